@@ -1,0 +1,300 @@
+"""CPU oracle for the LR-QAT linear layer (arXiv 2406.06385).
+
+TEST INFRASTRUCTURE ONLY.  This module is the independent reference that the
+CUDA path is checked against.  Only the test suite, ``__graft_entry__.smoke``
+and the CPU-baseline leg of ``bench.py`` may import it; the library itself never
+does.  It shares no code with the CUDA path and imports nothing from it: every
+function below is written from the paper's equations, in float64 unless the
+paper (or the reading stated next to the function) fixes another precision.
+
+Notation (Sec. 3 of the paper): a linear layer y = W x with W in R^{m x k}
+(m = out features, k = in features); tokens are stacked as rows, so
+Y[T, m] = X[T, k] W^T.  Bit-width b gives the symmetric integer grid
+[n, p] = [-2^{b-1}, 2^{b-1} - 1] (Eq. 1, Eq. 3).
+
+  * Eq. 6 / Eq. 7   Phi0 = phi(W0 / s0): frozen downcast of the pretrained weight
+  * Eq. 8           W_hat = s * clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p)
+  * Eq. 4 text      gradients w.r.t. A, B, s use the straight-through estimator
+                    d round(t) / dt = 1 (first introduced with Eq. 3)
+  * Sec. 3 end      after training W_Z = clip(...) is the integer weight, W_hat = s W_Z
+
+Readings where the paper is silent (all repeated in the design notes):
+  R1 round(.) is round-half-to-even (IEEE round-to-nearest; what PyTorch's
+     torch.round does, and the paper's implementation is PyTorch, App. B).
+  R2 the pre-round value u = phi^{-1}(Phi0) + (alpha/r) A B is formed at full
+     precision; integer codes are compared exactly except where the fp32
+     rendering of u lies within 1e-5 of a half-integer (see ``near_tie``).
+  R3 the STE clip mask is taken on the rounded value: M = 1[n <= round(u) <= p].
+  R4 ds is the plain gradient sum_j G_ij c_ij (no LSQ gradient scaling).
+  R5 per-channel scales are per output row; groups (g128) run along k.
+  R6 the nibble order of double packing: low nibble = even column, high nibble
+     = odd column, 4-bit two's complement.
+  R7 s0 comes from symmetric min-max range setting: max|W0| over the row (or
+     group) divided by p, in fp32; an all-zero row/group gets s0 = 1.
+  R8 W0 / s0 in the downcast is one fp32 IEEE division (the result then decides
+     an integer code, so both sides take it in the same precision).
+  R9 activation quantizer (weight-activation runs): per-tensor symmetric int8,
+     X_Z = clip(round(X / s_x), -128, 127) with X / s_x one fp32 division,
+     X_hat = s_x X_Z, STE with clip mask M_x = 1[-128 <= round(X/s_x) <= 127].
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import Dict, Optional
+
+import numpy as np
+
+PHI_QFIXED = 0
+PHI_INT_PACKED = 1
+
+NEAR_TIE_TOL = 1e-5
+
+
+@dataclass(frozen=True)
+class Layer:
+    """Quantizer settings of one layer, as the oracle sees them."""
+    m: int
+    k: int
+    r: int
+    alpha: float
+    bits: int
+    group_size: int = 0          # 0 = per output channel
+    phi_format: int = PHI_QFIXED
+    act_bits: int = 0            # 0 or 8
+
+
+def grid(bits: int):
+    """Symmetric b-bit integer grid [n, p] of Eq. 1 with z = 0."""
+    return -(2 ** (bits - 1)), 2 ** (bits - 1) - 1
+
+
+def frac_bits(layer: Layer) -> int:
+    """Fractional bits of the stored Phi0: 8 - b for Qb.(8-b) (Eq. 7), 0 for INT-b."""
+    return 8 - layer.bits if layer.phi_format == PHI_QFIXED else 0
+
+
+def expand_scale(s: np.ndarray, layer: Layer) -> np.ndarray:
+    """Broadcast a per-row [m] or per-group [m, k/g] scale to the full [m, k] shape (R5)."""
+    s = np.asarray(s, dtype=np.float64)
+    if layer.group_size == 0:
+        return np.repeat(s.reshape(layer.m, 1), layer.k, axis=1)
+    return np.repeat(s.reshape(layer.m, layer.k // layer.group_size), layer.group_size, axis=1)
+
+
+# ----------------------------------------------------------------------------
+# Range setting (App. B "PTQ initialization", min-max estimator) -- reading R7
+# ----------------------------------------------------------------------------
+def minmax_scale(W0: np.ndarray, layer: Layer) -> np.ndarray:
+    """s0 = max|W0| / p over each output row (or each g-wide group of a row), fp32."""
+    _, p = grid(layer.bits)
+    W0 = np.asarray(W0, dtype=np.float32)
+    if layer.group_size == 0:
+        amax = np.abs(W0).max(axis=1)
+    else:
+        amax = np.abs(W0.reshape(layer.m, layer.k // layer.group_size, layer.group_size)).max(axis=2)
+    safe = np.where(amax > 0, amax, np.float32(p)).astype(np.float32)
+    return np.divide(safe, np.float32(p), dtype=np.float32)
+
+
+# ----------------------------------------------------------------------------
+# Downcasting operator phi and its inverse (Sec. 3, Eq. 6, Eq. 7)
+# ----------------------------------------------------------------------------
+def pack_nibbles(codes: np.ndarray) -> np.ndarray:
+    """Double packing of INT-b values (b <= 4) into bytes, reading R6.
+
+    Byte j of a row holds column 2j in its low nibble and column 2j+1 in its
+    high nibble, each as a 4-bit two's complement number.
+    """
+    codes = np.asarray(codes).astype(np.int64)
+    assert codes.shape[1] % 2 == 0
+    assert codes.min(initial=0) >= -8 and codes.max(initial=0) <= 7
+    lo = codes[:, 0::2] & 0xF          # two's complement low 4 bits
+    hi = codes[:, 1::2] & 0xF
+    return (lo | (hi << 4)).astype(np.uint8)
+
+
+def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
+    """Inverse of ``pack_nibbles``: sign-extend each nibble back to an integer."""
+    packed = np.asarray(packed, dtype=np.uint8).astype(np.int64)
+    lo = packed & 0xF
+    hi = packed >> 4
+    out = np.empty((packed.shape[0], 2 * packed.shape[1]), dtype=np.int64)
+    out[:, 0::2] = np.where(lo >= 8, lo - 16, lo)
+    out[:, 1::2] = np.where(hi >= 8, hi - 16, hi)
+    return out.astype(np.int8)
+
+
+def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer) -> np.ndarray:
+    """Phi0 = phi(W0 / s0) (Eq. 6).
+
+    Q-fixed (Eq. 7): INT8(round(2^{8-b} * clip(x, n, p))), stored int8 [m, k].
+    INT-b (Sec. 3): clip(round(x), n, p), double-packed into uint8 [m, k/2].
+    x = W0 / s0 is a single fp32 division per element (reading R8).
+    """
+    n, p = grid(layer.bits)
+    W0 = np.asarray(W0, dtype=np.float32)
+    s_full = expand_scale(s0, layer).astype(np.float32)
+    x = np.divide(W0, s_full, dtype=np.float32)
+    if layer.phi_format == PHI_QFIXED:
+        y = np.clip(x.astype(np.float64), n, p) * 2.0 ** (8 - layer.bits)
+        return np.rint(y).astype(np.int8)
+    codes = np.clip(np.rint(x.astype(np.float64)), n, p).astype(np.int8)
+    return pack_nibbles(codes)
+
+
+def upcast(Phi0: np.ndarray, layer: Layer) -> np.ndarray:
+    """phi^{-1}(Phi0) as float64: Phi0 / 2^{8-b} (Eq. 7) or the unpacked INT-b value."""
+    if layer.phi_format == PHI_QFIXED:
+        return np.asarray(Phi0, dtype=np.int8).astype(np.float64) / 2.0 ** (8 - layer.bits)
+    return unpack_nibbles(Phi0).astype(np.float64)
+
+
+# ----------------------------------------------------------------------------
+# LR-QAT weight (Eq. 8) and its integer codes
+# ----------------------------------------------------------------------------
+def preround(Phi0: np.ndarray, A: np.ndarray, B: np.ndarray, layer: Layer) -> np.ndarray:
+    """u = phi^{-1}(Phi0) + (alpha / r) A B, the argument of round() in Eq. 8 (reading R2)."""
+    AB = np.asarray(A, dtype=np.float64) @ np.asarray(B, dtype=np.float64)
+    return upcast(Phi0, layer) + (layer.alpha / layer.r) * AB
+
+
+def codes_from_u(u: np.ndarray, layer: Layer):
+    """q = round(u) (R1), c = clip(q, n, p) (Eq. 8), M = 1[n <= q <= p] (R3)."""
+    n, p = grid(layer.bits)
+    q = np.rint(u)
+    c = np.clip(q, n, p)
+    M = ((q >= n) & (q <= p)).astype(np.float64)
+    return q, c, M
+
+
+def near_tie(u: np.ndarray, tol: float = NEAR_TIE_TOL) -> np.ndarray:
+    """Elements whose fp32 pre-round value lies within ``tol`` of a half-integer.
+
+    There the rounding decision depends on the last bits of the low-rank sum, so
+    two correct implementations may pick different codes.
+    """
+    u32 = np.asarray(u, dtype=np.float32).astype(np.float64)
+    return np.abs(u32 - (np.floor(u32) + 0.5)) <= tol
+
+
+def fake_quant_weight(Phi0, s, A, B, layer: Layer) -> Dict[str, np.ndarray]:
+    """W_hat = s * clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p)  (Eq. 8)."""
+    u = preround(Phi0, A, B, layer)
+    q, c, M = codes_from_u(u, layer)
+    return {"u": u, "q": q, "c": c, "M": M, "W_hat": expand_scale(s, layer) * c}
+
+
+def merge(Phi0, A, B, layer: Layer) -> np.ndarray:
+    """Integer weight W_Z = clip(round(...), n, p) that training leaves behind (Sec. 3, Eq. 8)."""
+    return codes_from_u(preround(Phi0, A, B, layer), layer)[1].astype(np.int8)
+
+
+# ----------------------------------------------------------------------------
+# Activation quantizer (weight-activation runs, Sec. 4 "Quantization") -- R9
+# ----------------------------------------------------------------------------
+def act_quant(X: np.ndarray, s_x: float):
+    """Per-tensor symmetric int8 fake quantization of activations (Eq. 1, z = 0, b = 8)."""
+    x = np.divide(np.asarray(X, dtype=np.float32), np.float32(s_x), dtype=np.float32)
+    q = np.rint(x.astype(np.float64))
+    codes = np.clip(q, -128, 127)
+    mask = ((q >= -128) & (q <= 127)).astype(np.float64)
+    return codes, float(np.float32(s_x)) * codes, mask
+
+
+# ----------------------------------------------------------------------------
+# Linear layer forward / backward with checkpointed W_hat (Sec. 3)
+# ----------------------------------------------------------------------------
+def _inputs(X, layer: Layer, s_x: Optional[float]):
+    X = np.asarray(X, dtype=np.float64)
+    if layer.act_bits == 8:
+        assert s_x is not None
+        _, Xh, Mx = act_quant(X, s_x)
+        return Xh, Mx
+    return X, np.ones_like(X)
+
+
+def linear_fwd(X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) -> np.ndarray:
+    """Y = X_hat W_hat^T with W_hat from Eq. 8; returns float64 [T, m]."""
+    Xh, _ = _inputs(X, layer, s_x)
+    return Xh @ fake_quant_weight(Phi0, s, A, B, layer)["W_hat"].T
+
+
+def linear_bwd(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) -> Dict[str, np.ndarray]:
+    """Gradients of the LR-QAT layer for an upstream gradient dY [T, m].
+
+    W_hat is recomputed from Phi0, A, B, s (the checkpointing of Sec. 3).  With
+    G = dY^T X_hat (the gradient w.r.t. W_hat) and the STE of Eq. 3/4:
+      dX = (dY W_hat) * M_x
+      dU = G * s * M                    (gradient w.r.t. u, mask from R3)
+      dA = (alpha/r) dU B^T,  dB = (alpha/r) A^T dU
+      ds = sum over the row (or group) of G * c   (reading R4)
+    """
+    dY = np.asarray(dY, dtype=np.float64)
+    Xh, Mx = _inputs(X, layer, s_x)
+    fq = fake_quant_weight(Phi0, s, A, B, layer)
+    dX = (dY @ fq["W_hat"]) * Mx
+    G = dY.T @ Xh
+    dU = G * expand_scale(s, layer) * fq["M"]
+    scale = layer.alpha / layer.r
+    dA = scale * (dU @ np.asarray(B, dtype=np.float64).T)
+    dB = scale * (np.asarray(A, dtype=np.float64).T @ dU)
+    Gc = G * fq["c"]
+    if layer.group_size == 0:
+        ds = Gc.sum(axis=1)
+    else:
+        ds = Gc.reshape(layer.m, layer.k // layer.group_size, layer.group_size).sum(axis=2)
+    return {"dX": dX, "dA": dA, "dB": dB, "ds": ds, "G": G, "fq": fq}
+
+
+def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) -> Dict[str, np.ndarray]:
+    """The same gradients as ``linear_bwd``, hand-expanded into scalar loops.
+
+    For tiny shapes only.  Each weight element is rebuilt from Eq. 8 with its
+    own rank-r dot product, and each gradient is accumulated term by term with
+    the chain rule through s * clip(round(.)) under the STE.
+    """
+    n, p = grid(layer.bits)
+    T = len(dY)
+    m, k, r = layer.m, layer.k, layer.r
+    P = upcast(Phi0, layer)
+    s_full = expand_scale(s, layer)
+    Xh, Mx = _inputs(X, layer, s_x)
+    A = np.asarray(A, dtype=np.float64)
+    B = np.asarray(B, dtype=np.float64)
+    dY = np.asarray(dY, dtype=np.float64)
+    scale = layer.alpha / layer.r
+    dX = np.zeros((T, k))
+    dA = np.zeros((m, r))
+    dB = np.zeros((r, k))
+    ds = np.zeros((m,) if layer.group_size == 0 else (m, k // layer.group_size))
+    for i in range(m):
+        for j in range(k):
+            lowrank = 0.0
+            for t in range(r):
+                lowrank += A[i, t] * B[t, j]
+            u = P[i, j] + scale * lowrank
+            q = float(np.rint(u))
+            c = min(max(q, n), p)
+            inside = 1.0 if n <= q <= p else 0.0
+            w = s_full[i, j] * c
+            g = 0.0                              # dL/dW_hat[i, j] = sum_tok dY[tok, i] X_hat[tok, j]
+            for tok in range(T):
+                g += dY[tok, i] * Xh[tok, j]
+                dX[tok, j] += dY[tok, i] * w * Mx[tok, j]
+            du = g * s_full[i, j] * inside       # STE through round, zero outside the clip range
+            for t in range(r):
+                dA[i, t] += scale * du * B[t, j]
+                dB[t, j] += scale * du * A[i, t]
+            if layer.group_size == 0:
+                ds[i] += g * c
+            else:
+                ds[i, j // layer.group_size] += g * c
+    return {"dX": dX, "dA": dA, "dB": dB, "ds": ds}
+
+
+def rel_fro(a: np.ndarray, b: np.ndarray) -> float:
+    """Relative Frobenius error ||a - b|| / ||b|| (the parity metric for float outputs)."""
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    den = np.linalg.norm(b)
+    return float(np.linalg.norm(a - b) / den) if den > 0 else float(np.linalg.norm(a - b))

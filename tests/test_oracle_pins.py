@@ -1,0 +1,321 @@
+"""Pins of the CPU oracle against facts the paper and the mathematics fix.
+
+None of these tests compares the oracle with itself: each checks it against a
+hand-worked example, a special case with a known answer, an exhaustive
+enumeration, an exact finite difference, or a library autograd of a closed form.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2406_06385_gb300 import workloads as WL
+
+
+# ---------------------------------------------------------------------------
+# Hand-worked example, Eq. 7 (phi = Q4.4) and Eq. 8, b = 4, r = 1, alpha = 1.
+# Every number below is a dyadic rational worked out by hand:
+#   x = W0 / s0 : row 0 [7, -3.5, 1.25, 0.3125], row 1 [-7, 3.75, 0.125, 6.5]
+#   Phi0 = 16 x : row 0 [112, -56, 20, 5],      row 1 [-112, 60, 2, 104]
+#   A B         : row 0 [0.75, 0.5, -0.25, 0.1875], row 1 [-0.375, -0.25, 0.125, -0.09375]
+#   u = Phi0/16 + A B : row 0 [7.75, -3.0, 1.0, 0.5], row 1 [-7.375, 3.5, 0.25, 6.40625]
+#   q = round-half-even(u) : row 0 [8, -3, 1, 0], row 1 [-7, 4, 0, 6]
+#   c = clip(q, -8, 7) : row 0 [7, -3, 1, 0], row 1 [-7, 4, 0, 6];  mask row 0 [0, 1, 1, 1]
+# ---------------------------------------------------------------------------
+HAND_LAYER = O.Layer(m=2, k=4, r=1, alpha=1.0, bits=4)
+HAND_W0 = np.array([[0.875, -0.4375, 0.15625, 0.0390625],
+                    [-1.75, 0.9375, 0.03125, 1.625]], dtype=np.float32)
+HAND_A = np.array([[0.5], [-0.25]])
+HAND_B = np.array([[1.5, 1.0, -0.5, 0.375]])
+HAND_S = np.array([0.25, 0.5])            # trained scale, differs from s0 on purpose
+HAND_X = np.array([[1.0, 2.0, -1.0, 0.5], [0.0, -1.0, 2.0, 1.0]])
+HAND_DY = np.array([[1.0, -1.0], [0.5, 2.0]])
+
+
+def test_hand_example_downcast_and_codes():
+    s0 = O.minmax_scale(HAND_W0, HAND_LAYER)
+    np.testing.assert_array_equal(s0, np.array([0.125, 0.25], dtype=np.float32))
+    phi0 = O.downcast(HAND_W0, s0, HAND_LAYER)
+    np.testing.assert_array_equal(phi0, [[112, -56, 20, 5], [-112, 60, 2, 104]])
+    fq = O.fake_quant_weight(phi0, HAND_S, HAND_A, HAND_B, HAND_LAYER)
+    np.testing.assert_array_equal(fq["u"], [[7.75, -3.0, 1.0, 0.5], [-7.375, 3.5, 0.25, 6.40625]])
+    np.testing.assert_array_equal(fq["q"], [[8, -3, 1, 0], [-7, 4, 0, 6]])
+    np.testing.assert_array_equal(fq["c"], [[7, -3, 1, 0], [-7, 4, 0, 6]])
+    np.testing.assert_array_equal(fq["M"], [[0, 1, 1, 1], [1, 1, 1, 1]])
+    np.testing.assert_array_equal(fq["W_hat"], [[1.75, -0.75, 0.25, 0.0], [-3.5, 2.0, 0.0, 3.0]])
+    np.testing.assert_array_equal(O.merge(phi0, HAND_A, HAND_B, HAND_LAYER), [[7, -3, 1, 0], [-7, 4, 0, 6]])
+
+
+def test_hand_example_forward_backward():
+    # Y = X W_hat^T; dX = dY W_hat; G = dY^T X; dU = G s M; dA = dU B^T; dB = A^T dU; ds = sum G c
+    #   G row 0 = [1, 1.5, 0, 1], row 1 = [-1, -4, 5, 1.5]
+    #   dU row 0 = 0.25 * G0 * [0,1,1,1] = [0, 0.375, 0, 0.25]; dU row 1 = 0.5 * G1 = [-0.5, -2, 2.5, 0.75]
+    phi0 = np.array([[112, -56, 20, 5], [-112, 60, 2, 104]], dtype=np.int8)
+    Y = O.linear_fwd(HAND_X, phi0, HAND_S, HAND_A, HAND_B, HAND_LAYER)
+    np.testing.assert_array_equal(Y, [[0.0, 2.0], [1.25, 1.0]])
+    g = O.linear_bwd(HAND_DY, HAND_X, phi0, HAND_S, HAND_A, HAND_B, HAND_LAYER)
+    np.testing.assert_array_equal(g["dX"], [[5.25, -2.75, 0.25, -3.0], [-6.125, 3.625, 0.125, 6.0]])
+    np.testing.assert_array_equal(g["G"], [[1.0, 1.5, 0.0, 1.0], [-1.0, -4.0, 5.0, 1.5]])
+    np.testing.assert_array_equal(g["dA"], [[0.46875], [-3.71875]])
+    np.testing.assert_array_equal(g["dB"], [[0.125, 0.6875, -0.625, -0.0625]])
+    np.testing.assert_array_equal(g["ds"], [2.5, 0.0])
+
+
+def test_hand_example_alpha_over_r_half():
+    # Same weights with alpha = 0.5, r = 1: (alpha/r) A B = row 0 [0.375, 0.25, -0.125, 0.09375],
+    # row 1 [-0.1875, -0.125, 0.0625, -0.046875];  u row 0 = [7.375, -3.25, 1.125, 0.40625] (no clip now),
+    # u row 1 = [-7.1875, 3.625, 0.1875, 6.453125];  q = [[7, -3, 1, 0], [-7, 4, 0, 6]], M = 1 everywhere.
+    # dU row 0 = 0.25 * [1, 1.5, 0, 1] = [0.25, 0.375, 0, 0.25]; dU row 1 = [-0.5, -2, 2.5, 0.75]
+    # dA = 0.5 * dU B^T = [[0.421875], [-1.859375]];  dB = 0.5 * A^T dU = [[0.125, 0.34375, -0.3125, -0.03125]]
+    layer = O.Layer(m=2, k=4, r=1, alpha=0.5, bits=4)
+    phi0 = np.array([[112, -56, 20, 5], [-112, 60, 2, 104]], dtype=np.int8)
+    fq = O.fake_quant_weight(phi0, HAND_S, HAND_A, HAND_B, layer)
+    np.testing.assert_array_equal(fq["u"], [[7.375, -3.25, 1.125, 0.40625], [-7.1875, 3.625, 0.1875, 6.453125]])
+    np.testing.assert_array_equal(fq["c"], [[7, -3, 1, 0], [-7, 4, 0, 6]])
+    assert fq["M"].min() == 1.0
+    g = O.linear_bwd(HAND_DY, HAND_X, phi0, HAND_S, HAND_A, HAND_B, layer)
+    np.testing.assert_array_equal(g["dA"], [[0.421875], [-1.859375]])
+    np.testing.assert_array_equal(g["dB"], [[0.125, 0.34375, -0.3125, -0.03125]])
+    np.testing.assert_array_equal(g["ds"], [2.5, 0.0])
+
+
+def test_hand_example_int4_packed():
+    # phi = INT-4 (Sec. 3): codes clip(round(x)) = row 0 [7, -4, 1, 0], row 1 [-7, 4, 0, 6]
+    # packed bytes: row 0 [0xC7, 0x01], row 1 [0x49, 0x60]
+    layer = O.Layer(m=2, k=4, r=1, alpha=1.0, bits=4, phi_format=O.PHI_INT_PACKED)
+    s0 = O.minmax_scale(HAND_W0, layer)
+    phi0 = O.downcast(HAND_W0, s0, layer)
+    np.testing.assert_array_equal(phi0, np.array([[0xC7, 0x01], [0x49, 0x60]], dtype=np.uint8))
+    np.testing.assert_array_equal(O.upcast(phi0, layer), [[7, -4, 1, 0], [-7, 4, 0, 6]])
+    # u row 0 = [7.75, -3.5, 0.75, 0.1875] -> q = [8, -4, 1, 0] (-3.5 ties to even -4)
+    fq = O.fake_quant_weight(phi0, HAND_S, HAND_A, HAND_B, layer)
+    np.testing.assert_array_equal(fq["q"][0], [8, -4, 1, 0])
+    np.testing.assert_array_equal(fq["c"][0], [7, -4, 1, 0])
+    np.testing.assert_array_equal(fq["M"][0], [0, 1, 1, 1])
+
+
+def test_hand_example_activation_quantizer():
+    # s_x = 0.5: X / s_x = [2, 4, -2, 1] ... all inside [-128, 127]
+    codes, xh, mask = O.act_quant(HAND_X, 0.5)
+    np.testing.assert_array_equal(codes, HAND_X * 2)
+    np.testing.assert_array_equal(xh, HAND_X)
+    assert mask.min() == 1.0
+    # s_x = 1/64: 2 * 64 = 128 -> clipped to 127, mask 0; -1 * 64 = -64 and -2 * 64 = -128 stay;
+    # 1.984375 * 64 = 127 stays; 1.9921875 * 64 = 127.5 ties to even 128 -> clipped, mask 0
+    codes, xh, mask = O.act_quant(np.array([[2.0, -1.0, -2.0, 1.984375, 1.9921875]]), 1.0 / 64)
+    np.testing.assert_array_equal(codes, [[127, -64, -128, 127, 127]])
+    np.testing.assert_array_equal(mask, [[0, 1, 1, 1, 0]])
+
+
+def test_minmax_zero_row_and_groups():
+    layer = O.Layer(m=2, k=256, r=1, alpha=1.0, bits=3, group_size=128)
+    W0 = np.zeros((2, 256), dtype=np.float32)
+    W0[0, 5] = -1.5          # group (0, 0): max 1.5 -> 1.5 / 3 = 0.5
+    W0[1, 200] = 0.75        # group (1, 1): 0.75 / 3 = 0.25
+    np.testing.assert_array_equal(O.minmax_scale(W0, layer), [[0.5, 1.0], [1.0, 0.25]])
+
+
+def test_near_tie_rule():
+    u = np.array([0.5, 0.500005, 0.5001, -2.499995, 3.0, 1.4999])
+    np.testing.assert_array_equal(O.near_tie(u), [True, True, False, True, False, False])
+
+
+# ---------------------------------------------------------------------------
+# Special cases with a textbook answer
+# ---------------------------------------------------------------------------
+def _rtn_python(x32: np.ndarray, n: int, p: int) -> np.ndarray:
+    """Round-to-nearest PTQ (Eq. 1 with z = 0) via Python's built-in round (half to even)."""
+    out = np.empty(x32.shape, dtype=np.int64)
+    for idx in np.ndindex(x32.shape):
+        out[idx] = min(max(round(float(x32[idx])), n), p)
+    return out
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_int_phi_with_zero_adapter_is_rtn(bits):
+    """phi = INT-b and B = 0: W_Z equals round-to-nearest quantization of W0 exactly."""
+    layer = O.Layer(m=24, k=64, r=4, alpha=4.0, bits=bits, phi_format=O.PHI_INT_PACKED)
+    spec = WL.LayerSpec("t", 24, 64, 4, 4.0, bits, 0, WL.PHI_INT_PACKED, outlier_frac=0.01)
+    d = WL.make_layer(spec, 1, seed=3, zero_B=True, with_activations=False)
+    s0 = O.minmax_scale(d.W0, layer)
+    x32 = np.divide(d.W0, s0[:, None].astype(np.float32), dtype=np.float32)
+    n, p = O.grid(bits)
+    wz = O.merge(O.downcast(d.W0, s0, layer), d.A, d.B, layer)
+    np.testing.assert_array_equal(wz, _rtn_python(x32, n, p))
+
+
+@pytest.mark.parametrize("bits", [3, 4])
+def test_qfixed_with_zero_adapter_is_rtn_except_double_rounding(bits):
+    """phi = Qb.(8-b) and B = 0: W_Z equals RTN of W0 except where the stored value
+    round(2^f x)/2^f lands exactly on a half-integer that x itself is not on
+    (double rounding); that set is predicted in closed form and must match exactly."""
+    layer = O.Layer(m=64, k=128, r=4, alpha=4.0, bits=bits)
+    spec = WL.LayerSpec("t", 64, 128, 4, 4.0, bits, 0, WL.PHI_QFIXED, outlier_frac=0.01)
+    d = WL.make_layer(spec, 1, seed=5, zero_B=True, with_activations=False)
+    s0 = O.minmax_scale(d.W0, layer)
+    x32 = np.divide(d.W0, s0[:, None].astype(np.float32), dtype=np.float32)
+    n, p = O.grid(bits)
+    f = 8 - bits
+    wz = O.merge(O.downcast(d.W0, s0, layer), d.A, d.B, layer).astype(np.int64)
+    rtn = _rtn_python(x32, n, p)
+    stored = np.array([round(min(max(float(v), n), p) * 2 ** f) / 2 ** f for v in x32.ravel()]).reshape(x32.shape)
+    on_half = (stored - np.floor(stored)) == 0.5
+    predicted = on_half & (np.vectorize(lambda a, b: round(a) != min(max(round(b), n), p))(stored, x32.astype(np.float64)))
+    mismatch = wz != rtn
+    np.testing.assert_array_equal(mismatch, predicted)
+    assert mismatch.sum() > 0   # the set is not empty on this draw
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 5, 6, 7])
+def test_qfixed_grid_round_trip_exhaustive(bits):
+    """Every Qb.(8-b) grid value j / 2^{8-b} survives phi^{-1}(phi(.)) exactly (Eq. 7)."""
+    n, p = O.grid(bits)
+    f = 8 - bits
+    js = np.arange(n * 2 ** f, p * 2 ** f + 1)
+    layer = O.Layer(m=1, k=len(js), r=1, alpha=1.0, bits=bits)
+    v = (js / 2 ** f).astype(np.float32)[None, :]
+    s0 = np.ones(1, dtype=np.float32)
+    phi = O.downcast(v, s0, layer)
+    np.testing.assert_array_equal(phi[0], js)
+    np.testing.assert_array_equal(O.upcast(phi, layer)[0], v[0])
+    np.testing.assert_array_equal(O.downcast(O.upcast(phi, layer).astype(np.float32), s0, layer), phi)
+    assert phi.min() == -128 and phi.max() == p * 2 ** f
+
+
+def test_nibble_packing_exhaustive():
+    """All 256 bytes unpack and re-pack to themselves; all 256 nibble pairs round-trip."""
+    allbytes = np.arange(256, dtype=np.uint8).reshape(1, 256)
+    np.testing.assert_array_equal(O.pack_nibbles(O.unpack_nibbles(allbytes)), allbytes)
+    pairs = np.array(list(itertools.product(range(-8, 8), repeat=2)), dtype=np.int64).reshape(1, -1)
+    np.testing.assert_array_equal(O.unpack_nibbles(O.pack_nibbles(pairs)), pairs)
+    # low nibble is the even column (reading R6)
+    np.testing.assert_array_equal(O.pack_nibbles(np.array([[1, -1]])), [[0xF1]])
+
+
+@pytest.mark.parametrize("phi_format,bits", [(O.PHI_QFIXED, 4), (O.PHI_QFIXED, 3), (O.PHI_INT_PACKED, 3)])
+def test_code_range_with_large_adapters(phi_format, bits):
+    """Codes stay on the b-bit grid whatever A B does; Phi0 stays in its storage range."""
+    layer = O.Layer(m=32, k=64, r=8, alpha=8.0, bits=bits, phi_format=phi_format)
+    spec = WL.LayerSpec("t", 32, 64, 8, 8.0, bits, 0, phi_format, a_std=2.0, b_std=2.0)
+    d = WL.make_layer(spec, 1, seed=7, with_activations=False)
+    s0 = O.minmax_scale(d.W0, layer)
+    phi0 = O.downcast(d.W0, s0, layer)
+    n, p = O.grid(bits)
+    if phi_format == O.PHI_QFIXED:
+        assert phi0.min() >= -128 and phi0.max() <= p * 2 ** (8 - bits)
+    fq = O.fake_quant_weight(phi0, s0, d.A, d.B, layer)
+    assert fq["c"].min() == n and fq["c"].max() == p     # large A B pushes both clip ends
+    assert 0 < fq["M"].mean() < 1
+
+
+@pytest.mark.parametrize("group_size", [0, 128])
+def test_merge_reproduces_fake_quant_weight(group_size):
+    """s * W_Z == W_hat element by element (Sec. 3: no loss when folding the adapters)."""
+    layer = O.Layer(m=16, k=256, r=4, alpha=4.0, bits=4, group_size=group_size)
+    spec = WL.LayerSpec("t", 16, 256, 4, 4.0, 4, group_size, WL.PHI_QFIXED, a_std=0.3, b_std=0.3)
+    d = WL.make_layer(spec, 1, seed=11, with_activations=False)
+    s0 = O.minmax_scale(d.W0, layer)
+    phi0 = O.downcast(d.W0, s0, layer)
+    s = s0 * np.float32(1.1)
+    wz = O.merge(phi0, d.A, d.B, layer)
+    fq = O.fake_quant_weight(phi0, s, d.A, d.B, layer)
+    np.testing.assert_array_equal(O.expand_scale(s, layer) * wz, fq["W_hat"])
+
+
+# ---------------------------------------------------------------------------
+# Gradients: matrix form vs hand-expanded loops, finite differences, autograd
+# ---------------------------------------------------------------------------
+LOOP_CASES = [
+    dict(m=4, k=6, r=2, bits=4, group_size=0, phi=O.PHI_QFIXED, act=0, std=0.3),
+    dict(m=4, k=6, r=2, bits=3, group_size=0, phi=O.PHI_QFIXED, act=0, std=2.0),      # clip active
+    dict(m=3, k=8, r=3, bits=4, group_size=0, phi=O.PHI_INT_PACKED, act=0, std=1.0),
+    dict(m=2, k=256, r=2, bits=4, group_size=128, phi=O.PHI_QFIXED, act=0, std=1.0),
+    dict(m=4, k=6, r=2, bits=4, group_size=0, phi=O.PHI_QFIXED, act=8, std=1.0),
+]
+
+
+def _tiny(case, T=3, seed=13):
+    layer = O.Layer(case["m"], case["k"], case["r"], float(case["r"]), case["bits"], case["group_size"],
+                    case["phi"], case["act"])
+    spec = WL.LayerSpec("t", case["m"], case["k"], case["r"], float(case["r"]), case["bits"],
+                        case["group_size"], case["phi"], a_std=case["std"], b_std=case["std"])
+    d = WL.make_layer(spec, T, seed=seed)
+    s0 = O.minmax_scale(d.W0, layer)
+    phi0 = O.downcast(d.W0, s0, layer)
+    s = s0 * np.float32(0.9)
+    s_x = float(np.abs(d.X).max()) / 200.0 if case["act"] else None   # small s_x: some clipping
+    return layer, d, phi0, s, s_x
+
+
+@pytest.mark.parametrize("case", LOOP_CASES)
+def test_ste_gradients_match_scalar_loops(case):
+    layer, d, phi0, s, s_x = _tiny(case)
+    ref = O.linear_bwd_loops(d.dY, d.X, phi0, s, d.A, d.B, layer, s_x)
+    got = O.linear_bwd(d.dY, d.X, phi0, s, d.A, d.B, layer, s_x)
+    for name in ("dX", "dA", "dB", "ds"):
+        np.testing.assert_allclose(got[name], ref[name], rtol=1e-12, atol=1e-12, err_msg=name)
+    if case["std"] == 2.0:
+        assert got["fq"]["M"].min() == 0.0       # the clip mask is exercised
+    if case["act"]:
+        assert O.act_quant(d.X, s_x)[2].min() == 0.0
+
+
+def _loss(dY, X, phi0, s, A, B, layer):
+    return float(np.sum(dY * O.linear_fwd(X, phi0, s, A, B, layer)))
+
+
+@pytest.mark.parametrize("case", LOOP_CASES[:4])
+def test_dX_and_ds_are_exact_gradients(case):
+    """Y is linear in X and in s (c does not depend on s, Eq. 5/8), so central
+    differences of <dY, Y> reproduce dX and ds up to float64 rounding."""
+    layer, d, phi0, s, _ = _tiny(case, T=4)
+    g = O.linear_bwd(d.dY, d.X, phi0, s, d.A, d.B, layer)
+    eps = 0.5
+    for (t, j) in [(0, 0), (1, layer.k - 1), (3, layer.k // 2)]:
+        Xp, Xm = d.X.astype(np.float64).copy(), d.X.astype(np.float64).copy()
+        Xp[t, j] += eps
+        Xm[t, j] -= eps
+        fd = (_loss(d.dY, Xp, phi0, s, d.A, d.B, layer) - _loss(d.dY, Xm, phi0, s, d.A, d.B, layer)) / (2 * eps)
+        assert abs(fd - g["dX"][t, j]) <= 1e-9 * max(1.0, abs(fd))
+    s64 = s.astype(np.float64)
+    for idx in [(0,) if s.ndim == 1 else (0, 0), (layer.m - 1,) if s.ndim == 1 else (layer.m - 1, 1)]:
+        sp, sm = s64.copy(), s64.copy()
+        sp[idx] += eps
+        sm[idx] -= eps
+        fd = (_loss(d.dY, d.X, phi0, sp, d.A, d.B, layer) - _loss(d.dY, d.X, phi0, sm, d.A, d.B, layer)) / (2 * eps)
+        assert abs(fd - g["ds"][idx]) <= 1e-9 * max(1.0, abs(fd))
+
+
+def test_adapter_gradients_equal_surrogate_autograd():
+    """Where no element is clipped (M = 1), the STE gradients w.r.t. A and B are the
+    exact gradients of the smooth surrogate s * (phi^{-1}(Phi0) + (alpha/r) A B)."""
+    torch = pytest.importorskip("torch")
+    layer = O.Layer(m=8, k=16, r=4, alpha=2.0, bits=4)
+    spec = WL.LayerSpec("t", 8, 16, 4, 2.0, 4, 0, WL.PHI_QFIXED, a_std=0.1, b_std=0.1)
+    d = WL.make_layer(spec, 5, seed=17)
+    s0 = O.minmax_scale(d.W0, layer) * np.float32(1.5)       # wide range: nothing clips
+    phi0 = O.downcast(d.W0, s0, layer)
+    g = O.linear_bwd(d.dY, d.X, phi0, s0, d.A, d.B, layer)
+    assert g["fq"]["M"].min() == 1.0
+    P = torch.tensor(O.upcast(phi0, layer), dtype=torch.float64)
+    A = torch.tensor(d.A, dtype=torch.float64, requires_grad=True)
+    B = torch.tensor(d.B, dtype=torch.float64, requires_grad=True)
+    s = torch.tensor(s0, dtype=torch.float64)[:, None]
+    W = s * (P + (layer.alpha / layer.r) * (A @ B))
+    loss = (torch.tensor(d.dY, dtype=torch.float64) * (torch.tensor(d.X, dtype=torch.float64) @ W.T)).sum()
+    loss.backward()
+    np.testing.assert_allclose(g["dA"], A.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(g["dB"], B.grad.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_workload_generator_is_deterministic_and_bf16_exact():
+    spec = WL.workload("tiny").layers[0]
+    a = WL.make_layer(spec, 64, seed=0)
+    b = WL.make_layer(spec, 64, seed=0)
+    for name in ("W0", "A_bits", "B_bits", "X_bits", "dY_bits"):
+        np.testing.assert_array_equal(getattr(a, name), getattr(b, name))
+    # bf16 values widen exactly and re-round to the same bits
+    np.testing.assert_array_equal(WL.bf16_bits(a.X), a.X_bits)
+    assert WL.bf16_bits(np.array([1.0 + 2.0 ** -8], dtype=np.float32))[0] == 0x3F80   # tie -> even
+    assert WL.bf16_bits(np.array([1.0 + 3 * 2.0 ** -8], dtype=np.float32))[0] == 0x3F82
