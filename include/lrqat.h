@@ -1,0 +1,145 @@
+/*
+ * lrqat.h -- C ABI of the GB300 (sm_103a) LR-QAT linear layer.
+ *
+ * LR-QAT (arXiv 2406.06385, Sec. 3) trains a quantized linear layer y = W x,
+ * W in R^{m x k}, through the fake-quantized weight of Eq. 8:
+ *
+ *     W_hat = s * clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p),
+ *     Phi0  = phi(W0 / s0)                                        (Eq. 6)
+ *
+ * with [n, p] = [-2^{b-1}, 2^{b-1}-1], a frozen downcast base Phi0, trainable
+ * rank-r adapters A [m, r], B [r, k] and a trainable scale s.  Tokens are
+ * stacked as rows: Y[T, m] = X[T, k] W_hat^T.
+ *
+ * Conventions for every call:
+ *   - Pointers are DEVICE pointers unless stated otherwise; arrays are dense
+ *     row-major; the caller owns every buffer and every buffer must be 16-byte
+ *     aligned (TMA).  bf16 tensors are passed as raw bfloat16 bits (uint16_t).
+ *   - Calls are asynchronous on `stream` (NULL = legacy default stream) and
+ *     allocate no device memory; scratch comes from the caller's workspace.
+ *   - Return value: LRQAT_OK or a negative lrqat_status.  Host-side argument
+ *     checks run before any CUDA work; the reason of the last failure on the
+ *     calling thread is available from lrqat_last_error().  Device-side bounded
+ *     waits that give up set a device status word, which
+ *     lrqat_get_device_status() reports as LRQAT_ERR_TIMEOUT.
+ *   - Rounding is round-half-to-even; the pre-round value
+ *     u = phi^{-1}(Phi0) + (alpha/r) A B is formed in fp32.
+ *   - Supported shapes: m and k multiples of 128, 1 <= r <= 64, T >= 1 (any
+ *     T; ragged token tails are handled), group_size 0 (per output channel)
+ *     or a multiple of 128 that divides k.
+ */
+#ifndef LRQAT_H
+#define LRQAT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t / CUstream. */
+typedef struct CUstream_st* lrqat_stream_t;
+
+typedef enum {
+  LRQAT_OK = 0,
+  LRQAT_ERR_INVALID_ARG = -1, /* null pointer, bad shape, bad bit-width ...          */
+  LRQAT_ERR_UNSUPPORTED = -2, /* valid for the method, not implemented (e.g. r > 64)  */
+  LRQAT_ERR_ALIGNMENT = -3,   /* a pointer is not 16-byte aligned                     */
+  LRQAT_ERR_WORKSPACE = -4,   /* workspace missing or smaller than required           */
+  LRQAT_ERR_CUDA = -5,        /* a CUDA runtime/driver call or launch failed          */
+  LRQAT_ERR_TIMEOUT = -6      /* a kernel's bounded wait gave up (device status)      */
+} lrqat_status;
+
+/* Storage format of the frozen base Phi0 (Sec. 3, "Downcasting operator"). */
+typedef enum {
+  /* Eq. 7, phi = Qb.(8-b): int8 [m, k], value round(2^{8-b} clip(W0/s0, n, p)). */
+  LRQAT_PHI_QFIXED = 0,
+  /* phi = INT-b, double-packed (b <= 4): uint8 [m, k/2]; byte j of a row holds
+   * column 2j in its low nibble and column 2j+1 in its high nibble, each a
+   * 4-bit two's complement integer clip(round(W0/s0), n, p). */
+  LRQAT_PHI_INT_PACKED = 1
+} lrqat_phi_format;
+
+/* Settings of one layer.  W is m x k (m = out features, k = in features). */
+typedef struct {
+  int64_t m;
+  int64_t k;
+  int32_t r;          /* adapter rank, 1..64                                        */
+  float alpha;        /* adapter scaling: (alpha / r) A B enters Eq. 8              */
+  int32_t bits;       /* b: 2..7 for QFIXED, 2..4 for INT_PACKED                    */
+  int32_t group_size; /* 0: one scale per output row (pc); else scales per g-wide
+                         group along k (g128 = 128), s has shape [m, k/g]           */
+  int32_t phi_format; /* lrqat_phi_format                                           */
+  int32_t act_bits;   /* 0: activations unquantized; 8: per-tensor symmetric int8
+                         X_hat = s_x clip(round(X/s_x), -128, 127) (Sec. 4,
+                         weight-activation quantization; Eq. 1 with z = 0)          */
+} lrqat_layer;
+
+/* Human-readable reason of the last non-OK status returned on this thread. */
+const char* lrqat_last_error(void);
+
+/* Symmetric min-max range setting (App. B, "PTQ initialization"):
+ *   s0[i] (or s0[i, g]) = max |W0[i, :]| (over the row or group) / p, fp32;
+ *   an all-zero row/group gets s0 = 1.
+ * W0: fp32 [m, k].  s0: fp32 [m] or [m, k/g] (output). */
+int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrqat_stream_t stream);
+
+/* Downcasting operator of Eq. 6 / Eq. 7: Phi0 = phi(W0 / s0), with W0 / s0 one
+ * fp32 IEEE division per element.
+ * W0: fp32 [m, k]; s0: fp32 [m] or [m, k/g];
+ * Phi0 (output): int8 [m, k] (QFIXED) or uint8 [m, k/2] (INT_PACKED). */
+int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0,
+                   lrqat_stream_t stream);
+
+/* Bytes of workspace lrqat_linear_fwd needs for T tokens (padded adapter
+ * copies; int8 activation codes when act_bits == 8). */
+size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
+
+/* Forward of the LR-QAT layer (Eq. 8 inside y = W_hat x):
+ *   Y = X_hat W_hat^T,  X_hat = X (act_bits 0) or s_x clip(round(X/s_x)) (act_bits 8).
+ * W_hat is rebuilt tile by tile inside the GEMM and never written to memory.
+ * X: bf16 [T, k]; Phi0 as produced by lrqat_downcast; s: fp32 [m] or [m, k/g];
+ * A: bf16 [m, r]; B: bf16 [r, k]; s_x: device fp32 scalar (required iff
+ * act_bits == 8, else may be NULL); Y (output): bf16 [T, m].
+ * workspace: device buffer of at least lrqat_fwd_workspace_bytes() bytes. */
+int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0,
+                     const float* s, const uint16_t* A, const uint16_t* B, const float* s_x,
+                     uint16_t* Y, void* workspace, size_t workspace_bytes, lrqat_stream_t stream);
+
+/* Bytes of workspace lrqat_linear_bwd needs for T tokens. */
+size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
+
+/* Backward of the LR-QAT layer for the upstream gradient dY, with W_hat
+ * recomputed rather than stored (the checkpointing of Sec. 3) and the
+ * straight-through estimator for round() (Eq. 3/4 text).  With G = dY^T X_hat,
+ * u, c = clip(round(u), n, p) and M = 1[n <= round(u) <= p]:
+ *   dX = (dY W_hat) * M_x          (M_x: activation clip mask, ones if act_bits 0)
+ *   dA = (alpha/r) (G * s * M) B^T,  dB = (alpha/r) A^T (G * s * M)
+ *   ds = sum over the row (or group) of G * c
+ * dY: bf16 [T, m]; X, Phi0, s, A, B, s_x as in lrqat_linear_fwd;
+ * dX (output): bf16 [T, k]; dA: fp32 [m, r]; dB: fp32 [r, k]; ds: fp32 like s.
+ * accumulate = 0 overwrites dA, dB, ds; 1 adds to them (gradient accumulation
+ * over micro-batches).  dX is always overwritten.
+ * workspace: device buffer of at least lrqat_bwd_workspace_bytes() bytes. */
+int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X,
+                     const void* Phi0, const float* s, const uint16_t* A, const uint16_t* B,
+                     const float* s_x, uint16_t* dX, float* dA, float* dB, float* ds, int accumulate,
+                     void* workspace, size_t workspace_bytes, lrqat_stream_t stream);
+
+/* Fold the adapters into the final integer weight (Sec. 3, after Eq. 8):
+ *   W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p),  so W_hat = s W_Z.
+ * W_Z (output): int8 [m, k] with values in [n, p]. */
+int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, const uint16_t* B,
+                int8_t* W_Z, lrqat_stream_t stream);
+
+/* Synchronizes `stream`, then reads and clears the device status word of the
+ * current device.  Returns LRQAT_OK, LRQAT_ERR_TIMEOUT (a kernel's bounded
+ * wait gave up since the last call) or LRQAT_ERR_CUDA. */
+int lrqat_get_device_status(lrqat_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LRQAT_H */

@@ -1,0 +1,406 @@
+// Fused weight-gradient kernel of the LR-QAT layer.  For a tile of 128 weight
+// rows i x (128 or 256) columns j and a range of tokens it computes
+//   G = dY^T X_hat                 (tcgen05, fp32 accumulator in TMEM, never stored)
+// and, in the epilogue, the straight-through gradients of Eq. 8:
+//   u = phi^{-1}(Phi0) + (alpha/r) A B   (low-rank tile by tcgen05, recomputed)
+//   M = 1[n <= round(u) <= p],  c = clip(round(u), n, p)
+//   dU = G * s * M  -> bf16 in shared memory
+//   dA_partial = dU B^T,  dB^T_partial = dU^T A   (tcgen05, N = r rounded to 16)
+//   ds_partial = sum_j G * c
+// The partials of dA, dB and ds are reduced deterministically by a later kernel.
+//
+// Roles (320 threads): warp 0 issues TMA, warp 1 issues tcgen05 MMAs and owns
+// TMEM, warps 2..9 run the epilogue.  Work units (row block, column tile, token
+// split) are distributed persistently over the CTAs.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "kernels.h"
+#include "ptx.cuh"
+#include "quant.cuh"
+
+namespace lrqat {
+namespace {
+
+constexpr int NS = 4;
+constexpr int BKT = 32;                        // tokens per pipeline stage
+constexpr int NUM_THREADS = 320;
+constexpr int NUM_EPI_WARPS = 8;
+
+constexpr uint32_t BOX_BYTES = 64 * 32 * 2;    // one 64-column x 32-token bf16 box (SW128)
+constexpr uint32_t STAGE_DY = 2 * BOX_BYTES;   // 128 rows i
+constexpr uint32_t STAGE_BYTES = STAGE_DY + 4 * BOX_BYTES;   // + up to 256 columns j
+constexpr uint32_t OFF_STAGES = 0;
+constexpr uint32_t OFF_APAD = OFF_STAGES + NS * STAGE_BYTES;   // A (padded to 64 cols), 128 rows, SW128
+constexpr uint32_t OFF_AT = OFF_APAD + 16384;                  // A^T: 2 boxes of r16 rows x 64 cols
+constexpr uint32_t OFF_PHI = OFF_AT + 16384;                   // Phi0 chunk 128 x 128 (packed: 128 x 64 B)
+constexpr uint32_t OFF_BT = OFF_PHI + 16384;                   // B^T (padded) chunk 128 rows, SW128
+constexpr uint32_t OFF_BP = OFF_BT + 16384;                    // B (padded) chunk: 2 boxes of r16 rows x 64 cols
+constexpr uint32_t OFF_DU = OFF_BP + 16384;                    // dU chunk: 2 atom columns of 128 rows x 128 B
+constexpr uint32_t SMEM_TILES = OFF_DU + 32768;
+constexpr uint32_t SMEM_BYTES = SMEM_TILES + 1024;
+static_assert(SMEM_BYTES <= 232448, "shared memory budget");
+
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t COL_G = 0;      // 256 columns
+constexpr uint32_t COL_L = 256;    // 128 columns
+constexpr uint32_t COL_DA = 384;   // up to 64 columns
+constexpr uint32_t COL_DBT = 448;  // up to 64 columns
+
+constexpr int BAR_FULL = 0;
+constexpr int BAR_EMPTY = BAR_FULL + NS;
+constexpr int BAR_EFFULL = BAR_EMPTY + NS;
+constexpr int BAR_EFEMPTY = BAR_EFFULL + 1;
+constexpr int BAR_ECFULL = BAR_EFEMPTY + 1;
+constexpr int BAR_ECEMPTY = BAR_ECFULL + 1;
+constexpr int BAR_ACCFULL = BAR_ECEMPTY + 1;
+constexpr int BAR_ACCEMPTY = BAR_ACCFULL + 1;
+constexpr int BAR_LFULL = BAR_ACCEMPTY + 1;
+constexpr int BAR_DUFULL = BAR_LFULL + 1;
+constexpr int BAR_DBFULL = BAR_DUFULL + 1;
+constexpr int BAR_DRAIN = BAR_DBFULL + 1;
+constexpr int NUM_BARS = BAR_DRAIN + 1;
+
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > timeout_ns) break;
+  }
+}
+
+struct Unit {
+  int ib, jt, sp, t0, nsteps;
+};
+
+__device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
+  Unit x;
+  x.ib = u % a.ni;
+  x.jt = (u / a.ni) % a.nj;
+  x.sp = u / (a.ni * a.nj);
+  x.t0 = x.sp * a.tchunk;
+  int t1 = x.t0 + a.tchunk;
+  if (t1 > a.T) t1 = a.T;
+  x.nsteps = (t1 - x.t0 + BKT - 1) / BKT;
+  return x;
+}
+
+template <bool PACKED>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    dw_kernel(const __grid_constant__ CUtensorMap tm_dy, const __grid_constant__ CUtensorMap tm_x,
+              const __grid_constant__ CUtensorMap tm_apad, const __grid_constant__ CUtensorMap tm_at,
+              const __grid_constant__ CUtensorMap tm_phi, const __grid_constant__ CUtensorMap tm_bt,
+              const __grid_constant__ CUtensorMap tm_b, const DwArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t bars[NUM_BARS];
+  __shared__ uint32_t tmem_base_s;
+  __shared__ volatile int abort_s;
+
+  const uint32_t smem = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  auto bar = [&](int i) { return smem_u32(&bars[i]); };
+  const int BN = 128 * args.nchunks;
+  const uint32_t rbox = static_cast<uint32_t>(args.r16) * 128u;   // bytes of one r16-row x 64-col box
+
+  if (threadIdx.x == 0) {
+    abort_s = 0;
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(bar(BAR_FULL + s), 1);
+      mbar_init(bar(BAR_EMPTY + s), 1);
+    }
+    mbar_init(bar(BAR_EFFULL), 1);
+    mbar_init(bar(BAR_EFEMPTY), 1);
+    mbar_init(bar(BAR_ECFULL), 1);
+    mbar_init(bar(BAR_ECEMPTY), 1);
+    mbar_init(bar(BAR_ACCFULL), 1);
+    mbar_init(bar(BAR_ACCEMPTY), NUM_EPI_WARPS);
+    mbar_init(bar(BAR_LFULL), 1);
+    mbar_init(bar(BAR_DUFULL), NUM_EPI_WARPS);
+    mbar_init(bar(BAR_DBFULL), 1);
+    mbar_init(bar(BAR_DRAIN), 1);
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc(smem_u32(&tmem_base_s), TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  const WaitCtl ctl{&abort_s, args.status, args.timeout_ns};
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      prefetch_tensormap(&tm_dy);
+      prefetch_tensormap(&tm_x);
+      const uint32_t stage_tx = STAGE_DY + 2u * args.nchunks * BOX_BYTES;
+      const uint32_t ef_tx = 16384u + 2u * rbox;
+      const uint32_t ec_tx = (PACKED ? 8192u : 16384u) + 16384u + 2u * rbox;
+      uint32_t g = 0, it = 0, cc = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
+        const Unit w = decode_unit(u, args);
+        for (int step = 0; step < w.nsteps; ++step) {
+          const uint32_t s = g % NS, ph = (g / NS) & 1u;
+          if (!(ok = wait_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1))) break;
+          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
+          const uint32_t fb = bar(BAR_FULL + s);
+          const int tok = w.t0 + step * BKT;
+          mbar_arrive_expect_tx(fb, stage_tx);
+          tma_load_2d(st, &tm_dy, w.ib * 128, tok, fb);
+          tma_load_2d(st + BOX_BYTES, &tm_dy, w.ib * 128 + 64, tok, fb);
+          for (int b = 0; b < 2 * args.nchunks; ++b)
+            tma_load_2d(st + STAGE_DY + b * BOX_BYTES, &tm_x, w.jt * BN + 64 * b, tok, fb);
+          ++g;
+        }
+        if (!ok) break;
+        if (!(ok = wait_bounded(bar(BAR_EFEMPTY), (it & 1u) ^ 1u, ctl, 2))) break;
+        mbar_arrive_expect_tx(bar(BAR_EFFULL), ef_tx);
+        tma_load_2d(smem + OFF_APAD, &tm_apad, 0, w.ib * 128, bar(BAR_EFFULL));
+        tma_load_2d(smem + OFF_AT, &tm_at, w.ib * 128, 0, bar(BAR_EFFULL));
+        tma_load_2d(smem + OFF_AT + rbox, &tm_at, w.ib * 128 + 64, 0, bar(BAR_EFFULL));
+        ++it;
+        for (int c = 0; c < args.nchunks; ++c) {
+          if (!(ok = wait_bounded(bar(BAR_ECEMPTY), (cc & 1u) ^ 1u, ctl, 3))) break;
+          const int j0 = w.jt * BN + 128 * c;
+          mbar_arrive_expect_tx(bar(BAR_ECFULL), ec_tx);
+          tma_load_2d(smem + OFF_PHI, &tm_phi, PACKED ? j0 / 2 : j0, w.ib * 128, bar(BAR_ECFULL));
+          tma_load_2d(smem + OFF_BT, &tm_bt, 0, j0, bar(BAR_ECFULL));
+          tma_load_2d(smem + OFF_BP, &tm_b, j0, 0, bar(BAR_ECFULL));
+          tma_load_2d(smem + OFF_BP + rbox, &tm_b, j0 + 64, 0, bar(BAR_ECFULL));
+          ++cc;
+        }
+      }
+      for (uint32_t s = 0; s < NS && s < g; ++s) {
+        const uint32_t last = s + NS * ((g - 1 - s) / NS);
+        drain_wait(bar(BAR_FULL + s), (last / NS) & 1u, args.timeout_ns);
+      }
+      if (it > 0) drain_wait(bar(BAR_EFFULL), (it - 1) & 1u, args.timeout_ns);
+      if (cc > 0) drain_wait(bar(BAR_ECFULL), (cc - 1) & 1u, args.timeout_ns);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc_g = make_idesc_bf16(128, BN, 1, 1);
+      const uint32_t idesc_l = make_idesc_bf16(128, 128, 0, 0);
+      const uint32_t idesc_da = make_idesc_bf16(128, args.r16, 0, 0);
+      const uint32_t idesc_db = make_idesc_bf16(128, args.r16, 1, 0);
+      const int lsteps = args.r16 / 16;
+      uint32_t g = 0, it = 0, cc = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
+        const Unit w = decode_unit(u, args);
+        if (!(ok = wait_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 4))) break;
+        tc_fence_after();
+        for (int step = 0; step < w.nsteps; ++step) {
+          const uint32_t s = g % NS, ph = (g / NS) & 1u;
+          if (!(ok = wait_bounded(bar(BAR_FULL + s), ph, ctl, 5))) break;
+          tc_fence_after();
+          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
+#pragma unroll
+          for (int ks = 0; ks < BKT / 16; ++ks) {
+            const uint64_t ad = make_sdesc(st + 2048u * ks, BOX_BYTES, 1024, SWZ_128B);
+            const uint64_t bd = make_sdesc(st + STAGE_DY + 2048u * ks, BOX_BYTES, 1024, SWZ_128B);
+            mma_bf16(tmem + COL_G, ad, bd, idesc_g, (step > 0 || ks > 0) ? 1u : 0u);
+          }
+          mma_commit(bar(BAR_EMPTY + s));
+          ++g;
+        }
+        if (!ok) break;
+        mma_commit(bar(BAR_ACCFULL));
+        if (!(ok = wait_bounded(bar(BAR_EFFULL), it & 1u, ctl, 6))) break;
+        for (int c = 0; c < args.nchunks; ++c) {
+          if (!(ok = wait_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 7))) break;
+          tc_fence_after();
+          // L = A_pad * (B^T chunk)^T : the low-rank tile of this 128 x 128 chunk
+          for (int ks = 0; ks < lsteps; ++ks) {
+            const uint64_t ad = make_sdesc(smem + OFF_APAD + 32u * ks, 16, 1024, SWZ_128B);
+            const uint64_t bd = make_sdesc(smem + OFF_BT + 32u * ks, 16, 1024, SWZ_128B);
+            mma_bf16(tmem + COL_L, ad, bd, idesc_l, ks > 0 ? 1u : 0u);
+          }
+          mma_commit(bar(BAR_LFULL));
+          if (!(ok = wait_bounded(bar(BAR_DUFULL), cc & 1u, ctl, 8))) break;
+          tc_fence_after();
+          // dA (+)= dU * B_chunk^T : M = 128 rows i, N = r16, K = 128 columns j
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint64_t ad = make_sdesc(smem + OFF_DU + 16384u * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+            const uint64_t bd = make_sdesc(smem + OFF_BP + rbox * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+            mma_bf16(tmem + COL_DA, ad, bd, idesc_da, (c > 0 || ks > 0) ? 1u : 0u);
+          }
+          // dB^T = dU^T * A : M = 128 columns j (dU read MN-major), N = r16, K = 128 rows i
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint64_t ad = make_sdesc(smem + OFF_DU + 2048u * ks, 16384, 1024, SWZ_128B);
+            const uint64_t bd = make_sdesc(smem + OFF_AT + rbox * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+            mma_bf16(tmem + COL_DBT, ad, bd, idesc_db, ks > 0 ? 1u : 0u);
+          }
+          mma_commit(bar(BAR_DBFULL));
+          mma_commit(bar(BAR_ECEMPTY));
+          ++cc;
+        }
+        if (!ok) break;
+        mma_commit(bar(BAR_EFEMPTY));
+        ++it;
+      }
+      mma_commit(bar(BAR_DRAIN));
+      drain_wait(bar(BAR_DRAIN), 0, args.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int pw = warp - 2;
+    const int q = warp & 3;
+    const int h = pw >> 2;
+    const int row = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const QuantParams qp = args.q;
+    const int nb = args.k / 128;
+    const float gscale = args.s_x != nullptr ? *args.s_x : 1.0f;
+    const int half_cols = args.r16 / 2;   // dA / dB^T columns read by this warp half
+    uint32_t it = 0, cc = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
+      const Unit w = decode_unit(u, args);
+      const int i_g = w.ib * 128 + row;
+      ok = wait_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 9);
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      for (int c = 0; c < args.nchunks; ++c) {
+        const int j0 = w.jt * BN + 128 * c;
+        const float s_i = args.s_ld ? args.s[static_cast<int64_t>(i_g) * args.s_ld + j0 / args.group_size]
+                                    : args.s[i_g];
+        ok = wait_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 10);
+        ok = ok && wait_bounded(bar(BAR_LFULL), cc & 1u, ctl, 11);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        tc_fence_after();
+        float ds_acc = 0.0f;
+#pragma unroll 1
+        for (int p = 0; p < 2; ++p) {
+          const int jl = 64 * h + 32 * p;   // column within the chunk
+          float G[32], Lv[32], v[32];
+          tmem_ld32(tmem + lane_off + COL_G + 128 * c + jl, G);
+          tmem_ld32(tmem + lane_off + COL_L + jl, Lv);
+          tmem_ld_wait();
+          if (PACKED) {
+            const uint4 raw = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 32, 64));
+            decode_i4x8(raw.x, v);
+            decode_i4x8(raw.y, v + 8);
+            decode_i4x8(raw.z, v + 16);
+            decode_i4x8(raw.w, v + 24);
+          } else {
+            const uint4 r0 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 16, 128));
+            const uint4 r1 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 16 + 1, 128));
+            decode_i8x4(r0.x, v);
+            decode_i8x4(r0.y, v + 4);
+            decode_i8x4(r0.z, v + 8);
+            decode_i8x4(r0.w, v + 12);
+            decode_i8x4(r1.x, v + 16);
+            decode_i8x4(r1.y, v + 20);
+            decode_i8x4(r1.z, v + 24);
+            decode_i8x4(r1.w, v + 28);
+          }
+          uint32_t du[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            float d2[2];
+#pragma unroll
+            for (int t = 0; t < 2; ++t) {
+              const int idx = 2 * e + t;
+              const float tm = magic_round(Lv[idx], v[idx], qp);
+              const bool inside = (tm >= qp.lo) && (tm <= qp.hi);
+              const float cval = code_from_magic(tm, qp);
+              const float gv = G[idx] * gscale;
+              ds_acc = __fmaf_rn(gv, cval, ds_acc);
+              d2[t] = inside ? gv * s_i : 0.0f;
+            }
+            du[e] = pack_rn_bf16x2(d2[0], d2[1]);
+          }
+          const uint32_t dub = smem + OFF_DU + 16384u * h;
+#pragma unroll
+          for (int wq = 0; wq < 4; ++wq)
+            st_shared_v4(dub + swz_offset(row, 4 * p + wq, 128), du[4 * wq], du[4 * wq + 1], du[4 * wq + 2],
+                         du[4 * wq + 3]);
+        }
+        // ds partial of this 128-column block (two halves h per row)
+        args.ds_part[(static_cast<int64_t>(w.sp * 2 + h) * args.m + i_g) * nb + j0 / 128] = ds_acc;
+        tc_fence_before();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(BAR_DUFULL));
+        ok = wait_bounded(bar(BAR_DBFULL), cc & 1u, ctl, 12);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        tc_fence_after();
+        // dB^T chunk: lanes = columns j of the chunk, TMEM columns = rank index
+        {
+          float* dst = args.dB_part + static_cast<int64_t>(w.ib * args.nsplit + w.sp) * args.r * args.k + j0 + row;
+          for (int c8 = 0; c8 < half_cols; c8 += 8) {
+            float vv[8];
+            tmem_ld8(tmem + lane_off + COL_DBT + h * half_cols + c8, vv);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const int t = h * half_cols + c8 + e;
+              if (t < args.r) dst[static_cast<int64_t>(t) * args.k] = vv[e];
+            }
+          }
+        }
+        if (c == args.nchunks - 1) {
+          float* dst = args.dA_part + (static_cast<int64_t>(w.jt * args.nsplit + w.sp) * args.m + i_g) * args.r;
+          for (int c8 = 0; c8 < half_cols; c8 += 8) {
+            float vv[8];
+            tmem_ld8(tmem + lane_off + COL_DA + h * half_cols + c8, vv);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const int t = h * half_cols + c8 + e;
+              if (t < args.r) dst[t] = vv[e];
+            }
+          }
+        }
+        ++cc;
+      }
+      if (!ok) break;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(BAR_ACCEMPTY));
+      ++it;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+template <bool PACKED>
+cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
+                       const CUtensorMap& e, const CUtensorMap& f, const CUtensorMap& g2, const DwArgs& args,
+                       int grid, cudaStream_t stream) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t err =
+        cudaFuncSetAttribute(dw_kernel<PACKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (err != cudaSuccess) return err;
+    configured = true;
+  }
+  dw_kernel<PACKED><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, f, g2, args);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int dw_smem_bytes(int, int) { return static_cast<int>(SMEM_BYTES); }
+
+cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_apad,
+                      const CUtensorMap& tm_at, const CUtensorMap& tm_phi, const CUtensorMap& tm_bt,
+                      const CUtensorMap& tm_b, const DwArgs& args, int grid, cudaStream_t stream) {
+  if (grid < 1 || args.r16 < 16 || args.r16 > 64 || (args.r16 & 15) || args.nchunks < 1 || args.nchunks > 2)
+    return cudaErrorInvalidValue;
+  return packed ? launch_one<true>(tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, args, grid, stream)
+                : launch_one<false>(tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, args, grid, stream);
+}
+
+}  // namespace lrqat

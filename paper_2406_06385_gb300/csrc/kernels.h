@@ -1,0 +1,91 @@
+// Internal launcher declarations shared by the translation units of liblrqat.
+// Every launcher enqueues on `stream` and returns the cudaError_t of the launch.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "quant.cuh"
+
+namespace lrqat {
+
+// ---- elementwise.cu --------------------------------------------------------
+cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int p, float* s0,
+                                cudaStream_t stream);
+cudaError_t launch_downcast(const float* W0, const float* s0, int64_t m, int64_t k, int group_size, int bits,
+                            int packed, void* phi0, cudaStream_t stream);
+cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
+                         int packed, const QuantParams& q, int8_t* wz, cudaStream_t stream);
+// codes = clip(round(X / s_x), -128, 127) as bf16; optional mask bits [k][ceil(T/32)].
+cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const float* s_x, uint16_t* codes,
+                             uint32_t* mask, cudaStream_t stream);
+// out[i][c] = c < r ? A[i][c] : 0 for c < 64 (A: [m, r] bf16 -> [m, 64]).
+cudaError_t launch_pad_rows64(const uint16_t* A, int64_t m, int r, uint16_t* out, cudaStream_t stream);
+// out[j][c] = c < r ? B[c][j] : 0 for c < 64 (B: [r, k] bf16 -> [k, 64]).
+cudaError_t launch_transpose_pad64(const uint16_t* B, int r, int64_t k, uint16_t* out, cudaStream_t stream);
+// out[c][i] = c < r ? A[i][c] : 0 for c < r16 (A: [m, r] -> [r16, m]).
+cudaError_t launch_transpose_rows(const uint16_t* A, int64_t m, int r, int r16, uint16_t* out,
+                                  cudaStream_t stream);
+// out[j][i] = stored integer of Phi0[i][j] (int8 raw, or sign-extended nibble), out: int8 [k, m].
+cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int packed, int8_t* out,
+                                 cudaStream_t stream);
+// Deterministic sums of the per-tile gradient partials written by the dW kernel.
+struct ReduceArgs {
+  const float* dA_part; int nA;      // [nA][m][r]
+  const float* dB_part; int nB;      // [nB][r][k]
+  const float* ds_part; int nS;      // [nS][m][k/128]
+  float* dA; float* dB; float* ds;
+  int64_t m, k; int r; int group_size;
+  float lr;                          // alpha / r
+  int accumulate;
+};
+cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream);
+
+// ---- fused_gemm.cu ---------------------------------------------------------
+enum FusedMode : int { FUSED_FWD_PC = 0, FUSED_FWD_GROUP = 1, FUSED_DX = 2 };
+
+struct FusedArgs {
+  int32_t rows;          // rows of the produced weight operand (m for fwd, k for dX)
+  int32_t kdim;          // contraction length (k for fwd, m for dX)
+  int32_t T;             // tokens
+  int32_t r16;           // adapter rank rounded up to 16
+  int32_t num_rb;        // rows / 128
+  int32_t num_tb;        // ceil(T / 448)
+  int32_t num_tiles;
+  QuantParams q;
+  const float* s;        // scale, [m] or [m, s_ld]
+  int32_t s_ld;          // groups per row (0 = per channel)
+  int32_t group_size;
+  const float* s_x;      // activation scale (device scalar) or nullptr
+  const uint32_t* xmask; // dX only: activation clip mask bits [k][xmask_ld], or nullptr
+  int32_t xmask_ld;
+  uint16_t* out;         // Y [T, m] (fwd) or dX [T, k] (dX)
+  int64_t out_ld;
+  int* status;
+  uint64_t timeout_ns;
+};
+int fused_smem_bytes();
+cudaError_t launch_fused(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
+                         const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
+                         cudaStream_t stream);
+
+// ---- dw.cu -------------------------------------------------------------------
+struct DwArgs {
+  int32_t m, k, T;
+  int32_t r, r16;
+  int32_t nchunks;       // 128-column chunks per tile (1 or 2)
+  int32_t ni, nj, nsplit, tchunk, num_units;
+  QuantParams q;
+  const float* s; int32_t s_ld; int32_t group_size;
+  const float* s_x;
+  float* dA_part; float* dB_part; float* ds_part;
+  int* status;
+  uint64_t timeout_ns;
+};
+int dw_smem_bytes(int r16, int packed);
+cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_apad,
+                      const CUtensorMap& tm_at, const CUtensorMap& tm_phi, const CUtensorMap& tm_bt,
+                      const CUtensorMap& tm_b, const DwArgs& args, int grid, cudaStream_t stream);
+
+}  // namespace lrqat

@@ -1,0 +1,530 @@
+// Host implementation of the C ABI declared in include/lrqat.h: argument
+// validation, workspace carving, TMA tensor-map encoding and kernel launches.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "kernels.h"
+#include "lrqat.h"
+
+namespace lrqat {
+namespace {
+
+// Device status word: kernels OR a bit into it when a bounded wait gives up.
+__device__ int g_device_status;
+
+constexpr uint64_t kWaitTimeoutNs = 2000000000ull;   // 2 s per wait
+constexpr int kMaxDevices = 64;
+
+thread_local std::string t_last_error;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  t_last_error = buf;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(LRQAT_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+struct DeviceInfo {
+  bool ready = false;
+  int sms = 0;
+  int* status = nullptr;
+};
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_dev_mu;
+
+int device_info(DeviceInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(LRQAT_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (!d.ready) {
+    e = cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_device_status);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
+    d.status = static_cast<int*>(p);
+    d.ready = true;
+  }
+  *out = &d;
+  return LRQAT_OK;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Row-major 2-D tensor [outer][inner] with rows of `row_bytes` bytes.
+int encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* ptr, uint64_t inner, uint64_t outer,
+              uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swz, const char* what) {
+  auto fn = tensor_map_encoder();
+  if (!fn) return fail(LRQAT_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = fn(map, dt, 2, const_cast<void*>(ptr), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(LRQAT_ERR_CUDA, "tensor map for %s failed (CUresult %d)", what, (int)r);
+  return LRQAT_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int frac_bits(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_QFIXED ? 8 - L.bits : 0; }
+int round16(int r) { return (r + 15) / 16 * 16; }
+
+int validate_layer(const lrqat_layer* L) {
+  if (!L) return fail(LRQAT_ERR_INVALID_ARG, "layer is NULL");
+  if (L->m <= 0 || L->k <= 0) return fail(LRQAT_ERR_INVALID_ARG, "m and k must be positive (m=%lld k=%lld)",
+                                          (long long)L->m, (long long)L->k);
+  if (L->m % 128 || L->k % 128)
+    return fail(LRQAT_ERR_UNSUPPORTED, "m and k must be multiples of 128 (m=%lld k=%lld)", (long long)L->m,
+                (long long)L->k);
+  if (L->m > (int64_t)1 << 30 || L->k > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "m or k too large");
+  if (L->r < 1) return fail(LRQAT_ERR_INVALID_ARG, "rank r must be >= 1 (r=%d)", L->r);
+  if (L->r > 64) return fail(LRQAT_ERR_UNSUPPORTED, "rank r=%d > 64 is not supported", L->r);
+  if (!std::isfinite(L->alpha)) return fail(LRQAT_ERR_INVALID_ARG, "alpha must be finite");
+  if (L->phi_format == LRQAT_PHI_QFIXED) {
+    if (L->bits < 2 || L->bits > 7) return fail(LRQAT_ERR_INVALID_ARG, "QFIXED needs 2 <= bits <= 7 (bits=%d)", L->bits);
+  } else if (L->phi_format == LRQAT_PHI_INT_PACKED) {
+    if (L->bits < 2 || L->bits > 4)
+      return fail(LRQAT_ERR_INVALID_ARG, "INT_PACKED needs 2 <= bits <= 4 (bits=%d)", L->bits);
+  } else {
+    return fail(LRQAT_ERR_INVALID_ARG, "unknown phi_format %d", L->phi_format);
+  }
+  if (L->group_size < 0) return fail(LRQAT_ERR_INVALID_ARG, "group_size must be >= 0");
+  if (L->group_size > 0 && (L->group_size % 128 || L->k % L->group_size))
+    return fail(LRQAT_ERR_UNSUPPORTED, "group_size %d must be a multiple of 128 dividing k", L->group_size);
+  if (L->act_bits != 0 && L->act_bits != 8)
+    return fail(LRQAT_ERR_UNSUPPORTED, "act_bits must be 0 or 8 (got %d)", L->act_bits);
+  return LRQAT_OK;
+}
+
+#define LRQAT_CHECK_PTR(p, name)                                                       \
+  do {                                                                                 \
+    if (!(p)) return fail(LRQAT_ERR_INVALID_ARG, "%s is NULL", name);                  \
+    if (!aligned16(p)) return fail(LRQAT_ERR_ALIGNMENT, "%s is not 16-byte aligned", name); \
+  } while (0)
+
+#define LRQAT_CUDA(expr, what)                          \
+  do {                                                  \
+    cudaError_t e_ = (expr);                            \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what);  \
+  } while (0)
+
+#define LRQAT_TRY(expr)          \
+  do {                           \
+    int st_ = (expr);            \
+    if (st_ != LRQAT_OK) return st_; \
+  } while (0)
+
+// Carves aligned sub-buffers out of a caller-provided workspace.
+struct Carver {
+  uintptr_t base;
+  size_t used = 0;
+  explicit Carver(void* p) : base(reinterpret_cast<uintptr_t>(p)) {}
+  void* take(size_t bytes) {
+    used = (used + 255) & ~size_t(255);
+    void* p = reinterpret_cast<void*>(base + used);
+    used += bytes;
+    return p;
+  }
+};
+
+// ----------------------------------------------------------------- planning --
+struct DwPlan {
+  int nchunks, ni, nj, nsplit, tchunk, units;
+};
+
+DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
+  DwPlan p;
+  p.nchunks = (L.k % 256 == 0) ? 2 : 1;
+  p.ni = static_cast<int>(L.m / 128);
+  p.nj = static_cast<int>(L.k / (128 * p.nchunks));
+  const int tiles = p.ni * p.nj;
+  const int64_t tsteps = (T + 31) / 32;
+  // Pick the token split that fills the SMs best; keep >= 256 tokens per split.
+  int best = 1;
+  double best_eff = 0.0;
+  for (int s = 1; s <= 8; ++s) {
+    if (s > 1 && tsteps / s < 8) break;
+    const int64_t units = static_cast<int64_t>(tiles) * s;
+    const int64_t waves = (units + sms - 1) / sms;
+    const double eff = static_cast<double>(units) / static_cast<double>(waves * sms) * (1.0 - 0.01 * (s - 1));
+    if (eff > best_eff + 1e-9) {
+      best_eff = eff;
+      best = s;
+    }
+  }
+  p.nsplit = best;
+  p.tchunk = static_cast<int>((tsteps + best - 1) / best) * 32;
+  p.nsplit = static_cast<int>((T + p.tchunk - 1) / p.tchunk);   // no empty splits
+  p.units = tiles * p.nsplit;
+  return p;
+}
+
+struct FwdWs {
+  uint16_t* a_pad;
+  uint16_t* bt_pad;
+  uint16_t* x_codes;
+};
+
+size_t fwd_ws_layout(const lrqat_layer& L, int64_t T, void* base, FwdWs* ws) {
+  Carver c(base);
+  FwdWs w{};
+  w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
+  w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  if (L.act_bits == 8) w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
+  if (ws) *ws = w;
+  return (c.used + 255) & ~size_t(255);
+}
+
+struct BwdWs {
+  uint16_t* a_pad;
+  uint16_t* bt_pad;
+  uint16_t* at;
+  uint16_t* b_pad;
+  int8_t* phit;
+  uint16_t* x_codes;
+  uint32_t* xmask;
+  float* dA_part;
+  float* dB_part;
+  float* ds_part;
+};
+
+size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* base, BwdWs* ws) {
+  Carver c(base);
+  BwdWs w{};
+  const int r16 = round16(L.r);
+  w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
+  w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  w.at = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.m * 2));
+  w.b_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.k * 2));
+  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
+  if (L.act_bits == 8) {
+    w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
+    w.xmask = static_cast<uint32_t*>(c.take(static_cast<size_t>(L.k) * ((T + 31) / 32) * 4));
+  }
+  w.dA_part = static_cast<float*>(c.take(static_cast<size_t>(p.nj) * p.nsplit * L.m * L.r * 4));
+  w.dB_part = static_cast<float*>(c.take(static_cast<size_t>(p.ni) * p.nsplit * L.r * L.k * 4));
+  w.ds_part = static_cast<float*>(c.take(static_cast<size_t>(2) * p.nsplit * L.m * (L.k / 128) * 4));
+  if (ws) *ws = w;
+  return (c.used + 255) & ~size_t(255);
+}
+
+int phi_map(CUtensorMap* map, const lrqat_layer& L, const void* phi0, uint32_t box_cols_elems, bool dw) {
+  // Forward: slices of 32 columns (32 B int8 rows, SW32; packed 16 B rows, no swizzle).
+  // dW: chunks of 128 columns (128 B int8 rows, SW128; packed 64 B rows, SW64).
+  if (L.phi_format == LRQAT_PHI_QFIXED)
+    return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k, L.m, L.k, box_cols_elems, 128,
+                     dw ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_32B, "Phi0");
+  return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k / 2, L.m, L.k / 2, box_cols_elems / 2, 128,
+                   dw ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_NONE, "Phi0 (packed)");
+}
+
+}  // namespace
+}  // namespace lrqat
+
+using namespace lrqat;
+
+extern "C" {
+
+const char* lrqat_last_error(void) { return t_last_error.c_str(); }
+
+int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  LRQAT_CHECK_PTR(W0, "W0");
+  LRQAT_CHECK_PTR(s0, "s0");
+  const lrqat_layer& L = *layer;
+  LRQAT_CUDA(launch_range_minmax(W0, L.m, L.k, L.group_size, (1 << (L.bits - 1)) - 1, s0, stream),
+             "range_minmax launch");
+  return LRQAT_OK;
+}
+
+int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0, lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  LRQAT_CHECK_PTR(W0, "W0");
+  LRQAT_CHECK_PTR(s0, "s0");
+  LRQAT_CHECK_PTR(Phi0, "Phi0");
+  const lrqat_layer& L = *layer;
+  LRQAT_CUDA(launch_downcast(W0, s0, L.m, L.k, L.group_size, L.bits, L.phi_format == LRQAT_PHI_INT_PACKED, Phi0,
+                             stream),
+             "downcast launch");
+  return LRQAT_OK;
+}
+
+size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
+  if (validate_layer(layer) != LRQAT_OK || T < 1) return 0;
+  return fwd_ws_layout(*layer, T, nullptr, nullptr);
+}
+
+int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0, const float* s,
+                     const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y, void* workspace,
+                     size_t workspace_bytes, lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  const lrqat_layer& L = *layer;
+  if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
+  if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
+  LRQAT_CHECK_PTR(X, "X");
+  LRQAT_CHECK_PTR(Phi0, "Phi0");
+  LRQAT_CHECK_PTR(s, "s");
+  if (!A) return fail(LRQAT_ERR_INVALID_ARG, "A is NULL");
+  if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
+  LRQAT_CHECK_PTR(Y, "Y");
+  if (L.act_bits == 8 && !s_x) return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8");
+  const size_t need = fwd_ws_layout(L, T, nullptr, nullptr);
+  if (!workspace || workspace_bytes < need)
+    return fail(LRQAT_ERR_WORKSPACE, "forward workspace of %zu bytes required, %zu given", need,
+                workspace ? workspace_bytes : (size_t)0);
+  if (!aligned16(workspace)) return fail(LRQAT_ERR_ALIGNMENT, "workspace is not 16-byte aligned");
+  DeviceInfo* dev = nullptr;
+  LRQAT_TRY(device_info(&dev));
+
+  FwdWs ws;
+  fwd_ws_layout(L, T, workspace, &ws);
+  const int r16 = round16(L.r);
+  LRQAT_CUDA(launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
+  LRQAT_CUDA(launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
+  const uint16_t* tok = X;
+  if (L.act_bits == 8) {
+    LRQAT_CUDA(launch_act_quant(X, T, L.k, s_x, ws.x_codes, nullptr, stream), "activation quantizer");
+    tok = ws.x_codes;
+  }
+  CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
+  LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 32, 224,
+                      CU_TENSOR_MAP_SWIZZLE_64B, "X"));
+  LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 32, false));
+  LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
+                      CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
+  LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 32,
+                      CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
+  FusedArgs a{};
+  a.rows = static_cast<int32_t>(L.m);
+  a.kdim = static_cast<int32_t>(L.k);
+  a.T = static_cast<int32_t>(T);
+  a.r16 = r16;
+  a.num_rb = static_cast<int32_t>(L.m / 128);
+  a.num_tb = static_cast<int32_t>((T + 447) / 448);
+  a.num_tiles = a.num_rb * a.num_tb;
+  a.q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+  a.s = s;
+  a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
+  a.group_size = L.group_size;
+  a.s_x = L.act_bits == 8 ? s_x : nullptr;
+  a.xmask = nullptr;
+  a.xmask_ld = 0;
+  a.out = Y;
+  a.out_ld = L.m;
+  a.status = dev->status;
+  a.timeout_ns = kWaitTimeoutNs;
+  const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
+  LRQAT_CUDA(launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, L.phi_format == LRQAT_PHI_INT_PACKED,
+                          tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+             "fused forward launch");
+  return LRQAT_OK;
+}
+
+size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
+  if (validate_layer(layer) != LRQAT_OK || T < 1) return 0;
+  DeviceInfo* dev = nullptr;
+  int sms = 152;
+  if (device_info(&dev) == LRQAT_OK) sms = dev->sms;
+  return bwd_ws_layout(*layer, T, plan_dw(*layer, T, sms), nullptr, nullptr);
+}
+
+int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X, const void* Phi0,
+                     const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* dX, float* dA,
+                     float* dB, float* ds, int accumulate, void* workspace, size_t workspace_bytes,
+                     lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  const lrqat_layer& L = *layer;
+  if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
+  if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
+  LRQAT_CHECK_PTR(dY, "dY");
+  LRQAT_CHECK_PTR(X, "X");
+  LRQAT_CHECK_PTR(Phi0, "Phi0");
+  LRQAT_CHECK_PTR(s, "s");
+  if (!A) return fail(LRQAT_ERR_INVALID_ARG, "A is NULL");
+  if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
+  LRQAT_CHECK_PTR(dX, "dX");
+  if (!dA || !dB || !ds) return fail(LRQAT_ERR_INVALID_ARG, "dA, dB and ds must not be NULL");
+  if (L.act_bits == 8 && !s_x) return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8");
+  DeviceInfo* dev = nullptr;
+  LRQAT_TRY(device_info(&dev));
+  const DwPlan plan = plan_dw(L, T, dev->sms);
+  const size_t need = bwd_ws_layout(L, T, plan, nullptr, nullptr);
+  if (!workspace || workspace_bytes < need)
+    return fail(LRQAT_ERR_WORKSPACE, "backward workspace of %zu bytes required, %zu given", need,
+                workspace ? workspace_bytes : (size_t)0);
+  if (!aligned16(workspace)) return fail(LRQAT_ERR_ALIGNMENT, "workspace is not 16-byte aligned");
+
+  BwdWs ws;
+  bwd_ws_layout(L, T, plan, workspace, &ws);
+  const int r16 = round16(L.r);
+  const bool packed = L.phi_format == LRQAT_PHI_INT_PACKED;
+  LRQAT_CUDA(launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
+  LRQAT_CUDA(launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
+  LRQAT_CUDA(launch_transpose_rows(A, L.m, L.r, r16, ws.at, stream), "transpose A");
+  LRQAT_CUDA(cudaMemsetAsync(ws.b_pad, 0, static_cast<size_t>(r16) * L.k * 2, stream), "clear B pad");
+  LRQAT_CUDA(cudaMemcpyAsync(ws.b_pad, B, static_cast<size_t>(L.r) * L.k * 2, cudaMemcpyDeviceToDevice, stream),
+             "copy B");
+  LRQAT_CUDA(launch_phi_transpose(Phi0, L.m, L.k, packed, ws.phit, stream), "transpose Phi0");
+  const uint16_t* xop = X;
+  if (L.act_bits == 8) {
+    LRQAT_CUDA(launch_act_quant(X, T, L.k, s_x, ws.x_codes, ws.xmask, stream), "activation quantizer");
+    xop = ws.x_codes;
+  }
+  const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+
+  // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
+  {
+    CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
+    LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 32, 224,
+                        CU_TENSOR_MAP_SWIZZLE_64B, "dY"));
+    LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.phit, L.m, L.k, L.m, 32, 128,
+                        CU_TENSOR_MAP_SWIZZLE_32B, "Phi0^T"));
+    LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
+    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 32,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
+    FusedArgs a{};
+    a.rows = static_cast<int32_t>(L.k);
+    a.kdim = static_cast<int32_t>(L.m);
+    a.T = static_cast<int32_t>(T);
+    a.r16 = r16;
+    a.num_rb = static_cast<int32_t>(L.k / 128);
+    a.num_tb = static_cast<int32_t>((T + 447) / 448);
+    a.num_tiles = a.num_rb * a.num_tb;
+    a.q = q;
+    a.s = s;
+    a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
+    a.group_size = L.group_size;
+    a.s_x = nullptr;
+    a.xmask = L.act_bits == 8 ? ws.xmask : nullptr;
+    a.xmask_ld = static_cast<int32_t>((T + 31) / 32);
+    a.out = dX;
+    a.out_ld = L.k;
+    a.status = dev->status;
+    a.timeout_ns = kWaitTimeoutNs;
+    const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
+    LRQAT_CUDA(launch_fused(FUSED_DX, 0, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream), "fused dX launch");
+  }
+  // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
+  {
+    CUtensorMap tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b;
+    LRQAT_TRY(encode_2d(&tm_dy, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 32,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "dY (dW)"));
+    LRQAT_TRY(encode_2d(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, xop, L.k, T, L.k * 2, 64, 32,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "X (dW)"));
+    LRQAT_TRY(encode_2d(&tm_apad, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A (padded, dW)"));
+    LRQAT_TRY(encode_2d(&tm_at, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "A^T"));
+    LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
+    LRQAT_TRY(encode_2d(&tm_bt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded, dW)"));
+    LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.b_pad, L.k, r16, L.k * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
+    DwArgs a{};
+    a.m = static_cast<int32_t>(L.m);
+    a.k = static_cast<int32_t>(L.k);
+    a.T = static_cast<int32_t>(T);
+    a.r = L.r;
+    a.r16 = r16;
+    a.nchunks = plan.nchunks;
+    a.ni = plan.ni;
+    a.nj = plan.nj;
+    a.nsplit = plan.nsplit;
+    a.tchunk = plan.tchunk;
+    a.num_units = plan.units;
+    a.q = q;
+    a.s = s;
+    a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
+    a.group_size = L.group_size;
+    a.s_x = L.act_bits == 8 ? s_x : nullptr;
+    a.dA_part = ws.dA_part;
+    a.dB_part = ws.dB_part;
+    a.ds_part = ws.ds_part;
+    a.status = dev->status;
+    a.timeout_ns = kWaitTimeoutNs;
+    const int grid = plan.units < dev->sms ? plan.units : dev->sms;
+    LRQAT_CUDA(launch_dw(packed, tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, a, grid, stream),
+               "fused dW launch");
+  }
+  ReduceArgs ra{};
+  ra.dA_part = ws.dA_part;
+  ra.nA = plan.nj * plan.nsplit;
+  ra.dB_part = ws.dB_part;
+  ra.nB = plan.ni * plan.nsplit;
+  ra.ds_part = ws.ds_part;
+  ra.nS = 2 * plan.nsplit;
+  ra.dA = dA;
+  ra.dB = dB;
+  ra.ds = ds;
+  ra.m = L.m;
+  ra.k = L.k;
+  ra.r = L.r;
+  ra.group_size = L.group_size;
+  ra.lr = static_cast<float>(static_cast<double>(L.alpha) / L.r);
+  ra.accumulate = accumulate ? 1 : 0;
+  LRQAT_CUDA(launch_reduce(ra, stream), "gradient reduction");
+  return LRQAT_OK;
+}
+
+int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, const uint16_t* B, int8_t* W_Z,
+                lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  const lrqat_layer& L = *layer;
+  LRQAT_CHECK_PTR(Phi0, "Phi0");
+  if (!A) return fail(LRQAT_ERR_INVALID_ARG, "A is NULL");
+  if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
+  LRQAT_CHECK_PTR(W_Z, "W_Z");
+  const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+  LRQAT_CUDA(launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format == LRQAT_PHI_INT_PACKED, q, W_Z, stream),
+             "merge launch");
+  return LRQAT_OK;
+}
+
+int lrqat_get_device_status(lrqat_stream_t stream) {
+  DeviceInfo* dev = nullptr;
+  LRQAT_TRY(device_info(&dev));
+  LRQAT_CUDA(cudaStreamSynchronize(stream), "cudaStreamSynchronize");
+  int h = 0;
+  LRQAT_CUDA(cudaMemcpy(&h, dev->status, sizeof(int), cudaMemcpyDeviceToHost), "read device status");
+  if (h != 0) {
+    LRQAT_CUDA(cudaMemset(dev->status, 0, sizeof(int)), "clear device status");
+    return fail(LRQAT_ERR_TIMEOUT, "a kernel's bounded wait gave up (status word 0x%x)", h);
+  }
+  return LRQAT_OK;
+}
+
+}  // extern "C"

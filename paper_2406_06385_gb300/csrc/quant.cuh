@@ -1,0 +1,103 @@
+// Device-side arithmetic of the LR-QAT quantizer (Eq. 7 and Eq. 8 of the paper),
+// written for throughput inside GEMM producer stages.
+//
+// With f fractional bits of the stored base (f = 8 - b for Qb.(8-b), 0 for INT-b)
+// and v the stored integer (Phi0 itself, or the unpacked nibble):
+//   u_f = v + 2^f (alpha/r) L            (= 2^f u, one fp32 FMA: scaling by 2^f is exact)
+//   t   = u_f + 1.5 * 2^(23+f)           (fp32 add: rounds u_f to a multiple of 2^f,
+//                                          ties to even, i.e. round-half-even of u)
+//   t   = clamp(t, magic + 2^f n, magic + 2^f p)
+//   c   = t * 2^-f - 1.5 * 2^23          (exact: the integer code clip(round(u), n, p))
+// Integer inputs are turned into floats with the 2^23 exponent trick (a byte
+// permute into 0x4B0000xx and one subtraction) instead of a conversion
+// instruction.
+#pragma once
+
+#include <cstdint>
+
+namespace lrqat {
+
+struct QuantParams {
+  float lr_scale;   // 2^f * alpha / r
+  float magic;      // 1.5 * 2^(23 + f)
+  float lo;         // magic + 2^f * n
+  float hi;         // magic + 2^f * p
+  float inv2f;      // 2^-f
+  float magic_c;    // 1.5 * 2^23
+};
+
+// Builds the constants above on the host.
+inline QuantParams make_quant_params(int bits, int frac_bits, float alpha, int r) {
+  QuantParams q;
+  const double two_f = static_cast<double>(1 << frac_bits);
+  const double n = -static_cast<double>(1 << (bits - 1));
+  const double p = static_cast<double>((1 << (bits - 1)) - 1);
+  q.lr_scale = static_cast<float>(two_f * static_cast<double>(alpha) / static_cast<double>(r));
+  q.magic = static_cast<float>(1.5 * 8388608.0 * two_f);
+  q.lo = static_cast<float>(1.5 * 8388608.0 * two_f + two_f * n);
+  q.hi = static_cast<float>(1.5 * 8388608.0 * two_f + two_f * p);
+  q.inv2f = static_cast<float>(1.0 / two_f);
+  q.magic_c = 12582912.0f;   // 1.5 * 2^23
+  return q;
+}
+
+// 4 signed bytes of `w` -> 4 exact floats.
+__device__ __forceinline__ void decode_i8x4(uint32_t w, float* v) {
+  const uint32_t x = w ^ 0x80808080u;   // v + 128 in each byte
+  v[0] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7540u)) - 8388736.0f;   // 2^23 + 128
+  v[1] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7541u)) - 8388736.0f;
+  v[2] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7542u)) - 8388736.0f;
+  v[3] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7543u)) - 8388736.0f;
+}
+
+// 8 signed nibbles of `w` (low nibble of byte b = element 2b, high = 2b+1) -> 8 exact floats.
+__device__ __forceinline__ void decode_i4x8(uint32_t w, float* v) {
+  const uint32_t x = w ^ 0x88888888u;   // v + 8 in each nibble
+  const uint32_t lo = x & 0x0F0F0F0Fu;
+  const uint32_t hi = (x >> 4) & 0x0F0F0F0Fu;
+#pragma unroll
+  for (int b = 0; b < 4; ++b) {
+    v[2 * b] = __uint_as_float(__byte_perm(lo, 0x4B000000u, 0x7540u + b)) - 8388616.0f;       // 2^23 + 8
+    v[2 * b + 1] = __uint_as_float(__byte_perm(hi, 0x4B000000u, 0x7540u + b)) - 8388616.0f;
+  }
+}
+
+// t = round-half-even(u_f / 2^f) in the magic domain, unclipped.
+__device__ __forceinline__ float magic_round(float L, float v, const QuantParams& q) {
+  const float u = __fmaf_rn(L, q.lr_scale, v);
+  return __fadd_rn(u, q.magic);
+}
+
+// Integer code c = clip(round(u), n, p) as an exact float.
+__device__ __forceinline__ float code_from_magic(float t, const QuantParams& q) {
+  const float tc = fminf(fmaxf(t, q.lo), q.hi);
+  return __fmaf_rn(tc, q.inv2f, -q.magic_c);
+}
+
+__device__ __forceinline__ float lrqat_code(float L, float v, const QuantParams& q) {
+  return code_from_magic(magic_round(L, v, q), q);
+}
+
+// Two small-integer floats (|c| <= 128) -> packed bf16x2, exact (bf16 keeps the top 16 bits).
+__device__ __forceinline__ uint32_t pack_exact_bf16x2(float lo, float hi) {
+  return __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x7632u);
+}
+
+// Two floats -> packed bf16x2 with round-to-nearest-even.
+__device__ __forceinline__ uint32_t pack_rn_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+__device__ __forceinline__ float bf16_to_float(uint16_t b) {
+  return __uint_as_float(static_cast<uint32_t>(b) << 16);
+}
+
+__device__ __forceinline__ uint16_t float_to_bf16_rn(float f) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(0.0f), "f"(f));
+  return static_cast<uint16_t>(r & 0xFFFFu);
+}
+
+}  // namespace lrqat

@@ -1,0 +1,130 @@
+"""Python binding of liblrqat (the C ABI in include/lrqat.h).
+
+Argument marshalling only: every function here forwards torch tensor pointers
+and the current CUDA stream to the C entry point of the same name and raises
+``LrqatError`` on a non-OK status.  All computation happens in the library's
+CUDA kernels; there is no fallback when the library is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "_lib", "liblrqat.so")
+
+PHI_QFIXED = 0
+PHI_INT_PACKED = 1
+
+STATUS = {0: "LRQAT_OK", -1: "LRQAT_ERR_INVALID_ARG", -2: "LRQAT_ERR_UNSUPPORTED", -3: "LRQAT_ERR_ALIGNMENT",
+          -4: "LRQAT_ERR_WORKSPACE", -5: "LRQAT_ERR_CUDA", -6: "LRQAT_ERR_TIMEOUT"}
+
+
+class LrqatError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+class Layer(ctypes.Structure):
+    """Mirror of the C struct lrqat_layer."""
+    _fields_ = [("m", ctypes.c_int64), ("k", ctypes.c_int64), ("r", ctypes.c_int32), ("alpha", ctypes.c_float),
+                ("bits", ctypes.c_int32), ("group_size", ctypes.c_int32), ("phi_format", ctypes.c_int32),
+                ("act_bits", ctypes.c_int32)]
+
+    @classmethod
+    def from_spec(cls, spec) -> "Layer":
+        return cls(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Loads liblrqat.so; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with `python -m paper_2406_06385_gb300.build`")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i64, sz, ip = ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t, ctypes.c_int
+        lp = ctypes.POINTER(Layer)
+        L.lrqat_last_error.restype = ctypes.c_char_p
+        L.lrqat_last_error.argtypes = []
+        sigs = {
+            "lrqat_range_minmax": [lp, vp, vp, vp],
+            "lrqat_downcast": [lp, vp, vp, vp, vp],
+            "lrqat_linear_fwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+            "lrqat_linear_bwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ip, vp, sz, vp],
+            "lrqat_merge": [lp, vp, vp, vp, vp, vp],
+            "lrqat_get_device_status": [vp],
+        }
+        for name, args in sigs.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = ctypes.c_int
+        for name in ("lrqat_fwd_workspace_bytes", "lrqat_bwd_workspace_bytes"):
+            fn = getattr(L, name)
+            fn.argtypes = [lp, i64]
+            fn.restype = ctypes.c_size_t
+        _lib = L
+    return _lib
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        raise LrqatError(status, lib().lrqat_last_error().decode())
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is not None:
+        return stream if isinstance(stream, int) else stream.cuda_stream
+    import torch
+    return torch.cuda.current_stream().cuda_stream
+
+
+def last_error() -> str:
+    return lib().lrqat_last_error().decode()
+
+
+def range_minmax(layer: Layer, W0, s0, stream=None) -> None:
+    _check(lib().lrqat_range_minmax(ctypes.byref(layer), _ptr(W0), _ptr(s0), _stream(stream)))
+
+
+def downcast(layer: Layer, W0, s0, Phi0, stream=None) -> None:
+    _check(lib().lrqat_downcast(ctypes.byref(layer), _ptr(W0), _ptr(s0), _ptr(Phi0), _stream(stream)))
+
+
+def fwd_workspace_bytes(layer: Layer, T: int) -> int:
+    return int(lib().lrqat_fwd_workspace_bytes(ctypes.byref(layer), T))
+
+
+def bwd_workspace_bytes(layer: Layer, T: int) -> int:
+    return int(lib().lrqat_bwd_workspace_bytes(ctypes.byref(layer), T))
+
+
+def linear_fwd(layer: Layer, T: int, X, Phi0, s, A, B, s_x, Y, workspace, stream=None) -> None:
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().lrqat_linear_fwd(ctypes.byref(layer), T, _ptr(X), _ptr(Phi0), _ptr(s), _ptr(A), _ptr(B), _ptr(s_x),
+                                  _ptr(Y), _ptr(workspace), nbytes, _stream(stream)))
+
+
+def linear_bwd(layer: Layer, T: int, dY, X, Phi0, s, A, B, s_x, dX, dA, dB, ds, accumulate: bool, workspace,
+               stream=None) -> None:
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().lrqat_linear_bwd(ctypes.byref(layer), T, _ptr(dY), _ptr(X), _ptr(Phi0), _ptr(s), _ptr(A), _ptr(B),
+                                  _ptr(s_x), _ptr(dX), _ptr(dA), _ptr(dB), _ptr(ds), 1 if accumulate else 0,
+                                  _ptr(workspace), nbytes, _stream(stream)))
+
+
+def merge(layer: Layer, Phi0, A, B, W_Z, stream=None) -> None:
+    _check(lib().lrqat_merge(ctypes.byref(layer), _ptr(Phi0), _ptr(A), _ptr(B), _ptr(W_Z), _stream(stream)))
+
+
+def get_device_status(stream=None) -> None:
+    _check(lib().lrqat_get_device_status(_stream(stream)))

@@ -1,0 +1,59 @@
+"""Helpers for the GPU parity tests: host arrays <-> device tensors, and the
+per-layer set-up that goes through the library's own entry points."""
+import numpy as np
+
+from paper_2406_06385_gb300 import lrqat as LQ
+from paper_2406_06385_gb300 import workloads as WL
+
+
+def torch():
+    import torch as _t
+    return _t
+
+
+def to_dev(a: np.ndarray):
+    t = torch()
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint16:
+        return t.from_numpy(a.view(np.int16)).cuda()
+    if a.dtype == np.uint8:
+        return t.from_numpy(a).cuda()
+    return t.from_numpy(a).cuda()
+
+
+def bits_to_f32(t) -> np.ndarray:
+    """Device bf16 bits (int16 tensor) -> host fp32 values."""
+    return WL.bf16_to_f32(t.cpu().numpy().view(np.uint16))
+
+
+def empty(shape, dtype):
+    t = torch()
+    return t.empty(shape, dtype=dtype, device="cuda")
+
+
+def oracle_layer(spec):
+    import oracle as O
+    return O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+
+
+class DeviceLayer:
+    """One layer's frozen base and adapters on the device, prepared with the
+    library's own range setting and downcast."""
+
+    def __init__(self, data: WL.LayerData, s_scale: float = 1.0):
+        t = torch()
+        spec = data.spec
+        self.spec = spec
+        self.layer = LQ.Layer.from_spec(spec)
+        self.W0 = to_dev(data.W0)
+        ng = spec.k // spec.group_size if spec.group_size else 1
+        self.s0 = t.empty((spec.m, ng) if spec.group_size else (spec.m,), dtype=t.float32, device="cuda")
+        LQ.range_minmax(self.layer, self.W0, self.s0)
+        if spec.phi_format == WL.PHI_QFIXED:
+            self.phi0 = t.empty((spec.m, spec.k), dtype=t.int8, device="cuda")
+        else:
+            self.phi0 = t.empty((spec.m, spec.k // 2), dtype=t.uint8, device="cuda")
+        LQ.downcast(self.layer, self.W0, self.s0, self.phi0)
+        self.s = (self.s0 * s_scale).contiguous()
+        self.A = to_dev(data.A_bits)
+        self.B = to_dev(data.B_bits)

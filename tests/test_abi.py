@@ -1,0 +1,83 @@
+"""The C-ABI library loads, exports every symbol include/lrqat.h declares, and
+rejects bad arguments on the host before any CUDA work (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2406_06385_gb300 import lrqat as LQ
+from paper_2406_06385_gb300.build import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build()
+    return LQ.lib()
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "lrqat.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\*?\s+\**(lrqat_[a-z_0-9]+)\s*\(", src, flags=re.M)))
+
+
+def test_header_declares_the_entry_points():
+    names = header_functions()
+    for expected in ("lrqat_range_minmax", "lrqat_downcast", "lrqat_linear_fwd", "lrqat_linear_bwd", "lrqat_merge",
+                     "lrqat_fwd_workspace_bytes", "lrqat_bwd_workspace_bytes", "lrqat_get_device_status",
+                     "lrqat_last_error"):
+        assert expected in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in header_functions():
+        assert hasattr(lib, name), name
+
+
+def _layer(**kw):
+    d = dict(m=256, k=256, r=4, alpha=4.0, bits=4, group_size=0, phi_format=LQ.PHI_QFIXED, act_bits=0)
+    d.update(kw)
+    return LQ.Layer(**d)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(m=100), -2), (dict(k=0), -1), (dict(r=0), -1), (dict(r=65), -2), (dict(bits=1), -1), (dict(bits=8), -1),
+    (dict(phi_format=LQ.PHI_INT_PACKED, bits=5), -1), (dict(group_size=64), -2), (dict(group_size=384), -2),
+    (dict(act_bits=4), -2), (dict(phi_format=7), -1),
+])
+def test_invalid_layers_are_rejected_on_host(lib, kw, status):
+    L = _layer(**kw)
+    got = lib.lrqat_linear_fwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, None, 16, 16, 1 << 20, None)
+    assert got == status, LQ.last_error()
+    assert LQ.last_error()
+
+
+def test_null_and_misaligned_pointers_are_rejected(lib):
+    L = _layer()
+    assert lib.lrqat_linear_fwd(ctypes.byref(L), 64, None, 16, 16, 16, 16, None, 16, 16, 1 << 20, None) == -1
+    assert lib.lrqat_linear_fwd(ctypes.byref(L), 64, 18, 16, 16, 16, 16, None, 16, 16, 1 << 20, None) == -3
+    assert lib.lrqat_linear_fwd(ctypes.byref(L), 0, 16, 16, 16, 16, 16, None, 16, 16, 1 << 20, None) == -1
+    # act_bits = 8 needs s_x
+    L8 = _layer(act_bits=8)
+    assert lib.lrqat_linear_fwd(ctypes.byref(L8), 64, 16, 16, 16, 16, 16, None, 16, 16, 1 << 30, None) == -1
+
+
+def test_short_workspace_is_rejected(lib):
+    L = _layer()
+    need = lib.lrqat_fwd_workspace_bytes(ctypes.byref(L), 64)
+    assert need > 0
+    assert lib.lrqat_linear_fwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, None, 16, 16, need - 1, None) == -4
+    assert lib.lrqat_linear_bwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, 16, None, 16, 16, 16, 16, 0, None, 0,
+                                None) in (-4, -5)   # -5 when no CUDA device is visible
+
+
+def test_workspace_grows_with_tokens_and_activation_quantizer(lib):
+    L = _layer()
+    L8 = _layer(act_bits=8)
+    assert lib.lrqat_fwd_workspace_bytes(ctypes.byref(L), 64) == lib.lrqat_fwd_workspace_bytes(ctypes.byref(L), 4096)
+    assert lib.lrqat_fwd_workspace_bytes(ctypes.byref(L8), 4096) >= 4096 * 256 * 2
+    assert lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 64) > 0
+    assert lib.lrqat_fwd_workspace_bytes(ctypes.byref(_layer(m=100)), 64) == 0

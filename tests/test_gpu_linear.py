@@ -1,0 +1,168 @@
+"""GPU parity of the fused LR-QAT forward and backward against the oracle.
+
+Sizes span several tiles in every dimension and leave ragged tails (token
+counts that are not multiples of the 448-token forward tile or the 32-token dW
+stage).  Float outputs are compared by relative Frobenius error (Y, dX: 1e-2;
+dA, dB, ds: 2e-2); the integer codes the fused producers build are extracted
+exactly with identity inputs and compared bit for bit, except near-ties.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2406_06385_gb300 import lrqat as LQ
+from paper_2406_06385_gb300 import workloads as WL
+
+from gpu_util import DeviceLayer, bits_to_f32, oracle_layer, to_dev, torch
+
+pytestmark = pytest.mark.gpu
+
+TOL_ACT = 1e-2
+TOL_GRAD = 2e-2
+
+
+def spec_of(name, m, k, r, bits=4, group=0, phi=WL.PHI_QFIXED, act=0, alpha=None, a_std=1 / 64, b_std=1e-3,
+            outliers=1e-3):
+    return WL.LayerSpec(name, m, k, r, float(r if alpha is None else alpha), bits, group, phi, act,
+                        outlier_frac=outliers, a_std=a_std, b_std=b_std)
+
+
+CASES = [
+    # id, spec, T
+    ("q44_pc_multi_tile", spec_of("a", 384, 512, 32), 1000),
+    ("q44_pc_alpha1", spec_of("b", 256, 256, 8, alpha=1.0, a_std=0.3, b_std=0.3), 448),
+    ("q35_pc_r64", spec_of("c", 128, 384, 64, bits=3, a_std=0.1, b_std=0.1), 97),
+    ("int3_packed", spec_of("d", 256, 512, 32, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.2, b_std=0.2), 513),
+    ("int4_packed_r4", spec_of("e", 128, 256, 4, bits=4, phi=WL.PHI_INT_PACKED, a_std=0.3, b_std=0.3), 64),
+    ("q44_g128_a8", spec_of("f", 256, 384, 16, group=128, act=8, a_std=0.2, b_std=0.2), 300),
+    ("q44_g256", spec_of("g", 128, 512, 32, group=256, a_std=0.2, b_std=0.2), 256),
+    ("q26_clip_heavy", spec_of("h", 128, 256, 16, bits=2, a_std=1.0, b_std=1.0), 200),
+    ("tokens_1", spec_of("i", 128, 128, 1), 1),
+]
+
+
+def _run(spec, T, seed=0, s_scale=1.0, sx_factor=1.0, zero_B=False):
+    t = torch()
+    data = WL.make_layer(spec, T, seed=seed, zero_B=zero_B)
+    dl = DeviceLayer(data, s_scale)
+    X, dY = to_dev(data.X_bits), to_dev(data.dY_bits)
+    s_x_host = None
+    s_x = None
+    if spec.act_bits == 8:
+        s_x_host = np.float32(np.float32(np.abs(data.X).max()) / np.float32(127.0) * np.float32(sx_factor))
+        s_x = t.tensor([s_x_host], dtype=t.float32, device="cuda")
+    L = dl.layer
+    Y = t.empty((T, spec.m), dtype=t.int16, device="cuda")
+    ws = t.empty(max(LQ.fwd_workspace_bytes(L, T), 16), dtype=t.uint8, device="cuda")
+    LQ.linear_fwd(L, T, X, dl.phi0, dl.s, dl.A, dl.B, s_x, Y, ws)
+    dX = t.empty((T, spec.k), dtype=t.int16, device="cuda")
+    dA = t.empty((spec.m, spec.r), dtype=t.float32, device="cuda")
+    dB = t.empty((spec.r, spec.k), dtype=t.float32, device="cuda")
+    ds = t.empty_like(dl.s)
+    wsb = t.empty(LQ.bwd_workspace_bytes(L, T), dtype=t.uint8, device="cuda")
+    LQ.linear_bwd(L, T, dY, X, dl.phi0, dl.s, dl.A, dl.B, s_x, dX, dA, dB, ds, False, wsb)
+    LQ.get_device_status()
+    # oracle side: its own range setting and downcast from the same W0
+    OL = oracle_layer(spec)
+    s0 = O.minmax_scale(data.W0, OL)
+    phi0 = O.downcast(data.W0, s0, OL)
+    s = (s0 * np.float32(s_scale)).astype(np.float32)
+    Y_ref = O.linear_fwd(data.X, phi0, s, data.A, data.B, OL, s_x_host)
+    g = O.linear_bwd(data.dY, data.X, phi0, s, data.A, data.B, OL, s_x_host)
+    got = dict(Y=bits_to_f32(Y), dX=bits_to_f32(dX), dA=dA.cpu().numpy(), dB=dB.cpu().numpy(),
+               ds=ds.cpu().numpy().reshape(g["ds"].shape))
+    ref = dict(Y=Y_ref, dX=g["dX"], dA=g["dA"], dB=g["dB"], ds=g["ds"])
+    return got, ref, g
+
+
+@pytest.mark.parametrize("cid,spec,T", CASES, ids=[c[0] for c in CASES])
+def test_fwd_bwd_parity(cid, spec, T):
+    got, ref, g = _run(spec, T, seed=1, s_scale=1.05)
+    errs = {k: O.rel_fro(got[k], ref[k]) for k in got}
+    assert errs["Y"] <= TOL_ACT and errs["dX"] <= TOL_ACT, errs
+    assert errs["dA"] <= TOL_GRAD and errs["dB"] <= TOL_GRAD and errs["ds"] <= TOL_GRAD, errs
+    if cid == "q26_clip_heavy":
+        assert g["fq"]["M"].mean() < 0.9    # the STE clip mask matters in this case
+
+
+def test_activation_clip_mask_in_dx():
+    """A small activation scale clips part of X; dX must vanish there (STE mask)."""
+    spec = spec_of("m", 128, 256, 16, group=128, act=8, a_std=0.2, b_std=0.2)
+    got, ref, _ = _run(spec, 160, seed=4, sx_factor=0.25)
+    assert (ref["dX"] == 0).mean() > 0.01
+    for k in ("Y", "dX"):
+        assert O.rel_fro(got[k], ref[k]) <= TOL_ACT, k
+    for k in ("dA", "dB", "ds"):
+        assert O.rel_fro(got[k], ref[k]) <= TOL_GRAD, k
+
+
+def test_gradient_accumulation():
+    """accumulate = 1 adds to dA, dB, ds; dX is overwritten."""
+    t = torch()
+    spec = spec_of("acc", 128, 256, 8, a_std=0.2, b_std=0.2)
+    data = WL.make_layer(spec, 96, seed=9)
+    dl = DeviceLayer(data)
+    X, dY = to_dev(data.X_bits), to_dev(data.dY_bits)
+    L = dl.layer
+    ws = t.empty(LQ.bwd_workspace_bytes(L, 96), dtype=t.uint8, device="cuda")
+    outs = []
+    for acc in (False, True):
+        dX = t.empty((96, 256), dtype=t.int16, device="cuda")
+        dA = t.zeros((128, 8), dtype=t.float32, device="cuda") if not acc else outs[0][1].clone()
+        dB = t.zeros((8, 256), dtype=t.float32, device="cuda") if not acc else outs[0][2].clone()
+        ds = t.zeros((128,), dtype=t.float32, device="cuda") if not acc else outs[0][3].clone()
+        LQ.linear_bwd(L, 96, dY, X, dl.phi0, dl.s, dl.A, dl.B, None, dX, dA, dB, ds, acc, ws)
+        outs.append((dX, dA, dB, ds))
+    LQ.get_device_status()
+    for i in (1, 2, 3):
+        np.testing.assert_allclose(outs[1][i].cpu().numpy(), 2 * outs[0][i].cpu().numpy(), rtol=1e-6, atol=1e-6)
+    np.testing.assert_array_equal(outs[1][0].cpu().numpy(), outs[0][0].cpu().numpy())
+
+
+CODE_CASES = [
+    ("q44_pc", spec_of("c1", 256, 256, 32, a_std=0.1, b_std=0.1)),
+    ("q35_pc", spec_of("c2", 128, 384, 16, bits=3, a_std=0.2, b_std=0.2)),
+    ("int3_packed", spec_of("c3", 128, 256, 8, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.3, b_std=0.3)),
+    ("q44_g128", spec_of("c4", 128, 256, 16, group=128, a_std=0.1, b_std=0.1)),
+]
+
+
+@pytest.mark.parametrize("cid,spec", CODE_CASES, ids=[c[0] for c in CODE_CASES])
+@pytest.mark.parametrize("zero_B", [False, True], ids=["lowrank", "ties"])
+def test_fused_codes_bit_exact(cid, spec, zero_B):
+    """With s = 1 and X = I (T = k) the forward returns Y = C^T exactly; with
+    dY = I (T = m) the dX kernel returns its own codes C.  Both must equal the
+    oracle's codes except at near-ties; B = 0 makes every Q-fixed half-integer an
+    exact tie, which both sides must round half to even."""
+    t = torch()
+    data = WL.make_layer(spec, 1, seed=5, with_activations=False, zero_B=zero_B)
+    dl = DeviceLayer(data)
+    dl.s = t.ones_like(dl.s)
+    L = dl.layer
+    m, k = spec.m, spec.k
+    eye_k = WL.bf16_bits(np.eye(k, dtype=np.float32))
+    eye_m = WL.bf16_bits(np.eye(m, dtype=np.float32))
+    Y = t.empty((k, m), dtype=t.int16, device="cuda")
+    ws = t.empty(max(LQ.fwd_workspace_bytes(L, k), 16), dtype=t.uint8, device="cuda")
+    LQ.linear_fwd(L, k, to_dev(eye_k), dl.phi0, dl.s, dl.A, dl.B, None, Y, ws)
+    T = m
+    dX = t.empty((T, k), dtype=t.int16, device="cuda")
+    dA = t.empty((m, spec.r), dtype=t.float32, device="cuda")
+    dB = t.empty((spec.r, k), dtype=t.float32, device="cuda")
+    ds = t.empty_like(dl.s)
+    Xz = t.zeros((T, k), dtype=t.int16, device="cuda")
+    wsb = t.empty(LQ.bwd_workspace_bytes(L, T), dtype=t.uint8, device="cuda")
+    LQ.linear_bwd(L, T, to_dev(eye_m), Xz, dl.phi0, dl.s, dl.A, dl.B, None, dX, dA, dB, ds, False, wsb)
+    LQ.get_device_status()
+    OL = oracle_layer(spec)
+    phi0 = O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL)
+    ones = np.ones((m, k // spec.group_size) if spec.group_size else (m,))
+    fq = O.fake_quant_weight(phi0, ones, data.A, data.B, OL)
+    exempt = O.near_tie(fq["u"]) if not zero_B else np.zeros_like(fq["c"], dtype=bool)
+    c_fwd = bits_to_f32(Y).T
+    c_dx = bits_to_f32(dX)
+    for name, c in (("fwd", c_fwd), ("dX", c_dx)):
+        bad = (c != fq["c"]) & ~exempt
+        assert bad.sum() == 0, f"{name}: {bad.sum()} code mismatches (near-ties exempt: {exempt.sum()})"
+    if zero_B and spec.phi_format == WL.PHI_QFIXED:
+        assert (np.abs(fq["u"] - np.floor(fq["u"]) - 0.5) == 0).sum() > 0   # exact ties were exercised
