@@ -1,0 +1,478 @@
+"""Throughput benchmark of the GB300 LR-QAT linear layer (fwd + bwd).
+
+One step = LR-QAT forward and backward of every layer of the workload over one
+batch of T tokens, with the fake-quantized weight rebuilt on chip in each of the
+three GEMMs (Eq. 8 of the paper, checkpointed as in Sec. 3).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+    python bench.py --impl reference ...     # the CPU oracle, timed on host cores
+
+Prints ONE JSON line (rank 0).  With N > 1 (torchrun) every rank runs an
+independent replica of the workload (weak scaling, no collective on the data
+path); the timed region is bracketed by a barrier and device synchronization,
+and the slowest rank's time is used.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+import hashlib
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "LR-QAT linear fwd+bwd tokens/s and TFLOP/s, fraction of GB300 bf16 dense peak"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+GEMM_KERNELS = ("fused_fwd", "fused_dx", "fused_dw")
+KERNEL_SOURCES = {"fused_fwd": "fused_gemm.cu", "fused_dx": "fused_gemm.cu", "fused_dw": "dw.cu"}
+
+
+# --------------------------------------------------------------------------- helpers
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {k: float(p[k]) for k in FALLBACK_PEAKS}, "measured"
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_source_hash(kernel: str) -> str:
+    """sha256 of the sources that define a kernel (its .cu file and the shared device headers)."""
+    csrc = os.path.join(ROOT, "paper_2406_06385_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in (KERNEL_SOURCES[kernel], "ptx.cuh", "quant.cuh", "kernels.h"):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary of this kernel and workload,
+    or None when there is none or the kernel's source changed since it was captured."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    mb = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    ms = re.search(r"source_sha256_16:\s*([0-9a-f]+)", text)
+    if not mb or not ms or ms.group(1) != kernel_source_hash(kernel):
+        return None
+    return float(mb.group(1))
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons every 200 ms while running."""
+
+    FIELDS = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="lrqat_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.out, stderr=subprocess.DEVNULL)
+            time.sleep(0.6)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.out.close()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 11:
+                    continue
+                rows.append(parts)
+        except OSError:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except OSError:
+                pass
+        mine = [r for r in rows if self.uuid and r[1] == self.uuid]
+        rows = mine or [r for r in rows if r[0] == rows[0][0]] if rows else rows
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        busy = [r for r in rows if _num(r[5]) is not None and _num(r[5]) >= 50] or rows
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({n for r in busy for n, v in zip(names, r[7:11]) if v.lower().startswith("active")})
+        sm = [_num(r[2]) for r in busy if _num(r[2]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": _num(busy[0][3]),
+                "power_w_max": max((_num(r[4]) or 0.0) for r in busy), "reasons": reasons, "samples": len(busy)}
+
+
+def _num(s):
+    try:
+        return float(s)
+    except (TypeError, ValueError):
+        return None
+
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def aggregate_over_ranks(ms: float, units: float):
+    """Slowest rank's time and the sum of units over ranks (no-op without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return ms, units
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    u = torch.tensor([units], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+# --------------------------------------------------------------------------- GPU arm
+class GpuWorkload:
+    """Device-resident layers of a workload, prepared through the library (range
+    setting and downcast), with `sets` distinct copies of the step inputs."""
+
+    def __init__(self, wl, sets: int, seed: int = 0):
+        import numpy as np
+        import torch
+        from paper_2406_06385_gb300 import lrqat as LQ
+        from paper_2406_06385_gb300 import workloads as WL
+        self.wl = wl
+        self.T = wl.tokens
+        self.layers = []
+        dev = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).cuda()
+        for li, spec in enumerate(wl.layers):
+            d = WL.make_layer(spec, self.T, seed=seed, layer_index=li)
+            L = LQ.Layer.from_spec(spec)
+            W0 = dev(d.W0)
+            ng = spec.k // spec.group_size if spec.group_size else 1
+            s = torch.empty((spec.m, ng) if spec.group_size else (spec.m,), dtype=torch.float32, device="cuda")
+            LQ.range_minmax(L, W0, s)
+            if spec.phi_format == WL.PHI_QFIXED:
+                phi0 = torch.empty((spec.m, spec.k), dtype=torch.int8, device="cuda")
+            else:
+                phi0 = torch.empty((spec.m, spec.k // 2), dtype=torch.uint8, device="cuda")
+            LQ.downcast(L, W0, s, phi0)
+            del W0
+            X = [dev(d.X_bits) for _ in range(sets)]
+            dY = [dev(d.dY_bits) for _ in range(sets)]
+            s_x = None
+            if spec.act_bits == 8:
+                sx = np.float32(np.float32(np.abs(d.X).max()) / np.float32(127.0))
+                s_x = torch.tensor([sx], dtype=torch.float32, device="cuda")
+            lay = dict(spec=spec, L=L, phi0=phi0, s=s, A=dev(d.A_bits), B=dev(d.B_bits), X=X, dY=dY, s_x=s_x,
+                       X_host=d.X_bits, dY_host=d.dY_bits,
+                       Y=torch.empty((self.T, spec.m), dtype=torch.int16, device="cuda"),
+                       dX=torch.empty((self.T, spec.k), dtype=torch.int16, device="cuda"),
+                       dA=torch.empty((spec.m, spec.r), dtype=torch.float32, device="cuda"),
+                       dB=torch.empty((spec.r, spec.k), dtype=torch.float32, device="cuda"),
+                       ds=torch.empty_like(s))
+            lay["wsf"] = torch.empty(max(LQ.fwd_workspace_bytes(L, self.T), 16), dtype=torch.uint8, device="cuda")
+            lay["wsb"] = torch.empty(LQ.bwd_workspace_bytes(L, self.T), dtype=torch.uint8, device="cuda")
+            self.layers.append(lay)
+            if wl.merge:
+                lay["WZ"] = torch.empty((spec.m, spec.k), dtype=torch.int8, device="cuda")
+        torch.cuda.synchronize()
+        self.sets = sets
+
+    def step(self, i: int, X=None, dY=None):
+        from paper_2406_06385_gb300 import lrqat as LQ
+        j = i % self.sets
+        for lay in self.layers:
+            x = lay["X"][j] if X is None else X[id(lay)]
+            dy = lay["dY"][j] if dY is None else dY[id(lay)]
+            LQ.linear_fwd(lay["L"], self.T, x, lay["phi0"], lay["s"], lay["A"], lay["B"], lay["s_x"], lay["Y"],
+                          lay["wsf"])
+            LQ.linear_bwd(lay["L"], self.T, dy, x, lay["phi0"], lay["s"], lay["A"], lay["B"], lay["s_x"], lay["dX"],
+                          lay["dA"], lay["dB"], lay["ds"], False, lay["wsb"])
+            if self.wl.merge:
+                LQ.merge(lay["L"], lay["phi0"], lay["A"], lay["B"], lay["WZ"])
+
+
+def time_steps(fn, steps: int, warmup: int):
+    import torch
+    for i in range(warmup):
+        fn(i)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(steps):
+        fn(i)
+    e1.record()
+    e1.synchronize()
+    torch.cuda.synchronize()
+    barrier()
+    return e0.elapsed_time(e1)
+
+
+def run_gpu(args):
+    import torch
+    from paper_2406_06385_gb300 import lrqat as LQ
+    from paper_2406_06385_gb300 import workloads as WL
+    from paper_2406_06385_gb300.build import build
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    if rank == 0:
+        build()
+    barrier()
+    LQ.lib()
+    wl = WL.workload(args.workload)
+    T = wl.tokens
+    flops = wl.flops_fwd_bwd()
+    gw = GpuWorkload(wl, sets=args.sets)
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    uuid = getattr(props, "uuid", None)
+    uuid = f"GPU-{uuid}" if uuid is not None and not str(uuid).startswith("GPU-") else (str(uuid) if uuid else None)
+
+    # 1) device-resident timed region (the headline value)
+    with ClockSampler(uuid) as clocks:
+        ms = time_steps(gw.step, args.steps, args.warmup)
+    LQ.get_device_status()
+    ms, units = aggregate_over_ranks(ms, float(T * args.steps))
+    value = units / (ms / 1e3)
+    ms_per_step = ms / args.steps
+
+    # 2) traced pass: per-kernel device time on the launching stream, launch counts
+    LQ.trace_enable(True)
+    ms_traced = time_steps(gw.step, args.steps, 0)
+    trace = LQ.trace_read()
+    LQ.trace_enable(False)
+    LQ.get_device_status()
+    launches = sum(n for n, _ in trace.values())
+    dom = max((k for k in trace if k in GEMM_KERNELS), key=lambda k: trace[k][1])
+    n_dom, ms_dom = trace[dom]
+    # algorithmic work of the kernel: 2 T m k per launch (one launch per layer per step)
+    dom_flops_total = (n_dom / len(gw.layers)) * sum(2.0 * T * l["spec"].m * l["spec"].k for l in gw.layers)
+    dom_flops = dom_flops_total / n_dom
+    avg_ms = ms_dom / n_dom
+    peaks, peak_src = load_peaks()
+    achieved = dom_flops_total / (ms_dom / 1e3) / 1e12
+    traffic = profiled_traffic(dom, args.workload)
+
+    # 3) end to end: pinned host inputs in, step results out, inside the timed region
+    import numpy as np
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16))).pin_memory()
+    hx = {id(l): pin(l["X_host"]) for l in gw.layers}
+    hdy = {id(l): pin(l["dY_host"]) for l in gw.layers}
+    dx = {id(l): l["X"][0] for l in gw.layers}
+    ddy = {id(l): l["dY"][0] for l in gw.layers}
+    outs = {id(l): {n: torch.empty(l[n].shape, dtype=l[n].dtype, pin_memory=True) for n in ("Y", "dX", "dA", "dB", "ds")}
+            for l in gw.layers}
+    h2d = sum(t.numel() * t.element_size() for t in list(hx.values()) + list(hdy.values()))
+    d2h = sum(t.numel() * t.element_size() for o in outs.values() for t in o.values())
+
+    def e2e_step(i):
+        for l in gw.layers:
+            dx[id(l)].copy_(hx[id(l)], non_blocking=True)
+            ddy[id(l)].copy_(hdy[id(l)], non_blocking=True)
+        gw.step(0, X=dx, dY=ddy)
+        for l in gw.layers:
+            for n, t in outs[id(l)].items():
+                t.copy_(l[n], non_blocking=True)
+
+    e2e_steps = max(3, min(args.steps, int(3000.0 / max(ms_per_step, 1e-3) / 2)))
+    ms_e2e = time_steps(e2e_step, e2e_steps, 2)
+    ms_e2e, units_e2e = aggregate_over_ranks(ms_e2e, float(T * e2e_steps))
+
+    clk = clocks.summary()
+    if rank != 0:
+        return None
+    spec0 = wl.layers[0]
+    cfg = {"workload": wl.name, "tokens": T, "layers": [f"{l.name}:{l.m}x{l.k}" for l in wl.layers],
+           "r": spec0.r, "alpha": spec0.alpha, "bits": spec0.bits,
+           "granularity": "per-channel" if spec0.group_size == 0 else f"g{spec0.group_size}",
+           "phi": "Q%d.%d int8" % (spec0.bits, 8 - spec0.bits) if spec0.phi_format == 0 else f"INT-{spec0.bits} packed",
+           "activations": "int8 per-tensor" if spec0.act_bits == 8 else "bf16",
+           "merge": wl.merge, "parallelism": "replicas" if world > 1 else "single",
+           "l2": f"inputs rotate over {args.sets} device copies ({args.sets * sum((l['X'][0].numel() + l['dY'][0].numel()) * 2 for l in gw.layers) / 2**20:.0f} MiB) > L2"}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded normal weights/activations, LLaMA-shaped layers)",
+        "config": cfg,
+        "tflops": flops * args.steps * world / (ms / 1e3) / 1e12,
+        "frac_of_bf16_peak": {"sustained": flops * args.steps * world / (ms / 1e3) / 1e12 / peaks["bf16_tflops_sustained"],
+                              "burst": flops * args.steps * world / (ms / 1e3) / 1e12 / peaks["bf16_tflops"],
+                              "peaks": peak_src},
+        "roofline": {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops_sustained"],
+                     "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops_sustained"], "traffic": traffic,
+                     "peak_kind": f"bf16 dense, sustained ({peak_src})",
+                     "launch_ms": avg_ms, "flops_per_launch": dom_flops},
+        "kernels": {k: {"launches": n, "total_ms": t, "share": t / sum(v[1] for v in trace.values())}
+                    for k, (n, t) in sorted(trace.items(), key=lambda kv: -kv[1][1])},
+        "traced_ms_per_step": ms_traced / args.steps,
+        "gpu_launches": launches,
+        "e2e": {"value": units_e2e / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+        "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
+                   "samples": clk["samples"], "power_w_max": clk.get("power_w_max")},
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, budget_s=args.cpu_budget)
+    return line
+
+
+# --------------------------------------------------------------------------- CPU oracle
+def _oracle_sample(wl, rows: int, tokens: int):
+    """One layer's data cut to `rows` output channels and `tokens` tokens (a smaller
+    LR-QAT layer with the same per-element arithmetic), prepared for the oracle."""
+    import numpy as np
+    import oracle as O
+    from paper_2406_06385_gb300 import workloads as WL
+    spec = wl.layers[0]
+    d = WL.make_layer(spec, wl.tokens, seed=0, layer_index=0)
+    OL = O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+    s0 = O.minmax_scale(d.W0, OL)
+    phi0 = O.downcast(d.W0, s0, OL)
+    sub = O.Layer(rows, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+    X = d.X[:tokens]
+    s_x = float(np.float32(np.abs(d.X).max()) / np.float32(127.0)) if spec.act_bits == 8 else None
+    return dict(OL=sub, phi0=phi0[:rows], s=s0[:rows], A=d.A[:rows], B=d.B, X=X, dY=d.dY[:tokens, :rows], s_x=s_x,
+                frac=rows / spec.m, tokens=tokens, m=spec.m)
+
+
+def _oracle_step(smp):
+    import oracle as O
+    O.linear_fwd(smp["X"], smp["phi0"], smp["s"], smp["A"], smp["B"], smp["OL"], smp["s_x"])
+    O.linear_bwd(smp["dY"], smp["X"], smp["phi0"], smp["s"], smp["A"], smp["B"], smp["OL"], smp["s_x"])
+
+
+def _calibrated_sample(wl, budget_s: float):
+    """A (rows, tokens) cut of the workload's first layer whose oracle step takes
+    between budget_s / 2 and budget_s seconds (cost roughly doubles with either)."""
+    rows, tokens = 128, min(256, wl.tokens)
+    smp = _oracle_sample(wl, rows, tokens)
+    t0 = time.perf_counter()
+    _oracle_step(smp)
+    t = time.perf_counter() - t0
+    m = wl.layers[0].m
+    while t < budget_s / 2:
+        if tokens < wl.tokens:
+            tokens = min(wl.tokens, tokens * 2)
+        elif rows < m:
+            rows = min(m, rows * 2)
+        else:
+            break
+        t *= 2
+    return _oracle_sample(wl, rows, tokens)
+
+
+def cpu_baseline(wl, budget_s: float = 15.0):
+    """The oracle as it stands, on this host's cores, over a bounded sample of the workload."""
+    smp = _calibrated_sample(wl, budget_s / 3)
+    reps = 0
+    t0 = time.perf_counter()
+    while True:
+        _oracle_step(smp)
+        reps += 1
+        dt = time.perf_counter() - t0
+        if dt >= budget_s or reps >= 20:
+            break
+    nlayers = len(wl.layers)
+    value = smp["tokens"] * smp["frac"] * reps / dt / nlayers
+    return {"value": value, "unit": UNIT, "cores": len(os.sched_getaffinity(0)), "kind": "oracle",
+            "seconds": dt,
+            "sample": (f"{reps} oracle fwd+bwd steps of the first layer ({wl.layers[0].m}x{wl.layers[0].k}) cut to "
+                       f"{smp['OL'].m} output channels and {smp['tokens']} tokens (float64 numpy, BLAS on all host "
+                       f"cores); value = tokens x (rows/m) x steps / time / {nlayers} layer(s), i.e. full-workload "
+                       f"tokens/s assuming equal per-layer cost")}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return None
+    from paper_2406_06385_gb300 import workloads as WL
+    wl = WL.workload(args.workload)
+    per_step = max(0.02, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    smp = _calibrated_sample(wl, per_step)
+    for _ in range(args.warmup):
+        _oracle_step(smp)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        _oracle_step(smp)
+    dt = time.perf_counter() - t0
+    nlayers = len(wl.layers)
+    value = smp["tokens"] * smp["frac"] * args.steps / dt / nlayers
+    cores = len(os.sched_getaffinity(0))
+    sample = (f"each step: first layer ({wl.layers[0].m}x{wl.layers[0].k}) cut to {smp['OL'].m} output channels "
+              f"and {smp['tokens']} tokens; value = tokens x (rows/m) / time / {nlayers} layer(s)")
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "tokens": wl.tokens}, "impl": "reference",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+
+
+def main(argv=None):
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", choices=("lrqat", "reference"), default="lrqat")
+    p.add_argument("--workload", default="llama2_7b_attn")
+    p.add_argument("--sets", type=int, default=4, help="distinct device copies of the step inputs (L2 rotation)")
+    p.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    args = p.parse_args(argv)
+    if args.warmup < 3:
+        p.error("--warmup must be >= 3")
+    line = run_reference(args) if args.impl == "reference" else run_gpu(args)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    try:
+        import torch.distributed as dist
+        if dist.is_available() and dist.is_initialized():
+            dist.destroy_process_group()
+    except Exception:
+        pass
+
+
+if __name__ == "__main__":
+    main()

@@ -138,6 +138,19 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
  * wait gave up since the last call) or LRQAT_ERR_CUDA. */
 int lrqat_get_device_status(lrqat_stream_t stream);
 
+/* ---------------------------------------------------------------------------
+ * Tracing (instrumentation; not part of the method).  While enabled, every
+ * kernel the library enqueues is bracketed by a pair of CUDA events recorded on
+ * the stream it runs on, and counted per kernel name.  Tracing is off by
+ * default and costs nothing then.
+ * ------------------------------------------------------------------------- */
+/* enable = 1 starts (and clears) a trace, 0 stops recording. */
+int lrqat_trace_enable(int enable);
+/* Synchronizes the recorded events and reports up to `max_entries` kernels:
+ * names[i] (static strings), launches[i] and total device milliseconds[i];
+ * *count receives the number of distinct kernels seen.  Host arrays. */
+int lrqat_trace_read(int max_entries, const char** names, int64_t* launches, double* total_ms, int* count);
+
 #ifdef __cplusplus
 }
 #endif

@@ -152,6 +152,14 @@ __global__ void pad_rows64_kernel(const uint16_t* __restrict__ A, int64_t m, int
   out[e] = c < r ? A[i * r + c] : static_cast<uint16_t>(0);
 }
 
+__global__ void pad_rows_kernel(const uint16_t* __restrict__ src, int rows, int rows_pad, int64_t cols,
+                                uint16_t* __restrict__ out) {
+  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  if (e >= static_cast<int64_t>(rows_pad) * cols) return;
+  const int c = static_cast<int>(e / cols);
+  out[e] = c < rows ? src[e] : static_cast<uint16_t>(0);
+}
+
 __global__ void transpose_pad64_kernel(const uint16_t* __restrict__ B, int r, int64_t k, uint16_t* __restrict__ out) {
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (e >= k * 64) return;
@@ -264,6 +272,13 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
 
 cudaError_t launch_pad_rows64(const uint16_t* A, int64_t m, int r, uint16_t* out, cudaStream_t stream) {
   pad_rows64_kernel<<<blocks_for(m * 64, kThreads), kThreads, 0, stream>>>(A, m, r, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pad_rows(const uint16_t* src, int rows, int rows_pad, int64_t cols, uint16_t* out,
+                            cudaStream_t stream) {
+  pad_rows_kernel<<<blocks_for(static_cast<int64_t>(rows_pad) * cols, kThreads), kThreads, 0, stream>>>(src, rows, rows_pad,
+                                                                                                      cols, out);
   return cudaGetLastError();
 }
 

@@ -22,6 +22,9 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
                              uint32_t* mask, cudaStream_t stream);
 // out[i][c] = c < r ? A[i][c] : 0 for c < 64 (A: [m, r] bf16 -> [m, 64]).
 cudaError_t launch_pad_rows64(const uint16_t* A, int64_t m, int r, uint16_t* out, cudaStream_t stream);
+// out[c][j] = c < rows ? src[c][j] : 0 for c < rows_pad (zero-padded rows).
+cudaError_t launch_pad_rows(const uint16_t* src, int rows, int rows_pad, int64_t cols, uint16_t* out,
+                            cudaStream_t stream);
 // out[j][c] = c < r ? B[c][j] : 0 for c < 64 (B: [r, k] bf16 -> [k, 64]).
 cudaError_t launch_transpose_pad64(const uint16_t* B, int r, int64_t k, uint16_t* out, cudaStream_t stream);
 // out[c][i] = c < r ? A[i][c] : 0 for c < r16 (A: [m, r] -> [r16, m]).

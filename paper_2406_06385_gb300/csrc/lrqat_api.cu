@@ -11,6 +11,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #include "kernels.h"
 #include "lrqat.h"
@@ -147,6 +148,67 @@ int validate_layer(const lrqat_layer* L) {
     if (st_ != LRQAT_OK) return st_; \
   } while (0)
 
+// ------------------------------------------------------------------ tracing --
+struct TraceRec {
+  const char* name;
+  int kernels;
+  cudaEvent_t start, stop;
+};
+std::mutex g_trace_mu;
+bool g_trace_on = false;
+std::vector<TraceRec> g_trace;
+std::vector<cudaEvent_t> g_event_pool;
+
+cudaEvent_t trace_event() {
+  if (!g_event_pool.empty()) {
+    cudaEvent_t e = g_event_pool.back();
+    g_event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+void trace_clear_locked() {
+  for (auto& r : g_trace) {
+    if (r.start) g_event_pool.push_back(r.start);
+    if (r.stop) g_event_pool.push_back(r.stop);
+  }
+  g_trace.clear();
+}
+
+// Brackets the kernels enqueued in its scope with events on `stream` while tracing is on.
+class TraceScope {
+ public:
+  TraceScope(const char* name, int kernels, cudaStream_t stream) : stream_(stream) {
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    if (!g_trace_on) return;
+    rec_.name = name;
+    rec_.kernels = kernels;
+    rec_.start = trace_event();
+    rec_.stop = trace_event();
+    if (rec_.start && rec_.stop && cudaEventRecord(rec_.start, stream) == cudaSuccess) active_ = true;
+  }
+  ~TraceScope() {
+    if (!active_) return;
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    if (cudaEventRecord(rec_.stop, stream_) == cudaSuccess) g_trace.push_back(rec_);
+  }
+
+ private:
+  cudaStream_t stream_;
+  TraceRec rec_{};
+  bool active_ = false;
+};
+
+#define LRQAT_LAUNCH(name, nkernels, stream, expr, what)        \
+  do {                                                          \
+    TraceScope ts_(name, nkernels, stream);                     \
+    cudaError_t e_ = (expr);                                    \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what);          \
+  } while (0)
+
 // Carves aligned sub-buffers out of a caller-provided workspace.
 struct Carver {
   uintptr_t base;
@@ -265,8 +327,9 @@ int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrq
   LRQAT_CHECK_PTR(W0, "W0");
   LRQAT_CHECK_PTR(s0, "s0");
   const lrqat_layer& L = *layer;
-  LRQAT_CUDA(launch_range_minmax(W0, L.m, L.k, L.group_size, (1 << (L.bits - 1)) - 1, s0, stream),
-             "range_minmax launch");
+  LRQAT_LAUNCH("range_minmax", 1, stream,
+               launch_range_minmax(W0, L.m, L.k, L.group_size, (1 << (L.bits - 1)) - 1, s0, stream),
+               "range_minmax launch");
   return LRQAT_OK;
 }
 
@@ -276,9 +339,10 @@ int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, v
   LRQAT_CHECK_PTR(s0, "s0");
   LRQAT_CHECK_PTR(Phi0, "Phi0");
   const lrqat_layer& L = *layer;
-  LRQAT_CUDA(launch_downcast(W0, s0, L.m, L.k, L.group_size, L.bits, L.phi_format == LRQAT_PHI_INT_PACKED, Phi0,
-                             stream),
-             "downcast launch");
+  LRQAT_LAUNCH("downcast", 1, stream,
+               launch_downcast(W0, s0, L.m, L.k, L.group_size, L.bits, L.phi_format == LRQAT_PHI_INT_PACKED, Phi0,
+                               stream),
+               "downcast launch");
   return LRQAT_OK;
 }
 
@@ -312,11 +376,12 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   FwdWs ws;
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
-  LRQAT_CUDA(launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
-  LRQAT_CUDA(launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
+  LRQAT_LAUNCH("pad_rows64", 1, stream, launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
+  LRQAT_LAUNCH("transpose_pad64", 1, stream, launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
   const uint16_t* tok = X;
   if (L.act_bits == 8) {
-    LRQAT_CUDA(launch_act_quant(X, T, L.k, s_x, ws.x_codes, nullptr, stream), "activation quantizer");
+    LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, ws.x_codes, nullptr, stream),
+                 "activation quantizer");
     tok = ws.x_codes;
   }
   CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
@@ -347,9 +412,10 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   a.status = dev->status;
   a.timeout_ns = kWaitTimeoutNs;
   const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
-  LRQAT_CUDA(launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, L.phi_format == LRQAT_PHI_INT_PACKED,
-                          tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
-             "fused forward launch");
+  LRQAT_LAUNCH("fused_fwd", 1, stream,
+               launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, L.phi_format == LRQAT_PHI_INT_PACKED,
+                            tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+               "fused forward launch");
   return LRQAT_OK;
 }
 
@@ -391,16 +457,16 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   bwd_ws_layout(L, T, plan, workspace, &ws);
   const int r16 = round16(L.r);
   const bool packed = L.phi_format == LRQAT_PHI_INT_PACKED;
-  LRQAT_CUDA(launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
-  LRQAT_CUDA(launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
-  LRQAT_CUDA(launch_transpose_rows(A, L.m, L.r, r16, ws.at, stream), "transpose A");
-  LRQAT_CUDA(cudaMemsetAsync(ws.b_pad, 0, static_cast<size_t>(r16) * L.k * 2, stream), "clear B pad");
-  LRQAT_CUDA(cudaMemcpyAsync(ws.b_pad, B, static_cast<size_t>(L.r) * L.k * 2, cudaMemcpyDeviceToDevice, stream),
-             "copy B");
-  LRQAT_CUDA(launch_phi_transpose(Phi0, L.m, L.k, packed, ws.phit, stream), "transpose Phi0");
+  LRQAT_LAUNCH("pad_rows64", 1, stream, launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
+  LRQAT_LAUNCH("transpose_pad64", 1, stream, launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
+  LRQAT_LAUNCH("transpose_rows", 1, stream, launch_transpose_rows(A, L.m, L.r, r16, ws.at, stream), "transpose A");
+  LRQAT_LAUNCH("pad_rows", 1, stream, launch_pad_rows(B, L.r, r16, L.k, ws.b_pad, stream), "pad B");
+  LRQAT_LAUNCH("phi_transpose", 1, stream, launch_phi_transpose(Phi0, L.m, L.k, packed, ws.phit, stream),
+               "transpose Phi0");
   const uint16_t* xop = X;
   if (L.act_bits == 8) {
-    LRQAT_CUDA(launch_act_quant(X, T, L.k, s_x, ws.x_codes, ws.xmask, stream), "activation quantizer");
+    LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, ws.x_codes, ws.xmask, stream),
+                 "activation quantizer");
     xop = ws.x_codes;
   }
   const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
@@ -436,7 +502,8 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
     const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
-    LRQAT_CUDA(launch_fused(FUSED_DX, 0, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream), "fused dX launch");
+    LRQAT_LAUNCH("fused_dx", 1, stream, launch_fused(FUSED_DX, 0, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+                 "fused dX launch");
   }
   // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
   {
@@ -477,8 +544,9 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
     const int grid = plan.units < dev->sms ? plan.units : dev->sms;
-    LRQAT_CUDA(launch_dw(packed, tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, a, grid, stream),
-               "fused dW launch");
+    LRQAT_LAUNCH("fused_dw", 1, stream,
+                 launch_dw(packed, tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, a, grid, stream),
+                 "fused dW launch");
   }
   ReduceArgs ra{};
   ra.dA_part = ws.dA_part;
@@ -496,7 +564,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   ra.group_size = L.group_size;
   ra.lr = static_cast<float>(static_cast<double>(L.alpha) / L.r);
   ra.accumulate = accumulate ? 1 : 0;
-  LRQAT_CUDA(launch_reduce(ra, stream), "gradient reduction");
+  LRQAT_LAUNCH("reduce_grads", 3, stream, launch_reduce(ra, stream), "gradient reduction");
   return LRQAT_OK;
 }
 
@@ -509,8 +577,9 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
   if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
   LRQAT_CHECK_PTR(W_Z, "W_Z");
   const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
-  LRQAT_CUDA(launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format == LRQAT_PHI_INT_PACKED, q, W_Z, stream),
-             "merge launch");
+  LRQAT_LAUNCH("merge", 1, stream,
+               launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format == LRQAT_PHI_INT_PACKED, q, W_Z, stream),
+               "merge launch");
   return LRQAT_OK;
 }
 
@@ -523,6 +592,45 @@ int lrqat_get_device_status(lrqat_stream_t stream) {
   if (h != 0) {
     LRQAT_CUDA(cudaMemset(dev->status, 0, sizeof(int)), "clear device status");
     return fail(LRQAT_ERR_TIMEOUT, "a kernel's bounded wait gave up (status word 0x%x)", h);
+  }
+  return LRQAT_OK;
+}
+
+int lrqat_trace_enable(int enable) {
+  std::lock_guard<std::mutex> lock(g_trace_mu);
+  if (enable) trace_clear_locked();
+  g_trace_on = enable != 0;
+  return LRQAT_OK;
+}
+
+int lrqat_trace_read(int max_entries, const char** names, int64_t* launches, double* total_ms, int* count) {
+  if (max_entries < 0 || (max_entries > 0 && (!names || !launches || !total_ms)) || !count)
+    return fail(LRQAT_ERR_INVALID_ARG, "trace_read: bad output arrays");
+  std::lock_guard<std::mutex> lock(g_trace_mu);
+  std::vector<const char*> keys;
+  std::vector<int64_t> n;
+  std::vector<double> ms;
+  for (auto& r : g_trace) {
+    cudaError_t e = cudaEventSynchronize(r.stop);
+    if (e != cudaSuccess) return cuda_fail(e, "trace_read: cudaEventSynchronize");
+    float t = 0.0f;
+    e = cudaEventElapsedTime(&t, r.start, r.stop);
+    if (e != cudaSuccess) return cuda_fail(e, "trace_read: cudaEventElapsedTime");
+    size_t i = 0;
+    while (i < keys.size() && std::strcmp(keys[i], r.name) != 0) ++i;
+    if (i == keys.size()) {
+      keys.push_back(r.name);
+      n.push_back(0);
+      ms.push_back(0.0);
+    }
+    n[i] += r.kernels;
+    ms[i] += t;
+  }
+  *count = static_cast<int>(keys.size());
+  for (int i = 0; i < max_entries && i < static_cast<int>(keys.size()); ++i) {
+    names[i] = keys[i];
+    launches[i] = n[i];
+    total_ms[i] = ms[i];
   }
   return LRQAT_OK;
 }

@@ -64,6 +64,11 @@ def lib() -> ctypes.CDLL:
             fn = getattr(L, name)
             fn.argtypes = args
             fn.restype = ctypes.c_int
+        L.lrqat_trace_enable.argtypes = [ip]
+        L.lrqat_trace_enable.restype = ctypes.c_int
+        L.lrqat_trace_read.argtypes = [ip, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_int64),
+                                       ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)]
+        L.lrqat_trace_read.restype = ctypes.c_int
         for name in ("lrqat_fwd_workspace_bytes", "lrqat_bwd_workspace_bytes"):
             fn = getattr(L, name)
             fn.argtypes = [lp, i64]
@@ -128,3 +133,17 @@ def merge(layer: Layer, Phi0, A, B, W_Z, stream=None) -> None:
 
 def get_device_status(stream=None) -> None:
     _check(lib().lrqat_get_device_status(_stream(stream)))
+
+
+def trace_enable(enable: bool = True) -> None:
+    _check(lib().lrqat_trace_enable(1 if enable else 0))
+
+
+def trace_read(max_entries: int = 32):
+    """Per-kernel {name: (launches, total_ms)} recorded since trace_enable(True)."""
+    names = (ctypes.c_char_p * max_entries)()
+    launches = (ctypes.c_int64 * max_entries)()
+    ms = (ctypes.c_double * max_entries)()
+    count = ctypes.c_int(0)
+    _check(lib().lrqat_trace_read(max_entries, names, launches, ms, ctypes.byref(count)))
+    return {names[i].decode(): (int(launches[i]), float(ms[i])) for i in range(min(count.value, max_entries))}
