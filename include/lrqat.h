@@ -107,6 +107,28 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
                      const float* s, const uint16_t* A, const uint16_t* B, const float* s_x,
                      uint16_t* Y, void* workspace, size_t workspace_bytes, lrqat_stream_t stream);
 
+/* Allocation-free forward (no counterpart in the paper: this is a deployment
+ * convenience).  Same computation and arguments as lrqat_linear_fwd, but the
+ * scratch comes from a fixed array inside the library instead of a caller
+ * workspace, for callers that cannot allocate device memory: runtimes that own
+ * all device memory and hand an operator only its inputs and outputs, or that
+ * forbid allocation after start-up because cudaMalloc can synchronize the
+ * device and stall other work.
+ *   - The array holds LRQAT_FWD_NOALLOC_SCRATCH_BYTES bytes; every device that
+ *     loads the library keeps it until the process exits.  A layer/T whose
+ *     scratch (lrqat_fwd_workspace_bytes) exceeds it is rejected with
+ *     LRQAT_ERR_WORKSPACE (in practice: act_bits = 8 with large T * k).
+ *   - The first call on a device looks the array's device address up (with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls share the one array: calls that overlap on the GPU (different
+ *     streams, or host threads without ordering) race; serialize them.
+ *   - Every call rewrites the parts of the scratch it reads, so nothing has to
+ *     be cleared between calls.  No device memory is allocated or freed. */
+#define LRQAT_FWD_NOALLOC_SCRATCH_BYTES ((size_t)4 << 20)
+int lrqat_linear_fwd_noalloc(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0,
+                             const float* s, const uint16_t* A, const uint16_t* B, const float* s_x,
+                             uint16_t* Y, lrqat_stream_t stream);
+
 /* Bytes of workspace lrqat_linear_bwd needs for T tokens. */
 size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
 

@@ -316,11 +316,69 @@ int phi_map(CUtensorMap* map, const lrqat_layer& L, const void* phi0, uint32_t b
 }  // namespace
 }  // namespace lrqat
 
+// Scratch of lrqat_linear_fwd_noalloc, for callers that cannot allocate device
+// memory (runtimes that own all device memory and give an operator only its
+// inputs and outputs, or that forbid allocation after start-up because
+// cudaMalloc can synchronize the device).  It is part of the library image, so
+// every device that loads the library holds these bytes until the process exits.
+static __device__ __align__(256) unsigned char g_fwd_noalloc_scratch[LRQAT_FWD_NOALLOC_SCRATCH_BYTES];
+
+namespace lrqat {
+namespace {
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  In host code the
+// array's name is only a host-side stand-in, so the address is looked up once per
+// device (with that device current) and cached.
+int noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(LRQAT_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_fwd_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(forward scratch)");
+    g_noalloc_addr[dev] = p;
+  }
+  *out = g_noalloc_addr[dev];
+  return LRQAT_OK;
+}
+
+}  // namespace
+}  // namespace lrqat
+
 using namespace lrqat;
 
 extern "C" {
 
 const char* lrqat_last_error(void) { return t_last_error.c_str(); }
+
+// The forward of lrqat_linear_fwd with its scratch taken from the fixed array
+// above instead of a caller workspace.  The first call on a device performs the
+// address look-up.  Calls share the array, so calls that overlap on the GPU
+// race; each call rewrites every scratch byte it later reads (padded adapter
+// copies, activation codes), so nothing needs clearing between calls.  Nothing
+// is allocated or freed here or in lrqat_linear_fwd.
+int lrqat_linear_fwd_noalloc(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0,
+                             const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y,
+                             lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
+  if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
+  const size_t need = fwd_ws_layout(*layer, T, nullptr, nullptr);
+  if (need > LRQAT_FWD_NOALLOC_SCRATCH_BYTES)
+    return fail(LRQAT_ERR_WORKSPACE,
+                "lrqat_linear_fwd_noalloc: this layer and T need %zu bytes of scratch but the fixed scratch holds "
+                "%zu bytes; use lrqat_linear_fwd with a workspace",
+                need, (size_t)LRQAT_FWD_NOALLOC_SCRATCH_BYTES);
+  void* scratch = nullptr;
+  LRQAT_TRY(noalloc_scratch(&scratch));
+  return lrqat_linear_fwd(layer, T, X, Phi0, s, A, B, s_x, Y, scratch, LRQAT_FWD_NOALLOC_SCRATCH_BYTES, stream);
+}
 
 int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrqat_stream_t stream) {
   LRQAT_TRY(validate_layer(layer));

@@ -56,6 +56,7 @@ def lib() -> ctypes.CDLL:
             "lrqat_range_minmax": [lp, vp, vp, vp],
             "lrqat_downcast": [lp, vp, vp, vp, vp],
             "lrqat_linear_fwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+            "lrqat_linear_fwd_noalloc": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp],
             "lrqat_linear_bwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ip, vp, sz, vp],
             "lrqat_merge": [lp, vp, vp, vp, vp, vp],
             "lrqat_get_device_status": [vp],
@@ -117,6 +118,12 @@ def linear_fwd(layer: Layer, T: int, X, Phi0, s, A, B, s_x, Y, workspace, stream
     nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
     _check(lib().lrqat_linear_fwd(ctypes.byref(layer), T, _ptr(X), _ptr(Phi0), _ptr(s), _ptr(A), _ptr(B), _ptr(s_x),
                                   _ptr(Y), _ptr(workspace), nbytes, _stream(stream)))
+
+
+def linear_fwd_noalloc(layer: Layer, T: int, X, Phi0, s, A, B, s_x, Y, stream=None) -> None:
+    """Forward that takes its scratch from the library's fixed device array (no workspace argument)."""
+    _check(lib().lrqat_linear_fwd_noalloc(ctypes.byref(layer), T, _ptr(X), _ptr(Phi0), _ptr(s), _ptr(A), _ptr(B),
+                                          _ptr(s_x), _ptr(Y), _stream(stream)))
 
 
 def linear_bwd(layer: Layer, T: int, dY, X, Phi0, s, A, B, s_x, dX, dA, dB, ds, accumulate: bool, workspace,
