@@ -9,9 +9,10 @@
 //   ds_partial = sum_j G * c
 // The partials of dA, dB and ds are reduced deterministically by a later kernel.
 //
-// Roles (320 threads): warp 0 issues TMA, warp 1 issues tcgen05 MMAs and owns
-// TMEM, warps 2..9 run the epilogue.  Work units (row block, column tile, token
-// split) are distributed persistently over the CTAs.
+// Roles (416 threads): warp 0 loads the epilogue operands, warp 1 issues tcgen05
+// MMAs and owns TMEM, warps 2..9 run the epilogue, warps 10..12 fill the pipeline
+// stages with TMA.  Work units (row block, column tile, token split) are
+// distributed persistently over the CTAs.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -23,20 +24,27 @@
 namespace lrqat {
 namespace {
 
-constexpr int NS = 4;
+constexpr int NS = 6;
 constexpr int BKT = 32;                        // tokens per pipeline stage
-constexpr int NUM_THREADS = 320;
 constexpr int NUM_EPI_WARPS = 8;
+// TMA instructions issued by one warp are processed one after another, so the
+// pipeline stages are filled round-robin by NUM_LOADERS warps (one box per lane);
+// warp 0 loads the per-unit epilogue operands.
+constexpr int NUM_LOADERS = 3;
+constexpr int FIRST_LOADER = 2 + NUM_EPI_WARPS;
+constexpr int NUM_THREADS = 32 * (FIRST_LOADER + NUM_LOADERS);
 
 constexpr uint32_t BOX_BYTES = 64 * 32 * 2;    // one 64-column x 32-token bf16 box (SW128)
 constexpr uint32_t STAGE_DY = 2 * BOX_BYTES;   // 128 rows i
 constexpr uint32_t STAGE_BYTES = STAGE_DY + 4 * BOX_BYTES;   // + up to 256 columns j
 constexpr uint32_t OFF_STAGES = 0;
-constexpr uint32_t OFF_APAD = OFF_STAGES + NS * STAGE_BYTES;   // A (padded to 64 cols), 128 rows, SW128
-constexpr uint32_t OFF_AT = OFF_APAD + 16384;                  // A^T: 2 boxes of r16 rows x 64 cols
+// A^T [r16 rows t, 128 columns i] (2 boxes of 64 i) serves as the MN-major A operand of
+// the low-rank tile and the K-major B operand of dU^T A; B (padded) [r16 rows t, 128
+// columns j] serves as the MN-major B operand of the low-rank tile and the K-major B
+// operand of dU B^T.
+constexpr uint32_t OFF_AT = OFF_STAGES + NS * STAGE_BYTES;     // A^T: 2 boxes of r16 rows x 64 cols
 constexpr uint32_t OFF_PHI = OFF_AT + 16384;                   // Phi0 chunk 128 x 128 (packed: 128 x 64 B)
-constexpr uint32_t OFF_BT = OFF_PHI + 16384;                   // B^T (padded) chunk 128 rows, SW128
-constexpr uint32_t OFF_BP = OFF_BT + 16384;                    // B (padded) chunk: 2 boxes of r16 rows x 64 cols
+constexpr uint32_t OFF_BP = OFF_PHI + 16384;                   // B (padded) chunk: 2 boxes of r16 rows x 64 cols
 constexpr uint32_t OFF_DU = OFF_BP + 16384;                    // dU chunk: 2 atom columns of 128 rows x 128 B
 constexpr uint32_t SMEM_TILES = OFF_DU + 32768;
 constexpr uint32_t SMEM_BYTES = SMEM_TILES + 1024;
@@ -88,8 +96,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
 template <bool PACKED>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     dw_kernel(const __grid_constant__ CUtensorMap tm_dy, const __grid_constant__ CUtensorMap tm_x,
-              const __grid_constant__ CUtensorMap tm_apad, const __grid_constant__ CUtensorMap tm_at,
-              const __grid_constant__ CUtensorMap tm_phi, const __grid_constant__ CUtensorMap tm_bt,
+              const __grid_constant__ CUtensorMap tm_at, const __grid_constant__ CUtensorMap tm_phi,
               const __grid_constant__ CUtensorMap tm_b, const DwArgs args) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t bars[NUM_BARS];
@@ -129,34 +136,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const WaitCtl ctl{&abort_s, args.status, args.timeout_ns};
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ---------------------------------------- epilogue operands (per unit/chunk)
     if (lane == 0) {
-      prefetch_tensormap(&tm_dy);
-      prefetch_tensormap(&tm_x);
-      const uint32_t stage_tx = STAGE_DY + 2u * args.nchunks * BOX_BYTES;
-      const uint32_t ef_tx = 16384u + 2u * rbox;
-      const uint32_t ec_tx = (PACKED ? 8192u : 16384u) + 16384u + 2u * rbox;
-      uint32_t g = 0, it = 0, cc = 0;
+      const uint32_t ef_tx = 2u * rbox;
+      const uint32_t ec_tx = (PACKED ? 8192u : 16384u) + 2u * rbox;
+      uint32_t it = 0, cc = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
         const Unit w = decode_unit(u, args);
-        for (int step = 0; step < w.nsteps; ++step) {
-          const uint32_t s = g % NS, ph = (g / NS) & 1u;
-          if (!(ok = wait_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1))) break;
-          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
-          const uint32_t fb = bar(BAR_FULL + s);
-          const int tok = w.t0 + step * BKT;
-          mbar_arrive_expect_tx(fb, stage_tx);
-          tma_load_2d(st, &tm_dy, w.ib * 128, tok, fb);
-          tma_load_2d(st + BOX_BYTES, &tm_dy, w.ib * 128 + 64, tok, fb);
-          for (int b = 0; b < 2 * args.nchunks; ++b)
-            tma_load_2d(st + STAGE_DY + b * BOX_BYTES, &tm_x, w.jt * BN + 64 * b, tok, fb);
-          ++g;
-        }
-        if (!ok) break;
         if (!(ok = wait_bounded(bar(BAR_EFEMPTY), (it & 1u) ^ 1u, ctl, 2))) break;
         mbar_arrive_expect_tx(bar(BAR_EFFULL), ef_tx);
-        tma_load_2d(smem + OFF_APAD, &tm_apad, 0, w.ib * 128, bar(BAR_EFFULL));
         tma_load_2d(smem + OFF_AT, &tm_at, w.ib * 128, 0, bar(BAR_EFFULL));
         tma_load_2d(smem + OFF_AT + rbox, &tm_at, w.ib * 128 + 64, 0, bar(BAR_EFFULL));
         ++it;
@@ -165,46 +154,86 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const int j0 = w.jt * BN + 128 * c;
           mbar_arrive_expect_tx(bar(BAR_ECFULL), ec_tx);
           tma_load_2d(smem + OFF_PHI, &tm_phi, PACKED ? j0 / 2 : j0, w.ib * 128, bar(BAR_ECFULL));
-          tma_load_2d(smem + OFF_BT, &tm_bt, 0, j0, bar(BAR_ECFULL));
           tma_load_2d(smem + OFF_BP, &tm_b, j0, 0, bar(BAR_ECFULL));
           tma_load_2d(smem + OFF_BP + rbox, &tm_b, j0 + 64, 0, bar(BAR_ECFULL));
           ++cc;
         }
       }
-      for (uint32_t s = 0; s < NS && s < g; ++s) {
-        const uint32_t last = s + NS * ((g - 1 - s) / NS);
-        drain_wait(bar(BAR_FULL + s), (last / NS) & 1u, args.timeout_ns);
-      }
       if (it > 0) drain_wait(bar(BAR_EFFULL), (it - 1) & 1u, args.timeout_ns);
       if (cc > 0) drain_wait(bar(BAR_ECFULL), (cc - 1) & 1u, args.timeout_ns);
+    }
+  } else if (warp >= FIRST_LOADER) {
+    // ------------------------------------------------ pipeline stage loaders
+    // Loader t fills the global steps g = t, t + NUM_LOADERS, ...; lane b issues box b
+    // (boxes 0-1: dY columns i, boxes 2..: X columns j).
+    const uint32_t t = warp - FIRST_LOADER;
+    if (lane == 0) {
+      prefetch_tensormap(&tm_dy);
+      prefetch_tensormap(&tm_x);
+    }
+    const uint32_t stage_tx = STAGE_DY + 2u * args.nchunks * BOX_BYTES;
+    const int nbox = 2 + 2 * args.nchunks;
+    uint32_t g = 0, last_g = 0xffffffffu;
+    bool ok = true;
+    for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
+      const Unit w = decode_unit(u, args);
+      for (int step = 0; step < w.nsteps; ++step, ++g) {
+        if (g % NUM_LOADERS != t) continue;
+        const uint32_t s = g % NS, ph = (g / NS) & 1u;
+        if (lane == 0) ok = wait_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
+        const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
+        const uint32_t fb = bar(BAR_FULL + s);
+        if (lane == 0) mbar_arrive_expect_tx(fb, stage_tx);
+        __syncwarp();
+        const int tok = w.t0 + step * BKT;
+        if (lane < 2) tma_load_2d(st + lane * BOX_BYTES, &tm_dy, w.ib * 128 + 64 * lane, tok, fb);
+        else if (lane < nbox)
+          tma_load_2d(st + STAGE_DY + (lane - 2) * BOX_BYTES, &tm_x, w.jt * BN + 64 * (lane - 2), tok, fb);
+        last_g = g;
+      }
+    }
+    // Let every issued copy land before the CTA can exit (the slots this loader used).
+    if (lane == 0 && last_g != 0xffffffffu) {
+      for (uint32_t k = 0; k < NS && k <= last_g; ++k) {
+        const uint32_t gg = last_g - k;
+        if (gg % NUM_LOADERS == t) drain_wait(bar(BAR_FULL + gg % NS), (gg / NS) & 1u, args.timeout_ns);
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc_g = make_idesc_bf16(128, BN, 1, 1);
-      const uint32_t idesc_l = make_idesc_bf16(128, 128, 0, 0);
+      const uint32_t idesc_l = make_idesc_bf16(128, 128, 1, 1);
       const uint32_t idesc_da = make_idesc_bf16(128, args.r16, 0, 0);
       const uint32_t idesc_db = make_idesc_bf16(128, args.r16, 1, 0);
       const int lsteps = args.r16 / 16;
+      // Keep this thread's work between MMAs short: stage-0 descriptors are built once;
+      // a stage adds STAGE_BYTES / 16 and a 16-token K step adds 2048 bytes (128 units).
+      const uint64_t d_dy0 = make_sdesc(smem + OFF_STAGES, BOX_BYTES, 1024, SWZ_128B);
+      const uint64_t d_x0 = make_sdesc(smem + OFF_STAGES + STAGE_DY, BOX_BYTES, 1024, SWZ_128B);
+      const uint32_t b_full = bar(BAR_FULL), b_empty = bar(BAR_EMPTY);
       uint32_t g = 0, it = 0, cc = 0;
+      uint32_t s = 0, ph = 0;   // stage and phase of global step g
       bool ok = true;
       for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
         const Unit w = decode_unit(u, args);
         if (!(ok = wait_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 4))) break;
         tc_fence_after();
         for (int step = 0; step < w.nsteps; ++step) {
-          const uint32_t s = g % NS, ph = (g / NS) & 1u;
-          if (!(ok = wait_bounded(bar(BAR_FULL + s), ph, ctl, 5))) break;
+          if (!(ok = wait_bounded(b_full + 8u * s, ph, ctl, 5))) break;
           tc_fence_after();
-          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
-#pragma unroll
-          for (int ks = 0; ks < BKT / 16; ++ks) {
-            const uint64_t ad = make_sdesc(st + 2048u * ks, BOX_BYTES, 1024, SWZ_128B);
-            const uint64_t bd = make_sdesc(st + STAGE_DY + 2048u * ks, BOX_BYTES, 1024, SWZ_128B);
-            mma_bf16(tmem + COL_G, ad, bd, idesc_g, (step > 0 || ks > 0) ? 1u : 0u);
-          }
-          mma_commit(bar(BAR_EMPTY + s));
+          const uint64_t a = d_dy0 + s * (STAGE_BYTES >> 4), b = d_x0 + s * (STAGE_BYTES >> 4);
+          static_assert(BKT == 32, "two 16-token K steps per stage");
+          mma_bf16(tmem + COL_G, a, b, idesc_g, step > 0 ? 1u : 0u);
+          mma_bf16(tmem + COL_G, a + 128, b + 128, idesc_g, 1u);
+          mma_commit(b_empty + 8u * s);
           ++g;
+          if (++s == NS) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (!ok) break;
         mma_commit(bar(BAR_ACCFULL));
@@ -212,10 +241,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int c = 0; c < args.nchunks; ++c) {
           if (!(ok = wait_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 7))) break;
           tc_fence_after();
-          // L = A_pad * (B^T chunk)^T : the low-rank tile of this 128 x 128 chunk
+          // L = A (rows i) * B (columns j of the chunk): both operands read MN-major from
+          // A^T and B, 16 rank rows (two 8-row groups) per K step.
           for (int ks = 0; ks < lsteps; ++ks) {
-            const uint64_t ad = make_sdesc(smem + OFF_APAD + 32u * ks, 16, 1024, SWZ_128B);
-            const uint64_t bd = make_sdesc(smem + OFF_BT + 32u * ks, 16, 1024, SWZ_128B);
+            const uint64_t ad = make_sdesc(smem + OFF_AT + 2048u * ks, rbox, 1024, SWZ_128B);
+            const uint64_t bd = make_sdesc(smem + OFF_BP + 2048u * ks, rbox, 1024, SWZ_128B);
             mma_bf16(tmem + COL_L, ad, bd, idesc_l, ks > 0 ? 1u : 0u);
           }
           mma_commit(bar(BAR_LFULL));
@@ -377,8 +407,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
 template <bool PACKED>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
-                       const CUtensorMap& e, const CUtensorMap& f, const CUtensorMap& g2, const DwArgs& args,
-                       int grid, cudaStream_t stream) {
+                       const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
   static bool configured = false;
   if (!configured) {
     cudaError_t err =
@@ -386,7 +415,7 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
     if (err != cudaSuccess) return err;
     configured = true;
   }
-  dw_kernel<PACKED><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, f, g2, args);
+  dw_kernel<PACKED><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
   return cudaGetLastError();
 }
 
@@ -394,13 +423,13 @@ cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtenso
 
 int dw_smem_bytes(int, int) { return static_cast<int>(SMEM_BYTES); }
 
-cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_apad,
-                      const CUtensorMap& tm_at, const CUtensorMap& tm_phi, const CUtensorMap& tm_bt,
-                      const CUtensorMap& tm_b, const DwArgs& args, int grid, cudaStream_t stream) {
+cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
+                      const CUtensorMap& tm_phi, const CUtensorMap& tm_b, const DwArgs& args, int grid,
+                      cudaStream_t stream) {
   if (grid < 1 || args.r16 < 16 || args.r16 > 64 || (args.r16 & 15) || args.nchunks < 1 || args.nchunks > 2)
     return cudaErrorInvalidValue;
-  return packed ? launch_one<true>(tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, args, grid, stream)
-                : launch_one<false>(tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, args, grid, stream);
+  return packed ? launch_one<true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
+                : launch_one<false>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
 }
 
 }  // namespace lrqat

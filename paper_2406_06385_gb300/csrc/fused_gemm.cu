@@ -2,22 +2,31 @@
 // (dX = dY W_hat), with W_hat rebuilt on chip and never stored (Eq. 8 of the
 // paper; the recompute replaces the checkpointing of Sec. 3).
 //
-// One persistent CTA per SM processes tiles of 128 weight rows x 448 tokens.
-// Per 32-wide slice of the contraction:
-//   * TMA brings the token operand (448 x 32 bf16, SW64), the stored base
-//     (128 x 32 int8, SW32; packed: 128 x 16 bytes) and a 32-row slice of the
-//     second low-rank factor (SW128).
-//   * The MMA warp computes the low-rank tile L = RF * SF^T (M=128, N=32,
-//     K=r rounded to 16) into TMEM with tcgen05.
-//   * Eight producer warps read L from TMEM, decode the stored base, form
-//     u = phi^{-1}(Phi0) + (alpha/r) L, round half to even, clip, (scale) and
-//     write the bf16 operand tile (SW64, K-major) into shared memory.
-//   * The MMA warp runs the main product into two 128 x 224 fp32 TMEM
-//     accumulators; the same eight warps drain them in the epilogue.
+// One persistent CTA per SM processes tiles of 128 weight rows x 448 tokens,
+// one 64-wide slice of the contraction per pipeline stage:
+//   * token ring (2 slots): two loader warps, one per slot, bring with TMA the
+//     token operand as 2 boxes of 224 x 64 bf16 (128-byte rows, SW128); each slot
+//     also holds the bf16 operand tile W_hat of its stage;
+//   * factor ring (4 slots): one loader warp brings the stored base (128 x 64
+//     int8, SW64; packed: 128 x 32 bytes, SW32) and a 64-row slice of the second
+//     low-rank factor (SW128);
+//   * the MMA warp computes the low-rank tile L = RF * SF^T (M=128, N=64, K=r
+//     rounded to 16) into a TMEM buffer, issued ahead of the main product of the
+//     previous stage so that it is ready when that product finishes;
+//   * sixteen producer warps (lane quarter q = warp % 4, column chunk c of 16)
+//     read L with tcgen05.ld, decode the stored base, form
+//     u = phi^{-1}(Phi0) + (alpha/r) L with packed fp32 arithmetic, round half to
+//     even, clip, (scale) and write W_hat (SW128, K-major) while the previous
+//     stage's product runs;
+//   * the MMA warp runs the main product, 8 MMAs of M=128, N=224, K=16, into two
+//     fp32 TMEM accumulators; the same sixteen warps drain them in the epilogue.
 // Forward: rows = m (weight rows), contraction = k, RF = A (padded), SF = B^T.
 // dX:      rows = k, contraction = m over the transposed base Phi0^T,
 //          RF = B^T (padded), SF = A (padded); the scale varies along the
 //          contraction, so the producer emits bf16(s * c).
+// Large 128-byte-row boxes matter: an SM's TMA throughput falls with the number
+// of boxes it processes, and loads issued by one warp are handled one at a time,
+// hence one loader warp per ring slot of the token operand.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -30,44 +39,53 @@ namespace lrqat {
 namespace {
 
 constexpr int BM = 128;
-constexpr int BK = 32;
+constexpr int BK = 64;
 constexpr int BN = 224;
 constexpr int NACC = 2;
-constexpr int BT = BN * NACC;
-constexpr int NS = 4;
-constexpr int NUM_THREADS = 320;
-constexpr int NUM_PROD_WARPS = 8;
+constexpr int BT = BN * NACC;                    // 448 tokens per tile
+constexpr int NT = 2;                            // token ring slots
+constexpr int NF = 4;                            // factor ring slots (power of two)
+constexpr int NUM_PROD_WARPS = 16;
+constexpr int FIRST_TMA_WARP = 2 + NUM_PROD_WARPS;
+constexpr int NUM_TMA_WARPS = NT + 1;            // token loaders + factor loader
+constexpr int NUM_THREADS = 32 * (FIRST_TMA_WARP + NUM_TMA_WARPS);
+constexpr int EPI_COLS = NACC * BN / 4;          // accumulator columns drained per warp (112)
 
-constexpr uint32_t RF_BYTES = 128 * 128;
-constexpr uint32_t TOK_HALF = BN * 64;
-constexpr uint32_t TOK_BYTES = BT * 64;
-constexpr uint32_t W_BYTES = 128 * 64;
-constexpr uint32_t PHI_BYTES = 128 * 32;
-constexpr uint32_t SF_BYTES = 32 * 128;
-constexpr uint32_t OFF_TOK = 0;
-constexpr uint32_t OFF_W = TOK_BYTES;
-constexpr uint32_t OFF_PHI = OFF_W + W_BYTES;
-constexpr uint32_t OFF_SF = OFF_PHI + PHI_BYTES;
-constexpr uint32_t STAGE_BYTES = OFF_SF + SF_BYTES;
+constexpr uint32_t RF_BYTES = 128 * 128;         // 128 rows x 64 rank columns (bf16)
+constexpr uint32_t TOK_HALF = BN * 128;          // 224 tokens x 64 bf16
+constexpr uint32_t TOK_BYTES = 2 * TOK_HALF;
+constexpr uint32_t W_BYTES = 128 * 128;          // 128 rows x 64 bf16
+constexpr uint32_t PHI_BYTES = 128 * 64;         // 128 rows x 64 int8 (packed: half)
+constexpr uint32_t SF_BYTES = 64 * 128;          // 64 slice rows x 64 rank columns (bf16)
+constexpr uint32_t TSLOT_BYTES = TOK_BYTES + W_BYTES;
+constexpr uint32_t FSLOT_BYTES = PHI_BYTES + SF_BYTES;
 constexpr uint32_t OFF_RF = 0;
-constexpr uint32_t OFF_STAGES = RF_BYTES;
-constexpr uint32_t SMEM_BYTES = OFF_STAGES + NS * STAGE_BYTES + 1024;   // + 1 KB for 1024-B alignment
+constexpr uint32_t OFF_TSLOTS = RF_BYTES;
+constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
+constexpr uint32_t TS_W = TOK_BYTES;             // offsets inside a token slot
+constexpr uint32_t FS_SF = PHI_BYTES;            // offsets inside a factor slot
+constexpr uint32_t SMEM_BYTES = OFF_FSLOTS + NF * FSLOT_BYTES + 1024;   // + 1 KB for 1024-B alignment
 
-static_assert(STAGE_BYTES % 1024 == 0 && TOK_HALF % 1024 == 0 && OFF_W % 1024 == 0 && OFF_PHI % 1024 == 0 &&
-                  OFF_SF % 1024 == 0,
+static_assert(TSLOT_BYTES % 1024 == 0 && FSLOT_BYTES % 1024 == 0 && TOK_HALF % 1024 == 0 && TS_W % 1024 == 0 &&
+                  FS_SF % 1024 == 0 && OFF_TSLOTS % 1024 == 0 && OFF_FSLOTS % 1024 == 0,
               "swizzled tiles must start on 1024-byte boundaries");
+static_assert(SMEM_BYTES + 512 <= 232448, "shared memory budget");
+static_assert((NF & (NF - 1)) == 0, "factor ring index uses a mask");
+static_assert(EPI_COLS % 16 == 0, "epilogue drains 16-column chunks");
 
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t COL_L = NACC * BN;   // two 32-column low-rank buffers at 448 and 480
-static_assert(COL_L + 2 * BK <= TMEM_COLS, "TMEM budget");
+constexpr uint32_t COL_L = NACC * BN;            // one 64-column low-rank buffer at 448
+static_assert(COL_L + BK <= TMEM_COLS, "TMEM budget");
 
 // barrier indices
-constexpr int BAR_FULL = 0;
-constexpr int BAR_EMPTY = BAR_FULL + NS;
-constexpr int BAR_WFULL = BAR_EMPTY + NS;
-constexpr int BAR_LFULL = BAR_WFULL + NS;
-constexpr int BAR_LEMPTY = BAR_LFULL + 2;
-constexpr int BAR_RFFULL = BAR_LEMPTY + 2;
+constexpr int BAR_TFULL = 0;
+constexpr int BAR_TEMPTY = BAR_TFULL + NT;       // main product of the slot finished
+constexpr int BAR_WFULL = BAR_TEMPTY + NT;       // W_hat tile of the slot written
+constexpr int BAR_FFULL = BAR_WFULL + NT;
+constexpr int BAR_FEMPTY = BAR_FFULL + NF;
+constexpr int BAR_LFULL = BAR_FEMPTY + NF;
+constexpr int BAR_LEMPTY = BAR_LFULL + 1;
+constexpr int BAR_RFFULL = BAR_LEMPTY + 1;
 constexpr int BAR_RFEMPTY = BAR_RFFULL + 1;
 constexpr int BAR_ACCFULL = BAR_RFEMPTY + 1;
 constexpr int BAR_ACCEMPTY = BAR_ACCFULL + 1;
@@ -83,6 +101,9 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64
   }
 }
 
+// Stages are numbered globally over the CTA's tiles (gg); the contraction has an
+// even number of slices, so stage gg uses token slot gg % 2 for the (gg / 2)-th
+// time and factor slot gg % NF for the (gg / NF)-th time.
 template <int MODE, bool PACKED>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
@@ -100,15 +121,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (threadIdx.x == 0) {
     abort_s = 0;
-    for (int s = 0; s < NS; ++s) {
-      mbar_init(bar(BAR_FULL + s), 1);
-      mbar_init(bar(BAR_EMPTY + s), 1);
+    for (int s = 0; s < NT; ++s) {
+      mbar_init(bar(BAR_TFULL + s), 1);
+      mbar_init(bar(BAR_TEMPTY + s), 1);
       mbar_init(bar(BAR_WFULL + s), NUM_PROD_WARPS);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(bar(BAR_LFULL + b), 1);
-      mbar_init(bar(BAR_LEMPTY + b), NUM_PROD_WARPS);
+    for (int s = 0; s < NF; ++s) {
+      mbar_init(bar(BAR_FFULL + s), 1);
+      // Freed by the producers once they have built W_hat of the stage: by then the
+      // low-rank MMA that read the factor slice has completed (they waited for it).
+      mbar_init(bar(BAR_FEMPTY + s), NUM_PROD_WARPS);
     }
+    mbar_init(bar(BAR_LFULL), 1);
+    mbar_init(bar(BAR_LEMPTY), NUM_PROD_WARPS);
     mbar_init(bar(BAR_RFFULL), 1);
     mbar_init(bar(BAR_RFEMPTY), 1);
     mbar_init(bar(BAR_ACCFULL), 1);
@@ -122,96 +147,133 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
   const WaitCtl ctl{&abort_s, args.status, args.timeout_ns};
-  const int nk = args.kdim / BK;
+  const int nk = args.kdim / BK;   // even, at least 2 (kdim is a multiple of 128)
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------- row factor (per tile)
     if (lane == 0) {
-      prefetch_tensormap(&tm_tok);
-      prefetch_tensormap(&tm_phi);
       prefetch_tensormap(&tm_rf);
-      prefetch_tensormap(&tm_sf);
-      const uint32_t stage_tx = TOK_BYTES + (PACKED ? PHI_BYTES / 2 : PHI_BYTES) + SF_BYTES;
-      uint32_t g = 0;
       uint32_t it = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+      for (int tile = blockIdx.x; tile < args.num_tiles; tile += gridDim.x) {
         const int rb = tile % args.num_rb;
-        const int tb = tile / args.num_rb;
-        if (!(ok = wait_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1))) break;
+        if (!wait_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1)) break;
         mbar_arrive_expect_tx(bar(BAR_RFFULL), RF_BYTES);
         tma_load_2d(smem + OFF_RF, &tm_rf, 0, rb * BM, bar(BAR_RFFULL));
         ++it;
-        for (int kk = 0; kk < nk; ++kk) {
-          const uint32_t s = g % NS, ph = (g / NS) & 1u;
-          if (!(ok = wait_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 2))) break;
-          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
-          const uint32_t fb = bar(BAR_FULL + s);
-          mbar_arrive_expect_tx(fb, stage_tx);
-          tma_load_2d(st + OFF_TOK, &tm_tok, kk * BK, tb * BT, fb);
-          tma_load_2d(st + OFF_TOK + TOK_HALF, &tm_tok, kk * BK, tb * BT + BN, fb);
-          tma_load_2d(st + OFF_PHI, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb * BM, fb);
-          tma_load_2d(st + OFF_SF, &tm_sf, 0, kk * BK, fb);
-          ++g;
-        }
-      }
-      // Let every issued copy land before the CTA can exit.
-      for (uint32_t s = 0; s < NS && s < g; ++s) {
-        const uint32_t last = s + NS * ((g - 1 - s) / NS);
-        drain_wait(bar(BAR_FULL + s), (last / NS) & 1u, args.timeout_ns);
       }
       if (it > 0) drain_wait(bar(BAR_RFFULL), (it - 1) & 1u, args.timeout_ns);
+    }
+  } else if (warp >= FIRST_TMA_WARP && warp < FIRST_TMA_WARP + NT) {
+    // ------------------------------------------- token loaders (one per slot)
+    const uint32_t t = warp - FIRST_TMA_WARP;
+    if (lane == 0) prefetch_tensormap(&tm_tok);
+    const uint32_t st = smem + OFF_TSLOTS + t * TSLOT_BYTES;
+    const uint32_t fb = bar(BAR_TFULL + t), eb = bar(BAR_TEMPTY + t);
+    uint32_t n = 0;   // uses of this slot so far
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+      const int tb = tile / args.num_rb;
+      for (int kk = t; kk < nk; kk += NT) {
+        if (lane == 0) ok = wait_bounded(eb, (n & 1u) ^ 1u, ctl, 2);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
+        if (lane == 0) mbar_arrive_expect_tx(fb, TOK_BYTES);
+        __syncwarp();
+        if (lane == 0) tma_load_2d(st, &tm_tok, kk * BK, tb * BT, fb);
+        if (lane == 1) tma_load_2d(st + TOK_HALF, &tm_tok, kk * BK, tb * BT + BN, fb);
+        ++n;
+      }
+    }
+    // Let every issued copy land before the CTA can exit.
+    if (lane == 0 && n > 0) drain_wait(fb, (n - 1) & 1u, args.timeout_ns);
+  } else if (warp == FIRST_TMA_WARP + NT) {
+    // ------------------------------------------------- factor-ring loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_phi);
+      prefetch_tensormap(&tm_sf);
+    }
+    constexpr uint32_t tx = (PACKED ? PHI_BYTES / 2 : PHI_BYTES) + SF_BYTES;
+    uint32_t gg = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
+      const int rb = tile % args.num_rb;
+      for (int kk = 0; kk < nk; ++kk, ++gg) {
+        const uint32_t s = gg & (NF - 1);
+        const uint32_t fb = bar(BAR_FFULL + s);
+        if (lane == 0) ok = wait_bounded(bar(BAR_FEMPTY + s), ((gg / NF) & 1u) ^ 1u, ctl, 3);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
+        if (lane == 0) mbar_arrive_expect_tx(fb, tx);
+        __syncwarp();
+        const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
+        if (lane == 0) tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb * BM, fb);
+        if (lane == 1) tma_load_2d(fs + FS_SF, &tm_sf, 0, kk * BK, fb);
+      }
+    }
+    if (lane == 0 && gg > 0) {
+      const uint32_t last = gg - 1;
+      drain_wait(bar(BAR_FFULL + (last & (NF - 1))), (last / NF) & 1u, args.timeout_ns);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
+      // This thread's instruction stream sits between consecutive MMAs, so keep it
+      // short: descriptors of slot 0 are built once; a slot adds its byte stride / 16
+      // to the encoded start address and a 16-element K step adds 32 bytes (2 units).
       const uint32_t idesc_main = make_idesc_bf16(128, BN, 0, 0);
       const uint32_t idesc_l = make_idesc_bf16(128, BK, 0, 0);
       const int lsteps = args.r16 / 16;
+      constexpr uint32_t TSLOT_D = TSLOT_BYTES >> 4, FSLOT_D = FSLOT_BYTES >> 4, TOKH_D = TOK_HALF >> 4;
+      const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
+      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + FS_SF, 16, 1024, SWZ_128B);
+      const uint64_t d_w0 = make_sdesc(smem + OFF_TSLOTS + TS_W, 16, 1024, SWZ_128B);
+      const uint64_t d_tok0 = make_sdesc(smem + OFF_TSLOTS, 16, 1024, SWZ_128B);
       uint32_t g = 0;
       uint32_t it = 0;
       bool ok = true;
+      // Low-rank tile of stage gg into the TMEM buffer, once its factor slice has
+      // landed and the producers have read the tile of stage gg - 1.
       auto issue_lowrank = [&](uint32_t gg) -> bool {
-        const uint32_t s = gg % NS, ph = (gg / NS) & 1u;
-        const uint32_t lb = gg & 1u, lph = (gg >> 1) & 1u;
-        if (!wait_bounded(bar(BAR_FULL + s), ph, ctl, 3)) return false;
-        if (!wait_bounded(bar(BAR_LEMPTY + lb), lph ^ 1u, ctl, 4)) return false;
+        const uint32_t s = gg & (NF - 1);
+        if (!wait_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4)) return false;
+        if (!wait_bounded(bar(BAR_LEMPTY), (gg & 1u) ^ 1u, ctl, 5)) return false;
         tc_fence_after();
-        const uint32_t sf = smem + OFF_STAGES + s * STAGE_BYTES + OFF_SF;
-        for (int ks = 0; ks < lsteps; ++ks) {
-          const uint64_t ad = make_sdesc(smem + OFF_RF + 32u * ks, 16, 1024, SWZ_128B);
-          const uint64_t bd = make_sdesc(sf + 32u * ks, 16, 1024, SWZ_128B);
-          mma_bf16(tmem + COL_L + BK * lb, ad, bd, idesc_l, ks > 0 ? 1u : 0u);
-        }
-        mma_commit(bar(BAR_LFULL + lb));
+        const uint64_t sf = d_sf0 + s * FSLOT_D;
+        const uint32_t dl = tmem + COL_L;
+        mma_bf16(dl, d_rf, sf, idesc_l, 0u);
+        if (lsteps > 1) mma_bf16(dl, d_rf + 2, sf + 2, idesc_l, 1u);
+        if (lsteps > 2) mma_bf16(dl, d_rf + 4, sf + 4, idesc_l, 1u);
+        if (lsteps > 3) mma_bf16(dl, d_rf + 6, sf + 6, idesc_l, 1u);
+        mma_commit(bar(BAR_LFULL));
         return true;
       };
       for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
-        if (!(ok = wait_bounded(bar(BAR_RFFULL), it & 1u, ctl, 5))) break;
+        if (!(ok = wait_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
         if (!(ok = issue_lowrank(g))) break;
-        if (nk == 1) mma_commit(bar(BAR_RFEMPTY));
-        if (!(ok = wait_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 6))) break;
+        if (!(ok = wait_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
         tc_fence_after();
         for (int kk = 0; kk < nk; ++kk) {
           const uint32_t gg = g + kk;
+          const uint32_t s = gg & 1u, ph = (gg >> 1) & 1u;
+          if (!(ok = wait_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
           if (kk + 1 < nk) {
             if (!(ok = issue_lowrank(gg + 1))) break;
-            if (kk + 2 == nk) mma_commit(bar(BAR_RFEMPTY));
+            if (kk + 2 == nk) mma_commit(bar(BAR_RFEMPTY));   // last read of the row factor issued
           }
-          const uint32_t s = gg % NS, ph = (gg / NS) & 1u;
-          if (!(ok = wait_bounded(bar(BAR_WFULL + s), ph, ctl, 7))) break;
+          if (!(ok = wait_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
           tc_fence_after();
-          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
-#pragma unroll
-          for (int a = 0; a < NACC; ++a) {
-#pragma unroll
-            for (int ks = 0; ks < BK / 16; ++ks) {
-              const uint64_t ad = make_sdesc(st + OFF_W + 32u * ks, 16, 512, SWZ_64B);
-              const uint64_t bd = make_sdesc(st + OFF_TOK + a * TOK_HALF + 32u * ks, 16, 512, SWZ_64B);
-              mma_bf16(tmem + a * BN, ad, bd, idesc_main, (kk > 0 || ks > 0) ? 1u : 0u);
-            }
-          }
-          mma_commit(bar(BAR_EMPTY + s));
+          const uint64_t w = d_w0 + s * TSLOT_D, t = d_tok0 + s * TSLOT_D;
+          const uint32_t acc = kk > 0 ? 1u : 0u;
+          static_assert(NACC == 2 && BK == 64, "issue sequence below is written for 2 accumulators x 4 K steps");
+          mma_bf16(tmem, w, t, idesc_main, acc);
+          mma_bf16(tmem, w + 2, t + 2, idesc_main, 1u);
+          mma_bf16(tmem, w + 4, t + 4, idesc_main, 1u);
+          mma_bf16(tmem, w + 6, t + 6, idesc_main, 1u);
+          mma_bf16(tmem + BN, w, t + TOKH_D, idesc_main, acc);
+          mma_bf16(tmem + BN, w + 2, t + TOKH_D + 2, idesc_main, 1u);
+          mma_bf16(tmem + BN, w + 4, t + TOKH_D + 4, idesc_main, 1u);
+          mma_bf16(tmem + BN, w + 6, t + TOKH_D + 6, idesc_main, 1u);
+          mma_commit(bar(BAR_TEMPTY + s));
         }
         if (!ok) break;
         mma_commit(bar(BAR_ACCFULL));
@@ -223,12 +285,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ------------------------------------------- W_hat producers + epilogue
-    const int pw = warp - 2;
-    const int q = warp & 3;           // TMEM lane quarter this warp may access
-    const int h = pw >> 2;            // half of the slice columns / accumulator index
-    const int row = q * 32 + lane;    // row of the tile handled by this thread
+    const int pw = warp - 2;              // 0..15
+    const int q = warp & 3;               // TMEM lane quarter this warp may access
+    const int c = pw >> 2;                // 16-column chunk of the 64-wide slice (and epilogue block)
+    const int row = q * 32 + lane;        // row of the tile handled by this thread
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const QuantParams qp = args.q;
+    const float dec_off = PACKED ? kDecodeOffsetI4 : kDecodeOffsetI8;
     uint32_t g = 0;
     uint32_t it = 0;
     bool ok = true;
@@ -238,8 +301,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int row_g = rb * BM + row;
       for (int kk = 0; kk < nk; ++kk) {
         const uint32_t gg = g + kk;
-        const uint32_t s = gg % NS, ph = (gg / NS) & 1u;
-        const uint32_t lb = gg & 1u, lph = (gg >> 1) & 1u;
         // Scales that multiply the operand (group-wise forward, dX).
         float sc[16];
         if (MODE == FUSED_FWD_GROUP) {
@@ -247,7 +308,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int e = 0; e < 16; ++e) sc[e] = v;
         } else if (MODE == FUSED_DX) {
-          const int i0 = kk * BK + 16 * h;
+          const int i0 = kk * BK + 16 * c;
           if (args.s_ld == 0) {
             const float4* sp = reinterpret_cast<const float4*>(args.s + i0);
 #pragma unroll
@@ -264,70 +325,92 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int e = 0; e < 16; ++e) sc[e] = __ldg(args.s + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
           }
         }
-        ok = wait_bounded(bar(BAR_LFULL + lb), lph, ctl, 8);
+        ok = wait_bounded(bar(BAR_LFULL), gg & 1u, ctl, 10);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
         float Lv[16];
-        tmem_ld16(tmem + lane_off + COL_L + BK * lb + 16 * h, Lv);
+        tmem_ld16(tmem + lane_off + COL_L + 16 * c, Lv);
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar(BAR_LEMPTY + lb));
-        ok = wait_bounded(bar(BAR_FULL + s), ph, ctl, 9);
+        if (lane == 0) mbar_arrive(bar(BAR_LEMPTY));
+        const uint32_t fslot = gg & (NF - 1);
+        ok = wait_bounded(bar(BAR_FFULL + fslot), (gg / NF) & 1u, ctl, 11);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-        const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
-        float v[16];
+        const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
+        float fd[16];
         if (PACKED) {
-          const uint2 raw = ld_shared_v2(st + OFF_PHI + row * 16 + 8 * h);
-          decode_i4x8(raw.x, v);
-          decode_i4x8(raw.y, v + 8);
+          const uint2 raw = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
+          decode_i4x8_raw(raw.x, fd);
+          decode_i4x8_raw(raw.y, fd + 8);
         } else {
-          const uint4 raw = ld_shared_v4(st + OFF_PHI + swz_offset(row, h, 32));
-          decode_i8x4(raw.x, v);
-          decode_i8x4(raw.y, v + 4);
-          decode_i8x4(raw.z, v + 8);
-          decode_i8x4(raw.w, v + 12);
+          const uint4 raw = ld_shared_v4(fs + swz_offset(row, c, 64));
+          decode_i8x4_raw(raw.x, fd);
+          decode_i8x4_raw(raw.y, fd + 4);
+          decode_i8x4_raw(raw.z, fd + 8);
+          decode_i8x4_raw(raw.w, fd + 12);
         }
         uint32_t w[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float c0 = lrqat_code(Lv[2 * e], v[2 * e], qp);
-          const float c1 = lrqat_code(Lv[2 * e + 1], v[2 * e + 1], qp);
-          if (MODE == FUSED_FWD_PC)
-            w[e] = pack_exact_bf16x2(c0, c1);
-          else
-            w[e] = pack_rn_bf16x2(c0 * sc[2 * e], c1 * sc[2 * e + 1]);
+          const float2 t2 = magic_round2(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(fd[2 * e], fd[2 * e + 1]),
+                                         dec_off, qp);
+          if (MODE == FUSED_FWD_PC) {
+            w[e] = codes_bf16x2(t2, qp);
+          } else {
+            const float2 c2 = codes_f32x2(t2, qp);
+            const float2 v2 = __fmul2_rn(c2, make_float2(sc[2 * e], sc[2 * e + 1]));
+            w[e] = pack_rn_bf16x2(v2.x, v2.y);
+          }
         }
-        const uint32_t wt = st + OFF_W;
-        st_shared_v4(wt + swz_offset(row, 2 * h, 64), w[0], w[1], w[2], w[3]);
-        st_shared_v4(wt + swz_offset(row, 2 * h + 1, 64), w[4], w[5], w[6], w[7]);
+        // The W_hat buffer of this token slot was last read by the product of stage gg - 2.
+        const uint32_t ts = gg & 1u;
+        ok = wait_bounded(bar(BAR_TEMPTY + ts), ((gg >> 1) & 1u) ^ 1u, ctl, 12);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        const uint32_t wt = smem + OFF_TSLOTS + ts * TSLOT_BYTES + TS_W;
+        st_shared_v4(wt + swz_offset(row, 2 * c, 128), w[0], w[1], w[2], w[3]);
+        st_shared_v4(wt + swz_offset(row, 2 * c + 1, 128), w[4], w[5], w[6], w[7]);
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) mbar_arrive(bar(BAR_WFULL + s));
+        if (lane == 0) {
+          mbar_arrive(bar(BAR_WFULL + ts));
+          mbar_arrive(bar(BAR_FEMPTY + fslot));
+        }
       }
       if (!ok) break;
       // ------------------------------------------------------------ epilogue
       float scale = 1.0f;
       if (MODE == FUSED_FWD_PC) scale = args.s[row_g];
       if (MODE != FUSED_DX && args.s_x != nullptr) scale *= *args.s_x;
-      ok = wait_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 10);
+      ok = wait_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 13);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
+      const bool odd = lane & 1;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        float acc[32];
-        tmem_ld32(tmem + lane_off + h * BN + 32 * c, acc);
+      for (int ch = 0; ch < EPI_COLS / 16; ++ch) {
+        float acc[16];
+        const int col = c * EPI_COLS + 16 * ch;   // accumulator column = token offset in the tile
+        tmem_ld16(tmem + lane_off + col, acc);
         tmem_ld_wait();
-        const int tok0 = tb * BT + h * BN + 32 * c;
+        const int tok0 = tb * BT + col;
         uint32_t mword = 0xffffffffu;
         if (MODE == FUSED_DX && args.xmask != nullptr && tok0 < args.T)
-          mword = args.xmask[static_cast<int64_t>(row_g) * args.xmask_ld + tok0 / 32];
-        uint16_t* dst = args.out + static_cast<int64_t>(tok0) * args.out_ld + row_g;
+          mword = args.xmask[static_cast<int64_t>(row_g) * args.xmask_ld + tok0 / 32] >> (tok0 & 31);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          if (tok0 + e < args.T) {
-            const float val = ((mword >> e) & 1u) ? acc[e] * scale : 0.0f;
-            dst[static_cast<int64_t>(e) * args.out_ld] = float_to_bf16_rn(val);
+        for (int e = 0; e < 16; ++e) acc[e] = ((mword >> e) & 1u) ? acc[e] * scale : 0.0f;
+        // Pair rows (lane, lane ^ 1): the even lane stores both rows of even tokens,
+        // the odd lane both rows of odd tokens, as 4-byte words.
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float mine = odd ? acc[2 * e] : acc[2 * e + 1];
+          const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
+          const int tt = tok0 + 2 * e + (odd ? 1 : 0);
+          const float lo = odd ? other : acc[2 * e];
+          const float hi = odd ? acc[2 * e + 1] : other;
+          if (tt < args.T) {
+            uint32_t* dst = reinterpret_cast<uint32_t*>(args.out + static_cast<int64_t>(tt) * args.out_ld +
+                                                        (row_g & ~1));
+            *dst = pack_rn_bf16x2(lo, hi);
           }
         }
       }
@@ -369,7 +452,7 @@ int fused_smem_bytes() { return static_cast<int>(SMEM_BYTES); }
 cudaError_t launch_fused(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
                          const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
                          cudaStream_t stream) {
-  if (grid < 1) return cudaErrorInvalidValue;
+  if (grid < 1 || (args.kdim % 128) != 0 || args.kdim < 128) return cudaErrorInvalidValue;
   switch (mode) {
     case FUSED_FWD_PC:
       return packed ? launch_one<FUSED_FWD_PC, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)

@@ -87,8 +87,8 @@ struct DwArgs {
   uint64_t timeout_ns;
 };
 int dw_smem_bytes(int r16, int packed);
-cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_apad,
-                      const CUtensorMap& tm_at, const CUtensorMap& tm_phi, const CUtensorMap& tm_bt,
-                      const CUtensorMap& tm_b, const DwArgs& args, int grid, cudaStream_t stream);
+cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
+                      const CUtensorMap& tm_phi, const CUtensorMap& tm_b, const DwArgs& args, int grid,
+                      cudaStream_t stream);
 
 }  // namespace lrqat

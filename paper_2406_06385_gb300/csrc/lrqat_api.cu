@@ -304,13 +304,13 @@ size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* bas
 }
 
 int phi_map(CUtensorMap* map, const lrqat_layer& L, const void* phi0, uint32_t box_cols_elems, bool dw) {
-  // Forward: slices of 32 columns (32 B int8 rows, SW32; packed 16 B rows, no swizzle).
+  // Forward: slices of 64 columns (64 B int8 rows, SW64; packed 32 B rows, SW32).
   // dW: chunks of 128 columns (128 B int8 rows, SW128; packed 64 B rows, SW64).
   if (L.phi_format == LRQAT_PHI_QFIXED)
     return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k, L.m, L.k, box_cols_elems, 128,
-                     dw ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_32B, "Phi0");
+                     dw ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, "Phi0");
   return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k / 2, L.m, L.k / 2, box_cols_elems / 2, 128,
-                   dw ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_NONE, "Phi0 (packed)");
+                   dw ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B, "Phi0 (packed)");
 }
 
 }  // namespace
@@ -443,12 +443,12 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
     tok = ws.x_codes;
   }
   CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
-  LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 32, 224,
-                      CU_TENSOR_MAP_SWIZZLE_64B, "X"));
-  LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 32, false));
+  LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 64, 224,
+                      CU_TENSOR_MAP_SWIZZLE_128B, "X"));
+  LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 64, false));
   LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
                       CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
-  LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 32,
+  LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 64,
                       CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
   FusedArgs a{};
   a.rows = static_cast<int32_t>(L.m);
@@ -532,13 +532,13 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
-    LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 32, 224,
-                        CU_TENSOR_MAP_SWIZZLE_64B, "dY"));
-    LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.phit, L.m, L.k, L.m, 32, 128,
-                        CU_TENSOR_MAP_SWIZZLE_32B, "Phi0^T"));
+    LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 224,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "dY"));
+    LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.phit, L.m, L.k, L.m, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_64B, "Phi0^T"));
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
-    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 32,
+    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 64,
                         CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
     FusedArgs a{};
     a.rows = static_cast<int32_t>(L.k);
@@ -565,18 +565,14 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   }
   // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
   {
-    CUtensorMap tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b;
+    CUtensorMap tm_dy, tm_x, tm_at, tm_phi, tm_b;
     LRQAT_TRY(encode_2d(&tm_dy, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 32,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY (dW)"));
     LRQAT_TRY(encode_2d(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, xop, L.k, T, L.k * 2, 64, 32,
                         CU_TENSOR_MAP_SWIZZLE_128B, "X (dW)"));
-    LRQAT_TRY(encode_2d(&tm_apad, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
-                        CU_TENSOR_MAP_SWIZZLE_128B, "A (padded, dW)"));
     LRQAT_TRY(encode_2d(&tm_at, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64,
                         static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "A^T"));
     LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
-    LRQAT_TRY(encode_2d(&tm_bt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
-                        CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded, dW)"));
     LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.b_pad, L.k, r16, L.k * 2, 64,
                         static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
     DwArgs a{};
@@ -603,7 +599,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.timeout_ns = kWaitTimeoutNs;
     const int grid = plan.units < dev->sms ? plan.units : dev->sms;
     LRQAT_LAUNCH("fused_dw", 1, stream,
-                 launch_dw(packed, tm_dy, tm_x, tm_apad, tm_at, tm_phi, tm_bt, tm_b, a, grid, stream),
+                 launch_dw(packed, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
                  "fused dW launch");
   }
   ReduceArgs ra{};

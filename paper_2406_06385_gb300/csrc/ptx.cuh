@@ -45,6 +45,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Like mbar_try_wait, but lets the thread sleep up to `hint_ns` while the phase is
+// incomplete; it resumes as soon as the phase completes.  Sleeping waiters leave
+// the issue slots of their SM sub-partition to the warps that have work.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
 // Control block shared by all roles of one CTA.
 struct WaitCtl {
   volatile int* abort;   // shared-memory flag: some role gave up
@@ -55,12 +70,14 @@ struct WaitCtl {
 // Waits until the phase of parity `parity` of barrier `bar` has completed.
 // Returns false (and stops waiting) when the time limit passes or another role
 // of the CTA has already given up.
+// Each retry sleeps in try_wait for up to 20 us (woken early when the phase
+// completes), so the abort flag and the time limit are checked every few retries.
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, const WaitCtl& ctl, int site) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 15u) == 0) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if ((it & 3u) == 0) {
       if (*ctl.abort) return false;
       if (global_timer_ns() - t0 > ctl.timeout_ns) {
         *ctl.abort = 1;

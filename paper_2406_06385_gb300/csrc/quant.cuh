@@ -24,6 +24,8 @@ struct QuantParams {
   float hi;         // magic + 2^f * p
   float inv2f;      // 2^-f
   float magic_c;    // 1.5 * 2^23
+  uint32_t n_bf16x2;  // bf16 bits of n in both halves
+  uint32_t p_bf16x2;  // bf16 bits of p in both halves
 };
 
 // Builds the constants above on the host.
@@ -38,7 +40,67 @@ inline QuantParams make_quant_params(int bits, int frac_bits, float alpha, int r
   q.hi = static_cast<float>(1.5 * 8388608.0 * two_f + two_f * p);
   q.inv2f = static_cast<float>(1.0 / two_f);
   q.magic_c = 12582912.0f;   // 1.5 * 2^23
+  const float nf = static_cast<float>(n), pf = static_cast<float>(p);
+  uint32_t nb, pb;
+  static_assert(sizeof(float) == sizeof(uint32_t), "float is 32-bit");
+  __builtin_memcpy(&nb, &nf, 4);
+  __builtin_memcpy(&pb, &pf, 4);
+  q.n_bf16x2 = (nb >> 16) * 0x10001u;   // small integers are exact in bf16 (top 16 bits)
+  q.p_bf16x2 = (pb >> 16) * 0x10001u;
   return q;
+}
+
+// Offsets that turn the exponent-trick floats of the decoders below into the
+// stored integer: 2^23 + 128 for int8 bytes, 2^23 + 8 for nibbles.
+constexpr float kDecodeOffsetI8 = 8388736.0f;
+constexpr float kDecodeOffsetI4 = 8388616.0f;
+
+// 4 signed bytes -> 4 floats 2^23 + (v + 128), exact (subtract kDecodeOffsetI8 for v).
+__device__ __forceinline__ void decode_i8x4_raw(uint32_t w, float* f) {
+  const uint32_t x = w ^ 0x80808080u;
+  f[0] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7540u));
+  f[1] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7541u));
+  f[2] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7542u));
+  f[3] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7543u));
+}
+
+// 8 signed nibbles (low nibble of byte b = element 2b) -> 8 floats 2^23 + (v + 8), exact.
+__device__ __forceinline__ void decode_i4x8_raw(uint32_t w, float* f) {
+  const uint32_t x = w ^ 0x88888888u;
+  const uint32_t lo = x & 0x0F0F0F0Fu;
+  const uint32_t hi = (x >> 4) & 0x0F0F0F0Fu;
+#pragma unroll
+  for (int b = 0; b < 4; ++b) {
+    f[2 * b] = __uint_as_float(__byte_perm(lo, 0x4B000000u, 0x7540u + b));
+    f[2 * b + 1] = __uint_as_float(__byte_perm(hi, 0x4B000000u, 0x7540u + b));
+  }
+}
+
+// Two elements at once with packed fp32 arithmetic: from exponent-trick floats
+// `fd` (decoder output), the low-rank values L and the decode offset, returns the
+// magic-domain values t (round-half-even already applied, unclipped).
+__device__ __forceinline__ float2 magic_round2(float2 L, float2 fd, float offset, const QuantParams& q) {
+  const float2 v = __fadd2_rn(fd, make_float2(-offset, -offset));
+  const float2 u = __ffma2_rn(L, make_float2(q.lr_scale, q.lr_scale), v);
+  return __fadd2_rn(u, make_float2(q.magic, q.magic));
+}
+
+// Exact integer codes of two elements as bf16x2, clipped to [n, p].  The
+// unclipped codes are exact in fp32; bf16 keeps them exactly up to |c| <= 256 and
+// truncation of larger ones keeps them beyond the clip limits, so clipping in bf16
+// after packing is exact.
+__device__ __forceinline__ uint32_t codes_bf16x2(float2 t, const QuantParams& q) {
+  const float2 c = __ffma2_rn(t, make_float2(q.inv2f, q.inv2f), make_float2(-q.magic_c, -q.magic_c));
+  uint32_t w = __byte_perm(__float_as_uint(c.x), __float_as_uint(c.y), 0x7632u);
+  asm("max.bf16x2 %0, %0, %1;" : "+r"(w) : "r"(q.n_bf16x2));
+  asm("min.bf16x2 %0, %0, %1;" : "+r"(w) : "r"(q.p_bf16x2));
+  return w;
+}
+
+// Clipped codes of two elements as fp32 (exact).
+__device__ __forceinline__ float2 codes_f32x2(float2 t, const QuantParams& q) {
+  const float2 tc = make_float2(fminf(fmaxf(t.x, q.lo), q.hi), fminf(fmaxf(t.y, q.lo), q.hi));
+  return __ffma2_rn(tc, make_float2(q.inv2f, q.inv2f), make_float2(-q.magic_c, -q.magic_c));
 }
 
 // 4 signed bytes of `w` -> 4 exact floats.
