@@ -255,11 +255,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int kk = 0; kk < nk; ++kk) {
           const uint32_t gg = g + kk;
           const uint32_t s = gg & 1u, ph = (gg >> 1) & 1u;
-          if (!(ok = wait_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
+          // The low-rank tile of the next stage goes into the tensor pipe ahead of this
+          // stage's product as soon as the producers have read the current one, so the
+          // W_hat build of the next stage overlaps this product.
           if (kk + 1 < nk) {
             if (!(ok = issue_lowrank(gg + 1))) break;
             if (kk + 2 == nk) mma_commit(bar(BAR_RFEMPTY));   // last read of the row factor issued
           }
+          if (!(ok = wait_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
           if (!(ok = wait_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
           tc_fence_after();
           const uint64_t w = d_w0 + s * TSLOT_D, t = d_tok0 + s * TSLOT_D;
@@ -325,6 +328,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int e = 0; e < 16; ++e) sc[e] = __ldg(args.s + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
           }
         }
+        // The stored base usually lands well before the low-rank tile: decode it first,
+        // keeping the low-rank read -> W_hat chain short.
+        const uint32_t fslot = gg & (NF - 1);
+        ok = wait_bounded(bar(BAR_FFULL + fslot), (gg / NF) & 1u, ctl, 11);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
+        float v[16];
+        if (PACKED) {
+          const uint2 raw = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
+          decode_i4x8_raw(raw.x, v);
+          decode_i4x8_raw(raw.y, v + 8);
+        } else {
+          const uint4 raw = ld_shared_v4(fs + swz_offset(row, c, 64));
+          decode_i8x4_raw(raw.x, v);
+          decode_i8x4_raw(raw.y, v + 4);
+          decode_i8x4_raw(raw.z, v + 8);
+          decode_i8x4_raw(raw.w, v + 12);
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float2 d = __fadd2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(-dec_off, -dec_off));
+          v[2 * e] = d.x;
+          v[2 * e + 1] = d.y;
+        }
         ok = wait_bounded(bar(BAR_LFULL), gg & 1u, ctl, 10);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
@@ -334,27 +361,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(BAR_LEMPTY));
-        const uint32_t fslot = gg & (NF - 1);
-        ok = wait_bounded(bar(BAR_FFULL + fslot), (gg / NF) & 1u, ctl, 11);
-        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-        const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
-        float fd[16];
-        if (PACKED) {
-          const uint2 raw = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
-          decode_i4x8_raw(raw.x, fd);
-          decode_i4x8_raw(raw.y, fd + 8);
-        } else {
-          const uint4 raw = ld_shared_v4(fs + swz_offset(row, c, 64));
-          decode_i8x4_raw(raw.x, fd);
-          decode_i8x4_raw(raw.y, fd + 4);
-          decode_i8x4_raw(raw.z, fd + 8);
-          decode_i8x4_raw(raw.w, fd + 12);
-        }
         uint32_t w[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float2 t2 = magic_round2(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(fd[2 * e], fd[2 * e + 1]),
-                                         dec_off, qp);
+          const float2 u = __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
+                                      make_float2(v[2 * e], v[2 * e + 1]));
+          const float2 t2 = __fadd2_rn(u, make_float2(qp.magic, qp.magic));
           if (MODE == FUSED_FWD_PC) {
             w[e] = codes_bf16x2(t2, qp);
           } else {

@@ -76,15 +76,6 @@ __device__ __forceinline__ void decode_i4x8_raw(uint32_t w, float* f) {
   }
 }
 
-// Two elements at once with packed fp32 arithmetic: from exponent-trick floats
-// `fd` (decoder output), the low-rank values L and the decode offset, returns the
-// magic-domain values t (round-half-even already applied, unclipped).
-__device__ __forceinline__ float2 magic_round2(float2 L, float2 fd, float offset, const QuantParams& q) {
-  const float2 v = __fadd2_rn(fd, make_float2(-offset, -offset));
-  const float2 u = __ffma2_rn(L, make_float2(q.lr_scale, q.lr_scale), v);
-  return __fadd2_rn(u, make_float2(q.magic, q.magic));
-}
-
 // Exact integer codes of two elements as bf16x2, clipped to [n, p].  The
 // unclipped codes are exact in fp32; bf16 keeps them exactly up to |c| <= 256 and
 // truncation of larger ones keeps them beyond the clip limits, so clipping in bf16
