@@ -144,78 +144,189 @@ __global__ void act_quant_kernel(const uint16_t* __restrict__ X, int64_t T, int6
 }
 
 // ---------------------------------------------------------------- re-layouts --
-__global__ void pad_rows64_kernel(const uint16_t* __restrict__ A, int64_t m, int r, uint16_t* __restrict__ out) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= m * 64) return;
-  const int64_t i = e / 64;
-  const int c = static_cast<int>(e % 64);
-  out[e] = c < r ? A[i * r + c] : static_cast<uint16_t>(0);
-}
-
-__global__ void pad_rows_kernel(const uint16_t* __restrict__ src, int rows, int rows_pad, int64_t cols,
-                                uint16_t* __restrict__ out) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= static_cast<int64_t>(rows_pad) * cols) return;
-  const int c = static_cast<int>(e / cols);
-  out[e] = c < rows ? src[e] : static_cast<uint16_t>(0);
-}
-
-__global__ void transpose_pad64_kernel(const uint16_t* __restrict__ B, int r, int64_t k, uint16_t* __restrict__ out) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= k * 64) return;
-  const int64_t j = e / 64;
-  const int c = static_cast<int>(e % 64);
-  out[e] = c < r ? B[static_cast<int64_t>(c) * k + j] : static_cast<uint16_t>(0);
-}
-
-__global__ void transpose_rows_kernel(const uint16_t* __restrict__ A, int64_t m, int r, int r16,
-                                      uint16_t* __restrict__ out) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= static_cast<int64_t>(r16) * m) return;
-  const int c = static_cast<int>(e / m);
-  const int64_t i = e % m;
-  out[e] = c < r ? A[i * r + c] : static_cast<uint16_t>(0);
+// The four TMA-friendly layouts of the adapters, in one launch; each thread writes
+// 8 consecutive bf16 (16 bytes) of one output.  Null outputs are skipped.
+//   A_pad  [m][64]   = A[i][c], zero for c >= r       (row factor of the forward)
+//   Bt_pad [k][64]   = B[c][j], zero for c >= r       (B^T, row factor of dX)
+//   At     [r16][m]  = A[i][c], zero rows for c >= r  (A^T, dW epilogue)
+//   B_pad  [r16][k]  = B[c][j], zero rows for c >= r  (dW epilogue)
+__global__ void adapter_layouts_kernel(const uint16_t* __restrict__ A, const uint16_t* __restrict__ B, int64_t m,
+                                       int64_t k, int r, int r16, uint4* __restrict__ A_pad,
+                                       uint4* __restrict__ Bt_pad, uint4* __restrict__ At,
+                                       uint4* __restrict__ B_pad, int b_aligned) {
+  const int64_t n0 = A_pad ? m * 8 : 0;
+  const int64_t n1 = Bt_pad ? k * 8 : 0;
+  const int64_t n2 = At ? static_cast<int64_t>(r16) * (m / 8) : 0;
+  const int64_t n3 = B_pad ? static_cast<int64_t>(r16) * (k / 8) : 0;
+  const int64_t total = n0 + n1 + n2 + n3;
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    uint32_t w[4];
+    if (t < n0) {
+      const int64_t i = t >> 3;
+      const int c0 = static_cast<int>(t & 7) * 8;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int c = c0 + 2 * e;
+        const uint32_t lo = c < r ? A[i * r + c] : 0u, hi = c + 1 < r ? A[i * r + c + 1] : 0u;
+        w[e] = lo | (hi << 16);
+      }
+      A_pad[t] = make_uint4(w[0], w[1], w[2], w[3]);
+    } else if (t < n0 + n1) {
+      const int64_t u = t - n0, j = u >> 3;
+      const int c0 = static_cast<int>(u & 7) * 8;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int c = c0 + 2 * e;
+        const uint32_t lo = c < r ? B[static_cast<int64_t>(c) * k + j] : 0u;
+        const uint32_t hi = c + 1 < r ? B[static_cast<int64_t>(c + 1) * k + j] : 0u;
+        w[e] = lo | (hi << 16);
+      }
+      Bt_pad[u] = make_uint4(w[0], w[1], w[2], w[3]);
+    } else if (t < n0 + n1 + n2) {
+      const int64_t u = t - n0 - n1;
+      const int c = static_cast<int>(u / (m / 8));
+      const int64_t i0 = (u % (m / 8)) * 8;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t lo = c < r ? A[(i0 + 2 * e) * r + c] : 0u, hi = c < r ? A[(i0 + 2 * e + 1) * r + c] : 0u;
+        w[e] = lo | (hi << 16);
+      }
+      At[u] = make_uint4(w[0], w[1], w[2], w[3]);
+    } else {
+      const int64_t u = t - n0 - n1 - n2;
+      const int c = static_cast<int>(u / (k / 8));
+      const int64_t j0 = (u % (k / 8)) * 8;
+      if (c >= r) {
+        B_pad[u] = make_uint4(0, 0, 0, 0);
+      } else if (b_aligned) {
+        B_pad[u] = *reinterpret_cast<const uint4*>(B + static_cast<int64_t>(c) * k + j0);
+      } else {
+        const uint16_t* src = B + static_cast<int64_t>(c) * k + j0;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) w[e] = static_cast<uint32_t>(src[2 * e]) | (static_cast<uint32_t>(src[2 * e + 1]) << 16);
+        B_pad[u] = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    }
+  }
 }
 
 // 64 x 64 tiles of Phi0 (rows i, columns j) -> out[j][i] as int8 stored integers.
-__global__ void phi_transpose_kernel(const void* __restrict__ phi0, int64_t m, int64_t k, int packed,
-                                     int8_t* __restrict__ out) {
-  __shared__ int8_t tile[64][64 + 4];
+// Each thread loads 16 stored integers of one row (16 bytes, or 8 packed bytes)
+// and writes 16 bytes of one transposed row; the tile passes through shared
+// memory with a 68-byte pitch (4-byte aligned rows, at most 2-way conflicts on the
+// column reads).
+__global__ void __launch_bounds__(256) phi_transpose_kernel(const void* __restrict__ phi0, int64_t m, int64_t k,
+                                                             int packed, int8_t* __restrict__ out) {
+  constexpr int PITCH = 68;
+  __shared__ __align__(16) int8_t tile[64 * PITCH];
   const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 64;
   const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 64;
-  for (int e = threadIdx.x; e < 64 * 64; e += blockDim.x) {
-    const int ii = e / 64, jj = e % 64;
-    const int64_t i = i0 + ii, j = j0 + jj;
-    int8_t v;
-    if (packed) {
-      const uint8_t byte = static_cast<const uint8_t*>(phi0)[i * (k / 2) + j / 2];
-      const int nib = (j & 1) ? (byte >> 4) : (byte & 0xF);
-      v = static_cast<int8_t>(nib >= 8 ? nib - 16 : nib);
-    } else {
-      v = static_cast<const int8_t*>(phi0)[i * k + j];
+  const int t = threadIdx.x;
+  const int ii = t >> 2, jq = (t & 3) * 16;
+  uint32_t v[4];
+  if (packed) {
+    const uint2 raw =
+        *reinterpret_cast<const uint2*>(static_cast<const uint8_t*>(phi0) + (i0 + ii) * (k / 2) + (j0 + jq) / 2);
+    const uint32_t src[2] = {raw.x, raw.y};
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      // 4 packed bytes -> 8 sign-extended nibbles (low nibble = even column)
+      const uint32_t x = src[h] ^ 0x88888888u;
+      const uint32_t lo = x & 0x0F0F0F0Fu, hi = (x >> 4) & 0x0F0F0F0Fu;
+      // bytes: (lo0, hi0, lo1, hi1) and (lo2, hi2, lo3, hi3), then subtract 8 from each byte
+      const uint32_t b01 = __byte_perm(lo, hi, 0x5140), b23 = __byte_perm(lo, hi, 0x7362);
+      v[2 * h] = __vsub4(b01, 0x08080808u);
+      v[2 * h + 1] = __vsub4(b23, 0x08080808u);
     }
-    tile[ii][jj] = v;
+  } else {
+    const uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const int8_t*>(phi0) + (i0 + ii) * k + j0 + jq);
+    v[0] = raw.x;
+    v[1] = raw.y;
+    v[2] = raw.z;
+    v[3] = raw.w;
   }
+  uint32_t* row = reinterpret_cast<uint32_t*>(tile + ii * PITCH + jq);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) row[e] = v[e];
   __syncthreads();
-  for (int e = threadIdx.x; e < 64 * 64; e += blockDim.x) {
-    const int jj = e / 64, ii = e % 64;
-    out[(j0 + jj) * m + i0 + ii] = tile[ii][jj];
+  // output row jj = t / 4 (column j0 + jj of Phi0), 16 bytes i = iq .. iq + 15
+  const int jj = t >> 2, iq = (t & 3) * 16;
+  uint32_t o[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const uint32_t b0 = static_cast<uint8_t>(tile[(iq + 4 * e) * PITCH + jj]);
+    const uint32_t b1 = static_cast<uint8_t>(tile[(iq + 4 * e + 1) * PITCH + jj]);
+    const uint32_t b2 = static_cast<uint8_t>(tile[(iq + 4 * e + 2) * PITCH + jj]);
+    const uint32_t b3 = static_cast<uint8_t>(tile[(iq + 4 * e + 3) * PITCH + jj]);
+    o[e] = b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
   }
+  *reinterpret_cast<uint4*>(out + (j0 + jj) * m + i0 + iq) = make_uint4(o[0], o[1], o[2], o[3]);
 }
 
 // ------------------------------------------------------------------- reduce --
-__global__ void reduce_rows_kernel(const float* __restrict__ part, int nparts, int64_t n, float lr, int accumulate,
-                                   float* __restrict__ dst) {
+// dst = lr * sum_p part[p] (+ dst), 4 elements per thread, parts summed in a fixed
+// order (four interleaved partial sums, then pairwise), so results are deterministic.
+__global__ void reduce_rows_kernel(const float4* __restrict__ part, int nparts, int64_t n4, float lr,
+                                   int accumulate, float4* __restrict__ dst) {
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= n) return;
-  float acc = 0.0f;
-  for (int p = 0; p < nparts; ++p) acc += part[static_cast<int64_t>(p) * n + e];
-  acc *= lr;
-  dst[e] = accumulate ? dst[e] + acc : acc;
+  if (e >= n4) return;
+  float4 acc[4];
+#pragma unroll
+  for (int a = 0; a < 4; ++a) acc[a] = make_float4(0.f, 0.f, 0.f, 0.f);
+  int p = 0;
+  for (; p + 4 <= nparts; p += 4) {
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+      const float4 v = __ldg(part + static_cast<int64_t>(p + a) * n4 + e);
+      acc[a].x += v.x;
+      acc[a].y += v.y;
+      acc[a].z += v.z;
+      acc[a].w += v.w;
+    }
+  }
+  for (; p < nparts; ++p) {
+    const float4 v = __ldg(part + static_cast<int64_t>(p) * n4 + e);
+    acc[0].x += v.x;
+    acc[0].y += v.y;
+    acc[0].z += v.z;
+    acc[0].w += v.w;
+  }
+  float4 s;
+  s.x = ((acc[0].x + acc[1].x) + (acc[2].x + acc[3].x)) * lr;
+  s.y = ((acc[0].y + acc[1].y) + (acc[2].y + acc[3].y)) * lr;
+  s.z = ((acc[0].z + acc[1].z) + (acc[2].z + acc[3].z)) * lr;
+  s.w = ((acc[0].w + acc[1].w) + (acc[2].w + acc[3].w)) * lr;
+  if (accumulate) {
+    const float4 d = dst[e];
+    s.x += d.x;
+    s.y += d.y;
+    s.z += d.z;
+    s.w += d.w;
+  }
+  dst[e] = s;
 }
 
-__global__ void reduce_ds_kernel(const float* __restrict__ part, int nparts, int64_t m, int64_t nb, int ngroups,
-                                 int blocks_per_group, int accumulate, float* __restrict__ ds) {
+// ds[i] (per channel): one warp per row; lane l sums blocks l, l + 32, ... of every
+// part, then a fixed shuffle tree adds the lanes.
+__global__ void reduce_ds_row_kernel(const float* __restrict__ part, int nparts, int64_t m, int64_t nb, int accumulate,
+                                     float* __restrict__ ds) {
+  const int64_t i = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (i >= m) return;
+  float acc = 0.0f;
+  for (int p = 0; p < nparts; ++p) {
+    const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
+    for (int64_t b = lane; b < nb; b += 32) acc += row[b];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (lane == 0) ds[i] = accumulate ? ds[i] + acc : acc;
+}
+
+// ds[i][g] (per group): one thread per (row, group), sequential over its blocks.
+__global__ void reduce_ds_group_kernel(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
+                                       int ngroups, int blocks_per_group, int accumulate, float* __restrict__ ds) {
   const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (e >= m * ngroups) return;
   const int64_t i = e / ngroups;
@@ -270,27 +381,19 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
   return cudaGetLastError();
 }
 
-cudaError_t launch_pad_rows64(const uint16_t* A, int64_t m, int r, uint16_t* out, cudaStream_t stream) {
-  pad_rows64_kernel<<<blocks_for(m * 64, kThreads), kThreads, 0, stream>>>(A, m, r, out);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_pad_rows(const uint16_t* src, int rows, int rows_pad, int64_t cols, uint16_t* out,
-                            cudaStream_t stream) {
-  pad_rows_kernel<<<blocks_for(static_cast<int64_t>(rows_pad) * cols, kThreads), kThreads, 0, stream>>>(src, rows, rows_pad,
-                                                                                                      cols, out);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_transpose_pad64(const uint16_t* B, int r, int64_t k, uint16_t* out, cudaStream_t stream) {
-  transpose_pad64_kernel<<<blocks_for(k * 64, kThreads), kThreads, 0, stream>>>(B, r, k, out);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_transpose_rows(const uint16_t* A, int64_t m, int r, int r16, uint16_t* out,
-                                  cudaStream_t stream) {
-  transpose_rows_kernel<<<blocks_for(static_cast<int64_t>(r16) * m, kThreads), kThreads, 0, stream>>>(A, m, r, r16,
-                                                                                                     out);
+cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
+                                   uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad,
+                                   cudaStream_t stream) {
+  if ((m % 8) != 0 || (k % 8) != 0) return cudaErrorInvalidValue;
+  const int b_aligned = (reinterpret_cast<uintptr_t>(B) & 15) == 0;
+  const int64_t total = (A_pad ? m * 8 : 0) + (Bt_pad ? k * 8 : 0) + (At ? static_cast<int64_t>(r16) * (m / 8) : 0) +
+                        (B_pad ? static_cast<int64_t>(r16) * (k / 8) : 0);
+  if (total == 0) return cudaSuccess;
+  const int64_t want = blocks_for(total, kThreads);
+  const unsigned grid = static_cast<unsigned>(want < 4096 ? want : 4096);
+  adapter_layouts_kernel<<<grid, kThreads, 0, stream>>>(A, B, m, k, r, r16, reinterpret_cast<uint4*>(A_pad),
+                                                        reinterpret_cast<uint4*>(Bt_pad), reinterpret_cast<uint4*>(At),
+                                                        reinterpret_cast<uint4*>(B_pad), b_aligned);
   return cudaGetLastError();
 }
 
@@ -302,14 +405,20 @@ cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int pac
 }
 
 cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream) {
-  const int64_t nA = a.m * a.r, nB = static_cast<int64_t>(a.r) * a.k;
-  reduce_rows_kernel<<<blocks_for(nA, kThreads), kThreads, 0, stream>>>(a.dA_part, a.nA, nA, a.lr, a.accumulate, a.dA);
-  reduce_rows_kernel<<<blocks_for(nB, kThreads), kThreads, 0, stream>>>(a.dB_part, a.nB, nB, a.lr, a.accumulate, a.dB);
+  const int64_t nA4 = a.m * a.r / 4, nB4 = static_cast<int64_t>(a.r) * a.k / 4;   // m, k are multiples of 128
+  reduce_rows_kernel<<<blocks_for(nA4, kThreads), kThreads, 0, stream>>>(
+      reinterpret_cast<const float4*>(a.dA_part), a.nA, nA4, a.lr, a.accumulate, reinterpret_cast<float4*>(a.dA));
+  reduce_rows_kernel<<<blocks_for(nB4, kThreads), kThreads, 0, stream>>>(
+      reinterpret_cast<const float4*>(a.dB_part), a.nB, nB4, a.lr, a.accumulate, reinterpret_cast<float4*>(a.dB));
   const int64_t nb = a.k / 128;
-  const int ngroups = a.group_size ? static_cast<int>(a.k / a.group_size) : 1;
-  const int bpg = a.group_size ? a.group_size / 128 : static_cast<int>(nb);
-  reduce_ds_kernel<<<blocks_for(a.m * ngroups, kThreads), kThreads, 0, stream>>>(a.ds_part, a.nS, a.m, nb, ngroups,
-                                                                                bpg, a.accumulate, a.ds);
+  if (a.group_size == 0) {
+    reduce_ds_row_kernel<<<blocks_for(a.m * 32, kThreads), kThreads, 0, stream>>>(a.ds_part, a.nS, a.m, nb,
+                                                                                 a.accumulate, a.ds);
+  } else {
+    const int ngroups = static_cast<int>(a.k / a.group_size);
+    reduce_ds_group_kernel<<<blocks_for(a.m * ngroups, kThreads), kThreads, 0, stream>>>(
+        a.ds_part, a.nS, a.m, nb, ngroups, a.group_size / 128, a.accumulate, a.ds);
+  }
   return cudaGetLastError();
 }
 

@@ -20,16 +20,12 @@ cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B,
 // codes = clip(round(X / s_x), -128, 127) as bf16; optional mask bits [k][ceil(T/32)].
 cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const float* s_x, uint16_t* codes,
                              uint32_t* mask, cudaStream_t stream);
-// out[i][c] = c < r ? A[i][c] : 0 for c < 64 (A: [m, r] bf16 -> [m, 64]).
-cudaError_t launch_pad_rows64(const uint16_t* A, int64_t m, int r, uint16_t* out, cudaStream_t stream);
-// out[c][j] = c < rows ? src[c][j] : 0 for c < rows_pad (zero-padded rows).
-cudaError_t launch_pad_rows(const uint16_t* src, int rows, int rows_pad, int64_t cols, uint16_t* out,
-                            cudaStream_t stream);
-// out[j][c] = c < r ? B[c][j] : 0 for c < 64 (B: [r, k] bf16 -> [k, 64]).
-cudaError_t launch_transpose_pad64(const uint16_t* B, int r, int64_t k, uint16_t* out, cudaStream_t stream);
-// out[c][i] = c < r ? A[i][c] : 0 for c < r16 (A: [m, r] -> [r16, m]).
-cudaError_t launch_transpose_rows(const uint16_t* A, int64_t m, int r, int r16, uint16_t* out,
-                                  cudaStream_t stream);
+// TMA-friendly adapter layouts in one launch (null outputs are skipped):
+// A_pad [m][64] = A zero-padded to 64 columns, Bt_pad [k][64] = B^T zero-padded,
+// At [r16][m] = A^T with zero rows r..r16-1, B_pad [r16][k] = B with zero rows.
+cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
+                                   uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad,
+                                   cudaStream_t stream);
 // out[j][i] = stored integer of Phi0[i][j] (int8 raw, or sign-extended nibble), out: int8 [k, m].
 cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int packed, int8_t* out,
                                  cudaStream_t stream);

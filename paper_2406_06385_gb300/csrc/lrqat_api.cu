@@ -434,8 +434,9 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   FwdWs ws;
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
-  LRQAT_LAUNCH("pad_rows64", 1, stream, launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
-  LRQAT_LAUNCH("transpose_pad64", 1, stream, launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
+  LRQAT_LAUNCH("adapter_layouts", 1, stream,
+               launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
+               "adapter layouts");
   const uint16_t* tok = X;
   if (L.act_bits == 8) {
     LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, ws.x_codes, nullptr, stream),
@@ -515,10 +516,9 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   bwd_ws_layout(L, T, plan, workspace, &ws);
   const int r16 = round16(L.r);
   const bool packed = L.phi_format == LRQAT_PHI_INT_PACKED;
-  LRQAT_LAUNCH("pad_rows64", 1, stream, launch_pad_rows64(A, L.m, L.r, ws.a_pad, stream), "pad A");
-  LRQAT_LAUNCH("transpose_pad64", 1, stream, launch_transpose_pad64(B, L.r, L.k, ws.bt_pad, stream), "transpose B");
-  LRQAT_LAUNCH("transpose_rows", 1, stream, launch_transpose_rows(A, L.m, L.r, r16, ws.at, stream), "transpose A");
-  LRQAT_LAUNCH("pad_rows", 1, stream, launch_pad_rows(B, L.r, r16, L.k, ws.b_pad, stream), "pad B");
+  LRQAT_LAUNCH("adapter_layouts", 1, stream,
+               launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, ws.at, ws.b_pad, stream),
+               "adapter layouts");
   LRQAT_LAUNCH("phi_transpose", 1, stream, launch_phi_transpose(Phi0, L.m, L.k, packed, ws.phit, stream),
                "transpose Phi0");
   const uint16_t* xop = X;
