@@ -86,61 +86,119 @@ __global__ void downcast_packed_kernel(const float4* __restrict__ W0, const floa
 }
 
 // -------------------------------------------------------------------- merge --
-// W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p); A B by fp32 FMAs over t = 0..r-1.
+// W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p).  Each thread owns a
+// register tile of 16 rows x 4 columns: per rank index t it reads 16 values of A
+// (shared memory, broadcast) and 4 of B, and does 64 FMAs, so the product A B runs
+// at FMA throughput; the 4 codes of a row go out as one 32-bit store.
 constexpr int kMergeRows = 16;
-__global__ void merge_kernel(const void* __restrict__ phi0, const uint16_t* __restrict__ A,
-                             const uint16_t* __restrict__ B, int64_t m, int64_t k, int r, int packed, QuantParams q,
-                             int8_t* __restrict__ wz) {
-  __shared__ float As[kMergeRows][64];
-  const int64_t j = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+constexpr int kMergeThreads = 128;
+constexpr int kMergeCols = 4 * kMergeThreads;   // 512 columns per block
+__global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __restrict__ phi0,
+                                                              const uint16_t* __restrict__ A,
+                                                              const uint16_t* __restrict__ B, int64_t m, int64_t k,
+                                                              int r, int packed, int b_aligned, QuantParams q,
+                                                              int8_t* __restrict__ wz) {
+  __shared__ __align__(16) float As[64][kMergeRows];   // A^T tile: [t][row]
   const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kMergeRows;
-  for (int e = threadIdx.x; e < kMergeRows * 64; e += blockDim.x) {
-    const int ii = e / 64, t = e % 64;
-    As[ii][t] = (i0 + ii < m && t < r) ? bf16_to_float(A[(i0 + ii) * r + t]) : 0.0f;
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * kMergeCols + 4 * threadIdx.x;
+  for (int e = threadIdx.x; e < kMergeRows * 64; e += kMergeThreads) {
+    const int t = e / kMergeRows, ii = e % kMergeRows;
+    As[t][ii] = (i0 + ii < m && t < r) ? bf16_to_float(A[(i0 + ii) * r + t]) : 0.0f;
   }
   __syncthreads();
   if (j >= k) return;
-  float bcol[64];
+  float acc[kMergeRows][4];
 #pragma unroll
-  for (int t = 0; t < 64; ++t) bcol[t] = t < r ? bf16_to_float(B[static_cast<int64_t>(t) * k + j]) : 0.0f;
-  for (int ii = 0; ii < kMergeRows && i0 + ii < m; ++ii) {
-    const int64_t i = i0 + ii;
-    float L = 0.0f;
+  for (int ii = 0; ii < kMergeRows; ++ii)
 #pragma unroll
-    for (int t = 0; t < 64; ++t)
-      if (t < r) L = __fmaf_rn(As[ii][t], bcol[t], L);
-    float v;
-    if (packed) {
-      const uint8_t byte = static_cast<const uint8_t*>(phi0)[i * (k / 2) + j / 2];
-      int nib = (j & 1) ? (byte >> 4) : (byte & 0xF);
-      v = static_cast<float>(nib >= 8 ? nib - 16 : nib);
+    for (int c = 0; c < 4; ++c) acc[ii][c] = 0.0f;
+  for (int t = 0; t < r; ++t) {
+    const uint16_t* brow = B + static_cast<int64_t>(t) * k + j;
+    uint2 braw;
+    if (b_aligned) {
+      braw = __ldg(reinterpret_cast<const uint2*>(brow));
     } else {
-      v = static_cast<float>(static_cast<const int8_t*>(phi0)[i * k + j]);
+      braw.x = static_cast<uint32_t>(brow[0]) | (static_cast<uint32_t>(brow[1]) << 16);
+      braw.y = static_cast<uint32_t>(brow[2]) | (static_cast<uint32_t>(brow[3]) << 16);
     }
-    wz[i * k + j] = static_cast<int8_t>(__float2int_rn(lrqat_code(L, v, q)));
+    const float b4[4] = {__uint_as_float(braw.x << 16), __uint_as_float(braw.x & 0xFFFF0000u),
+                         __uint_as_float(braw.y << 16), __uint_as_float(braw.y & 0xFFFF0000u)};
+    const float4* arow = reinterpret_cast<const float4*>(&As[t][0]);
+#pragma unroll
+    for (int g = 0; g < kMergeRows / 4; ++g) {
+      const float4 a4 = arow[g];
+      const float av[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[4 * g + u][c] = __fmaf_rn(av[u], b4[c], acc[4 * g + u][c]);
+    }
+  }
+#pragma unroll
+  for (int ii = 0; ii < kMergeRows; ++ii) {
+    const int64_t i = i0 + ii;
+    if (i >= m) break;
+    float v[4];
+    if (packed) {
+      // 4 columns = 2 packed bytes (low nibble = even column)
+      const uint16_t two = *reinterpret_cast<const uint16_t*>(static_cast<const uint8_t*>(phi0) + i * (k / 2) + j / 2);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int nib = (two >> (4 * c)) & 0xF;
+        v[c] = static_cast<float>(nib >= 8 ? nib - 16 : nib);
+      }
+    } else {
+      const uint32_t four = *reinterpret_cast<const uint32_t*>(static_cast<const int8_t*>(phi0) + i * k + j);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[c] = static_cast<float>(static_cast<int8_t>((four >> (8 * c)) & 0xFF));
+    }
+    uint32_t out = 0;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int code = __float2int_rn(lrqat_code(acc[ii][c], v[c], q));
+      out |= (static_cast<uint32_t>(code) & 0xFFu) << (8 * c);
+    }
+    *reinterpret_cast<uint32_t*>(wz + i * k + j) = out;
   }
 }
 
 // --------------------------------------------------------- activation quant --
 // X_Z = clip(round(X / s_x), -128, 127) stored as exact bf16; optional mask bits
 // M_x = 1[-128 <= round(X / s_x) <= 127], laid out [k][ceil(T/32)] (bit = token % 32).
-__global__ void act_quant_kernel(const uint16_t* __restrict__ X, int64_t T, int64_t k, const float* __restrict__ s_x,
-                                 uint16_t* __restrict__ codes, uint32_t* __restrict__ mask, int64_t mask_ld) {
-  const int64_t j = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (j >= k) return;
+// Each thread handles 8 consecutive columns (16-byte loads and stores) of 32 tokens;
+// the division is the IEEE one, so the integer decisions match a plain fp32 X / s_x.
+__global__ void act_quant_kernel(const uint4* __restrict__ X, int64_t T, int64_t k8, const float* __restrict__ s_x,
+                                 uint4* __restrict__ codes, uint32_t* __restrict__ mask, int64_t mask_ld) {
+  const int64_t j8 = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  if (j8 >= k8) return;
   const float sx = *s_x;
   const int64_t t0 = static_cast<int64_t>(blockIdx.y) * 32;
-  uint32_t word = 0;
+  uint32_t word[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   for (int tt = 0; tt < 32; ++tt) {
     const int64_t t = t0 + tt;
     if (t >= T) break;
-    const float x = bf16_to_float(X[t * k + j]);
-    const float qv = rintf(__fdiv_rn(x, sx));
-    const float c = fminf(fmaxf(qv, -128.0f), 127.0f);
-    codes[t * k + j] = static_cast<uint16_t>(__float_as_uint(c) >> 16);
-    if (qv >= -128.0f && qv <= 127.0f) word |= 1u << tt;
+    const uint4 raw = X[t * k8 + j8];
+    const uint32_t in[4] = {raw.x, raw.y, raw.z, raw.w};
+    uint32_t out[4];
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      uint32_t o = 0;
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float x = __uint_as_float(e ? (in[h] & 0xFFFF0000u) : (in[h] << 16));
+        const float qv = rintf(__fdiv_rn(x, sx));
+        const float c = fminf(fmaxf(qv, -128.0f), 127.0f);
+        o |= (__float_as_uint(c) >> 16) << (16 * e);
+        if (qv >= -128.0f && qv <= 127.0f) word[2 * h + e] |= 1u << tt;
+      }
+      out[h] = o;
+    }
+    codes[t * k8 + j8] = make_uint4(out[0], out[1], out[2], out[3]);
   }
-  if (mask) mask[j * mask_ld + blockIdx.y] = word;
+  if (mask) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) mask[(8 * j8 + e) * mask_ld + blockIdx.y] = word[e];
+  }
 }
 
 // ---------------------------------------------------------------- re-layouts --
@@ -369,15 +427,21 @@ cudaError_t launch_downcast(const float* W0, const float* s0, int64_t m, int64_t
 
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
                          int packed, const QuantParams& q, int8_t* wz, cudaStream_t stream) {
-  dim3 grid(static_cast<unsigned>((k + kThreads - 1) / kThreads), static_cast<unsigned>((m + kMergeRows - 1) / kMergeRows));
-  merge_kernel<<<grid, kThreads, 0, stream>>>(phi0, A, B, m, k, r, packed, q, wz);
+  if ((k % 4) != 0 || r > 64) return cudaErrorInvalidValue;
+  const int b_aligned = (reinterpret_cast<uintptr_t>(B) & 7) == 0;
+  dim3 grid(static_cast<unsigned>((k + kMergeCols - 1) / kMergeCols), static_cast<unsigned>((m + kMergeRows - 1) / kMergeRows));
+  merge_kernel<<<grid, kMergeThreads, 0, stream>>>(phi0, A, B, m, k, r, packed, b_aligned, q, wz);
   return cudaGetLastError();
 }
 
 cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const float* s_x, uint16_t* codes,
                              uint32_t* mask, cudaStream_t stream) {
-  dim3 grid(static_cast<unsigned>((k + 127) / 128), static_cast<unsigned>((T + 31) / 32));
-  act_quant_kernel<<<grid, 128, 0, stream>>>(X, T, k, s_x, codes, mask, (T + 31) / 32);
+  if ((k % 8) != 0 || (reinterpret_cast<uintptr_t>(X) & 15) != 0 || (reinterpret_cast<uintptr_t>(codes) & 15) != 0)
+    return cudaErrorInvalidValue;
+  const int64_t k8 = k / 8;
+  dim3 grid(static_cast<unsigned>((k8 + 127) / 128), static_cast<unsigned>((T + 31) / 32));
+  act_quant_kernel<<<grid, 128, 0, stream>>>(reinterpret_cast<const uint4*>(X), T, k8, s_x,
+                                             reinterpret_cast<uint4*>(codes), mask, (T + 31) / 32);
   return cudaGetLastError();
 }
 
