@@ -1,0 +1,146 @@
+"""GPU parity at the benchmark's full sizes, in the launch configuration that
+bench.py times: one lrqat_linear_fwd and one lrqat_linear_bwd call over all
+T = 8192 tokens of a LLaMA-shaped layer.
+
+The oracle cannot redo a full 8192-token layer in a test's time, so it checks
+what it can compute exactly, one piece at a time:
+  * every integer code of W_hat that the fused producers build, bit for bit
+    (identity inputs turn the forward output into C^T and the dX output into C;
+    near-ties exempt, as in the small-size tests);
+  * Y and dX at sampled token rows (all output columns of those rows);
+  * dA and ds at sampled weight rows and dB at sampled weight columns, from the
+    rows / columns of G = dY^T X_hat that the oracle forms in fp64.
+Sampled outputs are compared with the same relative Frobenius tolerances as the
+small-size tests (1e-2 for Y and dX, 2e-2 for the adapter and scale gradients).
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2406_06385_gb300 import lrqat as LQ
+from paper_2406_06385_gb300 import workloads as WL
+
+from gpu_util import DeviceLayer, bits_to_f32, oracle_layer, to_dev, torch
+
+pytestmark = pytest.mark.gpu
+
+TOL_ACT = 1e-2
+TOL_GRAD = 2e-2
+T_FULL = 8192
+
+# The bench layer (4096 x 4096, Q4.4 per channel), the largest projection of the
+# W4 g128 + A8 MLP (14336 x 4096) and the INT-3 packed down projection (4096 x 11008).
+FULL_CASES = [
+    ("llama2_7b_attn", WL.workload("llama2_7b_attn").layers[0]),
+    ("llama3_8b_gate_g128_a8", WL.workload("llama3_8b_mlp").layers[0]),
+    ("llama2_7b_down_int3", WL.workload("llama2_7b_mlp").layers[2]),
+]
+
+
+def _codes_spec(spec):
+    # the codes do not depend on the activation quantizer; identity inputs need it off
+    return WL.LayerSpec(spec.name, spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format,
+                        0, spec.w_std, spec.outlier_frac, spec.outlier_mult, spec.a_std, spec.b_std)
+
+
+@pytest.mark.parametrize("cid,spec", FULL_CASES, ids=[c[0] for c in FULL_CASES])
+def test_full_size_codes_bit_exact(cid, spec):
+    t = torch()
+    spec = _codes_spec(spec)
+    data = WL.make_layer(spec, 1, seed=3, with_activations=False)
+    dl = DeviceLayer(data)
+    dl.s = t.ones_like(dl.s)
+    L = dl.layer
+    m, k = spec.m, spec.k
+    # forward with X = I_k: Y[j, i] = c[i, j]
+    X = t.eye(k, dtype=t.bfloat16, device="cuda").view(t.int16)
+    Y = t.empty((k, m), dtype=t.int16, device="cuda")
+    ws = t.empty(max(LQ.fwd_workspace_bytes(L, k), 16), dtype=t.uint8, device="cuda")
+    LQ.linear_fwd(L, k, X, dl.phi0, dl.s, dl.A, dl.B, None, Y, ws)
+    c_fwd = bits_to_f32(Y).T
+    del X, Y, ws
+    # dX with dY = I_m: dX[i, j] = c[i, j]
+    dYe = t.eye(m, dtype=t.bfloat16, device="cuda").view(t.int16)
+    Xz = t.zeros((m, k), dtype=t.int16, device="cuda")
+    dX = t.empty((m, k), dtype=t.int16, device="cuda")
+    dA = t.empty((m, spec.r), dtype=t.float32, device="cuda")
+    dB = t.empty((spec.r, k), dtype=t.float32, device="cuda")
+    ds = t.empty_like(dl.s)
+    wsb = t.empty(LQ.bwd_workspace_bytes(L, m), dtype=t.uint8, device="cuda")
+    LQ.linear_bwd(L, m, dYe, Xz, dl.phi0, dl.s, dl.A, dl.B, None, dX, dA, dB, ds, False, wsb)
+    LQ.get_device_status()
+    c_dx = bits_to_f32(dX)
+    OL = oracle_layer(spec)
+    phi0 = O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL)
+    u = O.preround(phi0, data.A, data.B, OL)
+    c = O.codes_from_u(u, OL)[1]
+    exempt = O.near_tie(u)
+    for name, got in (("fwd", c_fwd), ("dX", c_dx)):
+        bad = (got != c) & ~exempt
+        assert bad.sum() == 0, f"{name}: {bad.sum()} code mismatches of {c.size} (near-ties exempt: {exempt.sum()})"
+
+
+@pytest.mark.parametrize("cid,spec", FULL_CASES, ids=[c[0] for c in FULL_CASES])
+def test_full_size_sampled_outputs(cid, spec):
+    t = torch()
+    T = T_FULL
+    data = WL.make_layer(spec, T, seed=11)
+    dl = DeviceLayer(data)
+    L = dl.layer
+    X, dY = to_dev(data.X_bits), to_dev(data.dY_bits)
+    s_x_host, s_x = None, None
+    if spec.act_bits == 8:
+        s_x_host = np.float32(np.float32(np.abs(data.X).max()) / np.float32(127.0))
+        s_x = t.tensor([s_x_host], dtype=t.float32, device="cuda")
+    Y = t.empty((T, spec.m), dtype=t.int16, device="cuda")
+    ws = t.empty(max(LQ.fwd_workspace_bytes(L, T), 16), dtype=t.uint8, device="cuda")
+    LQ.linear_fwd(L, T, X, dl.phi0, dl.s, dl.A, dl.B, s_x, Y, ws)
+    dX = t.empty((T, spec.k), dtype=t.int16, device="cuda")
+    dA = t.empty((spec.m, spec.r), dtype=t.float32, device="cuda")
+    dB = t.empty((spec.r, spec.k), dtype=t.float32, device="cuda")
+    ds = t.empty_like(dl.s)
+    wsb = t.empty(LQ.bwd_workspace_bytes(L, T), dtype=t.uint8, device="cuda")
+    LQ.linear_bwd(L, T, dY, X, dl.phi0, dl.s, dl.A, dl.B, s_x, dX, dA, dB, ds, False, wsb)
+    LQ.get_device_status()
+
+    OL = oracle_layer(spec)
+    s0 = O.minmax_scale(data.W0, OL)
+    phi0 = O.downcast(data.W0, s0, OL)
+    fq = O.fake_quant_weight(phi0, s0, data.A, data.B, OL)
+    if spec.act_bits == 8:
+        _, Xh, Mx = O.act_quant(data.X, s_x_host)
+    else:
+        Xh = data.X.astype(np.float64)
+        Mx = np.ones_like(Xh)
+    dYf = data.dY.astype(np.float64)
+    scale = OL.alpha / OL.r
+
+    # Y and dX at sampled token rows (every column)
+    ts = WL.token_sample(T, 24, seed=1)
+    Y_ref = Xh[ts] @ fq["W_hat"].T
+    dX_ref = (dYf[ts] @ fq["W_hat"]) * Mx[ts]
+    Y_got = bits_to_f32(Y[t.as_tensor(ts, device="cuda")])
+    dX_got = bits_to_f32(dX[t.as_tensor(ts, device="cuda")])
+    assert O.rel_fro(Y_got, Y_ref) <= TOL_ACT
+    assert O.rel_fro(dX_got, dX_ref) <= TOL_ACT
+
+    # dA and ds at sampled weight rows: rows of G, dU and the codes
+    rows = WL.token_sample(spec.m, 6, seed=2)
+    G_rows = dYf[:, rows].T @ Xh
+    s_rows = O.expand_scale(s0, OL)[rows]
+    dU_rows = G_rows * s_rows * fq["M"][rows]
+    dA_ref = scale * (dU_rows @ data.B.astype(np.float64).T)
+    Gc = G_rows * fq["c"][rows]
+    ds_ref = Gc.sum(axis=1) if spec.group_size == 0 else Gc.reshape(len(rows), -1, spec.group_size).sum(axis=2)
+    dA_got = dA.cpu().numpy()[rows]
+    ds_got = ds.cpu().numpy().reshape((spec.m, -1) if spec.group_size else (spec.m,))[rows]
+    assert O.rel_fro(dA_got, dA_ref) <= TOL_GRAD
+    assert O.rel_fro(ds_got, ds_ref) <= TOL_GRAD
+
+    # dB at sampled weight columns: columns of G and dU
+    cols = WL.token_sample(spec.k, 6, seed=3)
+    G_cols = dYf.T @ Xh[:, cols]
+    dU_cols = G_cols * O.expand_scale(s0, OL)[:, cols] * fq["M"][:, cols]
+    dB_ref = scale * (data.A.astype(np.float64).T @ dU_cols)
+    dB_got = dB.cpu().numpy()[:, cols]
+    assert O.rel_fro(dB_got, dB_ref) <= TOL_GRAD
