@@ -269,107 +269,136 @@ __global__ void adapter_layouts_kernel(const uint16_t* __restrict__ A, const uin
   }
 }
 
-// 64 x 64 tiles of Phi0 (rows i, columns j) -> out[j][i] as int8 stored integers.
-// Each thread loads 16 stored integers of one row (16 bytes, or 8 packed bytes)
-// and writes 16 bytes of one transposed row; the tile passes through shared
-// memory with a 68-byte pitch (4-byte aligned rows, at most 2-way conflicts on the
-// column reads).
+// 128 x 128 tiles of Phi0 (rows i, columns j) -> out[j][i] as int8 stored integers.
+// Load: each thread brings four pieces of 16 stored integers (16 bytes, or 8 packed
+// bytes) into a shared tile whose 16-byte groups are XOR-swizzled by the row's
+// 16-row block, so that the column gathers below hit 32 distinct banks.
+// Store: each thread transposes a 16-row x 4-column block with byte permutes and
+// writes four 16-byte pieces of transposed rows (8 threads cover one 128-byte row).
+__device__ __forceinline__ void unpack_i4x8(uint32_t packed4, uint32_t& lo_word, uint32_t& hi_word) {
+  // 4 packed bytes -> 8 sign-extended nibbles (low nibble = even column)
+  const uint32_t x = packed4 ^ 0x88888888u;
+  const uint32_t lo = x & 0x0F0F0F0Fu, hi = (x >> 4) & 0x0F0F0F0Fu;
+  lo_word = __vsub4(__byte_perm(lo, hi, 0x5140), 0x08080808u);
+  hi_word = __vsub4(__byte_perm(lo, hi, 0x7362), 0x08080808u);
+}
+
 __global__ void __launch_bounds__(256) phi_transpose_kernel(const void* __restrict__ phi0, int64_t m, int64_t k,
                                                              int packed, int8_t* __restrict__ out) {
-  constexpr int PITCH = 68;
-  __shared__ __align__(16) int8_t tile[64 * PITCH];
-  const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 64;
-  const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 64;
+  __shared__ __align__(16) uint32_t tile[128 * 32];   // 128 rows x 32 words
+  const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 128;
+  const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 128;
   const int t = threadIdx.x;
-  const int ii = t >> 2, jq = (t & 3) * 16;
-  uint32_t v[4];
+  uint4 v[4];
   if (packed) {
-    const uint2 raw =
-        *reinterpret_cast<const uint2*>(static_cast<const uint8_t*>(phi0) + (i0 + ii) * (k / 2) + (j0 + jq) / 2);
-    const uint32_t src[2] = {raw.x, raw.y};
+    const uint8_t* src = static_cast<const uint8_t*>(phi0);
+    uint2 raw[4];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      // 4 packed bytes -> 8 sign-extended nibbles (low nibble = even column)
-      const uint32_t x = src[h] ^ 0x88888888u;
-      const uint32_t lo = x & 0x0F0F0F0Fu, hi = (x >> 4) & 0x0F0F0F0Fu;
-      // bytes: (lo0, hi0, lo1, hi1) and (lo2, hi2, lo3, hi3), then subtract 8 from each byte
-      const uint32_t b01 = __byte_perm(lo, hi, 0x5140), b23 = __byte_perm(lo, hi, 0x7362);
-      v[2 * h] = __vsub4(b01, 0x08080808u);
-      v[2 * h + 1] = __vsub4(b23, 0x08080808u);
+    for (int x = 0; x < 4; ++x) {
+      const int u = t + 256 * x, R = u >> 3, q = u & 7;
+      raw[x] = *reinterpret_cast<const uint2*>(src + (i0 + R) * (k / 2) + (j0 + 16 * q) / 2);
+    }
+#pragma unroll
+    for (int x = 0; x < 4; ++x) {
+      unpack_i4x8(raw[x].x, v[x].x, v[x].y);
+      unpack_i4x8(raw[x].y, v[x].z, v[x].w);
     }
   } else {
-    const uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const int8_t*>(phi0) + (i0 + ii) * k + j0 + jq);
-    v[0] = raw.x;
-    v[1] = raw.y;
-    v[2] = raw.z;
-    v[3] = raw.w;
-  }
-  uint32_t* row = reinterpret_cast<uint32_t*>(tile + ii * PITCH + jq);
+    const int8_t* src = static_cast<const int8_t*>(phi0);
 #pragma unroll
-  for (int e = 0; e < 4; ++e) row[e] = v[e];
+    for (int x = 0; x < 4; ++x) {
+      const int u = t + 256 * x, R = u >> 3, q = u & 7;
+      v[x] = *reinterpret_cast<const uint4*>(src + (i0 + R) * k + j0 + 16 * q);
+    }
+  }
+#pragma unroll
+  for (int x = 0; x < 4; ++x) {
+    const int u = t + 256 * x, R = u >> 3, q = u & 7;
+    *reinterpret_cast<uint4*>(&tile[R * 32 + 4 * (q ^ ((R >> 4) & 7))]) = v[x];
+  }
   __syncthreads();
-  // output row jj = t / 4 (column j0 + jj of Phi0), 16 bytes i = iq .. iq + 15
-  const int jj = t >> 2, iq = (t & 3) * 16;
-  uint32_t o[4];
+  const int w = t >> 5, L = t & 31;
+  const int a = L & 7;                    // 16-row block of the tile (rows i)
+  const int c = 4 * w + (L >> 3);         // word column: columns j = 4c .. 4c + 3
+  const int wcol = 4 * (w ^ a) + (L >> 3);   // its swizzled position (all rows of block a)
+  uint32_t o[4][4];
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const uint32_t b0 = static_cast<uint8_t>(tile[(iq + 4 * e) * PITCH + jj]);
-    const uint32_t b1 = static_cast<uint8_t>(tile[(iq + 4 * e + 1) * PITCH + jj]);
-    const uint32_t b2 = static_cast<uint8_t>(tile[(iq + 4 * e + 2) * PITCH + jj]);
-    const uint32_t b3 = static_cast<uint8_t>(tile[(iq + 4 * e + 3) * PITCH + jj]);
-    o[e] = b0 | (b1 << 8) | (b2 << 16) | (b3 << 24);
+  for (int blk = 0; blk < 4; ++blk) {
+    const int R = 16 * a + 4 * blk;
+    const uint32_t x0 = tile[R * 32 + wcol], x1 = tile[(R + 1) * 32 + wcol];
+    const uint32_t x2 = tile[(R + 2) * 32 + wcol], x3 = tile[(R + 3) * 32 + wcol];
+    const uint32_t t01lo = __byte_perm(x0, x1, 0x5140), t01hi = __byte_perm(x0, x1, 0x7362);
+    const uint32_t t23lo = __byte_perm(x2, x3, 0x5140), t23hi = __byte_perm(x2, x3, 0x7362);
+    o[0][blk] = __byte_perm(t01lo, t23lo, 0x5410);
+    o[1][blk] = __byte_perm(t01lo, t23lo, 0x7632);
+    o[2][blk] = __byte_perm(t01hi, t23hi, 0x5410);
+    o[3][blk] = __byte_perm(t01hi, t23hi, 0x7632);
   }
-  *reinterpret_cast<uint4*>(out + (j0 + jj) * m + i0 + iq) = make_uint4(o[0], o[1], o[2], o[3]);
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+    *reinterpret_cast<uint4*>(out + (j0 + 4 * c + r) * m + i0 + 16 * a) = make_uint4(o[r][0], o[r][1], o[r][2], o[r][3]);
 }
 
 // ------------------------------------------------------------------- reduce --
-// dst = lr * sum_p part[p] (+ dst), 4 elements per thread, parts summed in a fixed
-// order (four interleaved partial sums, then pairwise), so results are deterministic.
-__global__ void reduce_rows_kernel(const float4* __restrict__ part, int nparts, int64_t n4, float lr,
-                                   int accumulate, float4* __restrict__ dst) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (e >= n4) return;
-  float4 acc[4];
-#pragma unroll
-  for (int a = 0; a < 4; ++a) acc[a] = make_float4(0.f, 0.f, 0.f, 0.f);
-  int p = 0;
-  for (; p + 4 <= nparts; p += 4) {
-#pragma unroll
-    for (int a = 0; a < 4; ++a) {
-      const float4 v = __ldg(part + static_cast<int64_t>(p + a) * n4 + e);
-      acc[a].x += v.x;
-      acc[a].y += v.y;
-      acc[a].z += v.z;
-      acc[a].w += v.w;
+// One launch sums every gradient partial. Block ranges: [0, nblk_a) dA, then dB, then ds.
+// dA / dB: a block owns 32 float4 columns; warp w adds parts w, w + 8, w + 16, ... in that
+// order, and the eight warp sums are added in a fixed tree, so results are deterministic.
+constexpr int kRedSlices = kThreads / 32;
+
+struct RedJob {
+  const float4* part;
+  int nparts;
+  int64_t n4;
+  float4* dst;
+};
+
+__device__ __forceinline__ void add4(float4& a, const float4& b) {
+  a.x += b.x;
+  a.y += b.y;
+  a.z += b.z;
+  a.w += b.w;
+}
+
+__device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk, float lr, int accumulate,
+                                                   float4 (*sm)[32]) {
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t e = blk * 32 + lane;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (e < j.n4) {
+    int p = w;
+    for (; p + 3 * kRedSlices < j.nparts; p += 4 * kRedSlices) {
+      const float4 v0 = __ldg(j.part + static_cast<int64_t>(p) * j.n4 + e);
+      const float4 v1 = __ldg(j.part + static_cast<int64_t>(p + kRedSlices) * j.n4 + e);
+      const float4 v2 = __ldg(j.part + static_cast<int64_t>(p + 2 * kRedSlices) * j.n4 + e);
+      const float4 v3 = __ldg(j.part + static_cast<int64_t>(p + 3 * kRedSlices) * j.n4 + e);
+      add4(acc, v0);
+      add4(acc, v1);
+      add4(acc, v2);
+      add4(acc, v3);
     }
+    for (; p < j.nparts; p += kRedSlices) add4(acc, __ldg(j.part + static_cast<int64_t>(p) * j.n4 + e));
   }
-  for (; p < nparts; ++p) {
-    const float4 v = __ldg(part + static_cast<int64_t>(p) * n4 + e);
-    acc[0].x += v.x;
-    acc[0].y += v.y;
-    acc[0].z += v.z;
-    acc[0].w += v.w;
+  sm[w][lane] = acc;
+  __syncthreads();
+  if (w == 0 && e < j.n4) {
+    float4 s[kRedSlices];
+#pragma unroll
+    for (int i = 0; i < kRedSlices; ++i) s[i] = sm[i][lane];
+#pragma unroll
+    for (int h = kRedSlices / 2; h > 0; h >>= 1)
+#pragma unroll
+      for (int i = 0; i < h; ++i) add4(s[i], s[i + h]);
+    float4 r = make_float4(s[0].x * lr, s[0].y * lr, s[0].z * lr, s[0].w * lr);
+    if (accumulate) add4(r, j.dst[e]);
+    j.dst[e] = r;
   }
-  float4 s;
-  s.x = ((acc[0].x + acc[1].x) + (acc[2].x + acc[3].x)) * lr;
-  s.y = ((acc[0].y + acc[1].y) + (acc[2].y + acc[3].y)) * lr;
-  s.z = ((acc[0].z + acc[1].z) + (acc[2].z + acc[3].z)) * lr;
-  s.w = ((acc[0].w + acc[1].w) + (acc[2].w + acc[3].w)) * lr;
-  if (accumulate) {
-    const float4 d = dst[e];
-    s.x += d.x;
-    s.y += d.y;
-    s.z += d.z;
-    s.w += d.w;
-  }
-  dst[e] = s;
 }
 
 // ds[i] (per channel): one warp per row; lane l sums blocks l, l + 32, ... of every
 // part, then a fixed shuffle tree adds the lanes.
-__global__ void reduce_ds_row_kernel(const float* __restrict__ part, int nparts, int64_t m, int64_t nb, int accumulate,
-                                     float* __restrict__ ds) {
-  const int64_t i = (blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x) >> 5;
+__device__ __forceinline__ void reduce_ds_row(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
+                                              int accumulate, float* __restrict__ ds, int64_t blk) {
+  const int64_t i = (blk * kThreads + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (i >= m) return;
   float acc = 0.0f;
@@ -383,9 +412,10 @@ __global__ void reduce_ds_row_kernel(const float* __restrict__ part, int nparts,
 }
 
 // ds[i][g] (per group): one thread per (row, group), sequential over its blocks.
-__global__ void reduce_ds_group_kernel(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
-                                       int ngroups, int blocks_per_group, int accumulate, float* __restrict__ ds) {
-  const int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+__device__ __forceinline__ void reduce_ds_group(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
+                                                int ngroups, int blocks_per_group, int accumulate,
+                                                float* __restrict__ ds, int64_t blk) {
+  const int64_t e = blk * kThreads + threadIdx.x;
   if (e >= m * ngroups) return;
   const int64_t i = e / ngroups;
   const int g = static_cast<int>(e % ngroups);
@@ -395,6 +425,22 @@ __global__ void reduce_ds_group_kernel(const float* __restrict__ part, int npart
     for (int b = g * blocks_per_group; b < (g + 1) * blocks_per_group; ++b) acc += row[b];
   }
   ds[e] = accumulate ? ds[e] + acc : acc;
+}
+
+__global__ void __launch_bounds__(kThreads) reduce_grads_kernel(RedJob ja, RedJob jb, int64_t nblk_a, int64_t nblk_b,
+                                                                ReduceArgs a, int64_t nb, int ngroups) {
+  __shared__ float4 sm[kRedSlices][32];
+  const int64_t blk = blockIdx.x;
+  if (blk < nblk_a) {
+    reduce_parts_block(ja, blk, a.lr, a.accumulate, sm);
+  } else if (blk < nblk_a + nblk_b) {
+    reduce_parts_block(jb, blk - nblk_a, a.lr, a.accumulate, sm);
+  } else if (a.group_size == 0) {
+    reduce_ds_row(a.ds_part, a.nS, a.m, nb, a.accumulate, a.ds, blk - nblk_a - nblk_b);
+  } else {
+    reduce_ds_group(a.ds_part, a.nS, a.m, nb, ngroups, a.group_size / 128, a.accumulate, a.ds,
+                    blk - nblk_a - nblk_b);
+  }
 }
 
 }  // namespace
@@ -463,26 +509,22 @@ cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t
 
 cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int packed, int8_t* out,
                                  cudaStream_t stream) {
-  dim3 grid(static_cast<unsigned>(k / 64), static_cast<unsigned>(m / 64));
+  if ((m % 128) != 0 || (k % 128) != 0) return cudaErrorInvalidValue;
+  dim3 grid(static_cast<unsigned>(k / 128), static_cast<unsigned>(m / 128));
   phi_transpose_kernel<<<grid, kThreads, 0, stream>>>(phi0, m, k, packed, out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream) {
   const int64_t nA4 = a.m * a.r / 4, nB4 = static_cast<int64_t>(a.r) * a.k / 4;   // m, k are multiples of 128
-  reduce_rows_kernel<<<blocks_for(nA4, kThreads), kThreads, 0, stream>>>(
-      reinterpret_cast<const float4*>(a.dA_part), a.nA, nA4, a.lr, a.accumulate, reinterpret_cast<float4*>(a.dA));
-  reduce_rows_kernel<<<blocks_for(nB4, kThreads), kThreads, 0, stream>>>(
-      reinterpret_cast<const float4*>(a.dB_part), a.nB, nB4, a.lr, a.accumulate, reinterpret_cast<float4*>(a.dB));
+  const RedJob ja{reinterpret_cast<const float4*>(a.dA_part), a.nA, nA4, reinterpret_cast<float4*>(a.dA)};
+  const RedJob jb{reinterpret_cast<const float4*>(a.dB_part), a.nB, nB4, reinterpret_cast<float4*>(a.dB)};
+  const int64_t nblk_a = (nA4 + 31) / 32, nblk_b = (nB4 + 31) / 32;
   const int64_t nb = a.k / 128;
-  if (a.group_size == 0) {
-    reduce_ds_row_kernel<<<blocks_for(a.m * 32, kThreads), kThreads, 0, stream>>>(a.ds_part, a.nS, a.m, nb,
-                                                                                 a.accumulate, a.ds);
-  } else {
-    const int ngroups = static_cast<int>(a.k / a.group_size);
-    reduce_ds_group_kernel<<<blocks_for(a.m * ngroups, kThreads), kThreads, 0, stream>>>(
-        a.ds_part, a.nS, a.m, nb, ngroups, a.group_size / 128, a.accumulate, a.ds);
-  }
+  const int ngroups = a.group_size ? static_cast<int>(a.k / a.group_size) : 1;
+  const int64_t nblk_s = a.group_size == 0 ? blocks_for(a.m * 32, kThreads) : blocks_for(a.m * ngroups, kThreads);
+  reduce_grads_kernel<<<static_cast<unsigned>(nblk_a + nblk_b + nblk_s), kThreads, 0, stream>>>(ja, jb, nblk_a, nblk_b,
+                                                                                               a, nb, ngroups);
   return cudaGetLastError();
 }
 

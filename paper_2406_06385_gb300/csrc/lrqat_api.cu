@@ -618,7 +618,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   ra.group_size = L.group_size;
   ra.lr = static_cast<float>(static_cast<double>(L.alpha) / L.r);
   ra.accumulate = accumulate ? 1 : 0;
-  LRQAT_LAUNCH("reduce_grads", 3, stream, launch_reduce(ra, stream), "gradient reduction");
+  LRQAT_LAUNCH("reduce_grads", 1, stream, launch_reduce(ra, stream), "gradient reduction");
   return LRQAT_OK;
 }
 
