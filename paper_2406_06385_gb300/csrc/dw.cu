@@ -350,6 +350,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             st_shared_v4(dub + swz_offset(row, 4 * p + wq, 128), du[4 * wq], du[4 * wq + 1], du[4 * wq + 2],
                          du[4 * wq + 3]);
         }
+        if (c == args.nchunks - 1) {
+          // Last read of G for this unit: hand the accumulator to the next unit's main
+          // loop, which then overlaps the adapter contractions and partial stores below.
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(BAR_ACCEMPTY));
+        }
         // ds partial of this 128-column block (two halves h per row)
         args.ds_part[(static_cast<int64_t>(w.sp * 2 + h) * args.m + i_g) * nb + j0 / 128] = ds_acc;
         tc_fence_before();
@@ -389,9 +396,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         ++cc;
       }
       if (!ok) break;
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(BAR_ACCEMPTY));
       ++it;
     }
   }

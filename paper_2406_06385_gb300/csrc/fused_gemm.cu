@@ -9,7 +9,8 @@
 //     also holds the bf16 operand tile W_hat of its stage;
 //   * factor ring (4 slots): one loader warp brings the stored base (128 x 64
 //     int8, SW64; packed: 128 x 32 bytes, SW32) and a 64-row slice of the second
-//     low-rank factor (SW128);
+//     low-rank factor, only its first r16 columns (rows of 32, 64 or 128 bytes,
+//     swizzled to the row width);
 //   * the MMA warp computes the low-rank tile L = RF * SF^T (M=128, N=64, K=r
 //     rounded to 16) into a TMEM buffer, issued ahead of the main product of the
 //     previous stage so that it is ready when that product finishes;
@@ -56,7 +57,7 @@ constexpr uint32_t TOK_HALF = BN * 128;          // 224 tokens x 64 bf16
 constexpr uint32_t TOK_BYTES = 2 * TOK_HALF;
 constexpr uint32_t W_BYTES = 128 * 128;          // 128 rows x 64 bf16
 constexpr uint32_t PHI_BYTES = 128 * 64;         // 128 rows x 64 int8 (packed: half)
-constexpr uint32_t SF_BYTES = 64 * 128;          // 64 slice rows x 64 rank columns (bf16)
+constexpr uint32_t SF_BYTES = 64 * 128;          // 64 slice rows x up to 64 rank columns (bf16)
 constexpr uint32_t TSLOT_BYTES = TOK_BYTES + W_BYTES;
 constexpr uint32_t FSLOT_BYTES = PHI_BYTES + SF_BYTES;
 constexpr uint32_t OFF_RF = 0;
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       prefetch_tensormap(&tm_phi);
       prefetch_tensormap(&tm_sf);
     }
-    constexpr uint32_t tx = (PACKED ? PHI_BYTES / 2 : PHI_BYTES) + SF_BYTES;
+    const uint32_t tx = (PACKED ? PHI_BYTES / 2 : PHI_BYTES) + static_cast<uint32_t>(BK * 2 * args.sf_cols);
     uint32_t gg = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
@@ -225,7 +226,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int lsteps = args.r16 / 16;
       constexpr uint32_t TSLOT_D = TSLOT_BYTES >> 4, FSLOT_D = FSLOT_BYTES >> 4, TOKH_D = TOK_HALF >> 4;
       const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
-      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + FS_SF, 16, 1024, SWZ_128B);
+      // The factor slice has rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to match).
+      const uint32_t sf_swz = args.sf_cols == 16 ? SWZ_32B : args.sf_cols == 32 ? SWZ_64B : SWZ_128B;
+      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + FS_SF, 16, 16u * args.sf_cols, sf_swz);
       const uint64_t d_w0 = make_sdesc(smem + OFF_TSLOTS + TS_W, 16, 1024, SWZ_128B);
       const uint64_t d_tok0 = make_sdesc(smem + OFF_TSLOTS, 16, 1024, SWZ_128B);
       uint32_t g = 0;

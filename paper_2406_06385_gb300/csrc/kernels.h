@@ -49,6 +49,7 @@ struct FusedArgs {
   int32_t kdim;          // contraction length (k for fwd, m for dX)
   int32_t T;             // tokens
   int32_t r16;           // adapter rank rounded up to 16
+  int32_t sf_cols;       // columns of the second factor loaded per stage (16, 32 or 64)
   int32_t num_rb;        // rows / 128
   int32_t num_tb;        // ceil(T / 448)
   int32_t num_tiles;

@@ -98,6 +98,15 @@ int encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* ptr, uint64_
   return LRQAT_OK;
 }
 
+// The fused GEMMs load only the first r16 columns of the second low-rank factor per
+// stage, as rows of 32, 64 or 128 bytes with the matching swizzle (rank 33..48 keeps
+// 64 columns: no swizzle mode has 96-byte rows).
+int sf_cols(int r16) { return r16 == 48 ? 64 : r16; }
+CUtensorMapSwizzle sf_swizzle(int r16) {
+  const int c = sf_cols(r16);
+  return c == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : c == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int frac_bits(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_QFIXED ? 8 - L.bits : 0; }
@@ -449,13 +458,14 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 64, false));
   LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
                       CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
-  LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 64,
-                      CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
+  LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, sf_cols(r16), 64,
+                      sf_swizzle(r16), "B^T (padded)"));
   FusedArgs a{};
   a.rows = static_cast<int32_t>(L.m);
   a.kdim = static_cast<int32_t>(L.k);
   a.T = static_cast<int32_t>(T);
   a.r16 = r16;
+  a.sf_cols = sf_cols(r16);
   a.num_rb = static_cast<int32_t>(L.m / 128);
   a.num_tb = static_cast<int32_t>((T + 447) / 448);
   a.num_tiles = a.num_rb * a.num_tb;
@@ -538,13 +548,14 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
                         CU_TENSOR_MAP_SWIZZLE_64B, "Phi0^T"));
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
-    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 64,
-                        CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
+    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16), 64,
+                        sf_swizzle(r16), "A (padded)"));
     FusedArgs a{};
     a.rows = static_cast<int32_t>(L.k);
     a.kdim = static_cast<int32_t>(L.m);
     a.T = static_cast<int32_t>(T);
     a.r16 = r16;
+    a.sf_cols = sf_cols(r16);
     a.num_rb = static_cast<int32_t>(L.k / 128);
     a.num_tb = static_cast<int32_t>((T + 447) / 448);
     a.num_tiles = a.num_rb * a.num_tb;

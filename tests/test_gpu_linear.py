@@ -38,6 +38,7 @@ CASES = [
     ("q44_g256", spec_of("g", 128, 512, 32, group=256, a_std=0.2, b_std=0.2), 256),
     ("q26_clip_heavy", spec_of("h", 128, 256, 16, bits=2, a_std=1.0, b_std=1.0), 200),
     ("tokens_1", spec_of("i", 128, 128, 1), 1),
+    ("q44_pc_r40", spec_of("j", 256, 256, 40, a_std=0.2, b_std=0.2), 130),
 ]
 
 
