@@ -373,9 +373,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (MODE == FUSED_FWD_PC) {
             w[e] = codes_bf16x2(t2, qp);
           } else {
-            const float2 c2 = codes_f32x2(t2, qp);
-            const float2 v2 = __fmul2_rn(c2, make_float2(sc[2 * e], sc[2 * e + 1]));
-            w[e] = pack_rn_bf16x2(v2.x, v2.y);
+            // bf16(bf16(s) * c): the exact bf16 codes times the bf16-rounded scales,
+            // one packed multiply instead of an fp32 clip, multiply and conversion.
+            w[e] = mul_bf16x2(codes_bf16x2(t2, qp), pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
           }
         }
         // The W_hat buffer of this token slot was last read by the product of stage gg - 2.

@@ -88,12 +88,6 @@ __device__ __forceinline__ uint32_t codes_bf16x2(float2 t, const QuantParams& q)
   return w;
 }
 
-// Clipped codes of two elements as fp32 (exact).
-__device__ __forceinline__ float2 codes_f32x2(float2 t, const QuantParams& q) {
-  const float2 tc = make_float2(fminf(fmaxf(t.x, q.lo), q.hi), fminf(fmaxf(t.y, q.lo), q.hi));
-  return __ffma2_rn(tc, make_float2(q.inv2f, q.inv2f), make_float2(-q.magic_c, -q.magic_c));
-}
-
 // 4 signed bytes of `w` -> 4 exact floats.
 __device__ __forceinline__ void decode_i8x4(uint32_t w, float* v) {
   const uint32_t x = w ^ 0x80808080u;   // v + 128 in each byte
@@ -140,6 +134,13 @@ __device__ __forceinline__ uint32_t pack_exact_bf16x2(float lo, float hi) {
 __device__ __forceinline__ uint32_t pack_rn_bf16x2(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Elementwise bf16x2 product, rounded to nearest even.
+__device__ __forceinline__ uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
   return r;
 }
 
