@@ -302,7 +302,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         ok = ok && wait_bounded(bar(BAR_LFULL), cc & 1u, ctl, 11);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
-        float ds_acc = 0.0f;
+        // Packed fp32x2 arithmetic per pair of columns: u = phi^-1 + (alpha/r) L, the
+        // unclipped code cu (round half to even by the magic add), the clipped code c,
+        // the STE mask M = [c == cu], dU = G * (s_x s) * M and the ds partial sum G * c
+        // (times s_x at the end).
+        const float gs_i = gscale * s_i;
+        const float dec_off = PACKED ? kDecodeOffsetI4 : kDecodeOffsetI8;
+        const float code_n = __fmaf_rn(qp.lo, qp.inv2f, -qp.magic_c);   // n and p as exact floats
+        const float code_p = __fmaf_rn(qp.hi, qp.inv2f, -qp.magic_c);
+        float2 ds2 = make_float2(0.0f, 0.0f);
 #pragma unroll 1
         for (int p = 0; p < 2; ++p) {
           const int jl = 64 * h + 32 * p;   // column within the chunk
@@ -312,37 +320,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           tmem_ld_wait();
           if (PACKED) {
             const uint4 raw = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 32, 64));
-            decode_i4x8(raw.x, v);
-            decode_i4x8(raw.y, v + 8);
-            decode_i4x8(raw.z, v + 16);
-            decode_i4x8(raw.w, v + 24);
+            decode_i4x8_raw(raw.x, v);
+            decode_i4x8_raw(raw.y, v + 8);
+            decode_i4x8_raw(raw.z, v + 16);
+            decode_i4x8_raw(raw.w, v + 24);
           } else {
             const uint4 r0 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 16, 128));
             const uint4 r1 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 16 + 1, 128));
-            decode_i8x4(r0.x, v);
-            decode_i8x4(r0.y, v + 4);
-            decode_i8x4(r0.z, v + 8);
-            decode_i8x4(r0.w, v + 12);
-            decode_i8x4(r1.x, v + 16);
-            decode_i8x4(r1.y, v + 20);
-            decode_i8x4(r1.z, v + 24);
-            decode_i8x4(r1.w, v + 28);
+            decode_i8x4_raw(r0.x, v);
+            decode_i8x4_raw(r0.y, v + 4);
+            decode_i8x4_raw(r0.z, v + 8);
+            decode_i8x4_raw(r0.w, v + 12);
+            decode_i8x4_raw(r1.x, v + 16);
+            decode_i8x4_raw(r1.y, v + 20);
+            decode_i8x4_raw(r1.z, v + 24);
+            decode_i8x4_raw(r1.w, v + 28);
           }
           uint32_t du[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
-            float d2[2];
-#pragma unroll
-            for (int t = 0; t < 2; ++t) {
-              const int idx = 2 * e + t;
-              const float tm = magic_round(Lv[idx], v[idx], qp);
-              const bool inside = (tm >= qp.lo) && (tm <= qp.hi);
-              const float cval = code_from_magic(tm, qp);
-              const float gv = G[idx] * gscale;
-              ds_acc = __fmaf_rn(gv, cval, ds_acc);
-              d2[t] = inside ? gv * s_i : 0.0f;
-            }
-            du[e] = pack_rn_bf16x2(d2[0], d2[1]);
+            const float2 g2 = make_float2(G[2 * e], G[2 * e + 1]);
+            const float2 v2 = __fadd2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(-dec_off, -dec_off));
+            const float2 u2 = __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
+                                         v2);
+            const float2 t2 = __fadd2_rn(u2, make_float2(qp.magic, qp.magic));
+            const float2 cu = __ffma2_rn(t2, make_float2(qp.inv2f, qp.inv2f), make_float2(-qp.magic_c, -qp.magic_c));
+            const float2 cc = make_float2(fminf(fmaxf(cu.x, code_n), code_p), fminf(fmaxf(cu.y, code_n), code_p));
+            ds2 = __ffma2_rn(g2, cc, ds2);
+            const float2 gs = __fmul2_rn(g2, make_float2(gs_i, gs_i));
+            du[e] = pack_rn_bf16x2(cc.x == cu.x ? gs.x : 0.0f, cc.y == cu.y ? gs.y : 0.0f);
           }
           const uint32_t dub = smem + OFF_DU + 16384u * h;
 #pragma unroll
@@ -357,6 +363,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(bar(BAR_ACCEMPTY));
         }
+        const float ds_acc = (ds2.x + ds2.y) * gscale;
         // ds partial of this 128-column block (two halves h per row)
         args.ds_part[(static_cast<int64_t>(w.sp * 2 + h) * args.m + i_g) * nb + j0 / 128] = ds_acc;
         tc_fence_before();

@@ -88,27 +88,6 @@ __device__ __forceinline__ uint32_t codes_bf16x2(float2 t, const QuantParams& q)
   return w;
 }
 
-// 4 signed bytes of `w` -> 4 exact floats.
-__device__ __forceinline__ void decode_i8x4(uint32_t w, float* v) {
-  const uint32_t x = w ^ 0x80808080u;   // v + 128 in each byte
-  v[0] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7540u)) - 8388736.0f;   // 2^23 + 128
-  v[1] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7541u)) - 8388736.0f;
-  v[2] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7542u)) - 8388736.0f;
-  v[3] = __uint_as_float(__byte_perm(x, 0x4B000000u, 0x7543u)) - 8388736.0f;
-}
-
-// 8 signed nibbles of `w` (low nibble of byte b = element 2b, high = 2b+1) -> 8 exact floats.
-__device__ __forceinline__ void decode_i4x8(uint32_t w, float* v) {
-  const uint32_t x = w ^ 0x88888888u;   // v + 8 in each nibble
-  const uint32_t lo = x & 0x0F0F0F0Fu;
-  const uint32_t hi = (x >> 4) & 0x0F0F0F0Fu;
-#pragma unroll
-  for (int b = 0; b < 4; ++b) {
-    v[2 * b] = __uint_as_float(__byte_perm(lo, 0x4B000000u, 0x7540u + b)) - 8388616.0f;       // 2^23 + 8
-    v[2 * b + 1] = __uint_as_float(__byte_perm(hi, 0x4B000000u, 0x7540u + b)) - 8388616.0f;
-  }
-}
-
 // t = round-half-even(u_f / 2^f) in the magic domain, unclipped.
 __device__ __forceinline__ float magic_round(float L, float v, const QuantParams& q) {
   const float u = __fmaf_rn(L, q.lr_scale, v);
@@ -123,11 +102,6 @@ __device__ __forceinline__ float code_from_magic(float t, const QuantParams& q) 
 
 __device__ __forceinline__ float lrqat_code(float L, float v, const QuantParams& q) {
   return code_from_magic(magic_round(L, v, q), q);
-}
-
-// Two small-integer floats (|c| <= 128) -> packed bf16x2, exact (bf16 keeps the top 16 bits).
-__device__ __forceinline__ uint32_t pack_exact_bf16x2(float lo, float hi) {
-  return __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x7632u);
 }
 
 // Two floats -> packed bf16x2 with round-to-nearest-even.
@@ -146,12 +120,6 @@ __device__ __forceinline__ uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
 
 __device__ __forceinline__ float bf16_to_float(uint16_t b) {
   return __uint_as_float(static_cast<uint32_t>(b) << 16);
-}
-
-__device__ __forceinline__ uint16_t float_to_bf16_rn(float f) {
-  uint32_t r;
-  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(0.0f), "f"(f));
-  return static_cast<uint16_t>(r & 0xFFFFu);
 }
 
 }  // namespace lrqat
