@@ -36,6 +36,15 @@ Readings where the paper is silent (all repeated in the design notes):
   R9 activation quantizer (weight-activation runs): per-tensor symmetric int8,
      X_Z = clip(round(X / s_x), -128, 127) with X / s_x one fp32 division,
      X_hat = s_x X_Z, STE with clip mask M_x = 1[-128 <= round(X/s_x) <= 127].
+  R10 asymmetric weights (the INT2 runs of Sec. 4; Eq. 1 with the zero offset z
+     outside the rounding, as the end of Sec. 3 states): W_hat = s (W_Z - z) with
+     W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B + z), n, p) and z frozen at its
+     range-setting value z0 (Sec. 4).  z is an integer, so round(x) + z = round(x + z)
+     and the oracle stores Phi0 = phi(W0 / s0 + z0): the frozen base already carries
+     the offset and Eq. 8's clip range stays [n, p].  Range setting is asymmetric
+     min-max: s0 = (max - min) / (2^b - 1) in fp32 and z0 = clip(round(n - min / s0),
+     n, p) with min / s0 one fp32 division and the rest exact.  The STE mask is
+     unchanged and ds = sum G (W_Z - z).
 """
 from __future__ import annotations
 
@@ -96,6 +105,34 @@ def minmax_scale(W0: np.ndarray, layer: Layer) -> np.ndarray:
     return np.divide(safe, np.float32(p), dtype=np.float32)
 
 
+def minmax_range_asym(W0: np.ndarray, layer: Layer):
+    """Asymmetric min-max range setting (reading R10): returns (s0, z0), both float32
+    and shaped like the scales; z0 holds integers in [n, p]."""
+    n, p = grid(layer.bits)
+    W0 = np.asarray(W0, dtype=np.float32)
+    if layer.group_size == 0:
+        seg = W0.reshape(layer.m, 1, layer.k)
+    else:
+        seg = W0.reshape(layer.m, layer.k // layer.group_size, layer.group_size)
+    lo = seg.min(axis=2).astype(np.float32)
+    hi = seg.max(axis=2).astype(np.float32)
+    span = np.subtract(hi, lo, dtype=np.float32)
+    span = np.where(span > 0, span, np.float32(2 ** layer.bits - 1)).astype(np.float32)
+    s0 = np.divide(span, np.float32(2 ** layer.bits - 1), dtype=np.float32)
+    q = np.divide(lo, s0, dtype=np.float32).astype(np.float64)
+    z0 = np.clip(np.rint(n - q), n, p).astype(np.float32)
+    if layer.group_size == 0:
+        return s0.reshape(layer.m), z0.reshape(layer.m)
+    return s0, z0
+
+
+def expand_zero(z: Optional[np.ndarray], layer: Layer) -> np.ndarray:
+    """The zero offsets broadcast to [m, k] (0 for a symmetric layer)."""
+    if z is None:
+        return np.zeros((layer.m, layer.k))
+    return expand_scale(z, layer)
+
+
 # ----------------------------------------------------------------------------
 # Downcasting operator phi and its inverse (Sec. 3, Eq. 6, Eq. 7)
 # ----------------------------------------------------------------------------
@@ -124,21 +161,24 @@ def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
     return out.astype(np.int8)
 
 
-def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer) -> np.ndarray:
-    """Phi0 = phi(W0 / s0) (Eq. 6).
+def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer, z0: Optional[np.ndarray] = None) -> np.ndarray:
+    """Phi0 = phi(W0 / s0) (Eq. 6); with zero offsets phi(W0 / s0 + z0) (reading R10).
 
     Q-fixed (Eq. 7): INT8(round(2^{8-b} * clip(x, n, p))), stored int8 [m, k].
     INT-b (Sec. 3): clip(round(x), n, p), double-packed into uint8 [m, k/2].
-    x = W0 / s0 is a single fp32 division per element (reading R8).
+    W0 / s0 is a single fp32 division per element (reading R8); adding the integer
+    offset is exact.
     """
     n, p = grid(layer.bits)
     W0 = np.asarray(W0, dtype=np.float32)
     s_full = expand_scale(s0, layer).astype(np.float32)
-    x = np.divide(W0, s_full, dtype=np.float32)
+    x = np.divide(W0, s_full, dtype=np.float32).astype(np.float64)
+    if z0 is not None:
+        x = x + expand_scale(z0, layer)
     if layer.phi_format == PHI_QFIXED:
-        y = np.clip(x.astype(np.float64), n, p) * 2.0 ** (8 - layer.bits)
+        y = np.clip(x, n, p) * 2.0 ** (8 - layer.bits)
         return np.rint(y).astype(np.int8)
-    codes = np.clip(np.rint(x.astype(np.float64)), n, p).astype(np.int8)
+    codes = np.clip(np.rint(x), n, p).astype(np.int8)
     return pack_nibbles(codes)
 
 
@@ -177,15 +217,18 @@ def near_tie(u: np.ndarray, tol: float = NEAR_TIE_TOL) -> np.ndarray:
     return np.abs(u32 - (np.floor(u32) + 0.5)) <= tol
 
 
-def fake_quant_weight(Phi0, s, A, B, layer: Layer) -> Dict[str, np.ndarray]:
-    """W_hat = s * clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p)  (Eq. 8)."""
+def fake_quant_weight(Phi0, s, A, B, layer: Layer, z: Optional[np.ndarray] = None) -> Dict[str, np.ndarray]:
+    """W_hat = s * clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p)  (Eq. 8);
+    with zero offsets W_hat = s * (clip(...) - z), the offset carried by Phi0 (R10)."""
     u = preround(Phi0, A, B, layer)
     q, c, M = codes_from_u(u, layer)
-    return {"u": u, "q": q, "c": c, "M": M, "W_hat": expand_scale(s, layer) * c}
+    cz = c - expand_zero(z, layer)
+    return {"u": u, "q": q, "c": c, "cz": cz, "M": M, "W_hat": expand_scale(s, layer) * cz}
 
 
 def merge(Phi0, A, B, layer: Layer) -> np.ndarray:
-    """Integer weight W_Z = clip(round(...), n, p) that training leaves behind (Sec. 3, Eq. 8)."""
+    """Integer weight W_Z = clip(round(...), n, p) that training leaves behind (Sec. 3, Eq. 8);
+    with zero offsets the dequantized weight is s (W_Z - z) (Eq. 1)."""
     return codes_from_u(preround(Phi0, A, B, layer), layer)[1].astype(np.int8)
 
 
@@ -213,13 +256,15 @@ def _inputs(X, layer: Layer, s_x: Optional[float]):
     return X, np.ones_like(X)
 
 
-def linear_fwd(X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) -> np.ndarray:
+def linear_fwd(X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None,
+               z: Optional[np.ndarray] = None) -> np.ndarray:
     """Y = X_hat W_hat^T with W_hat from Eq. 8; returns float64 [T, m]."""
     Xh, _ = _inputs(X, layer, s_x)
-    return Xh @ fake_quant_weight(Phi0, s, A, B, layer)["W_hat"].T
+    return Xh @ fake_quant_weight(Phi0, s, A, B, layer, z)["W_hat"].T
 
 
-def linear_bwd(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) -> Dict[str, np.ndarray]:
+def linear_bwd(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None,
+               z: Optional[np.ndarray] = None) -> Dict[str, np.ndarray]:
     """Gradients of the LR-QAT layer for an upstream gradient dY [T, m].
 
     W_hat is recomputed from Phi0, A, B, s (the checkpointing of Sec. 3).  With
@@ -227,18 +272,18 @@ def linear_bwd(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) 
       dX = (dY W_hat) * M_x
       dU = G * s * M                    (gradient w.r.t. u, mask from R3)
       dA = (alpha/r) dU B^T,  dB = (alpha/r) A^T dU
-      ds = sum over the row (or group) of G * c   (reading R4)
+      ds = sum over the row (or group) of G * c   (reading R4; G * (c - z), R10)
     """
     dY = np.asarray(dY, dtype=np.float64)
     Xh, Mx = _inputs(X, layer, s_x)
-    fq = fake_quant_weight(Phi0, s, A, B, layer)
+    fq = fake_quant_weight(Phi0, s, A, B, layer, z)
     dX = (dY @ fq["W_hat"]) * Mx
     G = dY.T @ Xh
     dU = G * expand_scale(s, layer) * fq["M"]
     scale = layer.alpha / layer.r
     dA = scale * (dU @ np.asarray(B, dtype=np.float64).T)
     dB = scale * (np.asarray(A, dtype=np.float64).T @ dU)
-    Gc = G * fq["c"]
+    Gc = G * fq["cz"]
     if layer.group_size == 0:
         ds = Gc.sum(axis=1)
     else:
@@ -246,7 +291,8 @@ def linear_bwd(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) 
     return {"dX": dX, "dA": dA, "dB": dB, "ds": ds, "G": G, "fq": fq}
 
 
-def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None) -> Dict[str, np.ndarray]:
+def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None,
+                     z: Optional[np.ndarray] = None) -> Dict[str, np.ndarray]:
     """The same gradients as ``linear_bwd``, hand-expanded into scalar loops.
 
     For tiny shapes only.  Each weight element is rebuilt from Eq. 8 with its
@@ -258,6 +304,7 @@ def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = 
     m, k, r = layer.m, layer.k, layer.r
     P = upcast(Phi0, layer)
     s_full = expand_scale(s, layer)
+    z_full = expand_zero(z, layer)
     Xh, Mx = _inputs(X, layer, s_x)
     A = np.asarray(A, dtype=np.float64)
     B = np.asarray(B, dtype=np.float64)
@@ -276,7 +323,7 @@ def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = 
             q = float(np.rint(u))
             c = min(max(q, n), p)
             inside = 1.0 if n <= q <= p else 0.0
-            w = s_full[i, j] * c
+            w = s_full[i, j] * (c - z_full[i, j])
             g = 0.0                              # dL/dW_hat[i, j] = sum_tok dY[tok, i] X_hat[tok, j]
             for tok in range(T):
                 g += dY[tok, i] * Xh[tok, j]
@@ -286,9 +333,9 @@ def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = 
                 dA[i, t] += scale * du * B[t, j]
                 dB[t, j] += scale * du * A[i, t]
             if layer.group_size == 0:
-                ds[i] += g * c
+                ds[i] += g * (c - z_full[i, j])
             else:
-                ds[i, j // layer.group_size] += g * c
+                ds[i, j // layer.group_size] += g * (c - z_full[i, j])
     return {"dX": dX, "dA": dA, "dB": dB, "ds": ds}
 
 

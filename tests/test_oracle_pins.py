@@ -319,3 +319,114 @@ def test_workload_generator_is_deterministic_and_bf16_exact():
     np.testing.assert_array_equal(WL.bf16_bits(a.X), a.X_bits)
     assert WL.bf16_bits(np.array([1.0 + 2.0 ** -8], dtype=np.float32))[0] == 0x3F80   # tie -> even
     assert WL.bf16_bits(np.array([1.0 + 3 * 2.0 ** -8], dtype=np.float32))[0] == 0x3F82
+
+
+# ---------------------------------------------------------------------------
+# Asymmetric weights with a frozen zero offset (INT2 runs of Sec. 4; Eq. 1 with
+# the offset outside the rounding, end of Sec. 3; reading R10)
+# ---------------------------------------------------------------------------
+def _asym_data(bits, phi, group=0, m=24, k=256, r=4, T=1, seed=7, std=0.01, zero_B=False):
+    """A layer whose rows are shifted by different offsets, so that the zero
+    offsets z0 of min-max range setting spread over the grid."""
+    layer = O.Layer(m, k, r, float(r), bits, group, phi)
+    spec = WL.LayerSpec("t", m, k, r, float(r), bits, group, phi, a_std=std, b_std=std)
+    d = WL.make_layer(spec, T, seed=seed, zero_B=zero_B)
+    rng = np.random.default_rng(seed + 100)
+    shift = rng.uniform(-0.05, 0.05, size=(m, 1)).astype(np.float32)
+    W0 = (d.W0 + shift).astype(np.float32)
+    return layer, d, W0
+
+
+@pytest.mark.parametrize("bits,phi,group", [(2, O.PHI_QFIXED, 0), (2, O.PHI_INT_PACKED, 128),
+                                            (3, O.PHI_INT_PACKED, 0), (4, O.PHI_QFIXED, 128)])
+def test_asym_minmax_range_covers_min_and_max(bits, phi, group):
+    """s0 = (max - min) / (2^b - 1) and z0 = round(n - min / s0): the dequantized grid
+    s0 (j - z0), j in [n, p], reaches min and max to within half a step."""
+    layer, _, W0 = _asym_data(bits, phi, group)
+    n, p = O.grid(bits)
+    s0, z0 = O.minmax_range_asym(W0, layer)
+    seg = W0.reshape(layer.m, -1, group if group else layer.k)
+    lo, hi = seg.min(axis=2).reshape(s0.shape), seg.max(axis=2).reshape(s0.shape)
+    np.testing.assert_array_equal(s0, np.float32(hi - lo) / np.float32(2 ** bits - 1))
+    assert np.all(z0 == np.rint(z0)) and z0.min() >= n and z0.max() <= p
+    assert len(np.unique(z0)) > 1                                  # the offsets really vary
+    inner = (z0 > n) & (z0 < p)                                    # z0 not clipped
+    step = s0.astype(np.float64)
+    assert np.all(np.abs(step * (n - z0) - lo)[inner] <= 0.5 * step[inner] * (1 + 1e-6))
+    assert np.all(np.abs(step * (p - z0) - hi)[inner] <= 0.5 * step[inner] * (1 + 1e-6))
+
+
+@pytest.mark.parametrize("bits,group", [(2, 0), (2, 128), (3, 0), (4, 128)])
+def test_asym_int_phi_with_zero_adapter_is_asymmetric_rtn(bits, group):
+    """phi = INT-b and A B = 0: W_Z is Eq. 1's clip(round(W0 / s0) + z0, n, p), taken
+    here in that order (round first, then add z0), and s0 (W_Z - z0) is Eq. 1's
+    dequantized W0."""
+    layer, d, W0 = _asym_data(bits, O.PHI_INT_PACKED, group, zero_B=True)
+    n, p = O.grid(bits)
+    s0, z0 = O.minmax_range_asym(W0, layer)
+    x32 = np.divide(W0, O.expand_scale(s0, layer).astype(np.float32), dtype=np.float32)
+    zf = O.expand_scale(z0, layer)
+    expect = np.clip(_rtn_python(x32, -10 ** 6, 10 ** 6) + zf, n, p)
+    phi0 = O.downcast(W0, s0, layer, z0)
+    wz = O.merge(phi0, d.A, d.B, layer).astype(np.int64)
+    np.testing.assert_array_equal(wz, expect)
+    fq = O.fake_quant_weight(phi0, s0, d.A, d.B, layer, z0)
+    np.testing.assert_array_equal(fq["W_hat"], O.expand_scale(s0, layer) * (expect - zf))
+
+
+def test_asym_zero_offsets_of_zero_reduce_to_symmetric():
+    """z = 0 everywhere gives exactly the symmetric path (Eq. 8)."""
+    layer, d, W0 = _asym_data(4, O.PHI_QFIXED, 0, T=3, std=0.3)
+    s0 = O.minmax_scale(W0, layer)
+    z0 = np.zeros_like(s0)
+    phi_s, phi_a = O.downcast(W0, s0, layer), O.downcast(W0, s0, layer, z0)
+    np.testing.assert_array_equal(phi_s, phi_a)
+    gs = O.linear_bwd(d.dY, d.X, phi_s, s0, d.A, d.B, layer)
+    ga = O.linear_bwd(d.dY, d.X, phi_a, s0, d.A, d.B, layer, None, z0)
+    for name in ("dX", "dA", "dB", "ds"):
+        np.testing.assert_array_equal(gs[name], ga[name], err_msg=name)
+
+
+ASYM_LOOP_CASES = [
+    dict(bits=2, phi=O.PHI_QFIXED, group=0, std=0.5),
+    dict(bits=2, phi=O.PHI_INT_PACKED, group=0, std=1.0),
+    dict(bits=3, phi=O.PHI_QFIXED, group=128, std=1.0),
+]
+
+
+@pytest.mark.parametrize("case", ASYM_LOOP_CASES)
+def test_asym_ste_gradients_match_scalar_loops_and_finite_differences(case):
+    """With zero offsets: the matrix-form gradients equal the hand-expanded loops, and
+    dX and ds equal central differences of <dY, Y> (Y is linear in X and in s; the
+    codes do not depend on s), while s (W_Z - z) reproduces W_hat."""
+    layer, d, W0 = _asym_data(case["bits"], case["phi"], case["group"], m=4, k=256, r=2, T=3,
+                              std=case["std"])
+    s0, z0 = O.minmax_range_asym(W0, layer)
+    phi0 = O.downcast(W0, s0, layer, z0)
+    s = s0 * np.float32(0.9)
+    ref = O.linear_bwd_loops(d.dY, d.X, phi0, s, d.A, d.B, layer, None, z0)
+    got = O.linear_bwd(d.dY, d.X, phi0, s, d.A, d.B, layer, None, z0)
+    for name in ("dX", "dA", "dB", "ds"):
+        np.testing.assert_allclose(got[name], ref[name], rtol=1e-12, atol=1e-12, err_msg=name)
+    assert got["fq"]["M"].min() == 0.0                              # the clip mask is exercised
+    wz = O.merge(phi0, d.A, d.B, layer).astype(np.float64)
+    np.testing.assert_array_equal(O.expand_scale(s, layer) * (wz - O.expand_scale(z0, layer)),
+                                  got["fq"]["W_hat"])
+
+    def loss(X, s_):
+        return float(np.sum(d.dY * O.linear_fwd(X, phi0, s_, d.A, d.B, layer, None, z0)))
+    eps = 0.5
+    X64 = d.X.astype(np.float64)
+    for (t, j) in [(0, 0), (2, layer.k - 1)]:
+        Xp, Xm = X64.copy(), X64.copy()
+        Xp[t, j] += eps
+        Xm[t, j] -= eps
+        fd = (loss(Xp, s) - loss(Xm, s)) / (2 * eps)
+        assert abs(fd - got["dX"][t, j]) <= 1e-9 * max(1.0, abs(fd))
+    s64 = s.astype(np.float64)
+    for idx in [(0,) if s.ndim == 1 else (0, 0), (layer.m - 1,) if s.ndim == 1 else (layer.m - 1, 1)]:
+        sp, sm = s64.copy(), s64.copy()
+        sp[idx] += eps
+        sm[idx] -= eps
+        fd = (loss(X64, sp) - loss(X64, sm)) / (2 * eps)
+        assert abs(fd - got["ds"][idx]) <= 1e-9 * max(1.0, abs(fd))
