@@ -179,10 +179,11 @@ class GpuWorkload:
         dev = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16) if a.dtype == np.uint16 else a)).cuda()
         for li, spec in enumerate(wl.layers):
             d = WL.make_layer(spec, self.T, seed=seed, layer_index=li)
-            L = LQ.Layer.from_spec(spec)
             W0 = dev(d.W0)
             ng = spec.k // spec.group_size if spec.group_size else 1
             s = torch.empty((spec.m, ng) if spec.group_size else (spec.m,), dtype=torch.float32, device="cuda")
+            z = torch.empty_like(s) if spec.asym else None   # zero offsets (asymmetric weights)
+            L = LQ.Layer.from_spec(spec, z.data_ptr() if spec.asym else 0)
             LQ.range_minmax(L, W0, s)
             if spec.phi_format == WL.PHI_QFIXED:
                 phi0 = torch.empty((spec.m, spec.k), dtype=torch.int8, device="cuda")
@@ -196,7 +197,7 @@ class GpuWorkload:
             if spec.act_bits == 8:
                 sx = np.float32(np.float32(np.abs(d.X).max()) / np.float32(127.0))
                 s_x = torch.tensor([sx], dtype=torch.float32, device="cuda")
-            lay = dict(spec=spec, L=L, phi0=phi0, s=s, A=dev(d.A_bits), B=dev(d.B_bits), X=X, dY=dY, s_x=s_x,
+            lay = dict(spec=spec, L=L, z=z, phi0=phi0, s=s, A=dev(d.A_bits), B=dev(d.B_bits), X=X, dY=dY, s_x=s_x,
                        X_host=d.X_bits, dY_host=d.dY_bits,
                        Y=torch.empty((self.T, spec.m), dtype=torch.int16, device="cuda"),
                        dX=torch.empty((self.T, spec.k), dtype=torch.int16, device="cuda"),

@@ -74,19 +74,31 @@ typedef struct {
   int32_t act_bits;   /* 0: activations unquantized; 8: per-tensor symmetric int8
                          X_hat = s_x clip(round(X/s_x), -128, 127) (Sec. 4,
                          weight-activation quantization; Eq. 1 with z = 0)          */
+  float* zero;        /* NULL: symmetric weight grid (Eq. 8 as written).  Otherwise
+                         asymmetric weights with a frozen zero offset (Eq. 1 with z
+                         outside the rounding, end of Sec. 3; the INT2 runs of Sec. 4):
+                         a device array shaped like s, 16-byte aligned, holding the
+                         integer offsets z as floats.  W_hat = s (W_Z - z) with
+                         W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p), where
+                         the stored base Phi0 = phi(W0 / s0 + z0) already carries the
+                         offset (z integer: round(x) + z = round(x + z)).
+                         lrqat_range_minmax writes z0; every other call reads z.     */
 } lrqat_layer;
 
 /* Human-readable reason of the last non-OK status returned on this thread. */
 const char* lrqat_last_error(void);
 
-/* Symmetric min-max range setting (App. B, "PTQ initialization"):
- *   s0[i] (or s0[i, g]) = max |W0[i, :]| (over the row or group) / p, fp32;
- *   an all-zero row/group gets s0 = 1.
+/* Min-max range setting (App. B, "PTQ initialization").  Symmetric (layer->zero
+ * == NULL): s0[i] (or s0[i, g]) = max |W0[i, :]| (over the row or group) / p, fp32;
+ * an all-zero row/group gets s0 = 1.  Asymmetric (layer->zero != NULL, written as
+ * an output): s0 = (max - min) / (2^b - 1) in fp32 (1 if max == min) and
+ * z0 = clip(round(n - min / s0), n, p), min / s0 one fp32 division.
  * W0: fp32 [m, k].  s0: fp32 [m] or [m, k/g] (output). */
 int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrqat_stream_t stream);
 
 /* Downcasting operator of Eq. 6 / Eq. 7: Phi0 = phi(W0 / s0), with W0 / s0 one
- * fp32 IEEE division per element.
+ * fp32 IEEE division per element; with zero offsets phi(W0 / s0 + z0), the
+ * integer offset added exactly.
  * W0: fp32 [m, k]; s0: fp32 [m] or [m, k/g];
  * Phi0 (output): int8 [m, k] (QFIXED) or uint8 [m, k/2] (INT_PACKED). */
 int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0,

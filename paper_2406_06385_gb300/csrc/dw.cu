@@ -93,7 +93,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   return x;
 }
 
-template <bool PACKED>
+template <bool PACKED, bool ZP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     dw_kernel(const __grid_constant__ CUtensorMap tm_dy, const __grid_constant__ CUtensorMap tm_x,
               const __grid_constant__ CUtensorMap tm_at, const __grid_constant__ CUtensorMap tm_phi,
@@ -298,14 +298,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int j0 = w.jt * BN + 128 * c;
         const float s_i = args.s_ld ? args.s[static_cast<int64_t>(i_g) * args.s_ld + j0 / args.group_size]
                                     : args.s[i_g];
+        // zero offset of the row (group) when the weights are asymmetric (ZP: args.zero set)
+        const float z_i = !ZP         ? 0.0f
+                          : args.s_ld ? args.zero[static_cast<int64_t>(i_g) * args.s_ld + j0 / args.group_size]
+                                      : args.zero[i_g];
         ok = wait_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 10);
         ok = ok && wait_bounded(bar(BAR_LFULL), cc & 1u, ctl, 11);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
         // Packed fp32x2 arithmetic per pair of columns: u = phi^-1 + (alpha/r) L, the
         // unclipped code cu (round half to even by the magic add), the clipped code c,
-        // the STE mask M = [c == cu], dU = G * (s_x s) * M and the ds partial sum G * c
-        // (times s_x at the end).
+        // the STE mask M = [c == cu], dU = G * (s_x s) * M and the ds partial sum G * (c - z)
+        // (times s_x at the end; z = 0 for symmetric weights).
         const float gs_i = gscale * s_i;
         const float dec_off = PACKED ? kDecodeOffsetI4 : kDecodeOffsetI8;
         const float code_n = __fmaf_rn(qp.lo, qp.inv2f, -qp.magic_c);   // n and p as exact floats
@@ -346,7 +350,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const float2 t2 = __fadd2_rn(u2, make_float2(qp.magic, qp.magic));
             const float2 cu = __ffma2_rn(t2, make_float2(qp.inv2f, qp.inv2f), make_float2(-qp.magic_c, -qp.magic_c));
             const float2 cc = make_float2(fminf(fmaxf(cu.x, code_n), code_p), fminf(fmaxf(cu.y, code_n), code_p));
-            ds2 = __ffma2_rn(g2, cc, ds2);
+            ds2 = __ffma2_rn(g2, ZP ? __fadd2_rn(cc, make_float2(-z_i, -z_i)) : cc, ds2);
             const float2 gs = __fmul2_rn(g2, make_float2(gs_i, gs_i));
             du[e] = pack_rn_bf16x2(cc.x == cu.x ? gs.x : 0.0f, cc.y == cu.y ? gs.y : 0.0f);
           }
@@ -416,17 +420,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <bool PACKED>
+template <bool PACKED, bool ZP>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
   static bool configured = false;
   if (!configured) {
     cudaError_t err =
-        cudaFuncSetAttribute(dw_kernel<PACKED>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+        cudaFuncSetAttribute(dw_kernel<PACKED, ZP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (err != cudaSuccess) return err;
     configured = true;
   }
-  dw_kernel<PACKED><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
+  dw_kernel<PACKED, ZP><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
   return cudaGetLastError();
 }
 
@@ -439,8 +443,11 @@ cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& t
                       cudaStream_t stream) {
   if (grid < 1 || args.r16 < 16 || args.r16 > 64 || (args.r16 & 15) || args.nchunks < 1 || args.nchunks > 2)
     return cudaErrorInvalidValue;
-  return packed ? launch_one<true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
-                : launch_one<false>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+  if (args.zero != nullptr)
+    return packed ? launch_one<true, true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
+                  : launch_one<false, true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+  return packed ? launch_one<true, false>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
+                : launch_one<false, false>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
 }
 
 }  // namespace lrqat

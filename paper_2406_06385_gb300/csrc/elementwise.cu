@@ -39,23 +39,75 @@ __global__ void range_minmax_kernel(const float* __restrict__ W0, int64_t k, int
   }
 }
 
+// Asymmetric min-max range setting (zero offsets, Eq. 1): per (row, group)
+// s0 = (max - min) / (2^b - 1) in fp32 (1 if max == min) and
+// z0 = clip(round(n - min / s0), n, p), min / s0 one fp32 division, the rest exact.
+__global__ void range_minmax_asym_kernel(const float* __restrict__ W0, int64_t k, int seg, int ngroups, int bits,
+                                         float* __restrict__ s0, float* __restrict__ z0) {
+  const int64_t row = blockIdx.x / ngroups;
+  const int g = blockIdx.x % ngroups;
+  const float* src = W0 + row * k + static_cast<int64_t>(g) * seg;
+  float lo = INFINITY, hi = -INFINITY;
+  for (int j = threadIdx.x; j < seg; j += blockDim.x) {
+    const float v = src[j];
+    lo = fminf(lo, v);
+    hi = fmaxf(hi, v);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  __shared__ float warp_lo[kThreads / 32], warp_hi[kThreads / 32];
+  if ((threadIdx.x & 31) == 0) {
+    warp_lo[threadIdx.x >> 5] = lo;
+    warp_hi[threadIdx.x >> 5] = hi;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) {
+      lo = fminf(lo, warp_lo[w]);
+      hi = fmaxf(hi, warp_hi[w]);
+    }
+    const float span = __fsub_rn(hi, lo);
+    const float s = span > 0.0f ? __fdiv_rn(span, static_cast<float>((1 << bits) - 1)) : 1.0f;
+    const double n = -static_cast<double>(1 << (bits - 1)), p = static_cast<double>((1 << (bits - 1)) - 1);
+    const double z = fmin(fmax(rint(n - static_cast<double>(__fdiv_rn(lo, s))), n), p);
+    s0[blockIdx.x] = s;
+    z0[blockIdx.x] = static_cast<float>(z);
+  }
+}
+
 // ----------------------------------------------------------------- downcast --
 // Q-fixed (Eq. 7): round(2^f clip(W0/s0, n, p)) -> int8; 4 elements per thread.
-__global__ void downcast_qfixed_kernel(const float4* __restrict__ W0, const float* __restrict__ s0, int64_t k,
-                                       int group_size, int ngroups, float n, float p, float two_f,
-                                       char4* __restrict__ out, int64_t n4) {
+// With zero offsets z0 (nullable): round(2^f clip(W0/s0 + z0, n, p)), the integer
+// offset added exactly in double precision.
+__global__ void downcast_qfixed_kernel(const float4* __restrict__ W0, const float* __restrict__ s0,
+                                       const float* __restrict__ z0, int64_t k, int group_size, int ngroups,
+                                       float n, float p, float two_f, char4* __restrict__ out, int64_t n4) {
   for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n4;
        e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int64_t row = (e * 4) / k;
     const int64_t col = (e * 4) % k;
-    const float s = group_size ? s0[row * ngroups + col / group_size] : s0[row];
+    const int64_t sidx = group_size ? row * ngroups + col / group_size : row;
+    const float s = s0[sidx];
     const float4 w = W0[e];
     const float x[4] = {w.x, w.y, w.z, w.w};
     int q[4];
+    if (z0 == nullptr) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float y = fminf(fmaxf(__fdiv_rn(x[i], s), n), p) * two_f;   // exact scaling by 2^f
-      q[i] = __float2int_rn(y);
+      for (int i = 0; i < 4; ++i) {
+        const float y = fminf(fmaxf(__fdiv_rn(x[i], s), n), p) * two_f;   // exact scaling by 2^f
+        q[i] = __float2int_rn(y);
+      }
+    } else {
+      const double z = z0[sidx];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const double y = fmin(fmax(static_cast<double>(__fdiv_rn(x[i], s)) + z, static_cast<double>(n)),
+                              static_cast<double>(p)) * two_f;
+        q[i] = __double2int_rn(y);
+      }
     }
     out[e] = make_char4(static_cast<signed char>(q[0]), static_cast<signed char>(q[1]),
                         static_cast<signed char>(q[2]), static_cast<signed char>(q[3]));
@@ -63,21 +115,25 @@ __global__ void downcast_qfixed_kernel(const float4* __restrict__ W0, const floa
 }
 
 // INT-b, double packed: clip(round(W0/s0), n, p), two nibbles per byte; 8 elements per thread.
-__global__ void downcast_packed_kernel(const float4* __restrict__ W0, const float* __restrict__ s0, int64_t k,
-                                       int group_size, int ngroups, int n, int p, uint32_t* __restrict__ out,
-                                       int64_t n8) {
+// With zero offsets z0 (nullable): clip(round(W0/s0 + z0), n, p).
+__global__ void downcast_packed_kernel(const float4* __restrict__ W0, const float* __restrict__ s0,
+                                       const float* __restrict__ z0, int64_t k, int group_size, int ngroups, int n,
+                                       int p, uint32_t* __restrict__ out, int64_t n8) {
   for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n8;
        e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int64_t row = (e * 8) / k;
     const int64_t col = (e * 8) % k;
-    const float s = group_size ? s0[row * ngroups + col / group_size] : s0[row];
+    const int64_t sidx = group_size ? row * ngroups + col / group_size : row;
+    const float s = s0[sidx];
+    const double z = z0 != nullptr ? static_cast<double>(z0[sidx]) : 0.0;
     const float4 w0 = W0[2 * e];
     const float4 w1 = W0[2 * e + 1];
     const float x[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
     uint32_t word = 0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      int c = __float2int_rn(__fdiv_rn(x[i], s));
+      int c = z0 == nullptr ? __float2int_rn(__fdiv_rn(x[i], s))
+                            : __double2int_rn(static_cast<double>(__fdiv_rn(x[i], s)) + z);
       c = c < n ? n : (c > p ? p : c);
       word |= (static_cast<uint32_t>(c) & 0xFu) << (4 * i);
     }
@@ -445,28 +501,34 @@ __global__ void __launch_bounds__(kThreads) reduce_grads_kernel(RedJob ja, RedJo
 
 }  // namespace
 
-cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int p, float* s0,
-                                cudaStream_t stream) {
+cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int bits, float* s0,
+                                float* z0, cudaStream_t stream) {
   const int ngroups = group_size ? static_cast<int>(k / group_size) : 1;
   const int seg = group_size ? group_size : static_cast<int>(k);
-  range_minmax_kernel<<<static_cast<unsigned>(m * ngroups), kThreads, 0, stream>>>(W0, k, seg, ngroups,
-                                                                                   static_cast<float>(p), s0);
+  const unsigned grid = static_cast<unsigned>(m * ngroups);
+  if (z0 == nullptr) {
+    range_minmax_kernel<<<grid, kThreads, 0, stream>>>(W0, k, seg, ngroups,
+                                                       static_cast<float>((1 << (bits - 1)) - 1), s0);
+  } else {
+    range_minmax_asym_kernel<<<grid, kThreads, 0, stream>>>(W0, k, seg, ngroups, bits, s0, z0);
+  }
   return cudaGetLastError();
 }
 
-cudaError_t launch_downcast(const float* W0, const float* s0, int64_t m, int64_t k, int group_size, int bits,
-                            int packed, void* phi0, cudaStream_t stream) {
+cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, int64_t m, int64_t k, int group_size,
+                            int bits, int packed, void* phi0, cudaStream_t stream) {
   const int ngroups = group_size ? static_cast<int>(k / group_size) : 1;
   const int n = -(1 << (bits - 1)), p = (1 << (bits - 1)) - 1;
   if (!packed) {
     const int64_t n4 = m * k / 4;
     downcast_qfixed_kernel<<<blocks_for(n4, kThreads), kThreads, 0, stream>>>(
-        reinterpret_cast<const float4*>(W0), s0, k, group_size, ngroups, static_cast<float>(n),
+        reinterpret_cast<const float4*>(W0), s0, z0, k, group_size, ngroups, static_cast<float>(n),
         static_cast<float>(p), static_cast<float>(1 << (8 - bits)), static_cast<char4*>(phi0), n4);
   } else {
     const int64_t n8 = m * k / 8;
     downcast_packed_kernel<<<blocks_for(n8, kThreads), kThreads, 0, stream>>>(
-        reinterpret_cast<const float4*>(W0), s0, k, group_size, ngroups, n, p, static_cast<uint32_t*>(phi0), n8);
+        reinterpret_cast<const float4*>(W0), s0, z0, k, group_size, ngroups, n, p, static_cast<uint32_t*>(phi0),
+        n8);
   }
   return cudaGetLastError();
 }

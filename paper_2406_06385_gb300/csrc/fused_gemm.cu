@@ -105,7 +105,7 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64
 // Stages are numbered globally over the CTA's tiles (gg); the contraction has an
 // even number of slices, so stage gg uses token slot gg % 2 for the (gg / 2)-th
 // time and factor slot gg % NF for the (gg / NF)-th time.
-template <int MODE, bool PACKED>
+template <int MODE, bool PACKED, bool ZP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
@@ -298,6 +298,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const QuantParams qp = args.q;
     const float dec_off = PACKED ? kDecodeOffsetI4 : kDecodeOffsetI8;
+    constexpr bool zp = ZP;   // zero offsets (asymmetric weights): args.zero != nullptr
     uint32_t g = 0;
     uint32_t it = 0;
     bool ok = true;
@@ -307,8 +308,39 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int row_g = rb * BM + row;
       for (int kk = 0; kk < nk; ++kk) {
         const uint32_t gg = g + kk;
-        // Scales that multiply the operand (group-wise forward, dX).
+        // Scales that multiply the operand (group-wise forward, dX), and the zero offsets
+        // subtracted from the codes (asymmetric weights) as bf16 pairs.
         float sc[16];
+        uint32_t zw[8];
+        if (zp) {
+          if (MODE == FUSED_DX) {
+            const int i0 = kk * BK + 16 * c;
+            float zv[16];
+            if (args.s_ld == 0) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float4 v = __ldg(reinterpret_cast<const float4*>(args.zero + i0) + e);
+                zv[4 * e] = v.x;
+                zv[4 * e + 1] = v.y;
+                zv[4 * e + 2] = v.z;
+                zv[4 * e + 3] = v.w;
+              }
+            } else {
+              const int gcol = row_g / args.group_size;
+#pragma unroll
+              for (int e = 0; e < 16; ++e) zv[e] = __ldg(args.zero + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) zw[e] = pack_rn_bf16x2(zv[2 * e], zv[2 * e + 1]);
+          } else {
+            const float zr = MODE == FUSED_FWD_GROUP
+                                 ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size]
+                                 : args.zero[row_g];
+            const uint32_t z2 = pack_rn_bf16x2(zr, zr);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) zw[e] = z2;
+          }
+        }
         if (MODE == FUSED_FWD_GROUP) {
           const float v = args.s[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size];
 #pragma unroll
@@ -370,12 +402,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const float2 u = __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
                                       make_float2(v[2 * e], v[2 * e + 1]));
           const float2 t2 = __fadd2_rn(u, make_float2(qp.magic, qp.magic));
+          uint32_t cw = codes_bf16x2(t2, qp);
+          if (zp) cw = sub_bf16x2(cw, zw[e]);   // c - z, exact small integers
           if (MODE == FUSED_FWD_PC) {
-            w[e] = codes_bf16x2(t2, qp);
+            w[e] = cw;
           } else {
             // bf16(bf16(s) * c): the exact bf16 codes times the bf16-rounded scales,
             // one packed multiply instead of an fp32 clip, multiply and conversion.
-            w[e] = mul_bf16x2(codes_bf16x2(t2, qp), pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
+            w[e] = mul_bf16x2(cw, pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
           }
         }
         // The W_hat buffer of this token slot was last read by the product of stage gg - 2.
@@ -446,18 +480,36 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <int MODE, bool PACKED>
+template <int MODE, bool PACKED, bool ZP>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const FusedArgs& args, int grid, cudaStream_t stream) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, PACKED>,
+    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, PACKED, ZP>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  fused_gemm_kernel<MODE, PACKED><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, args);
+  fused_gemm_kernel<MODE, PACKED, ZP><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, args);
   return cudaGetLastError();
+}
+
+template <bool ZP>
+cudaError_t launch_mode(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
+                        const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
+                        cudaStream_t stream) {
+  switch (mode) {
+    case FUSED_FWD_PC:
+      return packed ? launch_one<FUSED_FWD_PC, true, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
+                    : launch_one<FUSED_FWD_PC, false, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FUSED_FWD_GROUP:
+      return packed ? launch_one<FUSED_FWD_GROUP, true, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
+                    : launch_one<FUSED_FWD_GROUP, false, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FUSED_DX:
+      return launch_one<FUSED_DX, false, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    default:
+      return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace
@@ -468,18 +520,8 @@ cudaError_t launch_fused(int mode, int packed, const CUtensorMap& tm_tok, const 
                          const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
                          cudaStream_t stream) {
   if (grid < 1 || (args.kdim % 128) != 0 || args.kdim < 128) return cudaErrorInvalidValue;
-  switch (mode) {
-    case FUSED_FWD_PC:
-      return packed ? launch_one<FUSED_FWD_PC, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
-                    : launch_one<FUSED_FWD_PC, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
-    case FUSED_FWD_GROUP:
-      return packed ? launch_one<FUSED_FWD_GROUP, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
-                    : launch_one<FUSED_FWD_GROUP, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
-    case FUSED_DX:
-      return launch_one<FUSED_DX, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
-    default:
-      return cudaErrorInvalidValue;
-  }
+  return args.zero != nullptr ? launch_mode<true>(mode, packed, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
+                              : launch_mode<false>(mode, packed, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
 }
 
 }  // namespace lrqat

@@ -11,10 +11,11 @@
 namespace lrqat {
 
 // ---- elementwise.cu --------------------------------------------------------
-cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int p, float* s0,
-                                cudaStream_t stream);
-cudaError_t launch_downcast(const float* W0, const float* s0, int64_t m, int64_t k, int group_size, int bits,
-                            int packed, void* phi0, cudaStream_t stream);
+// z0 == nullptr: symmetric range setting (s0 only); else asymmetric (s0 and zero offsets z0).
+cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int bits, float* s0,
+                                float* z0, cudaStream_t stream);
+cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, int64_t m, int64_t k, int group_size,
+                            int bits, int packed, void* phi0, cudaStream_t stream);
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
                          int packed, const QuantParams& q, int8_t* wz, cudaStream_t stream);
 // codes = clip(round(X / s_x), -128, 127) as bf16; optional mask bits [k][ceil(T/32)].
@@ -64,6 +65,8 @@ struct FusedArgs {
   int64_t out_ld;
   int* status;
   uint64_t timeout_ns;
+  // Kept last: inserting it earlier shifted the fields above and slowed the producers.
+  const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
 };
 int fused_smem_bytes();
 cudaError_t launch_fused(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
@@ -82,6 +85,7 @@ struct DwArgs {
   float* dA_part; float* dB_part; float* ds_part;
   int* status;
   uint64_t timeout_ns;
+  const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
 };
 int dw_smem_bytes(int r16, int packed);
 cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,

@@ -136,6 +136,7 @@ int validate_layer(const lrqat_layer* L) {
     return fail(LRQAT_ERR_UNSUPPORTED, "group_size %d must be a multiple of 128 dividing k", L->group_size);
   if (L->act_bits != 0 && L->act_bits != 8)
     return fail(LRQAT_ERR_UNSUPPORTED, "act_bits must be 0 or 8 (got %d)", L->act_bits);
+  if (L->zero && !aligned16(L->zero)) return fail(LRQAT_ERR_ALIGNMENT, "zero (offsets) is not 16-byte aligned");
   return LRQAT_OK;
 }
 
@@ -395,7 +396,7 @@ int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrq
   LRQAT_CHECK_PTR(s0, "s0");
   const lrqat_layer& L = *layer;
   LRQAT_LAUNCH("range_minmax", 1, stream,
-               launch_range_minmax(W0, L.m, L.k, L.group_size, (1 << (L.bits - 1)) - 1, s0, stream),
+               launch_range_minmax(W0, L.m, L.k, L.group_size, L.bits, s0, L.zero, stream),
                "range_minmax launch");
   return LRQAT_OK;
 }
@@ -407,8 +408,8 @@ int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, v
   LRQAT_CHECK_PTR(Phi0, "Phi0");
   const lrqat_layer& L = *layer;
   LRQAT_LAUNCH("downcast", 1, stream,
-               launch_downcast(W0, s0, L.m, L.k, L.group_size, L.bits, L.phi_format == LRQAT_PHI_INT_PACKED, Phi0,
-                               stream),
+               launch_downcast(W0, s0, L.zero, L.m, L.k, L.group_size, L.bits,
+                               L.phi_format == LRQAT_PHI_INT_PACKED, Phi0, stream),
                "downcast launch");
   return LRQAT_OK;
 }
@@ -471,6 +472,7 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   a.num_tiles = a.num_rb * a.num_tb;
   a.q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
   a.s = s;
+  a.zero = L.zero;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
   a.s_x = L.act_bits == 8 ? s_x : nullptr;
@@ -561,6 +563,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.num_tiles = a.num_rb * a.num_tb;
     a.q = q;
     a.s = s;
+    a.zero = L.zero;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;
@@ -600,6 +603,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.num_units = plan.units;
     a.q = q;
     a.s = s;
+    a.zero = L.zero;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = L.act_bits == 8 ? s_x : nullptr;

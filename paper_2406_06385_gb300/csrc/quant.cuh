@@ -111,6 +111,14 @@ __device__ __forceinline__ uint32_t pack_rn_bf16x2(float lo, float hi) {
   return r;
 }
 
+// Elementwise bf16x2 difference, rounded to nearest even (exact for the small
+// integers it is used on).
+__device__ __forceinline__ uint32_t sub_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
 // Elementwise bf16x2 product, rounded to nearest even.
 __device__ __forceinline__ uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
   uint32_t r;

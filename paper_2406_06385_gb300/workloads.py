@@ -56,6 +56,8 @@ class LayerSpec:
     outlier_mult: float = 10.0
     a_std: float = 0.01
     b_std: float = 0.01
+    asym: bool = False     # asymmetric weights: zero offsets z (the INT2 runs of the paper)
+    w_row_shift: float = 0.0   # each row of W0 shifted by U(-w_row_shift, w_row_shift)
 
 
 @dataclass(frozen=True)
@@ -161,6 +163,9 @@ def make_layer(spec: LayerSpec, tokens: int, seed: int = 0, layer_index: int = 0
     if n_out > 0:
         pos = g_o.choice(m * k, size=n_out, replace=False)
         W0.reshape(-1)[pos] *= np.float32(spec.outlier_mult)
+    if spec.w_row_shift > 0:
+        g_s = np.random.Generator(np.random.PCG64(ss.spawn(1)[0]))
+        W0 += g_s.uniform(-spec.w_row_shift, spec.w_row_shift, size=(m, 1)).astype(np.float32)
     A_bits = bf16_bits(g_a.standard_normal((m, r), dtype=np.float32) * np.float32(spec.a_std))
     if zero_B:
         B_bits = np.zeros((r, k), dtype=np.uint16)

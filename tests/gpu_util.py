@@ -44,10 +44,12 @@ class DeviceLayer:
         t = torch()
         spec = data.spec
         self.spec = spec
-        self.layer = LQ.Layer.from_spec(spec)
         self.W0 = to_dev(data.W0)
         ng = spec.k // spec.group_size if spec.group_size else 1
         self.s0 = t.empty((spec.m, ng) if spec.group_size else (spec.m,), dtype=t.float32, device="cuda")
+        # asymmetric weights: the range setting writes the zero offsets, later calls read them
+        self.z = t.empty_like(self.s0) if spec.asym else None
+        self.layer = LQ.Layer.from_spec(spec, self.z.data_ptr() if spec.asym else 0)
         LQ.range_minmax(self.layer, self.W0, self.s0)
         if spec.phi_format == WL.PHI_QFIXED:
             self.phi0 = t.empty((spec.m, spec.k), dtype=t.int8, device="cuda")

@@ -71,3 +71,30 @@ def test_zero_row_gets_unit_scale_and_zero_codes():
     s0 = dl.s0.cpu().numpy()
     assert s0[5] == 1.0
     assert np.all(dl.phi0.cpu().numpy()[5] == 0)
+
+
+ASYM_CASES = [
+    # id, m, k, bits, group, phi
+    ("int2_q26_pc", 128, 256, 2, 0, WL.PHI_QFIXED),
+    ("int2_packed_g128", 256, 512, 2, 128, WL.PHI_INT_PACKED),
+    ("int3_packed_pc", 128, 384, 3, 0, WL.PHI_INT_PACKED),
+    ("q44_g256", 128, 512, 4, 256, WL.PHI_QFIXED),
+]
+
+
+@pytest.mark.parametrize("case", ASYM_CASES, ids=[c[0] for c in ASYM_CASES])
+def test_asym_range_and_downcast_bit_exact(case):
+    """Asymmetric min-max range setting (s0 and zero offsets z0) and the downcast
+    phi(W0 / s0 + z0) match the oracle exactly; the offsets really vary."""
+    name, m, k, bits, g, phi = case
+    spec = WL.LayerSpec(name, m, k, 4, 4.0, bits, g, phi, outlier_frac=1e-3, asym=True, w_row_shift=0.03)
+    data = WL.make_layer(spec, 1, seed=23, with_activations=False)
+    dl = DeviceLayer(data)
+    torch().cuda.synchronize()
+    L = oracle_layer(spec)
+    s0_ref, z0_ref = O.minmax_range_asym(data.W0, L)
+    np.testing.assert_array_equal(dl.s0.cpu().numpy().reshape(s0_ref.shape), s0_ref)
+    np.testing.assert_array_equal(dl.z.cpu().numpy().reshape(z0_ref.shape), z0_ref)
+    assert len(np.unique(z0_ref)) > 1
+    phi_ref = O.downcast(data.W0, s0_ref, L, z0_ref)
+    np.testing.assert_array_equal(dl.phi0.cpu().numpy().view(phi_ref.dtype), phi_ref)

@@ -22,9 +22,18 @@ TOL_GRAD = 2e-2
 
 
 def spec_of(name, m, k, r, bits=4, group=0, phi=WL.PHI_QFIXED, act=0, alpha=None, a_std=1 / 64, b_std=1e-3,
-            outliers=1e-3):
+            outliers=1e-3, asym=False, shift=0.0):
     return WL.LayerSpec(name, m, k, r, float(r if alpha is None else alpha), bits, group, phi, act,
-                        outlier_frac=outliers, a_std=a_std, b_std=b_std)
+                        outlier_frac=outliers, a_std=a_std, b_std=b_std, asym=asym, w_row_shift=shift)
+
+
+def oracle_base(data, OL):
+    """The oracle's own range setting and downcast: (s0, z0 or None, Phi0)."""
+    if data.spec.asym:
+        s0, z0 = O.minmax_range_asym(data.W0, OL)
+        return s0, z0, O.downcast(data.W0, s0, OL, z0)
+    s0 = O.minmax_scale(data.W0, OL)
+    return s0, None, O.downcast(data.W0, s0, OL)
 
 
 CASES = [
@@ -39,6 +48,12 @@ CASES = [
     ("q26_clip_heavy", spec_of("h", 128, 256, 16, bits=2, a_std=1.0, b_std=1.0), 200),
     ("tokens_1", spec_of("i", 128, 128, 1), 1),
     ("q44_pc_r40", spec_of("j", 256, 256, 40, a_std=0.2, b_std=0.2), 130),
+    # asymmetric weights with frozen zero offsets (the INT2 runs of the paper)
+    ("int2_asym_q26_pc", spec_of("k", 256, 512, 32, bits=2, asym=True, shift=0.03, a_std=0.2, b_std=0.2), 333),
+    ("int2_asym_packed_g128", spec_of("l", 128, 512, 16, bits=2, group=128, phi=WL.PHI_INT_PACKED, asym=True,
+                                      shift=0.03, a_std=0.3, b_std=0.3), 200),
+    ("q35_asym_g128_a8", spec_of("o", 256, 384, 32, bits=3, group=128, act=8, asym=True, shift=0.02,
+                                 a_std=0.2, b_std=0.2), 150),
 ]
 
 
@@ -65,11 +80,13 @@ def _run(spec, T, seed=0, s_scale=1.0, sx_factor=1.0, zero_B=False):
     LQ.get_device_status()
     # oracle side: its own range setting and downcast from the same W0
     OL = oracle_layer(spec)
-    s0 = O.minmax_scale(data.W0, OL)
-    phi0 = O.downcast(data.W0, s0, OL)
+    s0, z0, phi0 = oracle_base(data, OL)
+    if spec.asym:   # the device's zero offsets and base equal the oracle's exactly
+        np.testing.assert_array_equal(dl.z.cpu().numpy().reshape(z0.shape), z0)
+        np.testing.assert_array_equal(dl.phi0.cpu().numpy(), phi0)
     s = (s0 * np.float32(s_scale)).astype(np.float32)
-    Y_ref = O.linear_fwd(data.X, phi0, s, data.A, data.B, OL, s_x_host)
-    g = O.linear_bwd(data.dY, data.X, phi0, s, data.A, data.B, OL, s_x_host)
+    Y_ref = O.linear_fwd(data.X, phi0, s, data.A, data.B, OL, s_x_host, z0)
+    g = O.linear_bwd(data.dY, data.X, phi0, s, data.A, data.B, OL, s_x_host, z0)
     got = dict(Y=bits_to_f32(Y), dX=bits_to_f32(dX), dA=dA.cpu().numpy(), dB=dB.cpu().numpy(),
                ds=ds.cpu().numpy().reshape(g["ds"].shape))
     ref = dict(Y=Y_ref, dX=g["dX"], dA=g["dA"], dB=g["dB"], ds=g["ds"])
@@ -125,6 +142,9 @@ CODE_CASES = [
     ("q35_pc", spec_of("c2", 128, 384, 16, bits=3, a_std=0.2, b_std=0.2)),
     ("int3_packed", spec_of("c3", 128, 256, 8, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.3, b_std=0.3)),
     ("q44_g128", spec_of("c4", 128, 256, 16, group=128, a_std=0.1, b_std=0.1)),
+    ("int2_asym_q26", spec_of("c5", 128, 256, 16, bits=2, asym=True, shift=0.03, a_std=0.2, b_std=0.2)),
+    ("int2_asym_packed_g128", spec_of("c6", 128, 256, 8, bits=2, group=128, phi=WL.PHI_INT_PACKED, asym=True,
+                                      shift=0.03, a_std=0.3, b_std=0.3)),
 ]
 
 
@@ -132,9 +152,9 @@ CODE_CASES = [
 @pytest.mark.parametrize("zero_B", [False, True], ids=["lowrank", "ties"])
 def test_fused_codes_bit_exact(cid, spec, zero_B):
     """With s = 1 and X = I (T = k) the forward returns Y = C^T exactly; with
-    dY = I (T = m) the dX kernel returns its own codes C.  Both must equal the
-    oracle's codes except at near-ties; B = 0 makes every Q-fixed half-integer an
-    exact tie, which both sides must round half to even."""
+    dY = I (T = m) the dX kernel returns its own codes C (C - z with zero offsets).
+    Both must equal the oracle's codes except at near-ties; B = 0 makes every
+    Q-fixed half-integer an exact tie, which both sides must round half to even."""
     t = torch()
     data = WL.make_layer(spec, 1, seed=5, with_activations=False, zero_B=zero_B)
     dl = DeviceLayer(data)
@@ -156,14 +176,14 @@ def test_fused_codes_bit_exact(cid, spec, zero_B):
     LQ.linear_bwd(L, T, to_dev(eye_m), Xz, dl.phi0, dl.s, dl.A, dl.B, None, dX, dA, dB, ds, False, wsb)
     LQ.get_device_status()
     OL = oracle_layer(spec)
-    phi0 = O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL)
+    _, z0, phi0 = oracle_base(data, OL)
     ones = np.ones((m, k // spec.group_size) if spec.group_size else (m,))
-    fq = O.fake_quant_weight(phi0, ones, data.A, data.B, OL)
+    fq = O.fake_quant_weight(phi0, ones, data.A, data.B, OL, z0)
     exempt = O.near_tie(fq["u"]) if not zero_B else np.zeros_like(fq["c"], dtype=bool)
     c_fwd = bits_to_f32(Y).T
     c_dx = bits_to_f32(dX)
     for name, c in (("fwd", c_fwd), ("dX", c_dx)):
-        bad = (c != fq["c"]) & ~exempt
+        bad = (c != fq["cz"]) & ~exempt
         assert bad.sum() == 0, f"{name}: {bad.sum()} code mismatches (near-ties exempt: {exempt.sum()})"
     if zero_B and spec.phi_format == WL.PHI_QFIXED:
         assert (np.abs(fq["u"] - np.floor(fq["u"]) - 0.5) == 0).sum() > 0   # exact ties were exercised
