@@ -416,19 +416,24 @@ def _oracle_sample(wl, rows: int, tokens: int):
     spec = wl.layers[0]
     d = WL.make_layer(spec, wl.tokens, seed=0, layer_index=0)
     OL = O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
-    s0 = O.minmax_scale(d.W0, OL)
-    phi0 = O.downcast(d.W0, s0, OL)
+    if spec.asym:   # asymmetric weights: zero offsets from asymmetric range setting
+        s0, z0 = O.minmax_range_asym(d.W0, OL)
+        phi0 = O.downcast(d.W0, s0, OL, z0)
+        z0 = z0[:rows]
+    else:
+        s0, z0 = O.minmax_scale(d.W0, OL), None
+        phi0 = O.downcast(d.W0, s0, OL)
     sub = O.Layer(rows, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
     X = d.X[:tokens]
     s_x = float(np.float32(np.abs(d.X).max()) / np.float32(127.0)) if spec.act_bits == 8 else None
-    return dict(OL=sub, phi0=phi0[:rows], s=s0[:rows], A=d.A[:rows], B=d.B, X=X, dY=d.dY[:tokens, :rows], s_x=s_x,
-                frac=rows / spec.m, tokens=tokens, m=spec.m)
+    return dict(OL=sub, phi0=phi0[:rows], s=s0[:rows], z=z0, A=d.A[:rows], B=d.B, X=X, dY=d.dY[:tokens, :rows],
+                s_x=s_x, frac=rows / spec.m, tokens=tokens, m=spec.m)
 
 
 def _oracle_step(smp):
     import oracle as O
-    O.linear_fwd(smp["X"], smp["phi0"], smp["s"], smp["A"], smp["B"], smp["OL"], smp["s_x"])
-    O.linear_bwd(smp["dY"], smp["X"], smp["phi0"], smp["s"], smp["A"], smp["B"], smp["OL"], smp["s_x"])
+    O.linear_fwd(smp["X"], smp["phi0"], smp["s"], smp["A"], smp["B"], smp["OL"], smp["s_x"], smp["z"])
+    O.linear_bwd(smp["dY"], smp["X"], smp["phi0"], smp["s"], smp["A"], smp["B"], smp["OL"], smp["s_x"], smp["z"])
 
 
 def _calibrated_sample(wl, budget_s: float):

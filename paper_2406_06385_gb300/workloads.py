@@ -18,7 +18,7 @@ the fixed order W0, outlier positions, A, B, X, dY.
 """
 from __future__ import annotations
 
-from dataclasses import dataclass, field
+from dataclasses import dataclass, field, replace
 from typing import List, Optional
 
 import numpy as np
@@ -89,6 +89,8 @@ def workload(name: str) -> Workload:
     llama2_7b_mlp   : gate/up 4096->11008, down 11008->4096, T=8192, W3 per channel, packed INT-3
     llama3_8b_mlp   : 4096->14336->4096, T=8192, W4 g128, per-tensor int8 activations, Q4.4
     llama2_13b_layer: q/k/v/o 5120^2, gate/up 5120->13824, down 13824->5120, T=16384, W4 pc, Q4.4, merge
+    llama2_7b_attn_int2: 4096x4096, T=8192, r=32, W2 per channel asymmetric (frozen zero
+                      offsets, the paper's INT2 setting), Q2.6
     """
     if name == "tiny":
         return Workload(name, 64, [LayerSpec("proj", 256, 256, r=4, alpha=4.0, bits=4, group_size=0,
@@ -111,10 +113,13 @@ def workload(name: str) -> Workload:
         return Workload(name, 16384, [_llama_layer(n, 5120, 5120, **kw) for n in ("q", "k", "v", "o")]
                         + [_llama_layer("gate", 13824, 5120, **kw), _llama_layer("up", 13824, 5120, **kw),
                            _llama_layer("down", 5120, 13824, **kw)], merge=True)
+    if name == "llama2_7b_attn_int2":
+        spec = _llama_layer("attn", 4096, 4096, bits=2, group_size=0, phi_format=PHI_QFIXED)
+        return Workload(name, 8192, [replace(spec, asym=True)])
     raise KeyError(f"unknown workload {name!r}")
 
 
-WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer")
+WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer", "llama2_7b_attn_int2")
 
 
 @dataclass

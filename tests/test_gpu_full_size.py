@@ -34,13 +34,24 @@ FULL_CASES = [
     ("llama2_7b_attn", WL.workload("llama2_7b_attn").layers[0]),
     ("llama3_8b_gate_g128_a8", WL.workload("llama3_8b_mlp").layers[0]),
     ("llama2_7b_down_int3", WL.workload("llama2_7b_mlp").layers[2]),
+    ("llama2_7b_attn_int2_asym", WL.workload("llama2_7b_attn_int2").layers[0]),
 ]
+
+
+def _oracle_base(data, OL):
+    """The oracle's range setting and downcast: (s0, z0 or None, Phi0)."""
+    if data.spec.asym:
+        s0, z0 = O.minmax_range_asym(data.W0, OL)
+        return s0, z0, O.downcast(data.W0, s0, OL, z0)
+    s0 = O.minmax_scale(data.W0, OL)
+    return s0, None, O.downcast(data.W0, s0, OL)
 
 
 def _codes_spec(spec):
     # the codes do not depend on the activation quantizer; identity inputs need it off
     return WL.LayerSpec(spec.name, spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format,
-                        0, spec.w_std, spec.outlier_frac, spec.outlier_mult, spec.a_std, spec.b_std)
+                        0, spec.w_std, spec.outlier_frac, spec.outlier_mult, spec.a_std, spec.b_std, spec.asym,
+                        spec.w_row_shift)
 
 
 @pytest.mark.parametrize("cid,spec", FULL_CASES, ids=[c[0] for c in FULL_CASES])
@@ -71,9 +82,9 @@ def test_full_size_codes_bit_exact(cid, spec):
     LQ.get_device_status()
     c_dx = bits_to_f32(dX)
     OL = oracle_layer(spec)
-    phi0 = O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL)
+    _, z0, phi0 = _oracle_base(data, OL)
     u = O.preround(phi0, data.A, data.B, OL)
-    c = O.codes_from_u(u, OL)[1]
+    c = O.codes_from_u(u, OL)[1] - O.expand_zero(z0, OL)   # the operand holds c - z
     exempt = O.near_tie(u)
     for name, got in (("fwd", c_fwd), ("dX", c_dx)):
         bad = (got != c) & ~exempt
@@ -104,9 +115,8 @@ def test_full_size_sampled_outputs(cid, spec):
     LQ.get_device_status()
 
     OL = oracle_layer(spec)
-    s0 = O.minmax_scale(data.W0, OL)
-    phi0 = O.downcast(data.W0, s0, OL)
-    fq = O.fake_quant_weight(phi0, s0, data.A, data.B, OL)
+    s0, z0, phi0 = _oracle_base(data, OL)
+    fq = O.fake_quant_weight(phi0, s0, data.A, data.B, OL, z0)
     if spec.act_bits == 8:
         _, Xh, Mx = O.act_quant(data.X, s_x_host)
     else:
@@ -130,7 +140,7 @@ def test_full_size_sampled_outputs(cid, spec):
     s_rows = O.expand_scale(s0, OL)[rows]
     dU_rows = G_rows * s_rows * fq["M"][rows]
     dA_ref = scale * (dU_rows @ data.B.astype(np.float64).T)
-    Gc = G_rows * fq["c"][rows]
+    Gc = G_rows * fq["cz"][rows]
     ds_ref = Gc.sum(axis=1) if spec.group_size == 0 else Gc.reshape(len(rows), -1, spec.group_size).sum(axis=2)
     dA_got = dA.cpu().numpy()[rows]
     ds_got = ds.cpu().numpy().reshape((spec.m, -1) if spec.group_size else (spec.m,))[rows]
