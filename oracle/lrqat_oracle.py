@@ -45,6 +45,11 @@ Readings where the paper is silent (all repeated in the design notes):
      min-max: s0 = (max - min) / (2^b - 1) in fp32 and z0 = clip(round(n - min / s0),
      n, p) with min / s0 one fp32 division and the rest exact.  The STE mask is
      unchanged and ds = sum G (W_Z - z).
+  R11 per-token activations (the default of the weight-activation runs, Sec. 4):
+     dynamic absmax scale per token, s_x[t] = max_j |X[t, j]| / 127 in fp32 (1 for
+     an all-zero token), X_Z = clip(round(X / s_x[t]), -128, 127) with X / s_x[t] one
+     fp32 division, X_hat = s_x[t] X_Z; the scale is not differentiated (STE with
+     the clip mask, as R9).
 """
 from __future__ import annotations
 
@@ -70,6 +75,7 @@ class Layer:
     group_size: int = 0          # 0 = per output channel
     phi_format: int = PHI_QFIXED
     act_bits: int = 0            # 0 or 8
+    act_per_token: bool = False  # with act_bits 8: one dynamic scale per token (R11)
 
 
 def grid(bits: int):
@@ -244,11 +250,32 @@ def act_quant(X: np.ndarray, s_x: float):
     return codes, float(np.float32(s_x)) * codes, mask
 
 
+def act_scale_per_token(X: np.ndarray) -> np.ndarray:
+    """Dynamic per-token absmax scales s_x[t] = max_j |X[t, j]| / 127, fp32 (R11)."""
+    amax = np.abs(np.asarray(X, dtype=np.float32)).max(axis=1)
+    amax = np.where(amax > 0, amax, np.float32(127.0)).astype(np.float32)
+    return np.divide(amax, np.float32(127.0), dtype=np.float32)
+
+
+def act_quant_per_token(X: np.ndarray):
+    """Per-token int8 fake quantization (Eq. 1, z = 0, b = 8, one scale per token):
+    returns (codes, X_hat, mask, s_x)."""
+    s_x = act_scale_per_token(X)
+    x = np.divide(np.asarray(X, dtype=np.float32), s_x[:, None], dtype=np.float32)
+    q = np.rint(x.astype(np.float64))
+    codes = np.clip(q, -128, 127)
+    mask = ((q >= -128) & (q <= 127)).astype(np.float64)
+    return codes, s_x.astype(np.float64)[:, None] * codes, mask, s_x
+
+
 # ----------------------------------------------------------------------------
 # Linear layer forward / backward with checkpointed W_hat (Sec. 3)
 # ----------------------------------------------------------------------------
 def _inputs(X, layer: Layer, s_x: Optional[float]):
     X = np.asarray(X, dtype=np.float64)
+    if layer.act_bits == 8 and layer.act_per_token:
+        _, Xh, Mx, _ = act_quant_per_token(X)
+        return Xh, Mx
     if layer.act_bits == 8:
         assert s_x is not None
         _, Xh, Mx = act_quant(X, s_x)

@@ -430,3 +430,50 @@ def test_asym_ste_gradients_match_scalar_loops_and_finite_differences(case):
         sm[idx] -= eps
         fd = (loss(X64, sp) - loss(X64, sm)) / (2 * eps)
         assert abs(fd - got["ds"][idx]) <= 1e-9 * max(1.0, abs(fd))
+
+
+# ---------------------------------------------------------------------------
+# Per-token activations (default of the weight-activation runs, Sec. 4; reading R11)
+# ---------------------------------------------------------------------------
+def test_per_token_absmax_scale_and_error_bound():
+    """Each token's largest |X| lands on code +-127, nothing clips, and the rounding
+    error of every element is at most half of its token's step."""
+    rng = np.random.default_rng(31)
+    X = (rng.standard_normal((40, 96)) * rng.uniform(0.01, 10.0, size=(40, 1))).astype(np.float32)
+    X[7] = 0.0                                                      # an all-zero token
+    codes, Xh, mask, s_x = O.act_quant_per_token(X)
+    assert s_x[7] == 1.0 and np.all(codes[7] == 0)
+    live = np.arange(40) != 7
+    assert np.all(np.abs(codes[live]).max(axis=1) == 127)
+    assert mask.min() == 1.0
+    err = np.abs(Xh - X.astype(np.float64))
+    assert np.all(err <= 0.5 * s_x.astype(np.float64)[:, None] * (1 + 1e-6))
+
+
+def test_per_token_equals_per_tensor_for_equal_token_ranges():
+    """When every token has the same absmax, the per-token quantizer is the per-tensor
+    one (Eq. 1, z = 0) with that scale."""
+    rng = np.random.default_rng(32)
+    X = rng.standard_normal((12, 64)).astype(np.float32)
+    X /= np.abs(X).max(axis=1, keepdims=True)                       # every token's absmax is 1
+    X = (X * np.float32(3.0)).astype(np.float32)
+    c1, Xh1, m1, s_x = O.act_quant_per_token(X)
+    assert np.all(s_x == s_x[0])
+    c2, Xh2, m2 = O.act_quant(X, float(s_x[0]))
+    np.testing.assert_array_equal(c1, c2)
+    np.testing.assert_array_equal(Xh1, Xh2)
+
+
+def test_per_token_ste_gradients_match_scalar_loops():
+    layer = O.Layer(4, 6, 2, 2.0, 4, 0, O.PHI_QFIXED, 8, True)
+    spec = WL.LayerSpec("t", 4, 6, 2, 2.0, 4, 0, WL.PHI_QFIXED, a_std=0.5, b_std=0.5)
+    d = WL.make_layer(spec, 5, seed=19)
+    s0 = O.minmax_scale(d.W0, layer)
+    phi0 = O.downcast(d.W0, s0, layer)
+    ref = O.linear_bwd_loops(d.dY, d.X, phi0, s0, d.A, d.B, layer)
+    got = O.linear_bwd(d.dY, d.X, phi0, s0, d.A, d.B, layer)
+    for name in ("dX", "dA", "dB", "ds"):
+        np.testing.assert_allclose(got[name], ref[name], rtol=1e-12, atol=1e-12, err_msg=name)
+    Xh = O.act_quant_per_token(d.X)[1]
+    np.testing.assert_allclose(O.linear_fwd(d.X, phi0, s0, d.A, d.B, layer),
+                               Xh @ O.fake_quant_weight(phi0, s0, d.A, d.B, layer)["W_hat"].T, rtol=0, atol=0)
