@@ -194,7 +194,7 @@ class GpuWorkload:
             X = [dev(d.X_bits) for _ in range(sets)]
             dY = [dev(d.dY_bits) for _ in range(sets)]
             s_x = None
-            if spec.act_bits == 8:
+            if spec.act_bits == 8 and not spec.act_per_token:
                 sx = np.float32(np.float32(np.abs(d.X).max()) / np.float32(127.0))
                 s_x = torch.tensor([sx], dtype=torch.float32, device="cuda")
             lay = dict(spec=spec, L=L, z=z, phi0=phi0, s=s, A=dev(d.A_bits), B=dev(d.B_bits), X=X, dY=dY, s_x=s_x,
@@ -376,7 +376,8 @@ def run_gpu(args):
            "r": spec0.r, "alpha": spec0.alpha, "bits": spec0.bits,
            "granularity": "per-channel" if spec0.group_size == 0 else f"g{spec0.group_size}",
            "phi": "Q%d.%d int8" % (spec0.bits, 8 - spec0.bits) if spec0.phi_format == 0 else f"INT-{spec0.bits} packed",
-           "activations": "int8 per-tensor" if spec0.act_bits == 8 else "bf16",
+           "activations": ("int8 per-token" if spec0.act_per_token else "int8 per-tensor") if spec0.act_bits == 8
+           else "bf16",
            "merge": wl.merge, "parallelism": "replicas" if world > 1 else "single",
            "l2": f"inputs rotate over {args.sets} device copies ({args.sets * sum((l['X'][0].numel() + l['dY'][0].numel()) * 2 for l in gw.layers) / 2**20:.0f} MiB) > L2"}
     line = {
@@ -415,7 +416,8 @@ def _oracle_sample(wl, rows: int, tokens: int):
     from paper_2406_06385_gb300 import workloads as WL
     spec = wl.layers[0]
     d = WL.make_layer(spec, wl.tokens, seed=0, layer_index=0)
-    OL = O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+    OL = O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits,
+                 spec.act_per_token)
     if spec.asym:   # asymmetric weights: zero offsets from asymmetric range setting
         s0, z0 = O.minmax_range_asym(d.W0, OL)
         phi0 = O.downcast(d.W0, s0, OL, z0)
@@ -423,9 +425,11 @@ def _oracle_sample(wl, rows: int, tokens: int):
     else:
         s0, z0 = O.minmax_scale(d.W0, OL), None
         phi0 = O.downcast(d.W0, s0, OL)
-    sub = O.Layer(rows, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+    sub = O.Layer(rows, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits,
+                  spec.act_per_token)
     X = d.X[:tokens]
-    s_x = float(np.float32(np.abs(d.X).max()) / np.float32(127.0)) if spec.act_bits == 8 else None
+    s_x = (float(np.float32(np.abs(d.X).max()) / np.float32(127.0))
+           if spec.act_bits == 8 and not spec.act_per_token else None)
     return dict(OL=sub, phi0=phi0[:rows], s=s0[:rows], z=z0, A=d.A[:rows], B=d.B, X=X, dY=d.dY[:tokens, :rows],
                 s_x=s_x, frac=rows / spec.m, tokens=tokens, m=spec.m)
 

@@ -83,6 +83,13 @@ typedef struct {
                          the stored base Phi0 = phi(W0 / s0 + z0) already carries the
                          offset (z integer: round(x) + z = round(x + z)).
                          lrqat_range_minmax writes z0; every other call reads z.     */
+  int32_t act_per_token; /* with act_bits 8: 0 = one static scale s_x for the tensor
+                         (passed by the caller); 1 = one dynamic absmax scale per
+                         token, s_x[t] = max_j |X[t, j]| / 127 (the default of the
+                         weight-activation runs, Sec. 4), computed inside the calls
+                         (s_x may then be NULL).  It never clips, so dX
+                         has no activation mask; the GEMMs take X_hat =
+                         bf16(s_x[t] X_Z) as their token operand.                    */
 } lrqat_layer;
 
 /* Human-readable reason of the last non-OK status returned on this thread. */

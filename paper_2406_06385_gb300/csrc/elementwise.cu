@@ -218,6 +218,18 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __rest
   }
 }
 
+// round(fl(x / s)) with fl the IEEE fp32 division, without dividing in the common
+// case: y = x * r with r = fl(1 / s) is within |y| 2^-22 of x / s, and fl(x / s) within
+// |y| 2^-24, so unless y lies within |y| 2^-20 (+ a tiny absolute margin) of a
+// half-integer both round to the same integer; near a half-integer the exact
+// division decides.
+__device__ __forceinline__ float div_round(float x, float s, float r) {
+  const float y = x * r;
+  const float q = rintf(y);
+  if (fabsf(fabsf(y - q) - 0.5f) > fmaxf(fabsf(y), 1.0f) * 9.5367431640625e-07f) return q;   // 2^-20
+  return rintf(__fdiv_rn(x, s));
+}
+
 // --------------------------------------------------------- activation quant --
 // X_Z = clip(round(X / s_x), -128, 127) stored as exact bf16; optional mask bits
 // M_x = 1[-128 <= round(X / s_x) <= 127], laid out [k][ceil(T/32)] (bit = token % 32).
@@ -228,12 +240,18 @@ __global__ void act_quant_kernel(const uint4* __restrict__ X, int64_t T, int64_t
   const int64_t j8 = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (j8 >= k8) return;
   const float sx = *s_x;
+  const float rx = __frcp_rn(sx);
   const int64_t t0 = static_cast<int64_t>(blockIdx.y) * 32;
   uint32_t word[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  uint4 buf[4];
   for (int tt = 0; tt < 32; ++tt) {
     const int64_t t = t0 + tt;
     if (t >= T) break;
-    const uint4 raw = X[t * k8 + j8];
+    if ((tt & 3) == 0) {   // four tokens' loads in flight
+#pragma unroll
+      for (int i = 0; i < 4; ++i) buf[i] = t + i < T ? X[(t + i) * k8 + j8] : make_uint4(0u, 0u, 0u, 0u);
+    }
+    const uint4 raw = buf[tt & 3];
     const uint32_t in[4] = {raw.x, raw.y, raw.z, raw.w};
     uint32_t out[4];
 #pragma unroll
@@ -242,7 +260,7 @@ __global__ void act_quant_kernel(const uint4* __restrict__ X, int64_t T, int64_t
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const float x = __uint_as_float(e ? (in[h] & 0xFFFF0000u) : (in[h] << 16));
-        const float qv = rintf(__fdiv_rn(x, sx));
+        const float qv = div_round(x, sx, rx);
         const float c = fminf(fmaxf(qv, -128.0f), 127.0f);
         o |= (__float_as_uint(c) >> 16) << (16 * e);
         if (qv >= -128.0f && qv <= 127.0f) word[2 * h + e] |= 1u << tt;
@@ -254,6 +272,55 @@ __global__ void act_quant_kernel(const uint4* __restrict__ X, int64_t T, int64_t
   if (mask) {
 #pragma unroll
     for (int e = 0; e < 8; ++e) mask[(8 * j8 + e) * mask_ld + blockIdx.y] = word[e];
+  }
+}
+
+// Per-token dynamic int8 quantizer, one warp per token: s_x[t] = max_j |X[t, j]| / 127
+// (1 for an all-zero token), X_Z = clip(round(X / s_x[t]), -128, 127) with the IEEE
+// division, and X_hat = bf16(s_x[t] X_Z), the operand of the forward and dW GEMMs.
+// The first pass finds the absmax with 16-byte loads and a shuffle reduction; the
+// second pass rereads the row (from L1) and quantizes.  Absmax scaling never clips,
+// so no mask is needed.
+__global__ void __launch_bounds__(kThreads) act_quant_token_kernel(const uint4* __restrict__ X, int64_t T,
+                                                                   int64_t k8, uint4* __restrict__ out) {
+  const int64_t t = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (t >= T) return;
+  const uint4* row = X + t * k8;
+  float amax = 0.0f;
+  for (int64_t j0 = lane; j0 < k8; j0 += 128) {   // four 16-byte loads in flight per lane
+    uint4 v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = j0 + 32 * i < k8 ? row[j0 + 32 * i] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+      for (int h = 0; h < 4; ++h)
+        amax = fmaxf(amax, fmaxf(fabsf(__uint_as_float(in[h] << 16)), fabsf(__uint_as_float(in[h] & 0xFFFF0000u))));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+  const float sx = amax > 0.0f ? __fdiv_rn(amax, 127.0f) : 1.0f;
+  const float rx = __frcp_rn(sx);
+  for (int64_t j0 = lane; j0 < k8; j0 += 128) {
+    uint4 v[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = j0 + 32 * i < k8 ? row[j0 + 32 * i] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (j0 + 32 * i >= k8) break;
+      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+      uint32_t o[4];
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const float c0 = fminf(fmaxf(div_round(__uint_as_float(in[h] << 16), sx, rx), -128.0f), 127.0f);
+        const float c1 = fminf(fmaxf(div_round(__uint_as_float(in[h] & 0xFFFF0000u), sx, rx), -128.0f), 127.0f);
+        o[h] = pack_rn_bf16x2(sx * c0, sx * c1);
+      }
+      out[t * k8 + j0 + 32 * i] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
   }
 }
 
@@ -550,6 +617,14 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
   dim3 grid(static_cast<unsigned>((k8 + 127) / 128), static_cast<unsigned>((T + 31) / 32));
   act_quant_kernel<<<grid, 128, 0, stream>>>(reinterpret_cast<const uint4*>(X), T, k8, s_x,
                                              reinterpret_cast<uint4*>(codes), mask, (T + 31) / 32);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_act_quant_token(const uint16_t* X, int64_t T, int64_t k, uint16_t* x_hat, cudaStream_t stream) {
+  if ((k % 8) != 0 || (reinterpret_cast<uintptr_t>(X) & 15) != 0 || (reinterpret_cast<uintptr_t>(x_hat) & 15) != 0)
+    return cudaErrorInvalidValue;
+  act_quant_token_kernel<<<blocks_for(T * 32, kThreads), kThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(X), T, k / 8, reinterpret_cast<uint4*>(x_hat));
   return cudaGetLastError();
 }
 

@@ -19,6 +19,9 @@ cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, i
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
                          int packed, const QuantParams& q, int8_t* wz, cudaStream_t stream);
 // codes = clip(round(X / s_x), -128, 127) as bf16; optional mask bits [k][ceil(T/32)].
+// Per-token dynamic int8 quantizer: s_x[t] = max |X[t, :]| / 127, writes
+// X_hat = bf16(s_x[t] X_Z) [T, k].
+cudaError_t launch_act_quant_token(const uint16_t* X, int64_t T, int64_t k, uint16_t* x_hat, cudaStream_t stream);
 cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const float* s_x, uint16_t* codes,
                              uint32_t* mask, cudaStream_t stream);
 // TMA-friendly adapter layouts in one launch (null outputs are skipped):

@@ -137,6 +137,8 @@ int validate_layer(const lrqat_layer* L) {
   if (L->act_bits != 0 && L->act_bits != 8)
     return fail(LRQAT_ERR_UNSUPPORTED, "act_bits must be 0 or 8 (got %d)", L->act_bits);
   if (L->zero && !aligned16(L->zero)) return fail(LRQAT_ERR_ALIGNMENT, "zero (offsets) is not 16-byte aligned");
+  if (L->act_per_token != 0 && (L->act_per_token != 1 || L->act_bits != 8))
+    return fail(LRQAT_ERR_INVALID_ARG, "act_per_token must be 0, or 1 with act_bits == 8");
   return LRQAT_OK;
 }
 
@@ -267,7 +269,7 @@ DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
 struct FwdWs {
   uint16_t* a_pad;
   uint16_t* bt_pad;
-  uint16_t* x_codes;
+  uint16_t* x_codes;   // int8 codes (per tensor) or X_hat (per token), bf16
 };
 
 size_t fwd_ws_layout(const lrqat_layer& L, int64_t T, void* base, FwdWs* ws) {
@@ -432,7 +434,8 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   if (!A) return fail(LRQAT_ERR_INVALID_ARG, "A is NULL");
   if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
   LRQAT_CHECK_PTR(Y, "Y");
-  if (L.act_bits == 8 && !s_x) return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8");
+  if (L.act_bits == 8 && !L.act_per_token && !s_x)
+    return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8 (per-tensor scale)");
   const size_t need = fwd_ws_layout(L, T, nullptr, nullptr);
   if (!workspace || workspace_bytes < need)
     return fail(LRQAT_ERR_WORKSPACE, "forward workspace of %zu bytes required, %zu given", need,
@@ -448,7 +451,12 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
                launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
                "adapter layouts");
   const uint16_t* tok = X;
-  if (L.act_bits == 8) {
+  if (L.act_bits == 8 && L.act_per_token) {
+    // X_hat = bf16(s_x[t] X_Z): the per-token scales are folded into the token operand
+    LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant_token(X, T, L.k, ws.x_codes, stream),
+                 "activation quantizer");
+    tok = ws.x_codes;
+  } else if (L.act_bits == 8) {
     LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, ws.x_codes, nullptr, stream),
                  "activation quantizer");
     tok = ws.x_codes;
@@ -475,7 +483,7 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   a.zero = L.zero;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
-  a.s_x = L.act_bits == 8 ? s_x : nullptr;
+  a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;
   a.xmask = nullptr;
   a.xmask_ld = 0;
   a.out = Y;
@@ -514,7 +522,8 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
   LRQAT_CHECK_PTR(dX, "dX");
   if (!dA || !dB || !ds) return fail(LRQAT_ERR_INVALID_ARG, "dA, dB and ds must not be NULL");
-  if (L.act_bits == 8 && !s_x) return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8");
+  if (L.act_bits == 8 && !L.act_per_token && !s_x)
+    return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8 (per-tensor scale)");
   DeviceInfo* dev = nullptr;
   LRQAT_TRY(device_info(&dev));
   const DwPlan plan = plan_dw(L, T, dev->sms);
@@ -534,7 +543,12 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   LRQAT_LAUNCH("phi_transpose", 1, stream, launch_phi_transpose(Phi0, L.m, L.k, packed, ws.phit, stream),
                "transpose Phi0");
   const uint16_t* xop = X;
-  if (L.act_bits == 8) {
+  if (L.act_bits == 8 && L.act_per_token) {
+    // dW takes X_hat = bf16(s_x[t] X_Z); absmax scaling never clips, so dX needs no mask
+    LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant_token(X, T, L.k, ws.x_codes, stream),
+                 "activation quantizer");
+    xop = ws.x_codes;
+  } else if (L.act_bits == 8) {
     LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, ws.x_codes, ws.xmask, stream),
                  "activation quantizer");
     xop = ws.x_codes;
@@ -567,7 +581,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;
-    a.xmask = L.act_bits == 8 ? ws.xmask : nullptr;
+    a.xmask = L.act_bits == 8 && !L.act_per_token ? ws.xmask : nullptr;
     a.xmask_ld = static_cast<int32_t>((T + 31) / 32);
     a.out = dX;
     a.out_ld = L.k;
@@ -606,7 +620,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.zero = L.zero;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
-    a.s_x = L.act_bits == 8 ? s_x : nullptr;
+    a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;   // per token: folded into X_hat
     a.dA_part = ws.dA_part;
     a.dB_part = ws.dB_part;
     a.ds_part = ws.ds_part;

@@ -58,6 +58,7 @@ class LayerSpec:
     b_std: float = 0.01
     asym: bool = False     # asymmetric weights: zero offsets z (the INT2 runs of the paper)
     w_row_shift: float = 0.0   # each row of W0 shifted by U(-w_row_shift, w_row_shift)
+    act_per_token: bool = False   # with act_bits 8: dynamic per-token scales (else per tensor)
 
 
 @dataclass(frozen=True)
@@ -91,6 +92,8 @@ def workload(name: str) -> Workload:
     llama2_13b_layer: q/k/v/o 5120^2, gate/up 5120->13824, down 13824->5120, T=16384, W4 pc, Q4.4, merge
     llama2_7b_attn_int2: 4096x4096, T=8192, r=32, W2 per channel asymmetric (frozen zero
                       offsets, the paper's INT2 setting), Q2.6
+    llama2_7b_attn_w4a8: 4096x4096, T=8192, r=32, W4 per channel, Q4.4, per-token dynamic int8
+                      activations (the paper's weight-activation default)
     """
     if name == "tiny":
         return Workload(name, 64, [LayerSpec("proj", 256, 256, r=4, alpha=4.0, bits=4, group_size=0,
@@ -116,10 +119,14 @@ def workload(name: str) -> Workload:
     if name == "llama2_7b_attn_int2":
         spec = _llama_layer("attn", 4096, 4096, bits=2, group_size=0, phi_format=PHI_QFIXED)
         return Workload(name, 8192, [replace(spec, asym=True)])
+    if name == "llama2_7b_attn_w4a8":
+        spec = _llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=PHI_QFIXED, act_bits=8)
+        return Workload(name, 8192, [replace(spec, act_per_token=True)])
     raise KeyError(f"unknown workload {name!r}")
 
 
-WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer", "llama2_7b_attn_int2")
+WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer", "llama2_7b_attn_int2",
+             "llama2_7b_attn_w4a8")
 
 
 @dataclass

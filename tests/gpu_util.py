@@ -33,7 +33,8 @@ def empty(shape, dtype):
 
 def oracle_layer(spec):
     import oracle as O
-    return O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits)
+    return O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits,
+                   spec.act_per_token)
 
 
 class DeviceLayer:

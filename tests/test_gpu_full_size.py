@@ -35,6 +35,7 @@ FULL_CASES = [
     ("llama3_8b_gate_g128_a8", WL.workload("llama3_8b_mlp").layers[0]),
     ("llama2_7b_down_int3", WL.workload("llama2_7b_mlp").layers[2]),
     ("llama2_7b_attn_int2_asym", WL.workload("llama2_7b_attn_int2").layers[0]),
+    ("llama2_7b_attn_w4a8_token", WL.workload("llama2_7b_attn_w4a8").layers[0]),
 ]
 
 
@@ -51,7 +52,7 @@ def _codes_spec(spec):
     # the codes do not depend on the activation quantizer; identity inputs need it off
     return WL.LayerSpec(spec.name, spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format,
                         0, spec.w_std, spec.outlier_frac, spec.outlier_mult, spec.a_std, spec.b_std, spec.asym,
-                        spec.w_row_shift)
+                        spec.w_row_shift, False)
 
 
 @pytest.mark.parametrize("cid,spec", FULL_CASES, ids=[c[0] for c in FULL_CASES])
@@ -100,7 +101,7 @@ def test_full_size_sampled_outputs(cid, spec):
     L = dl.layer
     X, dY = to_dev(data.X_bits), to_dev(data.dY_bits)
     s_x_host, s_x = None, None
-    if spec.act_bits == 8:
+    if spec.act_bits == 8 and not spec.act_per_token:
         s_x_host = np.float32(np.float32(np.abs(data.X).max()) / np.float32(127.0))
         s_x = t.tensor([s_x_host], dtype=t.float32, device="cuda")
     Y = t.empty((T, spec.m), dtype=t.int16, device="cuda")
@@ -117,7 +118,9 @@ def test_full_size_sampled_outputs(cid, spec):
     OL = oracle_layer(spec)
     s0, z0, phi0 = _oracle_base(data, OL)
     fq = O.fake_quant_weight(phi0, s0, data.A, data.B, OL, z0)
-    if spec.act_bits == 8:
+    if spec.act_bits == 8 and spec.act_per_token:
+        _, Xh, Mx, _ = O.act_quant_per_token(data.X)
+    elif spec.act_bits == 8:
         _, Xh, Mx = O.act_quant(data.X, s_x_host)
     else:
         Xh = data.X.astype(np.float64)

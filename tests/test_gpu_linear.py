@@ -22,9 +22,10 @@ TOL_GRAD = 2e-2
 
 
 def spec_of(name, m, k, r, bits=4, group=0, phi=WL.PHI_QFIXED, act=0, alpha=None, a_std=1 / 64, b_std=1e-3,
-            outliers=1e-3, asym=False, shift=0.0):
+            outliers=1e-3, asym=False, shift=0.0, per_token=False):
     return WL.LayerSpec(name, m, k, r, float(r if alpha is None else alpha), bits, group, phi, act,
-                        outlier_frac=outliers, a_std=a_std, b_std=b_std, asym=asym, w_row_shift=shift)
+                        outlier_frac=outliers, a_std=a_std, b_std=b_std, asym=asym, w_row_shift=shift,
+                        act_per_token=per_token)
 
 
 def oracle_base(data, OL):
@@ -54,6 +55,10 @@ CASES = [
                                       shift=0.03, a_std=0.3, b_std=0.3), 200),
     ("q35_asym_g128_a8", spec_of("o", 256, 384, 32, bits=3, group=128, act=8, asym=True, shift=0.02,
                                  a_std=0.2, b_std=0.2), 150),
+    # per-token dynamic int8 activations (the paper's weight-activation default)
+    ("q44_pc_a8_token", spec_of("p", 256, 512, 32, act=8, per_token=True, a_std=0.2, b_std=0.2), 301),
+    ("int3_packed_g128_a8_token", spec_of("q", 128, 384, 16, bits=3, group=128, phi=WL.PHI_INT_PACKED, act=8,
+                                          per_token=True, a_std=0.3, b_std=0.3), 97),
 ]
 
 
@@ -64,7 +69,7 @@ def _run(spec, T, seed=0, s_scale=1.0, sx_factor=1.0, zero_B=False):
     X, dY = to_dev(data.X_bits), to_dev(data.dY_bits)
     s_x_host = None
     s_x = None
-    if spec.act_bits == 8:
+    if spec.act_bits == 8 and not spec.act_per_token:
         s_x_host = np.float32(np.float32(np.abs(data.X).max()) / np.float32(127.0) * np.float32(sx_factor))
         s_x = t.tensor([s_x_host], dtype=t.float32, device="cuda")
     L = dl.layer
