@@ -36,7 +36,7 @@ Readings where the paper is silent (all repeated in the design notes):
   R9 activation quantizer (weight-activation runs): per-tensor symmetric int8,
      X_Z = clip(round(X / s_x), -128, 127) with X / s_x one fp32 division,
      X_hat = s_x X_Z, STE with clip mask M_x = 1[-128 <= round(X/s_x) <= 127].
-  R10 asymmetric weights (the INT2 runs of Sec. 4; Eq. 1 with the zero offset z
+  R13 asymmetric weights (the INT2 runs of Sec. 4; Eq. 1 with the zero offset z
      outside the rounding, as the end of Sec. 3 states): W_hat = s (W_Z - z) with
      W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B + z), n, p) and z frozen at its
      range-setting value z0 (Sec. 4).  z is an integer, so round(x) + z = round(x + z)
@@ -45,7 +45,7 @@ Readings where the paper is silent (all repeated in the design notes):
      min-max: s0 = (max - min) / (2^b - 1) in fp32 and z0 = clip(round(n - min / s0),
      n, p) with min / s0 one fp32 division and the rest exact.  The STE mask is
      unchanged and ds = sum G (W_Z - z).
-  R11 per-token activations (the default of the weight-activation runs, Sec. 4):
+  R14 per-token activations (the default of the weight-activation runs, Sec. 4):
      dynamic absmax scale per token, s_x[t] = max_j |X[t, j]| / 127 in fp32 (1 for
      an all-zero token), X_Z = clip(round(X / s_x[t]), -128, 127) with X / s_x[t] one
      fp32 division, X_hat = s_x[t] X_Z; the scale is not differentiated (STE with
@@ -75,7 +75,7 @@ class Layer:
     group_size: int = 0          # 0 = per output channel
     phi_format: int = PHI_QFIXED
     act_bits: int = 0            # 0 or 8
-    act_per_token: bool = False  # with act_bits 8: one dynamic scale per token (R11)
+    act_per_token: bool = False  # with act_bits 8: one dynamic scale per token (R14)
 
 
 def grid(bits: int):
@@ -112,7 +112,7 @@ def minmax_scale(W0: np.ndarray, layer: Layer) -> np.ndarray:
 
 
 def minmax_range_asym(W0: np.ndarray, layer: Layer):
-    """Asymmetric min-max range setting (reading R10): returns (s0, z0), both float32
+    """Asymmetric min-max range setting (reading R13): returns (s0, z0), both float32
     and shaped like the scales; z0 holds integers in [n, p]."""
     n, p = grid(layer.bits)
     W0 = np.asarray(W0, dtype=np.float32)
@@ -168,7 +168,7 @@ def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
 
 
 def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer, z0: Optional[np.ndarray] = None) -> np.ndarray:
-    """Phi0 = phi(W0 / s0) (Eq. 6); with zero offsets phi(W0 / s0 + z0) (reading R10).
+    """Phi0 = phi(W0 / s0) (Eq. 6); with zero offsets phi(W0 / s0 + z0) (reading R13).
 
     Q-fixed (Eq. 7): INT8(round(2^{8-b} * clip(x, n, p))), stored int8 [m, k].
     INT-b (Sec. 3): clip(round(x), n, p), double-packed into uint8 [m, k/2].
@@ -225,7 +225,7 @@ def near_tie(u: np.ndarray, tol: float = NEAR_TIE_TOL) -> np.ndarray:
 
 def fake_quant_weight(Phi0, s, A, B, layer: Layer, z: Optional[np.ndarray] = None) -> Dict[str, np.ndarray]:
     """W_hat = s * clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p)  (Eq. 8);
-    with zero offsets W_hat = s * (clip(...) - z), the offset carried by Phi0 (R10)."""
+    with zero offsets W_hat = s * (clip(...) - z), the offset carried by Phi0 (R13)."""
     u = preround(Phi0, A, B, layer)
     q, c, M = codes_from_u(u, layer)
     cz = c - expand_zero(z, layer)
@@ -251,7 +251,7 @@ def act_quant(X: np.ndarray, s_x: float):
 
 
 def act_scale_per_token(X: np.ndarray) -> np.ndarray:
-    """Dynamic per-token absmax scales s_x[t] = max_j |X[t, j]| / 127, fp32 (R11)."""
+    """Dynamic per-token absmax scales s_x[t] = max_j |X[t, j]| / 127, fp32 (R14)."""
     amax = np.abs(np.asarray(X, dtype=np.float32)).max(axis=1)
     amax = np.where(amax > 0, amax, np.float32(127.0)).astype(np.float32)
     return np.divide(amax, np.float32(127.0), dtype=np.float32)
@@ -299,7 +299,7 @@ def linear_bwd(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = None,
       dX = (dY W_hat) * M_x
       dU = G * s * M                    (gradient w.r.t. u, mask from R3)
       dA = (alpha/r) dU B^T,  dB = (alpha/r) A^T dU
-      ds = sum over the row (or group) of G * c   (reading R4; G * (c - z), R10)
+      ds = sum over the row (or group) of G * c   (reading R4; G * (c - z), R13)
     """
     dY = np.asarray(dY, dtype=np.float64)
     Xh, Mx = _inputs(X, layer, s_x)

@@ -323,7 +323,7 @@ def test_workload_generator_is_deterministic_and_bf16_exact():
 
 # ---------------------------------------------------------------------------
 # Asymmetric weights with a frozen zero offset (INT2 runs of Sec. 4; Eq. 1 with
-# the offset outside the rounding, end of Sec. 3; reading R10)
+# the offset outside the rounding, end of Sec. 3; reading R13)
 # ---------------------------------------------------------------------------
 def _asym_data(bits, phi, group=0, m=24, k=256, r=4, T=1, seed=7, std=0.01, zero_B=False):
     """A layer whose rows are shifted by different offsets, so that the zero
@@ -433,7 +433,7 @@ def test_asym_ste_gradients_match_scalar_loops_and_finite_differences(case):
 
 
 # ---------------------------------------------------------------------------
-# Per-token activations (default of the weight-activation runs, Sec. 4; reading R11)
+# Per-token activations (default of the weight-activation runs, Sec. 4; reading R14)
 # ---------------------------------------------------------------------------
 def test_per_token_absmax_scale_and_error_bound():
     """Each token's largest |X| lands on code +-127, nothing clips, and the rounding
