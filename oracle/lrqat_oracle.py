@@ -50,6 +50,12 @@ Readings where the paper is silent (all repeated in the design notes):
      an all-zero token), X_Z = clip(round(X / s_x[t]), -128, 127) with X / s_x[t] one
      fp32 division, X_hat = s_x[t] X_Z; the scale is not differentiated (STE with
      the clip mask, as R9).
+  R17 optimizer step (App. B, Table B1): AdamW with decoupled weight decay
+     (Loshchilov & Hutter), (beta1, beta2) = (0.9, 0.95), bias-corrected moments,
+     eps = 1e-8 (not stated; the usual default), separate learning rates for A, B
+     and for s, weight decay 0 by default; before it, clipping of the global L2 norm
+     of all trainable gradients to max_norm = 1.0 with coefficient
+     min(1, max_norm / (norm + 1e-6)).  A and B are updated in fp32 master copies.
 """
 from __future__ import annotations
 
@@ -364,6 +370,33 @@ def linear_bwd_loops(dY, X, Phi0, s, A, B, layer: Layer, s_x: Optional[float] = 
             else:
                 ds[i, j // layer.group_size] += g * (c - z_full[i, j])
     return {"dX": dX, "dA": dA, "dB": dB, "ds": ds}
+
+
+# ----------------------------------------------------------------------------
+# Optimizer step on the trainable parameters A, B, s (App. B, Table B1) -- R17
+# ----------------------------------------------------------------------------
+def clip_coefficient(grads, max_norm: float) -> float:
+    """Global L2-norm clipping: all gradients are multiplied by this coefficient."""
+    total = float(np.sqrt(sum(float(np.sum(np.asarray(g, dtype=np.float64) ** 2)) for g in grads)))
+    return min(1.0, max_norm / (total + 1e-6))
+
+
+def adamw_update(p, g, m, v, step: int, lr: float, beta1: float = 0.9, beta2: float = 0.95, eps: float = 1e-8,
+                 weight_decay: float = 0.0):
+    """One AdamW step (decoupled weight decay) for one tensor; returns (p, m, v) as float64.
+
+    step counts from 1.  The moments are bias-corrected; the decay multiplies the
+    parameter by (1 - lr * weight_decay) before the Adam update, which is the same
+    as subtracting lr * weight_decay * p from it.
+    """
+    p = np.asarray(p, dtype=np.float64)
+    g = np.asarray(g, dtype=np.float64)
+    m = beta1 * np.asarray(m, dtype=np.float64) + (1.0 - beta1) * g
+    v = beta2 * np.asarray(v, dtype=np.float64) + (1.0 - beta2) * g * g
+    m_hat = m / (1.0 - beta1 ** step)
+    v_hat = v / (1.0 - beta2 ** step)
+    p = p * (1.0 - lr * weight_decay) - lr * m_hat / (np.sqrt(v_hat) + eps)
+    return p, m, v
 
 
 def rel_fro(a: np.ndarray, b: np.ndarray) -> float:

@@ -477,3 +477,53 @@ def test_per_token_ste_gradients_match_scalar_loops():
     Xh = O.act_quant_per_token(d.X)[1]
     np.testing.assert_allclose(O.linear_fwd(d.X, phi0, s0, d.A, d.B, layer),
                                Xh @ O.fake_quant_weight(phi0, s0, d.A, d.B, layer)["W_hat"].T, rtol=0, atol=0)
+
+
+# ---------------------------------------------------------------------------
+# Optimizer step (App. B, Table B1; reading R17)
+# ---------------------------------------------------------------------------
+def test_adamw_first_step_closed_form():
+    """Step 1 without decay: m_hat = g, v_hat = g^2, so p moves by -lr g / (|g| + eps)."""
+    rng = np.random.default_rng(41)
+    p0, g = rng.standard_normal(50), rng.standard_normal(50)
+    p1, m, v = O.adamw_update(p0, g, np.zeros(50), np.zeros(50), 1, lr=1e-3)
+    np.testing.assert_allclose(p1, p0 - 1e-3 * g / (np.abs(g) + 1e-8), rtol=1e-13, atol=1e-16)
+    np.testing.assert_allclose(m, 0.1 * g, rtol=1e-14)
+    np.testing.assert_allclose(v, 0.05 * g * g, rtol=1e-14)
+
+
+def test_clip_coefficient_cases():
+    g1, g2 = np.full(4, 0.25), np.full(12, 0.0)                    # norm 0.5 <= 1: untouched
+    assert O.clip_coefficient([g1, g2], 1.0) == 1.0
+    g3 = np.array([3.0, 4.0])                                      # norm 5: scaled to ~1
+    c = O.clip_coefficient([g3], 1.0)
+    assert abs(c * 5.0 - 1.0) < 1e-6
+
+
+def test_adamw_with_clipping_matches_torch_optimizer():
+    """Three clipped AdamW steps on A, B, s (two parameter groups with their own
+    learning rates, as in Table B1) agree with torch.optim.AdamW and
+    torch.nn.utils.clip_grad_norm_, an independent implementation."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(42)
+    shapes = {"A": (6, 3), "B": (3, 8), "s": (6,)}
+    lrs = {"A": 1e-3, "B": 1e-3, "s": 1e-4}
+    params = {k: rng.standard_normal(sh) for k, sh in shapes.items()}
+    tp = {k: torch.tensor(v, dtype=torch.float64, requires_grad=True) for k, v in params.items()}
+    opt = torch.optim.AdamW([{"params": [tp["A"], tp["B"]], "lr": lrs["A"]}, {"params": [tp["s"]], "lr": lrs["s"]}],
+                            betas=(0.9, 0.95), eps=1e-8, weight_decay=0.0)
+    state = {k: (np.zeros(sh), np.zeros(sh)) for k, sh in shapes.items()}
+    for step in range(1, 4):
+        grads = {k: rng.standard_normal(sh) * (3.0 if step == 2 else 0.1) for k, sh in shapes.items()}
+        coef = O.clip_coefficient(list(grads.values()), 1.0)
+        for k in shapes:
+            params[k], m, v = O.adamw_update(params[k], coef * grads[k], *state[k], step, lrs[k])
+            state[k] = (m, v)
+        opt.zero_grad()
+        for k in shapes:
+            tp[k].grad = torch.tensor(grads[k], dtype=torch.float64)
+        torch.nn.utils.clip_grad_norm_([tp[k] for k in shapes], 1.0)
+        opt.step()
+        for k in shapes:
+            np.testing.assert_allclose(params[k], tp[k].detach().numpy(), rtol=1e-12, atol=1e-15, err_msg=f"{k} {step}")
+    assert O.clip_coefficient([rng.standard_normal(10) * 3.0], 1.0) < 1.0    # clipping path was reachable
