@@ -174,6 +174,51 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
 int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, const uint16_t* B,
                 int8_t* W_Z, lrqat_stream_t stream);
 
+/* ---- Optimizer step on A, B, s (App. B, Table B1) ------------------------------
+ * AdamW with decoupled weight decay, bias-corrected moments, separate learning rates
+ * for the adapters and the scales, after clipping the global L2 norm of all
+ * trainable gradients (every layer's dA, dB, ds) with the coefficient
+ * min(1, max_grad_norm / (norm + 1e-6)).  Zero offsets stay frozen (Sec. 4). */
+typedef struct {
+  float lr_ab;           /* learning rate of A and B for this step (schedules are the caller's) */
+  float lr_s;            /* learning rate of s (0 freezes the scales, s = s0)                  */
+  float beta1, beta2;    /* (0.9, 0.95)                                                      */
+  float eps;             /* 1e-8                                                             */
+  float weight_decay_ab; /* 0                                                                */
+  float weight_decay_s;  /* 0                                                                */
+  float max_grad_norm;   /* 1.0; <= 0 disables clipping                                      */
+  int32_t step;          /* 1, 2, ...: bias correction 1 - beta^step                         */
+} lrqat_adamw;
+
+/* Optimizer state of one layer: device arrays owned by the caller, the moments zeroed
+ * and the master copies initialised from A and B before the first step.
+ * A32 [m, r] and B32 [r, k] fp32 master copies; first/second moments shaped like
+ * A, B and s.  All 16-byte aligned. */
+typedef struct {
+  float* A32;
+  float* B32;
+  float* mA;
+  float* vA;
+  float* mB;
+  float* vB;
+  float* ms;
+  float* vs;
+} lrqat_adamw_state;
+
+/* Adds the squared L2 norm of one layer's gradients dA [m, r], dB [r, k] and ds
+ * (shaped like s) to *sqnorm, a device fp32 scalar the caller zeroes once per step.
+ * Deterministic: a fixed summation order within the layer; layers add in stream
+ * order. */
+int lrqat_grad_sqnorm(const lrqat_layer* layer, const float* dA, const float* dB, const float* ds, float* sqnorm,
+                      lrqat_stream_t stream);
+
+/* One clipped AdamW step on a layer's A, B (fp32 masters in `state`; the bf16 copies
+ * A [m, r], B [r, k] are rewritten for the next forward) and s, with the step's global
+ * squared gradient norm *sqnorm (after every layer's lrqat_grad_sqnorm). */
+int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const float* sqnorm, const float* dA,
+                     const float* dB, const float* ds, const lrqat_adamw_state* state, float* s, uint16_t* A,
+                     uint16_t* B, lrqat_stream_t stream);
+
 /* Synchronizes `stream`, then reads and clears the device status word of the
  * current device.  Returns LRQAT_OK, LRQAT_ERR_TIMEOUT (a kernel's bounded
  * wait gave up since the last call) or LRQAT_ERR_CUDA. */

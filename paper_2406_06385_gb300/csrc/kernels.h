@@ -45,6 +45,22 @@ struct ReduceArgs {
 };
 cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream);
 
+// ---- optim.cu ----------------------------------------------------------------
+cudaError_t launch_grad_sqnorm(const float* dA, int64_t na, const float* dB, int64_t nb, const float* ds, int64_t nc,
+                               float* sqnorm, cudaStream_t stream);
+struct AdamwArgs {
+  const float* dA; const float* dB; const float* ds;
+  float* A32; float* B32; float* s;
+  float* mA; float* vA; float* mB; float* vB; float* ms; float* vs;
+  uint16_t* A; uint16_t* B;          // bf16 copies of the updated A, B
+  int64_t nA, nB, ns;
+  float lr_ab, lr_s, wd_ab, wd_s;
+  float beta1, beta2, eps, bc1, bc2;  // bc = 1 - beta^step
+  float max_norm;
+  const float* sqnorm;                // global squared gradient norm (device scalar)
+};
+cudaError_t launch_adamw(const AdamwArgs& a, cudaStream_t stream);
+
 // ---- fused_gemm.cu ---------------------------------------------------------
 enum FusedMode : int { FUSED_FWD_PC = 0, FUSED_FWD_GROUP = 1, FUSED_DX = 2 };
 

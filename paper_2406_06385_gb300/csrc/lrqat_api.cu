@@ -666,6 +666,64 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
   return LRQAT_OK;
 }
 
+int lrqat_grad_sqnorm(const lrqat_layer* layer, const float* dA, const float* dB, const float* ds, float* sqnorm,
+                      lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  const lrqat_layer& L = *layer;
+  if (!dA || !dB || !ds || !sqnorm) return fail(LRQAT_ERR_INVALID_ARG, "dA, dB, ds and sqnorm must be non-NULL");
+  const int64_t ns = L.group_size ? L.m * (L.k / L.group_size) : L.m;
+  LRQAT_LAUNCH("grad_sqnorm", 1, stream,
+               launch_grad_sqnorm(dA, L.m * L.r, dB, static_cast<int64_t>(L.r) * L.k, ds, ns, sqnorm, stream),
+               "gradient norm launch");
+  return LRQAT_OK;
+}
+
+int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const float* sqnorm, const float* dA,
+                     const float* dB, const float* ds, const lrqat_adamw_state* state, float* s, uint16_t* A,
+                     uint16_t* B, lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  if (!opt || !state) return fail(LRQAT_ERR_INVALID_ARG, "opt and state must be non-NULL");
+  if (opt->step < 1) return fail(LRQAT_ERR_INVALID_ARG, "step must be >= 1 (step=%d)", opt->step);
+  if (!(opt->beta1 >= 0.0f && opt->beta1 < 1.0f && opt->beta2 >= 0.0f && opt->beta2 < 1.0f))
+    return fail(LRQAT_ERR_INVALID_ARG, "betas must lie in [0, 1)");
+  if (!(opt->eps > 0.0f)) return fail(LRQAT_ERR_INVALID_ARG, "eps must be positive");
+  if (!dA || !dB || !ds || !sqnorm || !s || !A || !B || !state->A32 || !state->B32 || !state->mA || !state->vA ||
+      !state->mB || !state->vB || !state->ms || !state->vs)
+    return fail(LRQAT_ERR_INVALID_ARG, "gradients, parameters, state arrays and sqnorm must be non-NULL");
+  const lrqat_layer& L = *layer;
+  AdamwArgs a{};
+  a.dA = dA;
+  a.dB = dB;
+  a.ds = ds;
+  a.A32 = state->A32;
+  a.B32 = state->B32;
+  a.s = s;
+  a.mA = state->mA;
+  a.vA = state->vA;
+  a.mB = state->mB;
+  a.vB = state->vB;
+  a.ms = state->ms;
+  a.vs = state->vs;
+  a.A = A;
+  a.B = B;
+  a.nA = L.m * L.r;
+  a.nB = static_cast<int64_t>(L.r) * L.k;
+  a.ns = L.group_size ? L.m * (L.k / L.group_size) : L.m;
+  a.lr_ab = opt->lr_ab;
+  a.lr_s = opt->lr_s;
+  a.wd_ab = opt->weight_decay_ab;
+  a.wd_s = opt->weight_decay_s;
+  a.beta1 = opt->beta1;
+  a.beta2 = opt->beta2;
+  a.eps = opt->eps;
+  a.bc1 = static_cast<float>(1.0 - std::pow(static_cast<double>(opt->beta1), opt->step));
+  a.bc2 = static_cast<float>(1.0 - std::pow(static_cast<double>(opt->beta2), opt->step));
+  a.max_norm = opt->max_grad_norm;
+  a.sqnorm = sqnorm;
+  LRQAT_LAUNCH("adamw", 1, stream, launch_adamw(a, stream), "AdamW launch");
+  return LRQAT_OK;
+}
+
 int lrqat_get_device_status(lrqat_stream_t stream) {
   DeviceInfo* dev = nullptr;
   LRQAT_TRY(device_info(&dev));

@@ -40,6 +40,23 @@ class Layer(ctypes.Structure):
                    zero or None, int(getattr(spec, "act_per_token", False)))
 
 
+class AdamW(ctypes.Structure):
+    """Mirror of lrqat_adamw (App. B, Table B1 defaults)."""
+    _fields_ = [("lr_ab", ctypes.c_float), ("lr_s", ctypes.c_float), ("beta1", ctypes.c_float),
+                ("beta2", ctypes.c_float), ("eps", ctypes.c_float), ("weight_decay_ab", ctypes.c_float),
+                ("weight_decay_s", ctypes.c_float), ("max_grad_norm", ctypes.c_float), ("step", ctypes.c_int32)]
+
+    @classmethod
+    def make(cls, lr_ab: float, lr_s: float, step: int, beta1: float = 0.9, beta2: float = 0.95, eps: float = 1e-8,
+             weight_decay_ab: float = 0.0, weight_decay_s: float = 0.0, max_grad_norm: float = 1.0) -> "AdamW":
+        return cls(lr_ab, lr_s, beta1, beta2, eps, weight_decay_ab, weight_decay_s, max_grad_norm, step)
+
+
+class AdamWState(ctypes.Structure):
+    """Mirror of lrqat_adamw_state: device addresses of the fp32 masters and moments."""
+    _fields_ = [(n, ctypes.c_void_p) for n in ("A32", "B32", "mA", "vA", "mB", "vB", "ms", "vs")]
+
+
 _lib = None
 
 
@@ -62,6 +79,9 @@ def lib() -> ctypes.CDLL:
             "lrqat_linear_bwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ip, vp, sz, vp],
             "lrqat_merge": [lp, vp, vp, vp, vp, vp],
             "lrqat_get_device_status": [vp],
+            "lrqat_grad_sqnorm": [lp, vp, vp, vp, vp, vp],
+            "lrqat_adamw_step": [lp, ctypes.POINTER(AdamW), vp, vp, vp, vp, ctypes.POINTER(AdamWState), vp, vp, vp,
+                                 vp],
         }
         for name, args in sigs.items():
             fn = getattr(L, name)
@@ -138,6 +158,18 @@ def linear_bwd(layer: Layer, T: int, dY, X, Phi0, s, A, B, s_x, dX, dA, dB, ds, 
 
 def merge(layer: Layer, Phi0, A, B, W_Z, stream=None) -> None:
     _check(lib().lrqat_merge(ctypes.byref(layer), _ptr(Phi0), _ptr(A), _ptr(B), _ptr(W_Z), _stream(stream)))
+
+
+def grad_sqnorm(layer: Layer, dA, dB, ds, sqnorm, stream=None) -> None:
+    """Adds the squared L2 norm of the layer's gradients to the device scalar sqnorm."""
+    _check(lib().lrqat_grad_sqnorm(ctypes.byref(layer), _ptr(dA), _ptr(dB), _ptr(ds), _ptr(sqnorm), _stream(stream)))
+
+
+def adamw_step(layer: Layer, opt: AdamW, sqnorm, dA, dB, ds, state: dict, s, A, B, stream=None) -> None:
+    """One clipped AdamW step; `state` maps A32, B32, mA, vA, mB, vB, ms, vs to device tensors."""
+    st = AdamWState(*[_ptr(state[n]) for n, _ in AdamWState._fields_])
+    _check(lib().lrqat_adamw_step(ctypes.byref(layer), ctypes.byref(opt), _ptr(sqnorm), _ptr(dA), _ptr(dB), _ptr(ds),
+                                  ctypes.byref(st), _ptr(s), _ptr(A), _ptr(B), _stream(stream)))
 
 
 def get_device_status(stream=None) -> None:

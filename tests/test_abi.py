@@ -28,7 +28,7 @@ def test_header_declares_the_entry_points():
     names = header_functions()
     for expected in ("lrqat_range_minmax", "lrqat_downcast", "lrqat_linear_fwd", "lrqat_linear_bwd", "lrqat_merge",
                      "lrqat_fwd_workspace_bytes", "lrqat_bwd_workspace_bytes", "lrqat_get_device_status",
-                     "lrqat_last_error"):
+                     "lrqat_last_error", "lrqat_grad_sqnorm", "lrqat_adamw_step"):
         assert expected in names
 
 
@@ -81,3 +81,22 @@ def test_workspace_grows_with_tokens_and_activation_quantizer(lib):
     assert lib.lrqat_fwd_workspace_bytes(ctypes.byref(L8), 4096) >= 4096 * 256 * 2
     assert lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 64) > 0
     assert lib.lrqat_fwd_workspace_bytes(ctypes.byref(_layer(m=100)), 64) == 0
+
+
+def test_quantizer_setting_fields_are_checked_on_host(lib):
+    """act_per_token needs act_bits 8; the zero offsets must be 16-byte aligned."""
+    L = _layer(act_per_token=1)
+    assert lib.lrqat_linear_fwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, None, 16, 16, 1 << 20, None) == -1
+    L = _layer(zero=8)
+    assert lib.lrqat_linear_fwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, None, 16, 16, 1 << 20, None) == -3
+
+
+def test_adamw_arguments_are_checked_on_host(lib):
+    L = _layer()
+    st = LQ.AdamWState(*([16] * 8))
+    ok = LQ.AdamW.make(1e-3, 0.0, step=1)
+    args = lambda opt, state: (ctypes.byref(L), ctypes.byref(opt), 16, 16, 16, 16, state, 16, 16, 16, None)
+    assert lib.lrqat_adamw_step(*args(LQ.AdamW.make(1e-3, 0.0, step=0), ctypes.byref(st))) == -1
+    assert lib.lrqat_adamw_step(*args(LQ.AdamW.make(1e-3, 0.0, step=1, beta2=1.0), ctypes.byref(st))) == -1
+    assert lib.lrqat_adamw_step(*args(ok, None)) == -1
+    assert lib.lrqat_grad_sqnorm(ctypes.byref(L), None, 16, 16, 16, None) == -1
