@@ -56,6 +56,10 @@ Readings where the paper is silent (all repeated in the design notes):
      and for s, weight decay 0 by default; before it, clipping of the global L2 norm
      of all trainable gradients to max_norm = 1.0 with coefficient
      min(1, max_norm / (norm + 1e-6)).  A and B are updated in fp32 master copies.
+  R18 L^p range setting (App. B, the alternative to min-max): per row (or group)
+     the scale minimising sum |w - s clip(round(w / s), n, p)|^p over the candidates
+     s_j = fl32(s_minmax * j / N), j = 1..N (N = 100), w / s_j one fp32 division;
+     the smallest j wins a tie.  Symmetric grids only.
 """
 from __future__ import annotations
 
@@ -143,6 +147,35 @@ def expand_zero(z: Optional[np.ndarray], layer: Layer) -> np.ndarray:
     if z is None:
         return np.zeros((layer.m, layer.k))
     return expand_scale(z, layer)
+
+
+def lp_candidates(s_max: np.ndarray, n_cand: int) -> np.ndarray:
+    """Candidate scales s_j = fl32(s_max * j / N), j = 1..N, as float32 [..., N] (R18)."""
+    j = np.arange(1, n_cand + 1, dtype=np.float64)
+    return (np.asarray(s_max, dtype=np.float64)[..., None] * j / n_cand).astype(np.float32)
+
+
+def lp_loss(w: np.ndarray, s: float, bits: int, p_norm: float) -> float:
+    """sum |w - s clip(round(w / s), n, p)|^p for one row or group (Eq. 1 quantizer, z = 0)."""
+    n, p = grid(bits)
+    w32 = np.asarray(w, dtype=np.float32)
+    q = np.clip(np.rint(np.divide(w32, np.float32(s), dtype=np.float32).astype(np.float64)), n, p)
+    return float(np.sum(np.abs(w32.astype(np.float64) - float(s) * q) ** p_norm))
+
+
+def lp_range(W0: np.ndarray, layer: Layer, p_norm: float, n_cand: int = 100):
+    """L^p range setting (R18): returns (s0 float32 shaped like the scales, chosen j - 1)."""
+    s_max = minmax_scale(W0, layer)
+    W0 = np.asarray(W0, dtype=np.float32)
+    segs = W0.reshape(layer.m, -1, layer.group_size if layer.group_size else layer.k)
+    cands = lp_candidates(s_max.reshape(layer.m, -1), n_cand)
+    best = np.zeros(segs.shape[:2], dtype=np.int64)
+    for i in range(segs.shape[0]):
+        for g in range(segs.shape[1]):
+            losses = [lp_loss(segs[i, g], cands[i, g, j], layer.bits, p_norm) for j in range(n_cand)]
+            best[i, g] = int(np.argmin(losses))       # first minimum: the smallest j wins a tie
+    s0 = np.take_along_axis(cands, best[..., None], axis=2)[..., 0]
+    return s0.reshape(s_max.shape), best.reshape(s_max.shape)
 
 
 # ----------------------------------------------------------------------------

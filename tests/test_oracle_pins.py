@@ -527,3 +527,40 @@ def test_adamw_with_clipping_matches_torch_optimizer():
         for k in shapes:
             np.testing.assert_allclose(params[k], tp[k].detach().numpy(), rtol=1e-12, atol=1e-15, err_msg=f"{k} {step}")
     assert O.clip_coefficient([rng.standard_normal(10) * 3.0], 1.0) < 1.0    # clipping path was reachable
+
+
+# ---------------------------------------------------------------------------
+# L^p range setting (App. B; reading R18)
+# ---------------------------------------------------------------------------
+def test_lp_range_brute_force_and_properties():
+    """On a tiny layer the chosen scale is the brute-force minimiser over the candidate
+    grid (written independently, with Python's round), the last candidate is min-max
+    itself, and a row with an outlier clips it under L2 (a scale below min-max)."""
+    layer = O.Layer(4, 64, 2, 2.0, 3, 0, O.PHI_QFIXED)
+    rng = np.random.default_rng(51)
+    W0 = (rng.standard_normal((4, 64)) * 0.02).astype(np.float32)
+    W0[1, 5] = 0.3                                                  # an outlier row
+    s_mm = O.minmax_scale(W0, layer)
+    cands = O.lp_candidates(s_mm, 100)
+    assert np.all(cands[:, -1] == s_mm)
+    s2, j2 = O.lp_range(W0, layer, 2.0)
+    n, p = O.grid(3)
+    for i in range(4):
+        # brute force written independently: quantize-dequantize for every candidate
+        best, best_j = None, None
+        for j in range(100):
+            s = float(cands[i, j])
+            q = np.array([min(max(round(float(np.float32(w) / np.float32(s))), n), p) for w in W0[i]], dtype=np.float64)
+            loss = float(np.sum((W0[i].astype(np.float64) - s * q) ** 2))
+            if best is None or loss < best:
+                best, best_j = loss, j
+        assert j2[i] == best_j, (i, j2[i], best_j)
+    assert s2[1] < s_mm[1]                                          # the outlier row clips its outlier under L2
+
+
+def test_lp_range_groups_shape():
+    layer = O.Layer(2, 256, 2, 2.0, 4, 128, O.PHI_QFIXED)
+    W0 = (np.random.default_rng(52).standard_normal((2, 256)) * 0.02).astype(np.float32)
+    s0, j = O.lp_range(W0, layer, 2.4, n_cand=40)
+    assert s0.shape == (2, 2) and j.shape == (2, 2)
+    assert np.all(s0 <= O.minmax_scale(W0, layer))
