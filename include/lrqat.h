@@ -103,6 +103,17 @@ const char* lrqat_last_error(void);
  * W0: fp32 [m, k].  s0: fp32 [m] or [m, k/g] (output). */
 int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrqat_stream_t stream);
 
+/* L^p range setting (App. B, the alternative to min-max; symmetric grids only): per
+ * row (or group) the scale minimising sum |w - s clip(round(w/s), n, p)|^p over the
+ * candidates s_j = fl32(s_minmax * j / N), j = 1..N, with w/s one fp32 division; the
+ * smaller j wins a tie (losses in fp32, so nearly equal candidates may be ordered
+ * differently than in exact arithmetic).  p_norm > 0 (the paper uses 2, 2.4, 3,
+ * 3.5, 4, 5); 1 <= n_candidates <= 256; the row or group must fit in 200 KB of shared
+ * memory.  layer->zero must be NULL (LRQAT_ERR_UNSUPPORTED otherwise).
+ * W0: fp32 [m, k].  s0: fp32 [m] or [m, k/g] (output). */
+int lrqat_range_lp(const lrqat_layer* layer, const float* W0, float p_norm, int32_t n_candidates, float* s0,
+                   lrqat_stream_t stream);
+
 /* Downcasting operator of Eq. 6 / Eq. 7: Phi0 = phi(W0 / s0), with W0 / s0 one
  * fp32 IEEE division per element; with zero offsets phi(W0 / s0 + z0), the
  * integer offset added exactly.

@@ -324,6 +324,76 @@ __global__ void __launch_bounds__(kThreads) act_quant_token_kernel(const uint4* 
   }
 }
 
+// L^p range setting (symmetric), one block per (row, group): the segment is staged in
+// shared memory, s_max = max|w| / p as in min-max, and thread j < N evaluates the
+// candidate s_j = fl32(s_max (j + 1) / N): loss_j = sum |w - s_j clip(round(w / s_j), n, p)|^p
+// (w / s_j decided as one fp32 division, the error formed with one fused multiply-add,
+// |err|^p by multiplication for integer p).  The smallest loss wins, the smaller j on
+// a tie.
+__global__ void __launch_bounds__(kThreads) range_lp_kernel(const float* __restrict__ W0, int64_t k, int seg,
+                                                            int ngroups, int bits, float p_norm, int n_cand,
+                                                            float* __restrict__ s0) {
+  extern __shared__ float segw[];
+  const int64_t row = blockIdx.x / ngroups;
+  const int g = blockIdx.x % ngroups;
+  const float* src = W0 + row * k + static_cast<int64_t>(g) * seg;
+  float amax = 0.0f;
+  for (int j = threadIdx.x; j < seg; j += blockDim.x) {
+    const float v = src[j];
+    segw[j] = v;
+    amax = fmaxf(amax, fabsf(v));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+  __shared__ float warp_max[kThreads / 32];
+  __shared__ float best_loss[kThreads];
+  __shared__ int best_j[kThreads];
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = amax;
+  __syncthreads();
+  float a = 0.0f;
+  for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) a = fmaxf(a, warp_max[w]);
+  const float pmax = static_cast<float>((1 << (bits - 1)) - 1), nmin = -static_cast<float>(1 << (bits - 1));
+  const float s_max = a > 0.0f ? __fdiv_rn(a, pmax) : 1.0f;
+  const int j = threadIdx.x;
+  float loss = INFINITY;
+  if (j < n_cand) {
+    const float s = static_cast<float>(static_cast<double>(s_max) * (j + 1) / n_cand);
+    const float r = __frcp_rn(s);
+    const int ip = static_cast<int>(p_norm);
+    const bool int_p = static_cast<float>(ip) == p_norm && ip >= 1 && ip <= 8;
+    float acc0 = 0.0f, acc1 = 0.0f;
+    for (int e = 0; e < seg; ++e) {
+      const float w = segw[e];
+      const float q = fminf(fmaxf(div_round(w, s, r), nmin), pmax);
+      const float err = fabsf(fmaf(-s, q, w));
+      float t;
+      if (int_p) {
+        t = err;
+        for (int i = 1; i < ip; ++i) t *= err;
+      } else {
+        t = err > 0.0f ? powf(err, p_norm) : 0.0f;
+      }
+      if (e & 1) acc1 += t; else acc0 += t;
+    }
+    loss = acc0 + acc1;
+  }
+  best_loss[threadIdx.x] = loss;
+  best_j[threadIdx.x] = j;
+  __syncthreads();
+  for (int h = blockDim.x / 2; h > 0; h >>= 1) {
+    if (static_cast<int>(threadIdx.x) < h) {
+      const float lo = best_loss[threadIdx.x + h];
+      const int jo = best_j[threadIdx.x + h];
+      if (lo < best_loss[threadIdx.x] || (lo == best_loss[threadIdx.x] && jo < best_j[threadIdx.x])) {
+        best_loss[threadIdx.x] = lo;
+        best_j[threadIdx.x] = jo;
+      }
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) s0[blockIdx.x] = static_cast<float>(static_cast<double>(s_max) * (best_j[0] + 1) / n_cand);
+}
+
 // ---------------------------------------------------------------- re-layouts --
 // The four TMA-friendly layouts of the adapters, in one launch; each thread writes
 // 8 consecutive bf16 (16 bytes) of one output.  Null outputs are skipped.
@@ -579,6 +649,22 @@ cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group
   } else {
     range_minmax_asym_kernel<<<grid, kThreads, 0, stream>>>(W0, k, seg, ngroups, bits, s0, z0);
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_range_lp(const float* W0, int64_t m, int64_t k, int group_size, int bits, float p_norm, int n_cand,
+                            float* s0, cudaStream_t stream) {
+  const int ngroups = group_size ? static_cast<int>(k / group_size) : 1;
+  const int seg = group_size ? group_size : static_cast<int>(k);
+  const size_t smem = static_cast<size_t>(seg) * 4;
+  if (n_cand < 1 || n_cand > kThreads || smem > 200 * 1024) return cudaErrorInvalidValue;
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(range_lp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  range_lp_kernel<<<static_cast<unsigned>(m * ngroups), kThreads, smem, stream>>>(W0, k, seg, ngroups, bits, p_norm,
+                                                                                 n_cand, s0);
   return cudaGetLastError();
 }
 

@@ -14,6 +14,9 @@ namespace lrqat {
 // z0 == nullptr: symmetric range setting (s0 only); else asymmetric (s0 and zero offsets z0).
 cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int bits, float* s0,
                                 float* z0, cudaStream_t stream);
+// L^p range setting over N scaled min-max candidates (symmetric grids).
+cudaError_t launch_range_lp(const float* W0, int64_t m, int64_t k, int group_size, int bits, float p_norm, int n_cand,
+                            float* s0, cudaStream_t stream);
 cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, int64_t m, int64_t k, int group_size,
                             int bits, int packed, void* phi0, cudaStream_t stream);
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,

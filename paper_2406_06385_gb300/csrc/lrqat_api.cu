@@ -403,6 +403,24 @@ int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrq
   return LRQAT_OK;
 }
 
+int lrqat_range_lp(const lrqat_layer* layer, const float* W0, float p_norm, int32_t n_candidates, float* s0,
+                   lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  LRQAT_CHECK_PTR(W0, "W0");
+  LRQAT_CHECK_PTR(s0, "s0");
+  const lrqat_layer& L = *layer;
+  if (L.zero) return fail(LRQAT_ERR_UNSUPPORTED, "L^p range setting is implemented for symmetric grids only");
+  if (!(p_norm > 0.0f) || !std::isfinite(p_norm)) return fail(LRQAT_ERR_INVALID_ARG, "p_norm must be positive");
+  if (n_candidates < 1 || n_candidates > 256)
+    return fail(LRQAT_ERR_INVALID_ARG, "n_candidates must be in [1, 256] (got %d)", n_candidates);
+  const int64_t seg = L.group_size ? L.group_size : L.k;
+  if (seg * 4 > 200 * 1024) return fail(LRQAT_ERR_UNSUPPORTED, "row or group of %lld values too long", (long long)seg);
+  LRQAT_LAUNCH("range_lp", 1, stream,
+               launch_range_lp(W0, L.m, L.k, L.group_size, L.bits, p_norm, n_candidates, s0, stream),
+               "range_lp launch");
+  return LRQAT_OK;
+}
+
 int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0, lrqat_stream_t stream) {
   LRQAT_TRY(validate_layer(layer));
   LRQAT_CHECK_PTR(W0, "W0");

@@ -80,6 +80,7 @@ def lib() -> ctypes.CDLL:
             "lrqat_merge": [lp, vp, vp, vp, vp, vp],
             "lrqat_get_device_status": [vp],
             "lrqat_grad_sqnorm": [lp, vp, vp, vp, vp, vp],
+            "lrqat_range_lp": [lp, vp, ctypes.c_float, ctypes.c_int32, vp, vp],
             "lrqat_adamw_step": [lp, ctypes.POINTER(AdamW), vp, vp, vp, vp, ctypes.POINTER(AdamWState), vp, vp, vp,
                                  vp],
         }
@@ -158,6 +159,11 @@ def linear_bwd(layer: Layer, T: int, dY, X, Phi0, s, A, B, s_x, dX, dA, dB, ds, 
 
 def merge(layer: Layer, Phi0, A, B, W_Z, stream=None) -> None:
     _check(lib().lrqat_merge(ctypes.byref(layer), _ptr(Phi0), _ptr(A), _ptr(B), _ptr(W_Z), _stream(stream)))
+
+
+def range_lp(layer: Layer, W0, s0, p_norm: float, n_candidates: int = 100, stream=None) -> None:
+    """L^p range setting over n_candidates scaled min-max scales (symmetric grids)."""
+    _check(lib().lrqat_range_lp(ctypes.byref(layer), _ptr(W0), p_norm, n_candidates, _ptr(s0), _stream(stream)))
 
 
 def grad_sqnorm(layer: Layer, dA, dB, ds, sqnorm, stream=None) -> None:

@@ -28,7 +28,7 @@ def test_header_declares_the_entry_points():
     names = header_functions()
     for expected in ("lrqat_range_minmax", "lrqat_downcast", "lrqat_linear_fwd", "lrqat_linear_bwd", "lrqat_merge",
                      "lrqat_fwd_workspace_bytes", "lrqat_bwd_workspace_bytes", "lrqat_get_device_status",
-                     "lrqat_last_error", "lrqat_grad_sqnorm", "lrqat_adamw_step"):
+                     "lrqat_last_error", "lrqat_grad_sqnorm", "lrqat_adamw_step", "lrqat_range_lp"):
         assert expected in names
 
 
@@ -100,3 +100,15 @@ def test_adamw_arguments_are_checked_on_host(lib):
     assert lib.lrqat_adamw_step(*args(LQ.AdamW.make(1e-3, 0.0, step=1, beta2=1.0), ctypes.byref(st))) == -1
     assert lib.lrqat_adamw_step(*args(ok, None)) == -1
     assert lib.lrqat_grad_sqnorm(ctypes.byref(L), None, 16, 16, 16, None) == -1
+
+
+def test_lp_range_arguments_are_checked_on_host(lib):
+    L = _layer()
+    f = lib.lrqat_range_lp
+    assert f(ctypes.byref(L), 16, 0.0, 100, 16, None) == -1
+    assert f(ctypes.byref(L), 16, float("nan"), 100, 16, None) == -1
+    assert f(ctypes.byref(L), 16, 2.0, 0, 16, None) == -1
+    assert f(ctypes.byref(L), 16, 2.0, 257, 16, None) == -1
+    assert f(ctypes.byref(L), None, 2.0, 100, 16, None) == -1
+    assert f(ctypes.byref(_layer(zero=16)), 16, 2.0, 100, 16, None) == -2
+    assert f(ctypes.byref(_layer(k=65536)), 16, 2.0, 100, 16, None) == -2

@@ -98,3 +98,51 @@ def test_asym_range_and_downcast_bit_exact(case):
     assert len(np.unique(z0_ref)) > 1
     phi_ref = O.downcast(data.W0, s0_ref, L, z0_ref)
     np.testing.assert_array_equal(dl.phi0.cpu().numpy().view(phi_ref.dtype), phi_ref)
+
+
+LP_CASES = [
+    # id, m, k, bits, group, p_norm, n_candidates
+    ("q4_pc_p2.4", 128, 512, 4, 0, 2.4, 100),
+    ("q3_g128_p3", 128, 640, 3, 128, 3.0, 100),
+    ("q2_pc_p4", 128, 256, 2, 0, 4.0, 64),
+    ("q4_g256_p2_n256", 128, 512, 4, 256, 2.0, 256),
+    ("q4_long_row_p5", 128, 16384, 4, 0, 5.0, 100),    # 64 KB segment: opt-in shared memory
+    ("q3_pc_p3.5_n1", 128, 256, 3, 0, 3.5, 1),
+]
+
+
+@pytest.mark.parametrize("case", LP_CASES, ids=[c[0] for c in LP_CASES])
+def test_lp_range_matches_oracle(case):
+    """L^p range setting: each scale is exactly one of the candidates fl32(s_max j / N);
+    it is the oracle's choice, or (fp32 against fp64 losses) a candidate whose exact
+    loss is within 1e-4 of the oracle's minimum; a zero row gets the first candidate
+    of the unit scale, like min-max."""
+    name, m, k, bits, g, p_norm, n_cand = case
+    spec = WL.LayerSpec(name, m, k, 4, 4.0, bits, g, WL.PHI_QFIXED, outlier_frac=1e-3)
+    data = WL.make_layer(spec, 1, seed=24, with_activations=False)
+    data.W0[1, :] = 0.0
+    dl = DeviceLayer(data)
+    s0 = torch().empty_like(dl.s0)
+    LQ.range_lp(dl.layer, dl.W0, s0, p_norm, n_cand)
+    LQ.get_device_status()
+    got = s0.cpu().numpy().reshape(m, -1)
+    L = oracle_layer(spec)
+    s0_ref, best_ref = O.lp_range(data.W0, L, p_norm, n_cand)
+    s0_ref, best_ref = s0_ref.reshape(m, -1), best_ref.reshape(m, -1)
+    cands = O.lp_candidates(O.minmax_scale(data.W0, L).reshape(m, -1), n_cand)
+    segs = data.W0.reshape(m, got.shape[1], -1)
+    n_diff = 0
+    for i in range(m):
+        for j in range(got.shape[1]):
+            hit = np.nonzero(cands[i, j] == got[i, j])[0]
+            assert hit.size >= 1, (i, j, got[i, j])
+            if got[i, j] == s0_ref[i, j]:
+                continue
+            n_diff += 1
+            ref_loss = O.lp_loss(segs[i, j], s0_ref[i, j], bits, p_norm)
+            got_loss = O.lp_loss(segs[i, j], got[i, j], bits, p_norm)
+            assert got_loss <= ref_loss * (1 + 1e-4), (i, j, got_loss, ref_loss)
+    assert n_diff <= max(1, got.size // 20), n_diff
+    assert np.all(got[1] == cands[1, :, 0]) and np.all(cands[1, :, 0] == np.float32(1.0 / n_cand))
+    if n_cand > 1:
+        assert len(np.unique(best_ref[2:])) > 1    # the search is not stuck at one end
