@@ -60,6 +60,16 @@ Readings where the paper is silent (all repeated in the design notes):
      the scale minimising sum |w - s clip(round(w / s), n, p)|^p over the candidates
      s_j = fl32(s_minmax * j / N), j = 1..N (N = 100), w / s_j one fp32 division;
      the smallest j wins a tie.  Symmetric grids only.
+  R19 floating-point downcasting operators (Sec. 3 names FP16, BF16 and FP8 as the
+     simplest choices of phi): Phi0 = cast(fl32(W0 / s0)) with round-to-nearest-even
+     and no clipping inside phi (the clip of Eq. 8 follows the low-rank add); FP8 is
+     the OCP E4M3 (bias 7, no infinities, largest finite 448) or E5M2 (bias 15,
+     largest finite 57344) format, and casts beyond the largest finite value
+     saturate to it.  phi^{-1} is the exact value.  Stored as bit patterns: uint16
+     for BF16/FP16, uint8 for FP8.  Symmetric grids only.
+  R20 bf16 pre-round variant (the reading that R2 rejects, kept to measure it):
+     u = bf16(phi^{-1}(Phi0) + bf16((alpha/r) bf16(A B))), each product and sum
+     rounded to bf16 as an eager bf16 implementation would (A B from the exact sum).
 """
 from __future__ import annotations
 
@@ -70,6 +80,11 @@ import numpy as np
 
 PHI_QFIXED = 0
 PHI_INT_PACKED = 1
+PHI_BF16 = 2
+PHI_FP16 = 3
+PHI_FP8_E4M3 = 4
+PHI_FP8_E5M2 = 5
+FLOAT_PHI = (PHI_BF16, PHI_FP16, PHI_FP8_E4M3, PHI_FP8_E5M2)
 
 NEAR_TIE_TOL = 1e-5
 
@@ -86,6 +101,7 @@ class Layer:
     phi_format: int = PHI_QFIXED
     act_bits: int = 0            # 0 or 8
     act_per_token: bool = False  # with act_bits 8: one dynamic scale per token (R14)
+    u_bf16: bool = False         # pre-round value in bf16 (R20) instead of full precision (R2)
 
 
 def grid(bits: int):
@@ -206,18 +222,110 @@ def unpack_nibbles(packed: np.ndarray) -> np.ndarray:
     return out.astype(np.int8)
 
 
+# ----------------------------------------------------------------------------
+# Floating-point storage formats of phi (Sec. 3) -- reading R19
+# ----------------------------------------------------------------------------
+_FP8_LAYOUT = {PHI_FP8_E4M3: (4, 3, 7), PHI_FP8_E5M2: (5, 2, 15)}   # exponent bits, mantissa bits, bias
+
+
+def fp8_value(code: int, fmt: int) -> float:
+    """Value of one FP8 bit pattern from the format's definition (NaN for the
+    non-finite patterns): sign, biased exponent e, mantissa m; e = 0 is subnormal,
+    m / 2^M * 2^(1 - bias); otherwise (1 + m / 2^M) * 2^(e - bias).  E4M3 has no
+    infinities and only S.1111.111 is NaN; E5M2 reserves e = 31 as IEEE does."""
+    eb, mb, bias = _FP8_LAYOUT[fmt]
+    sign = -1.0 if code & 0x80 else 1.0
+    e = (code >> mb) & ((1 << eb) - 1)
+    m = code & ((1 << mb) - 1)
+    if fmt == PHI_FP8_E4M3 and e == 15 and m == 7:
+        return float("nan")
+    if fmt == PHI_FP8_E5M2 and e == 31:
+        return float("nan")
+    if e == 0:
+        return sign * (m / 2.0 ** mb) * 2.0 ** (1 - bias)
+    return sign * (1.0 + m / 2.0 ** mb) * 2.0 ** (e - bias)
+
+
+def fp8_encode(x: np.ndarray, fmt: int) -> np.ndarray:
+    """Round-to-nearest-even cast of fp32 values to FP8 bit patterns, saturating at
+    the largest finite magnitude (R19).  The nearest finite magnitude is found on
+    the table of all non-negative finite values (ascending with the code); on an
+    exact midpoint the even code (even mantissa) wins.  The sign bit is kept, so a
+    negative value that rounds to zero gives negative zero."""
+    mags = np.array([fp8_value(c, fmt) for c in range(128)])
+    finite = np.nonzero(np.isfinite(mags))[0]
+    grid_v, grid_c = mags[finite], finite
+    x = np.asarray(x, dtype=np.float32)
+    a = np.minimum(np.abs(x.astype(np.float64)), grid_v[-1])
+    hi = np.clip(np.searchsorted(grid_v, a, side="left"), 0, len(grid_v) - 1)
+    lo = np.maximum(hi - 1, 0)
+    d_lo, d_hi = a - grid_v[lo], grid_v[hi] - a
+    pick_hi = (d_hi < d_lo) | ((d_hi == d_lo) & (grid_c[hi] % 2 == 0))
+    code = np.where(pick_hi, grid_c[hi], grid_c[lo]).astype(np.uint8)
+    return code | np.where(np.signbit(x), np.uint8(0x80), np.uint8(0))
+
+
+def fp8_decode(codes: np.ndarray, fmt: int) -> np.ndarray:
+    table = np.array([fp8_value(c, fmt) for c in range(256)])
+    return table[np.asarray(codes, dtype=np.uint8).astype(np.int64)]
+
+
+def bf16_encode(x: np.ndarray) -> np.ndarray:
+    """Round-to-nearest-even of fp32 values to bf16 (the upper half of the fp32 bit
+    pattern), as uint16 bit patterns: add 0x7FFF plus the lowest kept bit, truncate.
+    (Finite inputs only; they never come near the fp32 overflow threshold here.)"""
+    b = np.asarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    return ((b + 0x7FFF + ((b >> 16) & 1)) >> 16).astype(np.uint16)
+
+
+def bf16_round(v: np.ndarray) -> np.ndarray:
+    """float64 values in bf16's normal range rounded (nearest, ties to even) to the 8
+    significant bits of bf16, in one step: v = m 2^e with m in [0.5, 1), keep
+    rint(m 2^8) 2^(e-8)."""
+    m, e = np.frexp(np.asarray(v, dtype=np.float64))
+    return np.ldexp(np.rint(np.ldexp(m, 8)), e - 8)
+
+
+def bf16_decode(bits: np.ndarray) -> np.ndarray:
+    return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def float_cast(x: np.ndarray, fmt: int) -> np.ndarray:
+    """phi for the floating-point formats: the stored bit patterns of x (R19)."""
+    if fmt == PHI_BF16:
+        return bf16_encode(x)
+    if fmt == PHI_FP16:
+        return np.asarray(x, dtype=np.float32).astype(np.float16).view(np.uint16)
+    return fp8_encode(x, fmt)
+
+
+def float_value(bits: np.ndarray, fmt: int) -> np.ndarray:
+    """phi^{-1} for the floating-point formats: the exact value as float64."""
+    if fmt == PHI_BF16:
+        return bf16_decode(bits)
+    if fmt == PHI_FP16:
+        return np.asarray(bits, dtype=np.uint16).view(np.float16).astype(np.float64)
+    return fp8_decode(bits, fmt)
+
+
 def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer, z0: Optional[np.ndarray] = None) -> np.ndarray:
     """Phi0 = phi(W0 / s0) (Eq. 6); with zero offsets phi(W0 / s0 + z0) (reading R13).
 
     Q-fixed (Eq. 7): INT8(round(2^{8-b} * clip(x, n, p))), stored int8 [m, k].
     INT-b (Sec. 3): clip(round(x), n, p), double-packed into uint8 [m, k/2].
+    BF16 / FP16 / FP8 (R19): the rounded cast of x, as bit patterns.
     W0 / s0 is a single fp32 division per element (reading R8); adding the integer
     offset is exact.
     """
     n, p = grid(layer.bits)
     W0 = np.asarray(W0, dtype=np.float32)
     s_full = expand_scale(s0, layer).astype(np.float32)
-    x = np.divide(W0, s_full, dtype=np.float32).astype(np.float64)
+    x32 = np.divide(W0, s_full, dtype=np.float32)
+    if layer.phi_format in FLOAT_PHI:
+        if z0 is not None:
+            raise ValueError("floating-point phi is defined for symmetric grids only (R19)")
+        return float_cast(x32, layer.phi_format)
+    x = x32.astype(np.float64)
     if z0 is not None:
         x = x + expand_scale(z0, layer)
     if layer.phi_format == PHI_QFIXED:
@@ -228,7 +336,10 @@ def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer, z0: Optional[np.ndarr
 
 
 def upcast(Phi0: np.ndarray, layer: Layer) -> np.ndarray:
-    """phi^{-1}(Phi0) as float64: Phi0 / 2^{8-b} (Eq. 7) or the unpacked INT-b value."""
+    """phi^{-1}(Phi0) as float64: Phi0 / 2^{8-b} (Eq. 7), the unpacked INT-b value, or
+    the exact value of a floating-point pattern (R19)."""
+    if layer.phi_format in FLOAT_PHI:
+        return float_value(Phi0, layer.phi_format)
     if layer.phi_format == PHI_QFIXED:
         return np.asarray(Phi0, dtype=np.int8).astype(np.float64) / 2.0 ** (8 - layer.bits)
     return unpack_nibbles(Phi0).astype(np.float64)
@@ -238,8 +349,12 @@ def upcast(Phi0: np.ndarray, layer: Layer) -> np.ndarray:
 # LR-QAT weight (Eq. 8) and its integer codes
 # ----------------------------------------------------------------------------
 def preround(Phi0: np.ndarray, A: np.ndarray, B: np.ndarray, layer: Layer) -> np.ndarray:
-    """u = phi^{-1}(Phi0) + (alpha / r) A B, the argument of round() in Eq. 8 (reading R2)."""
+    """u = phi^{-1}(Phi0) + (alpha / r) A B, the argument of round() in Eq. 8 (reading R2;
+    with ``layer.u_bf16`` each step rounded to bf16, reading R20)."""
     AB = np.asarray(A, dtype=np.float64) @ np.asarray(B, dtype=np.float64)
+    if layer.u_bf16:
+        bf = bf16_round
+        return bf(upcast(Phi0, layer) + bf((layer.alpha / layer.r) * bf(AB)))
     return upcast(Phi0, layer) + (layer.alpha / layer.r) * AB
 
 

@@ -25,6 +25,10 @@ import numpy as np
 
 PHI_QFIXED = 0       # int8 fixed point Qb.(8-b), Eq. 7
 PHI_INT_PACKED = 1   # two INT-b nibbles per byte (Sec. 3, downcasting operator)
+PHI_BF16 = 2         # floating-point casts of W0 / s0 (Sec. 3), stored as bit patterns
+PHI_FP16 = 3
+PHI_FP8_E4M3 = 4
+PHI_FP8_E5M2 = 5
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -49,7 +53,7 @@ class LayerSpec:
     alpha: float           # LoRA scaling numerator (alpha / r multiplies A B)
     bits: int              # weight bit-width b
     group_size: int        # 0 = per output channel, else group width along k
-    phi_format: int        # PHI_QFIXED or PHI_INT_PACKED
+    phi_format: int        # one of the PHI_* storage formats above
     act_bits: int = 0      # 0 = no activation quantizer, 8 = per-tensor int8
     w_std: float = 0.02
     outlier_frac: float = 0.0
@@ -122,11 +126,16 @@ def workload(name: str) -> Workload:
     if name == "llama2_7b_attn_w4a8":
         spec = _llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=PHI_QFIXED, act_bits=8)
         return Workload(name, 8192, [replace(spec, act_per_token=True)])
+    if name.startswith("llama2_7b_attn_phi_"):
+        # the same 4096 x 4096 W4 per-channel layer with a floating-point base (Table 2 ablation)
+        fmt = {"bf16": PHI_BF16, "fp16": PHI_FP16, "fp8": PHI_FP8_E4M3, "fp8e5m2": PHI_FP8_E5M2}[name[19:]]
+        return Workload(name, 8192, [_llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=fmt)])
     raise KeyError(f"unknown workload {name!r}")
 
 
 WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer", "llama2_7b_attn_int2",
-             "llama2_7b_attn_w4a8")
+             "llama2_7b_attn_w4a8", "llama2_7b_attn_phi_bf16", "llama2_7b_attn_phi_fp16", "llama2_7b_attn_phi_fp8",
+             "llama2_7b_attn_phi_fp8e5m2")
 
 
 @dataclass

@@ -232,6 +232,9 @@ LOOP_CASES = [
     dict(m=3, k=8, r=3, bits=4, group_size=0, phi=O.PHI_INT_PACKED, act=0, std=1.0),
     dict(m=2, k=256, r=2, bits=4, group_size=128, phi=O.PHI_QFIXED, act=0, std=1.0),
     dict(m=4, k=6, r=2, bits=4, group_size=0, phi=O.PHI_QFIXED, act=8, std=1.0),
+    dict(m=4, k=6, r=2, bits=4, group_size=0, phi=O.PHI_BF16, act=0, std=0.3),
+    dict(m=4, k=6, r=2, bits=3, group_size=0, phi=O.PHI_FP8_E4M3, act=0, std=2.0),    # clip active
+    dict(m=2, k=256, r=2, bits=4, group_size=128, phi=O.PHI_FP16, act=0, std=1.0),
 ]
 
 
@@ -265,7 +268,7 @@ def _loss(dY, X, phi0, s, A, B, layer):
     return float(np.sum(dY * O.linear_fwd(X, phi0, s, A, B, layer)))
 
 
-@pytest.mark.parametrize("case", LOOP_CASES[:4])
+@pytest.mark.parametrize("case", LOOP_CASES[:4] + LOOP_CASES[5:])
 def test_dX_and_ds_are_exact_gradients(case):
     """Y is linear in X and in s (c does not depend on s, Eq. 5/8), so central
     differences of <dY, Y> reproduce dX and ds up to float64 rounding."""
@@ -564,3 +567,138 @@ def test_lp_range_groups_shape():
     s0, j = O.lp_range(W0, layer, 2.4, n_cand=40)
     assert s0.shape == (2, 2) and j.shape == (2, 2)
     assert np.all(s0 <= O.minmax_scale(W0, layer))
+
+
+# ---------------------------------------------------------------------------
+# Floating-point downcasting operators (Sec. 3; reading R19)
+# ---------------------------------------------------------------------------
+FP8_TORCH = [(O.PHI_FP8_E4M3, "float8_e4m3fn", 448.0), (O.PHI_FP8_E5M2, "float8_e5m2", 57344.0)]
+
+
+@pytest.mark.parametrize("fmt,tname,vmax", FP8_TORCH)
+def test_fp8_decode_exhaustive_against_torch(fmt, tname, vmax):
+    """All 256 FP8 patterns decode (from the format definition) to torch's values; the
+    non-finite patterns are exactly torch's; the largest finite value is the format's."""
+    torch = pytest.importorskip("torch")
+    td = getattr(torch, tname, None)
+    if td is None:
+        pytest.skip(f"torch has no {tname}")
+    codes = np.arange(256, dtype=np.uint8)
+    ours = O.fp8_decode(codes, fmt)
+    ref = torch.from_numpy(codes).view(td).to(torch.float64).numpy()
+    fin = np.isfinite(ref)
+    np.testing.assert_array_equal(ours[fin], ref[fin])
+    assert np.all(np.isnan(ours[~fin]))
+    assert np.nanmax(ours) == vmax and np.nanmin(ours) == -vmax
+
+
+@pytest.mark.parametrize("fmt,tname,vmax", FP8_TORCH)
+def test_fp8_encode_against_torch_midpoints_and_saturation(fmt, tname, vmax):
+    """In range the cast equals torch's round-to-nearest-even cast bit for bit (signed
+    zeros included); every finite pattern round-trips; an exact midpoint between two
+    neighbours takes the even pattern; beyond the largest finite value it saturates."""
+    torch = pytest.importorskip("torch")
+    td = getattr(torch, tname, None)
+    if td is None:
+        pytest.skip(f"torch has no {tname}")
+    rng = np.random.default_rng(61)
+    x = (rng.standard_normal(200000) * 10.0 ** rng.uniform(-4, np.log10(vmax) - 0.5, 200000)).astype(np.float32)
+    x = np.concatenate([x[np.abs(x) <= vmax], np.float32([0.0, -0.0, 1e-30, -1e-30])])   # torch does not saturate
+    ref = torch.from_numpy(x).to(td).view(torch.uint8).numpy()
+    np.testing.assert_array_equal(O.fp8_encode(x, fmt), ref)
+    vals = O.fp8_decode(np.arange(256, dtype=np.uint8), fmt)
+    finite = np.nonzero(np.isfinite(vals))[0].astype(np.uint8)
+    np.testing.assert_array_equal(O.fp8_encode(vals[finite].astype(np.float32), fmt), finite)
+    pos = np.nonzero(np.isfinite(vals[:128]))[0]
+    mids = ((vals[pos[:-1]] + vals[pos[1:]]) / 2).astype(np.float32)     # exact in fp32
+    got = O.fp8_encode(mids, fmt)
+    assert np.all(got % 2 == 0)
+    assert np.all((got == pos[:-1]) | (got == pos[1:]))
+    big = np.float32([vmax * 1.01, 1e30, -1e30])
+    np.testing.assert_array_equal(O.fp8_decode(O.fp8_encode(big, fmt), fmt), [vmax, vmax, -vmax])
+
+
+def test_bf16_and_fp16_casts_against_torch():
+    """bf16 (written from the bit pattern) and fp16 casts equal torch's casts, including
+    constructed exact midpoints, which go to the even neighbour; bf16_round of an fp32
+    value is the same rounding."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(62)
+    x = (rng.standard_normal(100000) * 10.0 ** rng.uniform(-6, 3, 100000)).astype(np.float32)
+    mid = ((rng.integers(0, 1 << 15, 1000, dtype=np.uint32) << 16) | 0x8000).astype(np.uint32).view(np.float32)
+    mid = mid[np.isfinite(mid) & (np.abs(mid) < 1e30) & (np.abs(mid) > 1e-37)]   # bf16's normal range
+    for v in (x, mid):
+        np.testing.assert_array_equal(O.float_cast(v, O.PHI_BF16),
+                                      torch.from_numpy(v).bfloat16().view(torch.int16).numpy().view(np.uint16))
+        np.testing.assert_array_equal(O.bf16_round(v.astype(np.float64)), O.bf16_decode(O.bf16_encode(v)))
+    np.testing.assert_array_equal(O.bf16_encode(mid) & 1, 0)
+    np.testing.assert_array_equal(O.float_cast(x, O.PHI_FP16),
+                                  torch.from_numpy(x).half().view(torch.int16).numpy().view(np.uint16))
+
+
+# format, bound on the relative cast error: half a unit in the last place, 2^-s for
+# s significant bits (bf16 8, fp16 11, E4M3 4, E5M2 3)
+FLOAT_PHI_ERR = [(O.PHI_BF16, 2.0 ** -8), (O.PHI_FP16, 2.0 ** -11), (O.PHI_FP8_E4M3, 2.0 ** -4),
+                 (O.PHI_FP8_E5M2, 2.0 ** -3)]
+
+
+@pytest.mark.parametrize("fmt,rel", FLOAT_PHI_ERR)
+def test_float_phi_with_zero_adapter_is_rtn_near_ties_aside(fmt, rel):
+    """phi = a floating-point cast and B = 0: W_Z equals round-to-nearest quantization
+    of W0 (Python's round) except on elements within the cast's half-ulp of a
+    half-integer, where the cast may move x across or onto it; the stored value is
+    within that bound of x and never clipped inside phi."""
+    bits = 4
+    layer = O.Layer(m=64, k=128, r=4, alpha=4.0, bits=bits, phi_format=fmt)
+    spec = WL.LayerSpec("t", 64, 128, 4, 4.0, bits, 0, fmt, outlier_frac=0.01)
+    d = WL.make_layer(spec, 1, seed=63, zero_B=True, with_activations=False)
+    s0 = O.minmax_scale(d.W0, layer) * np.float32(0.5)       # half range: phi must keep |x| > p
+    x32 = np.divide(d.W0, s0[:, None].astype(np.float32), dtype=np.float32)
+    phi0 = O.downcast(d.W0, s0, layer)
+    stored = O.upcast(phi0, layer)
+    x = x32.astype(np.float64)
+    sub = 2.0 ** -10 if fmt in (O.PHI_FP8_E4M3, O.PHI_FP8_E5M2) else 0.0    # half the E4M3 subnormal step
+    assert np.all(np.abs(stored - x) <= rel * np.abs(x) + sub)
+    n, p = O.grid(bits)
+    assert np.abs(stored).max() > p                            # no clip inside phi
+    wz = O.merge(phi0, d.A, d.B, layer).astype(np.int64)
+    rtn = _rtn_python(x32, n, p)
+    near = np.abs(x - (np.floor(x) + 0.5)) <= rel * np.abs(x) + sub
+    assert np.all((wz == rtn) | near)
+
+
+def test_float_phi_rejects_zero_offsets():
+    layer = O.Layer(m=2, k=4, r=1, alpha=1.0, bits=2, phi_format=O.PHI_BF16)
+    with pytest.raises(ValueError):
+        O.downcast(np.ones((2, 4), np.float32), np.ones(2, np.float32), layer, np.zeros(2, np.float32))
+
+
+# ---------------------------------------------------------------------------
+# bf16 pre-round value (reading R20): what the R2 choice changes
+# ---------------------------------------------------------------------------
+def test_bf16_u_matches_exact_u_where_nothing_rounds():
+    """With B = 0 and a base that bf16 holds exactly (Q4.4: at most 8 significant bits;
+    phi = BF16), every bf16 rounding of R20 is exact: the codes equal R2's."""
+    for fmt in (O.PHI_QFIXED, O.PHI_BF16):
+        layer = O.Layer(m=32, k=64, r=4, alpha=4.0, bits=4, phi_format=fmt)
+        spec = WL.LayerSpec("t", 32, 64, 4, 4.0, 4, 0, fmt, outlier_frac=0.01)
+        d = WL.make_layer(spec, 1, seed=64, zero_B=True, with_activations=False)
+        s0 = O.minmax_scale(d.W0, layer)
+        phi0 = O.downcast(d.W0, s0, layer)
+        lay16 = O.Layer(32, 64, 4, 4.0, 4, 0, fmt, u_bf16=True)
+        np.testing.assert_array_equal(O.merge(phi0, d.A, d.B, lay16), O.merge(phi0, d.A, d.B, layer))
+
+
+def test_bf16_u_swallows_small_adapter_updates():
+    """A bf16 u cannot move a base value in [2, 4) by less than half its ulp (2^-7):
+    there the R20 code is round(phi^{-1}(Phi0)) whatever A B adds, while the exact u of
+    R2 lets the same update flip codes that sit on a half-integer (Q4.4 stores 2.5)."""
+    layer = O.Layer(m=1, k=8, r=1, alpha=1.0, bits=4)
+    lay16 = O.Layer(1, 8, 1, 1.0, 4, u_bf16=True)
+    P = np.array([[2.5, -2.5, 3.5, -3.5, 2.0625, 3.9375, -2.4375, 2.5]])
+    phi0 = (P * 16).astype(np.int8)
+    A = np.ones((1, 1))
+    B = np.array([[2.0 ** -8, 2.0 ** -8, -2.0 ** -8, 2.0 ** -8, 2.0 ** -9, -2.0 ** -9, 2.0 ** -8, -2.0 ** -8]])
+    np.testing.assert_array_equal(O.merge(phi0, A, B, lay16)[0], np.clip(np.rint(P[0]), -8, 7))
+    exact = O.merge(phi0, A, B, layer)[0]
+    np.testing.assert_array_equal(exact, [3, -2, 3, -3, 2, 4, -2, 2])
