@@ -37,6 +37,12 @@ KERNEL_SOURCES = {"fused_fwd": "fused_gemm.cu", "fused_dx": "fused_gemm.cu", "fu
 
 
 # --------------------------------------------------------------------------- helpers
+
+def phi_label(fmt: int, bits: int) -> str:
+    """Storage format of Phi0 (the lrqat_phi_format values) as a config label."""
+    return {0: "Q%d.%d int8" % (bits, 8 - bits), 1: f"INT-{bits} packed", 2: "BF16", 3: "FP16", 4: "FP8 E4M3",
+            5: "FP8 E5M2"}[fmt]
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -185,10 +191,12 @@ class GpuWorkload:
             z = torch.empty_like(s) if spec.asym else None   # zero offsets (asymmetric weights)
             L = LQ.Layer.from_spec(spec, z.data_ptr() if spec.asym else 0)
             LQ.range_minmax(L, W0, s)
-            if spec.phi_format == WL.PHI_QFIXED:
-                phi0 = torch.empty((spec.m, spec.k), dtype=torch.int8, device="cuda")
-            else:
+            if spec.phi_format == WL.PHI_INT_PACKED:
                 phi0 = torch.empty((spec.m, spec.k // 2), dtype=torch.uint8, device="cuda")
+            elif spec.phi_format in (WL.PHI_BF16, WL.PHI_FP16):
+                phi0 = torch.empty((spec.m, spec.k), dtype=torch.int16, device="cuda")
+            else:
+                phi0 = torch.empty((spec.m, spec.k), dtype=torch.int8, device="cuda")
             LQ.downcast(L, W0, s, phi0)
             del W0
             X = [dev(d.X_bits) for _ in range(sets)]
@@ -375,7 +383,7 @@ def run_gpu(args):
     cfg = {"workload": wl.name, "tokens": T, "layers": [f"{l.name}:{l.m}x{l.k}" for l in wl.layers],
            "r": spec0.r, "alpha": spec0.alpha, "bits": spec0.bits,
            "granularity": "per-channel" if spec0.group_size == 0 else f"g{spec0.group_size}",
-           "phi": "Q%d.%d int8" % (spec0.bits, 8 - spec0.bits) if spec0.phi_format == 0 else f"INT-{spec0.bits} packed",
+           "phi": phi_label(spec0.phi_format, spec0.bits),
            "activations": ("int8 per-token" if spec0.act_per_token else "int8 per-tensor") if spec0.act_bits == 8
            else "bf16",
            "merge": wl.merge, "parallelism": "replicas" if world > 1 else "single",

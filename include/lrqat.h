@@ -58,7 +58,17 @@ typedef enum {
   /* phi = INT-b, double-packed (b <= 4): uint8 [m, k/2]; byte j of a row holds
    * column 2j in its low nibble and column 2j+1 in its high nibble, each a
    * 4-bit two's complement integer clip(round(W0/s0), n, p). */
-  LRQAT_PHI_INT_PACKED = 1
+  LRQAT_PHI_INT_PACKED = 1,
+  /* Sec. 3's floating-point casts: Phi0 = cast(W0/s0) with W0/s0 one fp32 division,
+   * round to nearest even, no clipping inside phi; phi^{-1} is the exact value.
+   * Stored as bit patterns: uint16 [m, k] for BF16 and FP16, uint8 [m, k] for the
+   * OCP FP8 formats (E4M3: bias 7, largest finite 448; E5M2: bias 15, largest
+   * finite 57344); FP16 and FP8 casts saturate at the largest finite value.  Symmetric
+   * grids only (zero == NULL), 2 <= bits <= 8. */
+  LRQAT_PHI_BF16 = 2,
+  LRQAT_PHI_FP16 = 3,
+  LRQAT_PHI_FP8_E4M3 = 4,
+  LRQAT_PHI_FP8_E5M2 = 5
 } lrqat_phi_format;
 
 /* Settings of one layer.  W is m x k (m = out features, k = in features). */
@@ -67,7 +77,7 @@ typedef struct {
   int64_t k;
   int32_t r;          /* adapter rank, 1..64                                        */
   float alpha;        /* adapter scaling: (alpha / r) A B enters Eq. 8              */
-  int32_t bits;       /* b: 2..7 for QFIXED, 2..4 for INT_PACKED                    */
+  int32_t bits;       /* b: 2..7 for QFIXED, 2..4 for INT_PACKED, 2..8 for the casts */
   int32_t group_size; /* 0: one scale per output row (pc); else scales per g-wide
                          group along k (g128 = 128), s has shape [m, k/g]           */
   int32_t phi_format; /* lrqat_phi_format                                           */
@@ -118,7 +128,8 @@ int lrqat_range_lp(const lrqat_layer* layer, const float* W0, float p_norm, int3
  * fp32 IEEE division per element; with zero offsets phi(W0 / s0 + z0), the
  * integer offset added exactly.
  * W0: fp32 [m, k]; s0: fp32 [m] or [m, k/g];
- * Phi0 (output): int8 [m, k] (QFIXED) or uint8 [m, k/2] (INT_PACKED). */
+ * Phi0 (output): int8 [m, k] (QFIXED), uint8 [m, k/2] (INT_PACKED), uint16 [m, k]
+ * (BF16, FP16) or uint8 [m, k] (FP8) bit patterns. */
 int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0,
                    lrqat_stream_t stream);
 

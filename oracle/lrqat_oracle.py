@@ -64,8 +64,8 @@ Readings where the paper is silent (all repeated in the design notes):
      simplest choices of phi): Phi0 = cast(fl32(W0 / s0)) with round-to-nearest-even
      and no clipping inside phi (the clip of Eq. 8 follows the low-rank add); FP8 is
      the OCP E4M3 (bias 7, no infinities, largest finite 448) or E5M2 (bias 15,
-     largest finite 57344) format, and casts beyond the largest finite value
-     saturate to it.  phi^{-1} is the exact value.  Stored as bit patterns: uint16
+     largest finite 57344) format; FP16 and FP8 casts beyond the largest finite
+     value saturate to it.  phi^{-1} is the exact value.  Stored as bit patterns: uint16
      for BF16/FP16, uint8 for FP8.  Symmetric grids only.
   R20 bf16 pre-round variant (the reading that R2 rejects, kept to measure it):
      u = bf16(phi^{-1}(Phi0) + bf16((alpha/r) bf16(A B))), each product and sum
@@ -294,8 +294,8 @@ def float_cast(x: np.ndarray, fmt: int) -> np.ndarray:
     """phi for the floating-point formats: the stored bit patterns of x (R19)."""
     if fmt == PHI_BF16:
         return bf16_encode(x)
-    if fmt == PHI_FP16:
-        return np.asarray(x, dtype=np.float32).astype(np.float16).view(np.uint16)
+    if fmt == PHI_FP16:   # saturating at the largest finite fp16, 65504
+        return np.clip(np.asarray(x, dtype=np.float32), -65504.0, 65504.0).astype(np.float16).view(np.uint16)
     return fp8_encode(x, fmt)
 
 

@@ -9,6 +9,11 @@
 //   ds_partial = sum_j G * c
 // The partials of dA, dB and ds are reduced deterministically by a later kernel.
 //
+// A 16-bit base (BF16/FP16 storage) would need a 32 KB chunk in shared memory, which
+// the pipeline leaves no room for: the epilogue threads read it from global memory
+// instead (each thread 64 contiguous bytes of its own row per half chunk, issued
+// before the waits of the chunk so that the latency overlaps them).
+//
 // Roles (416 threads): warp 0 loads the epilogue operands, warp 1 issues tcgen05
 // MMAs and owns TMEM, warps 2..9 run the epilogue, warps 10..12 fill the pipeline
 // stages with TMA.  Work units (row block, column tile, token split) are
@@ -93,7 +98,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   return x;
 }
 
-template <bool PACKED, bool ZP>
+template <int FMT, bool ZP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     dw_kernel(const __grid_constant__ CUtensorMap tm_dy, const __grid_constant__ CUtensorMap tm_x,
               const __grid_constant__ CUtensorMap tm_at, const __grid_constant__ CUtensorMap tm_phi,
@@ -107,6 +112,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   auto bar = [&](int i) { return smem_u32(&bars[i]); };
+  constexpr bool PACKED = FMT == FMT_I4;
+  constexpr bool P16 = fmt_16bit(FMT);   // base read from global memory by the epilogue
   const int BN = 128 * args.nchunks;
   const uint32_t rbox = static_cast<uint32_t>(args.r16) * 128u;   // bytes of one r16-row x 64-col box
 
@@ -139,7 +146,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     // ---------------------------------------- epilogue operands (per unit/chunk)
     if (lane == 0) {
       const uint32_t ef_tx = 2u * rbox;
-      const uint32_t ec_tx = (PACKED ? 8192u : 16384u) + 2u * rbox;
+      const uint32_t ec_tx = (P16 ? 0u : PACKED ? 8192u : 16384u) + 2u * rbox;
       uint32_t it = 0, cc = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
@@ -153,7 +160,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (!(ok = wait_bounded(bar(BAR_ECEMPTY), (cc & 1u) ^ 1u, ctl, 3))) break;
           const int j0 = w.jt * BN + 128 * c;
           mbar_arrive_expect_tx(bar(BAR_ECFULL), ec_tx);
-          tma_load_2d(smem + OFF_PHI, &tm_phi, PACKED ? j0 / 2 : j0, w.ib * 128, bar(BAR_ECFULL));
+          if (!P16) tma_load_2d(smem + OFF_PHI, &tm_phi, PACKED ? j0 / 2 : j0, w.ib * 128, bar(BAR_ECFULL));
           tma_load_2d(smem + OFF_BP, &tm_b, j0, 0, bar(BAR_ECFULL));
           tma_load_2d(smem + OFF_BP + rbox, &tm_b, j0 + 64, 0, bar(BAR_ECFULL));
           ++cc;
@@ -296,6 +303,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       for (int c = 0; c < args.nchunks; ++c) {
         const int j0 = w.jt * BN + 128 * c;
+        // 16-bit base: this thread's 2 x 32 values of row i_g (columns 64 h .. 64 h + 63)
+        uint4 g16[8];
+        if (P16) {
+          const uint4* src = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(args.phi) +
+                                                            static_cast<int64_t>(i_g) * args.k + j0 + 64 * h);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) g16[e] = __ldg(src + e);
+        }
         const float s_i = args.s_ld ? args.s[static_cast<int64_t>(i_g) * args.s_ld + j0 / args.group_size]
                                     : args.s[i_g];
         // zero offset of the row (group) when the weights are asymmetric (ZP: args.zero set)
@@ -311,7 +326,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // the STE mask M = [c == cu], dU = G * (s_x s) * M and the ds partial sum G * (c - z)
         // (times s_x at the end; z = 0 for symmetric weights).
         const float gs_i = gscale * s_i;
-        const float dec_off = PACKED ? kDecodeOffsetI4 : kDecodeOffsetI8;
         const float code_n = __fmaf_rn(qp.lo, qp.inv2f, -qp.magic_c);   // n and p as exact floats
         const float code_p = __fmaf_rn(qp.hi, qp.inv2f, -qp.magic_c);
         float2 ds2 = make_float2(0.0f, 0.0f);
@@ -322,29 +336,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           tmem_ld32(tmem + lane_off + COL_G + 128 * c + jl, G);
           tmem_ld32(tmem + lane_off + COL_L + jl, Lv);
           tmem_ld_wait();
+          uint32_t raw[16];
           if (PACKED) {
-            const uint4 raw = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 32, 64));
-            decode_i4x8_raw(raw.x, v);
-            decode_i4x8_raw(raw.y, v + 8);
-            decode_i4x8_raw(raw.z, v + 16);
-            decode_i4x8_raw(raw.w, v + 24);
+            const uint4 r0 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 32, 64));
+            raw[0] = r0.x, raw[1] = r0.y, raw[2] = r0.z, raw[3] = r0.w;
+            decode16<FMT>(raw, v);
+            decode16<FMT>(raw + 2, v + 16);
+          } else if (P16) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const uint4 r0 = g16[4 * p + e];
+              raw[4 * e] = r0.x, raw[4 * e + 1] = r0.y, raw[4 * e + 2] = r0.z, raw[4 * e + 3] = r0.w;
+            }
+            decode16<FMT>(raw, v);
+            decode16<FMT>(raw + 8, v + 16);
           } else {
             const uint4 r0 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 16, 128));
             const uint4 r1 = ld_shared_v4(smem + OFF_PHI + swz_offset(row, jl / 16 + 1, 128));
-            decode_i8x4_raw(r0.x, v);
-            decode_i8x4_raw(r0.y, v + 4);
-            decode_i8x4_raw(r0.z, v + 8);
-            decode_i8x4_raw(r0.w, v + 12);
-            decode_i8x4_raw(r1.x, v + 16);
-            decode_i8x4_raw(r1.y, v + 20);
-            decode_i8x4_raw(r1.z, v + 24);
-            decode_i8x4_raw(r1.w, v + 28);
+            raw[0] = r0.x, raw[1] = r0.y, raw[2] = r0.z, raw[3] = r0.w;
+            raw[4] = r1.x, raw[5] = r1.y, raw[6] = r1.z, raw[7] = r1.w;
+            decode16<FMT>(raw, v);
+            decode16<FMT>(raw + 4, v + 16);
           }
           uint32_t du[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
             const float2 g2 = make_float2(G[2 * e], G[2 * e + 1]);
-            const float2 v2 = __fadd2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(-dec_off, -dec_off));
+            const float2 v2 = make_float2(v[2 * e], v[2 * e + 1]);
             const float2 u2 = __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
                                          v2);
             const float2 t2 = __fadd2_rn(u2, make_float2(qp.magic, qp.magic));
@@ -420,34 +438,51 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <bool PACKED, bool ZP>
+template <int FMT, bool ZP>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
   static bool configured = false;
   if (!configured) {
     cudaError_t err =
-        cudaFuncSetAttribute(dw_kernel<PACKED, ZP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+        cudaFuncSetAttribute(dw_kernel<FMT, ZP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (err != cudaSuccess) return err;
     configured = true;
   }
-  dw_kernel<PACKED, ZP><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
+  dw_kernel<FMT, ZP><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
   return cudaGetLastError();
+}
+
+template <int FMT>
+cudaError_t launch_fmt(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
+                       const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
+  if (fmt_float(FMT)) {   // zero offsets exist only with the integer formats
+    if (args.zero != nullptr) return cudaErrorInvalidValue;
+    return launch_one<FMT, false>(a, b, c, d, e, args, grid, stream);
+  }
+  return args.zero != nullptr ? launch_one<FMT, true>(a, b, c, d, e, args, grid, stream)
+                              : launch_one<FMT, false>(a, b, c, d, e, args, grid, stream);
 }
 
 }  // namespace
 
 int dw_smem_bytes(int, int) { return static_cast<int>(SMEM_BYTES); }
 
-cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
+cudaError_t launch_dw(int fmt, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
                       const CUtensorMap& tm_phi, const CUtensorMap& tm_b, const DwArgs& args, int grid,
                       cudaStream_t stream) {
   if (grid < 1 || args.r16 < 16 || args.r16 > 64 || (args.r16 & 15) || args.nchunks < 1 || args.nchunks > 2)
     return cudaErrorInvalidValue;
-  if (args.zero != nullptr)
-    return packed ? launch_one<true, true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
-                  : launch_one<false, true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
-  return packed ? launch_one<true, false>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
-                : launch_one<false, false>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+  if (fmt_16bit(fmt) && (args.phi == nullptr || (reinterpret_cast<uintptr_t>(args.phi) & 15u) || args.k % 128))
+    return cudaErrorInvalidValue;
+  switch (fmt) {
+    case FMT_Q8: return launch_fmt<FMT_Q8>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+    case FMT_I4: return launch_fmt<FMT_I4>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+    case FMT_BF16: return launch_fmt<FMT_BF16>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+    case FMT_F16: return launch_fmt<FMT_F16>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+    case FMT_E4M3: return launch_fmt<FMT_E4M3>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+    case FMT_E5M2: return launch_fmt<FMT_E5M2>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace lrqat

@@ -141,6 +141,85 @@ __global__ void downcast_packed_kernel(const float4* __restrict__ W0, const floa
   }
 }
 
+// Floating-point storage (Sec. 3, the cast choices of phi): Phi0 = cast(fl32(W0 / s0))
+// with round-to-nearest-even, no clipping inside phi, FP16 and FP8 saturating at their
+// largest finite value; 4 elements per thread.
+template <int FMT>
+__device__ __forceinline__ uint32_t pack_fp8x2(float lo, float hi) {
+  unsigned short r;
+  if (FMT == FMT_E4M3) asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  else asm("cvt.rn.satfinite.e5m2x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Saturating: values beyond 65504 (which round-to-nearest would turn into infinities)
+// are clamped to it first.
+__device__ __forceinline__ uint32_t pack_sat_f16x2(float lo, float hi) {
+  uint32_t r;
+  lo = fminf(fmaxf(lo, -65504.0f), 65504.0f);
+  hi = fminf(fmaxf(hi, -65504.0f), 65504.0f);
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+template <int FMT>
+__global__ void downcast_float_kernel(const float4* __restrict__ W0, const float* __restrict__ s0, int64_t k,
+                                      int group_size, int ngroups, void* __restrict__ out, int64_t n4) {
+  for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n4;
+       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t row = (e * 4) / k;
+    const int64_t col = (e * 4) % k;
+    const float s = s0[group_size ? row * ngroups + col / group_size : row];
+    const float4 w = W0[e];
+    const float x0 = __fdiv_rn(w.x, s), x1 = __fdiv_rn(w.y, s), x2 = __fdiv_rn(w.z, s), x3 = __fdiv_rn(w.w, s);
+    if (FMT == FMT_BF16) {
+      static_cast<uint2*>(out)[e] = make_uint2(pack_rn_bf16x2(x0, x1), pack_rn_bf16x2(x2, x3));
+    } else if (FMT == FMT_F16) {
+      static_cast<uint2*>(out)[e] = make_uint2(pack_sat_f16x2(x0, x1), pack_sat_f16x2(x2, x3));
+    } else {
+      static_cast<uint32_t*>(out)[e] = pack_fp8x2<FMT>(x0, x1) | (pack_fp8x2<FMT>(x2, x3) << 16);
+    }
+  }
+}
+
+// 4 stored values of a row -> phi^{-1}(Phi0) in the units of u_f (Eq. 7 / Eq. 8).
+__device__ __forceinline__ void decode_row4(const void* phi0, int64_t i, int64_t k, int64_t j, int fmt, float* v) {
+  if (fmt == FMT_I4) {
+    // 4 columns = 2 packed bytes (low nibble = even column)
+    const uint16_t two = *reinterpret_cast<const uint16_t*>(static_cast<const uint8_t*>(phi0) + i * (k / 2) + j / 2);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int nib = (two >> (4 * c)) & 0xF;
+      v[c] = static_cast<float>(nib >= 8 ? nib - 16 : nib);
+    }
+  } else if (fmt_16bit(fmt)) {
+    const uint2 w = *reinterpret_cast<const uint2*>(static_cast<const uint16_t*>(phi0) + i * k + j);
+    if (fmt == FMT_BF16) {
+      decode_16x2_raw<FMT_BF16>(w.x, v);
+      decode_16x2_raw<FMT_BF16>(w.y, v + 2);
+    } else {
+      decode_16x2_raw<FMT_F16>(w.x, v);
+      decode_16x2_raw<FMT_F16>(w.y, v + 2);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[c] *= kFloatRebias<FMT_F16>;
+    }
+  } else {
+    const uint32_t four = *reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(phi0) + i * k + j);
+    if (fmt == FMT_Q8) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[c] = static_cast<float>(static_cast<int8_t>((four >> (8 * c)) & 0xFF));
+    } else if (fmt == FMT_E4M3) {
+      decode_fp8x4_raw<FMT_E4M3>(four, v);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[c] *= kFloatRebias<FMT_E4M3>;
+    } else {
+      decode_fp8x4_raw<FMT_E5M2>(four, v);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[c] *= kFloatRebias<FMT_E5M2>;
+    }
+  }
+}
+
 // -------------------------------------------------------------------- merge --
 // W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p).  Each thread owns a
 // register tile of 16 rows x 4 columns: per rank index t it reads 16 values of A
@@ -152,7 +231,7 @@ constexpr int kMergeCols = 4 * kMergeThreads;   // 512 columns per block
 __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __restrict__ phi0,
                                                               const uint16_t* __restrict__ A,
                                                               const uint16_t* __restrict__ B, int64_t m, int64_t k,
-                                                              int r, int packed, int b_aligned, QuantParams q,
+                                                              int r, int fmt, int b_aligned, QuantParams q,
                                                               int8_t* __restrict__ wz) {
   __shared__ __align__(16) float As[64][kMergeRows];   // A^T tile: [t][row]
   const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kMergeRows;
@@ -195,19 +274,7 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __rest
     const int64_t i = i0 + ii;
     if (i >= m) break;
     float v[4];
-    if (packed) {
-      // 4 columns = 2 packed bytes (low nibble = even column)
-      const uint16_t two = *reinterpret_cast<const uint16_t*>(static_cast<const uint8_t*>(phi0) + i * (k / 2) + j / 2);
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int nib = (two >> (4 * c)) & 0xF;
-        v[c] = static_cast<float>(nib >= 8 ? nib - 16 : nib);
-      }
-    } else {
-      const uint32_t four = *reinterpret_cast<const uint32_t*>(static_cast<const int8_t*>(phi0) + i * k + j);
-#pragma unroll
-      for (int c = 0; c < 4; ++c) v[c] = static_cast<float>(static_cast<int8_t>((four >> (8 * c)) & 0xFF));
-    }
+    decode_row4(phi0, i, k, j, fmt, v);
     uint32_t out = 0;
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
@@ -532,6 +599,35 @@ __global__ void __launch_bounds__(256) phi_transpose_kernel(const void* __restri
     *reinterpret_cast<uint4*>(out + (j0 + 4 * c + r) * m + i0 + 16 * a) = make_uint4(o[r][0], o[r][1], o[r][2], o[r][3]);
 }
 
+// 16-bit bases: out[j][i] = Phi0[i][j] through a padded 64 x 64 shared tile (a row
+// stride of 33 words keeps the column reads free of bank conflicts).
+__global__ void __launch_bounds__(256) phi_transpose16_kernel(const uint16_t* __restrict__ in, int64_t m, int64_t k,
+                                                               uint16_t* __restrict__ out) {
+  __shared__ __align__(16) uint32_t tile[64 * 33];   // 64 rows x 64 values (+ 2 values of padding)
+  const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 64;
+  const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 64;
+  const int t = threadIdx.x;
+#pragma unroll
+  for (int x = 0; x < 2; ++x) {
+    const int u = t + 256 * x, R = u >> 3, q = u & 7;
+    const uint4 v = *reinterpret_cast<const uint4*>(in + (i0 + R) * k + j0 + 8 * q);
+    uint32_t* dst = &tile[R * 33 + 4 * q];
+    dst[0] = v.x, dst[1] = v.y, dst[2] = v.z, dst[3] = v.w;
+  }
+  __syncthreads();
+  const uint16_t* t16 = reinterpret_cast<const uint16_t*>(tile);
+#pragma unroll
+  for (int x = 0; x < 2; ++x) {
+    const int u = t + 256 * x, J = u >> 3, q = u & 7;   // output row j0 + J, values i0 + 8q .. + 7
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      o[e] = static_cast<uint32_t>(t16[(8 * q + 2 * e) * 66 + J]) |
+             (static_cast<uint32_t>(t16[(8 * q + 2 * e + 1) * 66 + J]) << 16);
+    *reinterpret_cast<uint4*>(out + (j0 + J) * m + i0 + 8 * q) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
 // ------------------------------------------------------------------- reduce --
 // One launch sums every gradient partial. Block ranges: [0, nblk_a) dA, then dB, then ds.
 // dA / dB: a block owns 32 float4 columns; warp w adds parts w, w + 8, w + 16, ... in that
@@ -669,10 +765,20 @@ cudaError_t launch_range_lp(const float* W0, int64_t m, int64_t k, int group_siz
 }
 
 cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, int64_t m, int64_t k, int group_size,
-                            int bits, int packed, void* phi0, cudaStream_t stream) {
+                            int bits, int fmt, void* phi0, cudaStream_t stream) {
   const int ngroups = group_size ? static_cast<int>(k / group_size) : 1;
   const int n = -(1 << (bits - 1)), p = (1 << (bits - 1)) - 1;
-  if (!packed) {
+  if (fmt_float(fmt)) {
+    if (z0 != nullptr) return cudaErrorInvalidValue;
+    const int64_t n4 = m * k / 4;
+    const unsigned grid = blocks_for(n4, kThreads);
+    const float4* w4 = reinterpret_cast<const float4*>(W0);
+    auto kernel = fmt == FMT_BF16   ? downcast_float_kernel<FMT_BF16>
+                  : fmt == FMT_F16  ? downcast_float_kernel<FMT_F16>
+                  : fmt == FMT_E4M3 ? downcast_float_kernel<FMT_E4M3>
+                                    : downcast_float_kernel<FMT_E5M2>;
+    kernel<<<grid, kThreads, 0, stream>>>(w4, s0, k, group_size, ngroups, phi0, n4);
+  } else if (fmt == FMT_Q8) {
     const int64_t n4 = m * k / 4;
     downcast_qfixed_kernel<<<blocks_for(n4, kThreads), kThreads, 0, stream>>>(
         reinterpret_cast<const float4*>(W0), s0, z0, k, group_size, ngroups, static_cast<float>(n),
@@ -687,11 +793,11 @@ cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, i
 }
 
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
-                         int packed, const QuantParams& q, int8_t* wz, cudaStream_t stream) {
+                         int fmt, const QuantParams& q, int8_t* wz, cudaStream_t stream) {
   if ((k % 4) != 0 || r > 64) return cudaErrorInvalidValue;
   const int b_aligned = (reinterpret_cast<uintptr_t>(B) & 7) == 0;
   dim3 grid(static_cast<unsigned>((k + kMergeCols - 1) / kMergeCols), static_cast<unsigned>((m + kMergeRows - 1) / kMergeRows));
-  merge_kernel<<<grid, kMergeThreads, 0, stream>>>(phi0, A, B, m, k, r, packed, b_aligned, q, wz);
+  merge_kernel<<<grid, kMergeThreads, 0, stream>>>(phi0, A, B, m, k, r, fmt, b_aligned, q, wz);
   return cudaGetLastError();
 }
 
@@ -730,11 +836,16 @@ cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t
   return cudaGetLastError();
 }
 
-cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int packed, int8_t* out,
-                                 cudaStream_t stream) {
+cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int fmt, void* out, cudaStream_t stream) {
   if ((m % 128) != 0 || (k % 128) != 0) return cudaErrorInvalidValue;
+  if (fmt_16bit(fmt)) {
+    dim3 grid(static_cast<unsigned>(k / 64), static_cast<unsigned>(m / 64));
+    phi_transpose16_kernel<<<grid, 256, 0, stream>>>(static_cast<const uint16_t*>(phi0), m, k,
+                                                     static_cast<uint16_t*>(out));
+    return cudaGetLastError();
+  }
   dim3 grid(static_cast<unsigned>(k / 128), static_cast<unsigned>(m / 128));
-  phi_transpose_kernel<<<grid, kThreads, 0, stream>>>(phi0, m, k, packed, out);
+  phi_transpose_kernel<<<grid, kThreads, 0, stream>>>(phi0, m, k, fmt == FMT_I4, static_cast<int8_t*>(out));
   return cudaGetLastError();
 }
 

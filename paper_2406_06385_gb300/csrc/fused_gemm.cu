@@ -7,10 +7,11 @@
 //   * token ring (2 slots): two loader warps, one per slot, bring with TMA the
 //     token operand as 2 boxes of 224 x 64 bf16 (128-byte rows, SW128); each slot
 //     also holds the bf16 operand tile W_hat of its stage;
-//   * factor ring (4 slots): one loader warp brings the stored base (128 x 64
-//     int8, SW64; packed: 128 x 32 bytes, SW32) and a 64-row slice of the second
-//     low-rank factor, only its first r16 columns (rows of 32, 64 or 128 bytes,
-//     swizzled to the row width);
+//   * factor ring (4 slots; 2 for 16-bit bases): one loader warp brings the stored
+//     base (128 x 64 bytes, SW64, for 8-bit formats; packed: 128 x 32 bytes, SW32;
+//     BF16/FP16: 128 x 128 bytes, SW128) and a 64-row slice of the second low-rank
+//     factor, only its first r16 columns (rows of 32, 64 or 128 bytes, swizzled to
+//     the row width);
 //   * the MMA warp computes the low-rank tile L = RF * SF^T (M=128, N=64, K=r
 //     rounded to 16) into a TMEM buffer, issued ahead of the main product of the
 //     previous stage so that it is ready when that product finishes;
@@ -45,7 +46,7 @@ constexpr int BN = 224;
 constexpr int NACC = 2;
 constexpr int BT = BN * NACC;                    // 448 tokens per tile
 constexpr int NT = 2;                            // token ring slots
-constexpr int NF = 4;                            // factor ring slots (power of two)
+constexpr int NF_MAX = 4;                        // factor ring slots (power of two; 2 for 16-bit bases)
 constexpr int NUM_PROD_WARPS = 16;
 constexpr int FIRST_TMA_WARP = 2 + NUM_PROD_WARPS;
 constexpr int NUM_TMA_WARPS = NT + 1;            // token loaders + factor loader
@@ -56,22 +57,31 @@ constexpr uint32_t RF_BYTES = 128 * 128;         // 128 rows x 64 rank columns (
 constexpr uint32_t TOK_HALF = BN * 128;          // 224 tokens x 64 bf16
 constexpr uint32_t TOK_BYTES = 2 * TOK_HALF;
 constexpr uint32_t W_BYTES = 128 * 128;          // 128 rows x 64 bf16
-constexpr uint32_t PHI_BYTES = 128 * 64;         // 128 rows x 64 int8 (packed: half)
 constexpr uint32_t SF_BYTES = 64 * 128;          // 64 slice rows x up to 64 rank columns (bf16)
 constexpr uint32_t TSLOT_BYTES = TOK_BYTES + W_BYTES;
-constexpr uint32_t FSLOT_BYTES = PHI_BYTES + SF_BYTES;
 constexpr uint32_t OFF_RF = 0;
 constexpr uint32_t OFF_TSLOTS = RF_BYTES;
 constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
 constexpr uint32_t TS_W = TOK_BYTES;             // offsets inside a token slot
-constexpr uint32_t FS_SF = PHI_BYTES;            // offsets inside a factor slot
-constexpr uint32_t SMEM_BYTES = OFF_FSLOTS + NF * FSLOT_BYTES + 1024;   // + 1 KB for 1024-B alignment
 
-static_assert(TSLOT_BYTES % 1024 == 0 && FSLOT_BYTES % 1024 == 0 && TOK_HALF % 1024 == 0 && TS_W % 1024 == 0 &&
-                  FS_SF % 1024 == 0 && OFF_TSLOTS % 1024 == 0 && OFF_FSLOTS % 1024 == 0,
+// Factor ring of a storage format: a 16-bit base tile (128 x 64 x 2 bytes) doubles
+// the slot, so that ring has 2 slots.
+template <int FMT>
+struct FactorRing {
+  static constexpr int NF = fmt_16bit(FMT) ? 2 : 4;
+  static constexpr uint32_t PHI_BYTES = fmt_16bit(FMT) ? 128 * 128 : 128 * 64;   // packed uses half
+  static constexpr uint32_t PHI_TX = FMT == FMT_I4 ? PHI_BYTES / 2 : PHI_BYTES;  // bytes one base tile brings
+  static constexpr uint32_t FSLOT_BYTES = PHI_BYTES + SF_BYTES;
+  static constexpr uint32_t FS_SF = PHI_BYTES;    // offset of the factor slice inside a slot
+  static constexpr uint32_t SMEM_BYTES = OFF_FSLOTS + NF * FSLOT_BYTES + 1024;   // + 1 KB for 1024-B alignment
+  static_assert(FSLOT_BYTES % 1024 == 0 && FS_SF % 1024 == 0, "swizzled tiles must start on 1024-byte boundaries");
+  static_assert(SMEM_BYTES + 512 <= 232448, "shared memory budget");
+  static_assert((NF & (NF - 1)) == 0 && NF <= NF_MAX, "factor ring index uses a mask");
+};
+
+static_assert(TSLOT_BYTES % 1024 == 0 && TOK_HALF % 1024 == 0 && TS_W % 1024 == 0 && OFF_TSLOTS % 1024 == 0 &&
+                  OFF_FSLOTS % 1024 == 0,
               "swizzled tiles must start on 1024-byte boundaries");
-static_assert(SMEM_BYTES + 512 <= 232448, "shared memory budget");
-static_assert((NF & (NF - 1)) == 0, "factor ring index uses a mask");
 static_assert(EPI_COLS % 16 == 0, "epilogue drains 16-column chunks");
 
 constexpr uint32_t TMEM_COLS = 512;
@@ -83,8 +93,8 @@ constexpr int BAR_TFULL = 0;
 constexpr int BAR_TEMPTY = BAR_TFULL + NT;       // main product of the slot finished
 constexpr int BAR_WFULL = BAR_TEMPTY + NT;       // W_hat tile of the slot written
 constexpr int BAR_FFULL = BAR_WFULL + NT;
-constexpr int BAR_FEMPTY = BAR_FFULL + NF;
-constexpr int BAR_LFULL = BAR_FEMPTY + NF;
+constexpr int BAR_FEMPTY = BAR_FFULL + NF_MAX;
+constexpr int BAR_LFULL = BAR_FEMPTY + NF_MAX;
 constexpr int BAR_LEMPTY = BAR_LFULL + 1;
 constexpr int BAR_RFFULL = BAR_LEMPTY + 1;
 constexpr int BAR_RFEMPTY = BAR_RFFULL + 1;
@@ -105,11 +115,15 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64
 // Stages are numbered globally over the CTA's tiles (gg); the contraction has an
 // even number of slices, so stage gg uses token slot gg % 2 for the (gg / 2)-th
 // time and factor slot gg % NF for the (gg / NF)-th time.
-template <int MODE, bool PACKED, bool ZP>
+template <int MODE, int FMT, bool ZP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
                       const FusedArgs args) {
+  using FR = FactorRing<FMT>;
+  constexpr int NF = FR::NF;
+  constexpr bool PACKED = FMT == FMT_I4;
+  constexpr uint32_t FSLOT_BYTES = FR::FSLOT_BYTES;
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t bars[NUM_BARS];
   __shared__ uint32_t tmem_base_s;
@@ -193,7 +207,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       prefetch_tensormap(&tm_phi);
       prefetch_tensormap(&tm_sf);
     }
-    const uint32_t tx = (PACKED ? PHI_BYTES / 2 : PHI_BYTES) + static_cast<uint32_t>(BK * 2 * args.sf_cols);
+    const uint32_t tx = FR::PHI_TX + static_cast<uint32_t>(BK * 2 * args.sf_cols);
     uint32_t gg = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
@@ -208,7 +222,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         __syncwarp();
         const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
         if (lane == 0) tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb * BM, fb);
-        if (lane == 1) tma_load_2d(fs + FS_SF, &tm_sf, 0, kk * BK, fb);
+        if (lane == 1) tma_load_2d(fs + FR::FS_SF, &tm_sf, 0, kk * BK, fb);
       }
     }
     if (lane == 0 && gg > 0) {
@@ -228,7 +242,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
       // The factor slice has rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to match).
       const uint32_t sf_swz = args.sf_cols == 16 ? SWZ_32B : args.sf_cols == 32 ? SWZ_64B : SWZ_128B;
-      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + FS_SF, 16, 16u * args.sf_cols, sf_swz);
+      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + FR::FS_SF, 16, 16u * args.sf_cols, sf_swz);
       const uint64_t d_w0 = make_sdesc(smem + OFF_TSLOTS + TS_W, 16, 1024, SWZ_128B);
       const uint64_t d_tok0 = make_sdesc(smem + OFF_TSLOTS, 16, 1024, SWZ_128B);
       uint32_t g = 0;
@@ -297,7 +311,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int row = q * 32 + lane;        // row of the tile handled by this thread
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const QuantParams qp = args.q;
-    const float dec_off = PACKED ? kDecodeOffsetI4 : kDecodeOffsetI8;
     constexpr bool zp = ZP;   // zero offsets (asymmetric weights): args.zero != nullptr
     uint32_t g = 0;
     uint32_t it = 0;
@@ -370,23 +383,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
         float v[16];
+        uint32_t raw[8];
         if (PACKED) {
-          const uint2 raw = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
-          decode_i4x8_raw(raw.x, v);
-          decode_i4x8_raw(raw.y, v + 8);
+          const uint2 r = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
+          raw[0] = r.x;
+          raw[1] = r.y;
+        } else if (fmt_16bit(FMT)) {
+          // 16 values = 32 bytes of a 128-byte row: 16-byte chunks 2c and 2c + 1 (SW128)
+          const uint4 r0 = ld_shared_v4(fs + swz_offset(row, 2 * c, 128));
+          const uint4 r1 = ld_shared_v4(fs + swz_offset(row, 2 * c + 1, 128));
+          raw[0] = r0.x, raw[1] = r0.y, raw[2] = r0.z, raw[3] = r0.w;
+          raw[4] = r1.x, raw[5] = r1.y, raw[6] = r1.z, raw[7] = r1.w;
         } else {
-          const uint4 raw = ld_shared_v4(fs + swz_offset(row, c, 64));
-          decode_i8x4_raw(raw.x, v);
-          decode_i8x4_raw(raw.y, v + 4);
-          decode_i8x4_raw(raw.z, v + 8);
-          decode_i8x4_raw(raw.w, v + 12);
+          const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
+          raw[0] = r.x, raw[1] = r.y, raw[2] = r.z, raw[3] = r.w;
         }
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float2 d = __fadd2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(-dec_off, -dec_off));
-          v[2 * e] = d.x;
-          v[2 * e + 1] = d.y;
-        }
+        decode16<FMT>(raw, v);
         ok = wait_bounded(bar(BAR_LFULL), gg & 1u, ctl, 10);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
@@ -480,48 +492,67 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <int MODE, bool PACKED, bool ZP>
+template <int MODE, int FMT, bool ZP>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const FusedArgs& args, int grid, cudaStream_t stream) {
+  constexpr uint32_t smem = FactorRing<FMT>::SMEM_BYTES;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, PACKED, ZP>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, FMT, ZP>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  fused_gemm_kernel<MODE, PACKED, ZP><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, args);
+  fused_gemm_kernel<MODE, FMT, ZP><<<grid, NUM_THREADS, smem, stream>>>(a, b, c, d, args);
   return cudaGetLastError();
 }
 
-template <bool ZP>
-cudaError_t launch_mode(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
-                        const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
-                        cudaStream_t stream) {
-  switch (mode) {
-    case FUSED_FWD_PC:
-      return packed ? launch_one<FUSED_FWD_PC, true, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
-                    : launch_one<FUSED_FWD_PC, false, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
-    case FUSED_FWD_GROUP:
-      return packed ? launch_one<FUSED_FWD_GROUP, true, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
-                    : launch_one<FUSED_FWD_GROUP, false, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
-    case FUSED_DX:
-      return launch_one<FUSED_DX, false, ZP>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
-    default:
-      return cudaErrorInvalidValue;
+// The operand of the dX product is the transposed base, never packed (the transpose
+// unpacks nibbles into bytes).  Zero offsets exist only with the integer formats.
+template <int MODE, int FMT>
+cudaError_t launch_fmt(const CUtensorMap& tm_tok, const CUtensorMap& tm_phi, const CUtensorMap& tm_rf,
+                       const CUtensorMap& tm_sf, const FusedArgs& args, int grid, cudaStream_t stream) {
+  if (fmt_float(FMT)) {
+    if (args.zero != nullptr) return cudaErrorInvalidValue;
+    return launch_one<MODE, FMT, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+  }
+  return args.zero != nullptr ? launch_one<MODE, FMT, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
+                              : launch_one<MODE, FMT, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+}
+
+template <int MODE>
+cudaError_t launch_mode(int fmt, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi, const CUtensorMap& tm_rf,
+                        const CUtensorMap& tm_sf, const FusedArgs& args, int grid, cudaStream_t stream) {
+  switch (fmt) {
+    case FMT_Q8: return launch_fmt<MODE, FMT_Q8>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FMT_I4:
+      if (MODE == FUSED_DX) return cudaErrorInvalidValue;
+      return launch_fmt<MODE, MODE == FUSED_DX ? FMT_Q8 : FMT_I4>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FMT_BF16: return launch_fmt<MODE, FMT_BF16>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FMT_F16: return launch_fmt<MODE, FMT_F16>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FMT_E4M3: return launch_fmt<MODE, FMT_E4M3>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FMT_E5M2: return launch_fmt<MODE, FMT_E5M2>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    default: return cudaErrorInvalidValue;
   }
 }
 
 }  // namespace
 
-int fused_smem_bytes() { return static_cast<int>(SMEM_BYTES); }
+int fused_smem_bytes(int fmt) {
+  return static_cast<int>(fmt_16bit(fmt) ? FactorRing<FMT_BF16>::SMEM_BYTES : FactorRing<FMT_Q8>::SMEM_BYTES);
+}
 
-cudaError_t launch_fused(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
+cudaError_t launch_fused(int mode, int fmt, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
                          const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
                          cudaStream_t stream) {
   if (grid < 1 || (args.kdim % 128) != 0 || args.kdim < 128) return cudaErrorInvalidValue;
-  return args.zero != nullptr ? launch_mode<true>(mode, packed, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
-                              : launch_mode<false>(mode, packed, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+  switch (mode) {
+    case FUSED_FWD_PC: return launch_mode<FUSED_FWD_PC>(fmt, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FUSED_FWD_GROUP:
+      return launch_mode<FUSED_FWD_GROUP>(fmt, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    case FUSED_DX: return launch_mode<FUSED_DX>(fmt, tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace lrqat

@@ -17,10 +17,11 @@ cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group
 // L^p range setting over N scaled min-max candidates (symmetric grids).
 cudaError_t launch_range_lp(const float* W0, int64_t m, int64_t k, int group_size, int bits, float p_norm, int n_cand,
                             float* s0, cudaStream_t stream);
+// fmt: a PhiFmt value (quant.cuh); zero offsets z0 only with the integer formats.
 cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, int64_t m, int64_t k, int group_size,
-                            int bits, int packed, void* phi0, cudaStream_t stream);
+                            int bits, int fmt, void* phi0, cudaStream_t stream);
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
-                         int packed, const QuantParams& q, int8_t* wz, cudaStream_t stream);
+                         int fmt, const QuantParams& q, int8_t* wz, cudaStream_t stream);
 // codes = clip(round(X / s_x), -128, 127) as bf16; optional mask bits [k][ceil(T/32)].
 // Per-token dynamic int8 quantizer: s_x[t] = max |X[t, :]| / 127, writes
 // X_hat = bf16(s_x[t] X_Z) [T, k].
@@ -33,9 +34,9 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
 cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
                                    uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad,
                                    cudaStream_t stream);
-// out[j][i] = stored integer of Phi0[i][j] (int8 raw, or sign-extended nibble), out: int8 [k, m].
-cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int packed, int8_t* out,
-                                 cudaStream_t stream);
+// out[j][i] = stored value of Phi0[i][j]: the raw byte (Q-fixed, FP8), the sign-extended
+// nibble as an int8 (packed INT-b), or the raw 16-bit pattern (BF16, FP16); out [k, m].
+cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int fmt, void* out, cudaStream_t stream);
 // Deterministic sums of the per-tile gradient partials written by the dW kernel.
 struct ReduceArgs {
   const float* dA_part; int nA;      // [nA][m][r]
@@ -90,8 +91,9 @@ struct FusedArgs {
   // Kept last: inserting it earlier shifted the fields above and slowed the producers.
   const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
 };
-int fused_smem_bytes();
-cudaError_t launch_fused(int mode, int packed, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
+int fused_smem_bytes(int fmt);
+// fmt: a PhiFmt value (quant.cuh); FMT_I4 only for the forward modes
+cudaError_t launch_fused(int mode, int fmt, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
                          const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
                          cudaStream_t stream);
 
@@ -108,9 +110,11 @@ struct DwArgs {
   int* status;
   uint64_t timeout_ns;
   const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
+  const void* phi;       // 16-bit bases only: Phi0 [m, k], read directly by the epilogue
 };
-int dw_smem_bytes(int r16, int packed);
-cudaError_t launch_dw(int packed, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
+int dw_smem_bytes(int r16, int fmt);
+// fmt: a PhiFmt value (quant.cuh)
+cudaError_t launch_dw(int fmt, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
                       const CUtensorMap& tm_phi, const CUtensorMap& tm_b, const DwArgs& args, int grid,
                       cudaStream_t stream);
 

@@ -110,6 +110,7 @@ CUtensorMapSwizzle sf_swizzle(int r16) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int frac_bits(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_QFIXED ? 8 - L.bits : 0; }
+bool phi_16bit(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_BF16 || L.phi_format == LRQAT_PHI_FP16; }
 int round16(int r) { return (r + 15) / 16 * 16; }
 
 int validate_layer(const lrqat_layer* L) {
@@ -128,6 +129,11 @@ int validate_layer(const lrqat_layer* L) {
   } else if (L->phi_format == LRQAT_PHI_INT_PACKED) {
     if (L->bits < 2 || L->bits > 4)
       return fail(LRQAT_ERR_INVALID_ARG, "INT_PACKED needs 2 <= bits <= 4 (bits=%d)", L->bits);
+  } else if (L->phi_format >= LRQAT_PHI_BF16 && L->phi_format <= LRQAT_PHI_FP8_E5M2) {
+    if (L->bits < 2 || L->bits > 8)
+      return fail(LRQAT_ERR_INVALID_ARG, "floating-point phi needs 2 <= bits <= 8 (bits=%d)", L->bits);
+    if (L->zero)
+      return fail(LRQAT_ERR_UNSUPPORTED, "zero offsets are implemented for the integer phi formats only");
   } else {
     return fail(LRQAT_ERR_INVALID_ARG, "unknown phi_format %d", L->phi_format);
   }
@@ -303,7 +309,7 @@ size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* bas
   w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
   w.at = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.m * 2));
   w.b_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.k * 2));
-  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
+  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k * (phi_16bit(L) ? 2 : 1)));
   if (L.act_bits == 8) {
     w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
     w.xmask = static_cast<uint32_t*>(c.take(static_cast<size_t>(L.k) * ((T + 31) / 32) * 4));
@@ -316,9 +322,14 @@ size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* bas
 }
 
 int phi_map(CUtensorMap* map, const lrqat_layer& L, const void* phi0, uint32_t box_cols_elems, bool dw) {
-  // Forward: slices of 64 columns (64 B int8 rows, SW64; packed 32 B rows, SW32).
-  // dW: chunks of 128 columns (128 B int8 rows, SW128; packed 64 B rows, SW64).
-  if (L.phi_format == LRQAT_PHI_QFIXED)
+  // Forward: slices of 64 columns (64 B rows of 8-bit values, SW64; packed 32 B rows,
+  // SW32; 16-bit values 128 B rows, SW128).
+  // dW: chunks of 128 columns (128 B rows, SW128; packed 64 B rows, SW64); 16-bit
+  // bases are read by the dW epilogue without the map (a 64-column box is encoded).
+  if (phi_16bit(L))
+    return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, phi0, L.k, L.m, L.k * 2, 64, 128,
+                     CU_TENSOR_MAP_SWIZZLE_128B, "Phi0 (16-bit)");
+  if (L.phi_format != LRQAT_PHI_INT_PACKED)
     return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k, L.m, L.k, box_cols_elems, 128,
                      dw ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, "Phi0");
   return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k / 2, L.m, L.k / 2, box_cols_elems / 2, 128,
@@ -428,8 +439,7 @@ int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, v
   LRQAT_CHECK_PTR(Phi0, "Phi0");
   const lrqat_layer& L = *layer;
   LRQAT_LAUNCH("downcast", 1, stream,
-               launch_downcast(W0, s0, L.zero, L.m, L.k, L.group_size, L.bits,
-                               L.phi_format == LRQAT_PHI_INT_PACKED, Phi0, stream),
+               launch_downcast(W0, s0, L.zero, L.m, L.k, L.group_size, L.bits, L.phi_format, Phi0, stream),
                "downcast launch");
   return LRQAT_OK;
 }
@@ -510,8 +520,8 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   a.timeout_ns = kWaitTimeoutNs;
   const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
   LRQAT_LAUNCH("fused_fwd", 1, stream,
-               launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, L.phi_format == LRQAT_PHI_INT_PACKED,
-                            tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+               launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, L.phi_format, tm_tok, tm_phi, tm_rf,
+                            tm_sf, a, grid, stream),
                "fused forward launch");
   return LRQAT_OK;
 }
@@ -554,11 +564,12 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   BwdWs ws;
   bwd_ws_layout(L, T, plan, workspace, &ws);
   const int r16 = round16(L.r);
-  const bool packed = L.phi_format == LRQAT_PHI_INT_PACKED;
+  // the transposed base of a packed layer holds one int8 code per byte
+  const int fmt_t = L.phi_format == LRQAT_PHI_INT_PACKED ? LRQAT_PHI_QFIXED : L.phi_format;
   LRQAT_LAUNCH("adapter_layouts", 1, stream,
                launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, ws.at, ws.b_pad, stream),
                "adapter layouts");
-  LRQAT_LAUNCH("phi_transpose", 1, stream, launch_phi_transpose(Phi0, L.m, L.k, packed, ws.phit, stream),
+  LRQAT_LAUNCH("phi_transpose", 1, stream, launch_phi_transpose(Phi0, L.m, L.k, L.phi_format, ws.phit, stream),
                "transpose Phi0");
   const uint16_t* xop = X;
   if (L.act_bits == 8 && L.act_per_token) {
@@ -578,8 +589,12 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
     LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 224,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY"));
-    LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.phit, L.m, L.k, L.m, 64, 128,
-                        CU_TENSOR_MAP_SWIZZLE_64B, "Phi0^T"));
+    if (phi_16bit(L))
+      LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT16, ws.phit, L.m, L.k, L.m * 2, 64, 128,
+                          CU_TENSOR_MAP_SWIZZLE_128B, "Phi0^T (16-bit)"));
+    else
+      LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.phit, L.m, L.k, L.m, 64, 128,
+                          CU_TENSOR_MAP_SWIZZLE_64B, "Phi0^T"));
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
     LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16), 64,
@@ -606,8 +621,8 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
     const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
-    LRQAT_LAUNCH("fused_dx", 1, stream, launch_fused(FUSED_DX, 0, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
-                 "fused dX launch");
+    LRQAT_LAUNCH("fused_dx", 1, stream,
+                 launch_fused(FUSED_DX, fmt_t, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream), "fused dX launch");
   }
   // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
   {
@@ -644,9 +659,10 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.ds_part = ws.ds_part;
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
+    a.phi = Phi0;
     const int grid = plan.units < dev->sms ? plan.units : dev->sms;
     LRQAT_LAUNCH("fused_dw", 1, stream,
-                 launch_dw(packed, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
+                 launch_dw(L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
                  "fused dW launch");
   }
   ReduceArgs ra{};
@@ -679,7 +695,7 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
   LRQAT_CHECK_PTR(W_Z, "W_Z");
   const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
   LRQAT_LAUNCH("merge", 1, stream,
-               launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format == LRQAT_PHI_INT_PACKED, q, W_Z, stream),
+               launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format, q, W_Z, stream),
                "merge launch");
   return LRQAT_OK;
 }

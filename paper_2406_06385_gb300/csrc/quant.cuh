@@ -17,6 +17,11 @@
 
 namespace lrqat {
 
+// Storage formats of Phi0 (the values of lrqat_phi_format).
+enum PhiFmt : int { FMT_Q8 = 0, FMT_I4 = 1, FMT_BF16 = 2, FMT_F16 = 3, FMT_E4M3 = 4, FMT_E5M2 = 5 };
+__host__ __device__ constexpr bool fmt_float(int f) { return f >= FMT_BF16; }
+__host__ __device__ constexpr bool fmt_16bit(int f) { return f == FMT_BF16 || f == FMT_F16; }
+
 struct QuantParams {
   float lr_scale;   // 2^f * alpha / r
   float magic;      // 1.5 * 2^(23 + f)
@@ -73,6 +78,81 @@ __device__ __forceinline__ void decode_i4x8_raw(uint32_t w, float* f) {
   for (int b = 0; b < 4; ++b) {
     f[2 * b] = __uint_as_float(__byte_perm(lo, 0x4B000000u, 0x7540u + b));
     f[2 * b + 1] = __uint_as_float(__byte_perm(hi, 0x4B000000u, 0x7540u + b));
+  }
+}
+
+// Floating-point patterns -> fp32 without conversion instructions.  The pattern sits
+// at the top of a 32-bit word; an arithmetic shift right by (8 - exponent bits) lines
+// its exponent and mantissa fields up with fp32's and keeps the sign at bit 31, the
+// mask clears the sign copies in between, and the result is the value times
+// 2^(bias - 127): kFloatRebias<FMT> = 2^(127 - bias) restores it with one exact
+// multiply (subnormal patterns become fp32 subnormals, which the multiply scales
+// exactly; the library is built without flush-to-zero).  BF16 is the top half of fp32
+// and needs nothing.  The non-finite patterns are never stored (casts saturate).
+template <int FMT> struct FloatBits;
+template <> struct FloatBits<FMT_E4M3> { static constexpr int kShift = 4; static constexpr uint32_t kMask = 0x87F00000u; };
+template <> struct FloatBits<FMT_E5M2> { static constexpr int kShift = 3; static constexpr uint32_t kMask = 0x8FE00000u; };
+template <> struct FloatBits<FMT_F16> { static constexpr int kShift = 3; static constexpr uint32_t kMask = 0x8FFFE000u; };
+template <int FMT>
+constexpr float kFloatRebias = FMT == FMT_E4M3 ? 1.329227995784916e36f    // 2^120
+                               : FMT == FMT_BF16 ? 1.0f
+                                                 : 5.192296858534828e33f;  // 2^112 (E5M2, F16)
+
+template <int FMT>
+__device__ __forceinline__ float float_bits_top(uint32_t top) {
+  return __uint_as_float(static_cast<uint32_t>(static_cast<int32_t>(top) >> FloatBits<FMT>::kShift) &
+                         FloatBits<FMT>::kMask);
+}
+
+// 4 FP8 patterns (byte b = element b) -> 4 floats, value * 2^(bias - 127).
+template <int FMT>
+__device__ __forceinline__ void decode_fp8x4_raw(uint32_t w, float* f) {
+  f[0] = float_bits_top<FMT>(__byte_perm(w, 0u, 0x0444u));
+  f[1] = float_bits_top<FMT>(__byte_perm(w, 0u, 0x1444u));
+  f[2] = float_bits_top<FMT>(__byte_perm(w, 0u, 0x2444u));
+  f[3] = float_bits_top<FMT>(__byte_perm(w, 0u, 0x3444u));
+}
+
+// 2 sixteen-bit patterns (low half = element 0) -> 2 floats (F16: value * 2^-112).
+template <int FMT>
+__device__ __forceinline__ void decode_16x2_raw(uint32_t w, float* f) {
+  if (FMT == FMT_BF16) {
+    f[0] = __uint_as_float(w << 16);
+    f[1] = __uint_as_float(w & 0xFFFF0000u);
+  } else {
+    f[0] = float_bits_top<FMT_F16>(w << 16);
+    f[1] = float_bits_top<FMT_F16>(w & 0xFFFF0000u);
+  }
+}
+
+// 16 consecutive stored values of a row -> the stored values v of Eq. 8's
+// u_f = v + 2^f (alpha/r) L, from the raw words (I4: 2 words, 8-bit formats: 4,
+// 16-bit formats: 8).
+template <int FMT>
+__device__ __forceinline__ void decode16(const uint32_t* w, float* v) {
+  if constexpr (FMT == FMT_I4) {
+    decode_i4x8_raw(w[0], v);
+    decode_i4x8_raw(w[1], v + 8);
+  } else if constexpr (FMT == FMT_Q8) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) decode_i8x4_raw(w[i], v + 4 * i);
+  } else if constexpr (fmt_16bit(FMT)) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) decode_16x2_raw<FMT>(w[i], v + 2 * i);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) decode_fp8x4_raw<FMT>(w[i], v + 4 * i);
+  }
+  if constexpr (FMT == FMT_BF16) return;
+  const float a = FMT == FMT_I4 ? 1.0f : FMT == FMT_Q8 ? 1.0f : kFloatRebias<FMT>;
+  const float b = FMT == FMT_I4 ? -kDecodeOffsetI4 : FMT == FMT_Q8 ? -kDecodeOffsetI8 : 0.0f;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    float2 d;
+    if (fmt_float(FMT)) d = __fmul2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(a, a));
+    else d = __fadd2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(b, b));
+    v[2 * e] = d.x;
+    v[2 * e + 1] = d.y;
   }
 }
 

@@ -16,6 +16,10 @@ LIB_PATH = os.path.join(PKG, "_lib", "liblrqat.so")
 
 PHI_QFIXED = 0
 PHI_INT_PACKED = 1
+PHI_BF16 = 2
+PHI_FP16 = 3
+PHI_FP8_E4M3 = 4
+PHI_FP8_E5M2 = 5
 
 STATUS = {0: "LRQAT_OK", -1: "LRQAT_ERR_INVALID_ARG", -2: "LRQAT_ERR_UNSUPPORTED", -3: "LRQAT_ERR_ALIGNMENT",
           -4: "LRQAT_ERR_WORKSPACE", -5: "LRQAT_ERR_CUDA", -6: "LRQAT_ERR_TIMEOUT"}

@@ -37,6 +37,25 @@ def oracle_layer(spec):
                    spec.act_per_token)
 
 
+PHI_HOST_DTYPE = {WL.PHI_QFIXED: np.int8, WL.PHI_INT_PACKED: np.uint8, WL.PHI_BF16: np.uint16,
+                  WL.PHI_FP16: np.uint16, WL.PHI_FP8_E4M3: np.uint8, WL.PHI_FP8_E5M2: np.uint8}
+
+
+def phi_buffer(spec):
+    """Device buffer of Phi0 in the layer's storage format (see lrqat_phi_format)."""
+    t = torch()
+    if spec.phi_format == WL.PHI_INT_PACKED:
+        return t.empty((spec.m, spec.k // 2), dtype=t.uint8, device="cuda")
+    if spec.phi_format in (WL.PHI_BF16, WL.PHI_FP16):
+        return t.empty((spec.m, spec.k), dtype=t.int16, device="cuda")
+    return t.empty((spec.m, spec.k), dtype=t.int8 if spec.phi_format == WL.PHI_QFIXED else t.uint8, device="cuda")
+
+
+def phi_host(phi0, spec) -> np.ndarray:
+    """Device Phi0 -> host array in the oracle's representation of the format."""
+    return phi0.cpu().numpy().view(PHI_HOST_DTYPE[spec.phi_format])
+
+
 class DeviceLayer:
     """One layer's frozen base and adapters on the device, prepared with the
     library's own range setting and downcast."""
@@ -52,10 +71,7 @@ class DeviceLayer:
         self.z = t.empty_like(self.s0) if spec.asym else None
         self.layer = LQ.Layer.from_spec(spec, self.z.data_ptr() if spec.asym else 0)
         LQ.range_minmax(self.layer, self.W0, self.s0)
-        if spec.phi_format == WL.PHI_QFIXED:
-            self.phi0 = t.empty((spec.m, spec.k), dtype=t.int8, device="cuda")
-        else:
-            self.phi0 = t.empty((spec.m, spec.k // 2), dtype=t.uint8, device="cuda")
+        self.phi0 = phi_buffer(spec)
         LQ.downcast(self.layer, self.W0, self.s0, self.phi0)
         self.s = (self.s0 * s_scale).contiguous()
         self.A = to_dev(data.A_bits)

@@ -7,7 +7,7 @@ import oracle as O
 from paper_2406_06385_gb300 import lrqat as LQ
 from paper_2406_06385_gb300 import workloads as WL
 
-from gpu_util import DeviceLayer, oracle_layer, to_dev, torch
+from gpu_util import DeviceLayer, oracle_layer, phi_buffer, phi_host, to_dev, torch
 
 pytestmark = pytest.mark.gpu
 
@@ -20,6 +20,11 @@ CASES = [
     ("int4_packed_g256", 128, 512, 8, 4, 256, WL.PHI_INT_PACKED, 0.1, 0.1),
     ("q26_clip_heavy", 128, 256, 64, 2, 0, WL.PHI_QFIXED, 1.0, 1.0),
     ("q71", 128, 128, 1, 7, 0, WL.PHI_QFIXED, 0.05, 0.05),
+    ("bf16_pc", 256, 512, 8, 4, 0, WL.PHI_BF16, 0.05, 0.05),
+    ("fp16_g128_w3", 128, 640, 16, 3, 128, WL.PHI_FP16, 0.1, 0.1),
+    ("fp8_e4m3_pc", 384, 256, 32, 4, 0, WL.PHI_FP8_E4M3, 0.1, 0.1),
+    ("fp8_e5m2_g128_w2", 128, 512, 8, 2, 128, WL.PHI_FP8_E5M2, 0.3, 0.3),
+    ("bf16_w8", 128, 256, 4, 8, 0, WL.PHI_BF16, 0.05, 0.05),
 ]
 
 
@@ -51,7 +56,7 @@ def test_merge_matches_oracle_codes(case):
     LQ.merge(dl.layer, dl.phi0, dl.A, dl.B, wz)
     LQ.get_device_status()
     L = oracle_layer(spec)
-    phi_ref = dl.phi0.cpu().numpy().view(np.int8 if spec.phi_format == WL.PHI_QFIXED else np.uint8)
+    phi_ref = phi_host(dl.phi0, spec)
     ones = np.ones((spec.m, spec.k // spec.group_size) if spec.group_size else (spec.m,))
     fq = O.fake_quant_weight(phi_ref, ones, data.A, data.B, L)
     ref = fq["c"].astype(np.int8)
@@ -146,3 +151,31 @@ def test_lp_range_matches_oracle(case):
     assert np.all(got[1] == cands[1, :, 0]) and np.all(cands[1, :, 0] == np.float32(1.0 / n_cand))
     if n_cand > 1:
         assert len(np.unique(best_ref[2:])) > 1    # the search is not stuck at one end
+
+
+@pytest.mark.parametrize("phi", [WL.PHI_FP8_E4M3, WL.PHI_FP8_E5M2, WL.PHI_BF16, WL.PHI_FP16])
+def test_float_downcast_saturates_and_keeps_signed_zeros(phi):
+    """Scales far below min-max push W0 / s0 beyond the FP8 and FP16 ranges: those casts
+    saturate at the largest finite value; huge scales round small values to signed zeros
+    (bf16 keeps them).  Bit for bit against the oracle."""
+    t = torch()
+    spec = WL.LayerSpec("sat", 128, 256, 4, 4.0, 4, 0, phi, outlier_frac=1e-3)
+    data = WL.make_layer(spec, 1, seed=25, with_activations=False)
+    L = oracle_layer(spec)
+    lay = LQ.Layer.from_spec(spec)
+    W0 = to_dev(data.W0)
+    s_host = O.minmax_scale(data.W0, L).copy()
+    s_host[: 64] *= np.float32(1e-4)       # |W0 / s| up to ~7e4: beyond E4M3 and E5M2
+    s_host[64:] *= np.float32(1e12)        # |W0 / s| below every subnormal: signed zeros
+    s_dev = t.from_numpy(s_host).cuda()
+    phi0 = phi_buffer(spec)
+    LQ.downcast(lay, W0, s_dev, phi0)
+    LQ.get_device_status()
+    ref = O.downcast(data.W0, s_host, L)
+    np.testing.assert_array_equal(phi_host(phi0, spec), ref)
+    if phi in (WL.PHI_FP8_E4M3, WL.PHI_FP8_E5M2):
+        vmax = 448.0 if phi == WL.PHI_FP8_E4M3 else 57344.0
+        assert np.abs(O.upcast(ref, L)[:64]).max() == vmax
+    if phi != WL.PHI_BF16:
+        small = O.upcast(ref, L)[64:]
+        assert np.any((small == 0) & np.signbit(small)) and np.any((small == 0) & ~np.signbit(small))

@@ -13,7 +13,7 @@ import oracle as O
 from paper_2406_06385_gb300 import lrqat as LQ
 from paper_2406_06385_gb300 import workloads as WL
 
-from gpu_util import DeviceLayer, bits_to_f32, oracle_layer, to_dev, torch
+from gpu_util import DeviceLayer, bits_to_f32, oracle_layer, phi_host, to_dev, torch
 
 pytestmark = pytest.mark.gpu
 
@@ -59,6 +59,13 @@ CASES = [
     ("q44_pc_a8_token", spec_of("p", 256, 512, 32, act=8, per_token=True, a_std=0.2, b_std=0.2), 301),
     ("int3_packed_g128_a8_token", spec_of("q", 128, 384, 16, bits=3, group=128, phi=WL.PHI_INT_PACKED, act=8,
                                           per_token=True, a_std=0.3, b_std=0.3), 97),
+    # floating-point bases (the cast choices of phi, Sec. 3)
+    ("bf16_pc", spec_of("r", 256, 512, 32, phi=WL.PHI_BF16, a_std=0.2, b_std=0.2), 300),
+    ("fp16_g128_w3", spec_of("s", 128, 384, 16, bits=3, group=128, phi=WL.PHI_FP16, a_std=0.2, b_std=0.2), 130),
+    ("fp8_e4m3_pc_a8_token", spec_of("t", 256, 256, 16, phi=WL.PHI_FP8_E4M3, act=8, per_token=True, a_std=0.2,
+                                     b_std=0.2), 200),
+    ("fp8_e5m2_w2_clip", spec_of("u", 128, 512, 32, bits=2, phi=WL.PHI_FP8_E5M2, a_std=1.0, b_std=1.0), 97),
+    ("bf16_w8_g128", spec_of("v", 128, 256, 8, bits=8, group=128, phi=WL.PHI_BF16, a_std=0.3, b_std=0.3), 64),
 ]
 
 
@@ -86,9 +93,9 @@ def _run(spec, T, seed=0, s_scale=1.0, sx_factor=1.0, zero_B=False):
     # oracle side: its own range setting and downcast from the same W0
     OL = oracle_layer(spec)
     s0, z0, phi0 = oracle_base(data, OL)
-    if spec.asym:   # the device's zero offsets and base equal the oracle's exactly
+    if spec.asym:   # the device's zero offsets equal the oracle's exactly
         np.testing.assert_array_equal(dl.z.cpu().numpy().reshape(z0.shape), z0)
-        np.testing.assert_array_equal(dl.phi0.cpu().numpy(), phi0)
+    np.testing.assert_array_equal(phi_host(dl.phi0, spec), phi0)   # and so does the stored base
     s = (s0 * np.float32(s_scale)).astype(np.float32)
     Y_ref = O.linear_fwd(data.X, phi0, s, data.A, data.B, OL, s_x_host, z0)
     g = O.linear_bwd(data.dY, data.X, phi0, s, data.A, data.B, OL, s_x_host, z0)
@@ -150,6 +157,10 @@ CODE_CASES = [
     ("int2_asym_q26", spec_of("c5", 128, 256, 16, bits=2, asym=True, shift=0.03, a_std=0.2, b_std=0.2)),
     ("int2_asym_packed_g128", spec_of("c6", 128, 256, 8, bits=2, group=128, phi=WL.PHI_INT_PACKED, asym=True,
                                       shift=0.03, a_std=0.3, b_std=0.3)),
+    ("bf16_pc", spec_of("c7", 256, 256, 32, phi=WL.PHI_BF16, a_std=0.1, b_std=0.1)),
+    ("fp16_g128", spec_of("c8", 128, 256, 16, group=128, phi=WL.PHI_FP16, a_std=0.1, b_std=0.1)),
+    ("fp8_e4m3_w3", spec_of("c9", 128, 384, 16, bits=3, phi=WL.PHI_FP8_E4M3, a_std=0.2, b_std=0.2)),
+    ("fp8_e5m2", spec_of("c10", 128, 256, 8, phi=WL.PHI_FP8_E5M2, a_std=0.3, b_std=0.3)),
 ]
 
 
@@ -190,5 +201,5 @@ def test_fused_codes_bit_exact(cid, spec, zero_B):
     for name, c in (("fwd", c_fwd), ("dX", c_dx)):
         bad = (c != fq["cz"]) & ~exempt
         assert bad.sum() == 0, f"{name}: {bad.sum()} code mismatches (near-ties exempt: {exempt.sum()})"
-    if zero_B and spec.phi_format == WL.PHI_QFIXED:
+    if zero_B and spec.phi_format in (WL.PHI_QFIXED, WL.PHI_BF16, WL.PHI_FP16, WL.PHI_FP8_E4M3):
         assert (np.abs(fq["u"] - np.floor(fq["u"]) - 0.5) == 0).sum() > 0   # exact ties were exercised

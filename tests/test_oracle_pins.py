@@ -632,8 +632,11 @@ def test_bf16_and_fp16_casts_against_torch():
                                       torch.from_numpy(v).bfloat16().view(torch.int16).numpy().view(np.uint16))
         np.testing.assert_array_equal(O.bf16_round(v.astype(np.float64)), O.bf16_decode(O.bf16_encode(v)))
     np.testing.assert_array_equal(O.bf16_encode(mid) & 1, 0)
-    np.testing.assert_array_equal(O.float_cast(x, O.PHI_FP16),
-                                  torch.from_numpy(x).half().view(torch.int16).numpy().view(np.uint16))
+    x16 = x[np.abs(x) <= 65504.0]
+    np.testing.assert_array_equal(O.float_cast(x16, O.PHI_FP16),
+                                  torch.from_numpy(x16).half().view(torch.int16).numpy().view(np.uint16))
+    sat = O.float_value(O.float_cast(np.float32([7e4, -1e30]), O.PHI_FP16), O.PHI_FP16)
+    np.testing.assert_array_equal(sat, [65504.0, -65504.0])
 
 
 # format, bound on the relative cast error: half a unit in the last place, 2^-s for
