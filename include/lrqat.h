@@ -100,6 +100,13 @@ typedef struct {
                          (s_x may then be NULL).  It never clips, so dX
                          has no activation mask; the GEMMs take X_hat =
                          bf16(s_x[t] X_Z) as their token operand.                    */
+  int32_t u_bf16;     /* 0: the pre-round value u = phi^{-1}(Phi0) + (alpha/r) A B of
+                         Eq. 8 is formed in fp32.  1: in bf16, as Sec. 3 assumes for
+                         "the rest of the computation": u = bf16(phi^{-1}(Phi0) +
+                         bf16((alpha/r) bf16(A B))) (A B accumulated in fp32 first).
+                         Needs alpha/r a power of two (then the product is exact), a
+                         base exact in bf16 (not FP16) and zero == NULL
+                         (LRQAT_ERR_UNSUPPORTED otherwise).                           */
 } lrqat_layer;
 
 /* Human-readable reason of the last non-OK status returned on this thread. */

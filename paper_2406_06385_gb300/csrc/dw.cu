@@ -98,7 +98,8 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   return x;
 }
 
-template <int FMT, bool ZP>
+// UB: pre-round value in bf16 (u_bf16x2) instead of one fp32 FMA.
+template <int FMT, bool ZP, bool UB>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     dw_kernel(const __grid_constant__ CUtensorMap tm_dy, const __grid_constant__ CUtensorMap tm_x,
               const __grid_constant__ CUtensorMap tm_at, const __grid_constant__ CUtensorMap tm_phi,
@@ -291,6 +292,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int row = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const QuantParams qp = args.q;
+    const uint32_t lr2 = pack_rn_bf16x2(qp.lr_scale, qp.lr_scale);   // exact: a power of two when UB
     const int nb = args.k / 128;
     const float gscale = args.s_x != nullptr ? *args.s_x : 1.0f;
     const int half_cols = args.r16 / 2;   // dA / dB^T columns read by this warp half
@@ -363,8 +365,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int e = 0; e < 16; ++e) {
             const float2 g2 = make_float2(G[2 * e], G[2 * e + 1]);
             const float2 v2 = make_float2(v[2 * e], v[2 * e + 1]);
-            const float2 u2 = __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
-                                         v2);
+            const float2 u2 = UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v2.x, v2.y, lr2)
+                                 : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]),
+                                              make_float2(qp.lr_scale, qp.lr_scale), v2);
             const float2 t2 = __fadd2_rn(u2, make_float2(qp.magic, qp.magic));
             const float2 cu = __ffma2_rn(t2, make_float2(qp.inv2f, qp.inv2f), make_float2(-qp.magic_c, -qp.magic_c));
             const float2 cc = make_float2(fminf(fmaxf(cu.x, code_n), code_p), fminf(fmaxf(cu.y, code_n), code_p));
@@ -438,29 +441,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <int FMT, bool ZP>
+template <int FMT, bool ZP, bool UB>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
   static bool configured = false;
   if (!configured) {
     cudaError_t err =
-        cudaFuncSetAttribute(dw_kernel<FMT, ZP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+        cudaFuncSetAttribute(dw_kernel<FMT, ZP, UB>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (err != cudaSuccess) return err;
     configured = true;
   }
-  dw_kernel<FMT, ZP><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
+  dw_kernel<FMT, ZP, UB><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
   return cudaGetLastError();
 }
 
 template <int FMT>
 cudaError_t launch_fmt(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
+  if (args.u_bf16) {   // bf16 pre-round value: no zero offsets, bases exact in bf16
+    if (FMT == FMT_F16 || args.zero != nullptr) return cudaErrorInvalidValue;
+    return launch_one<FMT == FMT_F16 ? FMT_Q8 : FMT, false, true>(a, b, c, d, e, args, grid, stream);
+  }
   if (fmt_float(FMT)) {   // zero offsets exist only with the integer formats
     if (args.zero != nullptr) return cudaErrorInvalidValue;
-    return launch_one<FMT, false>(a, b, c, d, e, args, grid, stream);
+    return launch_one<FMT, false, false>(a, b, c, d, e, args, grid, stream);
   }
-  return args.zero != nullptr ? launch_one<FMT, true>(a, b, c, d, e, args, grid, stream)
-                              : launch_one<FMT, false>(a, b, c, d, e, args, grid, stream);
+  return args.zero != nullptr ? launch_one<FMT, true, false>(a, b, c, d, e, args, grid, stream)
+                              : launch_one<FMT, false, false>(a, b, c, d, e, args, grid, stream);
 }
 
 }  // namespace

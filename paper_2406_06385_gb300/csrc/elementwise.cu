@@ -231,7 +231,7 @@ constexpr int kMergeCols = 4 * kMergeThreads;   // 512 columns per block
 __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __restrict__ phi0,
                                                               const uint16_t* __restrict__ A,
                                                               const uint16_t* __restrict__ B, int64_t m, int64_t k,
-                                                              int r, int fmt, int b_aligned, QuantParams q,
+                                                              int r, int fmt, int ub, int b_aligned, QuantParams q,
                                                               int8_t* __restrict__ wz) {
   __shared__ __align__(16) float As[64][kMergeRows];   // A^T tile: [t][row]
   const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kMergeRows;
@@ -275,6 +275,18 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __rest
     if (i >= m) break;
     float v[4];
     decode_row4(phi0, i, k, j, fmt, v);
+    if (ub) {
+      // bf16 pre-round value: u_f = bf16(v + bf16(lr_f bf16(L))); the code of an exact u_f
+      const uint32_t lr2 = pack_rn_bf16x2(q.lr_scale, q.lr_scale);
+#pragma unroll
+      for (int c = 0; c < 4; c += 2) {
+        const float2 u = u_bf16x2(acc[ii][c], acc[ii][c + 1], v[c], v[c + 1], lr2);
+        v[c] = u.x;
+        v[c + 1] = u.y;
+        acc[ii][c] = 0.0f;
+        acc[ii][c + 1] = 0.0f;
+      }
+    }
     uint32_t out = 0;
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
@@ -793,11 +805,11 @@ cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, i
 }
 
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
-                         int fmt, const QuantParams& q, int8_t* wz, cudaStream_t stream) {
+                         int fmt, int u_bf16, const QuantParams& q, int8_t* wz, cudaStream_t stream) {
   if ((k % 4) != 0 || r > 64) return cudaErrorInvalidValue;
   const int b_aligned = (reinterpret_cast<uintptr_t>(B) & 7) == 0;
   dim3 grid(static_cast<unsigned>((k + kMergeCols - 1) / kMergeCols), static_cast<unsigned>((m + kMergeRows - 1) / kMergeRows));
-  merge_kernel<<<grid, kMergeThreads, 0, stream>>>(phi0, A, B, m, k, r, fmt, b_aligned, q, wz);
+  merge_kernel<<<grid, kMergeThreads, 0, stream>>>(phi0, A, B, m, k, r, fmt, u_bf16, b_aligned, q, wz);
   return cudaGetLastError();
 }
 

@@ -115,7 +115,8 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64
 // Stages are numbered globally over the CTA's tiles (gg); the contraction has an
 // even number of slices, so stage gg uses token slot gg % 2 for the (gg / 2)-th
 // time and factor slot gg % NF for the (gg / NF)-th time.
-template <int MODE, int FMT, bool ZP>
+// UB: pre-round value in bf16 (u_bf16x2) instead of one fp32 FMA.
+template <int MODE, int FMT, bool ZP, bool UB>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
@@ -311,6 +312,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int row = q * 32 + lane;        // row of the tile handled by this thread
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const QuantParams qp = args.q;
+    const uint32_t lr2 = pack_rn_bf16x2(qp.lr_scale, qp.lr_scale);   // exact: a power of two when UB
     constexpr bool zp = ZP;   // zero offsets (asymmetric weights): args.zero != nullptr
     uint32_t g = 0;
     uint32_t it = 0;
@@ -411,8 +413,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t w[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float2 u = __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
-                                      make_float2(v[2 * e], v[2 * e + 1]));
+          const float2 u =
+              UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
+                 : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
+                              make_float2(v[2 * e], v[2 * e + 1]));
           const float2 t2 = __fadd2_rn(u, make_float2(qp.magic, qp.magic));
           uint32_t cw = codes_bf16x2(t2, qp);
           if (zp) cw = sub_bf16x2(cw, zw[e]);   // c - z, exact small integers
@@ -492,32 +496,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <int MODE, int FMT, bool ZP>
+template <int MODE, int FMT, bool ZP, bool UB>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const FusedArgs& args, int grid, cudaStream_t stream) {
   constexpr uint32_t smem = FactorRing<FMT>::SMEM_BYTES;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, FMT, ZP>,
+    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, FMT, ZP, UB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  fused_gemm_kernel<MODE, FMT, ZP><<<grid, NUM_THREADS, smem, stream>>>(a, b, c, d, args);
+  fused_gemm_kernel<MODE, FMT, ZP, UB><<<grid, NUM_THREADS, smem, stream>>>(a, b, c, d, args);
   return cudaGetLastError();
 }
 
 // The operand of the dX product is the transposed base, never packed (the transpose
-// unpacks nibbles into bytes).  Zero offsets exist only with the integer formats.
+// unpacks nibbles into bytes).  Zero offsets exist only with the integer formats; the
+// bf16 pre-round value only without them and with bases exact in bf16 (not FP16).
 template <int MODE, int FMT>
 cudaError_t launch_fmt(const CUtensorMap& tm_tok, const CUtensorMap& tm_phi, const CUtensorMap& tm_rf,
                        const CUtensorMap& tm_sf, const FusedArgs& args, int grid, cudaStream_t stream) {
+  if (args.u_bf16) {
+    if (FMT == FMT_F16 || args.zero != nullptr) return cudaErrorInvalidValue;
+    return launch_one<MODE, FMT == FMT_F16 ? FMT_Q8 : FMT, false, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid,
+                                                                          stream);
+  }
   if (fmt_float(FMT)) {
     if (args.zero != nullptr) return cudaErrorInvalidValue;
-    return launch_one<MODE, FMT, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+    return launch_one<MODE, FMT, false, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
   }
-  return args.zero != nullptr ? launch_one<MODE, FMT, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
-                              : launch_one<MODE, FMT, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+  return args.zero != nullptr ? launch_one<MODE, FMT, true, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
+                              : launch_one<MODE, FMT, false, false>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
 }
 
 template <int MODE>

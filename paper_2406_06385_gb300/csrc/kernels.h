@@ -21,7 +21,7 @@ cudaError_t launch_range_lp(const float* W0, int64_t m, int64_t k, int group_siz
 cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, int64_t m, int64_t k, int group_size,
                             int bits, int fmt, void* phi0, cudaStream_t stream);
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
-                         int fmt, const QuantParams& q, int8_t* wz, cudaStream_t stream);
+                         int fmt, int u_bf16, const QuantParams& q, int8_t* wz, cudaStream_t stream);
 // codes = clip(round(X / s_x), -128, 127) as bf16; optional mask bits [k][ceil(T/32)].
 // Per-token dynamic int8 quantizer: s_x[t] = max |X[t, :]| / 127, writes
 // X_hat = bf16(s_x[t] X_Z) [T, k].
@@ -90,6 +90,7 @@ struct FusedArgs {
   uint64_t timeout_ns;
   // Kept last: inserting it earlier shifted the fields above and slowed the producers.
   const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
+  int32_t u_bf16;        // pre-round value in bf16 (lrqat_layer.u_bf16)
 };
 int fused_smem_bytes(int fmt);
 // fmt: a PhiFmt value (quant.cuh); FMT_I4 only for the forward modes
@@ -111,6 +112,7 @@ struct DwArgs {
   uint64_t timeout_ns;
   const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
   const void* phi;       // 16-bit bases only: Phi0 [m, k], read directly by the epilogue
+  int32_t u_bf16;        // pre-round value in bf16 (lrqat_layer.u_bf16)
 };
 int dw_smem_bytes(int r16, int fmt);
 // fmt: a PhiFmt value (quant.cuh)

@@ -145,6 +145,15 @@ int validate_layer(const lrqat_layer* L) {
   if (L->zero && !aligned16(L->zero)) return fail(LRQAT_ERR_ALIGNMENT, "zero (offsets) is not 16-byte aligned");
   if (L->act_per_token != 0 && (L->act_per_token != 1 || L->act_bits != 8))
     return fail(LRQAT_ERR_INVALID_ARG, "act_per_token must be 0, or 1 with act_bits == 8");
+  if (L->u_bf16 != 0) {
+    if (L->u_bf16 != 1) return fail(LRQAT_ERR_INVALID_ARG, "u_bf16 must be 0 or 1");
+    if (L->phi_format == LRQAT_PHI_FP16)
+      return fail(LRQAT_ERR_UNSUPPORTED, "u_bf16 needs a base exact in bf16 (not FP16)");
+    if (L->zero) return fail(LRQAT_ERR_UNSUPPORTED, "u_bf16 is implemented for symmetric grids only");
+    int e = 0;
+    if (!(L->alpha > 0.0f) || std::frexp(static_cast<double>(L->alpha) / L->r, &e) != 0.5)
+      return fail(LRQAT_ERR_UNSUPPORTED, "u_bf16 needs alpha / r to be a power of two");
+  }
   return LRQAT_OK;
 }
 
@@ -509,6 +518,7 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   a.q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
   a.s = s;
   a.zero = L.zero;
+  a.u_bf16 = L.u_bf16;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
   a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;
@@ -611,6 +621,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.q = q;
     a.s = s;
     a.zero = L.zero;
+    a.u_bf16 = L.u_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;
@@ -651,6 +662,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.q = q;
     a.s = s;
     a.zero = L.zero;
+    a.u_bf16 = L.u_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;   // per token: folded into X_hat
@@ -695,7 +707,7 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
   LRQAT_CHECK_PTR(W_Z, "W_Z");
   const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
   LRQAT_LAUNCH("merge", 1, stream,
-               launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format, q, W_Z, stream),
+               launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format, L.u_bf16, q, W_Z, stream),
                "merge launch");
   return LRQAT_OK;
 }

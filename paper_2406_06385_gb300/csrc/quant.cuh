@@ -191,6 +191,19 @@ __device__ __forceinline__ uint32_t pack_rn_bf16x2(float lo, float hi) {
   return r;
 }
 
+// Pre-round value in bf16 (the bf16 reading of Sec. 3's computation) for two
+// elements, in the units of u_f: u_f = bf16(v + bf16(lr_f bf16(L))) with lr_f =
+// 2^f alpha / r a power of two, so the product is exact and one bf16 fma rounds
+// exactly as the definition does; v is exact in bf16 (an integer |v| <= 128, or a
+// BF16, FP8 or nibble value), its fp32 low half zero.
+__device__ __forceinline__ float2 u_bf16x2(float L0, float L1, float v0, float v1, uint32_t lr2) {
+  const uint32_t lb = pack_rn_bf16x2(L0, L1);
+  const uint32_t vb = __byte_perm(__float_as_uint(v0), __float_as_uint(v1), 0x7632u);
+  uint32_t u;
+  asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(u) : "r"(lb), "r"(lr2), "r"(vb));
+  return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
+}
+
 // Elementwise bf16x2 difference, rounded to nearest even (exact for the small
 // integers it is used on).
 __device__ __forceinline__ uint32_t sub_bf16x2(uint32_t a, uint32_t b) {

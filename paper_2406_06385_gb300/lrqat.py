@@ -35,13 +35,14 @@ class Layer(ctypes.Structure):
     """Mirror of the C struct lrqat_layer."""
     _fields_ = [("m", ctypes.c_int64), ("k", ctypes.c_int64), ("r", ctypes.c_int32), ("alpha", ctypes.c_float),
                 ("bits", ctypes.c_int32), ("group_size", ctypes.c_int32), ("phi_format", ctypes.c_int32),
-                ("act_bits", ctypes.c_int32), ("zero", ctypes.c_void_p), ("act_per_token", ctypes.c_int32)]
+                ("act_bits", ctypes.c_int32), ("zero", ctypes.c_void_p), ("act_per_token", ctypes.c_int32),
+                ("u_bf16", ctypes.c_int32)]
 
     @classmethod
     def from_spec(cls, spec, zero: int = 0) -> "Layer":
         """`zero`: device address of the zero offsets (asymmetric weights), 0 for none."""
         return cls(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits,
-                   zero or None, int(getattr(spec, "act_per_token", False)))
+                   zero or None, int(getattr(spec, "act_per_token", False)), int(getattr(spec, "u_bf16", False)))
 
 
 class AdamW(ctypes.Structure):

@@ -63,6 +63,7 @@ class LayerSpec:
     asym: bool = False     # asymmetric weights: zero offsets z (the INT2 runs of the paper)
     w_row_shift: float = 0.0   # each row of W0 shifted by U(-w_row_shift, w_row_shift)
     act_per_token: bool = False   # with act_bits 8: dynamic per-token scales (else per tensor)
+    u_bf16: bool = False   # pre-round value formed in bf16 instead of fp32
 
 
 @dataclass(frozen=True)
@@ -126,6 +127,10 @@ def workload(name: str) -> Workload:
     if name == "llama2_7b_attn_w4a8":
         spec = _llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=PHI_QFIXED, act_bits=8)
         return Workload(name, 8192, [replace(spec, act_per_token=True)])
+    if name == "llama2_7b_attn_ubf16":
+        # the bench layer with its pre-round value formed in bf16 (the bf16 reading of Sec. 3)
+        spec = _llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=PHI_QFIXED)
+        return Workload(name, 8192, [replace(spec, u_bf16=True)])
     if name.startswith("llama2_7b_attn_phi_"):
         # the same 4096 x 4096 W4 per-channel layer with a floating-point base (Table 2 ablation)
         fmt = {"bf16": PHI_BF16, "fp16": PHI_FP16, "fp8": PHI_FP8_E4M3, "fp8e5m2": PHI_FP8_E5M2}[name[19:]]
@@ -135,7 +140,7 @@ def workload(name: str) -> Workload:
 
 WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer", "llama2_7b_attn_int2",
              "llama2_7b_attn_w4a8", "llama2_7b_attn_phi_bf16", "llama2_7b_attn_phi_fp16", "llama2_7b_attn_phi_fp8",
-             "llama2_7b_attn_phi_fp8e5m2")
+             "llama2_7b_attn_phi_fp8e5m2", "llama2_7b_attn_ubf16")
 
 
 @dataclass

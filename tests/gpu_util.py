@@ -34,7 +34,7 @@ def empty(shape, dtype):
 def oracle_layer(spec):
     import oracle as O
     return O.Layer(spec.m, spec.k, spec.r, spec.alpha, spec.bits, spec.group_size, spec.phi_format, spec.act_bits,
-                   spec.act_per_token)
+                   spec.act_per_token, spec.u_bf16)
 
 
 PHI_HOST_DTYPE = {WL.PHI_QFIXED: np.int8, WL.PHI_INT_PACKED: np.uint8, WL.PHI_BF16: np.uint16,
@@ -49,6 +49,15 @@ def phi_buffer(spec):
     if spec.phi_format in (WL.PHI_BF16, WL.PHI_FP16):
         return t.empty((spec.m, spec.k), dtype=t.int16, device="cuda")
     return t.empty((spec.m, spec.k), dtype=t.int8 if spec.phi_format == WL.PHI_QFIXED else t.uint8, device="cuda")
+
+
+def near_bf16_boundary(A, B, rel: float = 2.0 ** -18) -> np.ndarray:
+    """Elements whose exact A B lies so close to a bf16 rounding boundary that the
+    fp32-accumulated product of the tensor cores may round to the other neighbour
+    (the bf16 pre-round reading rounds A B to bf16 first)."""
+    import oracle as O
+    ab = np.asarray(A, dtype=np.float64) @ np.asarray(B, dtype=np.float64)
+    return O.bf16_round(ab * (1 + rel)) != O.bf16_round(ab * (1 - rel))
 
 
 def phi_host(phi0, spec) -> np.ndarray:

@@ -112,3 +112,11 @@ def test_lp_range_arguments_are_checked_on_host(lib):
     assert f(ctypes.byref(L), None, 2.0, 100, 16, None) == -1
     assert f(ctypes.byref(_layer(zero=16)), 16, 2.0, 100, 16, None) == -2
     assert f(ctypes.byref(_layer(k=65536)), 16, 2.0, 100, 16, None) == -2
+
+
+def test_bf16_pre_round_is_checked_on_host(lib):
+    f = lambda L: lib.lrqat_linear_fwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, None, 16, 16, 1 << 20, None)
+    assert f(_layer(u_bf16=2)) == -1
+    assert f(_layer(u_bf16=1, phi_format=LQ.PHI_FP16)) == -2
+    assert f(_layer(u_bf16=1, alpha=3.0)) == -2            # alpha / r = 3/4: not a power of two
+    assert f(_layer(u_bf16=1, zero=16)) == -2

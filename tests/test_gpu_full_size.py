@@ -29,13 +29,16 @@ TOL_GRAD = 2e-2
 T_FULL = 8192
 
 # The bench layer (4096 x 4096, Q4.4 per channel), the largest projection of the
-# W4 g128 + A8 MLP (14336 x 4096) and the INT-3 packed down projection (4096 x 11008).
+# W4 g128 + A8 MLP (14336 x 4096), the INT-3 packed down projection (4096 x 11008),
+# and the 4096 x 4096 layer with asymmetric W2, per-token A8, and BF16 / FP8 bases.
 FULL_CASES = [
     ("llama2_7b_attn", WL.workload("llama2_7b_attn").layers[0]),
     ("llama3_8b_gate_g128_a8", WL.workload("llama3_8b_mlp").layers[0]),
     ("llama2_7b_down_int3", WL.workload("llama2_7b_mlp").layers[2]),
     ("llama2_7b_attn_int2_asym", WL.workload("llama2_7b_attn_int2").layers[0]),
     ("llama2_7b_attn_w4a8_token", WL.workload("llama2_7b_attn_w4a8").layers[0]),
+    ("llama2_7b_attn_phi_bf16", WL.workload("llama2_7b_attn_phi_bf16").layers[0]),
+    ("llama2_7b_attn_phi_fp8", WL.workload("llama2_7b_attn_phi_fp8").layers[0]),
 ]
 
 

@@ -13,7 +13,7 @@ import oracle as O
 from paper_2406_06385_gb300 import lrqat as LQ
 from paper_2406_06385_gb300 import workloads as WL
 
-from gpu_util import DeviceLayer, bits_to_f32, oracle_layer, phi_host, to_dev, torch
+from gpu_util import DeviceLayer, bits_to_f32, near_bf16_boundary, oracle_layer, phi_host, to_dev, torch
 
 pytestmark = pytest.mark.gpu
 
@@ -22,10 +22,10 @@ TOL_GRAD = 2e-2
 
 
 def spec_of(name, m, k, r, bits=4, group=0, phi=WL.PHI_QFIXED, act=0, alpha=None, a_std=1 / 64, b_std=1e-3,
-            outliers=1e-3, asym=False, shift=0.0, per_token=False):
+            outliers=1e-3, asym=False, shift=0.0, per_token=False, ub=False):
     return WL.LayerSpec(name, m, k, r, float(r if alpha is None else alpha), bits, group, phi, act,
                         outlier_frac=outliers, a_std=a_std, b_std=b_std, asym=asym, w_row_shift=shift,
-                        act_per_token=per_token)
+                        act_per_token=per_token, u_bf16=ub)
 
 
 def oracle_base(data, OL):
@@ -66,6 +66,12 @@ CASES = [
                                      b_std=0.2), 200),
     ("fp8_e5m2_w2_clip", spec_of("u", 128, 512, 32, bits=2, phi=WL.PHI_FP8_E5M2, a_std=1.0, b_std=1.0), 97),
     ("bf16_w8_g128", spec_of("v", 128, 256, 8, bits=8, group=128, phi=WL.PHI_BF16, a_std=0.3, b_std=0.3), 64),
+    # pre-round value in bf16 (the bf16 reading of the computation)
+    ("q44_pc_ubf16", spec_of("w", 256, 512, 32, ub=True, a_std=0.2, b_std=0.2), 300),
+    ("bf16_g128_ubf16_alpha1", spec_of("x", 128, 384, 16, group=128, phi=WL.PHI_BF16, alpha=1.0, ub=True,
+                                       a_std=0.3, b_std=0.3), 130),
+    ("int3_packed_ubf16_a8", spec_of("y", 128, 256, 16, bits=3, phi=WL.PHI_INT_PACKED, act=8, ub=True, a_std=0.3,
+                                     b_std=0.3), 97),
 ]
 
 
@@ -161,6 +167,9 @@ CODE_CASES = [
     ("fp16_g128", spec_of("c8", 128, 256, 16, group=128, phi=WL.PHI_FP16, a_std=0.1, b_std=0.1)),
     ("fp8_e4m3_w3", spec_of("c9", 128, 384, 16, bits=3, phi=WL.PHI_FP8_E4M3, a_std=0.2, b_std=0.2)),
     ("fp8_e5m2", spec_of("c10", 128, 256, 8, phi=WL.PHI_FP8_E5M2, a_std=0.3, b_std=0.3)),
+    ("q44_pc_ubf16", spec_of("c11", 256, 256, 32, ub=True, a_std=0.3, b_std=0.3)),
+    ("fp8_e4m3_ubf16_alpha1", spec_of("c12", 128, 384, 16, phi=WL.PHI_FP8_E4M3, alpha=1.0, ub=True, a_std=0.5,
+                                      b_std=0.5)),
 ]
 
 
@@ -196,6 +205,8 @@ def test_fused_codes_bit_exact(cid, spec, zero_B):
     ones = np.ones((m, k // spec.group_size) if spec.group_size else (m,))
     fq = O.fake_quant_weight(phi0, ones, data.A, data.B, OL, z0)
     exempt = O.near_tie(fq["u"]) if not zero_B else np.zeros_like(fq["c"], dtype=bool)
+    if spec.u_bf16:   # u is a bf16 value: only the bf16 rounding of A B can differ
+        exempt = near_bf16_boundary(data.A, data.B) if not zero_B else np.zeros_like(fq["c"], dtype=bool)
     c_fwd = bits_to_f32(Y).T
     c_dx = bits_to_f32(dX)
     for name, c in (("fwd", c_fwd), ("dX", c_dx)):
@@ -203,3 +214,25 @@ def test_fused_codes_bit_exact(cid, spec, zero_B):
         assert bad.sum() == 0, f"{name}: {bad.sum()} code mismatches (near-ties exempt: {exempt.sum()})"
     if zero_B and spec.phi_format in (WL.PHI_QFIXED, WL.PHI_BF16, WL.PHI_FP16, WL.PHI_FP8_E4M3):
         assert (np.abs(fq["u"] - np.floor(fq["u"]) - 0.5) == 0).sum() > 0   # exact ties were exercised
+
+
+def test_bf16_pre_round_moves_codes():
+    """The two readings of u differ on this layer (so the bf16 cases above test something):
+    the device codes follow the reading the layer asks for."""
+    t = torch()
+    spec = spec_of("ub", 128, 256, 8, a_std=0.05, b_std=0.05)
+    data = WL.make_layer(spec, 1, seed=6, with_activations=False)
+    codes = {}
+    for ub in (False, True):
+        sp = spec_of("ub", 128, 256, 8, a_std=0.05, b_std=0.05, ub=ub)
+        dl = DeviceLayer(WL.LayerData(sp, data.W0, data.A_bits, data.B_bits))
+        wz = t.empty((128, 256), dtype=t.int8, device="cuda")
+        LQ.merge(dl.layer, dl.phi0, dl.A, dl.B, wz)
+        LQ.get_device_status()
+        codes[ub] = wz.cpu().numpy()
+        OL = oracle_layer(sp)
+        ref = O.merge(O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL), data.A, data.B, OL)
+        exempt = near_bf16_boundary(data.A, data.B) if ub else O.near_tie(
+            O.preround(O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL), data.A, data.B, OL))
+        assert ((codes[ub] != ref) & ~exempt).sum() == 0
+    assert (codes[False] != codes[True]).mean() > 0.001
