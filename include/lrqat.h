@@ -140,6 +140,19 @@ int lrqat_range_lp(const lrqat_layer* layer, const float* W0, float p_norm, int3
 int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0,
                    lrqat_stream_t stream);
 
+/* Activation fake quantizer of the weight-activation runs (Sec. 4; Eq. 1 with z = 0,
+ * b = 8), the step lrqat_linear_fwd / lrqat_linear_bwd run first when act_bits == 8,
+ * on its own.  X: bf16 [T, k]; X_out: bf16 [T, k] (output); layer->act_bits must be 8.
+ *   act_per_token == 0: X_out = X_Z = clip(round(X / s_x), -128, 127) as exact bf16
+ *     codes, X / s_x one fp32 division, s_x a device scalar (required); mask
+ *     (nullable): uint32 [k, ceil(T/32)], bit t % 32 of word [j, t / 32] is
+ *     M_x = 1[-128 <= round(X[t, j] / s_x) <= 127];
+ *   act_per_token == 1: s_x[t] = max_j |X[t, j]| / 127 in fp32 (1 for an all-zero
+ *     token), X_out = bf16(s_x[t] X_Z); s_x and mask are not used (NULL allowed).
+ * X and X_out 16-byte aligned; mask 4-byte aligned. */
+int lrqat_act_quant(const lrqat_layer* layer, int64_t T, const uint16_t* X, const float* s_x, uint16_t* X_out,
+                    uint32_t* mask, lrqat_stream_t stream);
+
 /* Bytes of workspace lrqat_linear_fwd needs for T tokens (padded adapter
  * copies; int8 activation codes when act_bits == 8). */
 size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T);

@@ -310,96 +310,177 @@ __device__ __forceinline__ float div_round(float x, float s, float r) {
 }
 
 // --------------------------------------------------------- activation quant --
-// X_Z = clip(round(X / s_x), -128, 127) stored as exact bf16; optional mask bits
-// M_x = 1[-128 <= round(X / s_x) <= 127], laid out [k][ceil(T/32)] (bit = token % 32).
-// Each thread handles 8 consecutive columns (16-byte loads and stores) of 32 tokens;
-// the division is the IEEE one, so the integer decisions match a plain fp32 X / s_x.
-__global__ void act_quant_kernel(const uint4* __restrict__ X, int64_t T, int64_t k8, const float* __restrict__ s_x,
-                                 uint4* __restrict__ codes, uint32_t* __restrict__ mask, int64_t mask_ld) {
-  const int64_t j8 = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (j8 >= k8) return;
+// round(fl32(x / s)) for two values, dividing only near a tie: y = x r with r =
+// fl32(1 / s) lies within 2^-22 |y| of x / s, and so does fl32(x / s); for |y| < 2^10
+// that is below 2^-12, so a y more than 2^-11 away from a half-integer rounds like the
+// exact quotient.  A |y| >= 2^10 is far outside every grid quantized here (|code| <=
+// 128), so whichever integer it rounds to, it clips and masks the same way.
+__device__ __forceinline__ float2 div_round2(float2 x, float s, float r) {
+  const float2 y = __fmul2_rn(x, make_float2(r, r));
+  float2 q = make_float2(rintf(y.x), rintf(y.y));
+  const float2 d = __fadd2_rn(y, make_float2(-q.x, -q.y));
+  if (fabsf(d.x) > 0.49951171875f) q.x = rintf(__fdiv_rn(x.x, s));
+  if (fabsf(d.y) > 0.49951171875f) q.y = rintf(__fdiv_rn(x.y, s));
+  return q;
+}
+
+// Per-tensor quantizer: X_Z = clip(round(X / s_x), -128, 127) stored as exact bf16;
+// optional mask bits M_x = 1[-128 <= round(X / s_x) <= 127], laid out [k][ceil(T/32)]
+// (bit = token % 32).  A block covers 64 columns x 256 tokens; lane (colgroup =
+// lane / 4, token group g = lane % 4) of warp w handles 8 columns (16 bytes) of tokens
+// 32w + 8g .. + 7, so one load instruction covers four token rows of 128 contiguous
+// bytes, and a lane issues its 8 loads before it uses any.  The mask bytes gather in
+// shared memory, and each column's 8 words (256 tokens) go out as 32 contiguous bytes.
+// (A persistent grid that loads its next tile while quantizing the current one held
+// only two blocks per SM and ran slower.)
+constexpr int kAqWarps = 8;
+constexpr int kAqTokens = 32 * kAqWarps;
+__global__ void __launch_bounds__(32 * kAqWarps) act_quant_kernel(const uint4* __restrict__ X, int64_t T,
+                                                                  int64_t k8, const float* __restrict__ s_x,
+                                                                  uint4* __restrict__ codes,
+                                                                  uint32_t* __restrict__ mask, int64_t mask_ld) {
+  __shared__ __align__(16) uint8_t mbytes[64][4 * kAqWarps];   // [column][token byte]
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int cg = lane >> 2, g = lane & 3;
+  const int64_t c8 = static_cast<int64_t>(blockIdx.x) * 8 + cg;
+  const int64_t t0 = static_cast<int64_t>(blockIdx.y) * kAqTokens + 32 * w + 8 * g;
+  const bool col_ok = c8 < k8;
   const float sx = *s_x;
   const float rx = __frcp_rn(sx);
-  const int64_t t0 = static_cast<int64_t>(blockIdx.y) * 32;
-  uint32_t word[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-  uint4 buf[4];
-  for (int tt = 0; tt < 32; ++tt) {
-    const int64_t t = t0 + tt;
-    if (t >= T) break;
-    if ((tt & 3) == 0) {   // four tokens' loads in flight
+  uint4 v[8];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) buf[i] = t + i < T ? X[(t + i) * k8 + j8] : make_uint4(0u, 0u, 0u, 0u);
-    }
-    const uint4 raw = buf[tt & 3];
-    const uint32_t in[4] = {raw.x, raw.y, raw.z, raw.w};
-    uint32_t out[4];
+  for (int i = 0; i < 8; ++i)
+    v[i] = col_ok && t0 + i < T ? __ldg(X + (t0 + i) * k8 + c8) : make_uint4(0u, 0u, 0u, 0u);
+  uint32_t bits[8] = {0, 0, 0, 0, 0, 0, 0, 0};
 #pragma unroll
-    for (int h = 0; h < 4; ++h) {
-      uint32_t o = 0;
+  for (int i = 0; i < 8; ++i) {
+    if (col_ok && t0 + i < T) {
+      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+      uint32_t out[4];
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const float x = __uint_as_float(e ? (in[h] & 0xFFFF0000u) : (in[h] << 16));
-        const float qv = div_round(x, sx, rx);
-        const float c = fminf(fmaxf(qv, -128.0f), 127.0f);
-        o |= (__float_as_uint(c) >> 16) << (16 * e);
-        if (qv >= -128.0f && qv <= 127.0f) word[2 * h + e] |= 1u << tt;
+      for (int h = 0; h < 4; ++h) {
+        const float2 q =
+            div_round2(make_float2(__uint_as_float(in[h] << 16), __uint_as_float(in[h] & 0xFFFF0000u)), sx, rx);
+        out[h] = pack_rn_bf16x2(fminf(fmaxf(q.x, -128.0f), 127.0f), fminf(fmaxf(q.y, -128.0f), 127.0f));
+        bits[2 * h] |= static_cast<uint32_t>(q.x >= -128.0f && q.x <= 127.0f) << i;
+        bits[2 * h + 1] |= static_cast<uint32_t>(q.y >= -128.0f && q.y <= 127.0f) << i;
       }
-      out[h] = o;
+      codes[(t0 + i) * k8 + c8] = make_uint4(out[0], out[1], out[2], out[3]);
     }
-    codes[t * k8 + j8] = make_uint4(out[0], out[1], out[2], out[3]);
   }
-  if (mask) {
+  if (mask == nullptr) return;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) mask[(8 * j8 + e) * mask_ld + blockIdx.y] = word[e];
+  for (int e = 0; e < 8; ++e) mbytes[8 * cg + e][4 * w + g] = static_cast<uint8_t>(bits[e]);
+  __syncthreads();
+  // 64 columns x 8 words: thread -> column tid / 4, words 2 (tid % 4), + 1
+  const int col = threadIdx.x >> 2, q = threadIdx.x & 3;
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * 64 + col;
+  const int64_t w0 = static_cast<int64_t>(blockIdx.y) * kAqWarps + 2 * q;
+  if (j < 8 * k8) {
+    const uint2 pair = *reinterpret_cast<const uint2*>(&mbytes[col][8 * q]);
+    uint32_t* dst = mask + j * mask_ld + w0;
+    if (w0 + 1 < mask_ld && ((reinterpret_cast<uintptr_t>(dst) & 7u) == 0)) {
+      *reinterpret_cast<uint2*>(dst) = pair;
+    } else {
+      if (w0 < mask_ld) dst[0] = pair.x;
+      if (w0 + 1 < mask_ld) dst[1] = pair.y;
+    }
   }
 }
 
-// Per-token dynamic int8 quantizer, one warp per token: s_x[t] = max_j |X[t, j]| / 127
-// (1 for an all-zero token), X_Z = clip(round(X / s_x[t]), -128, 127) with the IEEE
-// division, and X_hat = bf16(s_x[t] X_Z), the operand of the forward and dW GEMMs.
-// The first pass finds the absmax with 16-byte loads and a shuffle reduction; the
-// second pass rereads the row (from L1) and quantizes.  Absmax scaling never clips,
-// so no mask is needed.
-__global__ void __launch_bounds__(kThreads) act_quant_token_kernel(const uint4* __restrict__ X, int64_t T,
-                                                                   int64_t k8, uint4* __restrict__ out) {
+// Per-token dynamic int8 quantizer: s_x[t] = max_j |X[t, j]| / 127 (1 for an all-zero
+// token), X_Z = clip(round(X / s_x[t]), -128, 127) with the IEEE division, and X_hat =
+// bf16(s_x[t] X_Z), the operand of the forward and dW GEMMs.  A token gets 2^tpt_log2
+// threads (32 .. 256, at most kAtLoads 16-byte loads each: k <= 16384), which keep its
+// row in registers from the absmax pass to the quantize pass, so the row is read from
+// memory once; a block of 256 threads holds 256 >> tpt_log2 tokens.  Absmax scaling
+// never clips, so no mask is needed.
+constexpr int kAtLoads = 8;
+__global__ void __launch_bounds__(256, 3) act_quant_token_kernel(const uint4* __restrict__ X, int64_t T, int64_t k8,
+                                                                 int tpt_log2, uint4* __restrict__ out) {
+  __shared__ float red[8];
+  const int tpt = 1 << tpt_log2;
+  const int sub = threadIdx.x & (tpt - 1);                        // thread within its token
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * (256 >> tpt_log2) + (threadIdx.x >> tpt_log2);
+  const bool live = t < T;
+  const uint4* row = X + (live ? t : 0) * k8;
+  uint4 v[kAtLoads];
+#pragma unroll
+  for (int i = 0; i < kAtLoads; ++i) {
+    const int64_t j = sub + static_cast<int64_t>(tpt) * i;
+    v[i] = live && j < k8 ? __ldg(row + j) : make_uint4(0u, 0u, 0u, 0u);
+  }
+  float amax = 0.0f;
+#pragma unroll
+  for (int i = 0; i < kAtLoads; ++i) {
+    const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+    for (int h = 0; h < 4; ++h)
+      amax = fmaxf(amax, fmaxf(fabsf(__uint_as_float(in[h] << 16)), fabsf(__uint_as_float(in[h] & 0xFFFF0000u))));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+  if (tpt > 32) {   // the warps of one token combine through shared memory
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = amax;
+    __syncthreads();
+    const int w0 = (threadIdx.x >> 5) & ~((tpt >> 5) - 1);
+    for (int w = 0; w < (tpt >> 5); ++w) amax = fmaxf(amax, red[w0 + w]);
+  }
+  if (!live) return;
+  const float sx = amax > 0.0f ? __fdiv_rn(amax, 127.0f) : 1.0f;
+  const float rx = __frcp_rn(sx);
+#pragma unroll
+  for (int i = 0; i < kAtLoads; ++i) {
+    const int64_t j = sub + static_cast<int64_t>(tpt) * i;
+    if (j < k8) {
+      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+      uint32_t o[4];
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const float2 q =
+            div_round2(make_float2(__uint_as_float(in[h] << 16), __uint_as_float(in[h] & 0xFFFF0000u)), sx, rx);
+        const float2 xh = __fmul2_rn(make_float2(fminf(fmaxf(q.x, -128.0f), 127.0f), fminf(fmaxf(q.y, -128.0f), 127.0f)),
+                                     make_float2(sx, sx));
+        o[h] = pack_rn_bf16x2(xh.x, xh.y);
+      }
+      out[t * k8 + j] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+  }
+}
+
+// The same for rows longer than the register-resident kernel holds (k > 16384): one
+// warp per token, the second pass rereads the row.
+__global__ void __launch_bounds__(kThreads) act_quant_token_wide_kernel(const uint4* __restrict__ X, int64_t T,
+                                                                        int64_t k8, uint4* __restrict__ out) {
   const int64_t t = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
   const uint4* row = X + t * k8;
   float amax = 0.0f;
-  for (int64_t j0 = lane; j0 < k8; j0 += 128) {   // four 16-byte loads in flight per lane
-    uint4 v[4];
+  for (int64_t j = lane; j < k8; j += 32) {
+    const uint4 v = row[j];
+    const uint32_t in[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) v[i] = j0 + 32 * i < k8 ? row[j0 + 32 * i] : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
-#pragma unroll
-      for (int h = 0; h < 4; ++h)
-        amax = fmaxf(amax, fmaxf(fabsf(__uint_as_float(in[h] << 16)), fabsf(__uint_as_float(in[h] & 0xFFFF0000u))));
-    }
+    for (int h = 0; h < 4; ++h)
+      amax = fmaxf(amax, fmaxf(fabsf(__uint_as_float(in[h] << 16)), fabsf(__uint_as_float(in[h] & 0xFFFF0000u))));
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
   const float sx = amax > 0.0f ? __fdiv_rn(amax, 127.0f) : 1.0f;
   const float rx = __frcp_rn(sx);
-  for (int64_t j0 = lane; j0 < k8; j0 += 128) {
-    uint4 v[4];
+  for (int64_t j = lane; j < k8; j += 32) {
+    const uint4 v = row[j];
+    const uint32_t in[4] = {v.x, v.y, v.z, v.w};
+    uint32_t o[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) v[i] = j0 + 32 * i < k8 ? row[j0 + 32 * i] : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      if (j0 + 32 * i >= k8) break;
-      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
-      uint32_t o[4];
-#pragma unroll
-      for (int h = 0; h < 4; ++h) {
-        const float c0 = fminf(fmaxf(div_round(__uint_as_float(in[h] << 16), sx, rx), -128.0f), 127.0f);
-        const float c1 = fminf(fmaxf(div_round(__uint_as_float(in[h] & 0xFFFF0000u), sx, rx), -128.0f), 127.0f);
-        o[h] = pack_rn_bf16x2(sx * c0, sx * c1);
-      }
-      out[t * k8 + j0 + 32 * i] = make_uint4(o[0], o[1], o[2], o[3]);
+    for (int h = 0; h < 4; ++h) {
+      const float2 q =
+          div_round2(make_float2(__uint_as_float(in[h] << 16), __uint_as_float(in[h] & 0xFFFF0000u)), sx, rx);
+      const float2 xh = __fmul2_rn(make_float2(fminf(fmaxf(q.x, -128.0f), 127.0f), fminf(fmaxf(q.y, -128.0f), 127.0f)),
+                                   make_float2(sx, sx));
+      o[h] = pack_rn_bf16x2(xh.x, xh.y);
     }
+    out[t * k8 + j] = make_uint4(o[0], o[1], o[2], o[3]);
   }
 }
 
@@ -818,17 +899,26 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
   if ((k % 8) != 0 || (reinterpret_cast<uintptr_t>(X) & 15) != 0 || (reinterpret_cast<uintptr_t>(codes) & 15) != 0)
     return cudaErrorInvalidValue;
   const int64_t k8 = k / 8;
-  dim3 grid(static_cast<unsigned>((k8 + 127) / 128), static_cast<unsigned>((T + 31) / 32));
-  act_quant_kernel<<<grid, 128, 0, stream>>>(reinterpret_cast<const uint4*>(X), T, k8, s_x,
-                                             reinterpret_cast<uint4*>(codes), mask, (T + 31) / 32);
+  dim3 grid(static_cast<unsigned>((k8 + 7) / 8), static_cast<unsigned>((T + kAqTokens - 1) / kAqTokens));
+  act_quant_kernel<<<grid, 32 * kAqWarps, 0, stream>>>(reinterpret_cast<const uint4*>(X), T, k8, s_x,
+                                                       reinterpret_cast<uint4*>(codes), mask, (T + 31) / 32);
   return cudaGetLastError();
 }
 
 cudaError_t launch_act_quant_token(const uint16_t* X, int64_t T, int64_t k, uint16_t* x_hat, cudaStream_t stream) {
   if ((k % 8) != 0 || (reinterpret_cast<uintptr_t>(X) & 15) != 0 || (reinterpret_cast<uintptr_t>(x_hat) & 15) != 0)
     return cudaErrorInvalidValue;
-  act_quant_token_kernel<<<blocks_for(T * 32, kThreads), kThreads, 0, stream>>>(
-      reinterpret_cast<const uint4*>(X), T, k / 8, reinterpret_cast<uint4*>(x_hat));
+  const int64_t k8 = k / 8;
+  if (k8 <= 256 * kAtLoads) {
+    int tpt_log2 = 5;
+    while ((static_cast<int64_t>(1) << tpt_log2) * kAtLoads < k8) ++tpt_log2;   // 32 .. 256 threads per token
+    const int64_t per_block = 256 >> tpt_log2;
+    act_quant_token_kernel<<<static_cast<unsigned>((T + per_block - 1) / per_block), 256, 0, stream>>>(
+        reinterpret_cast<const uint4*>(X), T, k8, tpt_log2, reinterpret_cast<uint4*>(x_hat));
+  } else {
+    act_quant_token_wide_kernel<<<blocks_for(T * 32, kThreads), kThreads, 0, stream>>>(
+        reinterpret_cast<const uint4*>(X), T, k8, reinterpret_cast<uint4*>(x_hat));
+  }
   return cudaGetLastError();
 }
 

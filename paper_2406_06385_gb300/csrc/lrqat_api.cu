@@ -441,6 +441,25 @@ int lrqat_range_lp(const lrqat_layer* layer, const float* W0, float p_norm, int3
   return LRQAT_OK;
 }
 
+int lrqat_act_quant(const lrqat_layer* layer, int64_t T, const uint16_t* X, const float* s_x, uint16_t* X_out,
+                    uint32_t* mask, lrqat_stream_t stream) {
+  LRQAT_TRY(validate_layer(layer));
+  const lrqat_layer& L = *layer;
+  if (L.act_bits != 8) return fail(LRQAT_ERR_INVALID_ARG, "lrqat_act_quant needs act_bits == 8");
+  if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
+  if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
+  LRQAT_CHECK_PTR(X, "X");
+  LRQAT_CHECK_PTR(X_out, "X_out");
+  if (L.act_per_token) {
+    LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant_token(X, T, L.k, X_out, stream), "activation quantizer");
+    return LRQAT_OK;
+  }
+  if (!s_x) return fail(LRQAT_ERR_INVALID_ARG, "s_x is required for the per-tensor quantizer");
+  if (mask && (reinterpret_cast<uintptr_t>(mask) & 3u)) return fail(LRQAT_ERR_ALIGNMENT, "mask is not 4-byte aligned");
+  LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, X_out, mask, stream), "activation quantizer");
+  return LRQAT_OK;
+}
+
 int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, void* Phi0, lrqat_stream_t stream) {
   LRQAT_TRY(validate_layer(layer));
   LRQAT_CHECK_PTR(W0, "W0");

@@ -86,6 +86,7 @@ def lib() -> ctypes.CDLL:
             "lrqat_get_device_status": [vp],
             "lrqat_grad_sqnorm": [lp, vp, vp, vp, vp, vp],
             "lrqat_range_lp": [lp, vp, ctypes.c_float, ctypes.c_int32, vp, vp],
+            "lrqat_act_quant": [lp, ctypes.c_int64, vp, vp, vp, vp, vp],
             "lrqat_adamw_step": [lp, ctypes.POINTER(AdamW), vp, vp, vp, vp, ctypes.POINTER(AdamWState), vp, vp, vp,
                                  vp],
         }
@@ -164,6 +165,12 @@ def linear_bwd(layer: Layer, T: int, dY, X, Phi0, s, A, B, s_x, dX, dA, dB, ds, 
 
 def merge(layer: Layer, Phi0, A, B, W_Z, stream=None) -> None:
     _check(lib().lrqat_merge(ctypes.byref(layer), _ptr(Phi0), _ptr(A), _ptr(B), _ptr(W_Z), _stream(stream)))
+
+
+def act_quant(layer: Layer, T: int, X, s_x, X_out, mask=None, stream=None) -> None:
+    """Activation quantizer on its own (per tensor: codes + optional mask; per token: X_hat)."""
+    _check(lib().lrqat_act_quant(ctypes.byref(layer), T, _ptr(X), _ptr(s_x), _ptr(X_out), _ptr(mask),
+                                 _stream(stream)))
 
 
 def range_lp(layer: Layer, W0, s0, p_norm: float, n_candidates: int = 100, stream=None) -> None:

@@ -28,7 +28,7 @@ def test_header_declares_the_entry_points():
     names = header_functions()
     for expected in ("lrqat_range_minmax", "lrqat_downcast", "lrqat_linear_fwd", "lrqat_linear_bwd", "lrqat_merge",
                      "lrqat_fwd_workspace_bytes", "lrqat_bwd_workspace_bytes", "lrqat_get_device_status",
-                     "lrqat_last_error", "lrqat_grad_sqnorm", "lrqat_adamw_step", "lrqat_range_lp"):
+                     "lrqat_last_error", "lrqat_grad_sqnorm", "lrqat_adamw_step", "lrqat_range_lp", "lrqat_act_quant"):
         assert expected in names
 
 
@@ -120,3 +120,12 @@ def test_bf16_pre_round_is_checked_on_host(lib):
     assert f(_layer(u_bf16=1, phi_format=LQ.PHI_FP16)) == -2
     assert f(_layer(u_bf16=1, alpha=3.0)) == -2            # alpha / r = 3/4: not a power of two
     assert f(_layer(u_bf16=1, zero=16)) == -2
+
+
+def test_act_quant_arguments_are_checked_on_host(lib):
+    f = lib.lrqat_act_quant
+    assert f(ctypes.byref(_layer()), 64, 16, 16, 16, None, None) == -1                 # act_bits 0
+    assert f(ctypes.byref(_layer(act_bits=8)), 64, 16, None, 16, None, None) == -1     # per tensor needs s_x
+    assert f(ctypes.byref(_layer(act_bits=8)), 0, 16, 16, 16, None, None) == -1
+    assert f(ctypes.byref(_layer(act_bits=8)), 64, 16, 16, 18, None, None) == -3
+    assert f(ctypes.byref(_layer(act_bits=8)), 64, 16, 16, 16, 18, None) == -3
