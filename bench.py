@@ -10,7 +10,10 @@ three GEMMs (Eq. 8 of the paper, checkpointed as in Sec. 3).
 Prints ONE JSON line (rank 0).  With N > 1 (torchrun) every rank runs an
 independent replica of the workload (weak scaling, no collective on the data
 path); the timed region is bracketed by a barrier and device synchronization,
-and the slowest rank's time is used.
+and the slowest rank's time is used.  The device-resident timed region replays
+each step's library calls from CUDA graphs captured once per input set (the same
+kernels; --no-graph times the eager calls); the end-to-end figure (host buffers,
+copies included) and the per-kernel traced pass use eager calls.
 """
 from __future__ import annotations
 
@@ -236,6 +239,28 @@ class GpuWorkload:
                 LQ.merge(lay["L"], lay["phi0"], lay["A"], lay["B"], lay["WZ"])
 
 
+def capture_steps(gw):
+    """One CUDA graph of gw.step(j) per input set j, captured after an eager pass over
+    every set (first calls configure kernels and cache device data).  Replaying them
+    runs the same library kernels without the per-call host work and launch gaps."""
+    import torch
+    for j in range(gw.sets):
+        gw.step(j)
+    torch.cuda.synchronize()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graphs = []
+    with torch.cuda.stream(side):
+        for j in range(gw.sets):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                gw.step(j)
+            graphs.append(g)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    return lambda i: graphs[i % gw.sets].replay()
+
+
 def time_steps(fn, steps: int, warmup: int):
     import torch
     for i in range(warmup):
@@ -279,9 +304,11 @@ def run_gpu(args):
     uuid = getattr(props, "uuid", None)
     uuid = f"GPU-{uuid}" if uuid is not None and not str(uuid).startswith("GPU-") else (str(uuid) if uuid else None)
 
-    # 1) device-resident timed region (the headline value)
+    # 1) device-resident timed region (the headline value): each step's library calls,
+    #    replayed from CUDA graphs (eager calls with --no-graph)
+    step_fn = gw.step if args.no_graph else capture_steps(gw)
     with ClockSampler(uuid) as clocks:
-        ms = time_steps(gw.step, args.steps, args.warmup)
+        ms = time_steps(step_fn, args.steps, args.warmup)
     LQ.get_device_status()
     ms, units = aggregate_over_ranks(ms, float(T * args.steps))
     value = units / (ms / 1e3)
@@ -387,6 +414,7 @@ def run_gpu(args):
            "activations": ("int8 per-token" if spec0.act_per_token else "int8 per-tensor") if spec0.act_bits == 8
            else "bf16",
            "merge": wl.merge, "parallelism": "replicas" if world > 1 else "single",
+           "launch": "eager library calls" if args.no_graph else "CUDA graph replay of each step's library calls",
            "l2": f"inputs rotate over {args.sets} device copies ({args.sets * sum((l['X'][0].numel() + l['dY'][0].numel()) * 2 for l in gw.layers) / 2**20:.0f} MiB) > L2"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -527,6 +555,7 @@ def main(argv=None):
     p.add_argument("--sets", type=int, default=4, help="distinct device copies of the step inputs (L2 rotation)")
     p.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-graph", action="store_true", help="time eager library calls instead of CUDA graph replays")
     args = p.parse_args(argv)
     if args.warmup < 3:
         p.error("--warmup must be >= 3")
