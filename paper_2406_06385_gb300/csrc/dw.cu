@@ -152,13 +152,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
         const Unit w = decode_unit(u, args);
-        if (!(ok = wait_bounded(bar(BAR_EFEMPTY), (it & 1u) ^ 1u, ctl, 2))) break;
+        if (!(ok = wait_spin_bounded(bar(BAR_EFEMPTY), (it & 1u) ^ 1u, ctl, 2))) break;
         mbar_arrive_expect_tx(bar(BAR_EFFULL), ef_tx);
         tma_load_2d(smem + OFF_AT, &tm_at, w.ib * 128, 0, bar(BAR_EFFULL));
         tma_load_2d(smem + OFF_AT + rbox, &tm_at, w.ib * 128 + 64, 0, bar(BAR_EFFULL));
         ++it;
         for (int c = 0; c < args.nchunks; ++c) {
-          if (!(ok = wait_bounded(bar(BAR_ECEMPTY), (cc & 1u) ^ 1u, ctl, 3))) break;
+          if (!(ok = wait_spin_bounded(bar(BAR_ECEMPTY), (cc & 1u) ^ 1u, ctl, 3))) break;
           const int j0 = w.jt * BN + 128 * c;
           mbar_arrive_expect_tx(bar(BAR_ECFULL), ec_tx);
           if (!P16) tma_load_2d(smem + OFF_PHI, &tm_phi, PACKED ? j0 / 2 : j0, w.ib * 128, bar(BAR_ECFULL));
@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int step = 0; step < w.nsteps; ++step, ++g) {
         if (g % NUM_LOADERS != t) continue;
         const uint32_t s = g % NS, ph = (g / NS) & 1u;
-        if (lane == 0) ok = wait_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1);
+        if (lane == 0) ok = wait_spin_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
         const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
@@ -227,10 +227,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
         const Unit w = decode_unit(u, args);
-        if (!(ok = wait_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 4))) break;
+        if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 4))) break;
         tc_fence_after();
         for (int step = 0; step < w.nsteps; ++step) {
-          if (!(ok = wait_bounded(b_full + 8u * s, ph, ctl, 5))) break;
+          if (!(ok = wait_spin_bounded(b_full + 8u * s, ph, ctl, 5))) break;
           tc_fence_after();
           const uint64_t a = d_dy0 + s * (STAGE_BYTES >> 4), b = d_x0 + s * (STAGE_BYTES >> 4);
           static_assert(BKT == 32, "two 16-token K steps per stage");
@@ -245,9 +245,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         if (!ok) break;
         mma_commit(bar(BAR_ACCFULL));
-        if (!(ok = wait_bounded(bar(BAR_EFFULL), it & 1u, ctl, 6))) break;
+        if (!(ok = wait_spin_bounded(bar(BAR_EFFULL), it & 1u, ctl, 6))) break;
         for (int c = 0; c < args.nchunks; ++c) {
-          if (!(ok = wait_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 7))) break;
+          if (!(ok = wait_spin_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 7))) break;
           tc_fence_after();
           // L = A (rows i) * B (columns j of the chunk): both operands read MN-major from
           // A^T and B, 16 rank rows (two 8-row groups) per K step.
@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             mma_bf16(tmem + COL_L, ad, bd, idesc_l, ks > 0 ? 1u : 0u);
           }
           mma_commit(bar(BAR_LFULL));
-          if (!(ok = wait_bounded(bar(BAR_DUFULL), cc & 1u, ctl, 8))) break;
+          if (!(ok = wait_spin_bounded(bar(BAR_DUFULL), cc & 1u, ctl, 8))) break;
           tc_fence_after();
           // dA (+)= dU * B_chunk^T : M = 128 rows i, N = r16, K = 128 columns j
 #pragma unroll

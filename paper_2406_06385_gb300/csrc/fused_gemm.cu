@@ -172,7 +172,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t it = 0;
       for (int tile = blockIdx.x; tile < args.num_tiles; tile += gridDim.x) {
         const int rb = tile % args.num_rb;
-        if (!wait_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1)) break;
+        if (!wait_spin_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1)) break;
         mbar_arrive_expect_tx(bar(BAR_RFFULL), RF_BYTES);
         tma_load_2d(smem + OFF_RF, &tm_rf, 0, rb * BM, bar(BAR_RFFULL));
         ++it;
@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
       const int tb = tile / args.num_rb;
       for (int kk = t; kk < nk; kk += NT) {
-        if (lane == 0) ok = wait_bounded(eb, (n & 1u) ^ 1u, ctl, 2);
+        if (lane == 0) ok = wait_spin_bounded(eb, (n & 1u) ^ 1u, ctl, 2);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
         if (lane == 0) mbar_arrive_expect_tx(fb, TOK_BYTES);
@@ -216,7 +216,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int kk = 0; kk < nk; ++kk, ++gg) {
         const uint32_t s = gg & (NF - 1);
         const uint32_t fb = bar(BAR_FFULL + s);
-        if (lane == 0) ok = wait_bounded(bar(BAR_FEMPTY + s), ((gg / NF) & 1u) ^ 1u, ctl, 3);
+        if (lane == 0) ok = wait_spin_bounded(bar(BAR_FEMPTY + s), ((gg / NF) & 1u) ^ 1u, ctl, 3);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) break;
         if (lane == 0) mbar_arrive_expect_tx(fb, tx);
@@ -253,8 +253,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // landed and the producers have read the tile of stage gg - 1.
       auto issue_lowrank = [&](uint32_t gg) -> bool {
         const uint32_t s = gg & (NF - 1);
-        if (!wait_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4)) return false;
-        if (!wait_bounded(bar(BAR_LEMPTY), (gg & 1u) ^ 1u, ctl, 5)) return false;
+        if (!wait_spin_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4)) return false;
+        if (!wait_spin_bounded(bar(BAR_LEMPTY), (gg & 1u) ^ 1u, ctl, 5)) return false;
         tc_fence_after();
         const uint64_t sf = d_sf0 + s * FSLOT_D;
         const uint32_t dl = tmem + COL_L;
@@ -266,9 +266,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         return true;
       };
       for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
-        if (!(ok = wait_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
+        if (!(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
         if (!(ok = issue_lowrank(g))) break;
-        if (!(ok = wait_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
+        if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
         tc_fence_after();
         for (int kk = 0; kk < nk; ++kk) {
           const uint32_t gg = g + kk;
@@ -280,8 +280,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (!(ok = issue_lowrank(gg + 1))) break;
             if (kk + 2 == nk) mma_commit(bar(BAR_RFEMPTY));   // last read of the row factor issued
           }
-          if (!(ok = wait_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
-          if (!(ok = wait_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
+          if (!(ok = wait_spin_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
+          if (!(ok = wait_spin_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
           tc_fence_after();
           const uint64_t w = d_w0 + s * TSLOT_D, t = d_tok0 + s * TSLOT_D;
           const uint32_t acc = kk > 0 ? 1u : 0u;

@@ -88,6 +88,38 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, cons
   }
 }
 
+// Spinning variant for the threads whose latency sets the pipeline's pace (the
+// MMA-issuing thread and the TMA loaders): a non-blocking test_wait in a loop, so the
+// thread never sleeps past the phase completion (measured: 1-1.4% off the fused GEMMs
+// against the sleeping wait); bounded like wait_bounded, checking the abort flag and the
+// time limit every 1024 polls.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool wait_spin_bounded(uint32_t bar, uint32_t parity, const WaitCtl& ctl, int site) {
+  if (mbar_test_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_test_wait(bar, parity)) return true;
+    if ((it & 1023u) == 0) {
+      if (*ctl.abort) return false;
+      if (global_timer_ns() - t0 > ctl.timeout_ns) {
+        *ctl.abort = 1;
+        atomicOr(ctl.status, 1 | (1 << (8 + (site & 15))));
+        return false;
+      }
+    }
+  }
+}
+
 // --------------------------------------------------------------------- TMA --
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t c0, int32_t c1,
                                             uint32_t bar) {
