@@ -447,7 +447,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       float scale = 1.0f;
       if (MODE == FUSED_FWD_PC) scale = args.s[row_g];
       if (MODE != FUSED_DX && args.s_x != nullptr) scale *= *args.s_x;
-      ok = wait_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 13);
+      // polled: the drain, and with it the next tile's start, follows this phase directly
+      ok = wait_spin_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 13);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       const bool odd = lane & 1;
