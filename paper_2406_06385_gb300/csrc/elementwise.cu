@@ -561,7 +561,7 @@ __global__ void __launch_bounds__(kThreads) range_lp_kernel(const float* __restr
 //   Bt_pad [k][64]   = B[c][j], zero for c >= r       (B^T, row factor of dX)
 //   At     [r16][m]  = A[i][c], zero rows for c >= r  (A^T, dW epilogue)
 //   B_pad  [r16][k]  = B[c][j], zero rows for c >= r  (dW epilogue)
-__global__ void adapter_layouts_kernel(const uint16_t* __restrict__ A, const uint16_t* __restrict__ B, int64_t m,
+__device__ __forceinline__ void adapter_layouts_body(int64_t blk, int64_t nblk, const uint16_t* __restrict__ A, const uint16_t* __restrict__ B, int64_t m,
                                        int64_t k, int r, int r16, uint4* __restrict__ A_pad,
                                        uint4* __restrict__ Bt_pad, uint4* __restrict__ At,
                                        uint4* __restrict__ B_pad, int b_aligned) {
@@ -570,8 +570,8 @@ __global__ void adapter_layouts_kernel(const uint16_t* __restrict__ A, const uin
   const int64_t n2 = At ? static_cast<int64_t>(r16) * (m / 8) : 0;
   const int64_t n3 = B_pad ? static_cast<int64_t>(r16) * (k / 8) : 0;
   const int64_t total = n0 + n1 + n2 + n3;
-  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  for (int64_t t = blk * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+       t += nblk * blockDim.x) {
     uint32_t w[4];
     if (t < n0) {
       const int64_t i = t >> 3;
@@ -621,6 +621,12 @@ __global__ void adapter_layouts_kernel(const uint16_t* __restrict__ A, const uin
     }
   }
 }
+__global__ void adapter_layouts_kernel(const uint16_t* __restrict__ A, const uint16_t* __restrict__ B, int64_t m,
+                                       int64_t k, int r, int r16, uint4* __restrict__ A_pad,
+                                       uint4* __restrict__ Bt_pad, uint4* __restrict__ At,
+                                       uint4* __restrict__ B_pad, int b_aligned) {
+  adapter_layouts_body(blockIdx.x, gridDim.x, A, B, m, k, r, r16, A_pad, Bt_pad, At, B_pad, b_aligned);
+}
 
 // 128 x 128 tiles of Phi0 (rows i, columns j) -> out[j][i] as int8 stored integers.
 // Load: each thread brings four pieces of 16 stored integers (16 bytes, or 8 packed
@@ -636,11 +642,11 @@ __device__ __forceinline__ void unpack_i4x8(uint32_t packed4, uint32_t& lo_word,
   hi_word = __vsub4(__byte_perm(lo, hi, 0x7362), 0x08080808u);
 }
 
-__global__ void __launch_bounds__(256) phi_transpose_kernel(const void* __restrict__ phi0, int64_t m, int64_t k,
+__device__ __forceinline__ void phi_transpose_body(int64_t bx, int64_t by, const void* __restrict__ phi0, int64_t m, int64_t k,
                                                              int packed, int8_t* __restrict__ out) {
   __shared__ __align__(16) uint32_t tile[128 * 32];   // 128 rows x 32 words
-  const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 128;
-  const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 128;
+  const int64_t i0 = by * 128;
+  const int64_t j0 = bx * 128;
   const int t = threadIdx.x;
   uint4 v[4];
   if (packed) {
@@ -694,11 +700,11 @@ __global__ void __launch_bounds__(256) phi_transpose_kernel(const void* __restri
 
 // 16-bit bases: out[j][i] = Phi0[i][j] through a padded 64 x 64 shared tile (a row
 // stride of 33 words keeps the column reads free of bank conflicts).
-__global__ void __launch_bounds__(256) phi_transpose16_kernel(const uint16_t* __restrict__ in, int64_t m, int64_t k,
+__device__ __forceinline__ void phi_transpose16_body(int64_t bx, int64_t by, const uint16_t* __restrict__ in, int64_t m, int64_t k,
                                                                uint16_t* __restrict__ out) {
   __shared__ __align__(16) uint32_t tile[64 * 33];   // 64 rows x 64 values (+ 2 values of padding)
-  const int64_t i0 = static_cast<int64_t>(blockIdx.y) * 64;
-  const int64_t j0 = static_cast<int64_t>(blockIdx.x) * 64;
+  const int64_t i0 = by * 64;
+  const int64_t j0 = bx * 64;
   const int t = threadIdx.x;
 #pragma unroll
   for (int x = 0; x < 2; ++x) {
@@ -718,6 +724,31 @@ __global__ void __launch_bounds__(256) phi_transpose16_kernel(const uint16_t* __
       o[e] = static_cast<uint32_t>(t16[(8 * q + 2 * e) * 66 + J]) |
              (static_cast<uint32_t>(t16[(8 * q + 2 * e + 1) * 66 + J]) << 16);
     *reinterpret_cast<uint4*>(out + (j0 + J) * m + i0 + 8 * q) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// The backward's preparation in one launch: blocks [0, n_layout) write the adapter
+// layouts (as adapter_layouts_kernel), the rest transpose the stored base (as the
+// 128 x 128 byte or 64 x 64 sixteen-bit transposes), one tile per block.
+struct LayoutJob {
+  const uint16_t* A; const uint16_t* B; int64_t m, k; int r, r16;
+  uint4* A_pad; uint4* Bt_pad; uint4* At; uint4* B_pad; int b_aligned;
+};
+struct TransposeJob {
+  const void* phi0; void* out; int64_t m, k; int fmt; int64_t nbx;   // tiles along k
+};
+__global__ void __launch_bounds__(256) bwd_prep_kernel(LayoutJob lj, int64_t n_layout, TransposeJob tj) {
+  if (static_cast<int64_t>(blockIdx.x) < n_layout) {
+    adapter_layouts_body(blockIdx.x, n_layout, lj.A, lj.B, lj.m, lj.k, lj.r, lj.r16, lj.A_pad, lj.Bt_pad, lj.At,
+                         lj.B_pad, lj.b_aligned);
+    return;
+  }
+  const int64_t b = blockIdx.x - n_layout;
+  if (fmt_16bit(tj.fmt)) {
+    phi_transpose16_body(b % tj.nbx, b / tj.nbx, static_cast<const uint16_t*>(tj.phi0), tj.m, tj.k,
+                         static_cast<uint16_t*>(tj.out));
+  } else {
+    phi_transpose_body(b % tj.nbx, b / tj.nbx, tj.phi0, tj.m, tj.k, tj.fmt == FMT_I4, static_cast<int8_t*>(tj.out));
   }
 }
 
@@ -938,16 +969,21 @@ cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t
   return cudaGetLastError();
 }
 
-cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int fmt, void* out, cudaStream_t stream) {
+cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
+                            uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad, const void* phi0,
+                            int fmt, void* phi_t, cudaStream_t stream) {
   if ((m % 128) != 0 || (k % 128) != 0) return cudaErrorInvalidValue;
-  if (fmt_16bit(fmt)) {
-    dim3 grid(static_cast<unsigned>(k / 64), static_cast<unsigned>(m / 64));
-    phi_transpose16_kernel<<<grid, 256, 0, stream>>>(static_cast<const uint16_t*>(phi0), m, k,
-                                                     static_cast<uint16_t*>(out));
-    return cudaGetLastError();
-  }
-  dim3 grid(static_cast<unsigned>(k / 128), static_cast<unsigned>(m / 128));
-  phi_transpose_kernel<<<grid, kThreads, 0, stream>>>(phi0, m, k, fmt == FMT_I4, static_cast<int8_t*>(out));
+  const LayoutJob lj{A, B, m, k, r, r16, reinterpret_cast<uint4*>(A_pad), reinterpret_cast<uint4*>(Bt_pad),
+                     reinterpret_cast<uint4*>(At), reinterpret_cast<uint4*>(B_pad),
+                     (reinterpret_cast<uintptr_t>(B) & 15) == 0};
+  const int64_t total = (A_pad ? m * 8 : 0) + (Bt_pad ? k * 8 : 0) + (At ? static_cast<int64_t>(r16) * (m / 8) : 0) +
+                        (B_pad ? static_cast<int64_t>(r16) * (k / 8) : 0);
+  const int64_t want = blocks_for(total, 256);
+  const int64_t n_layout = want < 4096 ? want : 4096;
+  const int64_t tile = fmt_16bit(fmt) ? 64 : 128;
+  const TransposeJob tj{phi0, phi_t, m, k, fmt, k / tile};
+  const int64_t blocks = n_layout + (k / tile) * (m / tile);
+  bwd_prep_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(lj, n_layout, tj);
   return cudaGetLastError();
 }
 

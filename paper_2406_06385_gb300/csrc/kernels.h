@@ -34,9 +34,13 @@ cudaError_t launch_act_quant(const uint16_t* X, int64_t T, int64_t k, const floa
 cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
                                    uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad,
                                    cudaStream_t stream);
-// out[j][i] = stored value of Phi0[i][j]: the raw byte (Q-fixed, FP8), the sign-extended
-// nibble as an int8 (packed INT-b), or the raw 16-bit pattern (BF16, FP16); out [k, m].
-cudaError_t launch_phi_transpose(const void* phi0, int64_t m, int64_t k, int fmt, void* out, cudaStream_t stream);
+// The backward's preparation in one launch: the adapter layouts (as launch_adapter_layouts)
+// and phi_t[j][i] = stored value of Phi0[i][j]: the raw byte (Q-fixed, FP8), the
+// sign-extended nibble as an int8 (packed INT-b), or the raw 16-bit pattern (BF16, FP16);
+// phi_t [k, m].
+cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
+                            uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad, const void* phi0,
+                            int fmt, void* phi_t, cudaStream_t stream);
 // Deterministic sums of the per-tile gradient partials written by the dW kernel.
 struct ReduceArgs {
   const float* dA_part; int nA;      // [nA][m][r]

@@ -595,11 +595,10 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   const int r16 = round16(L.r);
   // the transposed base of a packed layer holds one int8 code per byte
   const int fmt_t = L.phi_format == LRQAT_PHI_INT_PACKED ? LRQAT_PHI_QFIXED : L.phi_format;
-  LRQAT_LAUNCH("adapter_layouts", 1, stream,
-               launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, ws.at, ws.b_pad, stream),
-               "adapter layouts");
-  LRQAT_LAUNCH("phi_transpose", 1, stream, launch_phi_transpose(Phi0, L.m, L.k, L.phi_format, ws.phit, stream),
-               "transpose Phi0");
+  LRQAT_LAUNCH("bwd_prep", 1, stream,
+               launch_bwd_prep(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, ws.at, ws.b_pad, Phi0, L.phi_format,
+                               ws.phit, stream),
+               "adapter layouts and transposed base");
   const uint16_t* xop = X;
   if (L.act_bits == 8 && L.act_per_token) {
     // dW takes X_hat = bf16(s_x[t] X_Z); absmax scaling never clips, so dX needs no mask
