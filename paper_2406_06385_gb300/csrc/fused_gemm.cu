@@ -122,6 +122,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
                       const FusedArgs args) {
   using FR = FactorRing<FMT>;
+  // forward: the second factor's slice may come MN-major straight from B (compiled out of dX)
+  const bool sf_mn = MODE != FUSED_DX && args.sf_mn;
   constexpr int NF = FR::NF;
   constexpr bool PACKED = FMT == FMT_I4;
   constexpr uint32_t FSLOT_BYTES = FR::FSLOT_BYTES;
@@ -208,7 +210,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       prefetch_tensormap(&tm_phi);
       prefetch_tensormap(&tm_sf);
     }
-    const uint32_t tx = FR::PHI_TX + static_cast<uint32_t>(BK * 2 * args.sf_cols);
+    const uint32_t tx = FR::PHI_TX + static_cast<uint32_t>(BK * 2 * (sf_mn ? args.r16 : args.sf_cols));
     uint32_t gg = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
@@ -223,7 +225,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         __syncwarp();
         const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
         if (lane == 0) tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb * BM, fb);
-        if (lane == 1) tma_load_2d(fs + FR::FS_SF, &tm_sf, 0, kk * BK, fb);
+        if (lane == 1) {
+          if (sf_mn) tma_load_2d(fs + FR::FS_SF, &tm_sf, kk * BK, 0, fb);   // B rows, 64 columns
+          else tma_load_2d(fs + FR::FS_SF, &tm_sf, 0, kk * BK, fb);
+        }
       }
     }
     if (lane == 0 && gg > 0) {
@@ -237,13 +242,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // short: descriptors of slot 0 are built once; a slot adds its byte stride / 16
       // to the encoded start address and a 16-element K step adds 32 bytes (2 units).
       const uint32_t idesc_main = make_idesc_bf16(128, BN, 0, 0);
-      const uint32_t idesc_l = make_idesc_bf16(128, BK, 0, 0);
+      const uint32_t idesc_l = make_idesc_bf16(128, BK, 0, sf_mn ? 1 : 0);
       const int lsteps = args.r16 / 16;
       constexpr uint32_t TSLOT_D = TSLOT_BYTES >> 4, FSLOT_D = FSLOT_BYTES >> 4, TOKH_D = TOK_HALF >> 4;
+      // K-major operands advance 32 bytes (2 units) per 16-element K step; MN-major ones
+      // (SW128, 8-row atoms of 128-byte rows) advance 16 rows, 2048 bytes (128 units).
       const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
-      // The factor slice has rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to match).
-      const uint32_t sf_swz = args.sf_cols == 16 ? SWZ_32B : args.sf_cols == 32 ? SWZ_64B : SWZ_128B;
-      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + FR::FS_SF, 16, 16u * args.sf_cols, sf_swz);
+      // The K-major factor slice has rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to
+      // match); the MN-major one rows of 64 bf16.
+      const uint32_t sf_swz = sf_mn || args.sf_cols == 64 ? SWZ_128B : args.sf_cols == 32 ? SWZ_64B : SWZ_32B;
+      const uint64_t d_sf0 = sf_mn ? make_sdesc(smem + OFF_FSLOTS + FR::FS_SF, 128u * args.r16, 1024, sf_swz)
+                                   : make_sdesc(smem + OFF_FSLOTS + FR::FS_SF, 16, 16u * args.sf_cols, sf_swz);
+      const uint32_t sf_step = sf_mn ? 128u : 2u;
+      const uint64_t sk1 = sf_step, sk2 = 2 * sf_step, sk3 = 3 * sf_step;
       const uint64_t d_w0 = make_sdesc(smem + OFF_TSLOTS + TS_W, 16, 1024, SWZ_128B);
       const uint64_t d_tok0 = make_sdesc(smem + OFF_TSLOTS, 16, 1024, SWZ_128B);
       uint32_t g = 0;
@@ -259,9 +270,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const uint64_t sf = d_sf0 + s * FSLOT_D;
         const uint32_t dl = tmem + COL_L;
         mma_bf16(dl, d_rf, sf, idesc_l, 0u);
-        if (lsteps > 1) mma_bf16(dl, d_rf + 2, sf + 2, idesc_l, 1u);
-        if (lsteps > 2) mma_bf16(dl, d_rf + 4, sf + 4, idesc_l, 1u);
-        if (lsteps > 3) mma_bf16(dl, d_rf + 6, sf + 6, idesc_l, 1u);
+        if (lsteps > 1) mma_bf16(dl, d_rf + 2, sf + sk1, idesc_l, 1u);
+        if (lsteps > 2) mma_bf16(dl, d_rf + 4, sf + sk2, idesc_l, 1u);
+        if (lsteps > 3) mma_bf16(dl, d_rf + 6, sf + sk3, idesc_l, 1u);
         mma_commit(bar(BAR_LFULL));
         return true;
       };

@@ -95,6 +95,9 @@ struct FusedArgs {
   // Kept last: inserting it earlier shifted the fields above and slowed the producers.
   const float* zero;     // zero offsets shaped like s (asymmetric weights), or nullptr
   int32_t u_bf16;        // pre-round value in bf16 (lrqat_layer.u_bf16)
+  // Forward only: the second factor's slice read straight from B as one MN-major box
+  // of 64 columns x r16 rank rows (no padded B^T copy).
+  int32_t sf_mn;
 };
 int fused_smem_bytes(int fmt);
 // fmt: a PhiFmt value (quant.cuh); FMT_I4 only for the forward modes

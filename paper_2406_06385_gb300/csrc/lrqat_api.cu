@@ -109,6 +109,14 @@ CUtensorMapSwizzle sf_swizzle(int r16) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// The fused GEMMs read the factors straight from the caller's A [m, r] and B [r, k] when
+// TMA can address them (16-byte aligned rows: r a multiple of 8, aligned bases): A as
+// 64-column K-major boxes whose columns past r read as zeros (the same tile as the padded
+// copy), B as MN-major boxes of r16 rank rows whose rows past r read as zeros.
+bool direct_factors(const lrqat_layer& L, const void* A, const void* B) {
+  return L.r % 8 == 0 && aligned16(A) && aligned16(B);
+}
+
 int frac_bits(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_QFIXED ? 8 - L.bits : 0; }
 bool phi_16bit(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_BF16 || L.phi_format == LRQAT_PHI_FP16; }
 int round16(int r) { return (r + 15) / 16 * 16; }
@@ -503,9 +511,11 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   FwdWs ws;
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
-  LRQAT_LAUNCH("adapter_layouts", 1, stream,
-               launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
-               "adapter layouts");
+  const bool direct = direct_factors(L, A, B);
+  if (!direct)
+    LRQAT_LAUNCH("adapter_layouts", 1, stream,
+                 launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
+                 "adapter layouts");
   const uint16_t* tok = X;
   if (L.act_bits == 8 && L.act_per_token) {
     // X_hat = bf16(s_x[t] X_Z): the per-token scales are folded into the token operand
@@ -521,10 +531,17 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 64, 224,
                       CU_TENSOR_MAP_SWIZZLE_128B, "X"));
   LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 64, false));
-  LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
-                      CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
-  LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, sf_cols(r16), 64,
-                      sf_swizzle(r16), "B^T (padded)"));
+  if (direct) {
+    LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A"));
+    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B, L.k, L.r, L.k * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B"));
+  } else {
+    LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
+    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, sf_cols(r16), 64,
+                        sf_swizzle(r16), "B^T (padded)"));
+  }
   FusedArgs a{};
   a.rows = static_cast<int32_t>(L.m);
   a.kdim = static_cast<int32_t>(L.k);
@@ -538,6 +555,7 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   a.s = s;
   a.zero = L.zero;
   a.u_bf16 = L.u_bf16;
+  a.sf_mn = direct ? 1 : 0;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
   a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;
@@ -595,9 +613,12 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   const int r16 = round16(L.r);
   // the transposed base of a packed layer holds one int8 code per byte
   const int fmt_t = L.phi_format == LRQAT_PHI_INT_PACKED ? LRQAT_PHI_QFIXED : L.phi_format;
+  // with direct factors the dX GEMM reads its A slices from A itself; its row factor stays the
+  // padded B^T, and dW takes A^T and B padded
+  const bool direct = direct_factors(L, A, B);
   LRQAT_LAUNCH("bwd_prep", 1, stream,
-               launch_bwd_prep(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, ws.at, ws.b_pad, Phi0, L.phi_format,
-                               ws.phit, stream),
+               launch_bwd_prep(A, B, L.m, L.k, L.r, r16, direct ? nullptr : ws.a_pad, ws.bt_pad, ws.at, ws.b_pad,
+                               Phi0, L.phi_format, ws.phit, stream),
                "adapter layouts and transposed base");
   const uint16_t* xop = X;
   if (L.act_bits == 8 && L.act_per_token) {
@@ -625,8 +646,12 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
                           CU_TENSOR_MAP_SWIZZLE_64B, "Phi0^T"));
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
-    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16), 64,
-                        sf_swizzle(r16), "A (padded)"));
+    if (direct)
+      LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, sf_cols(r16), 64,
+                          sf_swizzle(r16), "A"));
+    else
+      LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16), 64,
+                          sf_swizzle(r16), "A (padded)"));
     FusedArgs a{};
     a.rows = static_cast<int32_t>(L.k);
     a.kdim = static_cast<int32_t>(L.m);
@@ -640,6 +665,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.s = s;
     a.zero = L.zero;
     a.u_bf16 = L.u_bf16;
+    a.sf_mn = 0;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;
