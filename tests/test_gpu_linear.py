@@ -236,3 +236,29 @@ def test_bf16_pre_round_moves_codes():
             O.preround(O.downcast(data.W0, O.minmax_scale(data.W0, OL), OL), data.A, data.B, OL))
         assert ((codes[ub] != ref) & ~exempt).sum() == 0
     assert (codes[False] != codes[True]).mean() > 0.001
+
+
+@pytest.mark.parametrize("r", [8, 32, 40])
+def test_direct_and_padded_factor_paths_agree(r):
+    """The forward reads A and B straight from the caller's arrays when they are 16-byte
+    aligned (r a multiple of 8), else through padded copies; both fill the same shared
+    tiles, so Y is bit-identical.  Factors shifted by one element force the padded path."""
+    t = torch()
+    spec = spec_of("dp", 256, 384, r, a_std=0.2, b_std=0.2)
+    T = 300
+    data = WL.make_layer(spec, T, seed=8)
+    dl = DeviceLayer(data)
+    X = to_dev(data.X_bits)
+    L = dl.layer
+    ws = t.empty(max(LQ.fwd_workspace_bytes(L, T), 16), dtype=t.uint8, device="cuda")
+    outs = []
+    for shift in (0, 1):
+        A = t.empty(dl.A.numel() + 8, dtype=t.int16, device="cuda")[shift:shift + dl.A.numel()].view(dl.A.shape)
+        B = t.empty(dl.B.numel() + 8, dtype=t.int16, device="cuda")[shift:shift + dl.B.numel()].view(dl.B.shape)
+        A.copy_(dl.A)
+        B.copy_(dl.B)
+        Y = t.empty((T, spec.m), dtype=t.int16, device="cuda")
+        LQ.linear_fwd(L, T, X, dl.phi0, dl.s, A, B, None, Y, ws)
+        outs.append(Y.cpu().numpy())
+    LQ.get_device_status()
+    np.testing.assert_array_equal(outs[0], outs[1])
