@@ -255,7 +255,9 @@ def fp8_encode(x: np.ndarray, fmt: int) -> np.ndarray:
     mags = np.array([fp8_value(c, fmt) for c in range(128)])
     finite = np.nonzero(np.isfinite(mags))[0]
     grid_v, grid_c = mags[finite], finite
-    x = np.asarray(x, dtype=np.float32)
+    x = np.asarray(x)
+    if x.dtype != np.float64:   # float64 inputs are rounded from their own value
+        x = x.astype(np.float32)
     a = np.minimum(np.abs(x.astype(np.float64)), grid_v[-1])
     hi = np.clip(np.searchsorted(grid_v, a, side="left"), 0, len(grid_v) - 1)
     lo = np.maximum(hi - 1, 0)
@@ -333,6 +335,32 @@ def downcast(W0: np.ndarray, s0: np.ndarray, layer: Layer, z0: Optional[np.ndarr
         return np.rint(y).astype(np.int8)
     codes = np.clip(np.rint(x), n, p).astype(np.int8)
     return pack_nibbles(codes)
+
+
+def downcast_fp64_changes(W0: np.ndarray, s0: np.ndarray, layer: Layer,
+                          z0: Optional[np.ndarray] = None) -> np.ndarray:
+    """Mask of the elements whose stored base would change if W0 / s0 were one float64
+    division instead of the fp32 IEEE division the downcast uses (reading R8): the
+    value phi^{-1}(Phi0) of ``downcast`` against the same format rounded from the
+    float64 quotient."""
+    n, p = grid(layer.bits)
+    ref = upcast(downcast(W0, s0, layer, z0), layer)
+    x = np.asarray(W0, dtype=np.float32).astype(np.float64) / expand_scale(s0, layer).astype(np.float32).astype(np.float64)
+    if z0 is not None:
+        x = x + expand_scale(z0, layer)
+    fmt = layer.phi_format
+    if fmt == PHI_QFIXED:
+        f = 2.0 ** (8 - layer.bits)
+        alt = np.rint(np.clip(x, n, p) * f) / f
+    elif fmt == PHI_INT_PACKED:
+        alt = np.clip(np.rint(x), n, p)
+    elif fmt == PHI_BF16:
+        alt = bf16_round(x)
+    elif fmt == PHI_FP16:
+        alt = np.clip(x, -65504.0, 65504.0).astype(np.float16).astype(np.float64)
+    else:
+        alt = fp8_decode(fp8_encode(x, fmt), fmt)
+    return ref != alt
 
 
 def upcast(Phi0: np.ndarray, layer: Layer) -> np.ndarray:

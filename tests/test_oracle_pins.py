@@ -705,3 +705,48 @@ def test_bf16_u_swallows_small_adapter_updates():
     np.testing.assert_array_equal(O.merge(phi0, A, B, lay16)[0], np.clip(np.rint(P[0]), -8, 7))
     exact = O.merge(phi0, A, B, layer)[0]
     np.testing.assert_array_equal(exact, [3, -2, 3, -3, 2, 4, -2, 2])
+
+
+# ---------------------------------------------------------------------------
+# Reading R8: the downcast divides in fp32; which codes a float64 division would move
+# ---------------------------------------------------------------------------
+def _fl32_exact(q):
+    """The fp32 value nearest to the rational q, ties to even (checked against both
+    neighbours of a first guess in exact arithmetic)."""
+    from fractions import Fraction
+    c = np.float32(float(q))
+    cands = [np.nextafter(c, np.float32(-np.inf)), c, np.nextafter(c, np.float32(np.inf))]
+    best = min(cands, key=lambda v: (abs(Fraction(float(v)) - q), int(np.float32(v).view(np.uint32)) & 1))
+    return Fraction(float(best))
+
+
+def test_fp64_division_changes_match_exact_arithmetic():
+    """Weights built to put W0 / s0 next to rounding boundaries of Q4.4 (x = (j + 1/2)/16)
+    and of INT-4 (x = j + 1/2), with their fp32 neighbours: the oracle's mask of elements whose base changes under a
+    float64 division equals the one found with exact rationals (the fp32 quotient as the
+    correctly rounded fp32 of W0 / s0, the float64 one as Python's correctly rounded float),
+    and it is not empty."""
+    from fractions import Fraction
+    s0 = np.float32(0.3)
+    for fmt, step in ((O.PHI_QFIXED, 16), (O.PHI_INT_PACKED, 1)):
+        js = np.arange(-120, 112) if step == 16 else np.arange(-8, 7)
+        mid = np.array([np.float32(float(s0) * (j + 0.5) / step) for j in js], dtype=np.float32)
+        vals = np.concatenate([mid, np.nextafter(mid, np.float32(np.inf)), np.nextafter(mid, np.float32(-np.inf))])
+        k = len(vals) + (-len(vals)) % 16
+        W0 = np.zeros((1, k), dtype=np.float32)
+        W0[0, :len(vals)] = vals
+        layer = O.Layer(1, k, 1, 1.0, 4, 0, fmt)
+        got = O.downcast_fp64_changes(W0, np.array([s0]), layer)[0]
+        n, p = O.grid(4)
+        want = np.zeros(k, dtype=bool)
+        for i, w in enumerate(W0[0]):
+            q = Fraction(float(w)) / Fraction(float(s0))
+            codes = []
+            for x in (_fl32_exact(q), Fraction(float(q))):
+                x = min(max(x, n), p)
+                y = x * step
+                r = round(y)                       # Python's round: half to even, exact on Fractions
+                codes.append(r)
+            want[i] = codes[0] != codes[1]
+        np.testing.assert_array_equal(got, want)
+        assert want.sum() > 0
