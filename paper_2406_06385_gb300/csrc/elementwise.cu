@@ -324,6 +324,31 @@ __device__ __forceinline__ float2 div_round2(float2 x, float s, float r) {
   return q;
 }
 
+// round(fl32(x / s)) for the 8 bf16 values of a 16-byte word, with one near-tie test for
+// all of them (the largest distance from a half-integer decides whether any needs the
+// IEEE division); same results as div_round2 on each pair.
+__device__ __forceinline__ void div_round8(const uint4& raw, float s, float r, float (&q)[8]) {
+  const uint32_t in[4] = {raw.x, raw.y, raw.z, raw.w};
+  float x[8], dmax = 0.0f;
+#pragma unroll
+  for (int h = 0; h < 4; ++h) {
+    x[2 * h] = __uint_as_float(in[h] << 16);
+    x[2 * h + 1] = __uint_as_float(in[h] & 0xFFFF0000u);
+    const float2 y = __fmul2_rn(make_float2(x[2 * h], x[2 * h + 1]), make_float2(r, r));
+    q[2 * h] = rintf(y.x);
+    q[2 * h + 1] = rintf(y.y);
+    const float2 d = __fadd2_rn(y, make_float2(-q[2 * h], -q[2 * h + 1]));
+    dmax = fmaxf(dmax, fmaxf(fabsf(d.x), fabsf(d.y)));
+  }
+  if (dmax > 0.49951171875f) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float y = x[e] * r;
+      if (fabsf(y - q[e]) > 0.49951171875f) q[e] = rintf(__fdiv_rn(x[e], s));
+    }
+  }
+}
+
 // Per-tensor quantizer: X_Z = clip(round(X / s_x), -128, 127) stored as exact bf16;
 // optional mask bits M_x = 1[-128 <= round(X / s_x) <= 127], laid out [k][ceil(T/32)]
 // (bit = token % 32).  A block covers 64 columns x 256 tokens; lane (colgroup =
@@ -355,15 +380,15 @@ __global__ void __launch_bounds__(32 * kAqWarps) act_quant_kernel(const uint4* _
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     if (col_ok && t0 + i < T) {
-      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+      float q[8];
+      div_round8(v[i], sx, rx, q);
       uint32_t out[4];
 #pragma unroll
       for (int h = 0; h < 4; ++h) {
-        const float2 q =
-            div_round2(make_float2(__uint_as_float(in[h] << 16), __uint_as_float(in[h] & 0xFFFF0000u)), sx, rx);
-        out[h] = pack_rn_bf16x2(fminf(fmaxf(q.x, -128.0f), 127.0f), fminf(fmaxf(q.y, -128.0f), 127.0f));
-        bits[2 * h] |= static_cast<uint32_t>(q.x >= -128.0f && q.x <= 127.0f) << i;
-        bits[2 * h + 1] |= static_cast<uint32_t>(q.y >= -128.0f && q.y <= 127.0f) << i;
+        const float c0 = fminf(fmaxf(q[2 * h], -128.0f), 127.0f), c1 = fminf(fmaxf(q[2 * h + 1], -128.0f), 127.0f);
+        out[h] = pack_rn_bf16x2(c0, c1);
+        bits[2 * h] |= static_cast<uint32_t>(c0 == q[2 * h]) << i;       // in range iff the clip kept it
+        bits[2 * h + 1] |= static_cast<uint32_t>(c1 == q[2 * h + 1]) << i;
       }
       codes[(t0 + i) * k8 + c8] = make_uint4(out[0], out[1], out[2], out[3]);
     }
@@ -433,14 +458,13 @@ __global__ void __launch_bounds__(256, 3) act_quant_token_kernel(const uint4* __
   for (int i = 0; i < kAtLoads; ++i) {
     const int64_t j = sub + static_cast<int64_t>(tpt) * i;
     if (j < k8) {
-      const uint32_t in[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+      // absmax scaling: |X / s_x| <= 127 (+ rounding), so the codes need no clip
+      float q[8];
+      div_round8(v[i], sx, rx, q);
       uint32_t o[4];
 #pragma unroll
       for (int h = 0; h < 4; ++h) {
-        const float2 q =
-            div_round2(make_float2(__uint_as_float(in[h] << 16), __uint_as_float(in[h] & 0xFFFF0000u)), sx, rx);
-        const float2 xh = __fmul2_rn(make_float2(fminf(fmaxf(q.x, -128.0f), 127.0f), fminf(fmaxf(q.y, -128.0f), 127.0f)),
-                                     make_float2(sx, sx));
+        const float2 xh = __fmul2_rn(make_float2(q[2 * h], q[2 * h + 1]), make_float2(sx, sx));
         o[h] = pack_rn_bf16x2(xh.x, xh.y);
       }
       out[t * k8 + j] = make_uint4(o[0], o[1], o[2], o[3]);
