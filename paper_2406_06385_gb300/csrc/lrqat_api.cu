@@ -750,6 +750,28 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
   if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
   LRQAT_CHECK_PTR(W_Z, "W_Z");
   const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+  if (direct_factors(L, A, B) && aligned16(Phi0) && aligned16(W_Z)) {
+    DeviceInfo* dev = nullptr;
+    LRQAT_TRY(device_info(&dev));
+    const int r16 = round16(L.r);
+    CUtensorMap tm_a, tm_b;
+    LRQAT_TRY(encode_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A"));
+    LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B, L.k, L.r, L.k * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B"));
+    MergeArgs a{};
+    a.phi0 = Phi0;
+    a.wz = W_Z;
+    a.m = L.m;
+    a.k = L.k;
+    a.r16 = r16;
+    a.q = q;
+    a.status = dev->status;
+    a.timeout_ns = kWaitTimeoutNs;
+    LRQAT_LAUNCH("merge", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, tm_a, tm_b, a, stream),
+                 "merge launch");
+    return LRQAT_OK;
+  }
   LRQAT_LAUNCH("merge", 1, stream,
                launch_merge(Phi0, A, B, L.m, L.k, L.r, L.phi_format, L.u_bf16, q, W_Z, stream),
                "merge launch");
