@@ -105,21 +105,6 @@ cudaError_t launch_fused(int mode, int fmt, const CUtensorMap& tm_tok, const CUt
                          const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int grid,
                          cudaStream_t stream);
 
-// ---- merge.cu ------------------------------------------------------------------
-// Merge on the tensor cores; A and B are read by TMA (tm_a over A [m, r], 64 x 128 boxes;
-// tm_b over B [r, k], 64 x r16 boxes; both 128-byte swizzled), so r % 8 == 0.
-struct MergeArgs {
-  const void* phi0;      // stored base [m, k] in its format
-  int8_t* wz;            // W_Z [m, k]
-  int64_t m, k;
-  int32_t r16;           // adapter rank rounded up to 16 (<= 64)
-  QuantParams q;
-  int* status;
-  uint64_t timeout_ns;
-};
-cudaError_t launch_merge_tc(int fmt, int u_bf16, const CUtensorMap& tm_a, const CUtensorMap& tm_b,
-                            const MergeArgs& args, cudaStream_t stream);
-
 // ---- dw.cu -------------------------------------------------------------------
 struct DwArgs {
   int32_t m, k, T;

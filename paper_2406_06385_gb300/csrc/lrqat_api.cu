@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "kernels.h"
+#include "merge.h"
 #include "lrqat.h"
 
 namespace lrqat {

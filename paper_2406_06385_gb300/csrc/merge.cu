@@ -14,6 +14,7 @@
 #include <cstdint>
 
 #include "kernels.h"
+#include "merge.h"
 #include "ptx.cuh"
 #include "quant.cuh"
 
