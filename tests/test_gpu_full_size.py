@@ -9,10 +9,13 @@ what it can compute exactly, one piece at a time:
     near-ties exempt, as in the small-size tests);
   * Y and dX at sampled token rows (all output columns of those rows);
   * dA and ds at sampled weight rows and dB at sampled weight columns, from the
-    rows / columns of G = dY^T X_hat that the oracle forms in fp64.
+    rows / columns of G = dY^T X_hat that the oracle forms in fp64;
+  * every code of W_Z from lrqat_merge at the largest merged projection.
 Sampled outputs are compared with the same relative Frobenius tolerances as the
 small-size tests (1e-2 for Y and dX, 2e-2 for the adapter and scale gradients).
 """
+import dataclasses
+
 import numpy as np
 import pytest
 
@@ -160,3 +163,39 @@ def test_full_size_sampled_outputs(cid, spec):
     dB_ref = scale * (data.A.astype(np.float64).T @ dU_cols)
     dB_got = dB.cpu().numpy()[:, cols]
     assert O.rel_fro(dB_got, dB_ref) <= TOL_GRAD
+
+
+# The merge of the largest projection of the 13B layer that bench.py times with merge
+# (the 5120 x 13824 down projection), plus the 4096 x 4096 layer with a
+# rank that is not a multiple of 8 (the CUDA-core merge) and with a BF16 base.  The
+# factors are drawn large enough (|A B| ~ 0.5 code steps) that many codes move away from
+# the base's.
+def _merge_spec(spec):
+    return dataclasses.replace(spec, a_std=0.25, b_std=0.25)
+
+
+MERGE_CASES = [
+    ("llama2_13b_down", _merge_spec(WL.workload("llama2_13b_layer").layers[6])),
+    ("llama2_7b_attn_r20", WL.LayerSpec("attn_r20", 4096, 4096, 20, 20.0, 4, 0, WL.PHI_QFIXED, a_std=0.25,
+                                        b_std=0.25)),
+    ("llama2_7b_attn_phi_bf16", _merge_spec(WL.workload("llama2_7b_attn_phi_bf16").layers[0])),
+]
+
+
+@pytest.mark.parametrize("cid,spec", MERGE_CASES, ids=[c[0] for c in MERGE_CASES])
+def test_full_size_merge_bit_exact(cid, spec):
+    """Every code of W_Z from lrqat_merge against the oracle's merge (near-ties exempt)."""
+    t = torch()
+    data = WL.make_layer(spec, 1, seed=5, with_activations=False)
+    dl = DeviceLayer(data)
+    wz = t.empty((spec.m, spec.k), dtype=t.int8, device="cuda")
+    LQ.merge(dl.layer, dl.phi0, dl.A, dl.B, wz)
+    LQ.get_device_status()
+    got = wz.cpu().numpy()
+    OL = oracle_layer(spec)
+    _, _, phi0 = _oracle_base(data, OL)
+    ref = O.merge(phi0, data.A, data.B, OL)
+    exempt = O.near_tie(O.preround(phi0, data.A, data.B, OL))
+    bad = (got != ref) & ~exempt
+    assert bad.sum() == 0, f"{bad.sum()} code mismatches of {ref.size} (near-ties exempt: {exempt.sum()})"
+    assert (ref != O.merge(phi0, data.A, np.zeros_like(data.B), OL)).mean() > 0.1   # the low-rank term matters
