@@ -215,6 +215,11 @@ class GpuWorkload:
                        dA=torch.empty((spec.m, spec.r), dtype=torch.float32, device="cuda"),
                        dB=torch.empty((spec.r, spec.k), dtype=torch.float32, device="cuda"),
                        ds=torch.empty_like(s))
+            if spec.act_bits == 8:
+                # the step quantizes X once and runs the forward and the backward on its codes
+                lay["Xq"] = torch.empty((self.T, spec.k), dtype=torch.int16, device="cuda")
+                lay["xmask"] = None if spec.act_per_token else torch.empty(
+                    (spec.k, (self.T + 31) // 32), dtype=torch.int32, device="cuda")
             lay["wsf"] = torch.empty(max(LQ.fwd_workspace_bytes(L, self.T), 16), dtype=torch.uint8, device="cuda")
             lay["wsb"] = torch.empty(LQ.bwd_workspace_bytes(L, self.T), dtype=torch.uint8, device="cuda")
             self.layers.append(lay)
@@ -231,10 +236,19 @@ class GpuWorkload:
             x = lay["X"][j] if X is None else X[id(lay)]
             dy = lay["dY"][j] if dY is None else dY[id(lay)]
             o = lay if outs is None else outs[id(lay)]
-            LQ.linear_fwd(lay["L"], self.T, x, lay["phi0"], lay["s"], lay["A"], lay["B"], lay["s_x"], o["Y"],
-                          lay["wsf"])
-            LQ.linear_bwd(lay["L"], self.T, dy, x, lay["phi0"], lay["s"], lay["A"], lay["B"], lay["s_x"], o["dX"],
-                          o["dA"], o["dB"], o["ds"], False, lay["wsb"])
+            if "Xq" in lay:
+                # int8 activations: one quantizer pass per step feeds both GEMM passes
+                LQ.act_quant(lay["L"], self.T, x, lay["s_x"], lay["Xq"], lay["xmask"])
+                LQ.linear_fwd_quantized(lay["L"], self.T, lay["Xq"], lay["phi0"], lay["s"], lay["A"], lay["B"],
+                                        lay["s_x"], o["Y"], lay["wsf"])
+                LQ.linear_bwd_quantized(lay["L"], self.T, dy, lay["Xq"], lay["xmask"], lay["phi0"], lay["s"],
+                                        lay["A"], lay["B"], lay["s_x"], o["dX"], o["dA"], o["dB"], o["ds"], False,
+                                        lay["wsb"])
+            else:
+                LQ.linear_fwd(lay["L"], self.T, x, lay["phi0"], lay["s"], lay["A"], lay["B"], lay["s_x"], o["Y"],
+                              lay["wsf"])
+                LQ.linear_bwd(lay["L"], self.T, dy, x, lay["phi0"], lay["s"], lay["A"], lay["B"], lay["s_x"],
+                              o["dX"], o["dA"], o["dB"], o["ds"], False, lay["wsb"])
             if self.wl.merge:
                 LQ.merge(lay["L"], lay["phi0"], lay["A"], lay["B"], lay["WZ"])
 

@@ -210,6 +210,30 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
                      const float* s_x, uint16_t* dX, float* dA, float* dB, float* ds, int accumulate,
                      void* workspace, size_t workspace_bytes, lrqat_stream_t stream);
 
+/* Forward and backward on activations the caller has already quantized with
+ * lrqat_act_quant (act_bits == 8 only), so that each input is quantized once per
+ * training step rather than once in the forward and again in the backward (a
+ * deployment convenience; the paper's computation is unchanged):
+ *   X_q: bf16 [T, k], the X_out of lrqat_act_quant for this X and layer (per tensor:
+ *     the codes X_Z; per token: X_hat = bf16(s_x[t] X_Z));
+ *   mask (backward): the clip mask lrqat_act_quant wrote for this X, uint32
+ *     [k, ceil(T/32)], 4-byte aligned; required per tensor, not used per token (NULL
+ *     allowed);
+ *   every other argument as in lrqat_linear_fwd / lrqat_linear_bwd, s_x included (the
+ *     per-tensor scale the codes were made with).
+ * The results equal those of lrqat_linear_fwd / lrqat_linear_bwd on X bit for bit (the
+ * same kernels read the same operands); no quantizer runs.  The workspace sizes of
+ * lrqat_fwd_workspace_bytes / lrqat_bwd_workspace_bytes suffice.  Errors as there, and
+ * LRQAT_ERR_INVALID_ARG when act_bits != 8 or a per-tensor mask is NULL. */
+int lrqat_linear_fwd_quantized(const lrqat_layer* layer, int64_t T, const uint16_t* X_q, const void* Phi0,
+                               const float* s, const uint16_t* A, const uint16_t* B, const float* s_x,
+                               uint16_t* Y, void* workspace, size_t workspace_bytes, lrqat_stream_t stream);
+int lrqat_linear_bwd_quantized(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X_q,
+                               const uint32_t* mask, const void* Phi0, const float* s, const uint16_t* A,
+                               const uint16_t* B, const float* s_x, uint16_t* dX, float* dA, float* dB,
+                               float* ds, int accumulate, void* workspace, size_t workspace_bytes,
+                               lrqat_stream_t stream);
+
 /* Fold the adapters into the final integer weight (Sec. 3, after Eq. 8):
  *   W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p),  so W_hat = s W_Z.
  * W_Z (output): int8 [m, k] with values in [n, p]. */

@@ -486,11 +486,15 @@ size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
   return fwd_ws_layout(*layer, T, nullptr, nullptr);
 }
 
-int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0, const float* s,
-                     const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y, void* workspace,
-                     size_t workspace_bytes, lrqat_stream_t stream) {
+// quantized: X is already the activation quantizer's output for this layer (per tensor: the
+// codes; per token: X_hat), so no quantizer runs.
+static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* X, bool quantized, const void* Phi0,
+                           const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y,
+                           void* workspace, size_t workspace_bytes, lrqat_stream_t stream) {
   LRQAT_TRY(validate_layer(layer));
   const lrqat_layer& L = *layer;
+  if (quantized && L.act_bits != 8)
+    return fail(LRQAT_ERR_INVALID_ARG, "quantized activations need act_bits == 8 (got %d)", L.act_bits);
   if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
   if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
   LRQAT_CHECK_PTR(X, "X");
@@ -518,7 +522,9 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
                  "adapter layouts");
   const uint16_t* tok = X;
-  if (L.act_bits == 8 && L.act_per_token) {
+  if (quantized) {
+    // the caller ran lrqat_act_quant on this X
+  } else if (L.act_bits == 8 && L.act_per_token) {
     // X_hat = bf16(s_x[t] X_Z): the per-token scales are folded into the token operand
     LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant_token(X, T, L.k, ws.x_codes, stream),
                  "activation quantizer");
@@ -574,6 +580,18 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
   return LRQAT_OK;
 }
 
+int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0, const float* s,
+                     const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y, void* workspace,
+                     size_t workspace_bytes, lrqat_stream_t stream) {
+  return linear_fwd_impl(layer, T, X, false, Phi0, s, A, B, s_x, Y, workspace, workspace_bytes, stream);
+}
+
+int lrqat_linear_fwd_quantized(const lrqat_layer* layer, int64_t T, const uint16_t* X_q, const void* Phi0,
+                               const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y,
+                               void* workspace, size_t workspace_bytes, lrqat_stream_t stream) {
+  return linear_fwd_impl(layer, T, X_q, true, Phi0, s, A, B, s_x, Y, workspace, workspace_bytes, stream);
+}
+
 size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
   if (validate_layer(layer) != LRQAT_OK || T < 1) return 0;
   DeviceInfo* dev = nullptr;
@@ -582,12 +600,22 @@ size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
   return bwd_ws_layout(*layer, T, plan_dw(*layer, T, sms), nullptr, nullptr);
 }
 
-int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X, const void* Phi0,
-                     const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* dX, float* dA,
-                     float* dB, float* ds, int accumulate, void* workspace, size_t workspace_bytes,
-                     lrqat_stream_t stream) {
+// quantized: X is already the activation quantizer's output (as for linear_fwd_impl) and
+// x_mask its clip mask (per tensor).
+static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X, bool quantized,
+                           const uint32_t* x_mask, const void* Phi0, const float* s, const uint16_t* A,
+                           const uint16_t* B, const float* s_x, uint16_t* dX, float* dA, float* dB, float* ds,
+                           int accumulate, void* workspace, size_t workspace_bytes, lrqat_stream_t stream) {
   LRQAT_TRY(validate_layer(layer));
   const lrqat_layer& L = *layer;
+  if (quantized) {
+    if (L.act_bits != 8)
+      return fail(LRQAT_ERR_INVALID_ARG, "quantized activations need act_bits == 8 (got %d)", L.act_bits);
+    if (!L.act_per_token && !x_mask)
+      return fail(LRQAT_ERR_INVALID_ARG, "the clip mask is required for per-tensor quantized activations");
+    if (x_mask && (reinterpret_cast<uintptr_t>(x_mask) & 3u))
+      return fail(LRQAT_ERR_ALIGNMENT, "mask is not 4-byte aligned");
+  }
   if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
   if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
   LRQAT_CHECK_PTR(dY, "dY");
@@ -622,7 +650,10 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
                                Phi0, L.phi_format, ws.phit, stream),
                "adapter layouts and transposed base");
   const uint16_t* xop = X;
-  if (L.act_bits == 8 && L.act_per_token) {
+  const uint32_t* xmask = nullptr;
+  if (quantized) {
+    xmask = L.act_per_token ? nullptr : x_mask;
+  } else if (L.act_bits == 8 && L.act_per_token) {
     // dW takes X_hat = bf16(s_x[t] X_Z); absmax scaling never clips, so dX needs no mask
     LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant_token(X, T, L.k, ws.x_codes, stream),
                  "activation quantizer");
@@ -631,6 +662,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     LRQAT_LAUNCH("act_quant", 1, stream, launch_act_quant(X, T, L.k, s_x, ws.x_codes, ws.xmask, stream),
                  "activation quantizer");
     xop = ws.x_codes;
+    xmask = ws.xmask;
   }
   const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
 
@@ -670,7 +702,7 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;
-    a.xmask = L.act_bits == 8 && !L.act_per_token ? ws.xmask : nullptr;
+    a.xmask = L.act_bits == 8 && !L.act_per_token ? xmask : nullptr;
     a.xmask_ld = static_cast<int32_t>((T + 31) / 32);
     a.out = dX;
     a.out_ld = L.k;
@@ -740,6 +772,22 @@ int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, co
   ra.accumulate = accumulate ? 1 : 0;
   LRQAT_LAUNCH("reduce_grads", 1, stream, launch_reduce(ra, stream), "gradient reduction");
   return LRQAT_OK;
+}
+
+int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X, const void* Phi0,
+                     const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* dX, float* dA,
+                     float* dB, float* ds, int accumulate, void* workspace, size_t workspace_bytes,
+                     lrqat_stream_t stream) {
+  return linear_bwd_impl(layer, T, dY, X, false, nullptr, Phi0, s, A, B, s_x, dX, dA, dB, ds, accumulate, workspace,
+                         workspace_bytes, stream);
+}
+
+int lrqat_linear_bwd_quantized(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X_q,
+                               const uint32_t* mask, const void* Phi0, const float* s, const uint16_t* A,
+                               const uint16_t* B, const float* s_x, uint16_t* dX, float* dA, float* dB, float* ds,
+                               int accumulate, void* workspace, size_t workspace_bytes, lrqat_stream_t stream) {
+  return linear_bwd_impl(layer, T, dY, X_q, true, mask, Phi0, s, A, B, s_x, dX, dA, dB, ds, accumulate, workspace,
+                         workspace_bytes, stream);
 }
 
 int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, const uint16_t* B, int8_t* W_Z,

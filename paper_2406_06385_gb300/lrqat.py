@@ -82,6 +82,8 @@ def lib() -> ctypes.CDLL:
             "lrqat_linear_fwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
             "lrqat_linear_fwd_noalloc": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp],
             "lrqat_linear_bwd": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ip, vp, sz, vp],
+            "lrqat_linear_fwd_quantized": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp],
+            "lrqat_linear_bwd_quantized": [lp, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ip, vp, sz, vp],
             "lrqat_merge": [lp, vp, vp, vp, vp, vp],
             "lrqat_get_device_status": [vp],
             "lrqat_grad_sqnorm": [lp, vp, vp, vp, vp, vp],
@@ -161,6 +163,23 @@ def linear_bwd(layer: Layer, T: int, dY, X, Phi0, s, A, B, s_x, dX, dA, dB, ds, 
     _check(lib().lrqat_linear_bwd(ctypes.byref(layer), T, _ptr(dY), _ptr(X), _ptr(Phi0), _ptr(s), _ptr(A), _ptr(B),
                                   _ptr(s_x), _ptr(dX), _ptr(dA), _ptr(dB), _ptr(ds), 1 if accumulate else 0,
                                   _ptr(workspace), nbytes, _stream(stream)))
+
+
+def linear_fwd_quantized(layer: Layer, T: int, X_q, Phi0, s, A, B, s_x, Y, workspace, stream=None) -> None:
+    """Forward on the output of act_quant (per tensor: codes; per token: X_hat)."""
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().lrqat_linear_fwd_quantized(ctypes.byref(layer), T, _ptr(X_q), _ptr(Phi0), _ptr(s), _ptr(A), _ptr(B),
+                                            _ptr(s_x), _ptr(Y), _ptr(workspace), nbytes, _stream(stream)))
+
+
+def linear_bwd_quantized(layer: Layer, T: int, dY, X_q, mask, Phi0, s, A, B, s_x, dX, dA, dB, ds, accumulate: bool,
+                         workspace, stream=None) -> None:
+    """Backward on the output of act_quant and its clip mask (per tensor; None per token)."""
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().lrqat_linear_bwd_quantized(ctypes.byref(layer), T, _ptr(dY), _ptr(X_q), _ptr(mask), _ptr(Phi0),
+                                            _ptr(s), _ptr(A), _ptr(B), _ptr(s_x), _ptr(dX), _ptr(dA), _ptr(dB),
+                                            _ptr(ds), 1 if accumulate else 0, _ptr(workspace), nbytes,
+                                            _stream(stream)))
 
 
 def merge(layer: Layer, Phi0, A, B, W_Z, stream=None) -> None:

@@ -129,3 +129,16 @@ def test_act_quant_arguments_are_checked_on_host(lib):
     assert f(ctypes.byref(_layer(act_bits=8)), 0, 16, 16, 16, None, None) == -1
     assert f(ctypes.byref(_layer(act_bits=8)), 64, 16, 16, 18, None, None) == -3
     assert f(ctypes.byref(_layer(act_bits=8)), 64, 16, 16, 16, 18, None) == -3
+
+
+def test_quantized_activation_entry_points_are_checked_on_host(lib):
+    fq, bq = lib.lrqat_linear_fwd_quantized, lib.lrqat_linear_bwd_quantized
+    a8, a8t = _layer(act_bits=8), _layer(act_bits=8, act_per_token=1)
+    assert fq(ctypes.byref(_layer()), 64, 16, 16, 16, 16, 16, 16, 16, 16, 1 << 20, None) == -1   # act_bits 0
+    bwd = lambda L, mask: bq(ctypes.byref(L), 64, 16, 16, mask, 16, 16, 16, 16, 16, 16, 16, 16, 16, 0, 16, 1 << 20,
+                             None)
+    assert bwd(_layer(), 16) == -1                 # act_bits 0
+    assert bwd(a8, None) == -1                     # per tensor needs the clip mask
+    assert bwd(a8, 18) == -3                       # mask not 4-byte aligned
+    assert bwd(a8t, 18) == -3
+    assert "mask" in LQ.last_error()

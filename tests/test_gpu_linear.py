@@ -262,3 +262,51 @@ def test_direct_and_padded_factor_paths_agree(r):
         outs.append(Y.cpu().numpy())
     LQ.get_device_status()
     np.testing.assert_array_equal(outs[0], outs[1])
+
+
+QUANTIZED_CASES = [
+    # id, spec, T, activation scale factor (< 1 clips part of X)
+    ("a8_tensor_g128_clip", spec_of("qa", 256, 384, 16, group=128, act=8, a_std=0.2, b_std=0.2), 300, 0.25),
+    ("a8_token", spec_of("qb", 256, 512, 32, act=8, per_token=True, a_std=0.2, b_std=0.2), 301, 1.0),
+    ("a8_tensor_packed_ubf16", spec_of("qc", 128, 256, 16, bits=3, phi=WL.PHI_INT_PACKED, act=8, ub=True,
+                                       a_std=0.3, b_std=0.3), 97, 1.0),
+]
+
+
+@pytest.mark.parametrize("cid,spec,T,sx_factor", QUANTIZED_CASES, ids=[c[0] for c in QUANTIZED_CASES])
+def test_quantized_activation_entry_points_bit_identical(cid, spec, T, sx_factor):
+    """lrqat_act_quant once, then lrqat_linear_fwd_quantized / lrqat_linear_bwd_quantized on its
+    codes (and clip mask): every output equals that of the entry points that quantize X
+    themselves, bit for bit."""
+    t = torch()
+    data = WL.make_layer(spec, T, seed=9)
+    dl = DeviceLayer(data)
+    X, dY = to_dev(data.X_bits), to_dev(data.dY_bits)
+    s_x = None
+    if not spec.act_per_token:
+        sx = np.float32(np.float32(np.abs(data.X).max()) / np.float32(127.0) * np.float32(sx_factor))
+        s_x = t.tensor([sx], dtype=t.float32, device="cuda")
+    L = dl.layer
+    ws = t.empty(max(LQ.fwd_workspace_bytes(L, T), 16), dtype=t.uint8, device="cuda")
+    wsb = t.empty(LQ.bwd_workspace_bytes(L, T), dtype=t.uint8, device="cuda")
+
+    def outputs():
+        return dict(Y=t.empty((T, spec.m), dtype=t.int16, device="cuda"),
+                    dX=t.empty((T, spec.k), dtype=t.int16, device="cuda"),
+                    dA=t.empty((spec.m, spec.r), dtype=t.float32, device="cuda"),
+                    dB=t.empty((spec.r, spec.k), dtype=t.float32, device="cuda"), ds=t.empty_like(dl.s))
+
+    a, b = outputs(), outputs()
+    LQ.linear_fwd(L, T, X, dl.phi0, dl.s, dl.A, dl.B, s_x, a["Y"], ws)
+    LQ.linear_bwd(L, T, dY, X, dl.phi0, dl.s, dl.A, dl.B, s_x, a["dX"], a["dA"], a["dB"], a["ds"], False, wsb)
+    Xq = t.empty((T, spec.k), dtype=t.int16, device="cuda")
+    mask = None if spec.act_per_token else t.empty((spec.k, (T + 31) // 32), dtype=t.int32, device="cuda")
+    LQ.act_quant(L, T, X, s_x, Xq, mask)
+    LQ.linear_fwd_quantized(L, T, Xq, dl.phi0, dl.s, dl.A, dl.B, s_x, b["Y"], ws)
+    LQ.linear_bwd_quantized(L, T, dY, Xq, mask, dl.phi0, dl.s, dl.A, dl.B, s_x, b["dX"], b["dA"], b["dB"], b["ds"],
+                            False, wsb)
+    LQ.get_device_status()
+    for key in a:
+        assert t.equal(a[key], b[key]), key
+    if sx_factor < 1.0:
+        assert (bits_to_f32(b["dX"]) == 0).mean() > 0.01   # the clip mask was applied
