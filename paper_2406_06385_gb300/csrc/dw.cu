@@ -98,6 +98,52 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   return x;
 }
 
+// This CTA's units (equal token splits, taken round robin), or (stream-K) its whole tiles
+// of the full waves followed by the segments of its tail range (cut at tile boundaries; a
+// segment's slot is its index among the tile's segments).
+struct WorkIter {
+  int64_t u;      // next unit, or next whole tile
+  int64_t next;   // next tail stage
+  int64_t end;
+};
+
+__device__ __forceinline__ WorkIter work_begin(const DwArgs& a) {
+  if (a.sched.stream_k)
+    return {static_cast<int64_t>(blockIdx.x), dw_range_begin(blockIdx.x, a.sched),
+            dw_range_begin(blockIdx.x + 1, a.sched)};
+  return {static_cast<int64_t>(blockIdx.x), 0, 0};
+}
+
+__device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, Unit& x) {
+  if (!a.sched.stream_k) {
+    if (it.u >= a.num_units) return false;
+    x = decode_unit(static_cast<int>(it.u), a);
+    it.u += gridDim.x;
+    return true;
+  }
+  if (it.u < a.sched.full_tiles) {
+    x.ib = static_cast<int>(it.u % a.ni);
+    x.jt = static_cast<int>(it.u / a.ni);
+    x.sp = 0;
+    x.t0 = 0;
+    x.nsteps = static_cast<int>(a.sched.tsteps);
+    it.u += gridDim.x;
+    return true;
+  }
+  if (it.next >= it.end) return false;
+  const int64_t t = it.next / a.sched.tsteps;   // tile within the tail
+  const int64_t t_end = (t + 1) * a.sched.tsteps;
+  const int64_t e = it.end < t_end ? it.end : t_end;
+  const int64_t tile = a.sched.full_tiles + t;
+  x.ib = static_cast<int>(tile % a.ni);
+  x.jt = static_cast<int>(tile / a.ni);
+  x.sp = static_cast<int>(blockIdx.x - dw_cta_of(t * a.sched.tsteps, a.sched));
+  x.t0 = static_cast<int>((it.next - t * a.sched.tsteps) * BKT);
+  x.nsteps = static_cast<int>(e - it.next);
+  it.next = e;
+  return true;
+}
+
 // UB: pre-round value in bf16 (u_bf16x2) instead of one fp32 FMA.
 template <int FMT, bool ZP, bool UB>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -150,8 +196,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t ec_tx = (P16 ? 0u : PACKED ? 8192u : 16384u) + 2u * rbox;
       uint32_t it = 0, cc = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
-        const Unit w = decode_unit(u, args);
+      WorkIter wi = work_begin(args);
+      Unit w;
+      while (ok && work_next(wi, args, w)) {
+        if (args.sched.stream_k && w.sp == 0) {   // the reduction reads which slots hold data
+          const int64_t tile = w.ib + static_cast<int64_t>(args.ni) * w.jt;
+          args.tile_segs[tile] = dw_tile_segments(tile, args.sched);
+        }
         if (!(ok = wait_spin_bounded(bar(BAR_EFEMPTY), (it & 1u) ^ 1u, ctl, 2))) break;
         mbar_arrive_expect_tx(bar(BAR_EFFULL), ef_tx);
         tma_load_2d(smem + OFF_AT, &tm_at, w.ib * 128, 0, bar(BAR_EFFULL));
@@ -183,8 +234,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int nbox = 2 + 2 * args.nchunks;
     uint32_t g = 0, last_g = 0xffffffffu;
     bool ok = true;
-    for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
-      const Unit w = decode_unit(u, args);
+    WorkIter wi = work_begin(args);
+    Unit w;
+    while (ok && work_next(wi, args, w)) {
       for (int step = 0; step < w.nsteps; ++step, ++g) {
         if (g % NUM_LOADERS != t) continue;
         const uint32_t s = g % NS, ph = (g / NS) & 1u;
@@ -225,8 +277,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t g = 0, it = 0, cc = 0;
       uint32_t s = 0, ph = 0;   // stage and phase of global step g
       bool ok = true;
-      for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
-        const Unit w = decode_unit(u, args);
+      WorkIter wi = work_begin(args);
+      Unit w;
+      while (ok && work_next(wi, args, w)) {
         if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 4))) break;
         tc_fence_after();
         for (int step = 0; step < w.nsteps; ++step) {
@@ -298,8 +351,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int half_cols = args.r16 / 2;   // dA / dB^T columns read by this warp half
     uint32_t it = 0, cc = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < args.num_units && ok; u += gridDim.x) {
-      const Unit w = decode_unit(u, args);
+    WorkIter wi = work_begin(args);
+    Unit w;
+    while (ok && work_next(wi, args, w)) {
       const int i_g = w.ib * 128 + row;
       ok = wait_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 9);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }

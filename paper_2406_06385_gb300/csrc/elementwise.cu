@@ -787,7 +787,18 @@ struct RedJob {
   int nparts;
   int64_t n4;
   float4* dst;
+  int kind;        // 0: dA [m][r] (slot p = jt * nsplit + sp), 1: dB [r][k] (p = ib * nsplit + sp)
+  int64_t width;   // r (dA) or k (dB): elements per row of a partial
 };
+
+// Whether partial slot sp of tile (ib, jt) was written by the dW kernel: every slot, unless
+// its work was split stream-K (then a tile has as many slots as segments, which the dW kernel
+// recorded).
+__device__ __forceinline__ bool slot_written(const ReduceArgs& a, int64_t ib, int64_t jt, int sp) {
+  if (!a.sched.stream_k || sp == 0) return true;
+  const int64_t tile = ib + a.ni * jt;
+  return tile >= a.sched.full_tiles && sp < __ldg(a.tile_segs + tile);
+}
 
 __device__ __forceinline__ void add4(float4& a, const float4& b) {
   a.x += b.x;
@@ -796,24 +807,65 @@ __device__ __forceinline__ void add4(float4& a, const float4& b) {
   a.w += b.w;
 }
 
-__device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk, float lr, int accumulate,
+__device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk, const ReduceArgs& a,
                                                    float4 (*sm)[32]) {
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t e = blk * 32 + lane;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (e < j.n4) {
+  auto part = [&](int64_t p) { return __ldg(j.part + p * j.n4 + e); };
+  if (e < j.n4 && !a.sched.stream_k) {
     int p = w;
     for (; p + 3 * kRedSlices < j.nparts; p += 4 * kRedSlices) {
-      const float4 v0 = __ldg(j.part + static_cast<int64_t>(p) * j.n4 + e);
-      const float4 v1 = __ldg(j.part + static_cast<int64_t>(p + kRedSlices) * j.n4 + e);
-      const float4 v2 = __ldg(j.part + static_cast<int64_t>(p + 2 * kRedSlices) * j.n4 + e);
-      const float4 v3 = __ldg(j.part + static_cast<int64_t>(p + 3 * kRedSlices) * j.n4 + e);
+      const float4 v0 = part(p);
+      const float4 v1 = part(p + kRedSlices);
+      const float4 v2 = part(p + 2 * kRedSlices);
+      const float4 v3 = part(p + 3 * kRedSlices);
       add4(acc, v0);
       add4(acc, v1);
       add4(acc, v2);
       add4(acc, v3);
     }
-    for (; p < j.nparts; p += kRedSlices) add4(acc, __ldg(j.part + static_cast<int64_t>(p) * j.n4 + e));
+    for (; p < j.nparts; p += kRedSlices) add4(acc, part(p));
+  } else if (e < j.n4) {
+    // Stream-K: slot 0 of every tile (always written), spread over the warps, then the further
+    // slots of the tail's tiles.  Slot p = o * nsplit + sp, o the other tile coordinate (jt for
+    // dA, ib for dB); the tile coordinate this element fixes is the same for the whole block.
+    const int ns = a.nsplit;
+    const int64_t n_other = j.nparts / ns;
+    const int64_t fixed = j.kind == 0 ? (4 * e / j.width) / 128 : ((4 * e) % j.width) / a.bn;
+    // first o whose tile (fixed + ni o for dA, o + ni fixed for dB) is past the whole tiles;
+    // this warp's first tail tile's segment count is requested before the slot-0 loads
+    const int64_t ft = a.sched.full_tiles;
+    const int64_t o_tail = j.kind == 0 ? (ft > fixed ? (ft - fixed + a.ni - 1) / a.ni : 0)
+                                       : (ft > a.ni * fixed ? ft - a.ni * fixed : 0);
+    auto tile_of = [&](int64_t oo) { return j.kind == 0 ? fixed + a.ni * oo : oo + a.ni * fixed; };
+    int segs0 = o_tail + w < n_other ? __ldg(a.tile_segs + tile_of(o_tail + w)) : 0;
+    int64_t o = w;
+    for (; o + 3 * kRedSlices < n_other; o += 4 * kRedSlices) {
+      const float4 v0 = part(o * ns);
+      const float4 v1 = part((o + kRedSlices) * ns);
+      const float4 v2 = part((o + 2 * kRedSlices) * ns);
+      const float4 v3 = part((o + 3 * kRedSlices) * ns);
+      add4(acc, v0);
+      add4(acc, v1);
+      add4(acc, v2);
+      add4(acc, v3);
+    }
+#pragma unroll 4
+    for (; o < n_other; o += kRedSlices) add4(acc, part(o * ns));
+    for (int64_t o2 = o_tail + w; o2 < n_other; o2 += kRedSlices) {
+      const int segs = segs0;
+      if (o2 + kRedSlices < n_other) segs0 = __ldg(a.tile_segs + tile_of(o2 + kRedSlices));
+      // slots 1 .. segs - 1, four loads in flight at a time
+      for (int sp = 1; sp < segs; sp += 4) {
+        float4 v[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          v[q] = sp + q < segs ? part(o2 * ns + sp + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) add4(acc, v[q]);
+      }
+    }
   }
   sm[w][lane] = acc;
   __syncthreads();
@@ -825,8 +877,8 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
     for (int h = kRedSlices / 2; h > 0; h >>= 1)
 #pragma unroll
       for (int i = 0; i < h; ++i) add4(s[i], s[i + h]);
-    float4 r = make_float4(s[0].x * lr, s[0].y * lr, s[0].z * lr, s[0].w * lr);
-    if (accumulate) add4(r, j.dst[e]);
+    float4 r = make_float4(s[0].x * a.lr, s[0].y * a.lr, s[0].z * a.lr, s[0].w * a.lr);
+    if (a.accumulate) add4(r, j.dst[e]);
     j.dst[e] = r;
   }
 }
@@ -834,14 +886,16 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
 // ds[i] (per channel): one warp per row; lane l sums blocks l, l + 32, ... of every
 // part, then a fixed shuffle tree adds the lanes.
 __device__ __forceinline__ void reduce_ds_row(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
-                                              int accumulate, float* __restrict__ ds, int64_t blk) {
+                                              int accumulate, float* __restrict__ ds, int64_t blk,
+                                              const ReduceArgs& a) {
   const int64_t i = (blk * kThreads + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (i >= m) return;
   float acc = 0.0f;
-  for (int p = 0; p < nparts; ++p) {
+  for (int p = 0; p < nparts; ++p) {   // slot p / 2, column half p % 2
     const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
-    for (int64_t b = lane; b < nb; b += 32) acc += row[b];
+    for (int64_t b = lane; b < nb; b += 32)
+      if (slot_written(a, i / 128, b * 128 / a.bn, p / 2)) acc += row[b];
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
@@ -851,15 +905,16 @@ __device__ __forceinline__ void reduce_ds_row(const float* __restrict__ part, in
 // ds[i][g] (per group): one thread per (row, group), sequential over its blocks.
 __device__ __forceinline__ void reduce_ds_group(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
                                                 int ngroups, int blocks_per_group, int accumulate,
-                                                float* __restrict__ ds, int64_t blk) {
+                                                float* __restrict__ ds, int64_t blk, const ReduceArgs& a) {
   const int64_t e = blk * kThreads + threadIdx.x;
   if (e >= m * ngroups) return;
   const int64_t i = e / ngroups;
   const int g = static_cast<int>(e % ngroups);
   float acc = 0.0f;
-  for (int p = 0; p < nparts; ++p) {
+  for (int p = 0; p < nparts; ++p) {   // slot p / 2, column half p % 2
     const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
-    for (int b = g * blocks_per_group; b < (g + 1) * blocks_per_group; ++b) acc += row[b];
+    for (int b = g * blocks_per_group; b < (g + 1) * blocks_per_group; ++b)
+      if (slot_written(a, i / 128, static_cast<int64_t>(b) * 128 / a.bn, p / 2)) acc += row[b];
   }
   ds[e] = accumulate ? ds[e] + acc : acc;
 }
@@ -869,14 +924,14 @@ __global__ void __launch_bounds__(kThreads) reduce_grads_kernel(RedJob ja, RedJo
   __shared__ float4 sm[kRedSlices][32];
   const int64_t blk = blockIdx.x;
   if (blk < nblk_a) {
-    reduce_parts_block(ja, blk, a.lr, a.accumulate, sm);
+    reduce_parts_block(ja, blk, a, sm);
   } else if (blk < nblk_a + nblk_b) {
-    reduce_parts_block(jb, blk - nblk_a, a.lr, a.accumulate, sm);
+    reduce_parts_block(jb, blk - nblk_a, a, sm);
   } else if (a.group_size == 0) {
-    reduce_ds_row(a.ds_part, a.nS, a.m, nb, a.accumulate, a.ds, blk - nblk_a - nblk_b);
+    reduce_ds_row(a.ds_part, a.nS, a.m, nb, a.accumulate, a.ds, blk - nblk_a - nblk_b, a);
   } else {
     reduce_ds_group(a.ds_part, a.nS, a.m, nb, ngroups, a.group_size / 128, a.accumulate, a.ds,
-                    blk - nblk_a - nblk_b);
+                    blk - nblk_a - nblk_b, a);
   }
 }
 
@@ -1013,8 +1068,8 @@ cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int
 
 cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream) {
   const int64_t nA4 = a.m * a.r / 4, nB4 = static_cast<int64_t>(a.r) * a.k / 4;   // m, k are multiples of 128
-  const RedJob ja{reinterpret_cast<const float4*>(a.dA_part), a.nA, nA4, reinterpret_cast<float4*>(a.dA)};
-  const RedJob jb{reinterpret_cast<const float4*>(a.dB_part), a.nB, nB4, reinterpret_cast<float4*>(a.dB)};
+  const RedJob ja{reinterpret_cast<const float4*>(a.dA_part), a.nA, nA4, reinterpret_cast<float4*>(a.dA), 0, a.r};
+  const RedJob jb{reinterpret_cast<const float4*>(a.dB_part), a.nB, nB4, reinterpret_cast<float4*>(a.dB), 1, a.k};
   const int64_t nblk_a = (nA4 + 31) / 32, nblk_b = (nB4 + 31) / 32;
   const int64_t nb = a.k / 128;
   const int ngroups = a.group_size ? static_cast<int>(a.k / a.group_size) : 1;

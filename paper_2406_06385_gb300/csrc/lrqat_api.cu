@@ -8,6 +8,7 @@
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -261,6 +262,7 @@ struct Carver {
 // ----------------------------------------------------------------- planning --
 struct DwPlan {
   int nchunks, ni, nj, nsplit, tchunk, units;
+  DwSched sched;
 };
 
 DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
@@ -287,6 +289,46 @@ DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
   p.tchunk = static_cast<int>((tsteps + best - 1) / best) * 32;
   p.nsplit = static_cast<int>((T + p.tchunk - 1) / p.tchunk);   // no empty splits
   p.units = tiles * p.nsplit;
+  const int grid_eq = p.units < sms ? p.units : sms;
+  p.sched = DwSched{0, grid_eq, tsteps, 0, 0};
+  // Against whole tiles for the full waves of every SM and a stream-K split of the rest, by the
+  // slowest CTA's cost in stage units: its stages plus kEpilogueStages for each unit or segment
+  // it finishes (the part of the epilogue that the next main loop waits for, ~12K cycles
+  // against ~400 per stage).  The tail needs at least one stage per CTA.
+  constexpr int64_t kEpilogueStages = 32;
+  const int64_t waves = (p.units + grid_eq - 1) / grid_eq;
+  const int64_t cost_eq = waves * (p.tchunk / 32 + kEpilogueStages);
+  const int64_t full_tiles = tiles / sms * sms;
+  const DwSched sk{1, sms, tsteps, full_tiles, (tiles - full_tiles) * tsteps};
+  bool sk_ok = sk.total_steps >= sms;
+  int64_t cost_sk = 0;
+  if (sk_ok) {
+    int64_t max_segs = 0;
+    for (int b = 0; b < sms; ++b) {
+      const int64_t g0 = dw_range_begin(b, sk), g1 = dw_range_begin(b + 1, sk);
+      const int64_t segs = (g1 - 1) / tsteps - g0 / tsteps + 1;
+      if (segs > max_segs) max_segs = segs;
+    }
+    cost_sk = full_tiles / sms * (tsteps + kEpilogueStages) + (sk.total_steps + sms - 1) / sms +
+              kEpilogueStages * max_segs;
+  }
+  // LRQAT_DW_SCHEDULE=stream_k / split overrides the choice (tests and timing of either schedule)
+  const char* force = std::getenv("LRQAT_DW_SCHEDULE");
+  const bool use_sk = !sk_ok ? false
+                      : force && std::strcmp(force, "stream_k") == 0 ? true
+                      : force && std::strcmp(force, "split") == 0    ? false
+                                                                     : cost_sk < cost_eq;
+  if (use_sk) {
+    int slots = 1;
+    for (int64_t tile = full_tiles; tile < tiles; ++tile) {
+      const int n = dw_tile_segments(tile, sk);
+      if (n > slots) slots = n;
+    }
+    p.sched = sk;
+    p.nsplit = slots;        // partial slots per tile
+    p.tchunk = 0;            // not used
+    p.units = sms;
+  }
   return p;
 }
 
@@ -317,6 +359,7 @@ struct BwdWs {
   float* dA_part;
   float* dB_part;
   float* ds_part;
+  int32_t* tile_segs;
 };
 
 size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* base, BwdWs* ws) {
@@ -335,6 +378,7 @@ size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* bas
   w.dA_part = static_cast<float*>(c.take(static_cast<size_t>(p.nj) * p.nsplit * L.m * L.r * 4));
   w.dB_part = static_cast<float*>(c.take(static_cast<size_t>(p.ni) * p.nsplit * L.r * L.k * 4));
   w.ds_part = static_cast<float*>(c.take(static_cast<size_t>(2) * p.nsplit * L.m * (L.k / 128) * 4));
+  w.tile_segs = static_cast<int32_t*>(c.take(static_cast<size_t>(p.ni) * p.nj * 4));
   if (ws) *ws = w;
   return (c.used + 255) & ~size_t(255);
 }
@@ -749,7 +793,9 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
     a.phi = Phi0;
-    const int grid = plan.units < dev->sms ? plan.units : dev->sms;
+    a.sched = plan.sched;
+    a.tile_segs = ws.tile_segs;
+    const int grid = plan.sched.grid;
     LRQAT_LAUNCH("fused_dw", 1, stream,
                  launch_dw(L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
                  "fused dW launch");
@@ -770,6 +816,11 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   ra.group_size = L.group_size;
   ra.lr = static_cast<float>(static_cast<double>(L.alpha) / L.r);
   ra.accumulate = accumulate ? 1 : 0;
+  ra.sched = plan.sched;
+  ra.ni = plan.ni;
+  ra.nsplit = plan.nsplit;
+  ra.bn = 128 * plan.nchunks;
+  ra.tile_segs = ws.tile_segs;
   LRQAT_LAUNCH("reduce_grads", 1, stream, launch_reduce(ra, stream), "gradient reduction");
   return LRQAT_OK;
 }

@@ -142,3 +142,15 @@ def test_quantized_activation_entry_points_are_checked_on_host(lib):
     assert bwd(a8, 18) == -3                       # mask not 4-byte aligned
     assert bwd(a8t, 18) == -3
     assert "mask" in LQ.last_error()
+
+
+def test_dw_schedule_override_changes_the_partial_slots(lib, monkeypatch):
+    """A 128 x 256 layer over 8192 tokens: equal splits keep at most 8 slots per tile; stream-K
+    over every SM cuts the one tile into a segment per CTA, so its backward workspace (the
+    gradient partials) grows."""
+    L = _layer(m=128, k=256)
+    sizes = {}
+    for sched in ("split", "stream_k"):
+        monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
+        sizes[sched] = lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192)
+    assert sizes["stream_k"] > 4 * sizes["split"] > 0

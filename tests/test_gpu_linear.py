@@ -310,3 +310,45 @@ def test_quantized_activation_entry_points_bit_identical(cid, spec, T, sx_factor
         assert t.equal(a[key], b[key]), key
     if sx_factor < 1.0:
         assert (bits_to_f32(b["dX"]) == 0).mean() > 0.01   # the clip mask was applied
+
+
+# Shapes with at least one 32-token stage per CTA in the stream-K tail (tiles x stages >= 152),
+# ragged token counts; the last case has a full wave of whole tiles (160 tiles) before its tail.
+STREAM_K_CASES = [
+    ("q44_pc", spec_of("a", 384, 512, 32), 1000),
+    ("int3_packed", spec_of("d", 256, 512, 32, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.2, b_std=0.2), 1500),
+    ("q44_g128_a8", spec_of("f", 256, 384, 16, group=128, act=8, a_std=0.2, b_std=0.2), 1700),
+    ("int2_asym_q26", spec_of("k", 256, 512, 32, bits=2, asym=True, shift=0.03, a_std=0.2, b_std=0.2), 1300),
+    ("a8_token", spec_of("p", 256, 512, 32, act=8, per_token=True, a_std=0.2, b_std=0.2), 1301),
+    ("bf16_pc", spec_of("r", 256, 512, 32, phi=WL.PHI_BF16, a_std=0.2, b_std=0.2), 1250),
+    ("whole_wave_then_tail", spec_of("z", 2048, 2560, 16, a_std=0.2, b_std=0.2), 650),
+]
+
+
+@pytest.mark.parametrize("cid,spec,T", STREAM_K_CASES, ids=[c[0] for c in STREAM_K_CASES])
+def test_fwd_bwd_parity_stream_k_dw(cid, spec, T, monkeypatch):
+    """The dW work split stream-K (whole tiles for the full waves, then each CTA an equal range
+    of the remaining 32-token stages, a tile's token ranges reduced as separate partial slots),
+    forced on shapes whose cost model picks equal splits: ragged token tails inside segments,
+    tiles cut across many CTAs, and slots that no segment writes."""
+    monkeypatch.setenv("LRQAT_DW_SCHEDULE", "stream_k")
+    got, ref, _ = _run(spec, T, seed=2, s_scale=1.05)
+    errs = {k: O.rel_fro(got[k], ref[k]) for k in got}
+    assert errs["Y"] <= TOL_ACT and errs["dX"] <= TOL_ACT, errs
+    assert errs["dA"] <= TOL_GRAD and errs["dB"] <= TOL_GRAD and errs["ds"] <= TOL_GRAD, errs
+
+
+def test_dw_schedules_agree(monkeypatch):
+    """Equal token splits and stream-K give the same Y and dX bit for bit and the same gradients
+    up to rounding: ds up to fp32 summation order; dA and dB also up to the bf16 rounding of
+    dU, which the epilogue applies per token range (about 2^-9 relative)."""
+    spec = spec_of("sk", 256, 512, 32, group=128, a_std=0.2, b_std=0.2)
+    outs = {}
+    for sched in ("split", "stream_k"):
+        monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
+        outs[sched], _, _ = _run(spec, 1555, seed=3)
+    for key in ("Y", "dX"):
+        np.testing.assert_array_equal(outs["split"][key], outs["stream_k"][key])
+    assert O.rel_fro(outs["stream_k"]["ds"], outs["split"]["ds"]) <= 1e-5
+    for key in ("dA", "dB"):
+        assert O.rel_fro(outs["stream_k"][key], outs["split"][key]) <= 1e-2, key
