@@ -204,7 +204,13 @@ size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
  * dX (output): bf16 [T, k]; dA: fp32 [m, r]; dB: fp32 [r, k]; ds: fp32 like s.
  * accumulate = 0 overwrites dA, dB, ds; 1 adds to them (gradient accumulation
  * over micro-batches).  dX is always overwritten.
- * workspace: device buffer of at least lrqat_bwd_workspace_bytes() bytes. */
+ * workspace: device buffer of at least lrqat_bwd_workspace_bytes() bytes.
+ * The weight-gradient work is spread over the SMs either as equal token splits of
+ * every tile or as whole tiles followed by a balanced (stream-K) split of the rest,
+ * chosen per call; the environment variable LRQAT_DW_SCHEDULE = "split" or
+ * "stream_k" forces one (read by lrqat_bwd_workspace_bytes and lrqat_linear_bwd
+ * alike, so keep it fixed between the two).  Both give the same dX bit for bit and
+ * the same dA, dB, ds up to rounding order. */
 int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X,
                      const void* Phi0, const float* s, const uint16_t* A, const uint16_t* B,
                      const float* s_x, uint16_t* dX, float* dA, float* dB, float* ds, int accumulate,
