@@ -883,6 +883,31 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
   }
 }
 
+// Sum over the 128-column blocks b = b0, b0 + step, ... < b_end of row i of the parts that the
+// stream-K tail wrote past slot 0 (tiles past the whole ones; their segment count read once per
+// block, the slots' loads issued together).
+__device__ __forceinline__ float ds_tail_slots(const float* __restrict__ part, int64_t m, int64_t nb, int64_t i,
+                                               int64_t b0, int64_t step, const ReduceArgs& a, int64_t b_end = -1) {
+  if (b_end < 0) b_end = nb;
+  float acc = 0.0f;
+  for (int64_t b = b0; b < b_end; b += step) {
+    const int64_t tile = i / 128 + a.ni * (b * 128 / a.bn);
+    if (tile < a.sched.full_tiles) continue;
+    const int segs = __ldg(a.tile_segs + tile);
+    for (int sp = 1; sp < segs; sp += 2) {
+      float v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int p = 2 * (sp + q / 2) + (q & 1);
+        v[q] = sp + q / 2 < segs ? __ldg(part + (static_cast<int64_t>(p) * m + i) * nb + b) : 0.0f;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc += v[q];
+    }
+  }
+  return acc;
+}
+
 // ds[i] (per channel): one warp per row; lane l sums blocks l, l + 32, ... of every
 // part, then a fixed shuffle tree adds the lanes.
 __device__ __forceinline__ void reduce_ds_row(const float* __restrict__ part, int nparts, int64_t m, int64_t nb,
@@ -892,11 +917,14 @@ __device__ __forceinline__ void reduce_ds_row(const float* __restrict__ part, in
   const int lane = threadIdx.x & 31;
   if (i >= m) return;
   float acc = 0.0f;
-  for (int p = 0; p < nparts; ++p) {   // slot p / 2, column half p % 2
+  // parts p = 2 sp + h (slot sp, column half h); stream-K: slot 0 of every block here, the
+  // written further slots of the tail's tiles below
+  const int dense = a.sched.stream_k ? 2 : nparts;
+  for (int p = 0; p < dense; ++p) {
     const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
-    for (int64_t b = lane; b < nb; b += 32)
-      if (slot_written(a, i / 128, b * 128 / a.bn, p / 2)) acc += row[b];
+    for (int64_t b = lane; b < nb; b += 32) acc += row[b];
   }
+  if (a.sched.stream_k) acc += ds_tail_slots(part, m, nb, i, lane, 32, a);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
   if (lane == 0) ds[i] = accumulate ? ds[i] + acc : acc;
@@ -911,11 +939,15 @@ __device__ __forceinline__ void reduce_ds_group(const float* __restrict__ part, 
   const int64_t i = e / ngroups;
   const int g = static_cast<int>(e % ngroups);
   float acc = 0.0f;
-  for (int p = 0; p < nparts; ++p) {   // slot p / 2, column half p % 2
+  // parts p = 2 sp + h as in reduce_ds_row
+  const int dense = a.sched.stream_k ? 2 : nparts;
+  for (int p = 0; p < dense; ++p) {
     const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
-    for (int b = g * blocks_per_group; b < (g + 1) * blocks_per_group; ++b)
-      if (slot_written(a, i / 128, static_cast<int64_t>(b) * 128 / a.bn, p / 2)) acc += row[b];
+    for (int b = g * blocks_per_group; b < (g + 1) * blocks_per_group; ++b) acc += row[b];
   }
+  if (a.sched.stream_k)
+    acc += ds_tail_slots(part, m, nb, i, static_cast<int64_t>(g) * blocks_per_group, 1, a,
+                         static_cast<int64_t>(g + 1) * blocks_per_group);
   ds[e] = accumulate ? ds[e] + acc : acc;
 }
 
