@@ -98,24 +98,19 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   return x;
 }
 
-// This CTA's units (equal token splits, taken round robin), or (stream-K) its whole tiles
-// of the full waves followed by the segments of its tail range (cut at tile boundaries; a
-// segment's slot is its index among the tile's segments).
+// This CTA's units (equal token splits, taken round robin), or (tail schedule) its whole
+// tiles of the full waves followed by its one part of a tail tile (slot = part index).
 struct WorkIter {
   int64_t u;      // next unit, or next whole tile
-  int64_t next;   // next tail stage
-  int64_t end;
+  bool tail;      // the tail part is still to come
 };
 
 __device__ __forceinline__ WorkIter work_begin(const DwArgs& a) {
-  if (a.sched.stream_k)
-    return {static_cast<int64_t>(blockIdx.x), dw_range_begin(blockIdx.x, a.sched),
-            dw_range_begin(blockIdx.x + 1, a.sched)};
-  return {static_cast<int64_t>(blockIdx.x), 0, 0};
+  return {static_cast<int64_t>(blockIdx.x), a.sched.tail != 0 && blockIdx.x < a.sched.tail_grid};
 }
 
 __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, Unit& x) {
-  if (!a.sched.stream_k) {
+  if (!a.sched.tail) {
     if (it.u >= a.num_units) return false;
     x = decode_unit(static_cast<int>(it.u), a);
     it.u += gridDim.x;
@@ -130,17 +125,18 @@ __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, Unit& x
     it.u += gridDim.x;
     return true;
   }
-  if (it.next >= it.end) return false;
-  const int64_t t = it.next / a.sched.tsteps;   // tile within the tail
-  const int64_t t_end = (t + 1) * a.sched.tsteps;
-  const int64_t e = it.end < t_end ? it.end : t_end;
+  if (!it.tail) return false;
+  it.tail = false;
+  int64_t t;
+  int j, q;
+  dw_tail_part(blockIdx.x, a.sched, t, j, q);
   const int64_t tile = a.sched.full_tiles + t;
+  const int64_t s0 = j * a.sched.tsteps / q, s1 = (j + 1) * a.sched.tsteps / q;
   x.ib = static_cast<int>(tile % a.ni);
   x.jt = static_cast<int>(tile / a.ni);
-  x.sp = static_cast<int>(blockIdx.x - dw_cta_of(t * a.sched.tsteps, a.sched));
-  x.t0 = static_cast<int>((it.next - t * a.sched.tsteps) * BKT);
-  x.nsteps = static_cast<int>(e - it.next);
-  it.next = e;
+  x.sp = j;
+  x.t0 = static_cast<int>(s0 * BKT);
+  x.nsteps = static_cast<int>(s1 - s0);
   return true;
 }
 
@@ -199,7 +195,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       WorkIter wi = work_begin(args);
       Unit w;
       while (ok && work_next(wi, args, w)) {
-        if (args.sched.stream_k && w.sp == 0) {   // the reduction reads which slots hold data
+        if (args.sched.tail && w.sp == 0) {   // the reduction reads which slots hold data
           const int64_t tile = w.ib + static_cast<int64_t>(args.ni) * w.jt;
           args.tile_segs[tile] = dw_tile_segments(tile, args.sched);
         }

@@ -792,10 +792,10 @@ struct RedJob {
 };
 
 // Whether partial slot sp of tile (ib, jt) was written by the dW kernel: every slot, unless
-// its work was split stream-K (then a tile has as many slots as segments, which the dW kernel
+// its schedule had a tail (then a tail tile has as many slots as parts, which the dW kernel
 // recorded).
 __device__ __forceinline__ bool slot_written(const ReduceArgs& a, int64_t ib, int64_t jt, int sp) {
-  if (!a.sched.stream_k || sp == 0) return true;
+  if (!a.sched.tail || sp == 0) return true;
   const int64_t tile = ib + a.ni * jt;
   return tile >= a.sched.full_tiles && sp < __ldg(a.tile_segs + tile);
 }
@@ -813,7 +813,7 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
   const int64_t e = blk * 32 + lane;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   auto part = [&](int64_t p) { return __ldg(j.part + p * j.n4 + e); };
-  if (e < j.n4 && !a.sched.stream_k) {
+  if (e < j.n4 && !a.sched.tail) {
     int p = w;
     for (; p + 3 * kRedSlices < j.nparts; p += 4 * kRedSlices) {
       const float4 v0 = part(p);
@@ -827,7 +827,7 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
     }
     for (; p < j.nparts; p += kRedSlices) add4(acc, part(p));
   } else if (e < j.n4) {
-    // Stream-K: slot 0 of every tile (always written), spread over the warps, then the further
+    // With a tail: slot 0 of every tile (always written), spread over the warps, then the further
     // slots of the tail's tiles.  Slot p = o * nsplit + sp, o the other tile coordinate (jt for
     // dA, ib for dB); the tile coordinate this element fixes is the same for the whole block.
     const int ns = a.nsplit;
@@ -884,8 +884,8 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
 }
 
 // Sum over the 128-column blocks b = b0, b0 + step, ... < b_end of row i of the parts that the
-// stream-K tail wrote past slot 0 (tiles past the whole ones; their segment count read once per
-// block, the slots' loads issued together).
+// tail wrote past slot 0 (tiles past the whole ones; their part count read once per block, the
+// slots' loads issued together).
 __device__ __forceinline__ float ds_tail_slots(const float* __restrict__ part, int64_t m, int64_t nb, int64_t i,
                                                int64_t b0, int64_t step, const ReduceArgs& a, int64_t b_end = -1) {
   if (b_end < 0) b_end = nb;
@@ -917,14 +917,14 @@ __device__ __forceinline__ void reduce_ds_row(const float* __restrict__ part, in
   const int lane = threadIdx.x & 31;
   if (i >= m) return;
   float acc = 0.0f;
-  // parts p = 2 sp + h (slot sp, column half h); stream-K: slot 0 of every block here, the
+  // parts p = 2 sp + h (slot sp, column half h); with a tail: slot 0 of every block here, the
   // written further slots of the tail's tiles below
-  const int dense = a.sched.stream_k ? 2 : nparts;
+  const int dense = a.sched.tail ? 2 : nparts;
   for (int p = 0; p < dense; ++p) {
     const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
     for (int64_t b = lane; b < nb; b += 32) acc += row[b];
   }
-  if (a.sched.stream_k) acc += ds_tail_slots(part, m, nb, i, lane, 32, a);
+  if (a.sched.tail) acc += ds_tail_slots(part, m, nb, i, lane, 32, a);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
   if (lane == 0) ds[i] = accumulate ? ds[i] + acc : acc;
@@ -940,12 +940,12 @@ __device__ __forceinline__ void reduce_ds_group(const float* __restrict__ part, 
   const int g = static_cast<int>(e % ngroups);
   float acc = 0.0f;
   // parts p = 2 sp + h as in reduce_ds_row
-  const int dense = a.sched.stream_k ? 2 : nparts;
+  const int dense = a.sched.tail ? 2 : nparts;
   for (int p = 0; p < dense; ++p) {
     const float* row = part + (static_cast<int64_t>(p) * m + i) * nb;
     for (int b = g * blocks_per_group; b < (g + 1) * blocks_per_group; ++b) acc += row[b];
   }
-  if (a.sched.stream_k)
+  if (a.sched.tail)
     acc += ds_tail_slots(part, m, nb, i, static_cast<int64_t>(g) * blocks_per_group, 1, a,
                          static_cast<int64_t>(g + 1) * blocks_per_group);
   ds[e] = accumulate ? ds[e] + acc : acc;

@@ -45,33 +45,41 @@ cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int
 // 128 * nchunks columns j; tile = ib + ni * jt) of tsteps 32-token stages each; G and the
 // gradients it feeds (dU, dA, dB, ds) are linear in the tokens, so any token range of a tile
 // can be reduced on its own and its contribution written as one partial slot.
-//   stream_k == 0: every tile is cut into nsplit equal token ranges (units), taken round robin.
-//   stream_k == 1: the first full_tiles tiles (whole waves of `grid`) are taken whole, round
-//     robin, so that the CTAs of a wave read the same token stages of neighbouring tiles; then
-//     CTA b takes the stages [b S / grid, (b + 1) S / grid) of the tile-major sequence of the
-//     remaining tiles' S stages, cut at tile boundaries into segments (the balanced tail); the
-//     segments of a tile write slots 0, 1, ... in CTA order, and the dW kernel records each
-//     tile's segment count in tile_segs for the reduction.
+//   tail == 0: every tile is cut into nsplit equal token ranges (units), taken round robin.
+//   tail == 1: the first full_tiles tiles (whole waves of `grid`) are taken whole, round robin,
+//     so that the CTAs of a wave read the same token stages of neighbouring tiles; then CTA
+//     b < tail_grid takes one part of a remaining tile: each of the tail_tiles tiles is cut into
+//     tail_grid / tail_tiles or one more equal token ranges (parts j = 0, 1, ... write slots
+//     j), so every CTA finishes one segment and the CTAs on neighbouring tiles start at the
+//     same token offsets.  The dW kernel records each tile's part count in tile_segs for the
+//     reduction.
 struct DwSched {
-  int32_t stream_k;
+  int32_t tail;
   int32_t grid;
   int64_t tsteps;        // stages of one tile: ceil(T / 32)
-  int64_t full_tiles;    // tiles taken whole before the balanced tail
-  int64_t total_steps;   // S: stages of the tail
+  int64_t full_tiles;    // tiles taken whole before the tail
+  int64_t tail_tiles;    // tiles cut into parts (<= tail_grid)
+  int64_t tail_grid;     // CTAs that take a tail part
 };
-// The CTA whose tail range holds tail stage g: the largest b with b S / grid <= g.
-__host__ __device__ inline int64_t dw_cta_of(int64_t g, const DwSched& s) {
-  return ((g + 1) * s.grid + s.total_steps - 1) / s.total_steps - 1;
+// CTA b's tail part (b < tail_grid): tail tile t (tile full_tiles + t), part j of q.
+__host__ __device__ inline void dw_tail_part(int64_t b, const DwSched& s, int64_t& t, int& j, int& q) {
+  const int64_t q_lo = s.tail_grid / s.tail_tiles, extra = s.tail_grid % s.tail_tiles;
+  const int64_t wide = extra * (q_lo + 1);   // CTAs of the tiles cut into q_lo + 1 parts
+  if (b < wide) {
+    t = b / (q_lo + 1);
+    j = static_cast<int>(b % (q_lo + 1));
+    q = static_cast<int>(q_lo + 1);
+  } else {
+    t = extra + (b - wide) / q_lo;
+    j = static_cast<int>((b - wide) % q_lo);
+    q = static_cast<int>(q_lo);
+  }
 }
-// First tail stage of CTA b's range.
-__host__ __device__ inline int64_t dw_range_begin(int64_t b, const DwSched& s) {
-  return b * s.total_steps / s.grid;
-}
-// Partial slots a tile's segments write (stream_k == 1).
+// Partial slots a tile's segments write (tail == 1).
 __host__ __device__ inline int dw_tile_segments(int64_t tile, const DwSched& s) {
   if (tile < s.full_tiles) return 1;
-  const int64_t t = tile - s.full_tiles;
-  return static_cast<int>(dw_cta_of((t + 1) * s.tsteps - 1, s) - dw_cta_of(t * s.tsteps, s) + 1);
+  const int64_t q_lo = s.tail_grid / s.tail_tiles, extra = s.tail_grid % s.tail_tiles;
+  return static_cast<int>(tile - s.full_tiles < extra ? q_lo + 1 : q_lo);
 }
 
 // Deterministic sums of the per-tile gradient partials written by the dW kernel.
@@ -83,10 +91,10 @@ struct ReduceArgs {
   int64_t m, k; int r; int group_size;
   float lr;                          // alpha / r
   int accumulate;
-  // which partial slots hold data (all of them unless the dW work was split stream-K)
+  // which partial slots hold data (all of them unless the dW work had a tail, sched.tail)
   DwSched sched;
   int ni, nsplit, bn;                // row blocks, slots per tile, columns per tile
-  const int32_t* tile_segs;          // stream-K: slots written per tile (by the dW kernel)
+  const int32_t* tile_segs;          // tail schedule: slots written per tile (by the dW kernel)
 };
 cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream);
 
@@ -158,7 +166,7 @@ struct DwArgs {
   const void* phi;       // 16-bit bases only: Phi0 [m, k], read directly by the epilogue
   int32_t u_bf16;        // pre-round value in bf16 (lrqat_layer.u_bf16)
   DwSched sched;         // kept last (argument layout)
-  int32_t* tile_segs;    // stream-K: [ni * nj] slots written per tile
+  int32_t* tile_segs;    // tail schedule: [ni * nj] slots written per tile
 };
 int dw_smem_bytes(int r16, int fmt);
 // fmt: a PhiFmt value (quant.cuh)

@@ -290,43 +290,35 @@ DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
   p.nsplit = static_cast<int>((T + p.tchunk - 1) / p.tchunk);   // no empty splits
   p.units = tiles * p.nsplit;
   const int grid_eq = p.units < sms ? p.units : sms;
-  p.sched = DwSched{0, grid_eq, tsteps, 0, 0};
-  // Against whole tiles for the full waves of every SM and a stream-K split of the rest, by the
-  // slowest CTA's cost in stage units: its stages plus kEpilogueStages for each unit or segment
-  // it finishes (the part of the epilogue that the next main loop waits for, ~12K cycles
-  // against ~400 per stage).  The tail needs at least one stage per CTA.
+  p.sched = DwSched{0, grid_eq, tsteps, 0, 0, 0};
+  // Against whole tiles for the full waves of every SM and the remaining tiles cut into equal
+  // token parts, one per CTA (at most 8 parts a tile, none shorter than a stage), by the
+  // slowest CTA's cost in stage units: its stages plus kEpilogueStages for each unit it
+  // finishes (the part of the epilogue that the next main loop waits for).
   constexpr int64_t kEpilogueStages = 32;
   const int64_t waves = (p.units + grid_eq - 1) / grid_eq;
   const int64_t cost_eq = waves * (p.tchunk / 32 + kEpilogueStages);
   const int64_t full_tiles = tiles / sms * sms;
-  const DwSched sk{1, sms, tsteps, full_tiles, (tiles - full_tiles) * tsteps};
-  bool sk_ok = sk.total_steps >= sms;
-  int64_t cost_sk = 0;
-  if (sk_ok) {
-    int64_t max_segs = 0;
-    for (int b = 0; b < sms; ++b) {
-      const int64_t g0 = dw_range_begin(b, sk), g1 = dw_range_begin(b + 1, sk);
-      const int64_t segs = (g1 - 1) / tsteps - g0 / tsteps + 1;
-      if (segs > max_segs) max_segs = segs;
-    }
-    cost_sk = full_tiles / sms * (tsteps + kEpilogueStages) + (sk.total_steps + sms - 1) / sms +
-              kEpilogueStages * max_segs;
+  const int64_t tail_tiles = tiles - full_tiles;
+  const int64_t q_cap = tsteps < 8 ? tsteps : 8;
+  const int64_t tail_grid = tail_tiles * q_cap < sms ? tail_tiles * q_cap : sms;
+  const DwSched tl{1, sms, tsteps, full_tiles, tail_tiles, tail_grid};
+  const bool tail_ok = tail_tiles > 0;
+  int64_t cost_tail = 0;
+  if (tail_ok) {
+    const int64_t q_min = tail_grid / tail_tiles;   // the longest parts
+    cost_tail = full_tiles / sms * (tsteps + kEpilogueStages) + (tsteps + q_min - 1) / q_min + kEpilogueStages;
   }
-  // LRQAT_DW_SCHEDULE=stream_k / split overrides the choice (tests and timing of either schedule)
+  // LRQAT_DW_SCHEDULE=tail / split overrides the choice (tests and timing of either schedule)
   const char* force = std::getenv("LRQAT_DW_SCHEDULE");
-  const bool use_sk = !sk_ok ? false
-                      : force && std::strcmp(force, "stream_k") == 0 ? true
-                      : force && std::strcmp(force, "split") == 0    ? false
-                                                                     : cost_sk < cost_eq;
-  if (use_sk) {
-    int slots = 1;
-    for (int64_t tile = full_tiles; tile < tiles; ++tile) {
-      const int n = dw_tile_segments(tile, sk);
-      if (n > slots) slots = n;
-    }
-    p.sched = sk;
-    p.nsplit = slots;        // partial slots per tile
-    p.tchunk = 0;            // not used
+  const bool use_tail = !tail_ok ? false
+                        : force && std::strcmp(force, "tail") == 0  ? true
+                        : force && std::strcmp(force, "split") == 0 ? false
+                                                                    : cost_tail < cost_eq;
+  if (use_tail) {
+    p.sched = tl;
+    p.nsplit = dw_tile_segments(full_tiles, tl);   // the first tail tile has the most parts
+    p.tchunk = 0;                                  // not used
     p.units = sms;
   }
   return p;

@@ -144,37 +144,26 @@ def test_quantized_activation_entry_points_are_checked_on_host(lib):
     assert "mask" in LQ.last_error()
 
 
-def test_dw_schedule_override_changes_the_partial_slots(lib, monkeypatch):
-    """A 128 x 256 layer over 8192 tokens: equal splits keep at most 8 slots per tile; stream-K
-    over every SM cuts the one tile into a segment per CTA, so its backward workspace (the
-    gradient partials) grows."""
-    L = _layer(m=128, k=256)
-    sizes = {}
-    for sched in ("split", "stream_k"):
-        monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
-        sizes[sched] = lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192)
-    assert sizes["stream_k"] > 4 * sizes["split"] > 0
-
-
 def test_dw_schedule_choice_of_the_cost_model(lib, monkeypatch):
     """The plan without the override (152 SMs assumed when no GPU is present):
-      - 4096 x 4096 at 8192 tokens, 512 tiles: whole-tile waves (3 x 152) and a stream-K tail
-        of 56 tiles beat two equal token splits per tile (4 partial slots per tile against 2);
-      - 2432 x 2048 at 8192 tokens, exactly 152 tiles: one wave of whole tiles, nothing left
-        for a tail, so equal splits are taken and the stream-K override cannot apply;
-      - 384 x 512 at 1000 tokens, 6 tiles: a stream-K split keeps all SMs busy (1-2 stages
-        each against 8 stages on 24 SMs), so it is taken.
+      - 4096 x 4096 at 8192 tokens, 512 tiles: whole-tile waves (3 x 152) and the 56 remaining
+        tiles cut into 2 or 3 token parts, one per CTA, beat two equal token splits per tile
+        (3 partial slots per tile against 2);
+      - 2432 x 2048 at 8192 tokens, exactly 152 tiles: one wave of whole tiles, no tail, so equal
+        splits are taken and the tail override cannot apply;
+      - 384 x 512 at 1000 tokens, 6 tiles: 8 parts a tile keep 48 SMs busy with 4 stages each,
+        against 24 SMs with 8 stages each, so the tail schedule is taken (8 slots against 4).
     The backward workspace sizes (the partial slots) show which plan was made."""
     cases = {"big": (_layer(m=4096, k=4096, r=32, alpha=32.0), 8192),
              "waves": (_layer(m=2432, k=2048, r=32, alpha=32.0), 8192),
              "tiny": (_layer(m=384, k=512, r=32, alpha=32.0), 1000)}
     sizes = {}
-    for sched in (None, "split", "stream_k"):
+    for sched in (None, "split", "tail"):
         if sched is None:
             monkeypatch.delenv("LRQAT_DW_SCHEDULE", raising=False)
         else:
             monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
         sizes[sched] = {n: lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), T) for n, (L, T) in cases.items()}
-    assert sizes[None]["big"] == sizes["stream_k"]["big"] > sizes["split"]["big"]
-    assert sizes[None]["waves"] == sizes["split"]["waves"] == sizes["stream_k"]["waves"]
-    assert sizes[None]["tiny"] == sizes["stream_k"]["tiny"] > sizes["split"]["tiny"]
+    assert sizes[None]["big"] == sizes["tail"]["big"] > sizes["split"]["big"]
+    assert sizes[None]["waves"] == sizes["split"]["waves"] == sizes["tail"]["waves"]
+    assert sizes[None]["tiny"] == sizes["tail"]["tiny"] > sizes["split"]["tiny"]

@@ -312,9 +312,9 @@ def test_quantized_activation_entry_points_bit_identical(cid, spec, T, sx_factor
         assert (bits_to_f32(b["dX"]) == 0).mean() > 0.01   # the clip mask was applied
 
 
-# Shapes with at least one 32-token stage per CTA in the stream-K tail (tiles x stages >= 152),
-# ragged token counts; the last case has a full wave of whole tiles (160 tiles) before its tail.
-STREAM_K_CASES = [
+# Ragged token counts; every tile is a tail tile (cut into token parts) except in the last case,
+# which has a full wave of whole tiles (160 tiles) before its tail.
+TAIL_CASES = [
     ("q44_pc", spec_of("a", 384, 512, 32), 1000),
     ("int3_packed", spec_of("d", 256, 512, 32, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.2, b_std=0.2), 1500),
     ("q44_g128_a8", spec_of("f", 256, 384, 16, group=128, act=8, a_std=0.2, b_std=0.2), 1700),
@@ -325,13 +325,13 @@ STREAM_K_CASES = [
 ]
 
 
-@pytest.mark.parametrize("cid,spec,T", STREAM_K_CASES, ids=[c[0] for c in STREAM_K_CASES])
-def test_fwd_bwd_parity_stream_k_dw(cid, spec, T, monkeypatch):
-    """The dW work split stream-K (whole tiles for the full waves, then each CTA an equal range
-    of the remaining 32-token stages, a tile's token ranges reduced as separate partial slots),
-    forced on shapes whose cost model picks equal splits: ragged token tails inside segments,
-    tiles cut across many CTAs, and slots that no segment writes."""
-    monkeypatch.setenv("LRQAT_DW_SCHEDULE", "stream_k")
+@pytest.mark.parametrize("cid,spec,T", TAIL_CASES, ids=[c[0] for c in TAIL_CASES])
+def test_fwd_bwd_parity_tail_dw(cid, spec, T, monkeypatch):
+    """The dW work with a tail (whole tiles for the full waves, then the remaining tiles cut
+    into up to 8 equal token parts, one per CTA, each reduced as its own partial slot), forced
+    on shapes whose cost model may pick equal splits: ragged token tails inside parts, tiles
+    with different part counts, and slots that no part writes."""
+    monkeypatch.setenv("LRQAT_DW_SCHEDULE", "tail")
     got, ref, _ = _run(spec, T, seed=2, s_scale=1.05)
     errs = {k: O.rel_fro(got[k], ref[k]) for k in got}
     assert errs["Y"] <= TOL_ACT and errs["dX"] <= TOL_ACT, errs
@@ -339,16 +339,16 @@ def test_fwd_bwd_parity_stream_k_dw(cid, spec, T, monkeypatch):
 
 
 def test_dw_schedules_agree(monkeypatch):
-    """Equal token splits and stream-K give the same Y and dX bit for bit and the same gradients
+    """Equal token splits and the tail schedule give the same Y and dX bit for bit and the same gradients
     up to rounding: ds up to fp32 summation order; dA and dB also up to the bf16 rounding of
     dU, which the epilogue applies per token range (about 2^-9 relative)."""
     spec = spec_of("sk", 256, 512, 32, group=128, a_std=0.2, b_std=0.2)
     outs = {}
-    for sched in ("split", "stream_k"):
+    for sched in ("split", "tail"):
         monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
         outs[sched], _, _ = _run(spec, 1555, seed=3)
     for key in ("Y", "dX"):
-        np.testing.assert_array_equal(outs["split"][key], outs["stream_k"][key])
-    assert O.rel_fro(outs["stream_k"]["ds"], outs["split"]["ds"]) <= 1e-5
+        np.testing.assert_array_equal(outs["split"][key], outs["tail"][key])
+    assert O.rel_fro(outs["tail"]["ds"], outs["split"]["ds"]) <= 1e-5
     for key in ("dA", "dB"):
-        assert O.rel_fro(outs["stream_k"][key], outs["split"][key]) <= 1e-2, key
+        assert O.rel_fro(outs["tail"][key], outs["split"][key]) <= 1e-2, key
