@@ -206,9 +206,9 @@ size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
  * over micro-batches).  dX is always overwritten.
  * workspace: device buffer of at least lrqat_bwd_workspace_bytes() bytes.
  * The weight-gradient work is spread over the SMs either as equal token splits of
- * every tile or as whole tiles followed by a balanced (stream-K) split of the rest,
- * chosen per call; the environment variable LRQAT_DW_SCHEDULE = "split" or
- * "stream_k" forces one (read by lrqat_bwd_workspace_bytes and lrqat_linear_bwd
+ * every tile or as whole tiles followed by the remaining tiles cut into token
+ * parts, one per SM, chosen per call; the environment variable LRQAT_DW_SCHEDULE =
+ * "split" or "tail" forces one (read by lrqat_bwd_workspace_bytes and lrqat_linear_bwd
  * alike, so keep it fixed between the two).  Both give the same dX bit for bit and
  * the same dA, dB, ds up to rounding order. */
 int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X,
