@@ -834,7 +834,7 @@ __device__ __forceinline__ void reduce_parts_block(const RedJob& j, int64_t blk,
     const int64_t n_other = j.nparts / ns;
     const int64_t fixed = j.kind == 0 ? (4 * e / j.width) / 128 : ((4 * e) % j.width) / a.bn;
     // first o whose tile (fixed + ni o for dA, o + ni fixed for dB) is past the whole tiles;
-    // this warp's first tail tile's segment count is requested before the slot-0 loads
+    // this warp's first tail tile's part count is requested before the slot-0 loads
     const int64_t ft = a.sched.full_tiles;
     const int64_t o_tail = j.kind == 0 ? (ft > fixed ? (ft - fixed + a.ni - 1) / a.ni : 0)
                                        : (ft > a.ni * fixed ? ft - a.ni * fixed : 0);
