@@ -207,10 +207,8 @@ size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
  * workspace: device buffer of at least lrqat_bwd_workspace_bytes() bytes.
  * The weight-gradient work is spread over the SMs either as equal token splits of
  * every tile or as whole tiles followed by the remaining tiles cut into token
- * parts, one per SM, chosen per call; the environment variable LRQAT_DW_SCHEDULE =
- * "split" or "tail" forces one (read by lrqat_bwd_workspace_bytes and lrqat_linear_bwd
- * alike, so keep it fixed between the two).  Both give the same dX bit for bit and
- * the same dA, dB, ds up to rounding order. */
+ * parts, one per SM, chosen per call unless lrqat_set_dw_schedule forces one.  Both
+ * give the same dX bit for bit and the same dA, dB, ds up to rounding order. */
 int lrqat_linear_bwd(const lrqat_layer* layer, int64_t T, const uint16_t* dY, const uint16_t* X,
                      const void* Phi0, const float* s, const uint16_t* A, const uint16_t* B,
                      const float* s_x, uint16_t* dX, float* dA, float* dB, float* ds, int accumulate,
@@ -290,6 +288,17 @@ int lrqat_grad_sqnorm(const lrqat_layer* layer, const float* dA, const float* dB
 int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const float* sqnorm, const float* dA,
                      const float* dB, const float* ds, const lrqat_adamw_state* state, float* s, uint16_t* A,
                      uint16_t* B, lrqat_stream_t stream);
+
+/* Tuning (no counterpart in the paper): the schedule of the weight-gradient work of
+ * lrqat_linear_bwd.  0 = chosen per call by a cost model (the default), 1 = equal token
+ * splits of every tile, 2 = whole tiles followed by the remaining tiles cut into token
+ * parts (falls back to 1 when every SM gets the same number of whole tiles).  The
+ * setting is process-wide and changes the size lrqat_bwd_workspace_bytes reports, so
+ * set it before querying sizes and keep it while those workspaces are in use.  The
+ * environment variable LRQAT_DW_SCHEDULE ("split" or "tail") gives the start value; it
+ * is read once, when the library is loaded.  Returns LRQAT_ERR_INVALID_ARG for other
+ * values. */
+int lrqat_set_dw_schedule(int schedule);
 
 /* Synchronizes `stream`, then reads and clears the device status word of the
  * current device.  Returns LRQAT_OK, LRQAT_ERR_TIMEOUT (a kernel's bounded

@@ -494,13 +494,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 template <int FMT, bool ZP, bool UB>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t err =
-        cudaFuncSetAttribute(dw_kernel<FMT, ZP, UB>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-    if (err != cudaSuccess) return err;
-    configured = true;
-  }
+  static bool configured[kMaxDevices] = {};
+  const cudaError_t err = ensure_smem_attr(reinterpret_cast<const void*>(dw_kernel<FMT, ZP, UB>),
+                                           static_cast<int>(SMEM_BYTES), configured);
+  if (err != cudaSuccess) return err;
   dw_kernel<FMT, ZP, UB><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
   return cudaGetLastError();
 }

@@ -990,8 +990,9 @@ cudaError_t launch_range_lp(const float* W0, int64_t m, int64_t k, int group_siz
   const size_t smem = static_cast<size_t>(seg) * 4;
   if (n_cand < 1 || n_cand > kThreads || smem > 200 * 1024) return cudaErrorInvalidValue;
   if (smem > 48 * 1024) {
-    const cudaError_t e = cudaFuncSetAttribute(range_lp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               static_cast<int>(smem));
+    // the largest row or group any call may need (200 KB), set once per device
+    static bool configured[kMaxDevices] = {};
+    const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(range_lp_kernel), 200 * 1024, configured);
     if (e != cudaSuccess) return e;
   }
   range_lp_kernel<<<static_cast<unsigned>(m * ngroups), kThreads, smem, stream>>>(W0, k, seg, ngroups, bits, p_norm,

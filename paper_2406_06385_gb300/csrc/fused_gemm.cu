@@ -512,13 +512,10 @@ template <int MODE, int FMT, bool ZP, bool UB>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const FusedArgs& args, int grid, cudaStream_t stream) {
   constexpr uint32_t smem = FactorRing<FMT>::SMEM_BYTES;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(fused_gemm_kernel<MODE, FMT, ZP, UB>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static bool configured[kMaxDevices] = {};
+  const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(fused_gemm_kernel<MODE, FMT, ZP, UB>),
+                                         static_cast<int>(smem), configured);
+  if (e != cudaSuccess) return e;
   fused_gemm_kernel<MODE, FMT, ZP, UB><<<grid, NUM_THREADS, smem, stream>>>(a, b, c, d, args);
   return cudaGetLastError();
 }

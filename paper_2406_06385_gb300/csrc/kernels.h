@@ -10,6 +10,25 @@
 
 namespace lrqat {
 
+// Devices a process may use with the library (ordinals 0 .. kMaxDevices - 1).
+constexpr int kMaxDevices = 64;
+
+// Raises a kernel's dynamic shared-memory limit to `bytes` on the current device,
+// once per device: the attribute belongs to the device's context, so a process
+// that uses several devices sets it on each.  `done` has kMaxDevices entries.
+inline cudaError_t ensure_smem_attr(const void* kernel, int bytes, bool* done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  if (!done[dev]) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  return cudaSuccess;
+}
+
 // ---- elementwise.cu --------------------------------------------------------
 // z0 == nullptr: symmetric range setting (s0 only); else asymmetric (s0 and zero offsets z0).
 cudaError_t launch_range_minmax(const float* W0, int64_t m, int64_t k, int group_size, int bits, float* s0,

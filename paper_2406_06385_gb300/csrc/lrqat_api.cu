@@ -4,6 +4,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdint>
@@ -25,7 +26,6 @@ namespace {
 __device__ int g_device_status;
 
 constexpr uint64_t kWaitTimeoutNs = 2000000000ull;   // 2 s per wait
-constexpr int kMaxDevices = 64;
 
 thread_local std::string t_last_error;
 
@@ -260,6 +260,18 @@ struct Carver {
 };
 
 // ----------------------------------------------------------------- planning --
+// Schedule of the weight-gradient work: 0 = chosen per call by the cost model below,
+// 1 = equal token splits, 2 = whole tiles and a tail.  The environment variable
+// LRQAT_DW_SCHEDULE ("split" / "tail") sets the start value once, when the library is
+// loaded; lrqat_set_dw_schedule changes it explicitly.
+int dw_schedule_from_env() {
+  const char* v = std::getenv("LRQAT_DW_SCHEDULE");
+  if (v && std::strcmp(v, "split") == 0) return 1;
+  if (v && std::strcmp(v, "tail") == 0) return 2;
+  return 0;
+}
+std::atomic<int> g_dw_schedule{dw_schedule_from_env()};
+
 struct DwPlan {
   int nchunks, ni, nj, nsplit, tchunk, units;
   DwSched sched;
@@ -309,12 +321,9 @@ DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
     const int64_t q_min = tail_grid / tail_tiles;   // the longest parts
     cost_tail = full_tiles / sms * (tsteps + kEpilogueStages) + (tsteps + q_min - 1) / q_min + kEpilogueStages;
   }
-  // LRQAT_DW_SCHEDULE=tail / split overrides the choice (tests and timing of either schedule)
-  const char* force = std::getenv("LRQAT_DW_SCHEDULE");
-  const bool use_tail = !tail_ok ? false
-                        : force && std::strcmp(force, "tail") == 0  ? true
-                        : force && std::strcmp(force, "split") == 0 ? false
-                                                                    : cost_tail < cost_eq;
+  // a forced schedule (lrqat_set_dw_schedule) overrides the choice; the tail needs tail tiles
+  const int force = g_dw_schedule.load(std::memory_order_relaxed);
+  const bool use_tail = !tail_ok ? false : force == 2 ? true : force == 1 ? false : cost_tail < cost_eq;
   if (use_tail) {
     p.sched = tl;
     p.nsplit = dw_tile_segments(full_tiles, tl);   // the first tail tile has the most parts
@@ -661,7 +670,11 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   if (!A) return fail(LRQAT_ERR_INVALID_ARG, "A is NULL");
   if (!B) return fail(LRQAT_ERR_INVALID_ARG, "B is NULL");
   LRQAT_CHECK_PTR(dX, "dX");
-  if (!dA || !dB || !ds) return fail(LRQAT_ERR_INVALID_ARG, "dA, dB and ds must not be NULL");
+  // the gradient reduction reads and writes dA and dB with 16-byte accesses; ds is written
+  // as scalars
+  LRQAT_CHECK_PTR(dA, "dA");
+  LRQAT_CHECK_PTR(dB, "dB");
+  if (!ds) return fail(LRQAT_ERR_INVALID_ARG, "ds is NULL");
   if (L.act_bits == 8 && !L.act_per_token && !s_x)
     return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8 (per-tensor scale)");
   DeviceInfo* dev = nullptr;
@@ -925,6 +938,12 @@ int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const flo
   a.max_norm = opt->max_grad_norm;
   a.sqnorm = sqnorm;
   LRQAT_LAUNCH("adamw", 1, stream, launch_adamw(a, stream), "AdamW launch");
+  return LRQAT_OK;
+}
+
+int lrqat_set_dw_schedule(int schedule) {
+  if (schedule < 0 || schedule > 2) return fail(LRQAT_ERR_INVALID_ARG, "dW schedule must be 0, 1 or 2 (got %d)", schedule);
+  g_dw_schedule.store(schedule, std::memory_order_relaxed);
   return LRQAT_OK;
 }
 

@@ -163,13 +163,10 @@ __global__ void __launch_bounds__(128) merge_tc_kernel(const __grid_constant__ C
 template <int FMT, bool UB>
 cudaError_t launch_merge_one(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const MergeArgs& args,
                              cudaStream_t stream) {
-  static bool configured = false;
-  if (!configured) {
-    const cudaError_t e = cudaFuncSetAttribute(merge_tc_kernel<FMT, UB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static bool configured[kMaxDevices] = {};
+  const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(merge_tc_kernel<FMT, UB>),
+                                         static_cast<int>(SMEM_BYTES), configured);
+  if (e != cudaSuccess) return e;
   dim3 grid(static_cast<unsigned>(args.k / 128), static_cast<unsigned>(args.m / 128));
   merge_tc_kernel<FMT, UB><<<grid, 128, SMEM_BYTES, stream>>>(tm_a, tm_b, args);
   return cudaGetLastError();

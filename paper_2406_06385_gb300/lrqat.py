@@ -96,6 +96,8 @@ def lib() -> ctypes.CDLL:
             fn = getattr(L, name)
             fn.argtypes = args
             fn.restype = ctypes.c_int
+        L.lrqat_set_dw_schedule.argtypes = [ip]
+        L.lrqat_set_dw_schedule.restype = ctypes.c_int
         L.lrqat_trace_enable.argtypes = [ip]
         L.lrqat_trace_enable.restype = ctypes.c_int
         L.lrqat_trace_read.argtypes = [ip, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_int64),
@@ -211,6 +213,14 @@ def adamw_step(layer: Layer, opt: AdamW, sqnorm, dA, dB, ds, state: dict, s, A, 
 
 def get_device_status(stream=None) -> None:
     _check(lib().lrqat_get_device_status(_stream(stream)))
+
+
+DW_SCHEDULES = {"auto": 0, "split": 1, "tail": 2}
+
+
+def set_dw_schedule(schedule: str) -> None:
+    """Process-wide schedule of the weight-gradient work: "auto", "split" or "tail"."""
+    _check(lib().lrqat_set_dw_schedule(DW_SCHEDULES[schedule]))
 
 
 def trace_enable(enable: bool = True) -> None:

@@ -10,3 +10,12 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA device (GB300, sm_103a) and the built library")
+
+
+@pytest.fixture
+def dw_schedule():
+    """Forces the schedule of the weight-gradient work for one test ("split" or "tail")
+    and restores the per-call choice afterwards."""
+    from paper_2406_06385_gb300 import lrqat as LQ
+    yield LQ.set_dw_schedule
+    LQ.set_dw_schedule("auto")

@@ -144,8 +144,8 @@ def test_quantized_activation_entry_points_are_checked_on_host(lib):
     assert "mask" in LQ.last_error()
 
 
-def test_dw_schedule_choice_of_the_cost_model(lib, monkeypatch):
-    """The plan without the override (152 SMs assumed when no GPU is present):
+def test_dw_schedule_choice_of_the_cost_model(lib, dw_schedule):
+    """The plan without an override (152 SMs assumed when no GPU is present):
       - 4096 x 4096 at 8192 tokens, 512 tiles: whole-tile waves (3 x 152) and the 56 remaining
         tiles cut into 2 or 3 token parts, one per CTA, beat two equal token splits per tile
         (3 partial slots per tile against 2);
@@ -158,12 +158,46 @@ def test_dw_schedule_choice_of_the_cost_model(lib, monkeypatch):
              "waves": (_layer(m=2432, k=2048, r=32, alpha=32.0), 8192),
              "tiny": (_layer(m=384, k=512, r=32, alpha=32.0), 1000)}
     sizes = {}
-    for sched in (None, "split", "tail"):
-        if sched is None:
-            monkeypatch.delenv("LRQAT_DW_SCHEDULE", raising=False)
-        else:
-            monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
+    for sched in ("auto", "split", "tail"):
+        dw_schedule(sched)
         sizes[sched] = {n: lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), T) for n, (L, T) in cases.items()}
-    assert sizes[None]["big"] == sizes["tail"]["big"] > sizes["split"]["big"]
-    assert sizes[None]["waves"] == sizes["split"]["waves"] == sizes["tail"]["waves"]
-    assert sizes[None]["tiny"] == sizes["tail"]["tiny"] > sizes["split"]["tiny"]
+    assert sizes["auto"]["big"] == sizes["tail"]["big"] > sizes["split"]["big"]
+    assert sizes["auto"]["waves"] == sizes["split"]["waves"] == sizes["tail"]["waves"]
+    assert sizes["auto"]["tiny"] == sizes["tail"]["tiny"] > sizes["split"]["tiny"]
+    assert lib.lrqat_set_dw_schedule(3) == -1 and lib.lrqat_set_dw_schedule(-1) == -1
+
+
+def test_dw_schedule_environment_is_read_once_at_load(lib, dw_schedule, monkeypatch):
+    """LRQAT_DW_SCHEDULE sets the start value when the library is loaded; changing the
+    environment afterwards changes no workspace size (so a size query and the call that
+    uses it always agree)."""
+    L = _layer(m=4096, k=4096, r=32, alpha=32.0)
+    dw_schedule("auto")
+    before = lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192)
+    monkeypatch.setenv("LRQAT_DW_SCHEDULE", "split")
+    assert lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192) == before
+    dw_schedule("split")
+    split = lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192)
+    assert split < before
+    # a fresh process that loads the library with the variable set starts from it
+    code = ("import ctypes, sys; sys.path.insert(0, %r); from paper_2406_06385_gb300 import lrqat as LQ; "
+            "L = LQ.Layer(4096, 4096, 32, 32.0, 4, 0, 0, 0); "
+            "print(LQ.lib().lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192))" % ROOT)
+    import subprocess
+    import sys
+    env = dict(os.environ, LRQAT_DW_SCHEDULE="split")
+    out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=120)
+    assert out.returncode == 0, out.stderr
+    assert int(out.stdout.strip()) == split
+
+
+def test_gradient_outputs_must_be_16_byte_aligned(lib):
+    """The gradient reduction reads and writes dA and dB with 16-byte accesses, so an
+    unaligned dA or dB is rejected on the host before any launch (ds may be unaligned)."""
+    L = _layer()
+    f = lambda dA, dB, ds: lib.lrqat_linear_bwd(ctypes.byref(L), 64, 16, 16, 16, 16, 16, 16, None, 16, dA, dB, ds, 0,
+                                                16, 1 << 30, None)
+    assert f(20, 16, 16) == -3 and "dA" in LQ.last_error()
+    assert f(16, 20, 16) == -3 and "dB" in LQ.last_error()
+    assert f(16, 16, None) == -1
+    assert f(None, 16, 16) == -1

@@ -97,3 +97,24 @@ def test_warmup_below_three_is_rejected():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--warmup", "2"],
                        capture_output=True, text=True, timeout=120, cwd=ROOT)
     assert r.returncode != 0
+
+
+def test_peak_kind_follows_the_clock_record():
+    """Burst peak at full clock without the power cap; sustained otherwise."""
+    assert bench.peak_kind({"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": []}) == "burst"
+    assert bench.peak_kind({"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"]}) == "sustained"
+    assert bench.peak_kind({"sm_mhz": 1462.0, "sm_max_mhz": 2070.0, "reasons": []}) == "sustained"
+    assert bench.peak_kind({"sm_mhz": None, "sm_max_mhz": None, "reasons": []}) == "burst"
+
+
+def test_algorithmic_bytes_of_a_gemm_launch():
+    """Two bf16 token operands of T rows, the stored base once (int8 here) and the adapters."""
+    from paper_2406_06385_gb300 import workloads as WL
+    spec = WL.workload("llama2_7b_attn").layers[0]
+    T = 8192
+    assert bench.kernel_bytes(T, spec) == 2 * T * 8192 + 4096 * 4096 + 2 * 32 * 8192
+
+
+def test_single_thread_baseline_child_runs_on_one_core():
+    d = bench.cpu_baseline_single_thread("tiny", budget_s=0.5)
+    assert d["cores"] == 1 and d["value"] > 0 and d["kind"] == "oracle", d

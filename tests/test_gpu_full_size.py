@@ -1,6 +1,7 @@
 """GPU parity at the benchmark's full sizes, in the launch configuration that
 bench.py times: one lrqat_linear_fwd and one lrqat_linear_bwd call over all
-T = 8192 tokens of a LLaMA-shaped layer.
+T tokens of a LLaMA-shaped layer (T = 16384 for the three projection shapes of
+the LLaMA-2-13B decoder layer, 8192 for the others).
 
 The oracle cannot redo a full 8192-token layer in a test's time, so it checks
 what it can compute exactly, one piece at a time:
@@ -13,8 +14,15 @@ what it can compute exactly, one piece at a time:
   * every code of W_Z from lrqat_merge at the largest merged projection.
 Sampled outputs are compared with the same relative Frobenius tolerances as the
 small-size tests (1e-2 for Y and dX, 2e-2 for the adapter and scale gradients).
+
+Every case reports what it found, pass or fail: the number of codes checked, the
+near-tie exemptions and mismatches, and the five relative errors, as one JSON line
+on stdout (shown by `pytest -rA`) and, when LRQAT_PARITY_REPORT names a file,
+appended to it.
 """
 import dataclasses
+import json
+import os
 
 import numpy as np
 import pytest
@@ -29,20 +37,35 @@ pytestmark = pytest.mark.gpu
 
 TOL_ACT = 1e-2
 TOL_GRAD = 2e-2
-T_FULL = 8192
 
-# The bench layer (4096 x 4096, Q4.4 per channel), the largest projection of the
-# W4 g128 + A8 MLP (14336 x 4096), the INT-3 packed down projection (4096 x 11008),
-# and the 4096 x 4096 layer with asymmetric W2, per-token A8, and BF16 / FP8 bases.
+# The three projection shapes of the LLaMA-2-13B decoder layer that bench.py times by
+# default (q/k/v/o 5120 x 5120, gate/up 13824 x 5120, down 5120 x 13824; T = 16384), the
+# 4096 x 4096 layer (Q4.4 per channel), the largest projection of the W4 g128 + A8 MLP
+# (14336 x 4096), the INT-3 packed down projection (4096 x 11008), and the 4096 x 4096
+# layer with asymmetric W2, per-token A8, and BF16 / FP8 bases (T = 8192).
+_L13 = WL.workload("llama2_13b_layer")
 FULL_CASES = [
-    ("llama2_7b_attn", WL.workload("llama2_7b_attn").layers[0]),
-    ("llama3_8b_gate_g128_a8", WL.workload("llama3_8b_mlp").layers[0]),
-    ("llama2_7b_down_int3", WL.workload("llama2_7b_mlp").layers[2]),
-    ("llama2_7b_attn_int2_asym", WL.workload("llama2_7b_attn_int2").layers[0]),
-    ("llama2_7b_attn_w4a8_token", WL.workload("llama2_7b_attn_w4a8").layers[0]),
-    ("llama2_7b_attn_phi_bf16", WL.workload("llama2_7b_attn_phi_bf16").layers[0]),
-    ("llama2_7b_attn_phi_fp8", WL.workload("llama2_7b_attn_phi_fp8").layers[0]),
+    ("llama2_13b_qkvo", _L13.layers[0], _L13.tokens),
+    ("llama2_13b_gate", _L13.layers[4], _L13.tokens),
+    ("llama2_13b_down", _L13.layers[6], _L13.tokens),
+    ("llama2_7b_attn", WL.workload("llama2_7b_attn").layers[0], 8192),
+    ("llama3_8b_gate_g128_a8", WL.workload("llama3_8b_mlp").layers[0], 8192),
+    ("llama2_7b_down_int3", WL.workload("llama2_7b_mlp").layers[2], 8192),
+    ("llama2_7b_attn_int2_asym", WL.workload("llama2_7b_attn_int2").layers[0], 8192),
+    ("llama2_7b_attn_w4a8_token", WL.workload("llama2_7b_attn_w4a8").layers[0], 8192),
+    ("llama2_7b_attn_phi_bf16", WL.workload("llama2_7b_attn_phi_bf16").layers[0], 8192),
+    ("llama2_7b_attn_phi_fp8", WL.workload("llama2_7b_attn_phi_fp8").layers[0], 8192),
 ]
+
+
+def _report(test: str, cid: str, **fields):
+    """One JSON line per case: on stdout and, with LRQAT_PARITY_REPORT set, in that file."""
+    line = json.dumps(dict(test=test, case=cid, **fields), sort_keys=True)
+    print(line)
+    path = os.environ.get("LRQAT_PARITY_REPORT")
+    if path:
+        with open(path, "a") as f:
+            f.write(line + "\n")
 
 
 def _oracle_base(data, OL):
@@ -61,8 +84,8 @@ def _codes_spec(spec):
                         spec.w_row_shift, False)
 
 
-@pytest.mark.parametrize("cid,spec", FULL_CASES, ids=[c[0] for c in FULL_CASES])
-def test_full_size_codes_bit_exact(cid, spec):
+@pytest.mark.parametrize("cid,spec,T", FULL_CASES, ids=[c[0] for c in FULL_CASES])
+def test_full_size_codes_bit_exact(cid, spec, T):
     t = torch()
     spec = _codes_spec(spec)
     data = WL.make_layer(spec, 1, seed=3, with_activations=False)
@@ -93,15 +116,16 @@ def test_full_size_codes_bit_exact(cid, spec):
     u = O.preround(phi0, data.A, data.B, OL)
     c = O.codes_from_u(u, OL)[1] - O.expand_zero(z0, OL)   # the operand holds c - z
     exempt = O.near_tie(u)
-    for name, got in (("fwd", c_fwd), ("dX", c_dx)):
-        bad = (got != c) & ~exempt
-        assert bad.sum() == 0, f"{name}: {bad.sum()} code mismatches of {c.size} (near-ties exempt: {exempt.sum()})"
+    bad = {name: int(((got != c) & ~exempt).sum()) for name, got in (("fwd", c_fwd), ("dX", c_dx))}
+    _report("codes", cid, codes=int(c.size), near_tie_exempt=int(exempt.sum()), mismatches_fwd=bad["fwd"],
+            mismatches_dx=bad["dX"], differ_at_exempt=int(((c_fwd != c) & exempt).sum()))
+    for name, n in bad.items():
+        assert n == 0, f"{name}: {n} code mismatches of {c.size} (near-ties exempt: {exempt.sum()})"
 
 
-@pytest.mark.parametrize("cid,spec", FULL_CASES, ids=[c[0] for c in FULL_CASES])
-def test_full_size_sampled_outputs(cid, spec):
+@pytest.mark.parametrize("cid,spec,T", FULL_CASES, ids=[c[0] for c in FULL_CASES])
+def test_full_size_sampled_outputs(cid, spec, T):
     t = torch()
-    T = T_FULL
     data = WL.make_layer(spec, T, seed=11)
     dl = DeviceLayer(data)
     L = dl.layer
@@ -140,8 +164,7 @@ def test_full_size_sampled_outputs(cid, spec):
     dX_ref = (dYf[ts] @ fq["W_hat"]) * Mx[ts]
     Y_got = bits_to_f32(Y[t.as_tensor(ts, device="cuda")])
     dX_got = bits_to_f32(dX[t.as_tensor(ts, device="cuda")])
-    assert O.rel_fro(Y_got, Y_ref) <= TOL_ACT
-    assert O.rel_fro(dX_got, dX_ref) <= TOL_ACT
+    errs = {"Y": O.rel_fro(Y_got, Y_ref), "dX": O.rel_fro(dX_got, dX_ref)}
 
     # dA and ds at sampled weight rows: rows of G, dU and the codes
     rows = WL.token_sample(spec.m, 6, seed=2)
@@ -153,8 +176,8 @@ def test_full_size_sampled_outputs(cid, spec):
     ds_ref = Gc.sum(axis=1) if spec.group_size == 0 else Gc.reshape(len(rows), -1, spec.group_size).sum(axis=2)
     dA_got = dA.cpu().numpy()[rows]
     ds_got = ds.cpu().numpy().reshape((spec.m, -1) if spec.group_size else (spec.m,))[rows]
-    assert O.rel_fro(dA_got, dA_ref) <= TOL_GRAD
-    assert O.rel_fro(ds_got, ds_ref) <= TOL_GRAD
+    errs["dA"] = O.rel_fro(dA_got, dA_ref)
+    errs["ds"] = O.rel_fro(ds_got, ds_ref)
 
     # dB at sampled weight columns: columns of G and dU
     cols = WL.token_sample(spec.k, 6, seed=3)
@@ -162,7 +185,13 @@ def test_full_size_sampled_outputs(cid, spec):
     dU_cols = G_cols * O.expand_scale(s0, OL)[:, cols] * fq["M"][:, cols]
     dB_ref = scale * (data.A.astype(np.float64).T @ dU_cols)
     dB_got = dB.cpu().numpy()[:, cols]
-    assert O.rel_fro(dB_got, dB_ref) <= TOL_GRAD
+    errs["dB"] = O.rel_fro(dB_got, dB_ref)
+    _report("sampled_outputs", cid, T=T, rel_err=errs, token_rows=len(ts), weight_rows=len(rows),
+            weight_cols=len(cols))
+    for key in ("Y", "dX"):
+        assert errs[key] <= TOL_ACT, errs
+    for key in ("dA", "dB", "ds"):
+        assert errs[key] <= TOL_GRAD, errs
 
 
 # The merge of the largest projection of the 13B layer that bench.py times with merge
@@ -197,5 +226,7 @@ def test_full_size_merge_bit_exact(cid, spec):
     ref = O.merge(phi0, data.A, data.B, OL)
     exempt = O.near_tie(O.preround(phi0, data.A, data.B, OL))
     bad = (got != ref) & ~exempt
+    _report("merge", cid, codes=int(ref.size), near_tie_exempt=int(exempt.sum()), mismatches=int(bad.sum()),
+            differ_at_exempt=int(((got != ref) & exempt).sum()))
     assert bad.sum() == 0, f"{bad.sum()} code mismatches of {ref.size} (near-ties exempt: {exempt.sum()})"
     assert (ref != O.merge(phi0, data.A, np.zeros_like(data.B), OL)).mean() > 0.1   # the low-rank term matters

@@ -326,26 +326,26 @@ TAIL_CASES = [
 
 
 @pytest.mark.parametrize("cid,spec,T", TAIL_CASES, ids=[c[0] for c in TAIL_CASES])
-def test_fwd_bwd_parity_tail_dw(cid, spec, T, monkeypatch):
+def test_fwd_bwd_parity_tail_dw(cid, spec, T, dw_schedule):
     """The dW work with a tail (whole tiles for the full waves, then the remaining tiles cut
     into up to 8 equal token parts, one per CTA, each reduced as its own partial slot), forced
     on shapes whose cost model may pick equal splits: ragged token tails inside parts, tiles
     with different part counts, and slots that no part writes."""
-    monkeypatch.setenv("LRQAT_DW_SCHEDULE", "tail")
+    dw_schedule("tail")
     got, ref, _ = _run(spec, T, seed=2, s_scale=1.05)
     errs = {k: O.rel_fro(got[k], ref[k]) for k in got}
     assert errs["Y"] <= TOL_ACT and errs["dX"] <= TOL_ACT, errs
     assert errs["dA"] <= TOL_GRAD and errs["dB"] <= TOL_GRAD and errs["ds"] <= TOL_GRAD, errs
 
 
-def test_dw_schedules_agree(monkeypatch):
+def test_dw_schedules_agree(dw_schedule):
     """Equal token splits and the tail schedule give the same Y and dX bit for bit and the same gradients
     up to rounding: ds up to fp32 summation order; dA and dB also up to the bf16 rounding of
     dU, which the epilogue applies per token range (about 2^-9 relative)."""
     spec = spec_of("sk", 256, 512, 32, group=128, a_std=0.2, b_std=0.2)
     outs = {}
     for sched in ("split", "tail"):
-        monkeypatch.setenv("LRQAT_DW_SCHEDULE", sched)
+        dw_schedule(sched)
         outs[sched], _, _ = _run(spec, 1555, seed=3)
     for key in ("Y", "dX"):
         np.testing.assert_array_equal(outs["split"][key], outs["tail"][key])

@@ -3,10 +3,14 @@
 Some callers cannot allocate device memory (runtimes that own all device memory
 and give an operator only its inputs and outputs, or that forbid allocation after
 start-up because cudaMalloc can synchronize the device); this entry point serves
-them from a fixed scratch array inside the library.  Its output must match the
-workspace-based lrqat_linear_fwd within the forward tolerance, on two calls in a
-row with different layers (the second call reuses the scratch the first one left
-behind), and layers whose scratch does not fit must be rejected cleanly.
+them from a fixed scratch array inside the library.  The cases below make the
+forward use that array: a rank that is not a multiple of 8 (the adapters are
+copied into padded layouts there) and per-tensor int8 activations (their codes
+live there).  Each output must equal the workspace-based lrqat_linear_fwd's bit
+for bit (the same kernels read the same operands) and the oracle's within the
+forward tolerance, on calls in a row with different layers (each call reuses the
+scratch the previous one left behind), and layers whose scratch does not fit must
+be rejected cleanly.
 
 This file is collected last on purpose, so that a run which stops at the first
 failure has already run every other test.
@@ -19,7 +23,7 @@ from paper_2406_06385_gb300 import lrqat as LQ
 from paper_2406_06385_gb300 import workloads as WL
 from paper_2406_06385_gb300.build import build
 
-from gpu_util import DeviceLayer, bits_to_f32, to_dev, torch
+from gpu_util import DeviceLayer, bits_to_f32, oracle_layer, to_dev, torch
 
 pytestmark = pytest.mark.gpu
 
@@ -37,27 +41,42 @@ def _spec(name, m, k, r, bits=4, phi=WL.PHI_QFIXED, group=0, act=0):
 
 
 def _forward_both(spec, T, seed):
+    """(no-alloc output, workspace output, oracle output) of one layer as fp32 arrays."""
     t = torch()
     data = WL.make_layer(spec, T, seed=seed)
     dl = DeviceLayer(data)
     X = to_dev(data.X_bits)
     L = dl.layer
+    s_x, s_x_host = None, None
+    if spec.act_bits == 8:
+        s_x_host = float(np.float32(np.abs(data.X).max()) / np.float32(127.0) * np.float32(0.7))   # some codes clip
+        s_x = t.tensor([s_x_host], dtype=t.float32, device="cuda")
+    assert LQ.fwd_workspace_bytes(L, T) <= (4 << 20)
     y_ref = t.empty((T, spec.m), dtype=t.int16, device="cuda")
     ws = t.empty(LQ.fwd_workspace_bytes(L, T), dtype=t.uint8, device="cuda")
-    LQ.linear_fwd(L, T, X, dl.phi0, dl.s, dl.A, dl.B, None, y_ref, ws)
+    LQ.linear_fwd(L, T, X, dl.phi0, dl.s, dl.A, dl.B, s_x, y_ref, ws)
     y_na = t.full((T, spec.m), 0x7FC0, dtype=t.int16, device="cuda")   # bf16 NaN everywhere beforehand
-    LQ.linear_fwd_noalloc(L, T, X, dl.phi0, dl.s, dl.A, dl.B, None, y_na)
+    LQ.linear_fwd_noalloc(L, T, X, dl.phi0, dl.s, dl.A, dl.B, s_x, y_na)
     LQ.get_device_status()
-    return bits_to_f32(y_na), bits_to_f32(y_ref)
+    OL = oracle_layer(spec)
+    s0 = O.minmax_scale(data.W0, OL)
+    y_or = O.linear_fwd(data.X, O.downcast(data.W0, s0, OL), s0, data.A, data.B, OL, s_x_host)
+    return bits_to_f32(y_na), bits_to_f32(y_ref), y_or
 
 
-def test_noalloc_forward_matches_workspace_forward_on_two_calls_in_a_row():
-    first = _forward_both(_spec("na1", 384, 512, 32), 1000, seed=31)
-    second = _forward_both(_spec("na2", 256, 512, 16, bits=3, phi=WL.PHI_INT_PACKED), 513, seed=32)
-    for got, ref in (first, second):
-        assert np.isfinite(got).all()
-        err = O.rel_fro(got, ref)
-        assert err <= TOL_Y, err
+def test_noalloc_forward_matches_workspace_forward_on_calls_in_a_row():
+    cases = [
+        (_spec("na_r20", 256, 512, 20), 1000, 31),                                   # padded adapters in the scratch
+        (_spec("na_a8", 384, 512, 32, act=8), 1500, 32),                             # int8 codes in the scratch
+        (_spec("na_r12_int3", 256, 768, 12, bits=3, phi=WL.PHI_INT_PACKED), 513, 33),
+        (_spec("na_r20", 256, 512, 20), 1000, 31),                                   # the first call again
+    ]
+    for spec, T, seed in cases:
+        got, ref, orc = _forward_both(spec, T, seed)
+        assert np.isfinite(got).all(), spec.name
+        np.testing.assert_array_equal(got, ref, err_msg=spec.name)
+        err = O.rel_fro(got, orc)
+        assert err <= TOL_Y, (spec.name, err)
 
 
 def test_noalloc_forward_rejects_scratch_beyond_its_limit():
