@@ -24,9 +24,15 @@
  *     lrqat_get_device_status() reports as LRQAT_ERR_TIMEOUT.
  *   - Rounding is round-half-to-even; the pre-round value
  *     u = phi^{-1}(Phi0) + (alpha/r) A B is formed in fp32.
- *   - Supported shapes: m and k multiples of 128, 1 <= r <= 64, T >= 1 (any
- *     T; ragged token tails are handled), group_size 0 (per output channel)
- *     or a multiple of 128 that divides k.
+ *   - Supported shapes: m and k multiples of 128, 1 <= r <= 256 (ranks above
+ *     64 with bits <= 7), T >= 1 (any T; ragged token tails are handled),
+ *     group_size 0 (per output channel) or a multiple of 128 that divides k.
+ *   - Ranks up to 64 rebuild W_hat entirely inside the GEMMs, the low-rank tile
+ *     (alpha/r) A B included.  Ranks above 64 first write the unclipped codes
+ *     round(phi^{-1}(Phi0) + (alpha/r) A B) of every weight (int8, saturated to
+ *     [-128, 127], which keeps the clip mask) into the workspace with one
+ *     tensor-core pass per call; the GEMMs then clip and scale those codes on
+ *     chip.  The results are the same codes, gradients and outputs.
  */
 #ifndef LRQAT_H
 #define LRQAT_H
@@ -44,7 +50,7 @@ typedef struct CUstream_st* lrqat_stream_t;
 typedef enum {
   LRQAT_OK = 0,
   LRQAT_ERR_INVALID_ARG = -1, /* null pointer, bad shape, bad bit-width ...          */
-  LRQAT_ERR_UNSUPPORTED = -2, /* valid for the method, not implemented (e.g. r > 64)  */
+  LRQAT_ERR_UNSUPPORTED = -2, /* valid for the method, not implemented (e.g. r > 256) */
   LRQAT_ERR_ALIGNMENT = -3,   /* a pointer is not 16-byte aligned                     */
   LRQAT_ERR_WORKSPACE = -4,   /* workspace missing or smaller than required           */
   LRQAT_ERR_CUDA = -5,        /* a CUDA runtime/driver call or launch failed          */
@@ -75,7 +81,7 @@ typedef enum {
 typedef struct {
   int64_t m;
   int64_t k;
-  int32_t r;          /* adapter rank, 1..64                                        */
+  int32_t r;          /* adapter rank, 1..256 (above 64: bits <= 7)                 */
   float alpha;        /* adapter scaling: (alpha / r) A B enters Eq. 8              */
   int32_t bits;       /* b: 2..7 for QFIXED, 2..4 for INT_PACKED, 2..8 for the casts */
   int32_t group_size; /* 0: one scale per output row (pc); else scales per g-wide
@@ -154,7 +160,8 @@ int lrqat_act_quant(const lrqat_layer* layer, int64_t T, const uint16_t* X, cons
                     uint32_t* mask, lrqat_stream_t stream);
 
 /* Bytes of workspace lrqat_linear_fwd needs for T tokens (padded adapter
- * copies; int8 activation codes when act_bits == 8). */
+ * copies; int8 activation codes when act_bits == 8; for ranks above 64 also
+ * the m x k int8 codes of the weights). */
 size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
 
 /* Forward of the LR-QAT layer (Eq. 8 inside y = W_hat x):

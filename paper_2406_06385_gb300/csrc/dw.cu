@@ -18,6 +18,14 @@
 // MMAs and owns TMEM, warps 2..9 run the epilogue, warps 10..12 fill the pipeline
 // stages with TMA.  Work units (row block, column tile, token split) are
 // distributed persistently over the CTAs.
+//
+// Ranks above 64 (NL): the base holds the unclipped codes round(u), low-rank term
+// included (the tensor-core code pass writes them once per call), so no low-rank tile
+// is computed, and the tiles are 128 columns wide.  The adapter contractions run in
+// rounds of 64 rank indices: per round the slices A^T[64 ranks, 128 rows] and B[64
+// ranks, 128 columns] land in the epilogue buffers, tcgen05 computes that round's 64
+// columns of dU B^T and dU^T A into one of two TMEM buffers, and the epilogue warps
+// write them out while the next round runs in the other buffer.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -60,6 +68,9 @@ constexpr uint32_t COL_G = 0;      // 256 columns
 constexpr uint32_t COL_L = 256;    // 128 columns
 constexpr uint32_t COL_DA = 384;   // up to 64 columns
 constexpr uint32_t COL_DBT = 448;  // up to 64 columns
+// NL: two buffers of a round's contractions, dA at COL_NL + 128 b, dB^T 64 columns further
+constexpr uint32_t COL_NL = 256;
+constexpr uint32_t NL_BOX = 64 * 128;   // one 64-rank-row x 64-column bf16 box
 
 constexpr int BAR_FULL = 0;
 constexpr int BAR_EMPTY = BAR_FULL + NS;
@@ -73,7 +84,10 @@ constexpr int BAR_LFULL = BAR_ACCEMPTY + 1;
 constexpr int BAR_DUFULL = BAR_LFULL + 1;
 constexpr int BAR_DBFULL = BAR_DUFULL + 1;
 constexpr int BAR_DRAIN = BAR_DBFULL + 1;
-constexpr int NUM_BARS = BAR_DRAIN + 1;
+// NL: the second buffer's contractions done, and each buffer read by the epilogue
+constexpr int BAR_DBFULL1 = BAR_DRAIN + 1;
+constexpr int BAR_DRAINED = BAR_DBFULL1 + 1;   // two barriers
+constexpr int NUM_BARS = BAR_DRAINED + 2;
 
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   const uint64_t t0 = global_timer_ns();
@@ -141,7 +155,9 @@ __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, Unit& x
 }
 
 // UB: pre-round value in bf16 (u_bf16x2) instead of one fp32 FMA.
-template <int FMT, bool ZP, bool UB>
+// NL: the base holds the unclipped codes (FMT_Q8, 0 fraction bits), no low-rank tile,
+// 128-column tiles, adapter contractions in rounds of 64 ranks.
+template <int FMT, bool ZP, bool UB, bool NL>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     dw_kernel(const __grid_constant__ CUtensorMap tm_dy, const __grid_constant__ CUtensorMap tm_x,
               const __grid_constant__ CUtensorMap tm_at, const __grid_constant__ CUtensorMap tm_phi,
@@ -176,6 +192,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     mbar_init(bar(BAR_DUFULL), NUM_EPI_WARPS);
     mbar_init(bar(BAR_DBFULL), 1);
     mbar_init(bar(BAR_DRAIN), 1);
+    mbar_init(bar(BAR_DBFULL1), 1);
+    mbar_init(bar(BAR_DRAINED), NUM_EPI_WARPS);
+    mbar_init(bar(BAR_DRAINED + 1), NUM_EPI_WARPS);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc(smem_u32(&tmem_base_s), TMEM_COLS);
@@ -187,7 +206,36 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (warp == 0) {
     // ---------------------------------------- epilogue operands (per unit/chunk)
-    if (lane == 0) {
+    if (NL && lane == 0) {
+      // the unit's code chunk, then its rank rounds (A^T and B slices of 64 ranks)
+      const int nrc = (args.r16 + 63) / 64;
+      uint32_t it = 0, cc = 0;
+      bool ok = true;
+      WorkIter wi = work_begin(args);
+      Unit w;
+      while (ok && work_next(wi, args, w)) {
+        if (args.sched.tail && w.sp == 0) {
+          const int64_t tile = w.ib + static_cast<int64_t>(args.ni) * w.jt;
+          args.tile_segs[tile] = dw_tile_segments(tile, args.sched);
+        }
+        if (!(ok = wait_spin_bounded(bar(BAR_ECEMPTY), (cc & 1u) ^ 1u, ctl, 3))) break;
+        const int j0 = w.jt * 128;
+        mbar_arrive_expect_tx(bar(BAR_ECFULL), 16384u);
+        tma_load_2d(smem + OFF_PHI, &tm_phi, j0, w.ib * 128, bar(BAR_ECFULL));
+        ++cc;
+        for (int rc = 0; rc < nrc; ++rc) {
+          if (!(ok = wait_spin_bounded(bar(BAR_EFEMPTY), (it & 1u) ^ 1u, ctl, 2))) break;
+          mbar_arrive_expect_tx(bar(BAR_EFFULL), 4u * NL_BOX);
+          tma_load_2d(smem + OFF_AT, &tm_at, w.ib * 128, 64 * rc, bar(BAR_EFFULL));
+          tma_load_2d(smem + OFF_AT + NL_BOX, &tm_at, w.ib * 128 + 64, 64 * rc, bar(BAR_EFFULL));
+          tma_load_2d(smem + OFF_BP, &tm_b, j0, 64 * rc, bar(BAR_EFFULL));
+          tma_load_2d(smem + OFF_BP + NL_BOX, &tm_b, j0 + 64, 64 * rc, bar(BAR_EFFULL));
+          ++it;
+        }
+      }
+      if (it > 0) drain_wait(bar(BAR_EFFULL), (it - 1) & 1u, args.timeout_ns);
+      if (cc > 0) drain_wait(bar(BAR_ECFULL), (cc - 1) & 1u, args.timeout_ns);
+    } else if (lane == 0) {
       const uint32_t ef_tx = 2u * rbox;
       const uint32_t ec_tx = (P16 ? 0u : PACKED ? 8192u : 16384u) + 2u * rbox;
       uint32_t it = 0, cc = 0;
@@ -271,6 +319,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint64_t d_x0 = make_sdesc(smem + OFF_STAGES + STAGE_DY, BOX_BYTES, 1024, SWZ_128B);
       const uint32_t b_full = bar(BAR_FULL), b_empty = bar(BAR_EMPTY);
       uint32_t g = 0, it = 0, cc = 0;
+      uint32_t rr = 0;          // NL: rank rounds issued
       uint32_t s = 0, ph = 0;   // stage and phase of global step g
       bool ok = true;
       WorkIter wi = work_begin(args);
@@ -294,6 +343,43 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         if (!ok) break;
         mma_commit(bar(BAR_ACCFULL));
+        if (NL) {
+          // dU of the unit written: the code chunk has been read, then the rank rounds
+          if (!(ok = wait_spin_bounded(bar(BAR_DUFULL), cc & 1u, ctl, 8))) break;
+          tc_fence_after();
+          mma_commit(bar(BAR_ECEMPTY));
+          const uint32_t idesc_da64 = make_idesc_bf16(128, 64, 0, 0);
+          const uint32_t idesc_db64 = make_idesc_bf16(128, 64, 1, 0);
+          for (int rc = 0; rc < (args.r16 + 63) / 64; ++rc) {
+            // rounds are the uses of the epilogue buffers (EF) in NL
+            if (!(ok = wait_spin_bounded(bar(BAR_EFFULL), rr & 1u, ctl, 6))) break;
+            const uint32_t b = rr & 1u, n = rr >> 1;
+            if (!(ok = wait_spin_bounded(bar(BAR_DRAINED + b), (n & 1u) ^ 1u, ctl, 13))) break;
+            tc_fence_after();
+            const uint32_t col = tmem + COL_NL + 128u * b;
+            // dA round = dU * B_round^T : M = 128 rows i, N = 64 ranks, K = 128 columns j
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks) {
+              const uint64_t ad = make_sdesc(smem + OFF_DU + 16384u * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+              const uint64_t bd = make_sdesc(smem + OFF_BP + NL_BOX * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+              mma_bf16(col, ad, bd, idesc_da64, ks > 0 ? 1u : 0u);
+            }
+            // dB^T round = dU^T * A_round : M = 128 columns j (dU MN-major), N = 64 ranks, K = 128 rows i
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks) {
+              const uint64_t ad = make_sdesc(smem + OFF_DU + 2048u * ks, 16384, 1024, SWZ_128B);
+              const uint64_t bd = make_sdesc(smem + OFF_AT + NL_BOX * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+              mma_bf16(col + 64, ad, bd, idesc_db64, ks > 0 ? 1u : 0u);
+            }
+            mma_commit(bar(b ? BAR_DBFULL1 : BAR_DBFULL));
+            mma_commit(bar(BAR_EFEMPTY));
+            ++rr;
+          }
+          if (!ok) break;
+          ++cc;
+          ++it;
+          continue;
+        }
         if (!(ok = wait_spin_bounded(bar(BAR_EFFULL), it & 1u, ctl, 6))) break;
         for (int c = 0; c < args.nchunks; ++c) {
           if (!(ok = wait_spin_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 7))) break;
@@ -346,6 +432,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const float gscale = args.s_x != nullptr ? *args.s_x : 1.0f;
     const int half_cols = args.r16 / 2;   // dA / dB^T columns read by this warp half
     uint32_t it = 0, cc = 0;
+    uint32_t rr = 0;   // NL: rank rounds drained
     bool ok = true;
     WorkIter wi = work_begin(args);
     Unit w;
@@ -370,7 +457,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                           : args.s_ld ? args.zero[static_cast<int64_t>(i_g) * args.s_ld + j0 / args.group_size]
                                       : args.zero[i_g];
         ok = wait_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 10);
-        ok = ok && wait_bounded(bar(BAR_LFULL), cc & 1u, ctl, 11);
+        if (!NL) ok = ok && wait_bounded(bar(BAR_LFULL), cc & 1u, ctl, 11);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
         // Packed fp32x2 arithmetic per pair of columns: u = phi^-1 + (alpha/r) L, the
@@ -386,7 +473,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const int jl = 64 * h + 32 * p;   // column within the chunk
           float G[32], Lv[32], v[32];
           tmem_ld32(tmem + lane_off + COL_G + 128 * c + jl, G);
-          tmem_ld32(tmem + lane_off + COL_L + jl, Lv);
+          if (!NL) tmem_ld32(tmem + lane_off + COL_L + jl, Lv);
           tmem_ld_wait();
           uint32_t raw[16];
           if (PACKED) {
@@ -415,9 +502,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int e = 0; e < 16; ++e) {
             const float2 g2 = make_float2(G[2 * e], G[2 * e + 1]);
             const float2 v2 = make_float2(v[2 * e], v[2 * e + 1]);
-            const float2 u2 = UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v2.x, v2.y, lr2)
-                                 : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]),
-                                              make_float2(qp.lr_scale, qp.lr_scale), v2);
+            const float2 u2 = NL   ? v2
+                              : UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v2.x, v2.y, lr2)
+                                   : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]),
+                                                make_float2(qp.lr_scale, qp.lr_scale), v2);
             const float2 t2 = __fadd2_rn(u2, make_float2(qp.magic, qp.magic));
             const float2 cu = __ffma2_rn(t2, make_float2(qp.inv2f, qp.inv2f), make_float2(-qp.magic_c, -qp.magic_c));
             const float2 cc = make_float2(fminf(fmaxf(cu.x, code_n), code_p), fminf(fmaxf(cu.y, code_n), code_p));
@@ -445,6 +533,41 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(bar(BAR_DUFULL));
+        if (NL) {
+          // rank rounds: this warp half writes 32 of each round's 64 rank columns of dB^T
+          // (lanes = columns j) and of dA (lanes = rows i)
+          float* dstB = args.dB_part + static_cast<int64_t>(w.ib * args.nsplit + w.sp) * args.r * args.k + j0 + row;
+          float* dstA = args.dA_part + (static_cast<int64_t>(w.jt * args.nsplit + w.sp) * args.m + i_g) * args.r;
+          for (int rc = 0; rc < (args.r16 + 63) / 64 && ok; ++rc) {
+            const uint32_t b = rr & 1u, n = rr >> 1;
+            ok = wait_bounded(bar(b ? BAR_DBFULL1 : BAR_DBFULL), n & 1u, ctl, 12);
+            if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t col = tmem + lane_off + COL_NL + 128u * b + 32u * h;
+#pragma unroll 1
+            for (int c8 = 0; c8 < 32; c8 += 8) {
+              float vb[8], va[8];
+              tmem_ld8(col + 64 + c8, vb);
+              tmem_ld8(col + c8, va);
+              tmem_ld_wait();
+#pragma unroll
+              for (int e = 0; e < 8; ++e) {
+                const int t = 64 * rc + 32 * h + c8 + e;
+                if (t < args.r) {
+                  dstB[static_cast<int64_t>(t) * args.k] = vb[e];
+                  dstA[t] = va[e];
+                }
+              }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(BAR_DRAINED + b));
+            ++rr;
+          }
+          if (!ok) break;
+          ++cc;
+          continue;
+        }
         ok = wait_bounded(bar(BAR_DBFULL), cc & 1u, ctl, 12);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after();
@@ -491,14 +614,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <int FMT, bool ZP, bool UB>
+template <int FMT, bool ZP, bool UB, bool NL = false>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const CUtensorMap& e, const DwArgs& args, int grid, cudaStream_t stream) {
   static bool configured[kMaxDevices] = {};
-  const cudaError_t err = ensure_smem_attr(reinterpret_cast<const void*>(dw_kernel<FMT, ZP, UB>),
+  const cudaError_t err = ensure_smem_attr(reinterpret_cast<const void*>(dw_kernel<FMT, ZP, UB, NL>),
                                            static_cast<int>(SMEM_BYTES), configured);
   if (err != cudaSuccess) return err;
-  dw_kernel<FMT, ZP, UB><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
+  dw_kernel<FMT, ZP, UB, NL><<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b, c, d, e, args);
   return cudaGetLastError();
 }
 
@@ -524,6 +647,14 @@ int dw_smem_bytes(int, int) { return static_cast<int>(SMEM_BYTES); }
 cudaError_t launch_dw(int fmt, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
                       const CUtensorMap& tm_phi, const CUtensorMap& tm_b, const DwArgs& args, int grid,
                       cudaStream_t stream) {
+  if (args.codes_base) {
+    // ranks above 64: the base holds int8 codes, 128-column tiles, rank rounds of 64
+    if (grid < 1 || fmt != FMT_Q8 || args.u_bf16 || args.nchunks != 1 || args.r16 < 16 || args.r16 > 256 ||
+        (args.r16 & 15))
+      return cudaErrorInvalidValue;
+    return args.zero != nullptr ? launch_one<FMT_Q8, true, false, true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream)
+                                : launch_one<FMT_Q8, false, false, true>(tm_dy, tm_x, tm_at, tm_phi, tm_b, args, grid, stream);
+  }
   if (grid < 1 || args.r16 < 16 || args.r16 > 64 || (args.r16 & 15) || args.nchunks < 1 || args.nchunks > 2)
     return cudaErrorInvalidValue;
   if (fmt_16bit(fmt) && (args.phi == nullptr || (reinterpret_cast<uintptr_t>(args.phi) & 15u) || args.k % 128))

@@ -233,21 +233,26 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __rest
                                                               const uint16_t* __restrict__ B, int64_t m, int64_t k,
                                                               int r, int fmt, int ub, int b_aligned, QuantParams q,
                                                               int8_t* __restrict__ wz) {
-  __shared__ __align__(16) float As[64][kMergeRows];   // A^T tile: [t][row]
+  __shared__ __align__(16) float As[64][kMergeRows];   // A^T tile of 64 rank indices: [t][row]
   const int64_t i0 = static_cast<int64_t>(blockIdx.y) * kMergeRows;
   const int64_t j = static_cast<int64_t>(blockIdx.x) * kMergeCols + 4 * threadIdx.x;
-  for (int e = threadIdx.x; e < kMergeRows * 64; e += kMergeThreads) {
-    const int t = e / kMergeRows, ii = e % kMergeRows;
-    As[t][ii] = (i0 + ii < m && t < r) ? bf16_to_float(A[(i0 + ii) * r + t]) : 0.0f;
-  }
-  __syncthreads();
-  if (j >= k) return;
   float acc[kMergeRows][4];
 #pragma unroll
   for (int ii = 0; ii < kMergeRows; ++ii)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[ii][c] = 0.0f;
-  for (int t = 0; t < r; ++t) {
+  // the rank in blocks of 64 indices, A staged in shared memory per block
+  for (int t0 = 0; t0 < r; t0 += 64) {
+  __syncthreads();   // the previous block's reads of As are done
+  for (int e = threadIdx.x; e < kMergeRows * 64; e += kMergeThreads) {
+    const int t = e / kMergeRows, ii = e % kMergeRows;
+    As[t][ii] = (i0 + ii < m && t0 + t < r) ? bf16_to_float(A[(i0 + ii) * r + t0 + t]) : 0.0f;
+  }
+  __syncthreads();
+  if (j < k) {
+  const int t_end = r - t0 < 64 ? r - t0 : 64;
+  for (int tt = 0; tt < t_end; ++tt) {
+    const int t = t0 + tt;
     const uint16_t* brow = B + static_cast<int64_t>(t) * k + j;
     uint2 braw;
     if (b_aligned) {
@@ -258,7 +263,7 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __rest
     }
     const float b4[4] = {__uint_as_float(braw.x << 16), __uint_as_float(braw.x & 0xFFFF0000u),
                          __uint_as_float(braw.y << 16), __uint_as_float(braw.y & 0xFFFF0000u)};
-    const float4* arow = reinterpret_cast<const float4*>(&As[t][0]);
+    const float4* arow = reinterpret_cast<const float4*>(&As[tt][0]);
 #pragma unroll
     for (int g = 0; g < kMergeRows / 4; ++g) {
       const float4 a4 = arow[g];
@@ -269,6 +274,9 @@ __global__ void __launch_bounds__(kMergeThreads) merge_kernel(const void* __rest
         for (int c = 0; c < 4; ++c) acc[4 * g + u][c] = __fmaf_rn(av[u], b4[c], acc[4 * g + u][c]);
     }
   }
+  }
+  }
+  if (j >= k) return;
 #pragma unroll
   for (int ii = 0; ii < kMergeRows; ++ii) {
     const int64_t i = i0 + ii;
@@ -1030,7 +1038,7 @@ cudaError_t launch_downcast(const float* W0, const float* s0, const float* z0, i
 
 cudaError_t launch_merge(const void* phi0, const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r,
                          int fmt, int u_bf16, const QuantParams& q, int8_t* wz, cudaStream_t stream) {
-  if ((k % 4) != 0 || r > 64) return cudaErrorInvalidValue;
+  if ((k % 4) != 0 || r > 256) return cudaErrorInvalidValue;
   const int b_aligned = (reinterpret_cast<uintptr_t>(B) & 7) == 0;
   dim3 grid(static_cast<unsigned>((k + kMergeCols - 1) / kMergeCols), static_cast<unsigned>((m + kMergeRows - 1) / kMergeRows));
   merge_kernel<<<grid, kMergeThreads, 0, stream>>>(phi0, A, B, m, k, r, fmt, u_bf16, b_aligned, q, wz);

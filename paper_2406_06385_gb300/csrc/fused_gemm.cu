@@ -29,6 +29,10 @@
 // Large 128-byte-row boxes matter: an SM's TMA throughput falls with the number
 // of boxes it processes, and loads issued by one warp are handled one at a time,
 // hence one loader warp per ring slot of the token operand.
+// Ranks above 64 (NL): the base operand already holds the codes round(u) of Eq. 8,
+// low-rank term included (written once per call by the tensor-core code pass), so no
+// factor is loaded and no low-rank tile is computed; the producers clip, (scale) and
+// store W_hat from the base alone.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -116,7 +120,8 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64
 // even number of slices, so stage gg uses token slot gg % 2 for the (gg / 2)-th
 // time and factor slot gg % NF for the (gg / NF)-th time.
 // UB: pre-round value in bf16 (u_bf16x2) instead of one fp32 FMA.
-template <int MODE, int FMT, bool ZP, bool UB>
+// NL: no low-rank term (the base holds the unclipped codes, FMT_Q8 with 0 fraction bits).
+template <int MODE, int FMT, bool ZP, bool UB, bool NL>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
@@ -169,7 +174,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (warp == 0) {
     // ------------------------------------------------- row factor (per tile)
-    if (lane == 0) {
+    if (!NL && lane == 0) {
       prefetch_tensormap(&tm_rf);
       uint32_t it = 0;
       for (int tile = blockIdx.x; tile < args.num_tiles; tile += gridDim.x) {
@@ -210,7 +215,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       prefetch_tensormap(&tm_phi);
       prefetch_tensormap(&tm_sf);
     }
-    const uint32_t tx = FR::PHI_TX + static_cast<uint32_t>(BK * 2 * (sf_mn ? args.r16 : args.sf_cols));
+    const uint32_t tx = FR::PHI_TX + (NL ? 0u : static_cast<uint32_t>(BK * 2 * (sf_mn ? args.r16 : args.sf_cols)));
     uint32_t gg = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
@@ -225,7 +230,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         __syncwarp();
         const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
         if (lane == 0) tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb * BM, fb);
-        if (lane == 1) {
+        if (!NL && lane == 1) {
           if (sf_mn) tma_load_2d(fs + FR::FS_SF, &tm_sf, kk * BK, 0, fb);   // B rows, 64 columns
           else tma_load_2d(fs + FR::FS_SF, &tm_sf, 0, kk * BK, fb);
         }
@@ -277,8 +282,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         return true;
       };
       for (int tile = blockIdx.x; tile < args.num_tiles && ok; tile += gridDim.x) {
-        if (!(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
-        if (!(ok = issue_lowrank(g))) break;
+        if (!NL && !(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
+        if (!NL && !(ok = issue_lowrank(g))) break;
         if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
         tc_fence_after();
         for (int kk = 0; kk < nk; ++kk) {
@@ -287,7 +292,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           // The low-rank tile of the next stage goes into the tensor pipe ahead of this
           // stage's product as soon as the producers have read the current one, so the
           // W_hat build of the next stage overlaps this product.
-          if (kk + 1 < nk) {
+          if (!NL && kk + 1 < nk) {
             if (!(ok = issue_lowrank(gg + 1))) break;
             if (kk + 2 == nk) mma_commit(bar(BAR_RFEMPTY));   // last read of the row factor issued
           }
@@ -412,22 +417,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           raw[0] = r.x, raw[1] = r.y, raw[2] = r.z, raw[3] = r.w;
         }
         decode16<FMT>(raw, v);
-        ok = wait_bounded(bar(BAR_LFULL), gg & 1u, ctl, 10);
-        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-        tc_fence_after();
         float Lv[16];
-        tmem_ld16(tmem + lane_off + COL_L + 16 * c, Lv);
-        tmem_ld_wait();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar(BAR_LEMPTY));
+        if (!NL) {
+          ok = wait_bounded(bar(BAR_LFULL), gg & 1u, ctl, 10);
+          if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+          tc_fence_after();
+          tmem_ld16(tmem + lane_off + COL_L + 16 * c, Lv);
+          tmem_ld_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(BAR_LEMPTY));
+        }
         uint32_t w[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const float2 u =
-              UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
-                 : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
-                              make_float2(v[2 * e], v[2 * e + 1]));
+              NL   ? make_float2(v[2 * e], v[2 * e + 1])
+              : UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
+                   : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
+                                make_float2(v[2 * e], v[2 * e + 1]));
           const float2 t2 = __fadd2_rn(u, make_float2(qp.magic, qp.magic));
           uint32_t cw = codes_bf16x2(t2, qp);
           if (zp) cw = sub_bf16x2(cw, zw[e]);   // c - z, exact small integers
@@ -508,15 +516,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
-template <int MODE, int FMT, bool ZP, bool UB>
+template <int MODE, int FMT, bool ZP, bool UB, bool NL = false>
 cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                        const FusedArgs& args, int grid, cudaStream_t stream) {
   constexpr uint32_t smem = FactorRing<FMT>::SMEM_BYTES;
   static bool configured[kMaxDevices] = {};
-  const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(fused_gemm_kernel<MODE, FMT, ZP, UB>),
+  const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(fused_gemm_kernel<MODE, FMT, ZP, UB, NL>),
                                          static_cast<int>(smem), configured);
   if (e != cudaSuccess) return e;
-  fused_gemm_kernel<MODE, FMT, ZP, UB><<<grid, NUM_THREADS, smem, stream>>>(a, b, c, d, args);
+  fused_gemm_kernel<MODE, FMT, ZP, UB, NL><<<grid, NUM_THREADS, smem, stream>>>(a, b, c, d, args);
   return cudaGetLastError();
 }
 
@@ -542,6 +550,13 @@ cudaError_t launch_fmt(const CUtensorMap& tm_tok, const CUtensorMap& tm_phi, con
 template <int MODE>
 cudaError_t launch_mode(int fmt, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi, const CUtensorMap& tm_rf,
                         const CUtensorMap& tm_sf, const FusedArgs& args, int grid, cudaStream_t stream) {
+  if (args.r16 == 0) {
+    // no low-rank term: the base holds int8 codes (0 fraction bits), the bf16 pre-round value
+    // (if any) was applied when they were written
+    if (fmt != FMT_Q8 || args.u_bf16) return cudaErrorInvalidValue;
+    return args.zero != nullptr ? launch_one<MODE, FMT_Q8, true, false, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream)
+                                : launch_one<MODE, FMT_Q8, false, false, true>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
+  }
   switch (fmt) {
     case FMT_Q8: return launch_fmt<MODE, FMT_Q8>(tm_tok, tm_phi, tm_rf, tm_sf, args, grid, stream);
     case FMT_I4:

@@ -140,7 +140,8 @@ struct FusedArgs {
   int32_t rows;          // rows of the produced weight operand (m for fwd, k for dX)
   int32_t kdim;          // contraction length (k for fwd, m for dX)
   int32_t T;             // tokens
-  int32_t r16;           // adapter rank rounded up to 16
+  int32_t r16;           // adapter rank rounded up to 16; 0: no low-rank term (the base holds
+                         // the unclipped int8 codes round(u), written for ranks above 64)
   int32_t sf_cols;       // columns of the second factor loaded per stage (16, 32 or 64)
   int32_t num_rb;        // rows / 128
   int32_t num_tb;        // ceil(T / 448)
@@ -186,6 +187,9 @@ struct DwArgs {
   int32_t u_bf16;        // pre-round value in bf16 (lrqat_layer.u_bf16)
   DwSched sched;         // kept last (argument layout)
   int32_t* tile_segs;    // tail schedule: [ni * nj] slots written per tile
+  // Ranks above 64: the base (tm_phi) holds the unclipped int8 codes round(u), low-rank
+  // term included; no low-rank tile, nchunks == 1, tm_at / tm_b boxes of 64 rank rows.
+  int32_t codes_base;
 };
 int dw_smem_bytes(int r16, int fmt);
 // fmt: a PhiFmt value (quant.cuh)

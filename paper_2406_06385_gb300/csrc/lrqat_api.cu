@@ -120,6 +120,13 @@ bool direct_factors(const lrqat_layer& L, const void* A, const void* B) {
 }
 
 int frac_bits(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_QFIXED ? 8 - L.bits : 0; }
+
+// Ranks above 64: one tensor-core pass per call writes the unclipped codes round(u) of every
+// weight (int8, saturated) into the workspace, and the three GEMMs read them as their base
+// with the low-rank term switched off (the factor slices of a rank above 64 do not fit next
+// to the GEMMs' token ring, and recomputing A B per 448-token tile would cost r/448 of the
+// GEMM's own tensor work).
+bool codes_base(const lrqat_layer& L) { return L.r > 64; }
 bool phi_16bit(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_BF16 || L.phi_format == LRQAT_PHI_FP16; }
 int round16(int r) { return (r + 15) / 16 * 16; }
 
@@ -132,7 +139,7 @@ int validate_layer(const lrqat_layer* L) {
                 (long long)L->k);
   if (L->m > (int64_t)1 << 30 || L->k > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "m or k too large");
   if (L->r < 1) return fail(LRQAT_ERR_INVALID_ARG, "rank r must be >= 1 (r=%d)", L->r);
-  if (L->r > 64) return fail(LRQAT_ERR_UNSUPPORTED, "rank r=%d > 64 is not supported", L->r);
+  if (L->r > 256) return fail(LRQAT_ERR_UNSUPPORTED, "rank r=%d > 256 is not supported", L->r);
   if (!std::isfinite(L->alpha)) return fail(LRQAT_ERR_INVALID_ARG, "alpha must be finite");
   if (L->phi_format == LRQAT_PHI_QFIXED) {
     if (L->bits < 2 || L->bits > 7) return fail(LRQAT_ERR_INVALID_ARG, "QFIXED needs 2 <= bits <= 7 (bits=%d)", L->bits);
@@ -150,6 +157,8 @@ int validate_layer(const lrqat_layer* L) {
   if (L->group_size < 0) return fail(LRQAT_ERR_INVALID_ARG, "group_size must be >= 0");
   if (L->group_size > 0 && (L->group_size % 128 || L->k % L->group_size))
     return fail(LRQAT_ERR_UNSUPPORTED, "group_size %d must be a multiple of 128 dividing k", L->group_size);
+  if (L->r > 64 && L->bits > 7)
+    return fail(LRQAT_ERR_UNSUPPORTED, "ranks above 64 need bits <= 7 (the unclipped codes are kept as int8)");
   if (L->act_bits != 0 && L->act_bits != 8)
     return fail(LRQAT_ERR_UNSUPPORTED, "act_bits must be 0 or 8 (got %d)", L->act_bits);
   if (L->zero && !aligned16(L->zero)) return fail(LRQAT_ERR_ALIGNMENT, "zero (offsets) is not 16-byte aligned");
@@ -279,7 +288,7 @@ struct DwPlan {
 
 DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
   DwPlan p;
-  p.nchunks = (L.k % 256 == 0) ? 2 : 1;
+  p.nchunks = (L.k % 256 == 0 && !codes_base(L)) ? 2 : 1;
   p.ni = static_cast<int>(L.m / 128);
   p.nj = static_cast<int>(L.k / (128 * p.nchunks));
   const int tiles = p.ni * p.nj;
@@ -337,13 +346,23 @@ struct FwdWs {
   uint16_t* a_pad;
   uint16_t* bt_pad;
   uint16_t* x_codes;   // int8 codes (per tensor) or X_hat (per token), bf16
+  uint16_t* at;        // ranks above 64: A^T [r16, m] and B [r16, k] zero-padded, codes [m, k]
+  uint16_t* b_pad;
+  int8_t* codes;
 };
 
 size_t fwd_ws_layout(const lrqat_layer& L, int64_t T, void* base, FwdWs* ws) {
   Carver c(base);
   FwdWs w{};
-  w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
-  w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  if (codes_base(L)) {
+    const size_t r16 = static_cast<size_t>(round16(L.r));
+    w.at = static_cast<uint16_t*>(c.take(r16 * L.m * 2));
+    w.b_pad = static_cast<uint16_t*>(c.take(r16 * L.k * 2));
+    w.codes = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
+  } else {
+    w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
+    w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  }
   if (L.act_bits == 8) w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
   if (ws) *ws = w;
   return (c.used + 255) & ~size_t(255);
@@ -361,17 +380,22 @@ struct BwdWs {
   float* dB_part;
   float* ds_part;
   int32_t* tile_segs;
+  int8_t* codes;       // ranks above 64: the unclipped codes [m, k] (phit then holds their transpose)
 };
 
 size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* base, BwdWs* ws) {
   Carver c(base);
   BwdWs w{};
   const int r16 = round16(L.r);
-  w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
-  w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  if (codes_base(L)) {
+    w.codes = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
+  } else {
+    w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
+    w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  }
   w.at = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.m * 2));
   w.b_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.k * 2));
-  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k * (phi_16bit(L) ? 2 : 1)));
+  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k * (phi_16bit(L) && !codes_base(L) ? 2 : 1)));
   if (L.act_bits == 8) {
     w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
     w.xmask = static_cast<uint32_t*>(c.take(static_cast<size_t>(L.k) * ((T + 31) / 32) * 4));
@@ -398,6 +422,21 @@ int phi_map(CUtensorMap* map, const lrqat_layer& L, const void* phi0, uint32_t b
   return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, phi0, L.k / 2, L.m, L.k / 2, box_cols_elems / 2, 128,
                    dw ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B, "Phi0 (packed)");
 }
+
+// Quantizer constants of the codes written for ranks above 64: the clamp bounds are the int8
+// range instead of [n, p] (the GEMMs clip and mask from the unclipped code).
+QuantParams saturating_params(const lrqat_layer& L) {
+  QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+  const QuantParams wide = make_quant_params(8, frac_bits(L), L.alpha, L.r);
+  q.lo = wide.lo;
+  q.hi = wide.hi;
+  return q;
+}
+
+// The codes pass: codes[i, j] = sat8(round(phi^{-1}(Phi0[i, j]) + (alpha/r) (A B)[i, j])) on the
+// tensor cores, from the zero-padded A^T [r16, m] and B [r16, k] (any rank up to 256).
+int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, const uint16_t* B_pad, int8_t* codes,
+                   const DeviceInfo* dev, cudaStream_t stream);
 
 }  // namespace
 }  // namespace lrqat
@@ -434,6 +473,30 @@ int noalloc_scratch(void** out) {
   return LRQAT_OK;
 }
 
+}  // namespace
+
+namespace {
+int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, const uint16_t* B_pad, int8_t* codes,
+                   const DeviceInfo* dev, cudaStream_t stream) {
+  const int r16 = round16(L.r);
+  CUtensorMap tm_a, tm_b;
+  LRQAT_TRY(encode_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, At, L.m, r16, L.m * 2, 64, static_cast<uint32_t>(r16),
+                      CU_TENSOR_MAP_SWIZZLE_128B, "A^T (padded)"));
+  LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B_pad, L.k, r16, L.k * 2, 64,
+                      static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
+  MergeArgs a{};
+  a.phi0 = Phi0;
+  a.wz = codes;
+  a.m = L.m;
+  a.k = L.k;
+  a.r16 = r16;
+  a.q = saturating_params(L);
+  a.status = dev->status;
+  a.timeout_ns = kWaitTimeoutNs;
+  LRQAT_LAUNCH("lowrank_codes", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 1, tm_a, tm_b, a, stream),
+               "low-rank code pass");
+  return LRQAT_OK;
+}
 }  // namespace
 }  // namespace lrqat
 
@@ -561,11 +624,19 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   FwdWs ws;
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
-  const bool direct = direct_factors(L, A, B);
-  if (!direct)
+  const bool cb = codes_base(L);
+  const bool direct = !cb && direct_factors(L, A, B);
+  if (cb) {
+    // ranks above 64: the codes of every weight, once per call
+    LRQAT_LAUNCH("adapter_layouts", 1, stream,
+                 launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
+                 "adapter layouts");
+    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, dev, stream));
+  } else if (!direct) {
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
                  "adapter layouts");
+  }
   const uint16_t* tok = X;
   if (quantized) {
     // the caller ran lrqat_act_quant on this X
@@ -582,8 +653,17 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
   LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 64, 224,
                       CU_TENSOR_MAP_SWIZZLE_128B, "X"));
-  LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 64, false));
-  if (direct) {
+  if (cb) {
+    // the codes as an 8-bit base; the factor maps are not read
+    LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.codes, L.k, L.m, L.k, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_64B, "codes"));
+    tm_rf = tm_phi;
+    tm_sf = tm_phi;
+  } else {
+    LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 64, false));
+  }
+  if (cb) {
+  } else if (direct) {
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "A"));
     LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B, L.k, L.r, L.k * 2, 64,
@@ -598,15 +678,15 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   a.rows = static_cast<int32_t>(L.m);
   a.kdim = static_cast<int32_t>(L.k);
   a.T = static_cast<int32_t>(T);
-  a.r16 = r16;
-  a.sf_cols = sf_cols(r16);
+  a.r16 = cb ? 0 : r16;
+  a.sf_cols = cb ? 0 : sf_cols(r16);
   a.num_rb = static_cast<int32_t>(L.m / 128);
   a.num_tb = static_cast<int32_t>((T + 447) / 448);
   a.num_tiles = a.num_rb * a.num_tb;
-  a.q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+  a.q = make_quant_params(L.bits, cb ? 0 : frac_bits(L), L.alpha, L.r);
   a.s = s;
   a.zero = L.zero;
-  a.u_bf16 = L.u_bf16;
+  a.u_bf16 = cb ? 0 : L.u_bf16;
   a.sf_mn = direct ? 1 : 0;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
@@ -619,8 +699,8 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   a.timeout_ns = kWaitTimeoutNs;
   const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
   LRQAT_LAUNCH("fused_fwd", 1, stream,
-               launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, L.phi_format, tm_tok, tm_phi, tm_rf,
-                            tm_sf, a, grid, stream),
+               launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, cb ? LRQAT_PHI_QFIXED : L.phi_format,
+                            tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
                "fused forward launch");
   return LRQAT_OK;
 }
@@ -693,11 +773,24 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   const int fmt_t = L.phi_format == LRQAT_PHI_INT_PACKED ? LRQAT_PHI_QFIXED : L.phi_format;
   // with direct factors the dX GEMM reads its A slices from A itself; its row factor stays the
   // padded B^T, and dW takes A^T and B padded
-  const bool direct = direct_factors(L, A, B);
-  LRQAT_LAUNCH("bwd_prep", 1, stream,
-               launch_bwd_prep(A, B, L.m, L.k, L.r, r16, direct ? nullptr : ws.a_pad, ws.bt_pad, ws.at, ws.b_pad,
-                               Phi0, L.phi_format, ws.phit, stream),
-               "adapter layouts and transposed base");
+  const bool cb = codes_base(L);
+  const bool direct = !cb && direct_factors(L, A, B);
+  if (cb) {
+    // ranks above 64: the codes of every weight, then their transpose for the dX GEMM
+    LRQAT_LAUNCH("adapter_layouts", 1, stream,
+                 launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
+                 "adapter layouts");
+    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, dev, stream));
+    LRQAT_LAUNCH("bwd_prep", 1, stream,
+                 launch_bwd_prep(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, nullptr, nullptr, ws.codes,
+                                 LRQAT_PHI_QFIXED, ws.phit, stream),
+                 "transposed codes");
+  } else {
+    LRQAT_LAUNCH("bwd_prep", 1, stream,
+                 launch_bwd_prep(A, B, L.m, L.k, L.r, r16, direct ? nullptr : ws.a_pad, ws.bt_pad, ws.at, ws.b_pad,
+                                 Phi0, L.phi_format, ws.phit, stream),
+                 "adapter layouts and transposed base");
+  }
   const uint16_t* xop = X;
   const uint32_t* xmask = nullptr;
   if (quantized) {
@@ -713,19 +806,24 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     xop = ws.x_codes;
     xmask = ws.xmask;
   }
-  const QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
+  // the codes base has no fraction bits
+  const QuantParams q = make_quant_params(L.bits, cb ? 0 : frac_bits(L), L.alpha, L.r);
 
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
     LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 224,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY"));
-    if (phi_16bit(L))
+    if (phi_16bit(L) && !cb)
       LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT16, ws.phit, L.m, L.k, L.m * 2, 64, 128,
                           CU_TENSOR_MAP_SWIZZLE_128B, "Phi0^T (16-bit)"));
     else
       LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.phit, L.m, L.k, L.m, 64, 128,
                           CU_TENSOR_MAP_SWIZZLE_64B, "Phi0^T"));
+    if (cb) {   // no factors are read
+      tm_rf = tm_phi;
+      tm_sf = tm_phi;
+    } else {
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
     if (direct)
@@ -734,19 +832,20 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     else
       LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16), 64,
                           sf_swizzle(r16), "A (padded)"));
+    }
     FusedArgs a{};
     a.rows = static_cast<int32_t>(L.k);
     a.kdim = static_cast<int32_t>(L.m);
     a.T = static_cast<int32_t>(T);
-    a.r16 = r16;
-    a.sf_cols = sf_cols(r16);
+    a.r16 = cb ? 0 : r16;
+    a.sf_cols = cb ? 0 : sf_cols(r16);
     a.num_rb = static_cast<int32_t>(L.k / 128);
     a.num_tb = static_cast<int32_t>((T + 447) / 448);
     a.num_tiles = a.num_rb * a.num_tb;
     a.q = q;
     a.s = s;
     a.zero = L.zero;
-    a.u_bf16 = L.u_bf16;
+    a.u_bf16 = cb ? 0 : L.u_bf16;
     a.sf_mn = 0;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
@@ -759,7 +858,8 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.timeout_ns = kWaitTimeoutNs;
     const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
     LRQAT_LAUNCH("fused_dx", 1, stream,
-                 launch_fused(FUSED_DX, fmt_t, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream), "fused dX launch");
+                 launch_fused(FUSED_DX, cb ? LRQAT_PHI_QFIXED : fmt_t, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+                 "fused dX launch");
   }
   // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
   {
@@ -768,11 +868,17 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY (dW)"));
     LRQAT_TRY(encode_2d(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, xop, L.k, T, L.k * 2, 64, 32,
                         CU_TENSOR_MAP_SWIZZLE_128B, "X (dW)"));
-    LRQAT_TRY(encode_2d(&tm_at, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64,
-                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "A^T"));
-    LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
-    LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.b_pad, L.k, r16, L.k * 2, 64,
-                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
+    // the codes base: boxes of 64 rank rows (one round of the adapter contractions)
+    const uint32_t rbox_rows = cb ? 64u : static_cast<uint32_t>(r16);
+    LRQAT_TRY(encode_2d(&tm_at, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64, rbox_rows,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A^T"));
+    if (cb)
+      LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.codes, L.k, L.m, L.k, 128, 128,
+                          CU_TENSOR_MAP_SWIZZLE_128B, "codes"));
+    else
+      LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
+    LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.b_pad, L.k, r16, L.k * 2, 64, rbox_rows,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
     DwArgs a{};
     a.m = static_cast<int32_t>(L.m);
     a.k = static_cast<int32_t>(L.k);
@@ -788,7 +894,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.q = q;
     a.s = s;
     a.zero = L.zero;
-    a.u_bf16 = L.u_bf16;
+    a.u_bf16 = cb ? 0 : L.u_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;   // per token: folded into X_hat
@@ -797,12 +903,13 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.ds_part = ws.ds_part;
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
-    a.phi = Phi0;
+    a.phi = cb ? static_cast<const void*>(ws.codes) : Phi0;
     a.sched = plan.sched;
     a.tile_segs = ws.tile_segs;
+    a.codes_base = cb ? 1 : 0;
     const int grid = plan.sched.grid;
     LRQAT_LAUNCH("fused_dw", 1, stream,
-                 launch_dw(L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
+                 launch_dw(cb ? LRQAT_PHI_QFIXED : L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
                  "fused dW launch");
   }
   ReduceArgs ra{};
@@ -873,7 +980,7 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
     a.q = q;
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
-    LRQAT_LAUNCH("merge", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, tm_a, tm_b, a, stream),
+    LRQAT_LAUNCH("merge", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 0, tm_a, tm_b, a, stream),
                  "merge launch");
     return LRQAT_OK;
   }

@@ -1,14 +1,19 @@
 // Merge on the tensor cores (Sec. 3: after training the integer weight is
-// W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p), and W_hat = s W_Z).
+// W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p), and W_hat = s W_Z), and the
+// same pass writing the unclipped codes for the GEMMs of ranks above 64.
 //
-// One CTA of four warps per 128 x 128 tile of W_Z: the tile's rows of A (one 64-column
-// K-major box read from A; columns past r read as zeros) and columns of B (two MN-major
-// boxes of r16 rank rows read from B; rows past r read as zeros) land by TMA, r16 / 16
-// tcgen05 MMAs write the low-rank tile L = A B into TMEM, and warp q turns rows
-// 32q .. 32q + 31 into codes (TMEM lane = row): it reads L 32 columns at a time, decodes
-// the stored base of the same 32 columns from global memory, rounds, clips and stores
-// 32 int8 codes as two 16-byte words.  The pass then moves the base and the codes once
-// (the product costs 2 m k r flops on the tensor cores instead of the CUDA cores).
+// One CTA of four warps per 128 x 128 tile: the tile's rows of A and columns of B land
+// by TMA, r16 / 16 tcgen05 MMAs write the low-rank tile L = A B into TMEM, and warp q
+// turns rows 32q .. 32q + 31 into codes (TMEM lane = row): it reads L 32 columns at a
+// time, decodes the stored base of the same 32 columns from global memory, rounds,
+// clamps to [lo, hi] of the quantizer constants and stores 32 int8 codes as two 16-byte
+// words.  The pass moves the base and the codes once (the product costs 2 m k r flops
+// on the tensor cores instead of the CUDA cores).
+//   A operand: K-major boxes of 64 rank columns read from A [m, r] (r % 8 == 0; columns
+//   past r read as zeros), or (AMN) two MN-major boxes of r16 rank rows x 64 rows read
+//   from the zero-padded A^T [r16, m].
+//   B operand: two MN-major boxes of r16 rank rows x 64 columns read from B [r, k] (rows
+//   past r read as zeros) or from the zero-padded B [r16, k].
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -21,13 +26,22 @@
 namespace lrqat {
 namespace {
 
-constexpr uint32_t OFF_A = 0;                      // 128 rows x 64 bf16 (128-byte rows, SW128)
-constexpr uint32_t OFF_B = 16384;                  // two boxes of r16 rows x 64 bf16 (SW128)
-// 16 KB of A, up to 16 KB of B and 1 KB for 1024-byte alignment, padded to 52 KB so that at
-// most four CTAs share an SM: four 128-column TMEM allocations fill its 512 columns, and a
-// fifth CTA would wait inside tcgen05.alloc.
-constexpr uint32_t SMEM_BYTES = 52 * 1024;
+// A: up to 64 KB (r16 = 256), then B: two boxes of r16 rows x 128 bytes.  Small ranks
+// pad the allocation to 52 KB so that at most four CTAs share an SM: four 128-column
+// TMEM allocations fill its 512 columns, and a fifth CTA would wait inside
+// tcgen05.alloc (ranks above 64 need more shared memory, so fewer CTAs fit anyway).
+constexpr uint32_t MIN_SMEM_BYTES = 52 * 1024;
+constexpr uint32_t MAX_SMEM_BYTES = 2 * 65536 + 1024;
 constexpr uint32_t TMEM_COLS = 128;
+
+__host__ __device__ constexpr uint32_t a_tile_bytes(int r16, bool amn) {
+  return amn ? 2u * 128u * static_cast<uint32_t>(r16) : 16384u * static_cast<uint32_t>((r16 + 63) / 64);
+}
+__host__ __device__ constexpr uint32_t smem_bytes(int r16, bool amn) {
+  return a_tile_bytes(r16, amn) + 2u * 128u * static_cast<uint32_t>(r16) + 1024u < MIN_SMEM_BYTES
+             ? MIN_SMEM_BYTES
+             : a_tile_bytes(r16, amn) + 2u * 128u * static_cast<uint32_t>(r16) + 1024u;
+}
 
 // Raw words of the stored base per 32 columns of a row: 16 bytes (packed nibbles),
 // 32 bytes (one byte per value) or 64 bytes (16-bit values).
@@ -59,7 +73,7 @@ __device__ __forceinline__ void decode32(const uint32_t* w, float (&v)[32]) {
   decode16<FMT>(w + raw_words<FMT>() / 2, v + 16);
 }
 
-template <int FMT, bool UB>
+template <int FMT, bool UB, bool AMN>
 __global__ void __launch_bounds__(128) merge_tc_kernel(const __grid_constant__ CUtensorMap tm_a,
                                                        const __grid_constant__ CUtensorMap tm_b, const MergeArgs args) {
   extern __shared__ uint8_t smem_raw[];
@@ -89,20 +103,32 @@ __global__ void __launch_bounds__(128) merge_tc_kernel(const __grid_constant__ C
   tc_fence_after();
   const uint32_t tmem = tmem_base_s;
   const WaitCtl ctl{&abort_s, args.status, args.timeout_ns};
-  const uint32_t rbox = 128u * static_cast<uint32_t>(args.r16);   // bytes of one r16-row x 64-column box of B
+  const int r16 = args.r16;
+  const uint32_t rbox = 128u * static_cast<uint32_t>(r16);   // bytes of one r16-row x 64-column box
+  const uint32_t off_b = a_tile_bytes(r16, AMN);
   if (threadIdx.x == 0) {
-    mbar_arrive_expect_tx(bar_load, 16384u + 2u * rbox);
-    tma_load_2d(smem + OFF_A, &tm_a, 0, static_cast<int32_t>(rb * 128), bar_load);
-    tma_load_2d(smem + OFF_B, &tm_b, static_cast<int32_t>(cb * 128), 0, bar_load);
-    tma_load_2d(smem + OFF_B + rbox, &tm_b, static_cast<int32_t>(cb * 128 + 64), 0, bar_load);
+    mbar_arrive_expect_tx(bar_load, off_b + 2u * rbox);
+    if (AMN) {
+      tma_load_2d(smem, &tm_a, static_cast<int32_t>(rb * 128), 0, bar_load);
+      tma_load_2d(smem + rbox, &tm_a, static_cast<int32_t>(rb * 128 + 64), 0, bar_load);
+    } else {
+      for (int kb = 0; kb < (r16 + 63) / 64; ++kb)
+        tma_load_2d(smem + 16384u * kb, &tm_a, 64 * kb, static_cast<int32_t>(rb * 128), bar_load);
+    }
+    tma_load_2d(smem + off_b, &tm_b, static_cast<int32_t>(cb * 128), 0, bar_load);
+    tma_load_2d(smem + off_b + rbox, &tm_b, static_cast<int32_t>(cb * 128 + 64), 0, bar_load);
     if (wait_bounded(bar_load, 0, ctl, 1)) {
       tc_fence_after();
-      // A: K-major, 32 bytes per 16-element K step; B: MN-major, two 64-column atoms
-      // (LBO = one box), 16 rank rows = 2048 bytes per K step.
-      const uint32_t idesc = make_idesc_bf16(128, 128, 0, 1);
-      const uint64_t da = make_sdesc(smem + OFF_A, 16, 1024, SWZ_128B);
-      const uint64_t db = make_sdesc(smem + OFF_B, rbox, 1024, SWZ_128B);
-      for (int ks = 0; ks < args.r16 / 16; ++ks) mma_bf16(tmem, da + 2 * ks, db + 128 * ks, idesc, ks > 0 ? 1u : 0u);
+      // A K-major: 32 bytes per 16-element K step inside a 64-column box, one box (16 KB)
+      // per 64 ranks; A and B MN-major: two 64-wide atoms (LBO = one box), 16 rank rows =
+      // 2048 bytes per K step.
+      const uint32_t idesc = make_idesc_bf16(128, 128, AMN ? 1 : 0, 1);
+      const uint64_t db = make_sdesc(smem + off_b, rbox, 1024, SWZ_128B);
+      for (int ks = 0; ks < r16 / 16; ++ks) {
+        const uint64_t da = AMN ? make_sdesc(smem + 2048u * ks, rbox, 1024, SWZ_128B)
+                                : make_sdesc(smem + 16384u * (ks >> 2) + 32u * (ks & 3), 16, 1024, SWZ_128B);
+        mma_bf16(tmem, da, db + 128 * ks, idesc, ks > 0 ? 1u : 0u);
+      }
       mma_commit(bar_mma);
     }
   }
@@ -160,39 +186,43 @@ __global__ void __launch_bounds__(128) merge_tc_kernel(const __grid_constant__ C
   }
 }
 
-template <int FMT, bool UB>
+template <int FMT, bool UB, bool AMN>
 cudaError_t launch_merge_one(const CUtensorMap& tm_a, const CUtensorMap& tm_b, const MergeArgs& args,
                              cudaStream_t stream) {
   static bool configured[kMaxDevices] = {};
-  const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(merge_tc_kernel<FMT, UB>),
-                                         static_cast<int>(SMEM_BYTES), configured);
+  const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(merge_tc_kernel<FMT, UB, AMN>),
+                                         static_cast<int>(MAX_SMEM_BYTES), configured);
   if (e != cudaSuccess) return e;
   dim3 grid(static_cast<unsigned>(args.k / 128), static_cast<unsigned>(args.m / 128));
-  merge_tc_kernel<FMT, UB><<<grid, 128, SMEM_BYTES, stream>>>(tm_a, tm_b, args);
+  merge_tc_kernel<FMT, UB, AMN><<<grid, 128, smem_bytes(args.r16, AMN), stream>>>(tm_a, tm_b, args);
   return cudaGetLastError();
 }
 
-template <bool UB>
+template <bool UB, bool AMN>
 cudaError_t launch_merge_ub(int fmt, const CUtensorMap& tm_a, const CUtensorMap& tm_b, const MergeArgs& args,
                             cudaStream_t stream) {
   switch (fmt) {
-    case FMT_Q8: return launch_merge_one<FMT_Q8, UB>(tm_a, tm_b, args, stream);
-    case FMT_I4: return launch_merge_one<FMT_I4, UB>(tm_a, tm_b, args, stream);
-    case FMT_BF16: return launch_merge_one<FMT_BF16, UB>(tm_a, tm_b, args, stream);
-    case FMT_F16: return UB ? cudaErrorInvalidValue : launch_merge_one<FMT_F16, false>(tm_a, tm_b, args, stream);
-    case FMT_E4M3: return launch_merge_one<FMT_E4M3, UB>(tm_a, tm_b, args, stream);
-    case FMT_E5M2: return launch_merge_one<FMT_E5M2, UB>(tm_a, tm_b, args, stream);
+    case FMT_Q8: return launch_merge_one<FMT_Q8, UB, AMN>(tm_a, tm_b, args, stream);
+    case FMT_I4: return launch_merge_one<FMT_I4, UB, AMN>(tm_a, tm_b, args, stream);
+    case FMT_BF16: return launch_merge_one<FMT_BF16, UB, AMN>(tm_a, tm_b, args, stream);
+    case FMT_F16: return UB ? cudaErrorInvalidValue : launch_merge_one<FMT_F16, false, AMN>(tm_a, tm_b, args, stream);
+    case FMT_E4M3: return launch_merge_one<FMT_E4M3, UB, AMN>(tm_a, tm_b, args, stream);
+    case FMT_E5M2: return launch_merge_one<FMT_E5M2, UB, AMN>(tm_a, tm_b, args, stream);
     default: return cudaErrorInvalidValue;
   }
 }
 
 }  // namespace
 
-cudaError_t launch_merge_tc(int fmt, int u_bf16, const CUtensorMap& tm_a, const CUtensorMap& tm_b,
+static_assert(smem_bytes(256, true) <= MAX_SMEM_BYTES && smem_bytes(256, false) <= MAX_SMEM_BYTES, "smem budget");
+
+cudaError_t launch_merge_tc(int fmt, int u_bf16, int a_mn, const CUtensorMap& tm_a, const CUtensorMap& tm_b,
                             const MergeArgs& args, cudaStream_t stream) {
-  if (args.m % 128 || args.k % 128 || args.r16 < 16 || args.r16 > 64 || (args.r16 & 15)) return cudaErrorInvalidValue;
-  return u_bf16 ? launch_merge_ub<true>(fmt, tm_a, tm_b, args, stream)
-                : launch_merge_ub<false>(fmt, tm_a, tm_b, args, stream);
+  if (args.m % 128 || args.k % 128 || args.r16 < 16 || args.r16 > 256 || (args.r16 & 15)) return cudaErrorInvalidValue;
+  if (a_mn) return u_bf16 ? launch_merge_ub<true, true>(fmt, tm_a, tm_b, args, stream)
+                          : launch_merge_ub<false, true>(fmt, tm_a, tm_b, args, stream);
+  return u_bf16 ? launch_merge_ub<true, false>(fmt, tm_a, tm_b, args, stream)
+                : launch_merge_ub<false, false>(fmt, tm_a, tm_b, args, stream);
 }
 
 }  // namespace lrqat

@@ -99,6 +99,7 @@ def workload(name: str) -> Workload:
                       offsets, the paper's INT2 setting), Q2.6
     llama2_7b_attn_w4a8: 4096x4096, T=8192, r=32, W4 per channel, Q4.4, per-token dynamic int8
                       activations (the paper's weight-activation default)
+    llama2_7b_attn_r256: the 4096x4096 layer at rank 256, alpha = 256
     """
     if name == "tiny":
         return Workload(name, 64, [LayerSpec("proj", 256, 256, r=4, alpha=4.0, bits=4, group_size=0,
@@ -131,6 +132,10 @@ def workload(name: str) -> Workload:
         # the bench layer with its pre-round value formed in bf16 (the bf16 reading of Sec. 3)
         spec = _llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=PHI_QFIXED)
         return Workload(name, 8192, [replace(spec, u_bf16=True)])
+    if name == "llama2_7b_attn_r256":
+        # the bench layer at the largest rank of the paper's rank ablation (Sec. 4.1, App. A)
+        spec = _llama_layer("attn", 4096, 4096, bits=4, group_size=0, phi_format=PHI_QFIXED)
+        return Workload(name, 8192, [replace(spec, r=256, alpha=256.0)])
     if name.startswith("llama2_7b_attn_phi_"):
         # the same 4096 x 4096 W4 per-channel layer with a floating-point base (Table 2 ablation)
         fmt = {"bf16": PHI_BF16, "fp16": PHI_FP16, "fp8": PHI_FP8_E4M3, "fp8e5m2": PHI_FP8_E5M2}[name[19:]]
@@ -140,7 +145,7 @@ def workload(name: str) -> Workload:
 
 WORKLOADS = ("tiny", "llama2_7b_attn", "llama2_7b_mlp", "llama3_8b_mlp", "llama2_13b_layer", "llama2_7b_attn_int2",
              "llama2_7b_attn_w4a8", "llama2_7b_attn_phi_bf16", "llama2_7b_attn_phi_fp16", "llama2_7b_attn_phi_fp8",
-             "llama2_7b_attn_phi_fp8e5m2", "llama2_7b_attn_ubf16")
+             "llama2_7b_attn_phi_fp8e5m2", "llama2_7b_attn_ubf16", "llama2_7b_attn_r256")
 
 
 @dataclass

@@ -44,7 +44,8 @@ def _layer(**kw):
 
 
 @pytest.mark.parametrize("kw,status", [
-    (dict(m=100), -2), (dict(k=0), -1), (dict(r=0), -1), (dict(r=65), -2), (dict(bits=1), -1), (dict(bits=8), -1),
+    (dict(m=100), -2), (dict(k=0), -1), (dict(r=0), -1), (dict(r=257), -2), (dict(bits=1), -1), (dict(bits=8), -1),
+    (dict(r=65, bits=8, phi_format=LQ.PHI_BF16), -2),
     (dict(phi_format=LQ.PHI_INT_PACKED, bits=5), -1), (dict(group_size=64), -2), (dict(group_size=384), -2),
     (dict(act_bits=4), -2), (dict(phi_format=7), -1),
 ])

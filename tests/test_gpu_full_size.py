@@ -55,6 +55,7 @@ FULL_CASES = [
     ("llama2_7b_attn_w4a8_token", WL.workload("llama2_7b_attn_w4a8").layers[0], 8192),
     ("llama2_7b_attn_phi_bf16", WL.workload("llama2_7b_attn_phi_bf16").layers[0], 8192),
     ("llama2_7b_attn_phi_fp8", WL.workload("llama2_7b_attn_phi_fp8").layers[0], 8192),
+    ("llama2_7b_attn_r256", WL.workload("llama2_7b_attn_r256").layers[0], 8192),
 ]
 
 
@@ -208,6 +209,8 @@ MERGE_CASES = [
     ("llama2_7b_attn_r20", WL.LayerSpec("attn_r20", 4096, 4096, 20, 20.0, 4, 0, WL.PHI_QFIXED, a_std=0.25,
                                         b_std=0.25)),
     ("llama2_7b_attn_phi_bf16", _merge_spec(WL.workload("llama2_7b_attn_phi_bf16").layers[0])),
+    ("llama2_7b_attn_r256", dataclasses.replace(WL.workload("llama2_7b_attn_r256").layers[0], a_std=0.15,
+                                                b_std=0.15)),
 ]
 
 

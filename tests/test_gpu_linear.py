@@ -72,6 +72,17 @@ CASES = [
                                        a_std=0.3, b_std=0.3), 130),
     ("int3_packed_ubf16_a8", spec_of("y", 128, 256, 16, bits=3, phi=WL.PHI_INT_PACKED, act=8, ub=True, a_std=0.3,
                                      b_std=0.3), 97),
+    # ranks above 64: the codes pass writes round(u) once per call, the GEMMs read it as their
+    # base and dW runs its adapter contractions in rounds of 64 ranks
+    ("q44_pc_r96", spec_of("lr1", 384, 512, 96, a_std=0.1, b_std=0.1), 700),
+    ("q44_pc_r128_ubf16", spec_of("lr2", 256, 512, 128, ub=True, a_std=0.1, b_std=0.1), 300),
+    ("q44_pc_r256", spec_of("lr3", 256, 640, 256, a_std=0.1, b_std=0.1), 1000),
+    ("int3_packed_r100", spec_of("lr4", 256, 512, 100, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.1, b_std=0.1), 513),
+    ("q44_g128_a8_r200", spec_of("lr5", 256, 384, 200, group=128, act=8, a_std=0.1, b_std=0.1), 300),
+    ("int2_asym_r72", spec_of("lr6", 256, 512, 72, bits=2, asym=True, shift=0.03, a_std=0.1, b_std=0.1), 333),
+    ("bf16_pc_a8_token_r160", spec_of("lr7", 256, 256, 160, phi=WL.PHI_BF16, act=8, per_token=True, a_std=0.1,
+                                      b_std=0.1), 200),
+    ("fp8_e4m3_w2_r256_clip", spec_of("lr8", 128, 512, 256, bits=2, phi=WL.PHI_FP8_E4M3, a_std=0.2, b_std=0.2), 97),
 ]
 
 
@@ -170,6 +181,11 @@ CODE_CASES = [
     ("q44_pc_ubf16", spec_of("c11", 256, 256, 32, ub=True, a_std=0.3, b_std=0.3)),
     ("fp8_e4m3_ubf16_alpha1", spec_of("c12", 128, 384, 16, phi=WL.PHI_FP8_E4M3, alpha=1.0, ub=True, a_std=0.5,
                                       b_std=0.5)),
+    ("q44_pc_r96", spec_of("c13", 256, 256, 96, a_std=0.1, b_std=0.1)),
+    ("int3_packed_r100", spec_of("c14", 128, 256, 100, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.1, b_std=0.1)),
+    ("int2_asym_g128_r256", spec_of("c15", 128, 256, 256, bits=2, group=128, asym=True, shift=0.03, a_std=0.1,
+                                    b_std=0.1)),
+    ("bf16_pc_r256_ubf16", spec_of("c16", 128, 256, 256, phi=WL.PHI_BF16, ub=True, a_std=0.1, b_std=0.1)),
 ]
 
 
@@ -238,7 +254,7 @@ def test_bf16_pre_round_moves_codes():
     assert (codes[False] != codes[True]).mean() > 0.001
 
 
-@pytest.mark.parametrize("r", [8, 32, 40])
+@pytest.mark.parametrize("r", [8, 32, 40, 256])
 def test_direct_and_padded_factor_paths_agree(r):
     """The forward reads A and B straight from the caller's arrays when they are 16-byte
     aligned (r a multiple of 8), else through padded copies; both fill the same shared
@@ -322,6 +338,7 @@ TAIL_CASES = [
     ("a8_token", spec_of("p", 256, 512, 32, act=8, per_token=True, a_std=0.2, b_std=0.2), 1301),
     ("bf16_pc", spec_of("r", 256, 512, 32, phi=WL.PHI_BF16, a_std=0.2, b_std=0.2), 1250),
     ("whole_wave_then_tail", spec_of("z", 2048, 2560, 16, a_std=0.2, b_std=0.2), 650),
+    ("q44_pc_r256", spec_of("lt", 256, 512, 256, a_std=0.1, b_std=0.1), 1000),
 ]
 
 
@@ -352,3 +369,34 @@ def test_dw_schedules_agree(dw_schedule):
     assert O.rel_fro(outs["tail"]["ds"], outs["split"]["ds"]) <= 1e-5
     for key in ("dA", "dB"):
         assert O.rel_fro(outs["tail"][key], outs["split"][key]) <= 1e-2, key
+
+
+MERGE_RANK_CASES = [
+    # tensor-core merge reading A and B directly (rank a multiple of 8), and the CUDA-core merge
+    # (rank 100; and rank 96 with the factors shifted off 16-byte alignment), both in rank blocks
+    ("q44_r256_tc", spec_of("mr1", 256, 384, 256, a_std=0.1, b_std=0.1), 0),
+    ("int3_packed_r96_tc", spec_of("mr2", 128, 512, 96, bits=3, phi=WL.PHI_INT_PACKED, a_std=0.1, b_std=0.1), 0),
+    ("q35_r100_cuda_cores", spec_of("mr3", 256, 256, 100, bits=3, a_std=0.1, b_std=0.1), 0),
+    ("fp8_r96_shifted", spec_of("mr4", 128, 256, 96, phi=WL.PHI_FP8_E4M3, a_std=0.1, b_std=0.1), 1),
+]
+
+
+@pytest.mark.parametrize("cid,spec,shift", MERGE_RANK_CASES, ids=[c[0] for c in MERGE_RANK_CASES])
+def test_merge_large_ranks(cid, spec, shift):
+    """lrqat_merge for ranks above 64: every code equals the oracle's merge outside near-ties."""
+    t = torch()
+    data = WL.make_layer(spec, 1, seed=12, with_activations=False)
+    dl = DeviceLayer(data)
+    A = t.empty(dl.A.numel() + 8, dtype=t.int16, device="cuda")[shift:shift + dl.A.numel()].view(dl.A.shape)
+    B = t.empty(dl.B.numel() + 8, dtype=t.int16, device="cuda")[shift:shift + dl.B.numel()].view(dl.B.shape)
+    A.copy_(dl.A)
+    B.copy_(dl.B)
+    wz = t.empty((spec.m, spec.k), dtype=t.int8, device="cuda")
+    LQ.merge(dl.layer, dl.phi0, A, B, wz)
+    LQ.get_device_status()
+    OL = oracle_layer(spec)
+    _, _, phi0 = oracle_base(data, OL)
+    ref = O.merge(phi0, data.A, data.B, OL)
+    exempt = O.near_tie(O.preround(phi0, data.A, data.B, OL))
+    assert ((wz.cpu().numpy() != ref) & ~exempt).sum() == 0
+    assert (ref != O.merge(phi0, data.A, np.zeros_like(data.B), OL)).mean() > 0.01   # the low-rank term matters
