@@ -366,24 +366,28 @@ def run_gpu(args):
     achieved = dom_flops_total / (ms_dom / 1e3) / 1e12
     traffic = profiled_traffic(dom, args.workload)
 
-    # 3) end to end: pinned host inputs in, step results out, inside the timed region.  Like a training
-    #    loop's data prefetch, step i+1's inputs are copied on a second stream while step i computes, and
-    #    step i's outputs are read back on a third stream while step i+1 computes (device inputs and
-    #    outputs double-buffered); every step's copies are inside the timed region.
+    # 3) end to end: pinned host inputs in, the step's result out, inside the timed region.  The inputs
+    #    are every layer's X and dY; the result is what the step produces for the optimizer, the
+    #    gradients dA, dB, ds of every layer (Y and dX stay on the device, where a network's adjacent
+    #    layers consume them).  Like a training loop's data prefetch, step i+1's inputs are copied on a
+    #    second stream while step i computes, and step i's gradients are read back on a third stream
+    #    while step i+1 computes (device inputs and outputs double-buffered); every step's copies are
+    #    inside the timed region.
     import numpy as np
     pin = lambda a: torch.from_numpy(np.ascontiguousarray(a.view(np.int16))).pin_memory()
     hx = {id(l): pin(l["X_host"]) for l in gw.layers}
     hdy = {id(l): pin(l["dY_host"]) for l in gw.layers}
-    out_names = ("Y", "dX", "dA", "dB", "ds")
+    out_names = ("Y", "dX", "dA", "dB", "ds")   # written by the step
+    result_names = ("dA", "dB", "ds")           # read back to the host
     d_in = [({id(l): l["X"][0] for l in gw.layers}, {id(l): l["dY"][0] for l in gw.layers}),
             ({id(l): torch.empty_like(l["X"][0]) for l in gw.layers},
              {id(l): torch.empty_like(l["dY"][0]) for l in gw.layers})]
     d_out = [{id(l): {n: l[n] for n in out_names} for l in gw.layers},
              {id(l): {n: torch.empty_like(l[n]) for n in out_names} for l in gw.layers}]
-    h_out = [{id(l): {n: torch.empty(l[n].shape, dtype=l[n].dtype, pin_memory=True) for n in out_names}
+    h_out = [{id(l): {n: torch.empty(l[n].shape, dtype=l[n].dtype, pin_memory=True) for n in result_names}
               for l in gw.layers} for _ in range(2)]
     h2d = sum(t.numel() * t.element_size() for t in list(hx.values()) + list(hdy.values()))
-    d2h = sum(t.numel() * t.element_size() for t in h_out[0][id(gw.layers[0])].values()) * len(gw.layers)
+    d2h = sum(t.numel() * t.element_size() for l in gw.layers for t in h_out[0][id(l)].values())
     comp = torch.cuda.current_stream()
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
     ev_in = [torch.cuda.Event() for _ in range(2)]
@@ -415,7 +419,7 @@ def run_gpu(args):
             with torch.cuda.stream(s_out):
                 s_out.wait_event(ev_comp[b])
                 for l in gw.layers:
-                    for n in out_names:
+                    for n in result_names:
                         h_out[b][id(l)][n].copy_(d_out[b][id(l)][n], non_blocking=True)
                 ev_out[b].record(s_out)
         comp.wait_stream(s_out)
@@ -477,7 +481,8 @@ def run_gpu(args):
         "traced_ms_per_step": ms_traced / args.steps,
         "gpu_launches": launches,
         "e2e": {"value": units_e2e / (ms_e2e / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                "d2h_bytes_per_step": d2h, "steps": e2e_steps, "h2d": "X and dY of every layer",
+                "d2h": "dA, dB and ds of every layer (the step's result)"},
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "samples": clk["samples"], "power_w_max": clk.get("power_w_max")},
     }
