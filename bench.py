@@ -389,16 +389,21 @@ def run_gpu(args):
     h2d = sum(t.numel() * t.element_size() for t in list(hx.values()) + list(hdy.values()))
     d2h = sum(t.numel() * t.element_size() for l in gw.layers for t in h_out[0][id(l)].values())
     comp = torch.cuda.current_stream()
-    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    # X and dY go up on two streams (two copy engines), the result comes back on a third
+    s_in, s_in2, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev_in = [torch.cuda.Event() for _ in range(2)]
     ev_comp = [torch.cuda.Event() for _ in range(2)]
     ev_out = [torch.cuda.Event() for _ in range(2)]
 
     def copy_in(b):
+        s_in2.wait_stream(s_in)
+        with torch.cuda.stream(s_in2):
+            for l in gw.layers:
+                d_in[b][1][id(l)].copy_(hdy[id(l)], non_blocking=True)
         with torch.cuda.stream(s_in):
             for l in gw.layers:
                 d_in[b][0][id(l)].copy_(hx[id(l)], non_blocking=True)
-                d_in[b][1][id(l)].copy_(hdy[id(l)], non_blocking=True)
+            s_in.wait_stream(s_in2)
             ev_in[b].record(s_in)
 
     def e2e_run(steps: int):
