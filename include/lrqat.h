@@ -307,6 +307,22 @@ int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const flo
  * values. */
 int lrqat_set_dw_schedule(int schedule);
 
+/* Tuning (no counterpart in the paper): the kernel of the forward and dX GEMMs.
+ * 1 = the one-SM kernel (128 weight rows x 448 tokens per SM); 2 = CTA pairs (tcgen05
+ * MMAs of 256 rows across the two SMs of a cluster, each SM holding half of the token
+ * operand; 256 rows x 384 tokens per pair) wherever the produced weight operand has a
+ * multiple of 256 rows (m for the forward, k for dX), the one-SM kernel otherwise;
+ * 0 (the default) = pairs where the base holds the precomputed codes (ranks above 64) and
+ * the one-SM kernel where the GEMM computes the low-rank tile itself, the faster of the two
+ * measured for each.  All give the same codes; outputs agree up to fp32 summation order.
+ * Process-wide; the environment variable LRQAT_GEMM_VARIANT ("auto", "single" or "pair")
+ * gives the start value, read once when the library is loaded.  Returns
+ * LRQAT_ERR_INVALID_ARG for other values. */
+int lrqat_set_gemm_variant(int variant);
+/* The current settings of lrqat_set_gemm_variant and lrqat_set_dw_schedule. */
+int lrqat_get_gemm_variant(void);
+int lrqat_get_dw_schedule(void);
+
 /* Synchronizes `stream`, then reads and clears the device status word of the
  * current device.  Returns LRQAT_OK, LRQAT_ERR_TIMEOUT (a kernel's bounded
  * wait gave up since the last call) or LRQAT_ERR_CUDA. */

@@ -1,0 +1,605 @@
+// Fused LR-QAT GEMM for the forward (Y = X W_hat^T) and the input gradient
+// (dX = dY W_hat) on CTA pairs: the same on-chip recompute of W_hat as the one-SM
+// kernel (Eq. 8; the recompute replaces the checkpointing of Sec. 3), with the main
+// product issued as tcgen05 MMAs of M = 256 rows across the two SMs of a cluster.
+//
+// Why pairs: the one-SM kernel is bound by its shared-memory port (each 64-wide stage of a
+// 128 x 448 tile moves ~192 KB through it, two thirds of it the token operand, written by
+// TMA and read by the MMAs).  In a pair each CTA holds its own 128 weight rows and only half
+// of every accumulator's tokens; the tensor cores of the pair exchange the token halves, so
+// each SM moves ~124 KB per stage for 128 rows x 384 tokens.
+//
+// A pair processes tiles of 256 weight rows (CTA rank c: rows 128 c .. 128 c + 127) x 384
+// tokens (two accumulators of 192 tokens; CTA c holds tokens 96 c .. 96 c + 95 of each), one
+// 64-wide slice of the contraction per stage:
+//   * token ring (4 slots per CTA): four loader warps, one per slot, bring this CTA's two
+//     96-token halves (SW128) with TMA whose completion lands on the leader's barrier; each
+//     slot also holds this CTA's W_hat tile of the stage;
+//   * factor ring (4 slots; 2 for 16-bit bases): the stored base of this CTA's rows (completion on its own
+//     barrier; only its own producers read it) and this CTA's half (32 rows) of the second
+//     factor's slice (completion on the leader's barrier: the low-rank MMA reads both halves);
+//   * the leader's MMA thread issues the low-rank tile L = RF SF^T (M = 256, N = 64) two
+//     stages ahead into one of two TMEM buffers, and the main product (M = 256, N = 192,
+//     8 MMAs per stage); every commit is multicast to both CTAs;
+//   * sixteen producer warps per CTA build this CTA's W_hat tile exactly as the one-SM kernel
+//     does, and drain this CTA's 128 rows of the accumulators in the epilogue.
+// The leader waits for the peer's "W_hat written", "L read" and "accumulators drained" events;
+// each peer warp reports them with a 16-byte copy into the leader's shared memory whose
+// completion counts on the leader's barrier (a thread-issued remote arrive is several times
+// slower under the pair's operand traffic), after fence.proxy.async has ordered its writes.
+// Ranks above 64 (NL): the base holds the codes (as in the one-SM kernel); no factors, no L.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "kernels.h"
+#include "ptx.cuh"
+#include "quant.cuh"
+
+namespace lrqat {
+namespace {
+
+constexpr int BM = 128;                          // weight rows per CTA (256 per pair)
+constexpr int BK = 64;
+constexpr int BNP = 192;                         // tokens per accumulator (N of the pair MMA)
+constexpr int BNH = BNP / 2;                     // tokens per accumulator held by one CTA
+constexpr int NACC = 2;
+constexpr int BTP = BNP * NACC;                  // 384 tokens per pair tile
+constexpr int NT = 4;                            // token ring slots
+constexpr int NF_MAX = 4;                        // factor ring slots (2 for 16-bit bases)
+constexpr int NUM_PROD_WARPS = 16;
+constexpr int FIRST_TMA_WARP = 2 + NUM_PROD_WARPS;
+constexpr int NUM_TMA_WARPS = NT + 1;
+constexpr int NUM_THREADS = 32 * (FIRST_TMA_WARP + NUM_TMA_WARPS);
+constexpr int EPI_COLS = NACC * BNP / 4;         // accumulator columns drained per warp (96)
+constexpr uint32_t SIG_TX = 16u * NUM_PROD_WARPS;   // bytes of the peer's per-warp signals
+
+constexpr uint32_t RF_BYTES = 128 * 128;         // 128 rows x 64 rank columns (bf16)
+constexpr uint32_t TOK_BOX = BNH * 128;          // 96 tokens x 64 bf16
+constexpr uint32_t TOK_BYTES = NACC * TOK_BOX;
+constexpr uint32_t W_BYTES = 128 * 128;          // 128 rows x 64 bf16
+constexpr uint32_t SFH_BYTES = 32 * 128;         // 32 slice rows x up to 64 rank columns (bf16)
+constexpr uint32_t TSLOT_BYTES = TOK_BYTES + W_BYTES;
+constexpr uint32_t OFF_RF = 0;
+constexpr uint32_t OFF_TSLOTS = RF_BYTES;
+constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
+constexpr uint32_t TS_W = TOK_BYTES;
+
+template <int FMT>
+struct PairRing {
+  static constexpr int NF = fmt_16bit(FMT) ? 2 : 4;
+  static constexpr uint32_t PHI_BYTES = fmt_16bit(FMT) ? 128 * 128 : 128 * 64;
+  static constexpr uint32_t PHI_TX = FMT == FMT_I4 ? PHI_BYTES / 2 : PHI_BYTES;
+  static constexpr uint32_t FSLOT_BYTES = PHI_BYTES + SFH_BYTES;
+  static constexpr uint32_t FS_SF = PHI_BYTES;
+  static constexpr uint32_t SMEM_BYTES = OFF_FSLOTS + NF * FSLOT_BYTES + 1024;
+  static_assert(FSLOT_BYTES % 1024 == 0 && FS_SF % 1024 == 0, "swizzled tiles must start on 1024-byte boundaries");
+  static_assert(SMEM_BYTES + 1024 <= 232448, "shared memory budget");
+};
+static_assert(TSLOT_BYTES % 1024 == 0 && TOK_BOX % 1024 == 0 && TS_W % 1024 == 0 && OFF_FSLOTS % 1024 == 0,
+              "swizzled tiles must start on 1024-byte boundaries");
+static_assert(EPI_COLS % 16 == 0, "epilogue drains 16-column chunks");
+
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t COL_L = NACC * BNP;           // two 64-column low-rank buffers at 384 and 448
+static_assert(COL_L + 2 * BK <= TMEM_COLS, "TMEM budget");
+
+constexpr int BAR_TFULL = 0;                     // leader: both token halves of the slot landed
+constexpr int BAR_TEMPTY = BAR_TFULL + NT;       // both: main product of the slot finished
+constexpr int BAR_WFULL = BAR_TEMPTY + NT;       // leader: both W_hat tiles of the slot written
+constexpr int BAR_PFULL = BAR_WFULL + NT;        // both: this CTA's base tile landed
+
+constexpr int BAR_FFULL = BAR_PFULL + NF_MAX;    // leader: both factor-slice halves landed
+constexpr int BAR_FEMPTY = BAR_FFULL + NF_MAX;   // both: slot read by this CTA's producers (after L)
+constexpr int BAR_LFULL = BAR_FEMPTY + NF_MAX;   // both: low-rank tile of the buffer computed
+constexpr int BAR_LEMPTY = BAR_LFULL + 2;        // leader: both CTAs read the buffer
+constexpr int BAR_RFFULL = BAR_LEMPTY + 2;       // leader: both row-factor halves landed
+constexpr int BAR_RFEMPTY = BAR_RFFULL + 1;      // both: last low-rank MMA of the tile finished
+constexpr int BAR_ACCFULL = BAR_RFEMPTY + 1;     // both: accumulators of the tile complete
+constexpr int BAR_ACCEMPTY = BAR_ACCFULL + 1;    // leader: both CTAs drained them
+constexpr int BAR_DRAIN = BAR_ACCEMPTY + 1;
+constexpr int NUM_BARS = BAR_DRAIN + 1;
+
+__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > timeout_ns) break;
+  }
+}
+
+// Stages are numbered globally over the pair's tiles (gg), identically in both CTAs: token
+// slot gg % NT, factor slot gg % NF, low-rank buffer gg % 2.
+template <int MODE, int FMT, bool ZP, bool UB, bool NL>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    fused_pair_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
+                      const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
+                      const FusedArgs args) {
+  using PR = PairRing<FMT>;
+  constexpr int NF = PR::NF;
+  constexpr bool PACKED = FMT == FMT_I4;
+  constexpr uint32_t FSLOT_BYTES = PR::FSLOT_BYTES;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t bars[NUM_BARS];
+  __shared__ __align__(16) uint32_t sig_buf[8];   // [0, 4): source of the peer's signals, [4, 8): their target
+  __shared__ uint32_t tmem_base_s;
+  __shared__ volatile int abort_s;
+
+  const uint32_t smem = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_cta_rank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  auto bar = [&](int i) { return smem_u32(&bars[i]); };
+  auto lbar = [&](int i) { return map_shared_rank(smem_u32(&bars[i]), 0); };   // the leader's copy
+
+  if (threadIdx.x == 0) {
+    abort_s = 0;
+    for (int s = 0; s < NT; ++s) {
+      mbar_init(bar(BAR_TFULL + s), 1);
+      mbar_init(bar(BAR_TEMPTY + s), 1);
+      mbar_init(bar(BAR_WFULL + s), NUM_PROD_WARPS);
+    }
+    for (int s = 0; s < NF; ++s) {
+      mbar_init(bar(BAR_PFULL + s), 1);
+      mbar_init(bar(BAR_FFULL + s), 1);
+      // freed by this CTA's producers after they built W_hat: by then they have waited for the
+      // low-rank tile, so the low-rank MMA that read the slot's factor half has completed
+      mbar_init(bar(BAR_FEMPTY + s), NUM_PROD_WARPS);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(bar(BAR_LFULL + b), 1);
+      mbar_init(bar(BAR_LEMPTY + b), NUM_PROD_WARPS);
+    }
+    mbar_init(bar(BAR_RFFULL), 1);
+    mbar_init(bar(BAR_RFEMPTY), 1);
+    mbar_init(bar(BAR_ACCFULL), 1);
+    mbar_init(bar(BAR_ACCEMPTY), NUM_PROD_WARPS);
+    mbar_init(bar(BAR_DRAIN), 1);
+    mbar_fence_init();
+  }
+  if (warp == 1) tmem_alloc_pair(smem_u32(&tmem_base_s), TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();   // both CTAs' barriers exist before either signals the other
+  tc_fence_after();
+  const uint32_t tmem = tmem_base_s;
+  const WaitCtl ctl{&abort_s, args.status, args.timeout_ns};
+  const int nk = args.kdim / BK;   // at least 2 (kdim is a multiple of 128)
+  const int num_rb2 = args.num_rb / 2;   // 256-row blocks
+  const int num_tiles = num_rb2 * ((args.T + BTP - 1) / BTP);
+  const uint32_t sig_src = smem_u32(&sig_buf[0]);
+  const uint32_t sig_dst_leader = map_shared_rank(smem_u32(&sig_buf[4]), 0);
+  // A producer warp's event on a leader barrier: the leader's warps arrive (warp 0 also
+  // announces the peer's 16 signal bytes per warp), the peer's warps send their signal.
+  auto report = [&](int b, int pw) {
+    if (leader) {
+      if (pw == 0) mbar_arrive_expect_tx(bar(b), SIG_TX);
+      else mbar_arrive(bar(b));
+    } else {
+      signal_remote16(sig_dst_leader, sig_src, lbar(b));
+    }
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------- row factor (per tile)
+    if (!NL && lane == 0) {
+      prefetch_tensormap(&tm_rf);
+      uint32_t it = 0;
+      for (int tile = pair; tile < num_tiles; tile += npairs) {
+        const int rb2 = tile % num_rb2;
+        if (!wait_spin_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1)) break;
+        if (leader) mbar_arrive_expect_tx(bar(BAR_RFFULL), 2u * RF_BYTES);
+        tma_load_2d_pair(smem + OFF_RF, &tm_rf, 0, rb2 * 2 * BM + static_cast<int>(rank) * BM, lbar(BAR_RFFULL));
+        ++it;
+      }
+    }
+  } else if (warp >= FIRST_TMA_WARP && warp < FIRST_TMA_WARP + NT) {
+    // ------------------------------------------- token loaders (one per slot)
+    const uint32_t t = warp - FIRST_TMA_WARP;
+    if (lane == 0) {
+      prefetch_tensormap(&tm_tok);
+      const uint32_t st = smem + OFF_TSLOTS + t * TSLOT_BYTES;
+      const uint32_t fb = lbar(BAR_TFULL + t), eb = bar(BAR_TEMPTY + t);
+      uint32_t g = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
+        const int tb = tile / num_rb2;
+        for (int kk = 0; kk < nk; ++kk) {
+          const uint32_t gg = g + kk;
+          if (gg % NT != t) continue;
+          const uint32_t n = gg / NT;
+          if (!(ok = wait_spin_bounded(eb, (n & 1u) ^ 1u, ctl, 2))) break;
+          if (leader) mbar_arrive_expect_tx(bar(BAR_TFULL + t), 2u * TOK_BYTES);
+          const int tok = tb * BTP + static_cast<int>(rank) * BNH;
+          tma_load_2d_pair(st, &tm_tok, kk * BK, tok, fb);
+          tma_load_2d_pair(st + TOK_BOX, &tm_tok, kk * BK, tok + BNP, fb);
+        }
+        g += nk;
+      }
+    }
+  } else if (warp == FIRST_TMA_WARP + NT) {
+    // ------------------------------------------------- factor-ring loader
+    if (lane == 0) {
+      prefetch_tensormap(&tm_phi);
+      if (!NL) prefetch_tensormap(&tm_sf);
+      const uint32_t sf_tx = static_cast<uint32_t>(32 * 2 * args.sf_cols);   // one CTA's half slice
+      uint32_t gg = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
+        const int rb2 = tile % num_rb2;
+        for (int kk = 0; kk < nk; ++kk, ++gg) {
+          const uint32_t s = gg % NF;
+          if (!(ok = wait_spin_bounded(bar(BAR_FEMPTY + s), ((gg / NF) & 1u) ^ 1u, ctl, 3))) break;
+          const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
+          mbar_arrive_expect_tx(bar(BAR_PFULL + s), PR::PHI_TX);
+          tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb2 * 2 * BM + static_cast<int>(rank) * BM,
+                      bar(BAR_PFULL + s));
+          if (!NL) {
+            if (leader) mbar_arrive_expect_tx(bar(BAR_FFULL + s), 2u * sf_tx);
+            tma_load_2d_pair(fs + PR::FS_SF, &tm_sf, 0, kk * BK + static_cast<int>(rank) * 32, lbar(BAR_FFULL + s));
+          }
+        }
+      }
+      if (gg > 0) {
+        const uint32_t last = gg - 1;
+        drain_wait(bar(BAR_PFULL + last % NF), (last / NF) & 1u, args.timeout_ns);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (the leader's)
+    if (leader && lane == 0) {
+      const uint32_t idesc_main = make_idesc_bf16(256, BNP, 0, 0);
+      const uint32_t idesc_l = make_idesc_bf16(256, BK, 0, 0);
+      const int lsteps = NL ? 0 : args.r16 / 16;
+      constexpr uint32_t TSLOT_D = TSLOT_BYTES >> 4, FSLOT_D = FSLOT_BYTES >> 4, TOKB_D = TOK_BOX >> 4;
+      const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
+      // the K-major half slice: 32 rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to match)
+      const uint32_t sf_swz = args.sf_cols == 64 ? SWZ_128B : args.sf_cols == 32 ? SWZ_64B : SWZ_32B;
+      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + PR::FS_SF, 16, 16u * args.sf_cols, sf_swz);
+      const uint64_t d_w0 = make_sdesc(smem + OFF_TSLOTS + TS_W, 16, 1024, SWZ_128B);
+      const uint64_t d_tok0 = make_sdesc(smem + OFF_TSLOTS, 16, 1024, SWZ_128B);
+      uint32_t g = 0, it = 0;
+      bool ok = true;
+      // L(gg) into buffer gg % 2 once both factor halves landed and both CTAs read L(gg - 2)
+      auto issue_lowrank = [&](uint32_t gg) -> bool {
+        const uint32_t s = gg % NF, b = gg & 1u;
+        if (!wait_spin_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4)) return false;
+        if (!wait_spin_bounded(bar(BAR_LEMPTY + b), ((gg >> 1) & 1u) ^ 1u, ctl, 5)) return false;
+        tc_fence_after();
+        const uint64_t sf = d_sf0 + s * FSLOT_D;
+        const uint32_t dl = tmem + COL_L + BK * b;
+        for (int ks = 0; ks < lsteps; ++ks) mma_bf16_pair(dl, d_rf + 2 * ks, sf + 2 * ks, idesc_l, ks > 0 ? 1u : 0u);
+        mma_commit_pair(bar(BAR_LFULL + b));
+        return true;
+      };
+      for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
+        if (!NL) {
+          if (!(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
+          if (!(ok = issue_lowrank(g))) break;
+          if (!(ok = issue_lowrank(g + 1))) break;
+          if (nk == 2) mma_commit_pair(bar(BAR_RFEMPTY));
+        }
+        if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
+        tc_fence_after();
+        for (int kk = 0; kk < nk; ++kk) {
+          const uint32_t gg = g + kk;
+          const uint32_t s = gg % NT, ph = (gg / NT) & 1u;
+          if (!NL && kk + 2 < nk) {
+            if (!(ok = issue_lowrank(gg + 2))) break;
+            if (kk + 3 == nk) mma_commit_pair(bar(BAR_RFEMPTY));   // last read of the row factor issued
+          }
+          if (!(ok = wait_spin_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
+          if (!(ok = wait_spin_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
+          tc_fence_after();
+          const uint64_t w = d_w0 + s * TSLOT_D, t = d_tok0 + s * TSLOT_D;
+          const uint32_t acc = kk > 0 ? 1u : 0u;
+          static_assert(NACC == 2 && BK == 64, "issue sequence below is written for 2 accumulators x 4 K steps");
+          mma_bf16_pair(tmem, w, t, idesc_main, acc);
+          mma_bf16_pair(tmem, w + 2, t + 2, idesc_main, 1u);
+          mma_bf16_pair(tmem, w + 4, t + 4, idesc_main, 1u);
+          mma_bf16_pair(tmem, w + 6, t + 6, idesc_main, 1u);
+          mma_bf16_pair(tmem + BNP, w, t + TOKB_D, idesc_main, acc);
+          mma_bf16_pair(tmem + BNP, w + 2, t + TOKB_D + 2, idesc_main, 1u);
+          mma_bf16_pair(tmem + BNP, w + 4, t + TOKB_D + 4, idesc_main, 1u);
+          mma_bf16_pair(tmem + BNP, w + 6, t + TOKB_D + 6, idesc_main, 1u);
+          mma_commit_pair(bar(BAR_TEMPTY + s));
+        }
+        if (!ok) break;
+        mma_commit_pair(bar(BAR_ACCFULL));
+        g += nk;
+        ++it;
+      }
+      if (ok) {
+        // the peer's last signals (the final drain, the reads of the last two low-rank
+        // tiles) land before the CTAs end
+        ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 10);
+        for (uint32_t gg = g >= 2 ? g - 2 : 0; ok && !NL && gg < g; ++gg)
+          ok = wait_spin_bounded(bar(BAR_LEMPTY + (gg & 1u)), (gg >> 1) & 1u, ctl, 11);
+      }
+      mma_commit_pair_self(bar(BAR_DRAIN));
+      drain_wait(bar(BAR_DRAIN), 0, args.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------- W_hat producers + epilogue
+    const int pw = warp - 2;              // 0..15
+    const int q = warp & 3;               // TMEM lane quarter this warp may access
+    const int c = pw >> 2;                // 16-column chunk of the 64-wide slice (and epilogue block)
+    const int row = q * 32 + lane;        // row of this CTA's tile handled by this thread
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const QuantParams qp = args.q;
+    const uint32_t lr2 = pack_rn_bf16x2(qp.lr_scale, qp.lr_scale);
+    uint32_t g = 0;
+    uint32_t it = 0;
+    bool ok = true;
+    for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
+      const int rb2 = tile % num_rb2;
+      const int tb = tile / num_rb2;
+      const int row_g = rb2 * 2 * BM + static_cast<int>(rank) * BM + row;
+      for (int kk = 0; kk < nk; ++kk) {
+        const uint32_t gg = g + kk;
+        float sc[16];
+        uint32_t zw[8];
+        if (ZP) {
+          if (MODE == FUSED_DX) {
+            const int i0 = kk * BK + 16 * c;
+            float zv[16];
+            if (args.s_ld == 0) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float4 v = __ldg(reinterpret_cast<const float4*>(args.zero + i0) + e);
+                zv[4 * e] = v.x;
+                zv[4 * e + 1] = v.y;
+                zv[4 * e + 2] = v.z;
+                zv[4 * e + 3] = v.w;
+              }
+            } else {
+              const int gcol = row_g / args.group_size;
+#pragma unroll
+              for (int e = 0; e < 16; ++e) zv[e] = __ldg(args.zero + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) zw[e] = pack_rn_bf16x2(zv[2 * e], zv[2 * e + 1]);
+          } else {
+            const float zr = MODE == FUSED_FWD_GROUP
+                                 ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size]
+                                 : args.zero[row_g];
+            const uint32_t z2 = pack_rn_bf16x2(zr, zr);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) zw[e] = z2;
+          }
+        }
+        if (MODE == FUSED_FWD_GROUP) {
+          const float v = args.s[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) sc[e] = v;
+        } else if (MODE == FUSED_DX) {
+          const int i0 = kk * BK + 16 * c;
+          if (args.s_ld == 0) {
+            const float4* sp = reinterpret_cast<const float4*>(args.s + i0);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float4 v = __ldg(sp + e);
+              sc[4 * e] = v.x;
+              sc[4 * e + 1] = v.y;
+              sc[4 * e + 2] = v.z;
+              sc[4 * e + 3] = v.w;
+            }
+          } else {
+            const int gcol = row_g / args.group_size;
+#pragma unroll
+            for (int e = 0; e < 16; ++e) sc[e] = __ldg(args.s + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
+          }
+        }
+        const uint32_t fslot = gg % NF;
+        ok = wait_bounded(bar(BAR_PFULL + fslot), (gg / NF) & 1u, ctl, 12);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
+        float v[16];
+        uint32_t raw[8];
+        if (PACKED) {
+          const uint2 r = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
+          raw[0] = r.x;
+          raw[1] = r.y;
+        } else if (fmt_16bit(FMT)) {
+          const uint4 r0 = ld_shared_v4(fs + swz_offset(row, 2 * c, 128));
+          const uint4 r1 = ld_shared_v4(fs + swz_offset(row, 2 * c + 1, 128));
+          raw[0] = r0.x, raw[1] = r0.y, raw[2] = r0.z, raw[3] = r0.w;
+          raw[4] = r1.x, raw[5] = r1.y, raw[6] = r1.z, raw[7] = r1.w;
+        } else {
+          const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
+          raw[0] = r.x, raw[1] = r.y, raw[2] = r.z, raw[3] = r.w;
+        }
+        decode16<FMT>(raw, v);
+        float Lv[16];
+        if (!NL) {
+          const uint32_t lb = gg & 1u;
+          ok = wait_bounded(bar(BAR_LFULL + lb), (gg >> 1) & 1u, ctl, 13);
+          if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+          tc_fence_after();
+          tmem_ld16(tmem + lane_off + COL_L + BK * lb + 16 * c, Lv);
+          tmem_ld_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) report(BAR_LEMPTY + lb, pw);
+        }
+        uint32_t w[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float2 u =
+              NL   ? make_float2(v[2 * e], v[2 * e + 1])
+              : UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
+                   : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
+                                make_float2(v[2 * e], v[2 * e + 1]));
+          const float2 t2 = __fadd2_rn(u, make_float2(qp.magic, qp.magic));
+          uint32_t cw = codes_bf16x2(t2, qp);
+          if (ZP) cw = sub_bf16x2(cw, zw[e]);
+          if (MODE == FUSED_FWD_PC) {
+            w[e] = cw;
+          } else {
+            w[e] = mul_bf16x2(cw, pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
+          }
+        }
+        // The W_hat buffer of this token slot was last read by the product of stage gg - NT.
+        const uint32_t ts = gg % NT;
+        ok = wait_bounded(bar(BAR_TEMPTY + ts), ((gg / NT) & 1u) ^ 1u, ctl, 14);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        const uint32_t wt = smem + OFF_TSLOTS + ts * TSLOT_BYTES + TS_W;
+        st_shared_v4(wt + swz_offset(row, 2 * c, 128), w[0], w[1], w[2], w[3]);
+        st_shared_v4(wt + swz_offset(row, 2 * c + 1, 128), w[4], w[5], w[6], w[7]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          report(BAR_WFULL + ts, pw);
+          mbar_arrive(bar(BAR_FEMPTY + fslot));
+        }
+      }
+      if (!ok) break;
+      // ------------------------------------------------------------ epilogue
+      float scale = 1.0f;
+      if (MODE == FUSED_FWD_PC) scale = args.s[row_g];
+      if (MODE != FUSED_DX && args.s_x != nullptr) scale *= *args.s_x;
+      ok = wait_spin_bounded(bar(BAR_ACCFULL), it & 1u, ctl, 15);
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      tc_fence_after();
+      const bool odd = lane & 1;
+#pragma unroll 1
+      for (int ch = 0; ch < EPI_COLS / 16; ++ch) {
+        float acc[16];
+        const int col = c * EPI_COLS + 16 * ch;   // accumulator column = token offset in the tile
+        tmem_ld16(tmem + lane_off + col, acc);
+        tmem_ld_wait();
+        const int tok0 = tb * BTP + col;
+        uint32_t mword = 0xffffffffu;
+        if (MODE == FUSED_DX && args.xmask != nullptr && tok0 < args.T)
+          mword = args.xmask[static_cast<int64_t>(row_g) * args.xmask_ld + tok0 / 32] >> (tok0 & 31);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) acc[e] = ((mword >> e) & 1u) ? acc[e] * scale : 0.0f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float mine = odd ? acc[2 * e] : acc[2 * e + 1];
+          const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
+          const int tt = tok0 + 2 * e + (odd ? 1 : 0);
+          const float lo = odd ? other : acc[2 * e];
+          const float hi = odd ? acc[2 * e + 1] : other;
+          if (tt < args.T) {
+            uint32_t* dst = reinterpret_cast<uint32_t*>(args.out + static_cast<int64_t>(tt) * args.out_ld +
+                                                        (row_g & ~1));
+            *dst = pack_rn_bf16x2(lo, hi);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) report(BAR_ACCEMPTY, pw);
+      g += nk;
+      ++it;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();   // neither CTA leaves while the other may still read its shared memory
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, TMEM_COLS);
+  }
+}
+
+template <int MODE, int FMT, bool ZP, bool UB, bool NL>
+cudaError_t launch_pair_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
+                            const FusedArgs& args, int npairs, cudaStream_t stream) {
+  constexpr uint32_t smem = PairRing<FMT>::SMEM_BYTES;
+  static bool configured[kMaxDevices] = {};
+  const void* fn = reinterpret_cast<const void*>(fused_pair_kernel<MODE, FMT, ZP, UB, NL>);
+  cudaError_t e = ensure_smem_attr(fn, static_cast<int>(smem), configured);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(2 * npairs), 1, 1);
+  cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // The persistent grid holds no more pairs than can be resident at once (an SM that has no
+  // partner in its GPC cannot host half of a pair), looked up once per device.
+  static int max_pairs[kMaxDevices] = {};
+  int dev = 0;
+  e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (max_pairs[dev] == 0) {
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, fused_pair_kernel<MODE, FMT, ZP, UB, NL>, &cfg);
+    if (e != cudaSuccess) return e;
+    if (n < 1) return cudaErrorInvalidConfiguration;
+    max_pairs[dev] = n;
+  }
+  if (npairs > max_pairs[dev]) {
+    npairs = max_pairs[dev];
+    cfg.gridDim = dim3(static_cast<unsigned>(2 * npairs), 1, 1);
+  }
+  e = cudaLaunchKernelEx(&cfg, fused_pair_kernel<MODE, FMT, ZP, UB, NL>, a, b, c, d, args);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+template <int MODE, int FMT>
+cudaError_t launch_pair_fmt(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
+                            const FusedArgs& args, int npairs, cudaStream_t stream) {
+  if (args.r16 == 0) {
+    if (FMT != FMT_Q8 || args.u_bf16) return cudaErrorInvalidValue;
+    return args.zero != nullptr ? launch_pair_one<MODE, FMT_Q8, true, false, true>(a, b, c, d, args, npairs, stream)
+                                : launch_pair_one<MODE, FMT_Q8, false, false, true>(a, b, c, d, args, npairs, stream);
+  }
+  if (args.u_bf16) {
+    if (FMT == FMT_F16 || args.zero != nullptr) return cudaErrorInvalidValue;
+    return launch_pair_one<MODE, FMT == FMT_F16 ? FMT_Q8 : FMT, false, true, false>(a, b, c, d, args, npairs, stream);
+  }
+  if (fmt_float(FMT)) {
+    if (args.zero != nullptr) return cudaErrorInvalidValue;
+    return launch_pair_one<MODE, FMT, false, false, false>(a, b, c, d, args, npairs, stream);
+  }
+  return args.zero != nullptr ? launch_pair_one<MODE, FMT, true, false, false>(a, b, c, d, args, npairs, stream)
+                              : launch_pair_one<MODE, FMT, false, false, false>(a, b, c, d, args, npairs, stream);
+}
+
+template <int MODE>
+cudaError_t launch_pair_mode(int fmt, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                             const CUtensorMap& d, const FusedArgs& args, int npairs, cudaStream_t stream) {
+  switch (fmt) {
+    case FMT_Q8: return launch_pair_fmt<MODE, FMT_Q8>(a, b, c, d, args, npairs, stream);
+    case FMT_I4:
+      if (MODE == FUSED_DX) return cudaErrorInvalidValue;
+      return launch_pair_fmt<MODE, MODE == FUSED_DX ? FMT_Q8 : FMT_I4>(a, b, c, d, args, npairs, stream);
+    case FMT_BF16: return launch_pair_fmt<MODE, FMT_BF16>(a, b, c, d, args, npairs, stream);
+    case FMT_F16: return launch_pair_fmt<MODE, FMT_F16>(a, b, c, d, args, npairs, stream);
+    case FMT_E4M3: return launch_pair_fmt<MODE, FMT_E4M3>(a, b, c, d, args, npairs, stream);
+    case FMT_E5M2: return launch_pair_fmt<MODE, FMT_E5M2>(a, b, c, d, args, npairs, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_fused_pair(int mode, int fmt, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
+                              const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int npairs,
+                              cudaStream_t stream) {
+  if (npairs < 1 || (args.kdim % 128) != 0 || args.kdim < 128 || (args.rows % 256) != 0 || args.sf_mn ||
+      args.num_rb != args.rows / 128)
+    return cudaErrorInvalidValue;
+  switch (mode) {
+    case FUSED_FWD_PC: return launch_pair_mode<FUSED_FWD_PC>(fmt, tm_tok, tm_phi, tm_rf, tm_sf, args, npairs, stream);
+    case FUSED_FWD_GROUP:
+      return launch_pair_mode<FUSED_FWD_GROUP>(fmt, tm_tok, tm_phi, tm_rf, tm_sf, args, npairs, stream);
+    case FUSED_DX: return launch_pair_mode<FUSED_DX>(fmt, tm_tok, tm_phi, tm_rf, tm_sf, args, npairs, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace lrqat

@@ -281,6 +281,25 @@ int dw_schedule_from_env() {
 }
 std::atomic<int> g_dw_schedule{dw_schedule_from_env()};
 
+// Kernel of the forward and dX GEMMs (lrqat_set_gemm_variant): 0 = the faster one measured for
+// the path (CTA pairs when the base holds the codes, ranks above 64; the one-SM kernel when the
+// low-rank tile is computed in the GEMM), 1 = the one-SM kernel (fused_gemm.cu) always, 2 = CTA
+// pairs (fused_pair.cu) always.  Pairs need a multiple of 256 produced rows; other shapes take
+// the one-SM kernel.  LRQAT_GEMM_VARIANT ("auto" / "single" / "pair") sets the start value once,
+// when the library is loaded.
+int gemm_variant_from_env() {
+  const char* v = std::getenv("LRQAT_GEMM_VARIANT");
+  if (v && std::strcmp(v, "single") == 0) return 1;
+  if (v && std::strcmp(v, "pair") == 0) return 2;
+  return 0;
+}
+std::atomic<int> g_gemm_variant{gemm_variant_from_env()};
+bool use_pair(int64_t rows, bool codes) {
+  const int v = g_gemm_variant.load(std::memory_order_relaxed);
+  return rows % 256 == 0 && (v == 2 || (v == 0 && codes));
+}
+constexpr int kPairTokens = 384;   // tokens per pair tile (two accumulators of 192)
+
 struct DwPlan {
   int nchunks, ni, nj, nsplit, tchunk, units;
   DwSched sched;
@@ -625,7 +644,9 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
   const bool cb = codes_base(L);
-  const bool direct = !cb && direct_factors(L, A, B);
+  const bool pair = use_pair(L.m, cb);
+  // the pair kernel reads K-major factor slices, so it takes B^T from the padded copy
+  const bool direct = !cb && !pair && direct_factors(L, A, B);
   if (cb) {
     // ranks above 64: the codes of every weight, once per call
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
@@ -651,7 +672,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     tok = ws.x_codes;
   }
   CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
-  LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 64, 224,
+  LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, tok, L.k, T, L.k * 2, 64, pair ? 96 : 224,
                       CU_TENSOR_MAP_SWIZZLE_128B, "X"));
   if (cb) {
     // the codes as an 8-bit base; the factor maps are not read
@@ -671,8 +692,8 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   } else {
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "A (padded)"));
-    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, sf_cols(r16), 64,
-                        sf_swizzle(r16), "B^T (padded)"));
+    LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, sf_cols(r16),
+                        pair ? 32 : 64, sf_swizzle(r16), "B^T (padded)"));
   }
   FusedArgs a{};
   a.rows = static_cast<int32_t>(L.m);
@@ -697,11 +718,18 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   a.out_ld = L.m;
   a.status = dev->status;
   a.timeout_ns = kWaitTimeoutNs;
-  const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
-  LRQAT_LAUNCH("fused_fwd", 1, stream,
-               launch_fused(L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC, cb ? LRQAT_PHI_QFIXED : L.phi_format,
-                            tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
-               "fused forward launch");
+  const int fmode = L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC;
+  const int ffmt = cb ? LRQAT_PHI_QFIXED : L.phi_format;
+  if (pair) {
+    const int64_t tiles = (L.m / 256) * ((T + kPairTokens - 1) / kPairTokens);
+    const int npairs = static_cast<int>(tiles < dev->sms / 2 ? tiles : dev->sms / 2);
+    LRQAT_LAUNCH("fused_fwd", 1, stream, launch_fused_pair(fmode, ffmt, tm_tok, tm_phi, tm_rf, tm_sf, a, npairs, stream),
+                 "fused forward launch (CTA pairs)");
+  } else {
+    const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
+    LRQAT_LAUNCH("fused_fwd", 1, stream, launch_fused(fmode, ffmt, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+                 "fused forward launch");
+  }
   return LRQAT_OK;
 }
 
@@ -811,8 +839,9 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
 
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
+    const bool pair = use_pair(L.k, cb);
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
-    LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 224,
+    LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, pair ? 96 : 224,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY"));
     if (phi_16bit(L) && !cb)
       LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT16, ws.phit, L.m, L.k, L.m * 2, 64, 128,
@@ -827,11 +856,11 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_TRY(encode_2d(&tm_rf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.bt_pad, 64, L.k, 128, 64, 128,
                         CU_TENSOR_MAP_SWIZZLE_128B, "B^T (padded)"));
     if (direct)
-      LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, sf_cols(r16), 64,
-                          sf_swizzle(r16), "A"));
+      LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, sf_cols(r16),
+                          pair ? 32 : 64, sf_swizzle(r16), "A"));
     else
-      LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16), 64,
-                          sf_swizzle(r16), "A (padded)"));
+      LRQAT_TRY(encode_2d(&tm_sf, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.a_pad, 64, L.m, 128, sf_cols(r16),
+                          pair ? 32 : 64, sf_swizzle(r16), "A (padded)"));
     }
     FusedArgs a{};
     a.rows = static_cast<int32_t>(L.k);
@@ -856,10 +885,18 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.out_ld = L.k;
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
-    const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
-    LRQAT_LAUNCH("fused_dx", 1, stream,
-                 launch_fused(FUSED_DX, cb ? LRQAT_PHI_QFIXED : fmt_t, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
-                 "fused dX launch");
+    const int dfmt = cb ? LRQAT_PHI_QFIXED : fmt_t;
+    if (pair) {
+      const int64_t tiles = (L.k / 256) * ((T + kPairTokens - 1) / kPairTokens);
+      const int npairs = static_cast<int>(tiles < dev->sms / 2 ? tiles : dev->sms / 2);
+      LRQAT_LAUNCH("fused_dx", 1, stream,
+                   launch_fused_pair(FUSED_DX, dfmt, tm_tok, tm_phi, tm_rf, tm_sf, a, npairs, stream),
+                   "fused dX launch (CTA pairs)");
+    } else {
+      const int grid = a.num_tiles < dev->sms ? a.num_tiles : dev->sms;
+      LRQAT_LAUNCH("fused_dx", 1, stream, launch_fused(FUSED_DX, dfmt, tm_tok, tm_phi, tm_rf, tm_sf, a, grid, stream),
+                   "fused dX launch");
+    }
   }
   // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
   {
@@ -1045,6 +1082,16 @@ int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const flo
   a.max_norm = opt->max_grad_norm;
   a.sqnorm = sqnorm;
   LRQAT_LAUNCH("adamw", 1, stream, launch_adamw(a, stream), "AdamW launch");
+  return LRQAT_OK;
+}
+
+int lrqat_get_gemm_variant(void) { return g_gemm_variant.load(std::memory_order_relaxed); }
+int lrqat_get_dw_schedule(void) { return g_dw_schedule.load(std::memory_order_relaxed); }
+
+int lrqat_set_gemm_variant(int variant) {
+  if (variant < 0 || variant > 2)
+    return fail(LRQAT_ERR_INVALID_ARG, "GEMM variant must be 0, 1 or 2 (got %d)", variant);
+  g_gemm_variant.store(variant, std::memory_order_relaxed);
   return LRQAT_OK;
 }
 

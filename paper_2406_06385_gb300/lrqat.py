@@ -96,6 +96,11 @@ def lib() -> ctypes.CDLL:
             fn = getattr(L, name)
             fn.argtypes = args
             fn.restype = ctypes.c_int
+        for name in ("lrqat_get_gemm_variant", "lrqat_get_dw_schedule"):
+            getattr(L, name).argtypes = []
+            getattr(L, name).restype = ctypes.c_int
+        L.lrqat_set_gemm_variant.argtypes = [ip]
+        L.lrqat_set_gemm_variant.restype = ctypes.c_int
         L.lrqat_set_dw_schedule.argtypes = [ip]
         L.lrqat_set_dw_schedule.restype = ctypes.c_int
         L.lrqat_trace_enable.argtypes = [ip]
@@ -221,6 +226,23 @@ DW_SCHEDULES = {"auto": 0, "split": 1, "tail": 2}
 def set_dw_schedule(schedule: str) -> None:
     """Process-wide schedule of the weight-gradient work: "auto", "split" or "tail"."""
     _check(lib().lrqat_set_dw_schedule(DW_SCHEDULES[schedule]))
+
+
+GEMM_VARIANTS = {"auto": 0, "single": 1, "pair": 2}
+
+
+def set_gemm_variant(variant: str) -> None:
+    """Process-wide kernel of the forward and dX GEMMs: "auto" (the faster one measured for the
+    path), "single" (one SM per tile) or "pair" (CTA pairs where the rows allow)."""
+    _check(lib().lrqat_set_gemm_variant(GEMM_VARIANTS[variant]))
+
+
+def gemm_variant() -> str:
+    return {v: k for k, v in GEMM_VARIANTS.items()}[lib().lrqat_get_gemm_variant()]
+
+
+def dw_schedule() -> str:
+    return {v: k for k, v in DW_SCHEDULES.items()}[lib().lrqat_get_dw_schedule()]
 
 
 def trace_enable(enable: bool = True) -> None:

@@ -15,7 +15,18 @@ def pytest_configure(config):
 @pytest.fixture
 def dw_schedule():
     """Forces the schedule of the weight-gradient work for one test ("split" or "tail")
-    and restores the per-call choice afterwards."""
+    and restores the previous setting afterwards."""
     from paper_2406_06385_gb300 import lrqat as LQ
+    before = LQ.dw_schedule()
     yield LQ.set_dw_schedule
-    LQ.set_dw_schedule("auto")
+    LQ.set_dw_schedule(before)
+
+
+@pytest.fixture
+def gemm_variant():
+    """Forces the kernel of the forward and dX GEMMs for one test ("pair" or "single") and
+    restores the previous setting afterwards."""
+    from paper_2406_06385_gb300 import lrqat as LQ
+    before = LQ.gemm_variant()
+    yield LQ.set_gemm_variant
+    LQ.set_gemm_variant(before)

@@ -401,3 +401,37 @@ def test_merge_large_ranks(cid, spec, shift):
     assert ((wz.cpu().numpy() != ref) & ~exempt).sum() == 0
     # the factors are drawn large enough (|A B| ~ 0.5 code steps or more) that the low-rank term moves codes
     assert (ref != O.merge(phi0, data.A, np.zeros_like(data.B), OL)).mean() > 0.01
+
+
+# The forward and dX GEMMs on CTA pairs (256 weight rows across two SMs) and on one SM: the
+# cases whose produced operand has a multiple of 256 rows (m for the forward, k for dX) run on
+# pairs when that variant is selected; both variants must match the oracle, give the same
+# integer codes, and agree with each other up to fp32 summation order.
+PAIR_CASES = [c for c in CASES if c[1].m % 256 == 0 or c[1].k % 256 == 0] + [
+    ("q44_pc_pair_tail", spec_of("pt", 512, 768, 32, a_std=0.2, b_std=0.2), 1111),
+    ("q44_g128_pair_r16", spec_of("pg", 768, 512, 16, group=128, a_std=0.2, b_std=0.2), 385),
+]
+
+
+@pytest.mark.parametrize("cid,spec,T", PAIR_CASES, ids=[c[0] for c in PAIR_CASES])
+def test_fwd_bwd_parity_gemm_variants(cid, spec, T, gemm_variant):
+    outs = {}
+    for variant in ("pair", "single"):
+        gemm_variant(variant)
+        got, ref, _ = _run(spec, T, seed=1, s_scale=1.05)
+        errs = {k: O.rel_fro(got[k], ref[k]) for k in got}
+        assert errs["Y"] <= TOL_ACT and errs["dX"] <= TOL_ACT, (variant, errs)
+        assert errs["dA"] <= TOL_GRAD and errs["dB"] <= TOL_GRAD and errs["ds"] <= TOL_GRAD, (variant, errs)
+        outs[variant] = got
+    for key in ("Y", "dX"):
+        assert O.rel_fro(outs["pair"][key], outs["single"][key]) <= 4e-3, key
+
+
+@pytest.mark.parametrize("cid,spec", [c for c in CODE_CASES if c[1].m % 256 == 0 and c[1].k % 256 == 0],
+                         ids=[c[0] for c in CODE_CASES if c[1].m % 256 == 0 and c[1].k % 256 == 0])
+def test_fused_codes_bit_exact_pair_gemm(cid, spec, gemm_variant):
+    """The integer codes the pair kernel's producers build, through the identity inputs of
+    test_fused_codes_bit_exact, with exact ties (B = 0) and with the low-rank term."""
+    gemm_variant("pair")
+    for zero_B in (False, True):
+        test_fused_codes_bit_exact(cid, spec, zero_B)
