@@ -312,9 +312,9 @@ int lrqat_set_dw_schedule(int schedule);
  * MMAs of 256 rows across the two SMs of a cluster, each SM holding half of the token
  * operand; 256 rows x 384 tokens per pair) wherever the produced weight operand has a
  * multiple of 256 rows (m for the forward, k for dX), the one-SM kernel otherwise;
- * 0 (the default) = pairs where the base holds the precomputed codes (ranks above 64) and
- * the one-SM kernel where the GEMM computes the low-rank tile itself, the faster of the two
- * measured for each.  All give the same codes; outputs agree up to fp32 summation order.
+ * 0 (the default) = the faster of the two measured for each GEMM: pairs for the forward,
+ * and for dX when the base holds the precomputed codes (ranks above 64); the one-SM kernel
+ * for dX when it computes the low-rank tile itself.  All give the same codes; outputs agree up to fp32 summation order.
  * Process-wide; the environment variable LRQAT_GEMM_VARIANT ("auto", "single" or "pair")
  * gives the start value, read once when the library is loaded.  Returns
  * LRQAT_ERR_INVALID_ARG for other values. */

@@ -18,9 +18,10 @@
 //   * factor ring (4 slots; 2 for 16-bit bases): the stored base of this CTA's rows (completion on its own
 //     barrier; only its own producers read it) and this CTA's half (32 rows) of the second
 //     factor's slice (completion on the leader's barrier: the low-rank MMA reads both halves);
-//   * the leader's MMA thread issues the low-rank tile L = RF SF^T (M = 256, N = 64) two
-//     stages ahead into one of two TMEM buffers, and the main product (M = 256, N = 192,
-//     8 MMAs per stage); every commit is multicast to both CTAs;
+//   * in the leader, one thread issues the low-rank tiles L = RF SF^T (M = 256, N = 64) into
+//     two TMEM buffers, up to two stages ahead of the producers, and another the main product
+//     (M = 256, N = 192, 8 MMAs per stage), so that neither waits behind the other's barriers;
+//     every commit is multicast to both CTAs;
 //   * sixteen producer warps per CTA build this CTA's W_hat tile exactly as the one-SM kernel
 //     does, and drain this CTA's 128 rows of the accumulators in the epilogue.
 // The leader waits for the peer's "W_hat written", "L read" and "accumulators drained" events;
@@ -182,16 +183,48 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   };
 
   if (warp == 0) {
-    // ------------------------------------------------- row factor (per tile)
+    // ------------------- row factor (per tile) and, in the leader, the low-rank MMAs
+    // A thread of its own issues the low-rank tiles, so that the main product never waits
+    // behind their barriers; each thread's commits track only its own MMAs.
     if (!NL && lane == 0) {
       prefetch_tensormap(&tm_rf);
-      uint32_t it = 0;
-      for (int tile = pair; tile < num_tiles; tile += npairs) {
+      const uint32_t idesc_l = make_idesc_bf16(256, BK, 0, 0);
+      const int lsteps = args.r16 / 16;
+      const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
+      // the K-major half slice: 32 rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to match)
+      const uint32_t sf_swz = args.sf_cols == 64 ? SWZ_128B : args.sf_cols == 32 ? SWZ_64B : SWZ_32B;
+      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + PR::FS_SF, 16, 16u * args.sf_cols, sf_swz);
+      constexpr uint32_t FSLOT_D = FSLOT_BYTES >> 4;
+      uint32_t it = 0, g = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
         const int rb2 = tile % num_rb2;
-        if (!wait_spin_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1)) break;
+        if (!(ok = wait_spin_bounded(bar(BAR_RFEMPTY), (it & 1u) ^ 1u, ctl, 1))) break;
         if (leader) mbar_arrive_expect_tx(bar(BAR_RFFULL), 2u * RF_BYTES);
         tma_load_2d_pair(smem + OFF_RF, &tm_rf, 0, rb2 * 2 * BM + static_cast<int>(rank) * BM, lbar(BAR_RFFULL));
+        if (leader) {
+          if (!(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
+          for (int kk = 0; kk < nk && ok; ++kk) {
+            // L(gg) into buffer gg % 2 once both factor halves landed and both CTAs read L(gg - 2)
+            const uint32_t gg = g + kk, s = gg % NF, b = gg & 1u;
+            if (!(ok = wait_spin_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4))) break;
+            if (!(ok = wait_spin_bounded(bar(BAR_LEMPTY + b), ((gg >> 1) & 1u) ^ 1u, ctl, 5))) break;
+            tc_fence_after();
+            const uint64_t sf = d_sf0 + s * FSLOT_D;
+            const uint32_t dl = tmem + COL_L + BK * b;
+            for (int ks = 0; ks < lsteps; ++ks) mma_bf16_pair(dl, d_rf + 2 * ks, sf + 2 * ks, idesc_l, ks > 0 ? 1u : 0u);
+            mma_commit_pair(bar(BAR_LFULL + b));
+          }
+          if (!ok) break;
+          mma_commit_pair(bar(BAR_RFEMPTY));   // last read of the row factor issued
+        }
+        g += nk;
         ++it;
+      }
+      if (leader && ok) {
+        // the peer's reports of the last two low-rank tiles land before the CTAs end
+        for (uint32_t gg = g >= 2 ? g - 2 : 0; ok && gg < g; ++gg)
+          ok = wait_spin_bounded(bar(BAR_LEMPTY + (gg & 1u)), (gg >> 1) & 1u, ctl, 11);
       }
     }
   } else if (warp >= FIRST_TMA_WARP && warp < FIRST_TMA_WARP + NT) {
@@ -247,48 +280,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer (the leader's)
+    // ------------------------------------ main-product MMA issuer (the leader's)
     if (leader && lane == 0) {
       const uint32_t idesc_main = make_idesc_bf16(256, BNP, 0, 0);
-      const uint32_t idesc_l = make_idesc_bf16(256, BK, 0, 0);
-      const int lsteps = NL ? 0 : args.r16 / 16;
-      constexpr uint32_t TSLOT_D = TSLOT_BYTES >> 4, FSLOT_D = FSLOT_BYTES >> 4, TOKB_D = TOK_BOX >> 4;
-      const uint64_t d_rf = make_sdesc(smem + OFF_RF, 16, 1024, SWZ_128B);
-      // the K-major half slice: 32 rows of sf_cols bf16 (32, 64 or 128 bytes, swizzled to match)
-      const uint32_t sf_swz = args.sf_cols == 64 ? SWZ_128B : args.sf_cols == 32 ? SWZ_64B : SWZ_32B;
-      const uint64_t d_sf0 = make_sdesc(smem + OFF_FSLOTS + PR::FS_SF, 16, 16u * args.sf_cols, sf_swz);
+      constexpr uint32_t TSLOT_D = TSLOT_BYTES >> 4, TOKB_D = TOK_BOX >> 4;
       const uint64_t d_w0 = make_sdesc(smem + OFF_TSLOTS + TS_W, 16, 1024, SWZ_128B);
       const uint64_t d_tok0 = make_sdesc(smem + OFF_TSLOTS, 16, 1024, SWZ_128B);
       uint32_t g = 0, it = 0;
       bool ok = true;
-      // L(gg) into buffer gg % 2 once both factor halves landed and both CTAs read L(gg - 2)
-      auto issue_lowrank = [&](uint32_t gg) -> bool {
-        const uint32_t s = gg % NF, b = gg & 1u;
-        if (!wait_spin_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4)) return false;
-        if (!wait_spin_bounded(bar(BAR_LEMPTY + b), ((gg >> 1) & 1u) ^ 1u, ctl, 5)) return false;
-        tc_fence_after();
-        const uint64_t sf = d_sf0 + s * FSLOT_D;
-        const uint32_t dl = tmem + COL_L + BK * b;
-        for (int ks = 0; ks < lsteps; ++ks) mma_bf16_pair(dl, d_rf + 2 * ks, sf + 2 * ks, idesc_l, ks > 0 ? 1u : 0u);
-        mma_commit_pair(bar(BAR_LFULL + b));
-        return true;
-      };
       for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
-        if (!NL) {
-          if (!(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
-          if (!(ok = issue_lowrank(g))) break;
-          if (!(ok = issue_lowrank(g + 1))) break;
-          if (nk == 2) mma_commit_pair(bar(BAR_RFEMPTY));
-        }
         if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
         tc_fence_after();
         for (int kk = 0; kk < nk; ++kk) {
           const uint32_t gg = g + kk;
           const uint32_t s = gg % NT, ph = (gg / NT) & 1u;
-          if (!NL && kk + 2 < nk) {
-            if (!(ok = issue_lowrank(gg + 2))) break;
-            if (kk + 3 == nk) mma_commit_pair(bar(BAR_RFEMPTY));   // last read of the row factor issued
-          }
           if (!(ok = wait_spin_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
           if (!(ok = wait_spin_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
           tc_fence_after();
@@ -310,13 +315,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         g += nk;
         ++it;
       }
-      if (ok) {
-        // the peer's last signals (the final drain, the reads of the last two low-rank
-        // tiles) land before the CTAs end
-        ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 10);
-        for (uint32_t gg = g >= 2 ? g - 2 : 0; ok && !NL && gg < g; ++gg)
-          ok = wait_spin_bounded(bar(BAR_LEMPTY + (gg & 1u)), (gg >> 1) & 1u, ctl, 11);
-      }
+      // the peer's last drain report lands before the CTAs end
+      if (ok) ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 10);
       mma_commit_pair_self(bar(BAR_DRAIN));
       drain_wait(bar(BAR_DRAIN), 0, args.timeout_ns);
     }

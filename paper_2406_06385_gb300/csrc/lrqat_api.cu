@@ -282,11 +282,12 @@ int dw_schedule_from_env() {
 std::atomic<int> g_dw_schedule{dw_schedule_from_env()};
 
 // Kernel of the forward and dX GEMMs (lrqat_set_gemm_variant): 0 = the faster one measured for
-// the path (CTA pairs when the base holds the codes, ranks above 64; the one-SM kernel when the
-// low-rank tile is computed in the GEMM), 1 = the one-SM kernel (fused_gemm.cu) always, 2 = CTA
-// pairs (fused_pair.cu) always.  Pairs need a multiple of 256 produced rows; other shapes take
-// the one-SM kernel.  LRQAT_GEMM_VARIANT ("auto" / "single" / "pair") sets the start value once,
-// when the library is loaded.
+// each GEMM (CTA pairs for the forward, and for dX when the base holds the codes of ranks above
+// 64; the one-SM kernel for dX when the GEMM computes the low-rank tile, whose producers' extra
+// scale multiply cannot keep up with the pair's shorter token tiles), 1 = the one-SM kernel
+// (fused_gemm.cu) always, 2 = CTA pairs (fused_pair.cu) always.  Pairs need a multiple of 256
+// produced rows; other shapes take the one-SM kernel.  LRQAT_GEMM_VARIANT ("auto" / "single" /
+// "pair") sets the start value once, when the library is loaded.
 int gemm_variant_from_env() {
   const char* v = std::getenv("LRQAT_GEMM_VARIANT");
   if (v && std::strcmp(v, "single") == 0) return 1;
@@ -294,9 +295,9 @@ int gemm_variant_from_env() {
   return 0;
 }
 std::atomic<int> g_gemm_variant{gemm_variant_from_env()};
-bool use_pair(int64_t rows, bool codes) {
+bool use_pair(int64_t rows, bool codes, bool dx) {
   const int v = g_gemm_variant.load(std::memory_order_relaxed);
-  return rows % 256 == 0 && (v == 2 || (v == 0 && codes));
+  return rows % 256 == 0 && (v == 2 || (v == 0 && (codes || !dx)));
 }
 constexpr int kPairTokens = 384;   // tokens per pair tile (two accumulators of 192)
 
@@ -644,7 +645,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
   const bool cb = codes_base(L);
-  const bool pair = use_pair(L.m, cb);
+  const bool pair = use_pair(L.m, cb, false);
   // the pair kernel reads K-major factor slices, so it takes B^T from the padded copy
   const bool direct = !cb && !pair && direct_factors(L, A, B);
   if (cb) {
@@ -839,7 +840,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
 
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
-    const bool pair = use_pair(L.k, cb);
+    const bool pair = use_pair(L.k, cb, true);
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
     LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, pair ? 96 : 224,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY"));
