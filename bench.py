@@ -36,7 +36,9 @@ METRIC = "LR-QAT linear fwd+bwd tokens/s and TFLOP/s, fraction of GB300 bf16 den
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 GEMM_KERNELS = ("fused_fwd", "fused_dx", "fused_dw")
-KERNEL_SOURCES = {"fused_fwd": "fused_gemm.cu", "fused_dx": "fused_gemm.cu", "fused_dw": "dw.cu"}
+# the sources whose kernels a traced name can refer to (the forward and dX run on CTA pairs or on one SM)
+KERNEL_SOURCES = {"fused_fwd": ("fused_gemm.cu", "fused_pair.cu"), "fused_dx": ("fused_gemm.cu", "fused_pair.cu"),
+                  "fused_dw": ("dw.cu",)}
 
 
 # --------------------------------------------------------------------------- helpers
@@ -60,7 +62,7 @@ def kernel_source_hash(kernel: str) -> str:
     """sha256 of the sources that define a kernel (its .cu file and the shared device headers)."""
     csrc = os.path.join(ROOT, "paper_2406_06385_gb300", "csrc")
     h = hashlib.sha256()
-    for name in (KERNEL_SOURCES[kernel], "ptx.cuh", "quant.cuh", "kernels.h"):
+    for name in KERNEL_SOURCES[kernel] + ("ptx.cuh", "quant.cuh", "kernels.h"):
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]

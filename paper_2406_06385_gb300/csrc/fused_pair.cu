@@ -42,21 +42,22 @@ namespace {
 
 constexpr int BM = 128;                          // weight rows per CTA (256 per pair)
 constexpr int BK = 64;
-constexpr int BNP = 192;                         // tokens per accumulator (N of the pair MMA)
+constexpr int BNP = 224;                         // tokens per accumulator (N of the pair MMA)
 constexpr int BNH = BNP / 2;                     // tokens per accumulator held by one CTA
 constexpr int NACC = 2;
-constexpr int BTP = BNP * NACC;                  // 384 tokens per pair tile
-constexpr int NT = 4;                            // token ring slots
+constexpr int BTP = BNP * NACC;                  // 448 tokens per pair tile
+constexpr int NT = 3;                            // token ring slots
+constexpr int NLB = 1;                           // low-rank TMEM buffers
 constexpr int NF_MAX = 4;                        // factor ring slots (2 for 16-bit bases)
 constexpr int NUM_PROD_WARPS = 16;
 constexpr int FIRST_TMA_WARP = 2 + NUM_PROD_WARPS;
 constexpr int NUM_TMA_WARPS = NT + 1;
 constexpr int NUM_THREADS = 32 * (FIRST_TMA_WARP + NUM_TMA_WARPS);
-constexpr int EPI_COLS = NACC * BNP / 4;         // accumulator columns drained per warp (96)
+constexpr int EPI_COLS = NACC * BNP / 4;         // accumulator columns drained per warp (112)
 constexpr uint32_t SIG_TX = 16u * NUM_PROD_WARPS;   // bytes of the peer's per-warp signals
 
 constexpr uint32_t RF_BYTES = 128 * 128;         // 128 rows x 64 rank columns (bf16)
-constexpr uint32_t TOK_BOX = BNH * 128;          // 96 tokens x 64 bf16
+constexpr uint32_t TOK_BOX = BNH * 128;          // 112 tokens x 64 bf16
 constexpr uint32_t TOK_BYTES = NACC * TOK_BOX;
 constexpr uint32_t W_BYTES = 128 * 128;          // 128 rows x 64 bf16
 constexpr uint32_t SFH_BYTES = 32 * 128;         // 32 slice rows x up to 64 rank columns (bf16)
@@ -82,8 +83,8 @@ static_assert(TSLOT_BYTES % 1024 == 0 && TOK_BOX % 1024 == 0 && TS_W % 1024 == 0
 static_assert(EPI_COLS % 16 == 0, "epilogue drains 16-column chunks");
 
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t COL_L = NACC * BNP;           // two 64-column low-rank buffers at 384 and 448
-static_assert(COL_L + 2 * BK <= TMEM_COLS, "TMEM budget");
+constexpr uint32_t COL_L = NACC * BNP;           // the 64-column low-rank buffer(s) after the accumulators
+static_assert(COL_L + NLB * BK <= TMEM_COLS, "TMEM budget");
 
 constexpr int BAR_TFULL = 0;                     // leader: both token halves of the slot landed
 constexpr int BAR_TEMPTY = BAR_TFULL + NT;       // both: main product of the slot finished
@@ -93,8 +94,8 @@ constexpr int BAR_PFULL = BAR_WFULL + NT;        // both: this CTA's base tile l
 constexpr int BAR_FFULL = BAR_PFULL + NF_MAX;    // leader: both factor-slice halves landed
 constexpr int BAR_FEMPTY = BAR_FFULL + NF_MAX;   // both: slot read by this CTA's producers (after L)
 constexpr int BAR_LFULL = BAR_FEMPTY + NF_MAX;   // both: low-rank tile of the buffer computed
-constexpr int BAR_LEMPTY = BAR_LFULL + 2;        // leader: both CTAs read the buffer
-constexpr int BAR_RFFULL = BAR_LEMPTY + 2;       // leader: both row-factor halves landed
+constexpr int BAR_LEMPTY = BAR_LFULL + NLB;      // leader: both CTAs read the buffer
+constexpr int BAR_RFFULL = BAR_LEMPTY + NLB;     // leader: both row-factor halves landed
 constexpr int BAR_RFEMPTY = BAR_RFFULL + 1;      // both: last low-rank MMA of the tile finished
 constexpr int BAR_ACCFULL = BAR_RFEMPTY + 1;     // both: accumulators of the tile complete
 constexpr int BAR_ACCEMPTY = BAR_ACCFULL + 1;    // leader: both CTAs drained them
@@ -148,7 +149,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // low-rank tile, so the low-rank MMA that read the slot's factor half has completed
       mbar_init(bar(BAR_FEMPTY + s), NUM_PROD_WARPS);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < NLB; ++b) {
       mbar_init(bar(BAR_LFULL + b), 1);
       mbar_init(bar(BAR_LEMPTY + b), NUM_PROD_WARPS);
     }
@@ -205,10 +206,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if (leader) {
           if (!(ok = wait_spin_bounded(bar(BAR_RFFULL), it & 1u, ctl, 6))) break;
           for (int kk = 0; kk < nk && ok; ++kk) {
-            // L(gg) into buffer gg % 2 once both factor halves landed and both CTAs read L(gg - 2)
-            const uint32_t gg = g + kk, s = gg % NF, b = gg & 1u;
+            // L(gg) into buffer gg % NLB once both factor halves landed and both CTAs read L(gg - NLB)
+            const uint32_t gg = g + kk, s = gg % NF, b = gg % NLB;
             if (!(ok = wait_spin_bounded(bar(BAR_FFULL + s), (gg / NF) & 1u, ctl, 4))) break;
-            if (!(ok = wait_spin_bounded(bar(BAR_LEMPTY + b), ((gg >> 1) & 1u) ^ 1u, ctl, 5))) break;
+            if (!(ok = wait_spin_bounded(bar(BAR_LEMPTY + b), ((gg / NLB) & 1u) ^ 1u, ctl, 5))) break;
             tc_fence_after();
             const uint64_t sf = d_sf0 + s * FSLOT_D;
             const uint32_t dl = tmem + COL_L + BK * b;
@@ -222,9 +223,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         ++it;
       }
       if (leader && ok) {
-        // the peer's reports of the last two low-rank tiles land before the CTAs end
-        for (uint32_t gg = g >= 2 ? g - 2 : 0; ok && gg < g; ++gg)
-          ok = wait_spin_bounded(bar(BAR_LEMPTY + (gg & 1u)), (gg >> 1) & 1u, ctl, 11);
+        // the peer's reports of the last low-rank tiles land before the CTAs end
+        for (uint32_t gg = g >= NLB ? g - NLB : 0; ok && gg < g; ++gg)
+          ok = wait_spin_bounded(bar(BAR_LEMPTY + gg % NLB), (gg / NLB) & 1u, ctl, 11);
       }
     }
   } else if (warp >= FIRST_TMA_WARP && warp < FIRST_TMA_WARP + NT) {
@@ -413,8 +414,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         decode16<FMT>(raw, v);
         float Lv[16];
         if (!NL) {
-          const uint32_t lb = gg & 1u;
-          ok = wait_bounded(bar(BAR_LFULL + lb), (gg >> 1) & 1u, ctl, 13);
+          const uint32_t lb = gg % NLB;
+          ok = wait_bounded(bar(BAR_LFULL + lb), (gg / NLB) & 1u, ctl, 13);
           if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
           tc_fence_after();
           tmem_ld16(tmem + lane_off + COL_L + BK * lb + 16 * c, Lv);

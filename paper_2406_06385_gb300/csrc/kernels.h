@@ -165,8 +165,8 @@ struct FusedArgs {
   int32_t sf_mn;
 };
 int fused_smem_bytes(int fmt);
-// The same GEMM on CTA pairs (fused_pair.cu): 256-row x 384-token tiles, npairs clusters of 2.
-// Needs rows % 256 == 0 and K-major factor slices (sf_mn == 0); tm_tok boxes of 96 tokens x
+// The same GEMM on CTA pairs (fused_pair.cu): 256-row x 448-token tiles, npairs clusters of 2.
+// Needs rows % 256 == 0 and K-major factor slices (sf_mn == 0); tm_tok boxes of 112 tokens x
 // 64, tm_sf boxes of 32 slice rows x sf_cols; tm_phi and tm_rf as for launch_fused.
 cudaError_t launch_fused_pair(int mode, int fmt, const CUtensorMap& tm_tok, const CUtensorMap& tm_phi,
                               const CUtensorMap& tm_rf, const CUtensorMap& tm_sf, const FusedArgs& args, int npairs,

@@ -228,12 +228,12 @@ def set_dw_schedule(schedule: str) -> None:
     _check(lib().lrqat_set_dw_schedule(DW_SCHEDULES[schedule]))
 
 
-GEMM_VARIANTS = {"auto": 0, "single": 1, "pair": 2}
+GEMM_VARIANTS = {"pair": 0, "single": 1}
 
 
 def set_gemm_variant(variant: str) -> None:
-    """Process-wide kernel of the forward and dX GEMMs: "auto" (the faster one measured for the
-    path), "single" (one SM per tile) or "pair" (CTA pairs where the rows allow)."""
+    """Process-wide kernel of the forward and dX GEMMs: "pair" (CTA pairs where the rows
+    allow, the default) or "single" (one SM per tile)."""
     _check(lib().lrqat_set_gemm_variant(GEMM_VARIANTS[variant]))
 
 
