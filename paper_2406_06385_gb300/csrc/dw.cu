@@ -112,6 +112,25 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   return x;
 }
 
+// Whole tile number u (u < full_tiles, in processing order) of the tail schedule.  The whole
+// tiles are the natural indices ib + ni jt < full_tiles; they are taken in groups of
+// kColGroup column tiles with the column tile varying fastest, so that a wave of CTAs covers
+// about (CTAs / kColGroup) row blocks x kColGroup column tiles: a rectangle of dY and X
+// columns rather than every row block (all of dY) per wave.  The part of the prefix that does
+// not fill a whole group keeps the natural order.
+constexpr int64_t kColGroup = 8;
+__device__ __forceinline__ void dw_whole_tile(int64_t u, int ni, int64_t full_tiles, int& ib, int& jt) {
+  const int64_t grouped = full_tiles / ni / kColGroup * kColGroup * ni;
+  if (u < grouped) {
+    const int64_t grp = u / (kColGroup * ni), r = u % (kColGroup * ni);
+    jt = static_cast<int>(grp * kColGroup + r % kColGroup);
+    ib = static_cast<int>(r / kColGroup);
+  } else {
+    ib = static_cast<int>(u % ni);
+    jt = static_cast<int>(u / ni);
+  }
+}
+
 // This CTA's units (equal token splits, taken round robin), or (tail schedule) its whole
 // tiles of the full waves followed by its one part of a tail tile (slot = part index).
 struct WorkIter {
@@ -131,8 +150,7 @@ __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, Unit& x
     return true;
   }
   if (it.u < a.sched.full_tiles) {
-    x.ib = static_cast<int>(it.u % a.ni);
-    x.jt = static_cast<int>(it.u / a.ni);
+    dw_whole_tile(it.u, a.ni, a.sched.full_tiles, x.ib, x.jt);
     x.sp = 0;
     x.t0 = 0;
     x.nsteps = static_cast<int>(a.sched.tsteps);
