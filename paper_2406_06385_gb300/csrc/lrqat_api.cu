@@ -282,15 +282,22 @@ int dw_schedule_from_env() {
 std::atomic<int> g_dw_schedule{dw_schedule_from_env()};
 
 // Kernel of the forward and dX GEMMs (lrqat_set_gemm_variant): 0 = CTA pairs (fused_pair.cu)
-// wherever the produced weight operand has a multiple of 256 rows, the one-SM kernel
-// (fused_gemm.cu) otherwise; 1 = the one-SM kernel always.  LRQAT_GEMM_VARIANT ("pair" /
-// "single") sets the start value once, when the library is loaded.
+// wherever they were measured faster: every GEMM whose produced weight operand has a multiple of
+// 256 rows, except dX with group-wise scales (its producers load a scale per element, which the
+// pair's per-SM share of the stage cannot absorb); 1 = the one-SM kernel (fused_gemm.cu) always;
+// 2 = pairs wherever the rows allow.  LRQAT_GEMM_VARIANT ("auto" / "single" / "pair") sets the
+// start value once, when the library is loaded.
 int gemm_variant_from_env() {
   const char* v = std::getenv("LRQAT_GEMM_VARIANT");
-  return v && std::strcmp(v, "single") == 0 ? 1 : 0;
+  if (v && std::strcmp(v, "single") == 0) return 1;
+  if (v && std::strcmp(v, "pair") == 0) return 2;
+  return 0;
 }
 std::atomic<int> g_gemm_variant{gemm_variant_from_env()};
-bool use_pair(int64_t rows) { return rows % 256 == 0 && g_gemm_variant.load(std::memory_order_relaxed) == 0; }
+bool use_pair(int64_t rows, bool group_dx) {
+  const int v = g_gemm_variant.load(std::memory_order_relaxed);
+  return rows % 256 == 0 && (v == 2 || (v == 0 && !group_dx));
+}
 constexpr int kPairTokens = 448;   // tokens per pair tile (two accumulators of 224)
 
 struct DwPlan {
@@ -637,7 +644,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   fwd_ws_layout(L, T, workspace, &ws);
   const int r16 = round16(L.r);
   const bool cb = codes_base(L);
-  const bool pair = use_pair(L.m);
+  const bool pair = use_pair(L.m, false);
   // the pair kernel reads K-major factor slices, so it takes B^T from the padded copy
   const bool direct = !cb && !pair && direct_factors(L, A, B);
   if (cb) {
@@ -832,7 +839,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
 
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
-    const bool pair = use_pair(L.k);
+    const bool pair = use_pair(L.k, L.group_size != 0);
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
     LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, pair ? 112 : 224,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY"));
@@ -1082,7 +1089,8 @@ int lrqat_get_gemm_variant(void) { return g_gemm_variant.load(std::memory_order_
 int lrqat_get_dw_schedule(void) { return g_dw_schedule.load(std::memory_order_relaxed); }
 
 int lrqat_set_gemm_variant(int variant) {
-  if (variant < 0 || variant > 1) return fail(LRQAT_ERR_INVALID_ARG, "GEMM variant must be 0 or 1 (got %d)", variant);
+  if (variant < 0 || variant > 2)
+    return fail(LRQAT_ERR_INVALID_ARG, "GEMM variant must be 0, 1 or 2 (got %d)", variant);
   g_gemm_variant.store(variant, std::memory_order_relaxed);
   return LRQAT_OK;
 }

@@ -228,12 +228,13 @@ def set_dw_schedule(schedule: str) -> None:
     _check(lib().lrqat_set_dw_schedule(DW_SCHEDULES[schedule]))
 
 
-GEMM_VARIANTS = {"pair": 0, "single": 1}
+GEMM_VARIANTS = {"auto": 0, "single": 1, "pair": 2}
 
 
 def set_gemm_variant(variant: str) -> None:
-    """Process-wide kernel of the forward and dX GEMMs: "pair" (CTA pairs where the rows
-    allow, the default) or "single" (one SM per tile)."""
+    """Process-wide kernel of the forward and dX GEMMs: "auto" (CTA pairs where they were
+    measured faster, the default), "single" (one SM per tile) or "pair" (CTA pairs wherever
+    the rows allow)."""
     _check(lib().lrqat_set_gemm_variant(GEMM_VARIANTS[variant]))
 
 
