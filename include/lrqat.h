@@ -160,8 +160,9 @@ int lrqat_act_quant(const lrqat_layer* layer, int64_t T, const uint16_t* X, cons
                     uint32_t* mask, lrqat_stream_t stream);
 
 /* Bytes of workspace lrqat_linear_fwd needs for T tokens (padded adapter
- * copies; int8 activation codes when act_bits == 8; for ranks above 64 also
- * the m x k int8 codes of the weights). */
+ * copies; int8 activation codes when act_bits == 8; the m x k int8 codes of the
+ * weights for the codes path of lrqat_set_lowrank_path).  The size covers every
+ * setting of lrqat_set_lowrank_path. */
 size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
 
 /* Forward of the LR-QAT layer (Eq. 8 inside y = W_hat x):
@@ -184,8 +185,10 @@ int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, con
  * device and stall other work.
  *   - The array holds LRQAT_FWD_NOALLOC_SCRATCH_BYTES bytes; every device that
  *     loads the library keeps it until the process exits.  A layer/T whose
- *     scratch (lrqat_fwd_workspace_bytes) exceeds it is rejected with
- *     LRQAT_ERR_WORKSPACE (in practice: act_bits = 8 with large T * k).
+ *     scratch exceeds it is rejected with LRQAT_ERR_WORKSPACE (in practice:
+ *     act_bits = 8 with large T * k, or a rank above 64 with a large m * k).
+ *     For ranks up to 64 this forward always computes the low-rank tile inside
+ *     the GEMM (lrqat_set_lowrank_path 1), so its scratch holds no weight codes.
  *   - The first call on a device looks the array's device address up (with
  *     that device current); make that first call before any stream capture.
  *   - All calls share the one array: calls that overlap on the GPU (different
@@ -197,7 +200,8 @@ int lrqat_linear_fwd_noalloc(const lrqat_layer* layer, int64_t T, const uint16_t
                              const float* s, const uint16_t* A, const uint16_t* B, const float* s_x,
                              uint16_t* Y, lrqat_stream_t stream);
 
-/* Bytes of workspace lrqat_linear_bwd needs for T tokens. */
+/* Bytes of workspace lrqat_linear_bwd needs for T tokens (covers every setting of
+ * lrqat_set_lowrank_path). */
 size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T);
 
 /* Backward of the LR-QAT layer for the upstream gradient dY, with W_hat
@@ -318,9 +322,26 @@ int lrqat_set_dw_schedule(int schedule);
  * "single" or "pair") gives the start value, read once when the library is loaded.
  * Returns LRQAT_ERR_INVALID_ARG for other values. */
 int lrqat_set_gemm_variant(int variant);
-/* The current settings of lrqat_set_gemm_variant and lrqat_set_dw_schedule. */
+
+/* Tuning (no counterpart in the paper): where the forward and dX GEMMs take the low-rank
+ * term (alpha/r) A B of Eq. 8 from.  1 = "tile": each GEMM stage computes the 64-column
+ * low-rank tile of its weight rows on the tensor cores next to the main product (ranks up
+ * to 64); 2 = "codes": one tensor-core pass per call writes round(u) of every weight as
+ * int8 (saturated to [-128, 127]) into the workspace and the GEMMs read those codes as
+ * their base, with no low-rank work in the stage; 0 (the default) = codes from 3072 tokens
+ * on, the tile below (the pass costs two bytes of HBM traffic per weight, the tile a low-rank
+ * MMA chain per stage).  Ranks above 64 always take the codes pass.  dW is unaffected: it
+ * computes its own low-rank tile for ranks up to 64.  All settings give the same codes up to
+ * fp32 summation order of A B.  Process-wide; the environment variable LRQAT_LOWRANK_PATH
+ * ("auto", "tile" or "codes") gives the start value, read once when the library is loaded.
+ * Returns LRQAT_ERR_INVALID_ARG for other values. */
+int lrqat_set_lowrank_path(int path);
+
+/* The current settings of lrqat_set_gemm_variant, lrqat_set_dw_schedule and
+ * lrqat_set_lowrank_path. */
 int lrqat_get_gemm_variant(void);
 int lrqat_get_dw_schedule(void);
+int lrqat_get_lowrank_path(void);
 
 /* Synchronizes `stream`, then reads and clears the device status word of the
  * current device.  Returns LRQAT_OK, LRQAT_ERR_TIMEOUT (a kernel's bounded

@@ -121,12 +121,33 @@ bool direct_factors(const lrqat_layer& L, const void* A, const void* B) {
 
 int frac_bits(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_QFIXED ? 8 - L.bits : 0; }
 
-// Ranks above 64: one tensor-core pass per call writes the unclipped codes round(u) of every
-// weight (int8, saturated) into the workspace, and the three GEMMs read them as their base
-// with the low-rank term switched off (the factor slices of a rank above 64 do not fit next
-// to the GEMMs' token ring, and recomputing A B per 448-token tile would cost r/448 of the
-// GEMM's own tensor work).
-bool codes_base(const lrqat_layer& L) { return L.r > 64; }
+// Where the forward and dX GEMMs take the low-rank term from (lrqat_set_lowrank_path):
+// 1 = the tile that each GEMM stage computes next to the main product (ranks up to 64);
+// 2 = the codes pass: one tensor-core pass per call writes the unclipped codes round(u) of every
+// weight (int8, saturated) into the workspace, and the GEMMs read them as their base with the
+// low-rank term switched off.  In the pair GEMM the in-stage tile is a chain of small MMAs
+// whose TMEM buffer holds one stage, so it paces the stage (measured on a 4096 x 4096 layer at
+// T = 8192: forward 218 -> 191 us, dX 254 -> 210 us with the codes, for a pass of 18 us), while
+// the pass moves ~2 bytes per weight through HBM whatever T is.  Measured fwd + bwd per call,
+// tile against codes: 4096 x 4096 at T = 2048 353 / 355 us, at T = 4096 511 / 500 us;
+// 5120 x 13824 at T = 2048 1017 / 1044 us, at T = 4096 1657 / 1625 us.  So 0 (auto) takes the
+// codes from kCodesMinTokens tokens on.  Ranks above 64 always take the codes: their factor slices do not
+// fit next to the GEMMs' token ring, and recomputing A B per 448-token tile would cost r/448 of
+// the GEMM's own tensor work.  The same holds for dW, which otherwise computes its own tile.
+int lowrank_path_from_env() {
+  const char* v = std::getenv("LRQAT_LOWRANK_PATH");
+  if (v && std::strcmp(v, "tile") == 0) return 1;
+  if (v && std::strcmp(v, "codes") == 0) return 2;
+  return 0;
+}
+std::atomic<int> g_lowrank_path{lowrank_path_from_env()};
+constexpr int64_t kCodesMinTokens = 3072;
+bool codes_dw(const lrqat_layer& L) { return L.r > 64; }
+bool codes_gemm(const lrqat_layer& L, int64_t T) {
+  if (L.r > 64) return true;
+  const int v = g_lowrank_path.load(std::memory_order_relaxed);
+  return v == 2 || (v == 0 && T >= kCodesMinTokens);
+}
 bool phi_16bit(const lrqat_layer& L) { return L.phi_format == LRQAT_PHI_BF16 || L.phi_format == LRQAT_PHI_FP16; }
 int round16(int r) { return (r + 15) / 16 * 16; }
 
@@ -307,7 +328,7 @@ struct DwPlan {
 
 DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
   DwPlan p;
-  p.nchunks = (L.k % 256 == 0 && !codes_base(L)) ? 2 : 1;
+  p.nchunks = (L.k % 256 == 0 && !codes_dw(L)) ? 2 : 1;
   p.ni = static_cast<int>(L.m / 128);
   p.nj = static_cast<int>(L.k / (128 * p.nchunks));
   const int tiles = p.ni * p.nj;
@@ -365,22 +386,24 @@ struct FwdWs {
   uint16_t* a_pad;
   uint16_t* bt_pad;
   uint16_t* x_codes;   // int8 codes (per tensor) or X_hat (per token), bf16
-  uint16_t* at;        // ranks above 64: A^T [r16, m] and B [r16, k] zero-padded, codes [m, k]
+  uint16_t* at;        // codes path: A^T [r16, m] and B [r16, k] zero-padded, codes [m, k]
   uint16_t* b_pad;
   int8_t* codes;
 };
 
-size_t fwd_ws_layout(const lrqat_layer& L, int64_t T, void* base, FwdWs* ws) {
+// with_codes: carve the buffers of the codes path too (ranks above 64 always have them).
+size_t fwd_ws_layout(const lrqat_layer& L, int64_t T, bool with_codes, void* base, FwdWs* ws) {
   Carver c(base);
   FwdWs w{};
-  if (codes_base(L)) {
+  if (L.r <= 64) {
+    w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
+    w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
+  }
+  if (with_codes || L.r > 64) {
     const size_t r16 = static_cast<size_t>(round16(L.r));
     w.at = static_cast<uint16_t*>(c.take(r16 * L.m * 2));
     w.b_pad = static_cast<uint16_t*>(c.take(r16 * L.k * 2));
     w.codes = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
-  } else {
-    w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
-    w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
   }
   if (L.act_bits == 8) w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
   if (ws) *ws = w;
@@ -399,22 +422,23 @@ struct BwdWs {
   float* dB_part;
   float* ds_part;
   int32_t* tile_segs;
-  int8_t* codes;       // ranks above 64: the unclipped codes [m, k] (phit then holds their transpose)
+  int8_t* codes;       // codes path: the unclipped codes [m, k] (phit then holds their transpose)
 };
 
 size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* base, BwdWs* ws) {
   Carver c(base);
   BwdWs w{};
   const int r16 = round16(L.r);
-  if (codes_base(L)) {
-    w.codes = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
-  } else {
+  // the buffers of both low-rank paths (lrqat_set_lowrank_path), so the size is the same for every setting
+  w.codes = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
+  if (L.r <= 64) {
     w.a_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.m) * 64 * 2));
     w.bt_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(L.k) * 64 * 2));
   }
   w.at = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.m * 2));
   w.b_pad = static_cast<uint16_t*>(c.take(static_cast<size_t>(r16) * L.k * 2));
-  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k * (phi_16bit(L) && !codes_base(L) ? 2 : 1)));
+  // the transposed base of the dX GEMM: 16-bit for a 16-bit base on the tile path, else int8
+  w.phit = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k * (phi_16bit(L) && L.r <= 64 ? 2 : 1)));
   if (L.act_bits == 8) {
     w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
     w.xmask = static_cast<uint32_t*>(c.take(static_cast<size_t>(L.k) * ((T + 31) / 32) * 4));
@@ -525,6 +549,10 @@ extern "C" {
 
 const char* lrqat_last_error(void) { return t_last_error.c_str(); }
 
+static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* X, bool quantized, const void* Phi0,
+                           const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y,
+                           void* workspace, size_t workspace_bytes, bool allow_codes, lrqat_stream_t stream);
+
 // The forward of lrqat_linear_fwd with its scratch taken from the fixed array
 // above instead of a caller workspace.  The first call on a device performs the
 // address look-up.  Calls share the array, so calls that overlap on the GPU
@@ -537,7 +565,8 @@ int lrqat_linear_fwd_noalloc(const lrqat_layer* layer, int64_t T, const uint16_t
   LRQAT_TRY(validate_layer(layer));
   if (T < 1) return fail(LRQAT_ERR_INVALID_ARG, "T must be >= 1 (T=%lld)", (long long)T);
   if (T > (int64_t)1 << 30) return fail(LRQAT_ERR_UNSUPPORTED, "T too large");
-  const size_t need = fwd_ws_layout(*layer, T, nullptr, nullptr);
+  // ranks up to 64 take the in-GEMM low-rank tile here: the codes of m x k weights would not fit
+  const size_t need = fwd_ws_layout(*layer, T, false, nullptr, nullptr);
   if (need > LRQAT_FWD_NOALLOC_SCRATCH_BYTES)
     return fail(LRQAT_ERR_WORKSPACE,
                 "lrqat_linear_fwd_noalloc: this layer and T need %zu bytes of scratch but the fixed scratch holds "
@@ -545,7 +574,8 @@ int lrqat_linear_fwd_noalloc(const lrqat_layer* layer, int64_t T, const uint16_t
                 need, (size_t)LRQAT_FWD_NOALLOC_SCRATCH_BYTES);
   void* scratch = nullptr;
   LRQAT_TRY(noalloc_scratch(&scratch));
-  return lrqat_linear_fwd(layer, T, X, Phi0, s, A, B, s_x, Y, scratch, LRQAT_FWD_NOALLOC_SCRATCH_BYTES, stream);
+  return linear_fwd_impl(layer, T, X, false, Phi0, s, A, B, s_x, Y, scratch, LRQAT_FWD_NOALLOC_SCRATCH_BYTES, false,
+                         stream);
 }
 
 int lrqat_range_minmax(const lrqat_layer* layer, const float* W0, float* s0, lrqat_stream_t stream) {
@@ -610,14 +640,15 @@ int lrqat_downcast(const lrqat_layer* layer, const float* W0, const float* s0, v
 
 size_t lrqat_fwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
   if (validate_layer(layer) != LRQAT_OK || T < 1) return 0;
-  return fwd_ws_layout(*layer, T, nullptr, nullptr);
+  return fwd_ws_layout(*layer, T, true, nullptr, nullptr);
 }
 
 // quantized: X is already the activation quantizer's output for this layer (per tensor: the
-// codes; per token: X_hat), so no quantizer runs.
+// codes; per token: X_hat), so no quantizer runs.  allow_codes: the workspace has the buffers
+// of the codes path (false for the allocation-free forward, whose scratch is sized without them).
 static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* X, bool quantized, const void* Phi0,
                            const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y,
-                           void* workspace, size_t workspace_bytes, lrqat_stream_t stream) {
+                           void* workspace, size_t workspace_bytes, bool allow_codes, lrqat_stream_t stream) {
   LRQAT_TRY(validate_layer(layer));
   const lrqat_layer& L = *layer;
   if (quantized && L.act_bits != 8)
@@ -632,7 +663,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   LRQAT_CHECK_PTR(Y, "Y");
   if (L.act_bits == 8 && !L.act_per_token && !s_x)
     return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8 (per-tensor scale)");
-  const size_t need = fwd_ws_layout(L, T, nullptr, nullptr);
+  const size_t need = fwd_ws_layout(L, T, allow_codes, nullptr, nullptr);
   if (!workspace || workspace_bytes < need)
     return fail(LRQAT_ERR_WORKSPACE, "forward workspace of %zu bytes required, %zu given", need,
                 workspace ? workspace_bytes : (size_t)0);
@@ -641,14 +672,14 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   LRQAT_TRY(device_info(&dev));
 
   FwdWs ws;
-  fwd_ws_layout(L, T, workspace, &ws);
+  fwd_ws_layout(L, T, allow_codes, workspace, &ws);
   const int r16 = round16(L.r);
-  const bool cb = codes_base(L);
+  const bool cb = L.r > 64 || (allow_codes && codes_gemm(L, T));
   const bool pair = use_pair(L.m, false);
   // the pair kernel reads K-major factor slices, so it takes B^T from the padded copy
   const bool direct = !cb && !pair && direct_factors(L, A, B);
   if (cb) {
-    // ranks above 64: the codes of every weight, once per call
+    // the codes of every weight, once per call
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
                  "adapter layouts");
@@ -736,13 +767,13 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
 int lrqat_linear_fwd(const lrqat_layer* layer, int64_t T, const uint16_t* X, const void* Phi0, const float* s,
                      const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y, void* workspace,
                      size_t workspace_bytes, lrqat_stream_t stream) {
-  return linear_fwd_impl(layer, T, X, false, Phi0, s, A, B, s_x, Y, workspace, workspace_bytes, stream);
+  return linear_fwd_impl(layer, T, X, false, Phi0, s, A, B, s_x, Y, workspace, workspace_bytes, true, stream);
 }
 
 int lrqat_linear_fwd_quantized(const lrqat_layer* layer, int64_t T, const uint16_t* X_q, const void* Phi0,
                                const float* s, const uint16_t* A, const uint16_t* B, const float* s_x, uint16_t* Y,
                                void* workspace, size_t workspace_bytes, lrqat_stream_t stream) {
-  return linear_fwd_impl(layer, T, X_q, true, Phi0, s, A, B, s_x, Y, workspace, workspace_bytes, stream);
+  return linear_fwd_impl(layer, T, X_q, true, Phi0, s, A, B, s_x, Y, workspace, workspace_bytes, true, stream);
 }
 
 size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
@@ -801,10 +832,13 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   const int fmt_t = L.phi_format == LRQAT_PHI_INT_PACKED ? LRQAT_PHI_QFIXED : L.phi_format;
   // with direct factors the dX GEMM reads its A slices from A itself; its row factor stays the
   // padded B^T, and dW takes A^T and B padded
-  const bool cb = codes_base(L);
+  // cb: the dX GEMM reads the codes (lrqat_set_lowrank_path); cbw: so does dW (ranks above 64)
+  const bool cb = codes_gemm(L, T);
+  const bool cbw = codes_dw(L);
   const bool direct = !cb && direct_factors(L, A, B);
   if (cb) {
-    // ranks above 64: the codes of every weight, then their transpose for the dX GEMM
+    // the codes of every weight, then their transpose for the dX GEMM; A^T and B padded serve
+    // the code pass and dW
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
                  "adapter layouts");
@@ -836,6 +870,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   }
   // the codes base has no fraction bits
   const QuantParams q = make_quant_params(L.bits, cb ? 0 : frac_bits(L), L.alpha, L.r);
+  const QuantParams qw = make_quant_params(L.bits, cbw ? 0 : frac_bits(L), L.alpha, L.r);
 
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
@@ -906,10 +941,10 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_TRY(encode_2d(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, xop, L.k, T, L.k * 2, 64, 32,
                         CU_TENSOR_MAP_SWIZZLE_128B, "X (dW)"));
     // the codes base: boxes of 64 rank rows (one round of the adapter contractions)
-    const uint32_t rbox_rows = cb ? 64u : static_cast<uint32_t>(r16);
+    const uint32_t rbox_rows = cbw ? 64u : static_cast<uint32_t>(r16);
     LRQAT_TRY(encode_2d(&tm_at, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64, rbox_rows,
                         CU_TENSOR_MAP_SWIZZLE_128B, "A^T"));
-    if (cb)
+    if (cbw)
       LRQAT_TRY(encode_2d(&tm_phi, CU_TENSOR_MAP_DATA_TYPE_UINT8, ws.codes, L.k, L.m, L.k, 128, 128,
                           CU_TENSOR_MAP_SWIZZLE_128B, "codes"));
     else
@@ -928,10 +963,10 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.nsplit = plan.nsplit;
     a.tchunk = plan.tchunk;
     a.num_units = plan.units;
-    a.q = q;
+    a.q = qw;
     a.s = s;
     a.zero = L.zero;
-    a.u_bf16 = cb ? 0 : L.u_bf16;
+    a.u_bf16 = cbw ? 0 : L.u_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;   // per token: folded into X_hat
@@ -940,13 +975,13 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.ds_part = ws.ds_part;
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
-    a.phi = cb ? static_cast<const void*>(ws.codes) : Phi0;
+    a.phi = cbw ? static_cast<const void*>(ws.codes) : Phi0;
     a.sched = plan.sched;
     a.tile_segs = ws.tile_segs;
-    a.codes_base = cb ? 1 : 0;
+    a.codes_base = cbw ? 1 : 0;
     const int grid = plan.sched.grid;
     LRQAT_LAUNCH("fused_dw", 1, stream,
-                 launch_dw(cb ? LRQAT_PHI_QFIXED : L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
+                 launch_dw(cbw ? LRQAT_PHI_QFIXED : L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
                  "fused dW launch");
   }
   ReduceArgs ra{};
@@ -1086,12 +1121,19 @@ int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const flo
 }
 
 int lrqat_get_gemm_variant(void) { return g_gemm_variant.load(std::memory_order_relaxed); }
+int lrqat_get_lowrank_path(void) { return g_lowrank_path.load(std::memory_order_relaxed); }
 int lrqat_get_dw_schedule(void) { return g_dw_schedule.load(std::memory_order_relaxed); }
 
 int lrqat_set_gemm_variant(int variant) {
   if (variant < 0 || variant > 2)
     return fail(LRQAT_ERR_INVALID_ARG, "GEMM variant must be 0, 1 or 2 (got %d)", variant);
   g_gemm_variant.store(variant, std::memory_order_relaxed);
+  return LRQAT_OK;
+}
+
+int lrqat_set_lowrank_path(int path) {
+  if (path < 0 || path > 2) return fail(LRQAT_ERR_INVALID_ARG, "low-rank path must be 0, 1 or 2 (got %d)", path);
+  g_lowrank_path.store(path, std::memory_order_relaxed);
   return LRQAT_OK;
 }
 

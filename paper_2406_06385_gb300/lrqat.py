@@ -96,13 +96,15 @@ def lib() -> ctypes.CDLL:
             fn = getattr(L, name)
             fn.argtypes = args
             fn.restype = ctypes.c_int
-        for name in ("lrqat_get_gemm_variant", "lrqat_get_dw_schedule"):
+        for name in ("lrqat_get_gemm_variant", "lrqat_get_dw_schedule", "lrqat_get_lowrank_path"):
             getattr(L, name).argtypes = []
             getattr(L, name).restype = ctypes.c_int
         L.lrqat_set_gemm_variant.argtypes = [ip]
         L.lrqat_set_gemm_variant.restype = ctypes.c_int
         L.lrqat_set_dw_schedule.argtypes = [ip]
         L.lrqat_set_dw_schedule.restype = ctypes.c_int
+        L.lrqat_set_lowrank_path.argtypes = [ip]
+        L.lrqat_set_lowrank_path.restype = ctypes.c_int
         L.lrqat_trace_enable.argtypes = [ip]
         L.lrqat_trace_enable.restype = ctypes.c_int
         L.lrqat_trace_read.argtypes = [ip, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_int64),
@@ -244,6 +246,20 @@ def gemm_variant() -> str:
 
 def dw_schedule() -> str:
     return {v: k for k, v in DW_SCHEDULES.items()}[lib().lrqat_get_dw_schedule()]
+
+
+LOWRANK_PATHS = {"auto": 0, "tile": 1, "codes": 2}
+
+
+def set_lowrank_path(path: str) -> None:
+    """Process-wide source of the low-rank term in the forward and dX GEMMs: "auto" (the
+    default), "tile" (computed inside each GEMM stage; ranks up to 64) or "codes" (one pass per
+    call writes the codes of every weight, which the GEMMs read)."""
+    _check(lib().lrqat_set_lowrank_path(LOWRANK_PATHS[path]))
+
+
+def lowrank_path() -> str:
+    return {v: k for k, v in LOWRANK_PATHS.items()}[lib().lrqat_get_lowrank_path()]
 
 
 def trace_enable(enable: bool = True) -> None:

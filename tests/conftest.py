@@ -30,3 +30,13 @@ def gemm_variant():
     before = LQ.gemm_variant()
     yield LQ.set_gemm_variant
     LQ.set_gemm_variant(before)
+
+
+@pytest.fixture
+def lowrank_path():
+    """Forces the source of the GEMMs' low-rank term for one test ("tile" or "codes") and
+    restores the previous setting afterwards."""
+    from paper_2406_06385_gb300 import lrqat as LQ
+    before = LQ.lowrank_path()
+    yield LQ.set_lowrank_path
+    LQ.set_lowrank_path(before)

@@ -192,6 +192,32 @@ def test_dw_schedule_environment_is_read_once_at_load(lib, dw_schedule, monkeypa
     assert int(out.stdout.strip()) == split
 
 
+def test_lowrank_path_setting(lib, lowrank_path, monkeypatch):
+    """The source of the GEMMs' low-rank term is a process-wide setting whose start value
+    comes from LRQAT_LOWRANK_PATH at load; the workspace sizes cover every setting (so a size
+    query and the call that uses it agree whatever the setting is), and the forward's size holds
+    the m x k int8 codes of the weights."""
+    L = _layer(m=4096, k=4096, r=32, alpha=32.0)
+    sizes = {}
+    for path in ("auto", "tile", "codes"):
+        lowrank_path(path)
+        assert LQ.lowrank_path() == path
+        sizes[path] = (lib.lrqat_fwd_workspace_bytes(ctypes.byref(L), 8192),
+                       lib.lrqat_bwd_workspace_bytes(ctypes.byref(L), 8192))
+    assert sizes["auto"] == sizes["tile"] == sizes["codes"]
+    assert sizes["auto"][0] >= 4096 * 4096 and sizes["auto"][1] >= 2 * 4096 * 4096
+    assert lib.lrqat_set_lowrank_path(3) == -1 and lib.lrqat_set_lowrank_path(-1) == -1
+    code = ("import sys; sys.path.insert(0, %r); from paper_2406_06385_gb300 import lrqat as LQ; "
+            "print(LQ.lowrank_path())" % ROOT)
+    import subprocess
+    import sys
+    for value, expect in (("tile", "tile"), ("codes", "codes"), ("bogus", "auto")):
+        env = dict(os.environ, LRQAT_LOWRANK_PATH=value)
+        out = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=120)
+        assert out.returncode == 0, out.stderr
+        assert out.stdout.strip() == expect
+
+
 def test_gradient_outputs_must_be_16_byte_aligned(lib):
     """The gradient reduction reads and writes dA and dB with 16-byte accesses, so an
     unaligned dA or dB is rejected on the host before any launch (ds may be unaligned)."""

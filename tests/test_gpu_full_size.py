@@ -59,6 +59,14 @@ FULL_CASES = [
 ]
 
 
+# The source of the GEMMs' low-rank term (lrqat_set_lowrank_path): at these token counts the
+# default takes the codes pass; the 13B q/k/v/o shape and the 4096 x 4096 layer also run with
+# the tile each GEMM stage computes.
+_BOTH_PATHS = ("llama2_13b_qkvo", "llama2_7b_attn")
+FULL_PATH_CASES = [pytest.param(*c, p, id=f"{c[0]}-{p}") for c in FULL_CASES
+                   for p in (("tile", "codes") if c[0] in _BOTH_PATHS else ("auto",))]
+
+
 def _report(test: str, cid: str, **fields):
     """One JSON line per case: on stdout and, with LRQAT_PARITY_REPORT set, in that file."""
     line = json.dumps(dict(test=test, case=cid, **fields), sort_keys=True)
@@ -85,8 +93,9 @@ def _codes_spec(spec):
                         spec.w_row_shift, False)
 
 
-@pytest.mark.parametrize("cid,spec,T", FULL_CASES, ids=[c[0] for c in FULL_CASES])
-def test_full_size_codes_bit_exact(cid, spec, T):
+@pytest.mark.parametrize("cid,spec,T,path", FULL_PATH_CASES)
+def test_full_size_codes_bit_exact(cid, spec, T, path, lowrank_path):
+    lowrank_path(path)
     t = torch()
     spec = _codes_spec(spec)
     data = WL.make_layer(spec, 1, seed=3, with_activations=False)
@@ -118,14 +127,15 @@ def test_full_size_codes_bit_exact(cid, spec, T):
     c = O.codes_from_u(u, OL)[1] - O.expand_zero(z0, OL)   # the operand holds c - z
     exempt = O.near_tie(u)
     bad = {name: int(((got != c) & ~exempt).sum()) for name, got in (("fwd", c_fwd), ("dX", c_dx))}
-    _report("codes", cid, codes=int(c.size), near_tie_exempt=int(exempt.sum()), mismatches_fwd=bad["fwd"],
+    _report("codes", cid, path=LQ.lowrank_path(), codes=int(c.size), near_tie_exempt=int(exempt.sum()), mismatches_fwd=bad["fwd"],
             mismatches_dx=bad["dX"], differ_at_exempt=int(((c_fwd != c) & exempt).sum()))
     for name, n in bad.items():
         assert n == 0, f"{name}: {n} code mismatches of {c.size} (near-ties exempt: {exempt.sum()})"
 
 
-@pytest.mark.parametrize("cid,spec,T", FULL_CASES, ids=[c[0] for c in FULL_CASES])
-def test_full_size_sampled_outputs(cid, spec, T):
+@pytest.mark.parametrize("cid,spec,T,path", FULL_PATH_CASES)
+def test_full_size_sampled_outputs(cid, spec, T, path, lowrank_path):
+    lowrank_path(path)
     t = torch()
     data = WL.make_layer(spec, T, seed=11)
     dl = DeviceLayer(data)
@@ -187,7 +197,7 @@ def test_full_size_sampled_outputs(cid, spec, T):
     dB_ref = scale * (data.A.astype(np.float64).T @ dU_cols)
     dB_got = dB.cpu().numpy()[:, cols]
     errs["dB"] = O.rel_fro(dB_got, dB_ref)
-    _report("sampled_outputs", cid, T=T, rel_err=errs, token_rows=len(ts), weight_rows=len(rows),
+    _report("sampled_outputs", cid, path=LQ.lowrank_path(), T=T, rel_err=errs, token_rows=len(ts), weight_rows=len(rows),
             weight_cols=len(cols))
     for key in ("Y", "dX"):
         assert errs[key] <= TOL_ACT, errs

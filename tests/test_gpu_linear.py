@@ -122,8 +122,20 @@ def _run(spec, T, seed=0, s_scale=1.0, sx_factor=1.0, zero_B=False):
     return got, ref, g
 
 
-@pytest.mark.parametrize("cid,spec,T", CASES, ids=[c[0] for c in CASES])
-def test_fwd_bwd_parity(cid, spec, T):
+def with_paths(cases):
+    """Each case of rank up to 64 on both sources of the GEMMs' low-rank term (the tile each
+    stage computes, and the codes one pass per call writes); ranks above 64 always take the
+    codes."""
+    out = []
+    for c in cases:
+        for path in (("tile", "codes") if c[1].r <= 64 else ("auto",)):
+            out.append(pytest.param(*c, path, id=f"{c[0]}-{path}"))
+    return out
+
+
+@pytest.mark.parametrize("cid,spec,T,path", with_paths(CASES))
+def test_fwd_bwd_parity(cid, spec, T, path, lowrank_path):
+    lowrank_path(path)
     got, ref, g = _run(spec, T, seed=1, s_scale=1.05)
     errs = {k: O.rel_fro(got[k], ref[k]) for k in got}
     assert errs["Y"] <= TOL_ACT and errs["dX"] <= TOL_ACT, errs
@@ -189,9 +201,15 @@ CODE_CASES = [
 ]
 
 
-@pytest.mark.parametrize("cid,spec", CODE_CASES, ids=[c[0] for c in CODE_CASES])
+@pytest.mark.parametrize("cid,spec,path", [pytest.param(c[0], c[1], p, id=f"{c[0]}-{p}") for c in CODE_CASES
+                                           for p in (("tile", "codes") if c[1].r <= 64 else ("auto",))])
 @pytest.mark.parametrize("zero_B", [False, True], ids=["lowrank", "ties"])
-def test_fused_codes_bit_exact(cid, spec, zero_B):
+def test_fused_codes_bit_exact(cid, spec, path, zero_B, lowrank_path):
+    lowrank_path(path)
+    check_codes_bit_exact(cid, spec, zero_B)
+
+
+def check_codes_bit_exact(cid, spec, zero_B):
     """With s = 1 and X = I (T = k) the forward returns Y = C^T exactly; with
     dY = I (T = m) the dX kernel returns its own codes C (C - z with zero offsets).
     Both must equal the oracle's codes except at near-ties; B = 0 makes every
@@ -413,8 +431,9 @@ PAIR_CASES = [c for c in CASES if c[1].m % 256 == 0 or c[1].k % 256 == 0] + [
 ]
 
 
-@pytest.mark.parametrize("cid,spec,T", PAIR_CASES, ids=[c[0] for c in PAIR_CASES])
-def test_fwd_bwd_parity_gemm_variants(cid, spec, T, gemm_variant):
+@pytest.mark.parametrize("cid,spec,T,path", with_paths(PAIR_CASES))
+def test_fwd_bwd_parity_gemm_variants(cid, spec, T, path, gemm_variant, lowrank_path):
+    lowrank_path(path)
     outs = {}
     for variant in ("pair", "single"):
         gemm_variant(variant)
@@ -429,9 +448,12 @@ def test_fwd_bwd_parity_gemm_variants(cid, spec, T, gemm_variant):
 
 @pytest.mark.parametrize("cid,spec", [c for c in CODE_CASES if c[1].m % 256 == 0 and c[1].k % 256 == 0],
                          ids=[c[0] for c in CODE_CASES if c[1].m % 256 == 0 and c[1].k % 256 == 0])
-def test_fused_codes_bit_exact_pair_gemm(cid, spec, gemm_variant):
+def test_fused_codes_bit_exact_pair_gemm(cid, spec, gemm_variant, lowrank_path):
     """The integer codes the pair kernel's producers build, through the identity inputs of
-    test_fused_codes_bit_exact, with exact ties (B = 0) and with the low-rank term."""
+    check_codes_bit_exact, with exact ties (B = 0) and with the low-rank term, from the
+    in-stage tile and from the codes pass."""
     gemm_variant("pair")
-    for zero_B in (False, True):
-        test_fused_codes_bit_exact(cid, spec, zero_B)
+    for path in (("tile", "codes") if spec.r <= 64 else ("auto",)):
+        lowrank_path(path)
+        for zero_B in (False, True):
+            check_codes_bit_exact(cid, spec, zero_B)
