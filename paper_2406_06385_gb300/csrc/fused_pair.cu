@@ -476,19 +476,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           mword = args.xmask[static_cast<int64_t>(row_g) * args.xmask_ld + tok0 / 32] >> (tok0 & 31);
 #pragma unroll
         for (int e = 0; e < 16; ++e) acc[e] = ((mword >> e) & 1u) ? acc[e] * scale : 0.0f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float mine = odd ? acc[2 * e] : acc[2 * e + 1];
-          const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
-          const int tt = tok0 + 2 * e + (odd ? 1 : 0);
-          const float lo = odd ? other : acc[2 * e];
-          const float hi = odd ? acc[2 * e + 1] : other;
-          if (tt < args.T) {
-            uint32_t* dst = reinterpret_cast<uint32_t*>(args.out + static_cast<int64_t>(tt) * args.out_ld +
-                                                        (row_g & ~1));
-            *dst = pack_rn_bf16x2(lo, hi);
-          }
-        }
+        store_row_pairs_bf16(acc, odd, args.out, args.out_ld, row_g, tok0, args.T);
       }
       tc_fence_before();
       __syncwarp();
