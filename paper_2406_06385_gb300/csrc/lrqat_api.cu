@@ -527,8 +527,9 @@ int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, c
                       CU_TENSOR_MAP_SWIZZLE_128B, "A^T (padded)"));
   LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B_pad, L.k, r16, L.k * 2, 64,
                       static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
+  CUtensorMap tm_phi;
+  LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
   MergeArgs a{};
-  a.phi0 = Phi0;
   a.wz = codes;
   a.m = L.m;
   a.k = L.k;
@@ -536,7 +537,7 @@ int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, c
   a.q = saturating_params(L);
   a.status = dev->status;
   a.timeout_ns = kWaitTimeoutNs;
-  LRQAT_LAUNCH("lowrank_codes", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 1, tm_a, tm_b, a, stream),
+  LRQAT_LAUNCH("lowrank_codes", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 1, tm_a, tm_b, tm_phi, a, stream),
                "low-rank code pass");
   return LRQAT_OK;
 }
@@ -1043,8 +1044,9 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
                         CU_TENSOR_MAP_SWIZZLE_128B, "A"));
     LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B, L.k, L.r, L.k * 2, 64,
                         static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B"));
+    CUtensorMap tm_phi;
+    LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
     MergeArgs a{};
-    a.phi0 = Phi0;
     a.wz = W_Z;
     a.m = L.m;
     a.k = L.k;
@@ -1052,7 +1054,7 @@ int lrqat_merge(const lrqat_layer* layer, const void* Phi0, const uint16_t* A, c
     a.q = q;
     a.status = dev->status;
     a.timeout_ns = kWaitTimeoutNs;
-    LRQAT_LAUNCH("merge", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 0, tm_a, tm_b, a, stream),
+    LRQAT_LAUNCH("merge", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 0, tm_a, tm_b, tm_phi, a, stream),
                  "merge launch");
     return LRQAT_OK;
   }

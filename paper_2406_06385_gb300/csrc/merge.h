@@ -17,9 +17,10 @@ namespace lrqat {
 //   a_mn == 0: tm_a over A [m, r] (r % 8 == 0, 16-byte aligned), 64 x 128 boxes, K-major;
 //   a_mn == 1: tm_a over the zero-padded A^T [r16, m], 64 x r16 boxes, MN-major.
 //   tm_b over B [r, k] or the zero-padded B [r16, k], 64 x r16 boxes.  All 128-byte swizzled;
-//   phi0 and wz 16-byte aligned.
+//   tm_phi over the stored base in 128-column chunks: 8-bit values 128 x 128 boxes (SW128),
+//   packed nibbles 64-byte x 128-row boxes (SW64), 16-bit values 64 x 128 boxes (SW128);
+//   wz 16-byte aligned.
 struct MergeArgs {
-  const void* phi0;      // stored base [m, k] in its format
   int8_t* wz;            // codes [m, k]
   int64_t m, k;
   int32_t r16;           // adapter rank rounded up to 16 (<= 256)
@@ -29,6 +30,6 @@ struct MergeArgs {
 };
 // fmt: a PhiFmt value (quant.cuh); u_bf16: the bf16 pre-round value (not with FP16 bases)
 cudaError_t launch_merge_tc(int fmt, int u_bf16, int a_mn, const CUtensorMap& tm_a, const CUtensorMap& tm_b,
-                            const MergeArgs& args, cudaStream_t stream);
+                            const CUtensorMap& tm_phi, const MergeArgs& args, cudaStream_t stream);
 
 }  // namespace lrqat
