@@ -18,7 +18,7 @@ BUILD_DIR = os.path.join(PKG, "_build")
 LIB_DIR = os.path.join(PKG, "_lib")
 LIB_PATH = os.path.join(LIB_DIR, "liblrqat.so")
 
-SOURCES = ["elementwise.cu", "fused_gemm.cu", "fused_pair.cu", "dw.cu", "merge.cu", "optim.cu", "lrqat_api.cu"]
+SOURCES = ["elementwise.cu", "fused_gemm.cu", "fused_pair.cu", "dw.cu", "dw_pair.cu", "merge.cu", "optim.cu", "lrqat_api.cu"]
 HEADERS = ["kernels.h", "ptx.cuh", "quant.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]

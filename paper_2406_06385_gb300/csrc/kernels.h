@@ -198,6 +198,16 @@ struct DwArgs {
   int32_t codes_base;
 };
 int dw_smem_bytes(int r16, int fmt);
+// The same kernel on CTA pairs (dw_pair.cu) for ranks up to 64, m and k multiples of 256:
+// units of 256 x 256 tiles (args.ni = m / 256, args.nj = k / 256, nchunks 2), npairs clusters of
+// two; tm_ath / tm_bh as tm_at / tm_b with boxes of r16 / 2 rank rows.  The partials are laid out
+// as launch_dw's (dB per 128-row block, tile_segs per 128-row tile).
+cudaError_t launch_dw_pair(int fmt, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
+                           const CUtensorMap& tm_ath, const CUtensorMap& tm_phi, const CUtensorMap& tm_b,
+                           const CUtensorMap& tm_bh, const DwArgs& args, int npairs, cudaStream_t stream);
+// Clusters of two of the pair dW kernel that can be resident at once on the current device
+// (0 when the query fails).
+int dw_pair_max_pairs();
 // fmt: a PhiFmt value (quant.cuh)
 cudaError_t launch_dw(int fmt, const CUtensorMap& tm_dy, const CUtensorMap& tm_x, const CUtensorMap& tm_at,
                       const CUtensorMap& tm_phi, const CUtensorMap& tm_b, const DwArgs& args, int grid,

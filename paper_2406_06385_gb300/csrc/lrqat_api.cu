@@ -321,18 +321,33 @@ bool use_pair(int64_t rows, bool group_dx) {
 }
 constexpr int kPairTokens = 448;   // tokens per pair tile (two accumulators of 224)
 
+constexpr int kDwPairTokensPerStage = 64;   // the pair dW kernel's stage (dw_pair.cu)
+// dW on CTA pairs (dw_pair.cu): 256 x 256 tiles, ranks up to 64, by the same setting as the
+// forward and dX GEMMs (lrqat_set_gemm_variant: not with 1, the one-SM kernels).
+bool use_pair_dw(const lrqat_layer& L) {
+  return L.m % 256 == 0 && L.k % 256 == 0 && !codes_dw(L) && g_gemm_variant.load(std::memory_order_relaxed) != 1;
+}
+
 struct DwPlan {
   int nchunks, ni, nj, nsplit, tchunk, units;
   DwSched sched;
+  bool pair;   // the pair kernel: ni counts 256-row tiles and sched.grid pairs
+  int ni128;   // 128-row blocks (the partial outputs)
+  int bkt;     // tokens per pipeline stage
 };
 
-DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
+// sms: the work slots of the persistent grid (SMs for the one-SM kernel, resident pairs for
+// the pair kernel).
+DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms, bool pair) {
   DwPlan p;
+  p.pair = pair;
   p.nchunks = (L.k % 256 == 0 && !codes_dw(L)) ? 2 : 1;
-  p.ni = static_cast<int>(L.m / 128);
+  p.ni128 = static_cast<int>(L.m / 128);
+  p.ni = static_cast<int>(pair ? L.m / 256 : L.m / 128);
   p.nj = static_cast<int>(L.k / (128 * p.nchunks));
   const int tiles = p.ni * p.nj;
-  const int64_t tsteps = (T + 31) / 32;
+  p.bkt = pair ? kDwPairTokensPerStage : 32;   // tokens per pipeline stage
+  const int64_t tsteps = (T + p.bkt - 1) / p.bkt;
   // Pick the token split that fills the SMs best; keep >= 256 tokens per split.
   int best = 1;
   double best_eff = 0.0;
@@ -347,7 +362,7 @@ DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
     }
   }
   p.nsplit = best;
-  p.tchunk = static_cast<int>((tsteps + best - 1) / best) * 32;
+  p.tchunk = static_cast<int>((tsteps + best - 1) / best) * p.bkt;
   p.nsplit = static_cast<int>((T + p.tchunk - 1) / p.tchunk);   // no empty splits
   p.units = tiles * p.nsplit;
   const int grid_eq = p.units < sms ? p.units : sms;
@@ -356,9 +371,9 @@ DwPlan plan_dw(const lrqat_layer& L, int64_t T, int sms) {
   // token parts, one per CTA (at most 8 parts a tile, none shorter than a stage), by the
   // slowest CTA's cost in stage units: its stages plus kEpilogueStages for each unit it
   // finishes (the part of the epilogue that the next main loop waits for).
-  constexpr int64_t kEpilogueStages = 32;
+  const int64_t kEpilogueStages = 32 * 32 / p.bkt;
   const int64_t waves = (p.units + grid_eq - 1) / grid_eq;
-  const int64_t cost_eq = waves * (p.tchunk / 32 + kEpilogueStages);
+  const int64_t cost_eq = waves * (p.tchunk / p.bkt + kEpilogueStages);
   const int64_t full_tiles = tiles / sms * sms;
   const int64_t tail_tiles = tiles - full_tiles;
   const int64_t q_cap = tsteps < 8 ? tsteps : 8;
@@ -444,9 +459,9 @@ size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* bas
     w.xmask = static_cast<uint32_t*>(c.take(static_cast<size_t>(L.k) * ((T + 31) / 32) * 4));
   }
   w.dA_part = static_cast<float*>(c.take(static_cast<size_t>(p.nj) * p.nsplit * L.m * L.r * 4));
-  w.dB_part = static_cast<float*>(c.take(static_cast<size_t>(p.ni) * p.nsplit * L.r * L.k * 4));
+  w.dB_part = static_cast<float*>(c.take(static_cast<size_t>(p.ni128) * p.nsplit * L.r * L.k * 4));
   w.ds_part = static_cast<float*>(c.take(static_cast<size_t>(2) * p.nsplit * L.m * (L.k / 128) * 4));
-  w.tile_segs = static_cast<int32_t*>(c.take(static_cast<size_t>(p.ni) * p.nj * 4));
+  w.tile_segs = static_cast<int32_t*>(c.take(static_cast<size_t>(p.ni128) * p.nj * 4));
   if (ws) *ws = w;
   return (c.used + 255) & ~size_t(255);
 }
@@ -782,7 +797,11 @@ size_t lrqat_bwd_workspace_bytes(const lrqat_layer* layer, int64_t T) {
   DeviceInfo* dev = nullptr;
   int sms = 152;
   if (device_info(&dev) == LRQAT_OK) sms = dev->sms;
-  return bwd_ws_layout(*layer, T, plan_dw(*layer, T, sms), nullptr, nullptr);
+  const bool pair = use_pair_dw(*layer);
+  int pairs = sms / 2;
+  if (pair && dev) pairs = dw_pair_max_pairs();
+  if (pair && pairs < 1) return 0;
+  return bwd_ws_layout(*layer, T, plan_dw(*layer, T, pair ? pairs : sms, pair), nullptr, nullptr);
 }
 
 // quantized: X is already the activation quantizer's output (as for linear_fwd_impl) and
@@ -819,7 +838,10 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     return fail(LRQAT_ERR_INVALID_ARG, "s_x is required when act_bits == 8 (per-tensor scale)");
   DeviceInfo* dev = nullptr;
   LRQAT_TRY(device_info(&dev));
-  const DwPlan plan = plan_dw(L, T, dev->sms);
+  const bool dw_pair = use_pair_dw(L);
+  const int dw_pairs = dw_pair ? dw_pair_max_pairs() : 0;
+  if (dw_pair && dw_pairs < 1) return fail(LRQAT_ERR_CUDA, "no cluster of two fits the dW kernel");
+  const DwPlan plan = plan_dw(L, T, dw_pair ? dw_pairs : dev->sms, dw_pair);
   const size_t need = bwd_ws_layout(L, T, plan, nullptr, nullptr);
   if (!workspace || workspace_bytes < need)
     return fail(LRQAT_ERR_WORKSPACE, "backward workspace of %zu bytes required, %zu given", need,
@@ -937,10 +959,10 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   // G = dY^T X_hat in TMEM, STE epilogue -> partials of dA, dB, ds.
   {
     CUtensorMap tm_dy, tm_x, tm_at, tm_phi, tm_b;
-    LRQAT_TRY(encode_2d(&tm_dy, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, 32,
-                        CU_TENSOR_MAP_SWIZZLE_128B, "dY (dW)"));
-    LRQAT_TRY(encode_2d(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, xop, L.k, T, L.k * 2, 64, 32,
-                        CU_TENSOR_MAP_SWIZZLE_128B, "X (dW)"));
+    LRQAT_TRY(encode_2d(&tm_dy, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64,
+                        static_cast<uint32_t>(plan.bkt), CU_TENSOR_MAP_SWIZZLE_128B, "dY (dW)"));
+    LRQAT_TRY(encode_2d(&tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, xop, L.k, T, L.k * 2, 64,
+                        static_cast<uint32_t>(plan.bkt), CU_TENSOR_MAP_SWIZZLE_128B, "X (dW)"));
     // the codes base: boxes of 64 rank rows (one round of the adapter contractions)
     const uint32_t rbox_rows = cbw ? 64u : static_cast<uint32_t>(r16);
     LRQAT_TRY(encode_2d(&tm_at, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64, rbox_rows,
@@ -981,15 +1003,27 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.tile_segs = ws.tile_segs;
     a.codes_base = cbw ? 1 : 0;
     const int grid = plan.sched.grid;
-    LRQAT_LAUNCH("fused_dw", 1, stream,
-                 launch_dw(cbw ? LRQAT_PHI_QFIXED : L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
-                 "fused dW launch");
+    if (plan.pair) {
+      // each CTA of a pair loads half of the ranks of the slices that serve as N-split B operands
+      CUtensorMap tm_ath, tm_bh;
+      LRQAT_TRY(encode_2d(&tm_ath, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.at, L.m, r16, L.m * 2, 64,
+                          static_cast<uint32_t>(r16 / 2), CU_TENSOR_MAP_SWIZZLE_128B, "A^T (rank halves)"));
+      LRQAT_TRY(encode_2d(&tm_bh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, ws.b_pad, L.k, r16, L.k * 2, 64,
+                          static_cast<uint32_t>(r16 / 2), CU_TENSOR_MAP_SWIZZLE_128B, "B (rank halves)"));
+      LRQAT_LAUNCH("fused_dw", 1, stream,
+                   launch_dw_pair(L.phi_format, tm_dy, tm_x, tm_at, tm_ath, tm_phi, tm_b, tm_bh, a, grid, stream),
+                   "fused dW launch (CTA pairs)");
+    } else {
+      LRQAT_LAUNCH("fused_dw", 1, stream,
+                   launch_dw(cbw ? LRQAT_PHI_QFIXED : L.phi_format, tm_dy, tm_x, tm_at, tm_phi, tm_b, a, grid, stream),
+                   "fused dW launch");
+    }
   }
   ReduceArgs ra{};
   ra.dA_part = ws.dA_part;
   ra.nA = plan.nj * plan.nsplit;
   ra.dB_part = ws.dB_part;
-  ra.nB = plan.ni * plan.nsplit;
+  ra.nB = plan.ni128 * plan.nsplit;
   ra.ds_part = ws.ds_part;
   ra.nS = 2 * plan.nsplit;
   ra.dA = dA;
@@ -1002,7 +1036,9 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   ra.lr = static_cast<float>(static_cast<double>(L.alpha) / L.r);
   ra.accumulate = accumulate ? 1 : 0;
   ra.sched = plan.sched;
-  ra.ni = plan.ni;
+  // the reduction counts 128-row tiles: a whole pair tile is two whole 128-row tiles
+  if (plan.pair) ra.sched.full_tiles *= 2;
+  ra.ni = plan.ni128;
   ra.nsplit = plan.nsplit;
   ra.bn = 128 * plan.nchunks;
   ra.tile_segs = ws.tile_segs;
