@@ -3,25 +3,24 @@
 // kernel (Eq. 8; the recompute replaces the checkpointing of Sec. 3), with the main
 // product issued as tcgen05 MMAs of M = 256 rows across the two SMs of a cluster.
 //
-// Why pairs: the one-SM kernel is bound by its shared-memory port (each 64-wide stage of a
-// 128 x 448 tile moves ~192 KB through it, two thirds of it the token operand, written by
-// TMA and read by the MMAs).  In a pair each CTA holds its own 128 weight rows and only half
-// of every accumulator's tokens; the tensor cores of the pair exchange the token halves, so
-// each SM moves ~124 KB per stage for 128 rows x 384 tokens.
+// Why pairs: the one-SM kernel (128 x 448 tiles) moves its whole 448-token operand through
+// each SM's shared memory every stage; in a pair each CTA holds its own 128 weight rows and only
+// half of every accumulator's tokens, and the tensor cores of the pair exchange the token halves
+// (measured on a 4096 x 4096 layer at T = 8192 on the codes: forward 276 -> 181 us).
 //
-// A pair processes tiles of 256 weight rows (CTA rank c: rows 128 c .. 128 c + 127) x 384
-// tokens (two accumulators of 192 tokens; CTA c holds tokens 96 c .. 96 c + 95 of each), one
+// A pair processes tiles of 256 weight rows (CTA rank c: rows 128 c .. 128 c + 127) x 448
+// tokens (two accumulators of 224 tokens; CTA c holds tokens 112 c .. 112 c + 111 of each), one
 // 64-wide slice of the contraction per stage:
-//   * token ring (4 slots per CTA): four loader warps, one per slot, bring this CTA's two
-//     96-token halves (SW128) with TMA whose completion lands on the leader's barrier; each
-//     slot also holds this CTA's W_hat tile of the stage;
-//   * factor ring (4 slots; 2 for 16-bit bases): the stored base of this CTA's rows (completion on its own
-//     barrier; only its own producers read it) and this CTA's half (32 rows) of the second
-//     factor's slice (completion on the leader's barrier: the low-rank MMA reads both halves);
-//   * in the leader, one thread issues the low-rank tiles L = RF SF^T (M = 256, N = 64) into
-//     two TMEM buffers, up to two stages ahead of the producers, and another the main product
-//     (M = 256, N = 192, 8 MMAs per stage), so that neither waits behind the other's barriers;
-//     every commit is multicast to both CTAs;
+//   * token ring (three slots per CTA, four on the codes): one loader warp per slot brings this
+//     CTA's two 112-token halves (SW128) with TMA whose completion lands on the leader's
+//     barrier; each slot also holds this CTA's W_hat tile of the stage;
+//   * factor ring (4 slots; 2 for 16-bit bases): the stored base of this CTA's rows (completion
+//     on its own barrier; only its own producers read it) and this CTA's half (32 rows) of the
+//     second factor's slice (completion on the leader's barrier: the low-rank MMA reads both);
+//   * in the leader, one thread issues the low-rank tile L = RF SF^T (M = 256, N = 64) of each
+//     stage into a TMEM buffer after the accumulators, and another the main product (M = 256,
+//     N = 224, 8 MMAs per stage), so that neither waits behind the other's barriers; every
+//     commit is multicast to both CTAs;
 //   * sixteen producer warps per CTA build this CTA's W_hat tile exactly as the one-SM kernel
 //     does, and drain this CTA's 128 rows of the accumulators in the epilogue.
 // The leader waits for the peer's "W_hat written", "L read" and "accumulators drained" events;
@@ -46,12 +45,12 @@ constexpr int BNP = 224;                         // tokens per accumulator (N of
 constexpr int BNH = BNP / 2;                     // tokens per accumulator held by one CTA
 constexpr int NACC = 2;
 constexpr int BTP = BNP * NACC;                  // 448 tokens per pair tile
-constexpr int NT = 3;                            // token ring slots
+constexpr int NT_MAX = 4;                        // token ring slots (3 with the low-rank tile)
 constexpr int NLB = 1;                           // low-rank TMEM buffers
 constexpr int NF_MAX = 4;                        // factor ring slots (2 for 16-bit bases)
 constexpr int NUM_PROD_WARPS = 16;
 constexpr int FIRST_TMA_WARP = 2 + NUM_PROD_WARPS;
-constexpr int NUM_TMA_WARPS = NT + 1;
+constexpr int NUM_TMA_WARPS = NT_MAX + 1;        // a token loader per slot, the factor loader
 constexpr int NUM_THREADS = 32 * (FIRST_TMA_WARP + NUM_TMA_WARPS);
 constexpr int EPI_COLS = NACC * BNP / 4;         // accumulator columns drained per warp (112)
 constexpr uint32_t SIG_TX = 16u * NUM_PROD_WARPS;   // bytes of the peer's per-warp signals
@@ -62,23 +61,31 @@ constexpr uint32_t TOK_BYTES = NACC * TOK_BOX;
 constexpr uint32_t W_BYTES = 128 * 128;          // 128 rows x 64 bf16
 constexpr uint32_t SFH_BYTES = 32 * 128;         // 32 slice rows x up to 64 rank columns (bf16)
 constexpr uint32_t TSLOT_BYTES = TOK_BYTES + W_BYTES;
-constexpr uint32_t OFF_RF = 0;
-constexpr uint32_t OFF_TSLOTS = RF_BYTES;
-constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
 constexpr uint32_t TS_W = TOK_BYTES;
 
-template <int FMT>
+// Shared-memory rings.  With the low-rank tile: the row factor, three token slots and per stage
+// the stored base and this CTA's half of the second factor's slice.  On the codes (NL): no
+// factors, so a fourth token slot fits (measured on a 4096 x 4096 layer at T = 8192: forward
+// 191 -> 181 us).
+template <int FMT, bool NL>
 struct PairRing {
+  static constexpr int NT = NL ? 4 : 3;
   static constexpr int NF = fmt_16bit(FMT) ? 2 : 4;
+  static constexpr uint32_t RF = NL ? 0u : RF_BYTES;
   static constexpr uint32_t PHI_BYTES = fmt_16bit(FMT) ? 128 * 128 : 128 * 64;
   static constexpr uint32_t PHI_TX = FMT == FMT_I4 ? PHI_BYTES / 2 : PHI_BYTES;
-  static constexpr uint32_t FSLOT_BYTES = PHI_BYTES + SFH_BYTES;
+  static constexpr uint32_t FSLOT_BYTES = PHI_BYTES + (NL ? 0u : SFH_BYTES);
   static constexpr uint32_t FS_SF = PHI_BYTES;
+  static constexpr uint32_t OFF_RF = 0;
+  static constexpr uint32_t OFF_TSLOTS = RF;
+  static constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
   static constexpr uint32_t SMEM_BYTES = OFF_FSLOTS + NF * FSLOT_BYTES + 1024;
-  static_assert(FSLOT_BYTES % 1024 == 0 && FS_SF % 1024 == 0, "swizzled tiles must start on 1024-byte boundaries");
+  static_assert(NT <= NT_MAX, "token slots");
+  static_assert(FSLOT_BYTES % 1024 == 0 && FS_SF % 1024 == 0 && OFF_FSLOTS % 1024 == 0,
+                "swizzled tiles must start on 1024-byte boundaries");
   static_assert(SMEM_BYTES + 1024 <= 232448, "shared memory budget");
 };
-static_assert(TSLOT_BYTES % 1024 == 0 && TOK_BOX % 1024 == 0 && TS_W % 1024 == 0 && OFF_FSLOTS % 1024 == 0,
+static_assert(TSLOT_BYTES % 1024 == 0 && TOK_BOX % 1024 == 0 && TS_W % 1024 == 0,
               "swizzled tiles must start on 1024-byte boundaries");
 static_assert(EPI_COLS % 16 == 0, "epilogue drains 16-column chunks");
 
@@ -87,9 +94,9 @@ constexpr uint32_t COL_L = NACC * BNP;           // the 64-column low-rank buffe
 static_assert(COL_L + NLB * BK <= TMEM_COLS, "TMEM budget");
 
 constexpr int BAR_TFULL = 0;                     // leader: both token halves of the slot landed
-constexpr int BAR_TEMPTY = BAR_TFULL + NT;       // both: main product of the slot finished
-constexpr int BAR_WFULL = BAR_TEMPTY + NT;       // leader: both W_hat tiles of the slot written
-constexpr int BAR_PFULL = BAR_WFULL + NT;        // both: this CTA's base tile landed
+constexpr int BAR_TEMPTY = BAR_TFULL + NT_MAX;   // both: main product of the slot finished
+constexpr int BAR_WFULL = BAR_TEMPTY + NT_MAX;   // leader: both W_hat tiles of the slot written
+constexpr int BAR_PFULL = BAR_WFULL + NT_MAX;    // both: this CTA's base tile landed
 
 constexpr int BAR_FFULL = BAR_PFULL + NF_MAX;    // leader: both factor-slice halves landed
 constexpr int BAR_FEMPTY = BAR_FFULL + NF_MAX;   // both: slot read by this CTA's producers (after L)
@@ -116,8 +123,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_pair_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
                       const FusedArgs args) {
-  using PR = PairRing<FMT>;
+  using PR = PairRing<FMT, NL>;
+  constexpr int NT = PR::NT;
   constexpr int NF = PR::NF;
+  constexpr uint32_t OFF_RF = PR::OFF_RF, OFF_TSLOTS = PR::OFF_TSLOTS, OFF_FSLOTS = PR::OFF_FSLOTS;
   constexpr bool PACKED = FMT == FMT_I4;
   constexpr uint32_t FSLOT_BYTES = PR::FSLOT_BYTES;
   extern __shared__ uint8_t smem_raw[];
@@ -228,10 +237,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           ok = wait_spin_bounded(bar(BAR_LEMPTY + gg % NLB), (gg / NLB) & 1u, ctl, 11);
       }
     }
-  } else if (warp >= FIRST_TMA_WARP && warp < FIRST_TMA_WARP + NT) {
+  } else if (warp >= FIRST_TMA_WARP && warp < FIRST_TMA_WARP + NT_MAX) {
     // ------------------------------------------- token loaders (one per slot)
-    const uint32_t t = warp - FIRST_TMA_WARP;
-    if (lane == 0) {
+    const uint32_t t = warp - FIRST_TMA_WARP;   // slots past NT have no loader work
+    if (lane == 0 && t < static_cast<uint32_t>(NT)) {
       prefetch_tensormap(&tm_tok);
       const uint32_t st = smem + OFF_TSLOTS + t * TSLOT_BYTES;
       const uint32_t fb = lbar(BAR_TFULL + t), eb = bar(BAR_TEMPTY + t);
@@ -252,7 +261,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         g += nk;
       }
     }
-  } else if (warp == FIRST_TMA_WARP + NT) {
+  } else if (warp == FIRST_TMA_WARP + NT_MAX) {
     // ------------------------------------------------- factor-ring loader
     if (lane == 0) {
       prefetch_tensormap(&tm_phi);
@@ -499,7 +508,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 template <int MODE, int FMT, bool ZP, bool UB, bool NL>
 cudaError_t launch_pair_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                             const FusedArgs& args, int npairs, cudaStream_t stream) {
-  constexpr uint32_t smem = PairRing<FMT>::SMEM_BYTES;
+  constexpr uint32_t smem = PairRing<FMT, NL>::SMEM_BYTES;
   static bool configured[kMaxDevices] = {};
   const void* fn = reinterpret_cast<const void*>(fused_pair_kernel<MODE, FMT, ZP, UB, NL>);
   cudaError_t e = ensure_smem_attr(fn, static_cast<int>(smem), configured);
