@@ -420,7 +420,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
           raw[0] = r.x, raw[1] = r.y, raw[2] = r.z, raw[3] = r.w;
         }
-        decode16<FMT>(raw, v);
+        if (NL && args.codes_ob) decode_ob16(raw, v);
+        else decode16<FMT>(raw, v);
         float Lv[16];
         if (!NL) {
           const uint32_t lb = gg % NLB;
@@ -441,8 +442,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               : UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
                    : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
                                 make_float2(v[2 * e], v[2 * e + 1]));
-          const float2 t2 = __fadd2_rn(u, make_float2(qp.magic, qp.magic));
-          uint32_t cw = codes_bf16x2(t2, qp);
+          uint32_t cw = NL ? (args.codes_ob ? pack_int_bf16x2(u.x, u.y) : int_codes_bf16x2(u.x, u.y, qp))
+                           : codes_bf16x2(__fadd2_rn(u, make_float2(qp.magic, qp.magic)), qp);
           if (ZP) cw = sub_bf16x2(cw, zw[e]);
           if (MODE == FUSED_FWD_PC) {
             w[e] = cw;

@@ -163,6 +163,9 @@ struct FusedArgs {
   // Forward only: the second factor's slice read straight from B as one MN-major box
   // of 64 columns x r16 rank rows (no padded B^T copy).
   int32_t sf_mn;
+  // Codes base (r16 == 0): 1 when the codes are clipped to [n, p] and stored offset-binary
+  // (byte = c + 128), so the producers neither flip the sign bit nor clamp; 0: saturated int8.
+  int32_t codes_ob;
 };
 int fused_smem_bytes(int fmt);
 // The same GEMM on CTA pairs (fused_pair.cu): 256-row x 448-token tiles, npairs clusters of 2.

@@ -492,9 +492,11 @@ QuantParams saturating_params(const lrqat_layer& L) {
 }
 
 // The codes pass: codes[i, j] = sat8(round(phi^{-1}(Phi0[i, j]) + (alpha/r) (A B)[i, j])) on the
-// tensor cores, from the zero-padded A^T [r16, m] and B [r16, k] (any rank up to 256).
+// tensor cores, from the zero-padded A^T [r16, m] and B [r16, k] (any rank up to 256).  clipped:
+// the codes clip(round(u), n, p) + 128 instead (offset-binary), for when only the forward and
+// dX GEMMs read them (dW of ranks above 64 needs the unclipped codes for its mask).
 int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, const uint16_t* B_pad, int8_t* codes,
-                   const DeviceInfo* dev, cudaStream_t stream);
+                   bool clipped, const DeviceInfo* dev, cudaStream_t stream);
 
 }  // namespace
 }  // namespace lrqat
@@ -535,7 +537,7 @@ int noalloc_scratch(void** out) {
 
 namespace {
 int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, const uint16_t* B_pad, int8_t* codes,
-                   const DeviceInfo* dev, cudaStream_t stream) {
+                   bool clipped, const DeviceInfo* dev, cudaStream_t stream) {
   const int r16 = round16(L.r);
   CUtensorMap tm_a, tm_b;
   LRQAT_TRY(encode_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, At, L.m, r16, L.m * 2, 64, static_cast<uint32_t>(r16),
@@ -549,7 +551,8 @@ int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, c
   a.m = L.m;
   a.k = L.k;
   a.r16 = r16;
-  a.q = saturating_params(L);
+  a.q = clipped ? make_quant_params(L.bits, frac_bits(L), L.alpha, L.r) : saturating_params(L);
+  a.xor_mask = clipped ? 0x80808080u : 0u;
   a.status = dev->status;
   a.timeout_ns = kWaitTimeoutNs;
   LRQAT_LAUNCH("lowrank_codes", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 1, tm_a, tm_b, tm_phi, a, stream),
@@ -699,7 +702,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
                  "adapter layouts");
-    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, dev, stream));
+    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, true, dev, stream));
   } else if (!direct) {
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
@@ -756,6 +759,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   a.zero = L.zero;
   a.u_bf16 = cb ? 0 : L.u_bf16;
   a.sf_mn = direct ? 1 : 0;
+  a.codes_ob = cb ? 1 : 0;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
   a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;
@@ -865,7 +869,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
                  "adapter layouts");
-    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, dev, stream));
+    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, !cbw, dev, stream));
     LRQAT_LAUNCH("bwd_prep", 1, stream,
                  launch_bwd_prep(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, nullptr, nullptr, ws.codes,
                                  LRQAT_PHI_QFIXED, ws.phit, stream),
@@ -934,6 +938,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.zero = L.zero;
     a.u_bf16 = cb ? 0 : L.u_bf16;
     a.sf_mn = 0;
+    a.codes_ob = cb && !cbw ? 1 : 0;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;

@@ -259,7 +259,8 @@ __global__ void __launch_bounds__(NUM_THREADS) merge_tc_kernel(const __grid_cons
             tb[e] = __float_as_uint(fminf(fmaxf(tt.x, q.lo), q.hi));
             tb[e + 1] = __float_as_uint(fminf(fmaxf(tt.y, q.lo), q.hi));
           }
-          o[g] = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040u), __byte_perm(tb[2], tb[3], 0x0040u), 0x5410u);
+          o[g] = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040u), __byte_perm(tb[2], tb[3], 0x0040u), 0x5410u) ^
+               args.xor_mask;
         }
         uint4* dst = reinterpret_cast<uint4*>(args.wz + row * args.k + colt + 32 * cc);
         dst[0] = make_uint4(o[0], o[1], o[2], o[3]);

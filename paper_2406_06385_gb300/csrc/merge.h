@@ -27,6 +27,7 @@ struct MergeArgs {
   QuantParams q;         // q.lo / q.hi: the clamp bounds in the magic domain
   int* status;
   uint64_t timeout_ns;
+  uint32_t xor_mask;     // applied to every 4 output bytes: 0x80808080 stores c + 128 (offset-binary)
 };
 // fmt: a PhiFmt value (quant.cuh); u_bf16: the bf16 pre-round value (not with FP16 bases)
 cudaError_t launch_merge_tc(int fmt, int u_bf16, int a_mn, const CUtensorMap& tm_a, const CUtensorMap& tm_b,

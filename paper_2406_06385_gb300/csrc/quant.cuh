@@ -168,6 +168,35 @@ __device__ __forceinline__ uint32_t codes_bf16x2(float2 t, const QuantParams& q)
   return w;
 }
 
+// 16 clipped codes stored offset-binary (byte = c + 128) -> their exact floats.
+__device__ __forceinline__ void decode_ob16(const uint32_t* w, float* v) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+#pragma unroll
+    for (int b = 0; b < 4; ++b) v[4 * i + b] = __uint_as_float(__byte_perm(w[i], 0x4B000000u, 0x7540u + b));
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const float2 d = __fadd2_rn(make_float2(v[2 * e], v[2 * e + 1]), make_float2(-kDecodeOffsetI8, -kDecodeOffsetI8));
+    v[2 * e] = d.x;
+    v[2 * e + 1] = d.y;
+  }
+}
+
+// Two exact small integers -> bf16x2 (the top halves of their floats).
+__device__ __forceinline__ uint32_t pack_int_bf16x2(float c0, float c1) {
+  return __byte_perm(__float_as_uint(c0), __float_as_uint(c1), 0x7632u);
+}
+
+// The same for two stored integer codes (the codes base: already rounded, 0 fraction bits):
+// their floats are exact, so their top halves are their bf16 values.
+__device__ __forceinline__ uint32_t int_codes_bf16x2(float c0, float c1, const QuantParams& q) {
+  uint32_t w = __byte_perm(__float_as_uint(c0), __float_as_uint(c1), 0x7632u);
+  asm("max.bf16x2 %0, %0, %1;" : "+r"(w) : "r"(q.n_bf16x2));
+  asm("min.bf16x2 %0, %0, %1;" : "+r"(w) : "r"(q.p_bf16x2));
+  return w;
+}
+
 // t = round-half-even(u_f / 2^f) in the magic domain, unclipped.
 __device__ __forceinline__ float magic_round(float L, float v, const QuantParams& q) {
   const float u = __fmaf_rn(L, q.lr_scale, v);
