@@ -1107,6 +1107,27 @@ cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int
   return cudaGetLastError();
 }
 
+__global__ void __launch_bounds__(kThreads) dx_scales_kernel(const float* __restrict__ s, const float* __restrict__ z,
+                                                             int64_t m, int groups, int s_ld, uint16_t* __restrict__ s_out,
+                                                             uint16_t* __restrict__ z_out) {
+  const int64_t n = m * groups;
+  for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < n;
+       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t g = e / m, i = e % m;
+    const int64_t src = s_ld ? i * s_ld + g : i;
+    s_out[e] = static_cast<uint16_t>(pack_rn_bf16x2(s[src], 0.0f) & 0xffffu);
+    if (z_out) z_out[e] = static_cast<uint16_t>(pack_rn_bf16x2(z[src], 0.0f) & 0xffffu);
+  }
+}
+
+cudaError_t launch_dx_scales(const float* s, const float* z, int64_t m, int groups, int s_ld, uint16_t* s_out,
+                             uint16_t* z_out, cudaStream_t stream) {
+  const int64_t n = m * groups;
+  const int grid = blocks_for(n, kThreads);
+  dx_scales_kernel<<<grid < 1024 ? grid : 1024, kThreads, 0, stream>>>(s, z, m, groups, s_ld, s_out, z_out);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_reduce(const ReduceArgs& a, cudaStream_t stream) {
   const int64_t nA4 = a.m * a.r / 4, nB4 = static_cast<int64_t>(a.r) * a.k / 4;   // m, k are multiples of 128
   const RedJob ja{reinterpret_cast<const float4*>(a.dA_part), a.nA, nA4, reinterpret_cast<float4*>(a.dA), 0, a.r};

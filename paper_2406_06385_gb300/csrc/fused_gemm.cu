@@ -342,27 +342,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // Scales that multiply the operand (group-wise forward, dX), and the zero offsets
         // subtracted from the codes (asymmetric weights) as bf16 pairs.
         float sc[16];
+        uint32_t scw[8];   // dX: bf16x2 scales
         uint32_t zw[8];
         if (zp) {
           if (MODE == FUSED_DX) {
-            const int i0 = kk * BK + 16 * c;
-            float zv[16];
-            if (args.s_ld == 0) {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const float4 v = __ldg(reinterpret_cast<const float4*>(args.zero + i0) + e);
-                zv[4 * e] = v.x;
-                zv[4 * e + 1] = v.y;
-                zv[4 * e + 2] = v.z;
-                zv[4 * e + 3] = v.w;
-              }
-            } else {
-              const int gcol = row_g / args.group_size;
-#pragma unroll
-              for (int e = 0; e < 16; ++e) zv[e] = __ldg(args.zero + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
-            }
-#pragma unroll
-            for (int e = 0; e < 8; ++e) zw[e] = pack_rn_bf16x2(zv[2 * e], zv[2 * e + 1]);
+            // 16 consecutive bf16 zero offsets of this stage's contraction indices
+            const uint16_t* zp = args.z_bf16 + (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
+                                 kk * BK + 16 * c;
+            const uint4 z0 = __ldg(reinterpret_cast<const uint4*>(zp));
+            const uint4 z1 = __ldg(reinterpret_cast<const uint4*>(zp) + 1);
+            zw[0] = z0.x, zw[1] = z0.y, zw[2] = z0.z, zw[3] = z0.w;
+            zw[4] = z1.x, zw[5] = z1.y, zw[6] = z1.z, zw[7] = z1.w;
           } else {
             const float zr = MODE == FUSED_FWD_GROUP
                                  ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size]
@@ -377,22 +367,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int e = 0; e < 16; ++e) sc[e] = v;
         } else if (MODE == FUSED_DX) {
-          const int i0 = kk * BK + 16 * c;
-          if (args.s_ld == 0) {
-            const float4* sp = reinterpret_cast<const float4*>(args.s + i0);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float4 v = __ldg(sp + e);
-              sc[4 * e] = v.x;
-              sc[4 * e + 1] = v.y;
-              sc[4 * e + 2] = v.z;
-              sc[4 * e + 3] = v.w;
-            }
-          } else {
-            const int gcol = row_g / args.group_size;
-#pragma unroll
-            for (int e = 0; e < 16; ++e) sc[e] = __ldg(args.s + static_cast<int64_t>(i0 + e) * args.s_ld + gcol);
-          }
+          // 16 consecutive bf16 scales of this stage's contraction indices, as bf16x2 words
+          const uint16_t* sp = args.s_bf16 + (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
+                               kk * BK + 16 * c;
+          const uint4 s0 = __ldg(reinterpret_cast<const uint4*>(sp));
+          const uint4 s1 = __ldg(reinterpret_cast<const uint4*>(sp) + 1);
+          scw[0] = s0.x, scw[1] = s0.y, scw[2] = s0.z, scw[3] = s0.w;
+          scw[4] = s1.x, scw[5] = s1.y, scw[6] = s1.z, scw[7] = s1.w;
         }
         // The stored base usually lands well before the low-rank tile: decode it first,
         // keeping the low-rank read -> W_hat chain short.
@@ -445,7 +426,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           } else {
             // bf16(bf16(s) * c): the exact bf16 codes times the bf16-rounded scales,
             // one packed multiply instead of an fp32 clip, multiply and conversion.
-            w[e] = mul_bf16x2(cw, pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
+            w[e] = mul_bf16x2(cw, MODE == FUSED_DX ? scw[e] : pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
           }
         }
         // The W_hat buffer of this token slot was last read by the product of stage gg - 2.

@@ -166,7 +166,15 @@ struct FusedArgs {
   // Codes base (r16 == 0): 1 when the codes are clipped to [n, p] and stored offset-binary
   // (byte = c + 128), so the producers neither flip the sign bit nor clamp; 0: saturated int8.
   int32_t codes_ob;
+  // dX only: the scales (and zero offsets, or nullptr) as bf16 rows along the contraction,
+  // [groups][kdim] (one row per channel scale), written by launch_dx_scales.
+  const uint16_t* s_bf16;
+  const uint16_t* z_bf16;
 };
+// s_out[g][i] = bf16(s[i][g]) (s [m] per channel: g = 0 only) and, with z, z_out likewise: the
+// dX GEMM's producers read 16 consecutive of them per stage with two 16-byte loads.
+cudaError_t launch_dx_scales(const float* s, const float* z, int64_t m, int groups, int s_ld, uint16_t* s_out,
+                             uint16_t* z_out, cudaStream_t stream);
 int fused_smem_bytes(int fmt);
 // The same GEMM on CTA pairs (fused_pair.cu): 256-row x 448-token tiles, npairs clusters of 2.
 // Needs rows % 256 == 0 and K-major factor slices (sf_mn == 0); tm_tok boxes of 112 tokens x

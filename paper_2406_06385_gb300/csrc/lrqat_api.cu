@@ -438,6 +438,8 @@ struct BwdWs {
   float* ds_part;
   int32_t* tile_segs;
   int8_t* codes;       // codes path: the unclipped codes [m, k] (phit then holds their transpose)
+  uint16_t* s_bf16;    // dX: the scales (and zero offsets) as bf16 rows [groups][m]
+  uint16_t* z_bf16;
 };
 
 size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* base, BwdWs* ws) {
@@ -462,6 +464,9 @@ size_t bwd_ws_layout(const lrqat_layer& L, int64_t T, const DwPlan& p, void* bas
   w.dB_part = static_cast<float*>(c.take(static_cast<size_t>(p.ni128) * p.nsplit * L.r * L.k * 4));
   w.ds_part = static_cast<float*>(c.take(static_cast<size_t>(2) * p.nsplit * L.m * (L.k / 128) * 4));
   w.tile_segs = static_cast<int32_t*>(c.take(static_cast<size_t>(p.ni128) * p.nj * 4));
+  const size_t groups = L.group_size ? static_cast<size_t>(L.k / L.group_size) : 1;
+  w.s_bf16 = static_cast<uint16_t*>(c.take(groups * L.m * 2));
+  if (L.zero) w.z_bf16 = static_cast<uint16_t*>(c.take(groups * L.m * 2));
   if (ws) *ws = w;
   return (c.used + 255) & ~size_t(255);
 }
@@ -901,6 +906,10 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
 
   // dX = dY W_hat (W_hat^T produced on chip from Phi0^T, B^T and A).
   {
+    const int groups = L.group_size ? static_cast<int>(L.k / L.group_size) : 1;
+    LRQAT_LAUNCH("dx_scales", 1, stream,
+                 launch_dx_scales(s, L.zero, L.m, groups, L.group_size ? groups : 0, ws.s_bf16, ws.z_bf16, stream),
+                 "dX scale rows");
     const bool pair = use_pair(L.k, L.group_size != 0);
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
     LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, pair ? 112 : 224,
@@ -939,6 +948,8 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.u_bf16 = cb ? 0 : L.u_bf16;
     a.sf_mn = 0;
     a.codes_ob = cb && !cbw ? 1 : 0;
+    a.s_bf16 = ws.s_bf16;
+    a.z_bf16 = ws.z_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
     a.group_size = L.group_size;
     a.s_x = nullptr;
