@@ -311,14 +311,14 @@ int lrqat_adamw_step(const lrqat_layer* layer, const lrqat_adamw* opt, const flo
  * values. */
 int lrqat_set_dw_schedule(int schedule);
 
-/* Tuning (no counterpart in the paper): the kernel of the forward and dX GEMMs.
+/* Tuning (no counterpart in the paper): the kernels of the forward, dX and dW GEMMs.
  * CTA pairs run tcgen05 MMAs of 256 rows across the two SMs of a cluster, each SM holding
  * half of the token operand (256 weight rows x 448 tokens per pair); they need a multiple
- * of 256 produced rows (m for the forward, k for dX).  The one-SM kernel takes 128 rows x
- * 448 tokens per SM.  0 (the default) = pairs wherever they were measured faster: every
- * GEMM whose rows allow, except dX with group-wise scales; 1 = the one-SM kernel always;
- * 2 = pairs wherever the rows allow.  All give the same codes; outputs agree up to fp32
- * summation order.  Process-wide; the environment variable LRQAT_GEMM_VARIANT ("auto",
+ * of 256 produced rows (m for the forward, k for dX; dW: ranks up to 64 and m, k multiples
+ * of 256, on 256 x 256 tiles).  The one-SM kernels take 128 rows per SM.  0 (the default) =
+ * pairs wherever they were measured faster, which is wherever the shapes allow; 1 = the
+ * one-SM kernels always; 2 = pairs wherever the shapes allow.  All give the same codes;
+ * outputs agree up to fp32 summation order.  Process-wide; the environment variable LRQAT_GEMM_VARIANT ("auto",
  * "single" or "pair") gives the start value, read once when the library is loaded.
  * Returns LRQAT_ERR_INVALID_ARG for other values. */
 int lrqat_set_gemm_variant(int variant);

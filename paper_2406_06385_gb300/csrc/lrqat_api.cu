@@ -303,9 +303,9 @@ int dw_schedule_from_env() {
 std::atomic<int> g_dw_schedule{dw_schedule_from_env()};
 
 // Kernel of the forward and dX GEMMs (lrqat_set_gemm_variant): 0 = CTA pairs (fused_pair.cu)
-// wherever they were measured faster: every GEMM whose produced weight operand has a multiple of
-// 256 rows, except dX with group-wise scales (its producers load a scale per element, which the
-// pair's per-SM share of the stage cannot absorb); 1 = the one-SM kernel (fused_gemm.cu) always;
+// wherever they were measured faster, which is every GEMM whose produced weight operand has a
+// multiple of 256 rows (with the dX scales read as bf16 rows, group-wise dX too: 916 -> 730 us on
+// the 14336 x 4096 g128 projection at T = 8192); 1 = the one-SM kernel (fused_gemm.cu) always;
 // 2 = pairs wherever the rows allow.  LRQAT_GEMM_VARIANT ("auto" / "single" / "pair") sets the
 // start value once, when the library is loaded.
 int gemm_variant_from_env() {
@@ -315,9 +315,9 @@ int gemm_variant_from_env() {
   return 0;
 }
 std::atomic<int> g_gemm_variant{gemm_variant_from_env()};
-bool use_pair(int64_t rows, bool group_dx) {
+bool use_pair(int64_t rows) {
   const int v = g_gemm_variant.load(std::memory_order_relaxed);
-  return rows % 256 == 0 && (v == 2 || (v == 0 && !group_dx));
+  return rows % 256 == 0 && v != 1;
 }
 constexpr int kPairTokens = 448;   // tokens per pair tile (two accumulators of 224)
 
@@ -699,7 +699,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   fwd_ws_layout(L, T, allow_codes, workspace, &ws);
   const int r16 = round16(L.r);
   const bool cb = L.r > 64 || (allow_codes && codes_gemm(L, T));
-  const bool pair = use_pair(L.m, false);
+  const bool pair = use_pair(L.m);
   // the pair kernel reads K-major factor slices, so it takes B^T from the padded copy
   const bool direct = !cb && !pair && direct_factors(L, A, B);
   if (cb) {
@@ -910,7 +910,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_LAUNCH("dx_scales", 1, stream,
                  launch_dx_scales(s, L.zero, L.m, groups, L.group_size ? groups : 0, ws.s_bf16, ws.z_bf16, stream),
                  "dX scale rows");
-    const bool pair = use_pair(L.k, L.group_size != 0);
+    const bool pair = use_pair(L.k);
     CUtensorMap tm_tok, tm_phi, tm_rf, tm_sf;
     LRQAT_TRY(encode_2d(&tm_tok, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, dY, L.m, T, L.m * 2, 64, pair ? 112 : 224,
                         CU_TENSOR_MAP_SWIZZLE_128B, "dY"));

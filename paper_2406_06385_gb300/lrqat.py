@@ -234,9 +234,9 @@ GEMM_VARIANTS = {"auto": 0, "single": 1, "pair": 2}
 
 
 def set_gemm_variant(variant: str) -> None:
-    """Process-wide kernel of the forward and dX GEMMs: "auto" (CTA pairs where they were
+    """Process-wide kernels of the forward, dX and dW GEMMs: "auto" (CTA pairs where they were
     measured faster, the default), "single" (one SM per tile) or "pair" (CTA pairs wherever
-    the rows allow)."""
+    the shapes allow)."""
     _check(lib().lrqat_set_gemm_variant(GEMM_VARIANTS[variant]))
 
 
