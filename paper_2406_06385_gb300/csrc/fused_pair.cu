@@ -401,8 +401,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
           raw[0] = r.x, raw[1] = r.y, raw[2] = r.z, raw[3] = r.w;
         }
-        if (NL && args.codes_ob) decode_ob16(raw, v);
-        else decode16<FMT>(raw, v);
+        // the codes base with the clipped codes stored as c + 64: bf16 straight from the bytes
+        const bool b64 = NL && args.codes_bias == 64;
+        uint32_t c8[8];
+        if (b64) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) decode_b64_bf16x4(raw[i], c8[2 * i], c8[2 * i + 1]);
+        } else if (NL && args.codes_bias == 128) {
+          decode_ob16(raw, v);
+        } else {
+          decode16<FMT>(raw, v);
+        }
         float Lv[16];
         if (!NL) {
           const uint32_t lb = gg % NLB;
@@ -418,13 +427,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t w[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float2 u =
-              NL   ? make_float2(v[2 * e], v[2 * e + 1])
-              : UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
-                   : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]), make_float2(qp.lr_scale, qp.lr_scale),
-                                make_float2(v[2 * e], v[2 * e + 1]));
-          uint32_t cw = NL ? (args.codes_ob ? pack_int_bf16x2(u.x, u.y) : int_codes_bf16x2(u.x, u.y, qp))
-                           : codes_bf16x2(__fadd2_rn(u, make_float2(qp.magic, qp.magic)), qp);
+          uint32_t cw;
+          if (NL) {
+            cw = b64                         ? c8[e]
+                 : args.codes_bias == 128    ? pack_int_bf16x2(v[2 * e], v[2 * e + 1])
+                                             : int_codes_bf16x2(v[2 * e], v[2 * e + 1], qp);
+          } else {
+            const float2 u = UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
+                                : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]),
+                                             make_float2(qp.lr_scale, qp.lr_scale), make_float2(v[2 * e], v[2 * e + 1]));
+            cw = codes_bf16x2(__fadd2_rn(u, make_float2(qp.magic, qp.magic)), qp);
+          }
           if (ZP) cw = sub_bf16x2(cw, zw[e]);
           if (MODE == FUSED_FWD_PC) {
             w[e] = cw;

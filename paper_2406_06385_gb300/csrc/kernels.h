@@ -163,9 +163,9 @@ struct FusedArgs {
   // Forward only: the second factor's slice read straight from B as one MN-major box
   // of 64 columns x r16 rank rows (no padded B^T copy).
   int32_t sf_mn;
-  // Codes base (r16 == 0): 1 when the codes are clipped to [n, p] and stored offset-binary
-  // (byte = c + 128), so the producers neither flip the sign bit nor clamp; 0: saturated int8.
-  int32_t codes_ob;
+  // Codes base (r16 == 0): 0: saturated int8 codes (the producers clamp them); 64 or 128: the
+  // codes clipped to [n, p] and stored as the unsigned byte c + 64 (b <= 7) or c + 128 (b = 8).
+  int32_t codes_bias;
   // dX only: the scales (and zero offsets, or nullptr) as bf16 rows along the contraction,
   // [groups][kdim] (one row per channel scale), written by launch_dx_scales.
   const uint16_t* s_bf16;

@@ -488,6 +488,11 @@ int phi_map(CUtensorMap* map, const lrqat_layer& L, const void* phi0, uint32_t b
 
 // Quantizer constants of the codes written for ranks above 64: the clamp bounds are the int8
 // range instead of [n, p] (the GEMMs clip and mask from the unclipped code).
+// The bias of the clipped codes the GEMMs read (merge.h, FusedArgs::codes_bias): c + 64 fits a
+// byte's low seven bits for b <= 7 (the GEMM producers then turn four codes into bf16 with two
+// byte permutes and two bf16 subtractions), c + 128 for b = 8.
+uint32_t codes_bias(const lrqat_layer& L) { return L.bits <= 7 ? 64u : 128u; }
+
 QuantParams saturating_params(const lrqat_layer& L) {
   QuantParams q = make_quant_params(L.bits, frac_bits(L), L.alpha, L.r);
   const QuantParams wide = make_quant_params(8, frac_bits(L), L.alpha, L.r);
@@ -557,7 +562,7 @@ int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, c
   a.k = L.k;
   a.r16 = r16;
   a.q = clipped ? make_quant_params(L.bits, frac_bits(L), L.alpha, L.r) : saturating_params(L);
-  a.xor_mask = clipped ? 0x80808080u : 0u;
+  a.code_bias = clipped ? codes_bias(L) : 0u;
   a.status = dev->status;
   a.timeout_ns = kWaitTimeoutNs;
   LRQAT_LAUNCH("lowrank_codes", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 1, tm_a, tm_b, tm_phi, a, stream),
@@ -764,7 +769,7 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   a.zero = L.zero;
   a.u_bf16 = cb ? 0 : L.u_bf16;
   a.sf_mn = direct ? 1 : 0;
-  a.codes_ob = cb ? 1 : 0;
+  a.codes_bias = cb ? static_cast<int32_t>(codes_bias(L)) : 0;
   a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
   a.group_size = L.group_size;
   a.s_x = L.act_bits == 8 && !L.act_per_token ? s_x : nullptr;
@@ -947,7 +952,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.zero = L.zero;
     a.u_bf16 = cb ? 0 : L.u_bf16;
     a.sf_mn = 0;
-    a.codes_ob = cb && !cbw ? 1 : 0;
+    a.codes_bias = cb && !cbw ? static_cast<int32_t>(codes_bias(L)) : 0;
     a.s_bf16 = ws.s_bf16;
     a.z_bf16 = ws.z_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;

@@ -240,7 +240,7 @@ __global__ void __launch_bounds__(NUM_THREADS) merge_tc_kernel(const __grid_cons
         }
         // t = u + magic rounds u half to even in units of 2^f; clamped to [lo, hi] its bit
         // pattern is the bits of magic (low byte zero) plus the integer code, so the code's
-        // int8 two's complement is t's low byte.
+        // int8 two's complement is t's low byte (code_bias added: the biased code's byte).
         uint32_t o[8];
 #pragma unroll
         for (int g = 0; g < 8; ++g) {
@@ -256,11 +256,10 @@ __global__ void __launch_bounds__(NUM_THREADS) merge_tc_kernel(const __grid_cons
                                           make_float2(v[j], v[j + 1]));
               tt = __fadd2_rn(u, make_float2(q.magic, q.magic));
             }
-            tb[e] = __float_as_uint(fminf(fmaxf(tt.x, q.lo), q.hi));
-            tb[e + 1] = __float_as_uint(fminf(fmaxf(tt.y, q.lo), q.hi));
+            tb[e] = __float_as_uint(fminf(fmaxf(tt.x, q.lo), q.hi)) + args.code_bias;
+            tb[e + 1] = __float_as_uint(fminf(fmaxf(tt.y, q.lo), q.hi)) + args.code_bias;
           }
-          o[g] = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040u), __byte_perm(tb[2], tb[3], 0x0040u), 0x5410u) ^
-               args.xor_mask;
+          o[g] = __byte_perm(__byte_perm(tb[0], tb[1], 0x0040u), __byte_perm(tb[2], tb[3], 0x0040u), 0x5410u);
         }
         uint4* dst = reinterpret_cast<uint4*>(args.wz + row * args.k + colt + 32 * cc);
         dst[0] = make_uint4(o[0], o[1], o[2], o[3]);

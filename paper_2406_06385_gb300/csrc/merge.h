@@ -27,7 +27,7 @@ struct MergeArgs {
   QuantParams q;         // q.lo / q.hi: the clamp bounds in the magic domain
   int* status;
   uint64_t timeout_ns;
-  uint32_t xor_mask;     // applied to every 4 output bytes: 0x80808080 stores c + 128 (offset-binary)
+  uint32_t code_bias;    // added to every stored code: 0 (two's complement), 64 or 128 (c + bias, unsigned)
 };
 // fmt: a PhiFmt value (quant.cuh); u_bf16: the bf16 pre-round value (not with FP16 bases)
 cudaError_t launch_merge_tc(int fmt, int u_bf16, int a_mn, const CUtensorMap& tm_a, const CUtensorMap& tm_b,

@@ -183,6 +183,11 @@ __device__ __forceinline__ void decode_ob16(const uint32_t* w, float* v) {
   }
 }
 
+// Four clipped codes stored as bytes c + 64 (|c| <= 64) -> two bf16x2 words: the byte becomes
+// the mantissa of bf16(128 + byte) = 0x43 : byte, and one exact bf16x2 subtraction of 192
+// leaves c.  w01 holds codes 0 and 1, w23 codes 2 and 3.
+__device__ __forceinline__ void decode_b64_bf16x4(uint32_t w, uint32_t& w01, uint32_t& w23);
+
 // Two exact small integers -> bf16x2 (the top halves of their floats).
 __device__ __forceinline__ uint32_t pack_int_bf16x2(float c0, float c1) {
   return __byte_perm(__float_as_uint(c0), __float_as_uint(c1), 0x7632u);
@@ -265,6 +270,11 @@ __device__ __forceinline__ uint32_t sub_bf16x2(uint32_t a, uint32_t b) {
   uint32_t r;
   asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
   return r;
+}
+
+__device__ __forceinline__ void decode_b64_bf16x4(uint32_t w, uint32_t& w01, uint32_t& w23) {
+  w01 = sub_bf16x2(__byte_perm(w, 0x43u, 0x4140u), 0x43404340u);
+  w23 = sub_bf16x2(__byte_perm(w, 0x43u, 0x4342u), 0x43404340u);
 }
 
 // Elementwise bf16x2 product, rounded to nearest even.
