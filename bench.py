@@ -38,7 +38,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 GEMM_KERNELS = ("fused_fwd", "fused_dx", "fused_dw")
 # the sources whose kernels a traced name can refer to (the forward and dX run on CTA pairs or on one SM)
 KERNEL_SOURCES = {"fused_fwd": ("fused_gemm.cu", "fused_pair.cu"), "fused_dx": ("fused_gemm.cu", "fused_pair.cu"),
-                  "fused_dw": ("dw.cu",)}
+                  "fused_dw": ("dw.cu", "dw_pair.cu")}
 
 
 # --------------------------------------------------------------------------- helpers
@@ -192,6 +192,23 @@ def barrier():
     import torch.distributed as dist
     if dist.is_available() and dist.is_initialized():
         dist.barrier()
+
+
+def workload_config(wl, args, world: int) -> dict:
+    """The `config` object of the JSON line: the workload by name, its layer shapes and
+    quantizer settings, and how the timed region launches and rotates its inputs.  Both
+    arms print the same object for the same arguments."""
+    spec0 = wl.layers[0]
+    in_bytes = args.sets * sum(2 * wl.tokens * (l.k + l.m) for l in wl.layers)
+    return {"workload": wl.name, "tokens": wl.tokens, "layers": [f"{l.name}:{l.m}x{l.k}" for l in wl.layers],
+            "r": spec0.r, "alpha": spec0.alpha, "bits": spec0.bits,
+            "granularity": "per-channel" if spec0.group_size == 0 else f"g{spec0.group_size}",
+            "phi": phi_label(spec0.phi_format, spec0.bits),
+            "activations": ("int8 per-token" if spec0.act_per_token else "int8 per-tensor") if spec0.act_bits == 8
+            else "bf16",
+            "merge": wl.merge, "parallelism": "replicas" if world > 1 else "single",
+            "launch": "eager library calls" if args.no_graph else "CUDA graph replay of each step's library calls",
+            "l2": f"inputs rotate over {args.sets} device copies ({in_bytes / 2**20:.0f} MiB) > L2"}
 
 
 # --------------------------------------------------------------------------- GPU arm
@@ -457,16 +474,7 @@ def run_gpu(args):
     # sustained peak (a seconds-long GEMM loop under the power cap) is.
     kind = peak_kind(clk)
     peak = peaks["bf16_tflops" if kind == "burst" else "bf16_tflops_sustained"]
-    spec0 = wl.layers[0]
-    cfg = {"workload": wl.name, "tokens": T, "layers": [f"{l.name}:{l.m}x{l.k}" for l in wl.layers],
-           "r": spec0.r, "alpha": spec0.alpha, "bits": spec0.bits,
-           "granularity": "per-channel" if spec0.group_size == 0 else f"g{spec0.group_size}",
-           "phi": phi_label(spec0.phi_format, spec0.bits),
-           "activations": ("int8 per-token" if spec0.act_per_token else "int8 per-tensor") if spec0.act_bits == 8
-           else "bf16",
-           "merge": wl.merge, "parallelism": "replicas" if world > 1 else "single",
-           "launch": "eager library calls" if args.no_graph else "CUDA graph replay of each step's library calls",
-           "l2": f"inputs rotate over {args.sets} device copies ({args.sets * sum((l['X'][0].numel() + l['dY'][0].numel()) * 2 for l in gw.layers) / 2**20:.0f} MiB) > L2"}
+    cfg = workload_config(wl, args, world)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -713,7 +721,7 @@ def run_reference(args):
     return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name, "tokens": wl.tokens}, "impl": "reference",
+            "config": workload_config(wl, args, world), "impl": "reference",
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}

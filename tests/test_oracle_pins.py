@@ -5,6 +5,8 @@ hand-worked example, a special case with a known answer, an exhaustive
 enumeration, an exact finite difference, or a library autograd of a closed form.
 """
 import itertools
+import json
+import os
 
 import numpy as np
 import pytest
@@ -14,52 +16,47 @@ from paper_2406_06385_gb300 import workloads as WL
 
 
 # ---------------------------------------------------------------------------
-# Hand-worked example, Eq. 7 (phi = Q4.4) and Eq. 8, b = 4, r = 1, alpha = 1.
-# Every number below is a dyadic rational worked out by hand:
-#   x = W0 / s0 : row 0 [7, -3.5, 1.25, 0.3125], row 1 [-7, 3.75, 0.125, 6.5]
-#   Phi0 = 16 x : row 0 [112, -56, 20, 5],      row 1 [-112, 60, 2, 104]
-#   A B         : row 0 [0.75, 0.5, -0.25, 0.1875], row 1 [-0.375, -0.25, 0.125, -0.09375]
-#   u = Phi0/16 + A B : row 0 [7.75, -3.0, 1.0, 0.5], row 1 [-7.375, 3.5, 0.25, 6.40625]
-#   q = round-half-even(u) : row 0 [8, -3, 1, 0], row 1 [-7, 4, 0, 6]
-#   c = clip(q, -8, 7) : row 0 [7, -3, 1, 0], row 1 [-7, 4, 0, 6];  mask row 0 [0, 1, 1, 1]
+# Hand-worked example, Eq. 7 (phi = Q4.4) and Eq. 8, b = 4, r = 1, alpha = 1: the inputs
+# and every intermediate value (dyadic rationals worked out by hand) are in
+# tests/golden/hand_example_q44.json.
 # ---------------------------------------------------------------------------
-HAND_LAYER = O.Layer(m=2, k=4, r=1, alpha=1.0, bits=4)
-HAND_W0 = np.array([[0.875, -0.4375, 0.15625, 0.0390625],
-                    [-1.75, 0.9375, 0.03125, 1.625]], dtype=np.float32)
-HAND_A = np.array([[0.5], [-0.25]])
-HAND_B = np.array([[1.5, 1.0, -0.5, 0.375]])
-HAND_S = np.array([0.25, 0.5])            # trained scale, differs from s0 on purpose
-HAND_X = np.array([[1.0, 2.0, -1.0, 0.5], [0.0, -1.0, 2.0, 1.0]])
-HAND_DY = np.array([[1.0, -1.0], [0.5, 2.0]])
+with open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "hand_example_q44.json")) as _f:
+    HAND = json.load(_f)
+_HL = HAND["layer"]
+HAND_LAYER = O.Layer(m=_HL["m"], k=_HL["k"], r=_HL["r"], alpha=_HL["alpha"], bits=_HL["bits"])
+HAND_W0 = np.array(HAND["inputs"]["W0"], dtype=np.float32)
+HAND_A = np.array(HAND["inputs"]["A"])
+HAND_B = np.array(HAND["inputs"]["B"])
+HAND_S = np.array(HAND["inputs"]["s"])            # trained scale, differs from s0 on purpose
+HAND_X = np.array(HAND["inputs"]["X"])
+HAND_DY = np.array(HAND["inputs"]["dY"])
+HAND_STEP = HAND["steps"]
 
 
 def test_hand_example_downcast_and_codes():
     s0 = O.minmax_scale(HAND_W0, HAND_LAYER)
-    np.testing.assert_array_equal(s0, np.array([0.125, 0.25], dtype=np.float32))
+    np.testing.assert_array_equal(s0, np.array(HAND_STEP["s0 = max|W0 row| / 7"], dtype=np.float32))
     phi0 = O.downcast(HAND_W0, s0, HAND_LAYER)
-    np.testing.assert_array_equal(phi0, [[112, -56, 20, 5], [-112, 60, 2, 104]])
+    np.testing.assert_array_equal(phi0, HAND_STEP["Phi0 = 16 x"])
     fq = O.fake_quant_weight(phi0, HAND_S, HAND_A, HAND_B, HAND_LAYER)
-    np.testing.assert_array_equal(fq["u"], [[7.75, -3.0, 1.0, 0.5], [-7.375, 3.5, 0.25, 6.40625]])
-    np.testing.assert_array_equal(fq["q"], [[8, -3, 1, 0], [-7, 4, 0, 6]])
-    np.testing.assert_array_equal(fq["c"], [[7, -3, 1, 0], [-7, 4, 0, 6]])
-    np.testing.assert_array_equal(fq["M"], [[0, 1, 1, 1], [1, 1, 1, 1]])
-    np.testing.assert_array_equal(fq["W_hat"], [[1.75, -0.75, 0.25, 0.0], [-3.5, 2.0, 0.0, 3.0]])
-    np.testing.assert_array_equal(O.merge(phi0, HAND_A, HAND_B, HAND_LAYER), [[7, -3, 1, 0], [-7, 4, 0, 6]])
+    np.testing.assert_array_equal(fq["u"], HAND_STEP["u = Phi0/16 + (alpha/r) A B"])
+    np.testing.assert_array_equal(fq["q"], HAND_STEP["q = round_half_even(u)"])
+    np.testing.assert_array_equal(fq["c"], HAND_STEP["c = clip(q, -8, 7)"])
+    np.testing.assert_array_equal(fq["M"], HAND_STEP["M = [n <= q <= p]"])
+    np.testing.assert_array_equal(fq["W_hat"], HAND_STEP["W_hat = s c"])
+    np.testing.assert_array_equal(O.merge(phi0, HAND_A, HAND_B, HAND_LAYER), HAND_STEP["c = clip(q, -8, 7)"])
 
 
 def test_hand_example_forward_backward():
-    # Y = X W_hat^T; dX = dY W_hat; G = dY^T X; dU = G s M; dA = dU B^T; dB = A^T dU; ds = sum G c
-    #   G row 0 = [1, 1.5, 0, 1], row 1 = [-1, -4, 5, 1.5]
-    #   dU row 0 = 0.25 * G0 * [0,1,1,1] = [0, 0.375, 0, 0.25]; dU row 1 = 0.5 * G1 = [-0.5, -2, 2.5, 0.75]
-    phi0 = np.array([[112, -56, 20, 5], [-112, 60, 2, 104]], dtype=np.int8)
+    phi0 = np.array(HAND_STEP["Phi0 = 16 x"], dtype=np.int8)
     Y = O.linear_fwd(HAND_X, phi0, HAND_S, HAND_A, HAND_B, HAND_LAYER)
-    np.testing.assert_array_equal(Y, [[0.0, 2.0], [1.25, 1.0]])
+    np.testing.assert_array_equal(Y, HAND_STEP["Y = X W_hat^T"])
     g = O.linear_bwd(HAND_DY, HAND_X, phi0, HAND_S, HAND_A, HAND_B, HAND_LAYER)
-    np.testing.assert_array_equal(g["dX"], [[5.25, -2.75, 0.25, -3.0], [-6.125, 3.625, 0.125, 6.0]])
-    np.testing.assert_array_equal(g["G"], [[1.0, 1.5, 0.0, 1.0], [-1.0, -4.0, 5.0, 1.5]])
-    np.testing.assert_array_equal(g["dA"], [[0.46875], [-3.71875]])
-    np.testing.assert_array_equal(g["dB"], [[0.125, 0.6875, -0.625, -0.0625]])
-    np.testing.assert_array_equal(g["ds"], [2.5, 0.0])
+    np.testing.assert_array_equal(g["dX"], HAND_STEP["dX = dY W_hat"])
+    np.testing.assert_array_equal(g["G"], HAND_STEP["G = dY^T X"])
+    np.testing.assert_array_equal(g["dA"], HAND_STEP["dA = (alpha/r) dU B^T"])
+    np.testing.assert_array_equal(g["dB"], HAND_STEP["dB = (alpha/r) A^T dU"])
+    np.testing.assert_array_equal(g["ds"], HAND_STEP["ds = sum_k G c"])
 
 
 def test_hand_example_alpha_over_r_half():
