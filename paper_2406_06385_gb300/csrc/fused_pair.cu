@@ -93,10 +93,11 @@ constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t COL_L = NACC * BNP;           // the 64-column low-rank buffer(s) after the accumulators
 static_assert(COL_L + NLB * BK <= TMEM_COLS, "TMEM budget");
 
-constexpr int BAR_TFULL = 0;                     // leader: both token halves of the slot landed
+// leader: the stage's operands are in place, i.e. both token halves of the slot landed and both
+// CTAs' producers wrote their W_hat tiles (one barrier, so that the MMA thread tests one per stage)
+constexpr int BAR_TFULL = 0;
 constexpr int BAR_TEMPTY = BAR_TFULL + NT_MAX;   // both: main product of the slot finished
-constexpr int BAR_WFULL = BAR_TEMPTY + NT_MAX;   // leader: both W_hat tiles of the slot written
-constexpr int BAR_PFULL = BAR_WFULL + NT_MAX;    // both: this CTA's base tile landed
+constexpr int BAR_PFULL = BAR_TEMPTY + NT_MAX;   // both: this CTA's base tile landed
 
 constexpr int BAR_FFULL = BAR_PFULL + NF_MAX;    // leader: both factor-slice halves landed
 constexpr int BAR_FEMPTY = BAR_FFULL + NF_MAX;   // both: slot read by this CTA's producers (after L)
@@ -147,9 +148,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0) {
     abort_s = 0;
     for (int s = 0; s < NT; ++s) {
-      mbar_init(bar(BAR_TFULL + s), 1);
+      mbar_init(bar(BAR_TFULL + s), 1 + NUM_PROD_WARPS);   // the leader's token loader and producer warps
       mbar_init(bar(BAR_TEMPTY + s), 1);
-      mbar_init(bar(BAR_WFULL + s), NUM_PROD_WARPS);
     }
     for (int s = 0; s < NF; ++s) {
       mbar_init(bar(BAR_PFULL + s), 1);
@@ -301,10 +301,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
         if (!(ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 7))) break;
         tc_fence_after();
+        // unrolled: the loop's own overhead between two stages' MMAs was ~120 cycles of idle tensor pipe
+#pragma unroll 4
         for (int kk = 0; kk < nk; ++kk) {
           const uint32_t gg = g + kk;
           const uint32_t s = gg % NT, ph = (gg / NT) & 1u;
-          if (!(ok = wait_spin_bounded(bar(BAR_WFULL + s), ph, ctl, 8))) break;
           if (!(ok = wait_spin_bounded(bar(BAR_TFULL + s), ph, ctl, 9))) break;
           tc_fence_after();
           const uint64_t w = d_w0 + s * TSLOT_D, t = d_tok0 + s * TSLOT_D;
@@ -455,7 +456,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          report(BAR_WFULL + ts, pw);
+          report(BAR_TFULL + ts, pw);
           mbar_arrive(bar(BAR_FEMPTY + fslot));
         }
       }
