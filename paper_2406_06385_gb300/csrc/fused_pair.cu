@@ -340,6 +340,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const QuantParams qp = args.q;
     const uint32_t lr2 = pack_rn_bf16x2(qp.lr_scale, qp.lr_scale);
+    // On the codes each warp builds two stages per iteration: both bases are read before either is
+    // decoded and one proxy fence covers both W_hat stores, so that the per-stage chain of
+    // shared-memory round trips (base read, W_hat store, fence, reports) is paid once per two
+    // stages (kdim is a multiple of 128, so nk is even).
+    constexpr int SPI = NL ? 2 : 1;
     uint32_t g = 0;
     uint32_t it = 0;
     bool ok = true;
@@ -347,117 +352,139 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int rb2 = tile % num_rb2;
       const int tb = tile / num_rb2;
       const int row_g = rb2 * 2 * BM + static_cast<int>(rank) * BM + row;
-      for (int kk = 0; kk < nk; ++kk) {
-        const uint32_t gg = g + kk;
-        float sc[16];
-        uint32_t scw[8];   // dX: bf16x2 scales
-        uint32_t zw[8];
-        if (ZP) {
-          if (MODE == FUSED_DX) {
-            // 16 consecutive bf16 zero offsets of this stage's contraction indices
-            const uint16_t* zp = args.z_bf16 + (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
-                                 kk * BK + 16 * c;
-            const uint4 z0 = __ldg(reinterpret_cast<const uint4*>(zp));
-            const uint4 z1 = __ldg(reinterpret_cast<const uint4*>(zp) + 1);
-            zw[0] = z0.x, zw[1] = z0.y, zw[2] = z0.z, zw[3] = z0.w;
-            zw[4] = z1.x, zw[5] = z1.y, zw[6] = z1.z, zw[7] = z1.w;
-          } else {
-            const float zr = MODE == FUSED_FWD_GROUP
-                                 ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size]
-                                 : args.zero[row_g];
-            const uint32_t z2 = pack_rn_bf16x2(zr, zr);
+      for (int kk = 0; kk < nk; kk += SPI) {
+        uint32_t scw[SPI][8];   // dX: the stage's 16 bf16 scales of its contraction indices, as bf16x2
+        uint32_t zw[SPI][8];    // zero offsets as bf16x2
+        uint32_t sgw[SPI];      // group-wise forward: the stage's scale as bf16x2
 #pragma unroll
-            for (int e = 0; e < 8; ++e) zw[e] = z2;
+        for (int j = 0; j < SPI; ++j) {
+          const int kj = kk + j;
+          if (ZP) {
+            if (MODE == FUSED_DX) {
+              // 16 consecutive bf16 zero offsets of this stage's contraction indices
+              const uint16_t* zp = args.z_bf16 +
+                                   (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
+                                   kj * BK + 16 * c;
+              const uint4 z0 = __ldg(reinterpret_cast<const uint4*>(zp));
+              const uint4 z1 = __ldg(reinterpret_cast<const uint4*>(zp) + 1);
+              zw[j][0] = z0.x, zw[j][1] = z0.y, zw[j][2] = z0.z, zw[j][3] = z0.w;
+              zw[j][4] = z1.x, zw[j][5] = z1.y, zw[j][6] = z1.z, zw[j][7] = z1.w;
+            } else {
+              const float zr = MODE == FUSED_FWD_GROUP
+                                   ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kj * BK) / args.group_size]
+                                   : args.zero[row_g];
+              const uint32_t z2 = pack_rn_bf16x2(zr, zr);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) zw[j][e] = z2;
+            }
+          }
+          if (MODE == FUSED_FWD_GROUP) {
+            const float v = args.s[static_cast<int64_t>(row_g) * args.s_ld + (kj * BK) / args.group_size];
+            sgw[j] = pack_rn_bf16x2(v, v);
+          } else if (MODE == FUSED_DX) {
+            const uint16_t* sp = args.s_bf16 +
+                                 (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
+                                 kj * BK + 16 * c;
+            const uint4 s0 = __ldg(reinterpret_cast<const uint4*>(sp));
+            const uint4 s1 = __ldg(reinterpret_cast<const uint4*>(sp) + 1);
+            scw[j][0] = s0.x, scw[j][1] = s0.y, scw[j][2] = s0.z, scw[j][3] = s0.w;
+            scw[j][4] = s1.x, scw[j][5] = s1.y, scw[j][6] = s1.z, scw[j][7] = s1.w;
           }
         }
-        if (MODE == FUSED_FWD_GROUP) {
-          const float v = args.s[static_cast<int64_t>(row_g) * args.s_ld + (kk * BK) / args.group_size];
+        // the stages' stored bases, each read as soon as it has landed
+        uint32_t raw[SPI][8];
 #pragma unroll
-          for (int e = 0; e < 16; ++e) sc[e] = v;
-        } else if (MODE == FUSED_DX) {
-          // 16 consecutive bf16 scales of this stage's contraction indices, as bf16x2 words
-          const uint16_t* sp = args.s_bf16 + (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
-                               kk * BK + 16 * c;
-          const uint4 s0 = __ldg(reinterpret_cast<const uint4*>(sp));
-          const uint4 s1 = __ldg(reinterpret_cast<const uint4*>(sp) + 1);
-          scw[0] = s0.x, scw[1] = s0.y, scw[2] = s0.z, scw[3] = s0.w;
-          scw[4] = s1.x, scw[5] = s1.y, scw[6] = s1.z, scw[7] = s1.w;
-        }
-        const uint32_t fslot = gg % NF;
-        ok = wait_bounded(bar(BAR_PFULL + fslot), (gg / NF) & 1u, ctl, 12);
-        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-        const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
-        float v[16];
-        uint32_t raw[8];
-        if (PACKED) {
-          const uint2 r = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
-          raw[0] = r.x;
-          raw[1] = r.y;
-        } else if (fmt_16bit(FMT)) {
-          const uint4 r0 = ld_shared_v4(fs + swz_offset(row, 2 * c, 128));
-          const uint4 r1 = ld_shared_v4(fs + swz_offset(row, 2 * c + 1, 128));
-          raw[0] = r0.x, raw[1] = r0.y, raw[2] = r0.z, raw[3] = r0.w;
-          raw[4] = r1.x, raw[5] = r1.y, raw[6] = r1.z, raw[7] = r1.w;
-        } else {
-          const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
-          raw[0] = r.x, raw[1] = r.y, raw[2] = r.z, raw[3] = r.w;
-        }
-        // the codes base with the clipped codes stored as c + 64: bf16 straight from the bytes
-        const bool b64 = NL && args.codes_bias == 64;
-        uint32_t c8[8];
-        if (b64) {
-#pragma unroll
-          for (int i = 0; i < 4; ++i) decode_b64_bf16x4(raw[i], c8[2 * i], c8[2 * i + 1]);
-        } else if (NL && args.codes_bias == 128) {
-          decode_ob16(raw, v);
-        } else {
-          decode16<FMT>(raw, v);
-        }
-        float Lv[16];
-        if (!NL) {
-          const uint32_t lb = gg % NLB;
-          ok = wait_bounded(bar(BAR_LFULL + lb), (gg / NLB) & 1u, ctl, 13);
+        for (int j = 0; j < SPI; ++j) {
+          const uint32_t gj = g + kk + j, fslot = gj % NF;
+          ok = wait_bounded(bar(BAR_PFULL + fslot), (gj / NF) & 1u, ctl, 12);
           if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-          tc_fence_after();
-          tmem_ld16(tmem + lane_off + COL_L + BK * lb + 16 * c, Lv);
-          tmem_ld_wait();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) report(BAR_LEMPTY + lb, pw);
+          const uint32_t fs = smem + OFF_FSLOTS + fslot * FSLOT_BYTES;
+          if (PACKED) {
+            const uint2 r = ld_shared_v2(fs + swz_offset(row, c >> 1, 32) + 8 * (c & 1));
+            raw[j][0] = r.x;
+            raw[j][1] = r.y;
+          } else if (fmt_16bit(FMT)) {
+            const uint4 r0 = ld_shared_v4(fs + swz_offset(row, 2 * c, 128));
+            const uint4 r1 = ld_shared_v4(fs + swz_offset(row, 2 * c + 1, 128));
+            raw[j][0] = r0.x, raw[j][1] = r0.y, raw[j][2] = r0.z, raw[j][3] = r0.w;
+            raw[j][4] = r1.x, raw[j][5] = r1.y, raw[j][6] = r1.z, raw[j][7] = r1.w;
+          } else {
+            const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
+            raw[j][0] = r.x, raw[j][1] = r.y, raw[j][2] = r.z, raw[j][3] = r.w;
+          }
         }
-        uint32_t w[8];
+        if (!ok) break;
+        uint32_t w[SPI][8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          uint32_t cw;
-          if (NL) {
-            cw = b64                         ? c8[e]
-                 : args.codes_bias == 128    ? pack_int_bf16x2(v[2 * e], v[2 * e + 1])
-                                             : int_codes_bf16x2(v[2 * e], v[2 * e + 1], qp);
+        for (int j = 0; j < SPI; ++j) {
+          const uint32_t gj = g + kk + j;
+          float v[16];
+          // the codes base with the clipped codes stored as c + 64: bf16 straight from the bytes
+          const bool b64 = NL && args.codes_bias == 64;
+          uint32_t c8[8];
+          if (b64) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) decode_b64_bf16x4(raw[j][i], c8[2 * i], c8[2 * i + 1]);
+          } else if (NL && args.codes_bias == 128) {
+            decode_ob16(raw[j], v);
           } else {
-            const float2 u = UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
-                                : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]),
-                                             make_float2(qp.lr_scale, qp.lr_scale), make_float2(v[2 * e], v[2 * e + 1]));
-            cw = codes_bf16x2(__fadd2_rn(u, make_float2(qp.magic, qp.magic)), qp);
+            decode16<FMT>(raw[j], v);
           }
-          if (ZP) cw = sub_bf16x2(cw, zw[e]);
-          if (MODE == FUSED_FWD_PC) {
-            w[e] = cw;
-          } else {
-            w[e] = mul_bf16x2(cw, MODE == FUSED_DX ? scw[e] : pack_rn_bf16x2(sc[2 * e], sc[2 * e + 1]));
+          float Lv[16];
+          if (!NL) {
+            const uint32_t lb = gj % NLB;
+            ok = wait_bounded(bar(BAR_LFULL + lb), (gj / NLB) & 1u, ctl, 13);
+            if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+            tc_fence_after();
+            tmem_ld16(tmem + lane_off + COL_L + BK * lb + 16 * c, Lv);
+            tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) report(BAR_LEMPTY + lb, pw);
+          }
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            uint32_t cw;
+            if (NL) {
+              cw = b64                         ? c8[e]
+                   : args.codes_bias == 128    ? pack_int_bf16x2(v[2 * e], v[2 * e + 1])
+                                               : int_codes_bf16x2(v[2 * e], v[2 * e + 1], qp);
+            } else {
+              const float2 u = UB ? u_bf16x2(Lv[2 * e], Lv[2 * e + 1], v[2 * e], v[2 * e + 1], lr2)
+                                  : __ffma2_rn(make_float2(Lv[2 * e], Lv[2 * e + 1]),
+                                               make_float2(qp.lr_scale, qp.lr_scale),
+                                               make_float2(v[2 * e], v[2 * e + 1]));
+              cw = codes_bf16x2(__fadd2_rn(u, make_float2(qp.magic, qp.magic)), qp);
+            }
+            if (ZP) cw = sub_bf16x2(cw, zw[j][e]);
+            if (MODE == FUSED_FWD_PC) {
+              w[j][e] = cw;
+            } else {
+              w[j][e] = mul_bf16x2(cw, MODE == FUSED_DX ? scw[j][e] : sgw[j]);
+            }
           }
         }
-        // The W_hat buffer of this token slot was last read by the product of stage gg - NT.
-        const uint32_t ts = gg % NT;
-        ok = wait_bounded(bar(BAR_TEMPTY + ts), ((gg / NT) & 1u) ^ 1u, ctl, 14);
-        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-        const uint32_t wt = smem + OFF_TSLOTS + ts * TSLOT_BYTES + TS_W;
-        st_shared_v4(wt + swz_offset(row, 2 * c, 128), w[0], w[1], w[2], w[3]);
-        st_shared_v4(wt + swz_offset(row, 2 * c + 1, 128), w[4], w[5], w[6], w[7]);
+        if (!ok) break;
+        // Each stage's W_hat buffer (in its token slot) was last read by the product of stage gj - NT.
+#pragma unroll
+        for (int j = 0; j < SPI; ++j) {
+          const uint32_t gj = g + kk + j, ts = gj % NT;
+          ok = wait_bounded(bar(BAR_TEMPTY + ts), ((gj / NT) & 1u) ^ 1u, ctl, 14);
+          if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+          const uint32_t wt = smem + OFF_TSLOTS + ts * TSLOT_BYTES + TS_W;
+          st_shared_v4(wt + swz_offset(row, 2 * c, 128), w[j][0], w[j][1], w[j][2], w[j][3]);
+          st_shared_v4(wt + swz_offset(row, 2 * c + 1, 128), w[j][4], w[j][5], w[j][6], w[j][7]);
+        }
+        if (!ok) break;
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          report(BAR_TFULL + ts, pw);
-          mbar_arrive(bar(BAR_FEMPTY + fslot));
+#pragma unroll
+          for (int j = 0; j < SPI; ++j) {
+            const uint32_t gj = g + kk + j;
+            report(BAR_TFULL + gj % NT, pw);
+            mbar_arrive(bar(BAR_FEMPTY + gj % NF));
+          }
         }
       }
       if (!ok) break;
