@@ -67,15 +67,19 @@ constexpr uint32_t TS_W = TOK_BYTES;
 // the stored base and this CTA's half of the second factor's slice.  On the codes (NL): no
 // factors, so a fourth token slot fits (measured on a 4096 x 4096 layer at T = 8192: forward
 // 191 -> 181 us).
-template <int FMT, bool NL>
+// DXS (dX): each factor slot also holds the stage's 64 bf16 scales (and zero offsets) of the
+// CTA's row group, copied by the factor loader, so that the producers read them from shared
+// memory with the base instead of from global memory.
+template <int FMT, bool NL, bool DXS>
 struct PairRing {
   static constexpr int NT = NL ? 4 : 3;
   static constexpr int NF = fmt_16bit(FMT) ? 2 : 4;
   static constexpr uint32_t RF = NL ? 0u : RF_BYTES;
   static constexpr uint32_t PHI_BYTES = fmt_16bit(FMT) ? 128 * 128 : 128 * 64;
   static constexpr uint32_t PHI_TX = FMT == FMT_I4 ? PHI_BYTES / 2 : PHI_BYTES;
-  static constexpr uint32_t FSLOT_BYTES = PHI_BYTES + (NL ? 0u : SFH_BYTES);
   static constexpr uint32_t FS_SF = PHI_BYTES;
+  static constexpr uint32_t FS_X = PHI_BYTES + (NL ? 0u : SFH_BYTES);   // dX: scales at +0, zero offsets at +128
+  static constexpr uint32_t FSLOT_BYTES = FS_X + (DXS ? 1024u : 0u);
   static constexpr uint32_t OFF_RF = 0;
   static constexpr uint32_t OFF_TSLOTS = RF;
   static constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
@@ -124,7 +128,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_pair_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
                       const FusedArgs args) {
-  using PR = PairRing<FMT, NL>;
+  using PR = PairRing<FMT, NL, MODE == FUSED_DX>;
   constexpr int NT = PR::NT;
   constexpr int NF = PR::NF;
   constexpr uint32_t OFF_RF = PR::OFF_RF, OFF_TSLOTS = PR::OFF_TSLOTS, OFF_FSLOTS = PR::OFF_FSLOTS;
@@ -275,9 +279,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t s = gg % NF;
           if (!(ok = wait_spin_bounded(bar(BAR_FEMPTY + s), ((gg / NF) & 1u) ^ 1u, ctl, 3))) break;
           const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
-          mbar_arrive_expect_tx(bar(BAR_PFULL + s), PR::PHI_TX);
+          constexpr uint32_t XTX = MODE == FUSED_DX ? (ZP ? 256u : 128u) : 0u;
+          mbar_arrive_expect_tx(bar(BAR_PFULL + s), PR::PHI_TX + XTX);
           tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb2 * 2 * BM + static_cast<int>(rank) * BM,
                       bar(BAR_PFULL + s));
+          if (MODE == FUSED_DX) {
+            // the stage's 64 scales (and zero offsets) of this CTA's row group (group sizes are
+            // multiples of 128, so a CTA's 128 rows lie in one group)
+            const int64_t xoff = (args.s_ld ? static_cast<int64_t>((rb2 * 2 * BM + static_cast<int>(rank) * BM) /
+                                                                   args.group_size) * args.kdim
+                                            : 0) + kk * BK;
+            bulk_load(fs + PR::FS_X, args.s_bf16 + xoff, 128u, bar(BAR_PFULL + s));
+            if (ZP) bulk_load(fs + PR::FS_X + 128u, args.z_bf16 + xoff, 128u, bar(BAR_PFULL + s));
+          }
           if (!NL) {
             if (leader) mbar_arrive_expect_tx(bar(BAR_FFULL + s), 2u * sf_tx);
             tma_load_2d_pair(fs + PR::FS_SF, &tm_sf, 0, kk * BK + static_cast<int>(rank) * 32, lbar(BAR_FFULL + s));
@@ -360,16 +374,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int j = 0; j < SPI; ++j) {
           const int kj = kk + j;
           if (ZP) {
-            if (MODE == FUSED_DX) {
-              // 16 consecutive bf16 zero offsets of this stage's contraction indices
-              const uint16_t* zp = args.z_bf16 +
-                                   (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
-                                   kj * BK + 16 * c;
-              const uint4 z0 = __ldg(reinterpret_cast<const uint4*>(zp));
-              const uint4 z1 = __ldg(reinterpret_cast<const uint4*>(zp) + 1);
-              zw[j][0] = z0.x, zw[j][1] = z0.y, zw[j][2] = z0.z, zw[j][3] = z0.w;
-              zw[j][4] = z1.x, zw[j][5] = z1.y, zw[j][6] = z1.z, zw[j][7] = z1.w;
-            } else {
+            if (MODE != FUSED_DX) {
               const float zr = MODE == FUSED_FWD_GROUP
                                    ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kj * BK) / args.group_size]
                                    : args.zero[row_g];
@@ -381,14 +386,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (MODE == FUSED_FWD_GROUP) {
             const float v = args.s[static_cast<int64_t>(row_g) * args.s_ld + (kj * BK) / args.group_size];
             sgw[j] = pack_rn_bf16x2(v, v);
-          } else if (MODE == FUSED_DX) {
-            const uint16_t* sp = args.s_bf16 +
-                                 (args.s_ld ? static_cast<int64_t>(row_g / args.group_size) * args.kdim : 0) +
-                                 kj * BK + 16 * c;
-            const uint4 s0 = __ldg(reinterpret_cast<const uint4*>(sp));
-            const uint4 s1 = __ldg(reinterpret_cast<const uint4*>(sp) + 1);
-            scw[j][0] = s0.x, scw[j][1] = s0.y, scw[j][2] = s0.z, scw[j][3] = s0.w;
-            scw[j][4] = s1.x, scw[j][5] = s1.y, scw[j][6] = s1.z, scw[j][7] = s1.w;
           }
         }
         // the stages' stored bases, each read as soon as it has landed
@@ -411,6 +408,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           } else {
             const uint4 r = ld_shared_v4(fs + swz_offset(row, c, 64));
             raw[j][0] = r.x, raw[j][1] = r.y, raw[j][2] = r.z, raw[j][3] = r.w;
+          }
+          if (MODE == FUSED_DX) {
+            // the 16 bf16 scales (zero offsets) of this warp's contraction indices, as bf16x2 words
+            const uint4 s0 = ld_shared_v4(fs + PR::FS_X + 32u * c), s1 = ld_shared_v4(fs + PR::FS_X + 32u * c + 16u);
+            scw[j][0] = s0.x, scw[j][1] = s0.y, scw[j][2] = s0.z, scw[j][3] = s0.w;
+            scw[j][4] = s1.x, scw[j][5] = s1.y, scw[j][6] = s1.z, scw[j][7] = s1.w;
+            if (ZP) {
+              const uint4 z0 = ld_shared_v4(fs + PR::FS_X + 128u + 32u * c);
+              const uint4 z1 = ld_shared_v4(fs + PR::FS_X + 128u + 32u * c + 16u);
+              zw[j][0] = z0.x, zw[j][1] = z0.y, zw[j][2] = z0.z, zw[j][3] = z0.w;
+              zw[j][4] = z1.x, zw[j][5] = z1.y, zw[j][6] = z1.z, zw[j][7] = z1.w;
+            }
           }
         }
         if (!ok) break;
@@ -531,7 +540,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 template <int MODE, int FMT, bool ZP, bool UB, bool NL>
 cudaError_t launch_pair_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                             const FusedArgs& args, int npairs, cudaStream_t stream) {
-  constexpr uint32_t smem = PairRing<FMT, NL>::SMEM_BYTES;
+  constexpr uint32_t smem = PairRing<FMT, NL, MODE == FUSED_DX>::SMEM_BYTES;
   static bool configured[kMaxDevices] = {};
   const void* fn = reinterpret_cast<const void*>(fused_pair_kernel<MODE, FMT, ZP, UB, NL>);
   cudaError_t e = ensure_smem_attr(fn, static_cast<int>(smem), configured);
