@@ -27,12 +27,17 @@
  *   - Supported shapes: m and k multiples of 128, 1 <= r <= 256 (ranks above
  *     64 with bits <= 7), T >= 1 (any T; ragged token tails are handled),
  *     group_size 0 (per output channel) or a multiple of 128 that divides k.
- *   - Ranks up to 64 rebuild W_hat entirely inside the GEMMs, the low-rank tile
- *     (alpha/r) A B included.  Ranks above 64 first write the unclipped codes
- *     round(phi^{-1}(Phi0) + (alpha/r) A B) of every weight (int8, saturated to
- *     [-128, 127], which keeps the clip mask) into the workspace with one
- *     tensor-core pass per call; the GEMMs then clip and scale those codes on
- *     chip.  The results are the same codes, gradients and outputs.
+ *   - W_hat is rebuilt on chip inside the GEMMs and never written.  Where the
+ *     low-rank term comes from is a tuning choice (lrqat_set_lowrank_path): for
+ *     ranks up to 64 and fewer than 3072 tokens each GEMM stage computes the
+ *     low-rank tile (alpha/r) A B next to the main product; otherwise one
+ *     tensor-core pass per call first writes one byte per weight into the
+ *     workspace, the clipped code c = clip(round(u), n, p) biased by 64 (128 for
+ *     8-bit weights) where only the forward and dX GEMMs read it, or the
+ *     unclipped round(u) saturated to [-128, 127] (which keeps the clip mask)
+ *     where the weight-gradient kernel needs the mask too (ranks above 64); the
+ *     GEMMs then turn those bytes into W_hat on chip.  The results are the same
+ *     codes, gradients and outputs.
  */
 #ifndef LRQAT_H
 #define LRQAT_H
@@ -326,9 +331,10 @@ int lrqat_set_gemm_variant(int variant);
 /* Tuning (no counterpart in the paper): where the forward and dX GEMMs take the low-rank
  * term (alpha/r) A B of Eq. 8 from.  1 = "tile": each GEMM stage computes the 64-column
  * low-rank tile of its weight rows on the tensor cores next to the main product (ranks up
- * to 64); 2 = "codes": one tensor-core pass per call writes round(u) of every weight as
- * int8 (saturated to [-128, 127]) into the workspace and the GEMMs read those codes as
- * their base, with no low-rank work in the stage; 0 (the default) = codes from 3072 tokens
+ * to 64); 2 = "codes": one tensor-core pass per call writes the code of every weight as one
+ * byte (clip(round(u), n, p) + 64, or + 128 for 8-bit weights) into the workspace and the
+ * GEMMs read those bytes as their base, with no low-rank work in the stage; 0 (the default)
+ * = codes from 3072 tokens
  * on, the tile below (the pass costs two bytes of HBM traffic per weight, the tile a low-rank
  * MMA chain per stage).  Ranks above 64 always take the codes pass.  dW is unaffected: it
  * computes its own low-rank tile for ranks up to 64.  All settings give the same codes up to

@@ -1,12 +1,15 @@
 // Merge on the tensor cores (Sec. 3: after training the integer weight is
 // W_Z = clip(round(phi^{-1}(Phi0) + (alpha/r) A B), n, p), and W_hat = s W_Z), and the
-// same pass writing the unclipped codes for the GEMMs of ranks above 64.
+// same pass writing the one-byte codes that the fused GEMMs read as their base (the codes
+// path): the clipped code plus a bias (64, or 128 for 8-bit weights) where only the forward
+// and dX GEMMs read them, the unclipped code saturated to int8 where dW needs the clip mask
+// (ranks above 64).
 //
 // Tiles of 128 x 128: the tile's rows of A and columns of B land by TMA, r16 / 16 tcgen05
 // MMAs write the low-rank tile L = A B into TMEM, and warp q turns rows 32q .. 32q + 31 into
-// codes (TMEM lane = row): it reads L 32 columns at a time, decodes the stored base of the same
-// 32 columns from global memory, rounds, clamps to [lo, hi] of the quantizer constants and
-// stores 32 int8 codes as two 16-byte words.  The CTAs are persistent and overlap one tile's
+// codes (TMEM lane = row): it reads L 32 columns at a time, takes the stored base of the same
+// 32 columns (staged by TMA into the operand slot), rounds, clamps to [lo, hi] of the quantizer
+// constants, adds the bias and stores 32 one-byte codes as two 16-byte words.  The CTAs are persistent and overlap one tile's
 // codes with the next tile's copies and MMAs (two TMEM buffers).  The pass moves the base and the codes once (the product costs 2 m k r flops
 // on the tensor cores instead of the CUDA cores).
 //   A operand: K-major boxes of 64 rank columns read from A [m, r] (r % 8 == 0; columns
