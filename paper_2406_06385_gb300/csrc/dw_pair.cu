@@ -27,9 +27,9 @@
 // The partial outputs are laid out as the one-SM kernel's (per 128-row block), so the same
 // reduction sums them.
 //
-// Roles (416 threads per CTA): warp 0 loads the epilogue operands, warp 1 owns TMEM and (in
-// the leader, rank 0) issues the MMAs, warps 2..9 run the epilogue, warps 10..12 fill the
-// stages.  Loads that the MMAs read complete on the leader's barriers (both CTAs' bytes);
+// Roles (448 threads per CTA): warp 0 loads the epilogue operands, warp 1 owns TMEM and (in
+// the leader, rank 0) issues the MMAs, warps 2..9 run the epilogue, warps 10..13 fill the
+// stages (one box of every stage each).  Loads that the MMAs read complete on the leader's barriers (both CTAs' bytes);
 // the leader waits for the peer's "dU written" and "accumulator drained" events, which each
 // peer warp reports with a 16-byte copy into the leader's shared memory.
 #include <cuda.h>
@@ -46,7 +46,7 @@ namespace {
 constexpr int NS = 4;
 constexpr int BKT = 64;                        // tokens per pipeline stage
 constexpr int NUM_EPI_WARPS = 8;
-constexpr int NUM_LOADERS = 3;
+constexpr int NUM_LOADERS = 4;                 // one per box of a stage
 constexpr int FIRST_LOADER = 2 + NUM_EPI_WARPS;
 constexpr int NUM_THREADS = 32 * (FIRST_LOADER + NUM_LOADERS);
 constexpr uint32_t SIG_TX = 16u * NUM_EPI_WARPS;   // bytes of the peer's per-warp signals
@@ -293,33 +293,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else if (warp >= FIRST_LOADER) {
     // ------------------------------------------------ pipeline stage loaders
-    // Loader t fills the global steps g = t, t + NUM_LOADERS, ...; lane b issues box b
-    // (boxes 0-1: this CTA's dY columns i, boxes 2-3: its X columns j).
-    const uint32_t t = warp - FIRST_LOADER;
+    // Loader b issues box b of every stage (boxes 0-1: this CTA's dY columns i, boxes 2-3: its X
+    // columns j): one warp's copies are handled one after another, so a stage's four boxes are
+    // fetched by four warps at once.  Loader 0 of the leader announces the stage's bytes.
+    const int b = warp - FIRST_LOADER;
     if (lane == 0) {
-      prefetch_tensormap(&tm_dy);
-      prefetch_tensormap(&tm_x);
-    }
-    uint32_t g = 0;
-    bool ok = true;
-    WorkIter wi = work_begin(args, pair);
-    Unit w;
-    while (ok && work_next(wi, args, pair, npairs, w)) {
-      const int i_own = w.ib * 256 + static_cast<int>(rank) * 128;
-      const int j_own = w.jt * BN + static_cast<int>(rank) * 128;
-      for (int step = 0; step < w.nsteps; ++step, ++g) {
-        if (g % NUM_LOADERS != t) continue;
-        const uint32_t s = g % NS, ph = (g / NS) & 1u;
-        if (lane == 0) ok = wait_spin_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1);
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (!ok) break;
-        const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
-        const uint32_t fb = lbar(BAR_FULL + s);
-        if (lane == 0 && leader) mbar_arrive_expect_tx(bar(BAR_FULL + s), 2u * STAGE_BYTES);
-        __syncwarp();
-        const int tok = w.t0 + step * BKT;
-        if (lane < 2) tma_load_2d_pair(st + lane * BOX_BYTES, &tm_dy, i_own + 64 * lane, tok, fb);
-        else if (lane < 4) tma_load_2d_pair(st + STAGE_DY + (lane - 2) * BOX_BYTES, &tm_x, j_own + 64 * (lane - 2), tok, fb);
+      if (b < 2) prefetch_tensormap(&tm_dy);
+      else prefetch_tensormap(&tm_x);
+      uint32_t g = 0;
+      bool ok = true;
+      WorkIter wi = work_begin(args, pair);
+      Unit w;
+      while (ok && work_next(wi, args, pair, npairs, w)) {
+        const int i_own = w.ib * 256 + static_cast<int>(rank) * 128;
+        const int j_own = w.jt * BN + static_cast<int>(rank) * 128;
+        for (int step = 0; step < w.nsteps; ++step, ++g) {
+          const uint32_t s = g % NS, ph = (g / NS) & 1u;
+          if (!(ok = wait_spin_bounded(bar(BAR_EMPTY + s), ph ^ 1u, ctl, 1))) break;
+          const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
+          const uint32_t fb = lbar(BAR_FULL + s);
+          if (b == 0 && leader) mbar_arrive_expect_tx(bar(BAR_FULL + s), 2u * STAGE_BYTES);
+          const int tok = w.t0 + step * BKT;
+          if (b < 2) tma_load_2d_pair(st + b * BOX_BYTES, &tm_dy, i_own + 64 * b, tok, fb);
+          else tma_load_2d_pair(st + STAGE_DY + (b - 2) * BOX_BYTES, &tm_x, j_own + 64 * (b - 2), tok, fb);
+        }
       }
     }
   } else if (warp == 1) {
