@@ -27,9 +27,10 @@
 // The partial outputs are laid out as the one-SM kernel's (per 128-row block), so the same
 // reduction sums them.
 //
-// Roles (448 threads per CTA): warp 0 loads the epilogue operands, warp 1 owns TMEM and (in
-// the leader, rank 0) issues the MMAs, warps 2..9 run the epilogue, warps 10..13 fill the
-// stages (one box of every stage each).  Loads that the MMAs read complete on the leader's barriers (both CTAs' bytes);
+// Roles (480 threads per CTA): warp 0 loads the epilogue operands, warp 1 owns TMEM and (in
+// the leader, rank 0) issues the main loop's MMAs, warps 2..9 run the epilogue, warps 10..13
+// fill the stages (one box of every stage each), warp 14 (in the leader) issues the epilogue's
+// MMAs (low-rank tiles and adapter contractions).  Loads that the MMAs read complete on the leader's barriers (both CTAs' bytes);
 // the leader waits for the peer's "dU written" and "accumulator drained" events, which each
 // peer warp reports with a 16-byte copy into the leader's shared memory.
 #include <cuda.h>
@@ -48,7 +49,8 @@ constexpr int BKT = 64;                        // tokens per pipeline stage
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int NUM_LOADERS = 4;                 // one per box of a stage
 constexpr int FIRST_LOADER = 2 + NUM_EPI_WARPS;
-constexpr int NUM_THREADS = 32 * (FIRST_LOADER + NUM_LOADERS);
+constexpr int EPI_MMA_WARP = FIRST_LOADER + NUM_LOADERS;   // the leader's epilogue MMAs
+constexpr int NUM_THREADS = 32 * (EPI_MMA_WARP + 1);
 constexpr uint32_t SIG_TX = 16u * NUM_EPI_WARPS;   // bytes of the peer's per-warp signals
 
 constexpr uint32_t BOX_BYTES = 64 * BKT * 2;   // one 64-column x 64-token bf16 box (SW128)
@@ -90,8 +92,9 @@ constexpr int BAR_ACCEMPTY = BAR_ACCFULL + 1;  // leader: both CTAs read G
 constexpr int BAR_LFULL = BAR_ACCEMPTY + 1;    // both: L of the chunk complete
 constexpr int BAR_DUFULL = BAR_LFULL + 1;      // leader: both CTAs wrote dU of the chunk
 constexpr int BAR_DBFULL = BAR_DUFULL + 1;     // both: dA / dB^T of the chunk complete
-constexpr int BAR_DRAIN = BAR_DBFULL + 1;
-constexpr int NUM_BARS = BAR_DRAIN + 1;
+constexpr int BAR_DRAIN = BAR_DBFULL + 1;        // the main-loop MMAs' last completion
+constexpr int BAR_DRAIN_E = BAR_DRAIN + 1;       // the epilogue MMAs' last completion
+constexpr int NUM_BARS = BAR_DRAIN_E + 1;
 
 __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   const uint64_t t0 = global_timer_ns();
@@ -229,6 +232,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     mbar_init(bar(BAR_DUFULL), NUM_EPI_WARPS);
     mbar_init(bar(BAR_DBFULL), 1);
     mbar_init(bar(BAR_DRAIN), 1);
+    mbar_init(bar(BAR_DRAIN_E), 1);
     mbar_fence_init();
   }
   if (warp == 1) tmem_alloc_pair(smem_u32(&tmem_base_s), TMEM_COLS);
@@ -291,7 +295,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       // the leader's barriers are all waited for by its MMA thread)
       if (!P16 && cc > 0) drain_wait(bar(BAR_PFULL), (cc - 1) & 1u, args.timeout_ns);
     }
-  } else if (warp >= FIRST_LOADER) {
+  } else if (warp >= FIRST_LOADER && warp < FIRST_LOADER + NUM_LOADERS) {
     // ------------------------------------------------ pipeline stage loaders
     // Loader b issues box b of every stage (boxes 0-1: this CTA's dY columns i, boxes 2-3: its X
     // columns j): one warp's copies are handled one after another, so a stage's four boxes are
@@ -323,14 +327,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     // ------------------------------------------------------ MMA issuer (the leader's)
     if (lane == 0 && leader) {
       const uint32_t idesc_g = make_idesc_bf16(256, BN, 1, 1);
-      const uint32_t idesc_l = make_idesc_bf16(256, 128, 1, 1);
-      const uint32_t idesc_da = make_idesc_bf16(256, args.r16, 0, 0);
-      const uint32_t idesc_db = make_idesc_bf16(256, args.r16, 1, 0);
-      const int lsteps = args.r16 / 16;
       const uint64_t d_dy0 = make_sdesc(smem + OFF_STAGES, BOX_BYTES, 1024, SWZ_128B);
       const uint64_t d_x0 = make_sdesc(smem + OFF_STAGES + STAGE_DY, BOX_BYTES, 1024, SWZ_128B);
       const uint32_t b_full = bar(BAR_FULL);
-      uint32_t it = 0, cc = 0;
+      uint32_t it = 0;
       uint32_t s = 0, ph = 0;   // stage and phase of the global step
       bool ok = true;
       WorkIter wi = work_begin(args, pair);
@@ -353,12 +353,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         if (!ok) break;
         mma_commit_pair(bar(BAR_ACCFULL));
+        ++it;
+      }
+      // the peer's last drain report lands before the CTAs end
+      if (ok) ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 14);
+      mma_commit_pair_self(bar(BAR_DRAIN));
+      drain_wait(bar(BAR_DRAIN), 0, args.timeout_ns);
+    }
+  } else if (warp == EPI_MMA_WARP) {
+    // -------------------------------------------- epilogue MMA issuer (the leader's)
+    // The low-rank tiles and the adapter contractions of every unit, issued by a thread of their
+    // own: the next unit's main loop (warp 1) starts as soon as the epilogue has read G, and
+    // the first chunk's low-rank tile is computed while the unit's main loop still runs.
+    if (lane == 0 && leader) {
+      const uint32_t idesc_l = make_idesc_bf16(256, 128, 1, 1);
+      const uint32_t idesc_da = make_idesc_bf16(256, args.r16, 0, 0);
+      const uint32_t idesc_db = make_idesc_bf16(256, args.r16, 1, 0);
+      const int lsteps = args.r16 / 16;
+      uint32_t it = 0, cc = 0;
+      bool ok = true;
+      WorkIter wi = work_begin(args, pair);
+      Unit w;
+      while (ok && work_next(wi, args, pair, npairs, w)) {
         if (!(ok = wait_spin_bounded(bar(BAR_EFFULL), it & 1u, ctl, 6))) break;
         for (int c = 0; c < 2; ++c) {
           if (!(ok = wait_spin_bounded(bar(BAR_ECFULL), cc & 1u, ctl, 7))) break;
           tc_fence_after();
           // L = A (rows i) * B (the chunk's columns j): both operands MN-major, 16 rank rows
-          // (two 8-row groups) per K step; each CTA supplies its 64 columns of B.
+          // (two 8-row groups) per K step; each CTA supplies its 64 columns of B.  Both CTAs'
+          // epilogue warps read the previous chunk's L before they reported its dU (DUFULL).
           for (int ks = 0; ks < lsteps; ++ks) {
             const uint64_t ad = make_sdesc(smem + OFF_AT + 2048u * ks, rbox, 1024, SWZ_128B);
             const uint64_t bd = make_sdesc(smem + OFF_BPL + 2048u * ks, rbox, 1024, SWZ_128B);
@@ -394,10 +417,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         mma_commit_pair(bar(BAR_EFEMPTY));
         ++it;
       }
-      // the peer's last drain report lands before the CTAs end
-      if (ok) ok = wait_spin_bounded(bar(BAR_ACCEMPTY), (it & 1u) ^ 1u, ctl, 14);
-      mma_commit_pair_self(bar(BAR_DRAIN));
-      drain_wait(bar(BAR_DRAIN), 0, args.timeout_ns);
+      mma_commit_pair_self(bar(BAR_DRAIN_E));
+      drain_wait(bar(BAR_DRAIN_E), 0, args.timeout_ns);
     }
   } else {
     // ------------------------------------------------------------ epilogue
