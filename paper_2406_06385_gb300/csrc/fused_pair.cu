@@ -67,10 +67,11 @@ constexpr uint32_t TS_W = TOK_BYTES;
 // the stored base and this CTA's half of the second factor's slice.  On the codes (NL): no
 // factors, so a fourth token slot fits (measured on a 4096 x 4096 layer at T = 8192: forward
 // 191 -> 181 us).
-// DXS (dX): each factor slot also holds the stage's 64 bf16 scales (and zero offsets) of the
-// CTA's row group, copied by the factor loader, so that the producers read them from shared
-// memory with the base instead of from global memory.
-template <int FMT, bool NL, bool DXS>
+// XS: each factor slot also holds the stage's scales (and zero offsets) as bf16, copied by the
+// factor loader, so that the producers read them from shared memory with the base instead of
+// from global memory: for dX the 64 scales of the stage's contraction indices in the CTA's row
+// group, for the group-wise forward the 128 scales of the CTA's rows in the stage's group.
+template <int FMT, bool NL, bool XS>
 struct PairRing {
   static constexpr int NT = NL ? 4 : 3;
   static constexpr int NF = fmt_16bit(FMT) ? 2 : 4;
@@ -78,8 +79,9 @@ struct PairRing {
   static constexpr uint32_t PHI_BYTES = fmt_16bit(FMT) ? 128 * 128 : 128 * 64;
   static constexpr uint32_t PHI_TX = FMT == FMT_I4 ? PHI_BYTES / 2 : PHI_BYTES;
   static constexpr uint32_t FS_SF = PHI_BYTES;
-  static constexpr uint32_t FS_X = PHI_BYTES + (NL ? 0u : SFH_BYTES);   // dX: scales at +0, zero offsets at +128
-  static constexpr uint32_t FSLOT_BYTES = FS_X + (DXS ? 1024u : 0u);
+  // scales at +0, zero offsets at +512 (dX: 128 bytes each, group-wise forward: 256)
+  static constexpr uint32_t FS_X = PHI_BYTES + (NL ? 0u : SFH_BYTES);
+  static constexpr uint32_t FSLOT_BYTES = FS_X + (XS ? 1024u : 0u);
   static constexpr uint32_t OFF_RF = 0;
   static constexpr uint32_t OFF_TSLOTS = RF;
   static constexpr uint32_t OFF_FSLOTS = OFF_TSLOTS + NT * TSLOT_BYTES;
@@ -128,7 +130,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fused_pair_kernel(const __grid_constant__ CUtensorMap tm_tok, const __grid_constant__ CUtensorMap tm_phi,
                       const __grid_constant__ CUtensorMap tm_rf, const __grid_constant__ CUtensorMap tm_sf,
                       const FusedArgs args) {
-  using PR = PairRing<FMT, NL, MODE == FUSED_DX>;
+  using PR = PairRing<FMT, NL, MODE == FUSED_DX || MODE == FUSED_FWD_GROUP>;
   constexpr int NT = PR::NT;
   constexpr int NF = PR::NF;
   constexpr uint32_t OFF_RF = PR::OFF_RF, OFF_TSLOTS = PR::OFF_TSLOTS, OFF_FSLOTS = PR::OFF_FSLOTS;
@@ -279,7 +281,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t s = gg % NF;
           if (!(ok = wait_spin_bounded(bar(BAR_FEMPTY + s), ((gg / NF) & 1u) ^ 1u, ctl, 3))) break;
           const uint32_t fs = smem + OFF_FSLOTS + s * FSLOT_BYTES;
-          constexpr uint32_t XTX = MODE == FUSED_DX ? (ZP ? 256u : 128u) : 0u;
+          constexpr uint32_t XTX = MODE == FUSED_DX        ? (ZP ? 256u : 128u)
+                                   : MODE == FUSED_FWD_GROUP ? (ZP ? 512u : 256u)
+                                                             : 0u;
           mbar_arrive_expect_tx(bar(BAR_PFULL + s), PR::PHI_TX + XTX);
           tma_load_2d(fs, &tm_phi, PACKED ? kk * (BK / 2) : kk * BK, rb2 * 2 * BM + static_cast<int>(rank) * BM,
                       bar(BAR_PFULL + s));
@@ -290,7 +294,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                                                    args.group_size) * args.kdim
                                             : 0) + kk * BK;
             bulk_load(fs + PR::FS_X, args.s_bf16 + xoff, 128u, bar(BAR_PFULL + s));
-            if (ZP) bulk_load(fs + PR::FS_X + 128u, args.z_bf16 + xoff, 128u, bar(BAR_PFULL + s));
+            if (ZP) bulk_load(fs + PR::FS_X + 512u, args.z_bf16 + xoff, 128u, bar(BAR_PFULL + s));
+          } else if (MODE == FUSED_FWD_GROUP) {
+            // the 128 scales (and zero offsets) of this CTA's rows in the stage's group, from the
+            // bf16 rows [groups][m] (a group holds a multiple of 128 contraction indices, so two
+            // stages never straddle it)
+            const int64_t xoff = static_cast<int64_t>((kk * BK) / args.group_size) * args.rows + rb2 * 2 * BM +
+                                 static_cast<int>(rank) * BM;
+            bulk_load(fs + PR::FS_X, args.s_bf16 + xoff, 256u, bar(BAR_PFULL + s));
+            if (ZP) bulk_load(fs + PR::FS_X + 512u, args.z_bf16 + xoff, 256u, bar(BAR_PFULL + s));
           }
           if (!NL) {
             if (leader) mbar_arrive_expect_tx(bar(BAR_FFULL + s), 2u * sf_tx);
@@ -370,23 +382,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t scw[SPI][8];   // dX: the stage's 16 bf16 scales of its contraction indices, as bf16x2
         uint32_t zw[SPI][8];    // zero offsets as bf16x2
         uint32_t sgw[SPI];      // group-wise forward: the stage's scale as bf16x2
+        if (ZP && MODE == FUSED_FWD_PC) {
+          // per-channel forward: this row's zero offset (dX and the group-wise forward read theirs
+          // from the factor slot below)
+          const uint32_t z2 = pack_rn_bf16x2(args.zero[row_g], args.zero[row_g]);
 #pragma unroll
-        for (int j = 0; j < SPI; ++j) {
-          const int kj = kk + j;
-          if (ZP) {
-            if (MODE != FUSED_DX) {
-              const float zr = MODE == FUSED_FWD_GROUP
-                                   ? args.zero[static_cast<int64_t>(row_g) * args.s_ld + (kj * BK) / args.group_size]
-                                   : args.zero[row_g];
-              const uint32_t z2 = pack_rn_bf16x2(zr, zr);
+          for (int j = 0; j < SPI; ++j)
 #pragma unroll
-              for (int e = 0; e < 8; ++e) zw[j][e] = z2;
-            }
-          }
-          if (MODE == FUSED_FWD_GROUP) {
-            const float v = args.s[static_cast<int64_t>(row_g) * args.s_ld + (kj * BK) / args.group_size];
-            sgw[j] = pack_rn_bf16x2(v, v);
-          }
+            for (int e = 0; e < 8; ++e) zw[j][e] = z2;
         }
         // the stages' stored bases, each read as soon as it has landed
         uint32_t raw[SPI][8];
@@ -415,10 +418,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             scw[j][0] = s0.x, scw[j][1] = s0.y, scw[j][2] = s0.z, scw[j][3] = s0.w;
             scw[j][4] = s1.x, scw[j][5] = s1.y, scw[j][6] = s1.z, scw[j][7] = s1.w;
             if (ZP) {
-              const uint4 z0 = ld_shared_v4(fs + PR::FS_X + 128u + 32u * c);
-              const uint4 z1 = ld_shared_v4(fs + PR::FS_X + 128u + 32u * c + 16u);
+              const uint4 z0 = ld_shared_v4(fs + PR::FS_X + 512u + 32u * c);
+              const uint4 z1 = ld_shared_v4(fs + PR::FS_X + 512u + 32u * c + 16u);
               zw[j][0] = z0.x, zw[j][1] = z0.y, zw[j][2] = z0.z, zw[j][3] = z0.w;
               zw[j][4] = z1.x, zw[j][5] = z1.y, zw[j][6] = z1.z, zw[j][7] = z1.w;
+            }
+          } else if (MODE == FUSED_FWD_GROUP) {
+            // this thread's row's scale (and zero offset) in the stage's group, as bf16x2
+            const uint32_t sv = ld_shared_u16(fs + PR::FS_X + 2u * row);
+            sgw[j] = sv | (sv << 16);
+            if (ZP) {
+              const uint32_t zv = ld_shared_u16(fs + PR::FS_X + 512u + 2u * row);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) zw[j][e] = zv | (zv << 16);
             }
           }
         }
@@ -540,7 +552,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 template <int MODE, int FMT, bool ZP, bool UB, bool NL>
 cudaError_t launch_pair_one(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const CUtensorMap& d,
                             const FusedArgs& args, int npairs, cudaStream_t stream) {
-  constexpr uint32_t smem = PairRing<FMT, NL, MODE == FUSED_DX>::SMEM_BYTES;
+  constexpr uint32_t smem = PairRing<FMT, NL, MODE == FUSED_DX || MODE == FUSED_FWD_GROUP>::SMEM_BYTES;
   static bool configured[kMaxDevices] = {};
   const void* fn = reinterpret_cast<const void*>(fused_pair_kernel<MODE, FMT, ZP, UB, NL>);
   cudaError_t e = ensure_smem_attr(fn, static_cast<int>(smem), configured);

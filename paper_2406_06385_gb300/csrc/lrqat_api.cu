@@ -404,6 +404,8 @@ struct FwdWs {
   uint16_t* at;        // codes path: A^T [r16, m] and B [r16, k] zero-padded, codes [m, k]
   uint16_t* b_pad;
   int8_t* codes;
+  uint16_t* s_bf16;    // group-wise: the scales (and zero offsets) as bf16 rows [groups][m]
+  uint16_t* z_bf16;
 };
 
 // with_codes: carve the buffers of the codes path too (ranks above 64 always have them).
@@ -421,6 +423,11 @@ size_t fwd_ws_layout(const lrqat_layer& L, int64_t T, bool with_codes, void* bas
     w.codes = static_cast<int8_t*>(c.take(static_cast<size_t>(L.m) * L.k));
   }
   if (L.act_bits == 8) w.x_codes = static_cast<uint16_t*>(c.take(static_cast<size_t>(T) * L.k * 2));
+  if (L.group_size) {
+    const size_t groups = static_cast<size_t>(L.k / L.group_size);
+    w.s_bf16 = static_cast<uint16_t*>(c.take(groups * L.m * 2));
+    if (L.zero) w.z_bf16 = static_cast<uint16_t*>(c.take(groups * L.m * 2));
+  }
   if (ws) *ws = w;
   return (c.used + 255) & ~size_t(255);
 }
@@ -781,6 +788,14 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   a.timeout_ns = kWaitTimeoutNs;
   const int fmode = L.group_size ? FUSED_FWD_GROUP : FUSED_FWD_PC;
   const int ffmt = cb ? LRQAT_PHI_QFIXED : L.phi_format;
+  if (pair && L.group_size) {
+    // the pair kernel's producers read the group scales as bf16 rows [groups][m], staged per stage
+    const int groups = static_cast<int>(L.k / L.group_size);
+    LRQAT_LAUNCH("scale_rows", 1, stream,
+                 launch_dx_scales(s, L.zero, L.m, groups, groups, ws.s_bf16, ws.z_bf16, stream), "scale rows");
+    a.s_bf16 = ws.s_bf16;
+    a.z_bf16 = ws.z_bf16;
+  }
   if (pair) {
     const int64_t tiles = (L.m / 256) * ((T + kPairTokens - 1) / kPairTokens);
     const int npairs = static_cast<int>(tiles < dev->sms / 2 ? tiles : dev->sms / 2);
