@@ -509,11 +509,13 @@ QuantParams saturating_params(const lrqat_layer& L) {
 }
 
 // The codes pass: codes[i, j] = sat8(round(phi^{-1}(Phi0[i, j]) + (alpha/r) (A B)[i, j])) on the
-// tensor cores, from the zero-padded A^T [r16, m] and B [r16, k] (any rank up to 256).  clipped:
-// the codes clip(round(u), n, p) + 128 instead (offset-binary), for when only the forward and
-// dX GEMMs read them (dW of ranks above 64 needs the unclipped codes for its mask).
-int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, const uint16_t* B_pad, int8_t* codes,
-                   bool clipped, const DeviceInfo* dev, cudaStream_t stream);
+// tensor cores (any rank up to 256), from A [m, r] and B [r, k] themselves when the factors are
+// direct (rank a multiple of 8, 16-byte aligned: TMA boxes past r read as zeros), else from the
+// zero-padded A^T [r16, m] and B [r16, k].  clipped: the codes clip(round(u), n, p) plus the bias
+// (codes_bias) instead, for when only the forward and dX GEMMs read them (dW of ranks above 64
+// needs the unclipped codes for its mask).
+int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* A, const uint16_t* B, const uint16_t* At,
+                   const uint16_t* B_pad, int8_t* codes, bool clipped, const DeviceInfo* dev, cudaStream_t stream);
 
 }  // namespace
 }  // namespace lrqat
@@ -553,14 +555,22 @@ int noalloc_scratch(void** out) {
 }  // namespace
 
 namespace {
-int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, const uint16_t* B_pad, int8_t* codes,
-                   bool clipped, const DeviceInfo* dev, cudaStream_t stream) {
+int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* A, const uint16_t* B, const uint16_t* At,
+                   const uint16_t* B_pad, int8_t* codes, bool clipped, const DeviceInfo* dev, cudaStream_t stream) {
   const int r16 = round16(L.r);
+  const bool direct = direct_factors(L, A, B);
   CUtensorMap tm_a, tm_b;
-  LRQAT_TRY(encode_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, At, L.m, r16, L.m * 2, 64, static_cast<uint32_t>(r16),
-                      CU_TENSOR_MAP_SWIZZLE_128B, "A^T (padded)"));
-  LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B_pad, L.k, r16, L.k * 2, 64,
-                      static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
+  if (direct) {
+    LRQAT_TRY(encode_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, A, L.r, L.m, L.r * 2, 64, 128,
+                        CU_TENSOR_MAP_SWIZZLE_128B, "A"));
+    LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B, L.k, L.r, L.k * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B"));
+  } else {
+    LRQAT_TRY(encode_2d(&tm_a, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, At, L.m, r16, L.m * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "A^T (padded)"));
+    LRQAT_TRY(encode_2d(&tm_b, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, B_pad, L.k, r16, L.k * 2, 64,
+                        static_cast<uint32_t>(r16), CU_TENSOR_MAP_SWIZZLE_128B, "B (padded)"));
+  }
   CUtensorMap tm_phi;
   LRQAT_TRY(phi_map(&tm_phi, L, Phi0, 128, true));
   MergeArgs a{};
@@ -572,7 +582,8 @@ int run_codes_pass(const lrqat_layer& L, const void* Phi0, const uint16_t* At, c
   a.code_bias = clipped ? codes_bias(L) : 0u;
   a.status = dev->status;
   a.timeout_ns = kWaitTimeoutNs;
-  LRQAT_LAUNCH("lowrank_codes", 1, stream, launch_merge_tc(L.phi_format, L.u_bf16, 1, tm_a, tm_b, tm_phi, a, stream),
+  LRQAT_LAUNCH("lowrank_codes", 1, stream,
+               launch_merge_tc(L.phi_format, L.u_bf16, direct ? 0 : 1, tm_a, tm_b, tm_phi, a, stream),
                "low-rank code pass");
   return LRQAT_OK;
 }
@@ -715,11 +726,12 @@ static int linear_fwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   // the pair kernel reads K-major factor slices, so it takes B^T from the padded copy
   const bool direct = !cb && !pair && direct_factors(L, A, B);
   if (cb) {
-    // the codes of every weight, once per call
-    LRQAT_LAUNCH("adapter_layouts", 1, stream,
-                 launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
-                 "adapter layouts");
-    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, true, dev, stream));
+    // the codes of every weight, once per call (from A and B themselves when the factors are direct)
+    if (!direct_factors(L, A, B))
+      LRQAT_LAUNCH("adapter_layouts", 1, stream,
+                   launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
+                   "adapter layouts");
+    LRQAT_TRY(run_codes_pass(L, Phi0, A, B, ws.at, ws.b_pad, ws.codes, true, dev, stream));
   } else if (!direct) {
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, ws.a_pad, ws.bt_pad, nullptr, nullptr, stream),
@@ -888,13 +900,21 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
   const bool cb = codes_gemm(L, T);
   const bool cbw = codes_dw(L);
   const bool direct = !cb && direct_factors(L, A, B);
-  if (cb) {
+  if (cb && direct_factors(L, A, B)) {
+    // the codes of every weight from A and B themselves, then one launch for A^T and B padded
+    // (dW's operands) and the transposed codes (the dX GEMM's base)
+    LRQAT_TRY(run_codes_pass(L, Phi0, A, B, ws.at, ws.b_pad, ws.codes, !cbw, dev, stream));
+    LRQAT_LAUNCH("bwd_prep", 1, stream,
+                 launch_bwd_prep(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, ws.codes,
+                                 LRQAT_PHI_QFIXED, ws.phit, stream),
+                 "adapter layouts and transposed codes");
+  } else if (cb) {
     // the codes of every weight, then their transpose for the dX GEMM; A^T and B padded serve
     // the code pass and dW
     LRQAT_LAUNCH("adapter_layouts", 1, stream,
                  launch_adapter_layouts(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, stream),
                  "adapter layouts");
-    LRQAT_TRY(run_codes_pass(L, Phi0, ws.at, ws.b_pad, ws.codes, !cbw, dev, stream));
+    LRQAT_TRY(run_codes_pass(L, Phi0, A, B, ws.at, ws.b_pad, ws.codes, !cbw, dev, stream));
     LRQAT_LAUNCH("bwd_prep", 1, stream,
                  launch_bwd_prep(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, nullptr, nullptr, ws.codes,
                                  LRQAT_PHI_QFIXED, ws.phit, stream),
