@@ -118,6 +118,7 @@ __device__ __forceinline__ void mma_bf16_pair_half(uint32_t d_tmem, uint64_t a_d
 
 struct Unit {
   int ib, jt, sp, t0, nsteps;   // ib: 256-row block of the pair
+  int rev;                      // stages in descending token order
 };
 
 __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
@@ -129,6 +130,7 @@ __device__ __forceinline__ Unit decode_unit(int u, const DwArgs& a) {
   int t1 = x.t0 + a.tchunk;
   if (t1 > a.T) t1 = a.T;
   x.nsteps = (t1 - x.t0 + BKT - 1) / BKT;
+  x.rev = 0;
   return x;
 }
 
@@ -159,9 +161,12 @@ __device__ __forceinline__ WorkIter work_begin(const DwArgs& a, int pair) {
 }
 
 __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, int pair, int npairs, Unit& x) {
+  // Odd waves run their stages in descending token order: a wave shares its column (or row) blocks
+  // with the wave before it, whose last stages are then still in L2 when it starts.
   if (!a.sched.tail) {
     if (it.u >= a.num_units) return false;
     x = decode_unit(static_cast<int>(it.u), a);
+    x.rev = static_cast<int>((it.u / npairs) & 1);
     it.u += npairs;
     return true;
   }
@@ -170,6 +175,7 @@ __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, int pai
     x.sp = 0;
     x.t0 = 0;
     x.nsteps = static_cast<int>(a.sched.tsteps);
+    x.rev = static_cast<int>((it.u / npairs) & 1);
     it.u += npairs;
     return true;
   }
@@ -185,6 +191,7 @@ __device__ __forceinline__ bool work_next(WorkIter& it, const DwArgs& a, int pai
   x.sp = j;
   x.t0 = static_cast<int>(s0 * BKT);
   x.nsteps = static_cast<int>(s1 - s0);
+  x.rev = 0;
   return true;
 }
 
@@ -317,7 +324,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t st = smem + OFF_STAGES + s * STAGE_BYTES;
           const uint32_t fb = lbar(BAR_FULL + s);
           if (b == 0 && leader) mbar_arrive_expect_tx(bar(BAR_FULL + s), 2u * STAGE_BYTES);
-          const int tok = w.t0 + step * BKT;
+          const int tok = w.t0 + (w.rev ? w.nsteps - 1 - step : step) * BKT;
           if (b < 2) tma_load_2d_pair(st + b * BOX_BYTES, &tm_dy, i_own + 64 * b, tok, fb);
           else tma_load_2d_pair(st + STAGE_DY + (b - 2) * BOX_BYTES, &tm_x, j_own + 64 * (b - 2), tok, fb);
         }
