@@ -15,19 +15,25 @@
 //     CTA's two 112-token halves (SW128) with TMA whose completion lands on the leader's
 //     barrier; each slot also holds this CTA's W_hat tile of the stage;
 //   * factor ring (4 slots; 2 for 16-bit bases): the stored base of this CTA's rows (completion
-//     on its own barrier; only its own producers read it) and this CTA's half (32 rows) of the
-//     second factor's slice (completion on the leader's barrier: the low-rank MMA reads both);
-//   * in the leader, one thread issues the low-rank tile L = RF SF^T (M = 256, N = 64) of each
-//     stage into a TMEM buffer after the accumulators, and another the main product (M = 256,
-//     N = 224, 8 MMAs per stage), so that neither waits behind the other's barriers; every
-//     commit is multicast to both CTAs;
+//     on its own barrier; only its own producers read it), with it the stage's scales (and zero
+//     offsets) where the producers apply them (dX, group-wise forward), and with the low-rank tile
+//     this CTA's half (32 rows) of the second factor's slice (completion on the leader's
+//     barrier: the low-rank MMA reads both halves);
+//   * in the leader, one thread issues the main product (M = 256, N = 224, 8 MMAs per stage) and,
+//     with the low-rank tile in the stage, another the tile L = RF SF^T (M = 256, N = 64) into a
+//     TMEM buffer after the accumulators, so that neither waits behind the other's barriers;
+//     every commit is multicast to both CTAs;
 //   * sixteen producer warps per CTA build this CTA's W_hat tile exactly as the one-SM kernel
-//     does, and drain this CTA's 128 rows of the accumulators in the epilogue.
-// The leader waits for the peer's "W_hat written", "L read" and "accumulators drained" events;
-// each peer warp reports them with a 16-byte copy into the leader's shared memory whose
-// completion counts on the leader's barrier (a thread-issued remote arrive is several times
-// slower under the pair's operand traffic), after fence.proxy.async has ordered its writes.
-// Ranks above 64 (NL): the base holds the codes (as in the one-SM kernel); no factors, no L.
+//     does (on the codes, two stages per iteration), and drain this CTA's 128 rows of the
+//     accumulators in the epilogue.
+// One barrier per slot in the leader counts the stage's token bytes and both CTAs' "W_hat
+// written" events, so the MMA thread tests one barrier per stage; the peer's events ("W_hat
+// written", "L read", "accumulators drained") travel as 16-byte copies into the leader's shared
+// memory whose completion counts on the leader's barrier (a thread-issued remote arrive is
+// several times slower under the pair's operand traffic), after fence.proxy.async has ordered
+// the peer's writes.
+// On the codes (NL: every rank from 3072 tokens on, and ranks above 64) the base holds the
+// one-byte codes of the codes pass; no factors, no L.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
