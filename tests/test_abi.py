@@ -84,6 +84,17 @@ def test_workspace_grows_with_tokens_and_activation_quantizer(lib):
     assert lib.lrqat_fwd_workspace_bytes(ctypes.byref(_layer(m=100)), 64) == 0
 
 
+def test_group_wise_forward_workspace_holds_the_scale_rows(lib):
+    """A group-wise forward stages its scales (and zero offsets) as bf16 rows [groups][m], so
+    its workspace covers groups x m x 2 bytes per array beyond the per-channel layer's."""
+    m, k, g = 512, 1024, 128
+    pc = lib.lrqat_fwd_workspace_bytes(ctypes.byref(_layer(m=m, k=k)), 64)
+    gw = lib.lrqat_fwd_workspace_bytes(ctypes.byref(_layer(m=m, k=k, group_size=g)), 64)
+    gz = lib.lrqat_fwd_workspace_bytes(ctypes.byref(_layer(m=m, k=k, group_size=g, zero=256)), 64)
+    assert gw - pc >= (k // g) * m * 2
+    assert gz - gw >= (k // g) * m * 2
+
+
 def test_quantizer_setting_fields_are_checked_on_host(lib):
     """act_per_token needs act_bits 8; the zero offsets must be 16-byte aligned."""
     L = _layer(act_per_token=1)

@@ -5,9 +5,10 @@ and give an operator only its inputs and outputs, or that forbid allocation afte
 start-up because cudaMalloc can synchronize the device); this entry point serves
 them from a fixed scratch array inside the library.  The cases below make the
 forward use that array: a rank that is not a multiple of 8 (the adapters are
-copied into padded layouts there) and per-tensor int8 activations (their codes
-live there).  Each output must equal the workspace-based lrqat_linear_fwd's bit
-for bit (the same kernels read the same operands) and the oracle's within the
+copied into padded layouts there), per-tensor int8 activations (their codes
+live there) and a group-wise layer on CTA pairs (its scales go there as bf16
+rows).  Each output must equal the workspace-based lrqat_linear_fwd's bit for
+bit (the same kernels read the same operands) and the oracle's within the
 forward tolerance, on calls in a row with different layers (each call reuses the
 scratch the previous one left behind), and layers whose scratch does not fit must
 be rejected cleanly.
@@ -72,6 +73,7 @@ def test_noalloc_forward_matches_workspace_forward_on_calls_in_a_row(lowrank_pat
         (_spec("na_r20", 256, 512, 20), 1000, 31),                                   # padded adapters in the scratch
         (_spec("na_a8", 384, 512, 32, act=8), 1500, 32),                             # int8 codes in the scratch
         (_spec("na_r12_int3", 256, 768, 12, bits=3, phi=WL.PHI_INT_PACKED), 513, 33),
+        (_spec("na_g128", 256, 512, 32, group=128), 700, 34),                        # scale rows in the scratch
         (_spec("na_r20", 256, 512, 20), 1000, 31),                                   # the first call again
     ]
     for spec, T, seed in cases:
