@@ -674,8 +674,11 @@ __device__ __forceinline__ void unpack_i4x8(uint32_t packed4, uint32_t& lo_word,
   hi_word = __vsub4(__byte_perm(lo, hi, 0x7362), 0x08080808u);
 }
 
+// clip_lo/clip_hi (clip != 0): int8 codes are clamped to [clip_lo, clip_hi] (each byte of the
+// word the same bound) and biased by 64 on the way, for a consumer that reads clip(c) + 64.
 __device__ __forceinline__ void phi_transpose_body(int64_t bx, int64_t by, const void* __restrict__ phi0, int64_t m, int64_t k,
-                                                             int packed, int8_t* __restrict__ out) {
+                                                             int packed, int8_t* __restrict__ out, int clip = 0,
+                                                             uint32_t clip_lo = 0, uint32_t clip_hi = 0) {
   __shared__ __align__(16) uint32_t tile[128 * 32];   // 128 rows x 32 words
   const int64_t i0 = by * 128;
   const int64_t j0 = bx * 128;
@@ -700,6 +703,12 @@ __device__ __forceinline__ void phi_transpose_body(int64_t bx, int64_t by, const
     for (int x = 0; x < 4; ++x) {
       const int u = t + 256 * x, R = u >> 3, q = u & 7;
       v[x] = *reinterpret_cast<const uint4*>(src + (i0 + R) * k + j0 + 16 * q);
+    }
+    if (clip) {
+      // per byte: max, min (signed), then + 64 without carries between bytes
+      auto cb = [&](uint32_t w) { return __vadd4(__vmins4(__vmaxs4(w, clip_lo), clip_hi), 0x40404040u); };
+#pragma unroll
+      for (int x = 0; x < 4; ++x) v[x] = make_uint4(cb(v[x].x), cb(v[x].y), cb(v[x].z), cb(v[x].w));
     }
   }
 #pragma unroll
@@ -768,6 +777,7 @@ struct LayoutJob {
 };
 struct TransposeJob {
   const void* phi0; void* out; int64_t m, k; int fmt; int64_t nbx;   // tiles along k
+  int clip; uint32_t clip_lo, clip_hi;   // int8 codes: clamp to [lo, hi] and add 64 (bytes x4)
 };
 __global__ void __launch_bounds__(256) bwd_prep_kernel(LayoutJob lj, int64_t n_layout, TransposeJob tj) {
   if (static_cast<int64_t>(blockIdx.x) < n_layout) {
@@ -780,7 +790,8 @@ __global__ void __launch_bounds__(256) bwd_prep_kernel(LayoutJob lj, int64_t n_l
     phi_transpose16_body(b % tj.nbx, b / tj.nbx, static_cast<const uint16_t*>(tj.phi0), tj.m, tj.k,
                          static_cast<uint16_t*>(tj.out));
   } else {
-    phi_transpose_body(b % tj.nbx, b / tj.nbx, tj.phi0, tj.m, tj.k, tj.fmt == FMT_I4, static_cast<int8_t*>(tj.out));
+    phi_transpose_body(b % tj.nbx, b / tj.nbx, tj.phi0, tj.m, tj.k, tj.fmt == FMT_I4, static_cast<int8_t*>(tj.out),
+                       tj.clip, tj.clip_lo, tj.clip_hi);
   }
 }
 
@@ -1091,7 +1102,7 @@ cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t
 
 cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
                             uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad, const void* phi0,
-                            int fmt, void* phi_t, cudaStream_t stream) {
+                            int fmt, void* phi_t, cudaStream_t stream, int clip_bits) {
   if ((m % 128) != 0 || (k % 128) != 0) return cudaErrorInvalidValue;
   const LayoutJob lj{A, B, m, k, r, r16, reinterpret_cast<uint4*>(A_pad), reinterpret_cast<uint4*>(Bt_pad),
                      reinterpret_cast<uint4*>(At), reinterpret_cast<uint4*>(B_pad),
@@ -1101,7 +1112,14 @@ cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int
   const int64_t want = blocks_for(total, 256);
   const int64_t n_layout = want < 4096 ? want : 4096;
   const int64_t tile = fmt_16bit(fmt) ? 64 : 128;
-  const TransposeJob tj{phi0, phi_t, m, k, fmt, k / tile};
+  TransposeJob tj{phi0, phi_t, m, k, fmt, k / tile, 0, 0u, 0u};
+  if (clip_bits > 0) {
+    if (fmt != FMT_Q8 || clip_bits > 7) return cudaErrorInvalidValue;
+    const uint32_t lo = static_cast<uint8_t>(-(1 << (clip_bits - 1))), hi = static_cast<uint8_t>((1 << (clip_bits - 1)) - 1);
+    tj.clip = 1;
+    tj.clip_lo = lo * 0x01010101u;
+    tj.clip_hi = hi * 0x01010101u;
+  }
   const int64_t blocks = n_layout + (k / tile) * (m / tile);
   bwd_prep_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(lj, n_layout, tj);
   return cudaGetLastError();

@@ -56,10 +56,11 @@ cudaError_t launch_adapter_layouts(const uint16_t* A, const uint16_t* B, int64_t
 // The backward's preparation in one launch: the adapter layouts (as launch_adapter_layouts)
 // and phi_t[j][i] = stored value of Phi0[i][j]: the raw byte (Q-fixed, FP8), the
 // sign-extended nibble as an int8 (packed INT-b), or the raw 16-bit pattern (BF16, FP16);
-// phi_t [k, m].
+// phi_t [k, m].  clip_bits > 0 (int8 codes only): each value is clamped to the signed
+// clip_bits-bit grid and biased by 64 on the way (the GEMMs' clip(c) + 64 codes).
 cudaError_t launch_bwd_prep(const uint16_t* A, const uint16_t* B, int64_t m, int64_t k, int r, int r16,
                             uint16_t* A_pad, uint16_t* Bt_pad, uint16_t* At, uint16_t* B_pad, const void* phi0,
-                            int fmt, void* phi_t, cudaStream_t stream);
+                            int fmt, void* phi_t, cudaStream_t stream, int clip_bits = 0);
 // Schedule of the dW work over its persistent CTAs.  The work is ni x nj tiles (128 rows i x
 // 128 * nchunks columns j; tile = ib + ni * jt) of tsteps 32-token stages each; G and the
 // gradients it feeds (dU, dA, dB, ds) are linear in the tokens, so any token range of a tile

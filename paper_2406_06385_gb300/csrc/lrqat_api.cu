@@ -906,7 +906,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_TRY(run_codes_pass(L, Phi0, A, B, ws.at, ws.b_pad, ws.codes, !cbw, dev, stream));
     LRQAT_LAUNCH("bwd_prep", 1, stream,
                  launch_bwd_prep(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, ws.at, ws.b_pad, ws.codes,
-                                 LRQAT_PHI_QFIXED, ws.phit, stream),
+                                 LRQAT_PHI_QFIXED, ws.phit, stream, cbw ? L.bits : 0),
                  "adapter layouts and transposed codes");
   } else if (cb) {
     // the codes of every weight, then their transpose for the dX GEMM; A^T and B padded serve
@@ -917,7 +917,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     LRQAT_TRY(run_codes_pass(L, Phi0, A, B, ws.at, ws.b_pad, ws.codes, !cbw, dev, stream));
     LRQAT_LAUNCH("bwd_prep", 1, stream,
                  launch_bwd_prep(A, B, L.m, L.k, L.r, r16, nullptr, nullptr, nullptr, nullptr, ws.codes,
-                                 LRQAT_PHI_QFIXED, ws.phit, stream),
+                                 LRQAT_PHI_QFIXED, ws.phit, stream, cbw ? L.bits : 0),
                  "transposed codes");
   } else {
     LRQAT_LAUNCH("bwd_prep", 1, stream,
@@ -987,7 +987,7 @@ static int linear_bwd_impl(const lrqat_layer* layer, int64_t T, const uint16_t* 
     a.zero = L.zero;
     a.u_bf16 = cb ? 0 : L.u_bf16;
     a.sf_mn = 0;
-    a.codes_bias = cb && !cbw ? static_cast<int32_t>(codes_bias(L)) : 0;
+    a.codes_bias = cb ? static_cast<int32_t>(codes_bias(L)) : 0;   // ranks above 64: clipped and biased in the transpose
     a.s_bf16 = ws.s_bf16;
     a.z_bf16 = ws.z_bf16;
     a.s_ld = L.group_size ? static_cast<int32_t>(L.k / L.group_size) : 0;
