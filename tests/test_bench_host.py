@@ -93,6 +93,22 @@ def test_reference_arm_prints_one_json_line():
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["metric"] == bench.METRIC
 
 
+def test_reference_arm_names_the_gpu_arms_config():
+    """Both arms print the same `config` object for the same arguments (workload, shapes,
+    quantizer settings, launch mode and input rotation), so their lines describe one workload."""
+    import argparse
+    from paper_2406_06385_gb300 import workloads as WL
+    args = argparse.Namespace(sets=4, no_graph=False)
+    wl = WL.workload("llama2_13b_layer")
+    cfg = bench.workload_config(wl, args, 1)
+    assert cfg["workload"] == "llama2_13b_layer" and cfg["tokens"] == 16384 and len(cfg["layers"]) == 7
+    assert cfg["merge"] is True and cfg["phi"] == "Q4.4 int8" and cfg["granularity"] == "per-channel"
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "2", "--warmup", "3"], capture_output=True, text=True, timeout=600)
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    assert d["config"] == bench.workload_config(WL.workload("tiny"), args, 1)
+
+
 def test_warmup_below_three_is_rejected():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--warmup", "2"],
                        capture_output=True, text=True, timeout=120, cwd=ROOT)
